@@ -1,0 +1,262 @@
+"""CPU oracle of MSV-Prune, multi-layer semantic visual-token pruning (§4.1, Eq. 1-3, Alg. 1 stage 1).
+
+TEST INFRASTRUCTURE. Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg may import
+this module. It shares no code with the CUDA path. It is plain and slow, and computes in fp64.
+
+The paper is silent or ambiguous on several points. The readings taken here (ties, roundings,
+K-means initialisation, the per-token reading of the pairwise score) are the ones the CUDA path
+implements, and each is stated where it is used.
+
+Pinned by tests/test_oracle_prune.py against brute force, closed forms and invariants.
+"""
+from __future__ import annotations
+
+from fractions import Fraction
+
+import numpy as np
+
+
+def attention_importance(attn_tile: np.ndarray, form: int) -> np.ndarray:
+    """a_v for one tile: the head-mean of the encoder self-attention (§4.1.1).
+
+    form 0 (CLIP-like): attn_tile is the [CLS] row per head, [H][1+n]. Column 0 (CLS attending to
+    itself) is not a patch and is dropped. form 1 (no CLS): attn_tile is the attention each patch
+    receives per head, [H][n].
+    """
+    a = np.asarray(attn_tile, dtype=np.float64)
+    if form == 0:
+        a = a[:, 1:]
+    return a.mean(axis=0)
+
+
+def n_anchor_tokens(keep: int, anchor_ratio: float) -> int:
+    """N_anc = round(keep * r), half away from zero, evaluated in double (§4.1, Eq. 1 budget n R r).
+
+    keep = n R is the retained count. N_cmp = keep - N_anc, so the two parts always add up to keep.
+    """
+    return int(np.floor(keep * anchor_ratio + 0.5))
+
+
+def select_anchors(a_v: np.ndarray, n_anc: int) -> np.ndarray:
+    """Eq. 1: the anchor set is the n_anc tokens of largest a_v.
+
+    The threshold form (the smallest tau with at most n R r scores >= tau) names exactly this
+    top-n_anc set. Equal scores are broken toward the lower token index. Returns indices ascending.
+    """
+    n = len(a_v)
+    order = sorted(range(n), key=lambda i: (-a_v[i], i))
+    return np.array(sorted(order[:n_anc]), dtype=np.int64)
+
+
+def unit_rows(f: np.ndarray) -> np.ndarray:
+    """Rows divided by their Euclidean norm, so that dot products are cosine similarities."""
+    f = np.asarray(f, dtype=np.float64)
+    return f / np.sqrt((f * f).sum(axis=1, keepdims=True))
+
+
+def anchor_similarity(fl_unit: np.ndarray, anchors: np.ndarray) -> np.ndarray:
+    """max over anchors p of sim(F^L_i, F^L_p), for every token i (Eq. 3, second bracket).
+
+    With no anchors (r = 0) the term is absent and 0 is returned.
+    """
+    if len(anchors) == 0:
+        return np.zeros(len(fl_unit))
+    return (fl_unit @ fl_unit[anchors].T).max(axis=1)
+
+
+def kmeans(x: np.ndarray, k: int, iters: int):
+    """K-means (Lloyd) on the rows of x, the final-layer features of the non-anchor tokens (§4.1.2).
+
+    The paper names K-means on F^L and nothing more. Readings taken here:
+    * initial centroids are the rows at positions floor(j * m / K), j = 0..K-1, of the non-anchor
+      tokens in ascending token order;
+    * the distance is the squared Euclidean distance sum_d (x_d - c_d)^2;
+    * each step assigns every point to its nearest centroid (ties to the lower cluster id);
+    * at most `iters` assignment steps, stopping early once the assignment repeats;
+    * each assignment step is followed by a centroid update (mean of the members); an empty
+      cluster keeps its previous centroid.
+
+    Returns (assignment [m], min relative margin (second - best) / best over all steps and points).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    m = len(x)
+    if m == 0:
+        return np.zeros(0, dtype=np.int64), np.inf
+    c = np.stack([x[(j * m) // k] for j in range(k)])
+    assign = None
+    margin = np.inf
+    for _ in range(iters):
+        d2 = ((x[:, None, :] - c[None, :, :]) ** 2).sum(axis=2)
+        new = np.argmin(d2, axis=1)
+        if k > 1:
+            srt = np.sort(d2, axis=1)
+            margin = min(margin, float(((srt[:, 1] - srt[:, 0]) / np.maximum(srt[:, 0], 1e-300)).min()))
+        if assign is not None and np.array_equal(new, assign):
+            break
+        assign = new
+        for j in range(k):
+            members = x[assign == j]
+            if len(members):
+                c[j] = members.mean(axis=0)
+    return assign, margin
+
+
+def _round_half_away(fr: Fraction) -> int:
+    return int((fr * 2 + 1) // 2)  # fr >= 0 here
+
+
+def cluster_quotas(sizes, n_cmp: int):
+    """Eq. 2: N_k = max(1, round(N_cmp |C_k| / sum_j |C_j|)), made to add up to N_cmp.
+
+    Eq. 2 alone need not sum to N_cmp, and its floor of 1 cannot hold when N_cmp is smaller than the
+    number of non-empty clusters. Reading taken (exact rational arithmetic):
+    * q_k = N_cmp |C_k| / sum|C|; N_k = max(1, round_half_away(q_k)) for non-empty clusters, 0 for
+      empty ones, capped at |C_k|;
+    * if N_cmp < number of non-empty clusters: one each to the largest clusters (ties to lower k);
+    * if the sum is short: passes over the clusters in descending fractional part of q_k (ties to
+      lower k) add 1 to each cluster that has room, until the sum is N_cmp;
+    * if the sum is over: passes in ascending fractional part (ties to higher k) take 1 from each
+      cluster with N_k > 1, until the sum is N_cmp.
+    """
+    sizes = [int(s) for s in sizes]
+    K = len(sizes)
+    total = sum(sizes)
+    quota = [0] * K
+    if n_cmp <= 0 or total == 0:
+        return quota
+    nonempty = [k for k in range(K) if sizes[k] > 0]
+    if n_cmp < len(nonempty):
+        for k in sorted(nonempty, key=lambda k: (-sizes[k], k))[:n_cmp]:
+            quota[k] = 1
+        return quota
+    q = [Fraction(n_cmp * sizes[k], total) for k in range(K)]
+    frac = [qk - (qk.numerator // qk.denominator) for qk in q]
+    for k in nonempty:
+        quota[k] = min(sizes[k], max(1, _round_half_away(q[k])))
+    while sum(quota) < n_cmp:
+        for k in sorted(range(K), key=lambda k: (-frac[k], k)):
+            if sum(quota) < n_cmp and quota[k] < sizes[k]:
+                quota[k] += 1
+    while sum(quota) > n_cmp:
+        for k in sorted(range(K), key=lambda k: (frac[k], -k)):
+            if sum(quota) > n_cmp and quota[k] > 1:
+                quota[k] -= 1
+    return quota
+
+
+def pairwise_scores(members, units_final, units_other, other_weights, a_anchor):
+    """Eq. 3 for the tokens of one cluster, reduced to one score per token.
+
+    S_ij = sim(F^L_i, F^L_j) + sim(F^M_i, F^M_j) + max_p sim(F^L_i, F^L_p) + max_p sim(F^L_j, F^L_p).
+    The paper selects "the N_k lowest-scoring tokens" of each cluster from this pairwise score; the
+    per-token score read here is the mean of S_ij over the other members j != i of the cluster. The
+    intra-cluster term sums every tapped non-final layer with its weight (one middle layer with
+    weight 1 in the paper). A singleton cluster has no pair; its token scores 2 * a_i.
+
+    Computed literally: the full |C| x |C| matrix of S_ij, diagonal excluded.
+    """
+    members = np.asarray(members)
+    c = len(members)
+    a = a_anchor[members]
+    if c == 1:
+        return 2.0 * a
+    u = units_final[members]
+    s = u @ u.T
+    for w, uo in zip(other_weights, units_other):
+        v = uo[members]
+        s = s + w * (v @ v.T)
+    s = s + a[:, None] + a[None, :]
+    np.fill_diagonal(s, 0.0)
+    return s.sum(axis=1) / (c - 1)
+
+
+def prune_tile(feats, attn_tile, *, has_cls: bool, attn_form: int, final_layer: int, keep: int,
+               n_clusters: int = 4, kmeans_iters: int = 10, anchor_ratio: float = 0.7,
+               layer_weight=None):
+    """MSV-Prune of one tile (Alg. 1 stage 1): anchors, clustering, scoring, per-cluster selection.
+
+    feats: list over tapped layers of [n_tok][d] arrays (row 0 is [CLS] when has_cls, never kept).
+    Returns a dict with keep_idx (ascending patch indices, length keep), kind (0 dropped, 1 anchor,
+    2 complementary), cluster (-1 for anchors), scores (Eq. 3 per-token score; +inf for anchors),
+    quotas, a_v, anchor_sim, and margins of every discrete decision (anchor cut, K-means, per-cluster
+    cuts) for input conditioning.
+    """
+    off = 1 if has_cls else 0
+    patch = [np.asarray(f, dtype=np.float64)[off:] for f in feats]
+    n = patch[0].shape[0]
+    if not 1 <= keep <= n:
+        raise ValueError("keep must lie in [1, n_patch]")
+    n_layers = len(patch)
+    if layer_weight is None:
+        layer_weight = [1.0] * n_layers
+    others = [l for l in range(n_layers) if l != final_layer]
+
+    a_v = attention_importance(attn_tile, attn_form)
+    n_anc = n_anchor_tokens(keep, anchor_ratio)
+    n_cmp = keep - n_anc
+    anchors = select_anchors(a_v, n_anc)
+    is_anchor = np.zeros(n, dtype=bool)
+    is_anchor[anchors] = True
+    rest = np.flatnonzero(~is_anchor)
+
+    units_final = unit_rows(patch[final_layer])
+    units_other = [unit_rows(patch[l]) for l in others]
+    a_sim = anchor_similarity(units_final, anchors)
+
+    assign, km_margin = kmeans(patch[final_layer][rest], n_clusters, kmeans_iters)
+    sizes = [int((assign == k).sum()) for k in range(n_clusters)]
+    quotas = cluster_quotas(sizes, n_cmp)
+
+    scores = np.full(n, np.inf)
+    cluster = np.full(n, -1, dtype=np.int64)
+    cluster[rest] = assign
+    selected = []
+    cut_gap = np.inf
+    for k in range(n_clusters):
+        members = rest[assign == k]
+        if len(members) == 0:
+            continue
+        s = pairwise_scores(members, units_final, units_other,
+                            [layer_weight[l] for l in others], a_sim)
+        scores[members] = s
+        order = sorted(range(len(members)), key=lambda j: (s[j], members[j]))
+        selected.extend(members[order[:quotas[k]]].tolist())
+        if 0 < quotas[k] < len(members):
+            cut_gap = min(cut_gap, float(s[order[quotas[k]]] - s[order[quotas[k] - 1]]))
+
+    kind = np.zeros(n, dtype=np.uint8)
+    kind[anchors] = 1
+    kind[np.array(selected, dtype=np.int64)] = 2
+    keep_idx = np.flatnonzero(kind > 0)
+    srt = np.sort(a_v)[::-1]
+    anchor_gap = float((srt[n_anc - 1] - srt[n_anc]) / srt[n_anc - 1]) if 0 < n_anc < n else np.inf
+    return dict(keep_idx=keep_idx, kind=kind, cluster=cluster, scores=scores, quotas=quotas,
+                sizes=sizes, a_v=a_v, anchor_sim=a_sim, n_anchor=n_anc,
+                margins=dict(anchor_gap=anchor_gap, kmeans=km_margin, cut_gap=cut_gap))
+
+
+def prune(feats, attn, *, has_cls=True, attn_form=0, final_layer=-1, keep=64, n_clusters=4,
+          kmeans_iters=10, anchor_ratio=0.7, layer_weight=None):
+    """MSV-Prune of every tile independently (AnyRes: same rule and budget per tile, §5.1).
+
+    feats: list over tapped layers of [n_tiles][n_tok][d]; attn: [n_tiles][H][n_att].
+    """
+    final_layer = final_layer % len(feats)
+    out = []
+    for t in range(attn.shape[0]):
+        out.append(prune_tile([f[t] for f in feats], attn[t], has_cls=has_cls, attn_form=attn_form,
+                              final_layer=final_layer, keep=keep, n_clusters=n_clusters,
+                              kmeans_iters=kmeans_iters, anchor_ratio=anchor_ratio,
+                              layer_weight=layer_weight))
+    return out
+
+
+def well_conditioned(result, gap: float = 1e-3) -> bool:
+    """True when every discrete decision of a prune_tile result has a margin above `gap`.
+
+    Used to pick seeded inputs on which an fp32 implementation and this fp64 oracle must agree
+    index for index: anchor cut (relative a_v gap), K-means (relative distance margin), and the
+    per-cluster selection cuts (absolute score gap).
+    """
+    m = result["margins"]
+    return m["anchor_gap"] > gap and m["kmeans"] > gap and m["cut_gap"] > gap

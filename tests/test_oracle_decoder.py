@@ -1,0 +1,194 @@
+"""Pins of the decoder-prefill oracle (§3.2 VSkip layers, Alg. 1 stage 2) and of the FLOP model.
+
+Expected values come from libraries (torch's bf16 cast and GELU), closed forms (rotation
+invariance, one-key attention), an independent textbook forward, and the paper's Table 1 totals.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import decoder as od
+from paper_2609_34977_gb300 import flops, synth
+
+
+def tiny_model(seed=5, cfg=None, std=0.05):
+    cfg = dict(cfg or synth.TINY_DECODER)
+    w = synth.decoder_weights(seed, cfg, std=std)
+    return od.model_from_torch(w, cfg), cfg
+
+
+def test_bf16_round_matches_torch_cast():
+    r = np.random.default_rng(0)
+    x = np.concatenate([r.standard_normal(20000) * 10.0 ** r.integers(-5, 5, 20000),
+                        [0.0, -0.0, 1.0, 1.00390625, 1.01171875]]).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).float().numpy()
+    np.testing.assert_array_equal(od.bf16_round(x.astype(np.float64)), ref.astype(np.float64))
+
+
+def test_rmsnorm_output_has_unit_rms_times_gain():
+    r = np.random.default_rng(1)
+    h = r.standard_normal((5, 64)) * 3
+    g = r.uniform(0.5, 2, 64)
+    y = od.rmsnorm(h, g, 0.0)
+    np.testing.assert_allclose(np.sqrt(((y / g) ** 2).mean(1)), 1.0, rtol=1e-12)
+
+
+def test_rope_is_a_rotation_depending_on_relative_position():
+    r = np.random.default_rng(2)
+    H, hd = 2, 16
+    q, k = r.standard_normal((1, H * hd)), r.standard_normal((1, H * hd))
+    np.testing.assert_allclose(od.rope(q, np.array([0]), H, hd, 1e4), q, atol=1e-15)
+    for p in (1, 7, 300):
+        rq = od.rope(q, np.array([p]), H, hd, 1e4)
+        np.testing.assert_allclose(np.linalg.norm(rq), np.linalg.norm(q), rtol=1e-12)
+    dots = []
+    for shift in (0, 5, 123):
+        rq = od.rope(q, np.array([9 + shift]), H, hd, 1e4).reshape(H, hd)
+        rk = od.rope(k, np.array([4 + shift]), H, hd, 1e4).reshape(H, hd)
+        dots.append((rq * rk).sum(1))
+    np.testing.assert_allclose(dots[0], dots[1], rtol=1e-10)
+    np.testing.assert_allclose(dots[0], dots[2], rtol=1e-10)
+
+
+def test_rope_pairs_first_and_second_half():
+    # rotate-half: dimension j is paired with j + hd/2 (not with j+1); angle pos * theta^(-2j/hd)
+    hd = 8
+    x = np.zeros((1, hd))
+    x[0, 1] = 1.0
+    y = od.rope(x, np.array([3]), 1, hd, 100.0)[0]
+    ang = 3 * 100.0 ** (-2.0 / hd)
+    expect = np.zeros(hd)
+    expect[1], expect[5] = np.cos(ang), np.sin(ang)
+    np.testing.assert_allclose(y, expect, atol=1e-15)
+
+
+def test_attention_closed_forms():
+    r = np.random.default_rng(3)
+    H, hd = 2, 4
+    q = r.standard_normal((3, H * hd))
+    k = np.tile(r.standard_normal((1, H * hd)), (3, 1))   # identical keys: uniform weights
+    v = r.standard_normal((3, H * hd))
+    out = od.causal_attention(q, k, v, np.arange(3), np.arange(3), H, H, hd)
+    np.testing.assert_allclose(out[0], v[0], atol=1e-15)            # first token sees only itself
+    np.testing.assert_allclose(out[2], v.mean(0), atol=1e-14)       # uniform over three keys
+    np.testing.assert_allclose(out[1], v[:2].mean(0), atol=1e-14)
+
+
+def test_gqa_head_grouping():
+    r = np.random.default_rng(4)
+    H, Hkv, hd = 4, 2, 4
+    q = r.standard_normal((2, H * hd))
+    k, v = r.standard_normal((2, Hkv * hd)), r.standard_normal((2, Hkv * hd))
+    out = od.causal_attention(q, k, v, np.arange(2), np.arange(2), H, Hkv, hd)
+    # heads 0,1 read kv head 0; heads 2,3 read kv head 1; first token sees only its own value
+    np.testing.assert_allclose(out[0, 0:hd], v[0, 0:hd])
+    np.testing.assert_allclose(out[0, hd:2 * hd], v[0, 0:hd])
+    np.testing.assert_allclose(out[0, 2 * hd:3 * hd], v[0, hd:2 * hd])
+
+
+def test_gelu_matches_torch():
+    x = np.linspace(-6, 6, 101)
+    ref = torch.nn.functional.gelu(torch.from_numpy(x)).numpy()
+    np.testing.assert_allclose(od.gelu(x), ref, rtol=1e-12, atol=1e-15)
+
+
+@pytest.mark.parametrize("kv", [4, 2])
+def test_prefill_with_empty_plan_equals_textbook_forward(kv):
+    cfg = dict(synth.TINY_DECODER, n_layers=2, d_model=64, n_heads=4, n_kv_heads=kv, head_dim=16,
+               d_ffn=96, vocab=50)
+    m, cfg = tiny_model(6, cfg)
+    T = 9
+    x = od.bf16_round(np.random.default_rng(7).standard_normal((T, 64)))
+    mask = np.zeros((2, T), dtype=np.uint8)
+    for rnd in (od.identity, od.bf16_round):
+        h, logits = od.prefill(m, x, [0, T], mask, round_fn=rnd)
+        h2, logits2 = od.dense_forward(m, x, round_fn=rnd)
+        tol = 1e-12 if rnd is od.identity else 1e-6
+        np.testing.assert_allclose(h, h2, rtol=0, atol=tol * np.abs(h2).max())
+        np.testing.assert_allclose(logits[0], logits2, rtol=0, atol=tol * np.abs(logits2).max())
+
+
+def test_packed_sequences_are_independent():
+    m, cfg = tiny_model(8)
+    r = np.random.default_rng(9)
+    xa = od.bf16_round(r.standard_normal((5, 256)))
+    xb = od.bf16_round(r.standard_normal((7, 256)))
+    zero = lambda T: np.zeros((2, T), dtype=np.uint8)
+    ha, la = od.prefill(m, xa, [0, 5], zero(5))
+    hb, lb = od.prefill(m, xb, [0, 7], zero(7))
+    h, lg = od.prefill(m, np.concatenate([xa, xb]), [0, 5, 12], zero(12))
+    np.testing.assert_allclose(h, np.concatenate([ha, hb]), rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lg, np.stack([la[0], lb[0]]), rtol=0, atol=1e-12)
+
+
+def test_skipped_sublayer_is_identity_on_residual():
+    m, cfg = tiny_model(10)
+    T = 12
+    x = od.bf16_round(np.random.default_rng(11).standard_normal((T, 256)))
+    admit = np.array([-1, 0, 1, 0, -1, 1, 0, -1, -1, 0, 1, -1], dtype=np.int16)
+    target = np.array([0, 1, 2, 2, 0, 1, 1, 0, 0, 2, 2, 0], dtype=np.uint8)
+    mask = od.expand_adaptive_plan(admit, target, 2)
+    trace = []
+    od.prefill(m, x, [0, T], mask, trace=trace)
+    before = [np.array(x, dtype=np.float64)] + trace[:-1]
+    for l in range(2):
+        for sub, bit in ((0, 1), (1, 2)):
+            hin, hout = before[2 * l + sub], trace[2 * l + sub]
+            skipped = (mask[l] & bit) != 0
+            assert skipped.any()
+            np.testing.assert_array_equal(hout[skipped], hin[skipped])
+            assert np.abs(hout[~skipped] - hin[~skipped]).max() > 1e-3
+
+
+def test_skip_attn_token_still_serves_as_key_and_value():
+    cfg = dict(synth.TINY_DECODER, n_layers=1)
+    m, cfg = tiny_model(12, cfg)
+    T, j = 8, 3
+    r = np.random.default_rng(13)
+    x = od.bf16_round(r.standard_normal((T, 256)))
+    mask = np.zeros((1, T), dtype=np.uint8)
+    mask[0, j] = 1
+    x2 = x.copy()
+    x2[j] = od.bf16_round(x[j] + r.standard_normal(256))
+    t1, t2 = [], []
+    h1, _ = od.prefill(m, x, [0, T], mask, trace=t1)
+    h2, _ = od.prefill(m, x2, [0, T], mask, trace=t2)
+    np.testing.assert_array_equal(t1[0][j], x[j])                 # not a query, residual untouched
+    np.testing.assert_array_equal(h1[:j], h2[:j])                 # causal: earlier tokens unaffected
+    assert np.abs(t1[0][j + 1:] - t2[0][j + 1:]).max() > 1e-3     # later tokens read j's K/V
+
+
+def test_plan_expansions():
+    admit = np.array([-1, 0, 2, 3], dtype=np.int16)
+    target = np.array([0, 1, 2, 1], dtype=np.uint8)
+    m = od.expand_adaptive_plan(admit, target, 4)
+    expect = np.array([[0, 1, 0, 0], [0, 1, 0, 0], [0, 1, 2, 0], [0, 1, 2, 1]], dtype=np.uint8)
+    np.testing.assert_array_equal(m, expect)
+    s = od.expand_static_plan([0, 2, 3], [1, 1, 0])
+    np.testing.assert_array_equal(s, [[0, 0, 0], [2, 2, 0], [3, 3, 0]])
+
+
+def test_projector_against_torch_layers():
+    cfg = dict(synth.TINY_DECODER, d_vis=32, d_proj=48, d_model=256)
+    w = synth.decoder_weights(14, cfg)
+    m = od.model_from_torch(w, cfg)
+    vis = od.bf16_round(np.random.default_rng(15).standard_normal((6, 32)))
+    got = od.project(m, vis, round_fn=od.identity)
+    t = torch.from_numpy(vis)
+    hid = torch.nn.functional.gelu(t @ w["proj_w1"].double().T + w["proj_b1"].double())
+    ref = hid @ w["proj_w2"].double().T + w["proj_b2"].double()
+    np.testing.assert_allclose(got, ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_flop_model_reproduces_table1_vanilla_totals():
+    # Table 1: LLaVA-1.5-7B vanilla 8.5 TFLOPs (576 visual + 64 text), LLaVA-NeXT-7B 42.7 TFLOPs.
+    assert abs(flops.paper_prefill_flops(576 + 64) / 1e12 - 8.5) < 0.05
+    assert abs(flops.paper_prefill_flops(2880 + 64) / 1e12 - 42.7) < 0.05
+
+
+def test_table9_covers_every_layer_once():
+    for name in synth.TABLE9:
+        t = synth.TABLE9[name]
+        assert sorted(t["attn"] + t["ffn"]) == list(range(32))
+    assert (synth.skip_targets("llava-1.5-7b") == 2).sum() == 5
+    assert (synth.skip_targets("llava-next-7b") == 2).sum() == 7
