@@ -1,0 +1,227 @@
+/*
+ * spider.h - C ABI of libspider.so, SPIDER's accelerated multimodal prefill on one GB300 (sm_103a).
+ *
+ * Two stages, as in Alg. 1 of the paper:
+ *   1. MSV-Prune (Sec. 4.1, Eq. 1-3): score, select and compact the visual tokens of each tile.
+ *   2. Decoder prefill with adaptive sub-layer skipping (Sec. 3.2, 4.2-4.3): every layer's attention
+ *      and FFN sub-layers run or are bypassed per token, following a skip mask.
+ *
+ * Conventions for every entry point:
+ *   - Pointers marked (dev) are device memory of the current CUDA device; (host) are host memory.
+ *     bf16 data is passed as uint16_t bit patterns. Matrices are row-major.
+ *   - The caller owns every buffer. Work is enqueued on `stream` (a cudaStream_t, NULL = legacy
+ *     default stream) and is asynchronous unless stated otherwise.
+ *   - spd_prune, spd_project and spd_prefill allocate nothing: they run in a caller-provided
+ *     workspace whose size the matching *_workspace_size call returns. A workspace must not be
+ *     shared by calls that may overlap on the GPU.
+ *   - Every call returns SPD_OK (0) or a negative spd_status. Argument errors are detected on the
+ *     host before any launch and leave the device untouched; spd_last_error() describes the last
+ *     failure of the calling thread. Device-side failures (a bounded wait that gave up) are
+ *     recorded in the workspace's status word, read back by spd_workspace_status().
+ */
+#ifndef SPIDER_H
+#define SPIDER_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SPD_OK = 0,
+  SPD_EINVAL = -1,       /* invalid argument or configuration (checked on the host) */
+  SPD_ENOSPC = -2,       /* workspace smaller than the size query returned */
+  SPD_ECUDA = -3,        /* a CUDA runtime/driver call failed */
+  SPD_ETIMEOUT = -4,     /* a bounded device-side wait gave up (kernel returned early) */
+  SPD_EUNSUPPORTED = -5  /* shape outside what the kernels implement (e.g. head_dim) */
+} spd_status;
+
+#define SPD_MAX_FEAT_LAYERS 4
+#define SPD_MAX_CLUSTERS 16
+
+/* Message of the last failed call on this thread (static storage, never NULL). */
+const char* spd_last_error(void);
+
+/* Reads and clears the device status word at the start of a workspace (synchronises `stream`).
+ * *status receives SPD_OK or the first device-side failure recorded since the last read. */
+int spd_workspace_status(void* ws, void* stream, int* status);
+
+/* Failure-detection self-test (no counterpart in the paper): launches one CTA whose thread waits,
+ * with the same bounded wait every pipelined kernel here uses, on a barrier that nothing ever
+ * arrives on. After `budget_cycles` SM clock cycles the wait gives up and records SPD_ETIMEOUT in
+ * the status word of `ws` (at least 4 bytes of device memory). No fault, trap or hang: the
+ * context stays usable. Asynchronous; read the result with spd_workspace_status. */
+int spd_selftest_bounded_wait(void* ws, long long budget_cycles, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Stage 1: MSV-Prune (Sec. 4.1)                                                                */
+/* ------------------------------------------------------------------------------------------ */
+
+typedef struct {
+  int n_tiles;      /* independent tiles (images, or AnyRes crops pruned separately, Sec. 5.1) */
+  int n_tok;        /* rows per tile in the feature arrays, including the [CLS] row if has_cls */
+  int has_cls;      /* 1: row 0 of every tile is [CLS]; it is never kept */
+  int d_feat;       /* feature width, a multiple of 4, at most 4096 */
+  int n_layers;     /* tapped encoder layers, 1..SPD_MAX_FEAT_LAYERS */
+  int final_layer;  /* index of the tapped layer that is F^L (final-layer features) */
+  int n_heads;      /* encoder attention heads in `attn` */
+  int attn_form;    /* 0: [CLS] attention row per head, [n_heads][n_tok] (column 0 = CLS->CLS);
+                       1: attention received by each patch per head, [n_heads][n_tok - has_cls] */
+  int keep;         /* tokens kept per tile, 1..n_patch (n_patch = n_tok - has_cls, <= 4096) */
+  int n_clusters;   /* K of the coarse clustering, 1..SPD_MAX_CLUSTERS (paper default 4) */
+  int kmeans_iters; /* maximum Lloyd assignment steps, >= 1 (stops early on a repeated assignment) */
+  double anchor_ratio; /* r in [0, 1]; N_anc = floor(keep * r + 0.5), N_cmp = keep - N_anc */
+  float layer_weight[SPD_MAX_FEAT_LAYERS]; /* weight of each non-final layer's intra-cluster cosine
+                       term in the score; 1 everywhere reproduces Eq. 3 (entry of final_layer unused) */
+} spd_prune_cfg;
+
+/* Bytes of device workspace spd_prune needs for `cfg` (0 if cfg is invalid). */
+size_t spd_prune_workspace_size(const spd_prune_cfg* cfg);
+
+/* MSV-Prune of every tile (Sec. 4.1; Alg. 1 stage 1):
+ *   a_v = head-mean of the attention (Sec. 4.1.1); anchors = the N_anc tokens of largest a_v
+ *   (Eq. 1, ties to the lower index); K-means (Lloyd, squared Euclidean, seeds at the quantiles
+ *   floor(k m / K) of the m non-anchor tokens in index order, empty clusters keep their centroid)
+ *   on F^L of the non-anchor tokens; quotas N_k by Eq. 2 made to sum to N_cmp; per-token score =
+ *   mean over the other members j of the cluster of S_ij (Eq. 3); in each cluster the N_k
+ *   lowest-scoring tokens (ties to the lower index) join the anchors; kept indices ascending.
+ * feats    (host array of n_layers dev pointers) each [n_tiles][n_tok][d_feat] fp32.
+ * attn     (dev) fp32, [n_tiles][n_heads][n_tok] (form 0) or [n_tiles][n_heads][n_patch] (form 1).
+ * keep_idx (dev) int32 [n_tiles][keep]: kept patch indices (0-based, CLS excluded), ascending.
+ * kind     (dev, may be NULL) uint8 [n_tiles][n_patch]: 0 dropped, 1 anchor, 2 complementary.
+ * cluster  (dev, may be NULL) int8 [n_tiles][n_patch]: K-means cluster, -1 for anchors.
+ * scores   (dev, may be NULL) fp32 [n_tiles][n_patch]: per-token Eq. 3 score, +inf for anchors.
+ * All pointers 16-byte aligned. Errors: SPD_EINVAL, SPD_ENOSPC, SPD_ECUDA. */
+int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, const float* attn,
+              int32_t* keep_idx, uint8_t* kind, int8_t* cluster, float* scores,
+              void* ws, size_t ws_bytes, void* stream);
+
+/* Gathers the kept rows of a per-tile payload (e.g. F^L) into packed bf16 rows for the projector:
+ * dst[t * keep + j][:] = bf16(src[t][row_offset + idx[t][j]][:]), round to nearest even.
+ * src (dev) fp32 [n_tiles][n_tok][d]; idx (dev) int32 [n_tiles][keep]; dst (dev) bf16
+ * [n_tiles * keep][d]. d a multiple of 4. Indices outside [0, n_tok - row_offset) are skipped and
+ * reported as SPD_EINVAL through the status word of `ws` (may be NULL: no report). */
+int spd_gather_rows_bf16(const float* src, int n_tiles, int n_tok, int d, int row_offset,
+                         const int32_t* idx, int keep, uint16_t* dst, void* ws, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Stage 2: decoder prefill with sub-layer skipping (Sec. 3.2, 4.2, 4.3)                        */
+/* ------------------------------------------------------------------------------------------ */
+
+typedef struct {
+  int n_layers, d_model, n_heads, n_kv_heads, head_dim, d_ffn, vocab;
+  float rope_theta;  /* rotary base; pairs (j, j + head_dim/2) rotate by pos * theta^(-2j/head_dim) */
+  float rms_eps;     /* RMSNorm epsilon */
+  int d_vis;         /* projector input width (vision features); 0 = no projector */
+  int d_proj;        /* projector hidden width */
+} spd_model_cfg;
+
+/* One decoder layer's weights, bf16 (dev), [out][in] row-major (y = x W^T). */
+typedef struct {
+  const uint16_t* attn_norm; /* [d_model] RMSNorm gain before attention */
+  const uint16_t* wq;        /* [n_heads * head_dim][d_model] */
+  const uint16_t* wk;        /* [n_kv_heads * head_dim][d_model] */
+  const uint16_t* wv;        /* [n_kv_heads * head_dim][d_model] */
+  const uint16_t* wo;        /* [d_model][n_heads * head_dim] */
+  const uint16_t* ffn_norm;  /* [d_model] */
+  const uint16_t* w_gate;    /* [d_ffn][d_model] */
+  const uint16_t* w_up;      /* [d_ffn][d_model] */
+  const uint16_t* w_down;    /* [d_model][d_ffn] */
+} spd_layer_weights;
+
+typedef struct {
+  const spd_layer_weights* layers; /* (host) array of n_layers */
+  const uint16_t* final_norm;      /* [d_model] */
+  const uint16_t* lm_head;         /* [vocab][d_model] */
+  const uint16_t* proj_w1;         /* [d_proj][d_vis]   (only if d_vis > 0) */
+  const uint16_t* proj_b1;         /* [d_proj] */
+  const uint16_t* proj_w2;         /* [d_model][d_proj] */
+  const uint16_t* proj_b2;         /* [d_model] */
+} spd_model_weights;
+
+typedef struct spd_model spd_model;
+
+/* Copies the weights into a handle, re-laid out for the GEMM kernels (device memory is allocated
+ * here, and only here). Synchronous. The caller's weight buffers may be freed afterwards.
+ * Requirements: head_dim in {64, 128}; n_heads a multiple of n_kv_heads; d_model, d_ffn, d_vis and
+ * d_proj multiples of 8. Errors: SPD_EINVAL, SPD_EUNSUPPORTED, SPD_ECUDA. */
+int spd_model_create(const spd_model_cfg* cfg, const spd_model_weights* w, spd_model** out);
+void spd_model_destroy(spd_model* m);
+
+/* Expands Alg. 1's per-token plan into per-layer skip bits (host only):
+ * a token with admit[i] >= 0 bypasses sub-layer target[i] (1 attention, 2 FFN) in every layer
+ * l >= admit[i] (the target is frozen at admission, Sec. 4.2). admit -1 = never.
+ * mask (host) uint8 [n_layers][n_tokens]: bit 0 skip attention, bit 1 skip FFN. */
+int spd_plan_adaptive(int n_layers, int n_tokens, const int16_t* admit, const uint8_t* target,
+                      uint8_t* mask);
+
+/* Static sparse-layer replacement (Sec. 3.2): layer l bypasses the sub-layers in layer_mask[l]
+ * (same bits) for every token with token_sel[i] != 0 (the visual tokens). Host only. */
+int spd_plan_static(int n_layers, int n_tokens, const uint8_t* layer_mask, const uint8_t* token_sel,
+                    uint8_t* mask);
+
+/* Workspace bytes of spd_project for up to `rows` visual rows. */
+size_t spd_project_workspace_size(const spd_model* m, int rows);
+
+/* LLaVA MLP projector on gathered visual rows: x[out_rows[r]] = bf16(W2 bf16(GELU(W1 v_r + b1)) + b2)
+ * (exact erf GELU). vis (dev) bf16 [rows][d_vis]; out_rows (dev) int32 [rows]; x (dev) bf16
+ * [*][d_model], the decoder's input sequence. Errors: SPD_EINVAL (no projector), SPD_ENOSPC. */
+int spd_project(const spd_model* m, const uint16_t* vis, int rows, const int32_t* out_rows,
+                uint16_t* x, void* ws, size_t ws_bytes, void* stream);
+
+/* Copies bf16 rows: dst[rows_map[r]][:] = src[r][:] (dev, d_model wide), e.g. text embeddings
+ * into the decoder's input sequence. */
+int spd_scatter_rows(const spd_model* m, const uint16_t* src, int rows, const int32_t* rows_map,
+                     uint16_t* dst, void* stream);
+
+/* Workspace bytes of spd_prefill for up to `max_tokens` packed tokens in up to `max_seqs` sequences. */
+size_t spd_prefill_workspace_size(const spd_model* m, int max_tokens, int max_seqs);
+
+/* Decoder prefill with per-token sub-layer bypass (Sec. 3.2 VSkip-Attn / VSkip-FFN; Alg. 1 "Forward
+ * layer l, bypassing sub-layer target(i)"), LLaMA-style layers:
+ *   h = x;  per layer l:  a = RMSNorm(h); K, V = RoPE(a Wk^T), a Wv^T for ALL tokens;
+ *           for attention-active tokens i: h_i += Wo . Attn(RoPE(a_i Wq^T), K, V) (causal, own sequence);
+ *           for FFN-active tokens i: h_i += Wdown (SiLU(Wgate b_i) * (Wup b_i)), b_i = RMSNorm(h_i).
+ *   A token whose mask bit is set at layer l is not a query there (bit 0) and/or skips the FFN
+ *   (bit 1): its residual row passes through that sub-layer bit-exactly; with bit 0 it still serves
+ *   as a key and a value. Sub-layers with no active token launch nothing.
+ *   logits[b] = lm_head . RMSNorm(h[last token of sequence b]).
+ * x (dev) bf16 [n_tokens][d_model]: packed sequences; cu_seqlens (host) int32 [n_seqs + 1],
+ * increasing from 0 to n_tokens; positions restart at 0 in every sequence.
+ * skip_mask (host) uint8 [n_layers][n_tokens] (spd_plan_* produce it); NULL = no skipping.
+ * h (dev) fp32 [n_tokens][d_model]: receives the final residual stream.
+ * logits (dev, may be NULL) fp32 [n_seqs][vocab].
+ * Returns once all work is enqueued. Errors: SPD_EINVAL, SPD_ENOSPC, SPD_ECUDA. */
+int spd_prefill(const spd_model* m, const uint16_t* x, int n_tokens, const int32_t* cu_seqlens,
+                int n_seqs, const uint8_t* skip_mask, float* h, float* logits, void* ws,
+                size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* Single kernels, exposed for composition and per-kernel tests                                 */
+/* ------------------------------------------------------------------------------------------ */
+
+typedef enum {
+  SPD_EPI_F32 = 0,       /* out fp32 [M][N] = acc */
+  SPD_EPI_BF16 = 1,      /* out bf16 [M][N] = bf16(acc) */
+  SPD_EPI_BIAS_BF16 = 2, /* out bf16 = bf16(acc + bias[n]) */
+  SPD_EPI_BIAS_GELU_BF16 = 3, /* out bf16 = bf16(GELU(acc + bias[n])) */
+  SPD_EPI_ADD_F32 = 4    /* out fp32 [rows[m]][n] += acc (residual update; rows may be NULL = m) */
+} spd_epilogue;
+
+/* Workspace bytes of spd_linear for an M x N output. */
+size_t spd_linear_workspace_size(int M, int N);
+
+/* out = epilogue(X W^T) on the tcgen05 tensor cores, fp32 accumulation.
+ * X (dev) bf16 [M][K]; W (dev) bf16 [N][K]; K a multiple of 8; N a multiple of 128 (or equal to
+ * a padded weight count whose extra rows are never written); bias (dev) bf16 [N] or NULL; rows (dev)
+ * int32 [M] or NULL; out (dev) as described by the epilogue, row stride ldo elements. */
+int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, int N, int epilogue,
+               const uint16_t* bias, const int32_t* rows, void* out, int ldo, void* ws,
+               size_t ws_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SPIDER_H */

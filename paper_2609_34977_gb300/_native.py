@@ -1,0 +1,239 @@
+"""ctypes binding of libspider.so: the C ABI declared in include/spider.h, same names, argument
+marshalling only (torch tensors -> device pointers, numpy arrays -> host pointers).
+
+Importing this module loads nothing; the first call loads the in-tree library and raises if it
+is missing. There is no fallback: every computation runs in the CUDA library.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "lib", "libspider.so")
+
+SPD_OK, SPD_EINVAL, SPD_ENOSPC, SPD_ECUDA, SPD_ETIMEOUT, SPD_EUNSUPPORTED = 0, -1, -2, -3, -4, -5
+SPD_MAX_FEAT_LAYERS = 4
+EPI_F32, EPI_BF16, EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_ADD_F32 = 0, 1, 2, 3, 4
+
+# every symbol include/spider.h declares
+EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait",
+           "spd_prune_workspace_size", "spd_prune", "spd_gather_rows_bf16", "spd_model_create",
+           "spd_model_destroy", "spd_plan_adaptive", "spd_plan_static", "spd_project_workspace_size",
+           "spd_project", "spd_scatter_rows", "spd_prefill_workspace_size", "spd_prefill",
+           "spd_linear_workspace_size", "spd_linear")
+
+
+class SpiderError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"spider error {code}: {msg}")
+        self.code = code
+
+
+class PruneCfg(C.Structure):
+    _fields_ = [("n_tiles", C.c_int), ("n_tok", C.c_int), ("has_cls", C.c_int), ("d_feat", C.c_int),
+                ("n_layers", C.c_int), ("final_layer", C.c_int), ("n_heads", C.c_int),
+                ("attn_form", C.c_int), ("keep", C.c_int), ("n_clusters", C.c_int),
+                ("kmeans_iters", C.c_int), ("anchor_ratio", C.c_double),
+                ("layer_weight", C.c_float * SPD_MAX_FEAT_LAYERS)]
+
+
+class ModelCfg(C.Structure):
+    _fields_ = [("n_layers", C.c_int), ("d_model", C.c_int), ("n_heads", C.c_int),
+                ("n_kv_heads", C.c_int), ("head_dim", C.c_int), ("d_ffn", C.c_int),
+                ("vocab", C.c_int), ("rope_theta", C.c_float), ("rms_eps", C.c_float),
+                ("d_vis", C.c_int), ("d_proj", C.c_int)]
+
+
+class LayerWeights(C.Structure):
+    _fields_ = [(k, C.c_void_p) for k in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate",
+                                          "w_up", "w_down")]
+
+
+class ModelWeights(C.Structure):
+    _fields_ = [("layers", C.POINTER(LayerWeights))] + [
+        (k, C.c_void_p) for k in ("final_norm", "lm_head", "proj_w1", "proj_b1", "proj_w2", "proj_b2")]
+
+
+_lib = None
+
+
+def lib():
+    """The loaded library (loads it on first use; raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with __graft_entry__.build()")
+        L = C.CDLL(LIB_PATH)
+        vp, i, sz, ll = C.c_void_p, C.c_int, C.c_size_t, C.c_longlong
+        sig = {
+            "spd_last_error": (C.c_char_p, []),
+            "spd_workspace_status": (i, [vp, vp, C.POINTER(i)]),
+            "spd_selftest_bounded_wait": (i, [vp, ll, vp]),
+            "spd_prune_workspace_size": (sz, [C.POINTER(PruneCfg)]),
+            "spd_prune": (i, [C.POINTER(PruneCfg), C.POINTER(vp), vp, vp, vp, vp, vp, vp, sz, vp]),
+            "spd_gather_rows_bf16": (i, [vp, i, i, i, i, vp, i, vp, vp, vp]),
+            "spd_model_create": (i, [C.POINTER(ModelCfg), C.POINTER(ModelWeights), C.POINTER(vp)]),
+            "spd_model_destroy": (None, [vp]),
+            "spd_plan_adaptive": (i, [i, i, vp, vp, vp]),
+            "spd_plan_static": (i, [i, i, vp, vp, vp]),
+            "spd_project_workspace_size": (sz, [vp, i]),
+            "spd_project": (i, [vp, vp, i, vp, vp, vp, sz, vp]),
+            "spd_scatter_rows": (i, [vp, vp, i, vp, vp, vp]),
+            "spd_prefill_workspace_size": (sz, [vp, i, i]),
+            "spd_prefill": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, sz, vp]),
+            "spd_linear_workspace_size": (sz, [i, i]),
+            "spd_linear": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, sz, vp]),
+        }
+        for name, (res, args) in sig.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(rc: int):
+    if rc != SPD_OK:
+        raise SpiderError(rc, lib().spd_last_error().decode())
+
+
+def _p(t):
+    """Device (torch) or host (numpy) pointer, or NULL for None."""
+    if t is None:
+        return None
+    if isinstance(t, np.ndarray):
+        assert t.flags["C_CONTIGUOUS"]
+        return t.ctypes.data
+    assert t.is_contiguous(), "tensors passed to libspider must be contiguous"
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return int(stream)
+
+
+def spd_last_error() -> str:
+    return lib().spd_last_error().decode()
+
+
+def spd_workspace_status(ws, stream=None) -> int:
+    v = C.c_int(0)
+    _check(lib().spd_workspace_status(_p(ws), _stream(stream), C.byref(v)))
+    return v.value
+
+
+def spd_selftest_bounded_wait(ws, budget_cycles: int, stream=None):
+    _check(lib().spd_selftest_bounded_wait(_p(ws), int(budget_cycles), _stream(stream)))
+
+
+def prune_cfg(n_tiles, n_tok, d_feat, n_layers, final_layer, n_heads, keep, *, has_cls=True,
+              attn_form=0, n_clusters=4, kmeans_iters=10, anchor_ratio=0.7, layer_weight=None):
+    w = list(layer_weight) if layer_weight is not None else [1.0] * SPD_MAX_FEAT_LAYERS
+    w = w + [1.0] * (SPD_MAX_FEAT_LAYERS - len(w))
+    return PruneCfg(n_tiles, n_tok, int(has_cls), d_feat, n_layers, final_layer, n_heads, attn_form,
+                    keep, n_clusters, kmeans_iters, float(anchor_ratio),
+                    (C.c_float * SPD_MAX_FEAT_LAYERS)(*w))
+
+
+def spd_prune_workspace_size(cfg: PruneCfg) -> int:
+    return int(lib().spd_prune_workspace_size(C.byref(cfg)))
+
+
+def spd_prune(cfg, feats, attn, keep_idx, kind=None, cluster=None, scores=None, ws=None, stream=None):
+    arr = (C.c_void_p * len(feats))(*[_p(f) for f in feats])
+    _check(lib().spd_prune(C.byref(cfg), arr, _p(attn), _p(keep_idx), _p(kind), _p(cluster),
+                           _p(scores), _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def spd_gather_rows_bf16(src, n_tiles, n_tok, d, row_offset, idx, keep, dst, ws=None, stream=None):
+    _check(lib().spd_gather_rows_bf16(_p(src), n_tiles, n_tok, d, row_offset, _p(idx), keep, _p(dst),
+                                      _p(ws), _stream(stream)))
+
+
+class SpdModel:
+    """Owner of an spd_model handle (spd_model_create / spd_model_destroy)."""
+
+    def __init__(self, cfg: dict, weights: dict):
+        self.cfg = dict(cfg)
+        mc = ModelCfg(cfg["n_layers"], cfg["d_model"], cfg["n_heads"], cfg["n_kv_heads"],
+                      cfg["head_dim"], cfg["d_ffn"], cfg["vocab"], float(cfg["rope_theta"]),
+                      float(cfg["rms_eps"]), cfg.get("d_vis", 0) if cfg.get("d_proj") else 0,
+                      cfg.get("d_proj", 0))
+        layers = (LayerWeights * cfg["n_layers"])()
+        for l, lw in enumerate(weights["layers"]):
+            for k, _ in LayerWeights._fields_:
+                setattr(layers[l], k, _p(lw[k]))
+        mw = ModelWeights(layers, _p(weights["final_norm"]), _p(weights["lm_head"]),
+                          *[_p(weights.get(k)) for k in ("proj_w1", "proj_b1", "proj_w2", "proj_b2")])
+        h = C.c_void_p()
+        import torch
+        torch.cuda.synchronize()
+        _check(lib().spd_model_create(C.byref(mc), C.byref(mw), C.byref(h)))
+        self.handle = h
+
+    def close(self):
+        if getattr(self, "handle", None):
+            lib().spd_model_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def spd_plan_adaptive(n_layers: int, admit: np.ndarray, target: np.ndarray) -> np.ndarray:
+    admit = np.ascontiguousarray(admit, dtype=np.int16)
+    target = np.ascontiguousarray(target, dtype=np.uint8)
+    mask = np.zeros((n_layers, len(admit)), dtype=np.uint8)
+    _check(lib().spd_plan_adaptive(n_layers, len(admit), _p(admit), _p(target), _p(mask)))
+    return mask
+
+
+def spd_plan_static(layer_mask: np.ndarray, token_sel: np.ndarray) -> np.ndarray:
+    layer_mask = np.ascontiguousarray(layer_mask, dtype=np.uint8)
+    token_sel = np.ascontiguousarray(token_sel, dtype=np.uint8)
+    mask = np.zeros((len(layer_mask), len(token_sel)), dtype=np.uint8)
+    _check(lib().spd_plan_static(len(layer_mask), len(token_sel), _p(layer_mask), _p(token_sel),
+                                 _p(mask)))
+    return mask
+
+
+def spd_project_workspace_size(model: SpdModel, rows: int) -> int:
+    return int(lib().spd_project_workspace_size(model.handle, rows))
+
+
+def spd_project(model: SpdModel, vis, rows, out_rows, x, ws, stream=None):
+    _check(lib().spd_project(model.handle, _p(vis), rows, _p(out_rows), _p(x), _p(ws),
+                             ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def spd_scatter_rows(model: SpdModel, src, rows, rows_map, dst, stream=None):
+    _check(lib().spd_scatter_rows(model.handle, _p(src), rows, _p(rows_map), _p(dst), _stream(stream)))
+
+
+def spd_prefill_workspace_size(model: SpdModel, max_tokens: int, max_seqs: int) -> int:
+    return int(lib().spd_prefill_workspace_size(model.handle, max_tokens, max_seqs))
+
+
+def spd_prefill(model: SpdModel, x, n_tokens, cu_seqlens, skip_mask, h, logits, ws, stream=None):
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    mask = None if skip_mask is None else np.ascontiguousarray(skip_mask, dtype=np.uint8)
+    _check(lib().spd_prefill(model.handle, _p(x), n_tokens, _p(cu), len(cu) - 1, _p(mask), _p(h),
+                             _p(logits), _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def spd_linear_workspace_size(M: int, N: int) -> int:
+    return int(lib().spd_linear_workspace_size(M, N))
+
+
+def spd_linear(X, M, K, W, N, epilogue, out, ldo, ws, bias=None, rows=None, stream=None):
+    _check(lib().spd_linear(_p(X), M, K, _p(W), N, epilogue, _p(bias), _p(rows), _p(out), ldo, _p(ws),
+                            ws.numel() * ws.element_size(), _stream(stream)))

@@ -1,0 +1,596 @@
+// C ABI of libspider.so: errors, model handle (weight re-layout for the GEMM epilogues), skip-plan
+// expansion, the projector, and the decoder-prefill executor (Alg. 1 stage 2).
+#include <cuda_bf16.h>
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <mutex>
+#include <vector>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace spd {
+
+int attention_run(const void* q, int ldq, const void* kv, int ldkv, int v_off, void* o, int ldo,
+                  const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads,
+                  int head_dim, cudaStream_t stream);
+int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float eps,
+                const int32_t* in_rows, void* out, const int32_t* map2, void* out2,
+                cudaStream_t stream);
+int bf16_to_f32_run(const uint16_t* x, float* h, size_t n, cudaStream_t stream);
+int scatter_rows_run(const uint16_t* src, int n_rows, int D, const int32_t* rows, uint16_t* dst,
+                     cudaStream_t stream);
+
+static thread_local char g_err[512] = "no error";
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int num_sms() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : 1;
+}
+
+namespace {
+
+// dst[dst_rows[i]][:] = src[src_rows[i]][:] for rows of `cols` bf16.
+__global__ void copy_rows_kernel(const uint16_t* __restrict__ src, uint16_t* __restrict__ dst,
+                                 int cols, const int32_t* __restrict__ src_rows,
+                                 const int32_t* __restrict__ dst_rows, int n) {
+  const int i = blockIdx.x;
+  if (i >= n) return;
+  const uint16_t* s = src + size_t(src_rows[i]) * cols;
+  uint16_t* d = dst + size_t(dst_rows[i]) * cols;
+  for (int c = threadIdx.x; c < cols; c += blockDim.x) d[c] = s[c];
+}
+
+// Bounded wait on a barrier that nothing arrives on: exercises the timeout path.
+__global__ void bounded_wait_probe_kernel(int* status, long long budget) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !mbar_wait(&bar, 0, &abort_flag, budget)) set_status(status, SPD_ETIMEOUT);
+}
+
+int copy_rows(const void* src, void* dst, int cols, const std::vector<int32_t>& sr,
+              const std::vector<int32_t>& dr) {
+  if (sr.empty()) return SPD_OK;
+  int32_t* d = nullptr;
+  SPD_CUDA_TRY(cudaMalloc(&d, sr.size() * 2 * sizeof(int32_t)));
+  cudaMemcpy(d, sr.data(), sr.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+  cudaMemcpy(d + sr.size(), dr.data(), dr.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+  copy_rows_kernel<<<int(sr.size()), 256>>>(static_cast<const uint16_t*>(src),
+                                            static_cast<uint16_t*>(dst), cols, d, d + sr.size(),
+                                            int(sr.size()));
+  cudaError_t e = cudaDeviceSynchronize();
+  cudaFree(d);
+  if (e != cudaSuccess) return fail(SPD_ECUDA, "weight packing failed: %s", cudaGetErrorString(e));
+  return SPD_OK;
+}
+
+// Row order of a Q/K weight inside each head: TMEM lanes l and l + 16 of a warp hold the rotary
+// pair (j, j + head_dim/2), so the epilogue rotates with one shuffle.
+int rope_source_dim(int r, int hd) {
+  const int g = r / 32, l = r % 32;
+  return (l < 16) ? 16 * g + l : hd / 2 + 16 * g + (l - 16);
+}
+
+}  // namespace
+}  // namespace spd
+
+using namespace spd;
+
+struct spd_model {
+  spd_model_cfg cfg;
+  struct Layer {
+    uint16_t *attn_norm, *ffn_norm, *wq, *wkv, *wo, *wgu, *wd;
+    CUtensorMap m_q, m_kv, m_o, m_gu, m_d;
+  };
+  std::vector<Layer> layers;
+  uint16_t *final_norm = nullptr, *lm_head = nullptr;
+  uint16_t *pw1 = nullptr, *pb1 = nullptr, *pw2 = nullptr, *pb2 = nullptr;
+  CUtensorMap m_lm, m_p1, m_p2;
+  float* inv_freq = nullptr;
+  int gu_rows = 0;
+  void* pool = nullptr;
+};
+
+extern "C" const char* spd_last_error(void) { return g_err; }
+
+extern "C" int spd_workspace_status(void* ws, void* stream, int* status) {
+  if (!ws || !status) return fail(SPD_EINVAL, "null workspace or status");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int v = 0;
+  SPD_CUDA_TRY(cudaMemcpyAsync(&v, ws, sizeof(int), cudaMemcpyDeviceToHost, st));
+  SPD_CUDA_TRY(cudaStreamSynchronize(st));
+  SPD_CUDA_TRY(cudaMemsetAsync(ws, 0, sizeof(int), st));
+  *status = v;
+  return SPD_OK;
+}
+
+extern "C" int spd_selftest_bounded_wait(void* ws, long long budget_cycles, void* stream) {
+  if (!ws) return fail(SPD_EINVAL, "null workspace");
+  bounded_wait_probe_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<int*>(ws),
+                                                                             budget_cycles);
+  SPD_CUDA_TRY(cudaGetLastError());
+  return SPD_OK;
+}
+
+extern "C" int spd_model_create(const spd_model_cfg* c, const spd_model_weights* w, spd_model** out) {
+  if (!c || !w || !out || !w->layers) return fail(SPD_EINVAL, "null model arguments");
+  *out = nullptr;
+  if (c->n_layers < 1 || c->d_model < 8 || c->n_heads < 1 || c->n_kv_heads < 1 ||
+      c->n_heads % c->n_kv_heads || c->d_ffn < 8 || c->vocab < 1)
+    return fail(SPD_EINVAL, "invalid model shape");
+  if (c->head_dim != 64 && c->head_dim != 128)
+    return fail(SPD_EUNSUPPORTED, "head_dim must be 64 or 128");
+  if (c->d_model % 8 || c->d_ffn % 8 || (c->d_vis && (c->d_vis % 8 || c->d_proj % 8 || c->d_proj < 8)))
+    return fail(SPD_EINVAL, "d_model, d_ffn, d_vis, d_proj must be multiples of 8");
+  if ((c->n_heads * c->head_dim) % 128 || (c->n_kv_heads * c->head_dim) % 128)
+    return fail(SPD_EUNSUPPORTED, "heads * head_dim must be a multiple of 128");
+  const size_t D = c->d_model, F = c->d_ffn, hd = c->head_dim;
+  const size_t q_rows = c->n_heads * hd, kv_rows = c->n_kv_heads * hd;
+  const int gu_rows = int((F + 63) / 64 * 128);
+  auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
+  const size_t per_layer = al(D * 2) * 2 + al(q_rows * D * 2) + al(2 * kv_rows * D * 2) +
+                           al(D * q_rows * 2) + al(size_t(gu_rows) * D * 2) + al(D * F * 2);
+  size_t total = per_layer * c->n_layers + al(D * 2) + al(size_t(c->vocab) * D * 2) + al(hd * 4);
+  if (c->d_vis)
+    total += al(size_t(c->d_proj) * c->d_vis * 2) + al(size_t(c->d_proj) * 2) +
+             al(D * c->d_proj * 2) + al(D * 2);
+  spd_model* m = new spd_model();
+  m->cfg = *c;
+  m->gu_rows = gu_rows;
+  if (cudaMalloc(&m->pool, total) != cudaSuccess) {
+    delete m;
+    return fail(SPD_ECUDA, "cudaMalloc of %zu bytes for the model failed", total);
+  }
+  cudaMemset(m->pool, 0, total);
+  uint8_t* cur = static_cast<uint8_t*>(m->pool);
+  auto take = [&](size_t b) {
+    uint8_t* p = cur;
+    cur += al(b);
+    return reinterpret_cast<uint16_t*>(p);
+  };
+  int rc = SPD_OK;
+  auto fin = [&](int code) {
+    if (code) {
+      cudaFree(m->pool);
+      delete m;
+    }
+    return code;
+  };
+  std::vector<int32_t> sr, dr;
+  m->layers.resize(c->n_layers);
+  for (int l = 0; l < c->n_layers && !rc; ++l) {
+    const spd_layer_weights& s = w->layers[l];
+    spd_model::Layer& L = m->layers[l];
+    if (!s.attn_norm || !s.wq || !s.wk || !s.wv || !s.wo || !s.ffn_norm || !s.w_gate || !s.w_up ||
+        !s.w_down)
+      return fin(fail(SPD_EINVAL, "null weight in layer %d", l));
+    L.attn_norm = take(D * 2);
+    L.ffn_norm = take(D * 2);
+    L.wq = take(q_rows * D * 2);
+    L.wkv = take(2 * kv_rows * D * 2);
+    L.wo = take(D * q_rows * 2);
+    L.wgu = take(size_t(gu_rows) * D * 2);
+    L.wd = take(D * F * 2);
+    cudaMemcpy(L.attn_norm, s.attn_norm, D * 2, cudaMemcpyDeviceToDevice);
+    cudaMemcpy(L.ffn_norm, s.ffn_norm, D * 2, cudaMemcpyDeviceToDevice);
+    cudaMemcpy(L.wo, s.wo, D * q_rows * 2, cudaMemcpyDeviceToDevice);
+    cudaMemcpy(L.wd, s.w_down, D * F * 2, cudaMemcpyDeviceToDevice);
+    // Q rows in rotary-pair order
+    sr.clear();
+    dr.clear();
+    for (size_t r = 0; r < q_rows; ++r) {
+      dr.push_back(int32_t(r));
+      sr.push_back(int32_t((r / hd) * hd + rope_source_dim(int(r % hd), int(hd))));
+    }
+    if ((rc = copy_rows(s.wq, L.wq, int(D), sr, dr))) break;
+    // K rows in rotary-pair order, then V rows as they are
+    sr.clear();
+    dr.clear();
+    for (size_t r = 0; r < kv_rows; ++r) {
+      dr.push_back(int32_t(r));
+      sr.push_back(int32_t((r / hd) * hd + rope_source_dim(int(r % hd), int(hd))));
+    }
+    if ((rc = copy_rows(s.wk, L.wkv, int(D), sr, dr))) break;
+    cudaMemcpy(L.wkv + kv_rows * D, s.wv, kv_rows * D * 2, cudaMemcpyDeviceToDevice);
+    // gate/up interleaved in half-warps: 128-row tile i, row 32 w + l holds gate (l < 16) or up
+    // (l >= 16) of FFN channel 64 i + 16 w + (l mod 16)
+    std::vector<int32_t> gs, gd, us, ud;
+    for (int r = 0; r < gu_rows; ++r) {
+      const int tile = r / 128, w32 = (r % 128) / 32, l32 = r % 32;
+      const int f = tile * 64 + w32 * 16 + (l32 & 15);
+      if (f >= int(F)) continue;
+      if (l32 < 16) { gs.push_back(f); gd.push_back(r); }
+      else { us.push_back(f); ud.push_back(r); }
+    }
+    if ((rc = copy_rows(s.w_gate, L.wgu, int(D), gs, gd))) break;
+    if ((rc = copy_rows(s.w_up, L.wgu, int(D), us, ud))) break;
+    if ((rc = make_weight_map(&L.m_q, L.wq, int(q_rows), int(D)))) break;
+    if ((rc = make_weight_map(&L.m_kv, L.wkv, int(2 * kv_rows), int(D)))) break;
+    if ((rc = make_weight_map(&L.m_o, L.wo, int(D), int(q_rows)))) break;
+    if ((rc = make_weight_map(&L.m_gu, L.wgu, gu_rows, int(D)))) break;
+    if ((rc = make_weight_map(&L.m_d, L.wd, int(D), int(F)))) break;
+  }
+  if (rc) return fin(rc);
+  if (!w->final_norm || !w->lm_head) return fin(fail(SPD_EINVAL, "null final_norm or lm_head"));
+  m->final_norm = take(D * 2);
+  m->lm_head = take(size_t(c->vocab) * D * 2);
+  cudaMemcpy(m->final_norm, w->final_norm, D * 2, cudaMemcpyDeviceToDevice);
+  cudaMemcpy(m->lm_head, w->lm_head, size_t(c->vocab) * D * 2, cudaMemcpyDeviceToDevice);
+  if ((rc = make_weight_map(&m->m_lm, m->lm_head, c->vocab, int(D)))) return fin(rc);
+  m->inv_freq = reinterpret_cast<float*>(take(hd * 4));
+  std::vector<float> inv(hd / 2);
+  for (size_t j = 0; j < hd / 2; ++j)
+    inv[j] = float(pow(double(c->rope_theta), -2.0 * double(j) / double(hd)));
+  cudaMemcpy(m->inv_freq, inv.data(), inv.size() * 4, cudaMemcpyHostToDevice);
+  if (c->d_vis) {
+    if (!w->proj_w1 || !w->proj_b1 || !w->proj_w2 || !w->proj_b2)
+      return fin(fail(SPD_EINVAL, "null projector weight"));
+    m->pw1 = take(size_t(c->d_proj) * c->d_vis * 2);
+    m->pb1 = take(size_t(c->d_proj) * 2);
+    m->pw2 = take(D * c->d_proj * 2);
+    m->pb2 = take(D * 2);
+    cudaMemcpy(m->pw1, w->proj_w1, size_t(c->d_proj) * c->d_vis * 2, cudaMemcpyDeviceToDevice);
+    cudaMemcpy(m->pb1, w->proj_b1, size_t(c->d_proj) * 2, cudaMemcpyDeviceToDevice);
+    cudaMemcpy(m->pw2, w->proj_w2, D * c->d_proj * 2, cudaMemcpyDeviceToDevice);
+    cudaMemcpy(m->pb2, w->proj_b2, D * 2, cudaMemcpyDeviceToDevice);
+    if ((rc = make_weight_map(&m->m_p1, m->pw1, c->d_proj, c->d_vis))) return fin(rc);
+    if ((rc = make_weight_map(&m->m_p2, m->pw2, int(D), c->d_proj))) return fin(rc);
+  }
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return fin(fail(SPD_ECUDA, "model upload: %s", cudaGetErrorString(e)));
+  *out = m;
+  return SPD_OK;
+}
+
+extern "C" void spd_model_destroy(spd_model* m) {
+  if (!m) return;
+  cudaFree(m->pool);
+  delete m;
+}
+
+extern "C" int spd_plan_adaptive(int n_layers, int n_tokens, const int16_t* admit,
+                                 const uint8_t* target, uint8_t* mask) {
+  if (n_layers < 1 || n_tokens < 0 || (n_tokens && (!admit || !target)) || !mask)
+    return fail(SPD_EINVAL, "bad plan arguments");
+  memset(mask, 0, size_t(n_layers) * n_tokens);
+  for (int i = 0; i < n_tokens; ++i) {
+    if (admit[i] < 0) continue;
+    if (target[i] != 1 && target[i] != 2) return fail(SPD_EINVAL, "token %d: target must be 1 or 2", i);
+    for (int l = admit[i]; l < n_layers; ++l) mask[size_t(l) * n_tokens + i] = target[i];
+  }
+  return SPD_OK;
+}
+
+extern "C" int spd_plan_static(int n_layers, int n_tokens, const uint8_t* layer_mask,
+                               const uint8_t* token_sel, uint8_t* mask) {
+  if (n_layers < 1 || n_tokens < 0 || !layer_mask || (n_tokens && !token_sel) || !mask)
+    return fail(SPD_EINVAL, "bad plan arguments");
+  for (int l = 0; l < n_layers; ++l) {
+    if (layer_mask[l] > 3) return fail(SPD_EINVAL, "layer %d: mask bits must be in 0..3", l);
+    for (int i = 0; i < n_tokens; ++i)
+      mask[size_t(l) * n_tokens + i] = token_sel[i] ? layer_mask[l] : 0;
+  }
+  return SPD_OK;
+}
+
+// ---- linear (single GEMM) --------------------------------------------------------------------
+extern "C" size_t spd_linear_workspace_size(int, int) { return 256 + gemm_scratch_bytes(); }
+
+static GemmScratch scratch_from(Carve& cv) {
+  GemmScratch s;
+  s.partial_floats = size_t(16) << 20;
+  s.partial = cv.take<float>(s.partial_floats);
+  s.n_counters = 1 << 16;
+  s.counters = cv.take<int>(s.n_counters);
+  s.status = cv.status();
+  return s;
+}
+
+extern "C" int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, int N, int epilogue,
+                          const uint16_t* bias, const int32_t* rows, void* out, int ldo, void* ws,
+                          size_t ws_bytes, void* stream) {
+  if (!X || !W || !out || !ws || M < 0 || K < 8 || N < 1 || ldo < N)
+    return fail(SPD_EINVAL, "bad linear arguments");
+  if (epilogue < SPD_EPI_F32 || epilogue > SPD_EPI_ADD_F32) return fail(SPD_EINVAL, "bad epilogue");
+  if ((epilogue == SPD_EPI_BIAS_BF16 || epilogue == SPD_EPI_BIAS_GELU_BF16) && !bias)
+    return fail(SPD_EINVAL, "epilogue needs a bias");
+  Carve cv(ws, ws_bytes);
+  GemmScratch s = scratch_from(cv);
+  if (!cv.fits()) return fail(SPD_ENOSPC, "linear workspace too small");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SPD_CUDA_TRY(cudaMemsetAsync(s.counters, 0, s.n_counters * sizeof(int), st));
+  GemmProblem p{};
+  p.w = W;
+  p.x = X;
+  p.n_out = N;
+  p.n_tok = M;
+  p.k = K;
+  p.epi = epilogue;
+  p.out = out;
+  p.ldo = ldo;
+  p.rows = rows;
+  p.bias = bias;
+  p.out_cols = N;
+  return gemm_run(p, s, st);
+}
+
+// ---- projector and sequence assembly --------------------------------------------------------
+extern "C" size_t spd_project_workspace_size(const spd_model* m, int rows) {
+  if (!m || rows < 0) return 0;
+  Carve cv(nullptr, ~size_t(0));
+  scratch_from(cv);
+  cv.take<uint16_t>(size_t(rows) * (m->cfg.d_proj > 0 ? m->cfg.d_proj : 1));
+  return cv.used;
+}
+
+extern "C" int spd_project(const spd_model* m, const uint16_t* vis, int rows, const int32_t* out_rows,
+                           uint16_t* x, void* ws, size_t ws_bytes, void* stream) {
+  if (!m || !vis || !out_rows || !x || !ws || rows < 0) return fail(SPD_EINVAL, "bad project arguments");
+  if (!m->cfg.d_vis) return fail(SPD_EINVAL, "model has no projector");
+  Carve cv(ws, ws_bytes);
+  GemmScratch s = scratch_from(cv);
+  uint16_t* hid = cv.take<uint16_t>(size_t(rows) * m->cfg.d_proj);
+  if (!cv.fits()) return fail(SPD_ENOSPC, "project workspace too small");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SPD_CUDA_TRY(cudaMemsetAsync(s.counters, 0, s.n_counters * sizeof(int), st));
+  GemmProblem p{};
+  p.map_w = &m->m_p1;
+  p.x = vis;
+  p.n_out = m->cfg.d_proj;
+  p.n_tok = rows;
+  p.k = m->cfg.d_vis;
+  p.epi = EPI_BIAS_GELU_BF16;
+  p.out = hid;
+  p.ldo = m->cfg.d_proj;
+  p.bias = m->pb1;
+  if (int rc = gemm_run(p, s, st)) return rc;
+  p.map_w = &m->m_p2;
+  p.x = hid;
+  p.n_out = m->cfg.d_model;
+  p.k = m->cfg.d_proj;
+  p.epi = EPI_BIAS_BF16;
+  p.out = x;
+  p.ldo = m->cfg.d_model;
+  p.bias = m->pb2;
+  p.rows = out_rows;
+  return gemm_run(p, s, st);
+}
+
+extern "C" int spd_scatter_rows(const spd_model* m, const uint16_t* src, int rows,
+                                const int32_t* rows_map, uint16_t* dst, void* stream) {
+  if (!m || !src || !rows_map || !dst || rows < 0) return fail(SPD_EINVAL, "bad scatter arguments");
+  return scatter_rows_run(src, rows, m->cfg.d_model, rows_map, dst, static_cast<cudaStream_t>(stream));
+}
+
+// ---- prefill executor ------------------------------------------------------------------------
+namespace {
+
+struct PrefillBufs {
+  uint16_t *xa, *xq, *q, *kv, *o, *y, *act, *z;
+  int32_t* lists;
+  size_t list_ints;
+  GemmScratch gs;
+};
+
+size_t list_ints_for(int L, int T, int B) {
+  // per layer: arows[T], amap[T], apos[T], frows[T], tiles[(T / 64 + B + 1) * 4]
+  // plus pos_all[T], last[B]
+  return size_t(L) * (4 * size_t(T) + 4 * (size_t(T) / 64 + B + 1)) + T + B + 16;
+}
+
+PrefillBufs carve_prefill(const spd_model_cfg& c, int T, int B, Carve& cv) {
+  PrefillBufs b;
+  const size_t D = c.d_model, qd = size_t(c.n_heads) * c.head_dim, kvd = size_t(c.n_kv_heads) * c.head_dim;
+  b.gs = scratch_from(cv);
+  b.xa = cv.take<uint16_t>(size_t(T) * D);
+  b.xq = cv.take<uint16_t>(size_t(T) * D);
+  b.q = cv.take<uint16_t>(size_t(T) * qd);
+  b.kv = cv.take<uint16_t>(size_t(T) * 2 * kvd);
+  b.o = cv.take<uint16_t>(size_t(T) * qd);
+  b.y = cv.take<uint16_t>(size_t(T) * D);
+  b.act = cv.take<uint16_t>(size_t(T) * c.d_ffn);
+  b.z = cv.take<uint16_t>(size_t(B) * D);
+  b.list_ints = list_ints_for(c.n_layers, T, B);
+  b.lists = cv.take<int32_t>(b.list_ints);
+  return b;
+}
+
+}  // namespace
+
+extern "C" size_t spd_prefill_workspace_size(const spd_model* m, int max_tokens, int max_seqs) {
+  if (!m || max_tokens < 1 || max_seqs < 1) return 0;
+  Carve cv(nullptr, ~size_t(0));
+  carve_prefill(m->cfg, max_tokens, max_seqs, cv);
+  return cv.used;
+}
+
+extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const int32_t* cu, int B,
+                           const uint8_t* mask, float* h, float* logits, void* ws, size_t ws_bytes,
+                           void* stream) {
+  if (!m || !x || !cu || !h || !ws || T < 1 || B < 1) return fail(SPD_EINVAL, "bad prefill arguments");
+  if (cu[0] != 0 || cu[B] != T) return fail(SPD_EINVAL, "cu_seqlens must run from 0 to n_tokens");
+  for (int b = 0; b < B; ++b)
+    if (cu[b + 1] <= cu[b]) return fail(SPD_EINVAL, "sequence %d is empty or cu_seqlens decreases", b);
+  if (mask)
+    for (size_t i = 0; i < size_t(m->cfg.n_layers) * T; ++i)
+      if (mask[i] > 3) return fail(SPD_EINVAL, "skip mask entries must be in 0..3");
+  const spd_model_cfg& c = m->cfg;
+  Carve cv(ws, ws_bytes);
+  PrefillBufs bf = carve_prefill(c, T, B, cv);
+  if (!cv.fits()) return fail(SPD_ENOSPC, "prefill workspace too small (%zu < %zu)", ws_bytes, cv.used);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int L = c.n_layers, D = c.d_model, hd = c.head_dim;
+  const int qd = c.n_heads * hd, kvd = c.n_kv_heads * hd;
+
+  // Host: per-layer row lists (the plan is control data: it decides which launches happen).
+  static thread_local std::vector<int32_t> hl;
+  hl.assign(bf.list_ints, 0);
+  std::vector<int> pos_all(T), seq_of(T);
+  for (int b = 0; b < B; ++b)
+    for (int t = cu[b]; t < cu[b + 1]; ++t) {
+      pos_all[t] = t - cu[b];
+      seq_of[t] = b;
+    }
+  struct LayerLists { size_t arows, amap, apos, frows, tiles; int na, nf, ntiles; };
+  std::vector<LayerLists> ll(L);
+  size_t off = 0;
+  const size_t pos_off = off;
+  for (int t = 0; t < T; ++t) hl[off + t] = pos_all[t];
+  off += T;
+  const size_t last_off = off;
+  for (int b = 0; b < B; ++b) hl[off + b] = cu[b + 1] - 1;
+  off += B;
+  for (int l = 0; l < L; ++l) {
+    LayerLists& q = ll[l];
+    const uint8_t* mk = mask ? mask + size_t(l) * T : nullptr;
+    q.arows = off; off += T;
+    q.amap = off; off += T;
+    q.apos = off; off += T;
+    q.frows = off; off += T;
+    q.tiles = off;
+    q.na = q.nf = q.ntiles = 0;
+    for (int t = 0; t < T; ++t) {
+      const int bits = mk ? mk[t] : 0;
+      if (!(bits & 1)) {
+        hl[q.amap + t] = q.na;
+        hl[q.apos + q.na] = pos_all[t];
+        hl[q.arows + q.na++] = t;
+      } else {
+        hl[q.amap + t] = -1;
+      }
+      if (!(bits & 2)) hl[q.frows + q.nf++] = t;
+    }
+    // attention tiles: 64 active queries of one sequence each
+    int a = 0;
+    for (int b = 0; b < B; ++b) {
+      int a_end = a;
+      while (a_end < q.na && seq_of[hl[q.arows + a_end]] == b) ++a_end;
+      for (int s0 = a; s0 < a_end; s0 += 64) {
+        int32_t* tl = &hl[q.tiles + 4 * size_t(q.ntiles++)];
+        tl[0] = s0;
+        tl[1] = (a_end - s0 < 64) ? a_end - s0 : 64;
+        tl[2] = cu[b];
+        tl[3] = cu[b + 1] - cu[b];
+      }
+      a = a_end;
+    }
+    off += 4 * (size_t(T) / 64 + B + 1);
+  }
+  int32_t* dl = bf.lists;
+  SPD_CUDA_TRY(cudaMemcpyAsync(dl, hl.data(), off * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
+  if (int rc = bf16_to_f32_run(x, h, size_t(T) * D, st)) return rc;
+
+  int rc = SPD_OK;
+  for (int l = 0; l < L && !rc; ++l) {
+    const spd_model::Layer& W = m->layers[l];
+    const LayerLists& q = ll[l];
+    // attention sub-layer: norm of every row (K/V need all tokens) + compact copy of query rows
+    rc = rmsnorm_run(h, T, D, W.attn_norm, c.rms_eps, nullptr, bf.xa, q.na ? dl + q.amap : nullptr,
+                     bf.xq, st);
+    if (rc) break;
+    GemmProblem kvp{};
+    kvp.map_w = &W.m_kv;
+    kvp.x = bf.xa;
+    kvp.n_out = 2 * kvd;
+    kvp.n_tok = T;
+    kvp.k = D;
+    kvp.epi = EPI_ROPE_BF16;
+    kvp.out = bf.kv;
+    kvp.ldo = 2 * kvd;
+    kvp.pos = dl + pos_off;
+    kvp.inv_freq = m->inv_freq;
+    kvp.rope_rows = kvd;
+    kvp.head_dim = hd;
+    if ((rc = gemm_run(kvp, bf.gs, st))) break;
+    if (q.na > 0) {
+      GemmProblem qp = kvp;
+      qp.map_w = &W.m_q;
+      qp.x = bf.xq;
+      qp.n_out = qd;
+      qp.n_tok = q.na;
+      qp.out = bf.q;
+      qp.ldo = qd;
+      qp.pos = dl + q.apos;
+      qp.rope_rows = qd;
+      if ((rc = gemm_run(qp, bf.gs, st))) break;
+      if ((rc = attention_run(bf.q, qd, bf.kv, 2 * kvd, kvd, bf.o, qd,
+                              reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
+                              c.n_heads, c.n_kv_heads, hd, st)))
+        break;
+      GemmProblem op{};
+      op.map_w = &W.m_o;
+      op.x = bf.o;
+      op.n_out = D;
+      op.n_tok = q.na;
+      op.k = qd;
+      op.epi = EPI_ADD_F32;
+      op.out = h;
+      op.ldo = D;
+      op.rows = dl + q.arows;
+      if ((rc = gemm_run(op, bf.gs, st))) break;
+    }
+    if (q.nf > 0) {
+      if ((rc = rmsnorm_run(h, q.nf, D, W.ffn_norm, c.rms_eps, dl + q.frows, bf.y, nullptr, nullptr,
+                            st)))
+        break;
+      GemmProblem gp{};
+      gp.map_w = &W.m_gu;
+      gp.x = bf.y;
+      gp.n_out = m->gu_rows;
+      gp.n_tok = q.nf;
+      gp.k = D;
+      gp.epi = EPI_SWIGLU_BF16;
+      gp.out = bf.act;
+      gp.ldo = c.d_ffn;
+      gp.out_cols = c.d_ffn;
+      if ((rc = gemm_run(gp, bf.gs, st))) break;
+      GemmProblem dp{};
+      dp.map_w = &W.m_d;
+      dp.x = bf.act;
+      dp.n_out = D;
+      dp.n_tok = q.nf;
+      dp.k = c.d_ffn;
+      dp.epi = EPI_ADD_F32;
+      dp.out = h;
+      dp.ldo = D;
+      dp.rows = dl + q.frows;
+      if ((rc = gemm_run(dp, bf.gs, st))) break;
+    }
+  }
+  if (rc) return rc;
+  if (logits) {
+    if ((rc = rmsnorm_run(h, B, D, m->final_norm, c.rms_eps, dl + last_off, bf.z, nullptr, nullptr, st)))
+      return rc;
+    GemmProblem lp{};
+    lp.map_w = &m->m_lm;
+    lp.x = bf.z;
+    lp.n_out = c.vocab;
+    lp.n_tok = B;
+    lp.k = D;
+    lp.epi = EPI_F32;
+    lp.out = logits;
+    lp.ldo = c.vocab;
+    if ((rc = gemm_run(lp, bf.gs, st))) return rc;
+  }
+  return SPD_OK;
+}

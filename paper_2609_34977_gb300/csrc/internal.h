@@ -1,0 +1,84 @@
+// Internal declarations shared by the translation units of libspider.so.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "spider.h"
+
+namespace spd {
+
+// ---- errors ----------------------------------------------------------------------------------
+int fail(int code, const char* fmt, ...);  // records the thread's message, returns code
+#define SPD_CUDA_TRY(expr)                                                              \
+  do {                                                                                  \
+    cudaError_t e_ = (expr);                                                            \
+    if (e_ != cudaSuccess)                                                              \
+      return ::spd::fail(SPD_ECUDA, "%s failed: %s (%s:%d)", #expr, cudaGetErrorString(e_), \
+                         __FILE__, __LINE__);                                           \
+  } while (0)
+
+// Clock budget of every bounded device-side wait (about half a second at 2 GHz).
+constexpr long long kWaitBudget = 1ll << 30;
+
+int num_sms();  // SM count of the current device
+
+// Bump allocator over a caller-provided workspace. The first 256 bytes hold the status word.
+struct Carve {
+  uint8_t* base;
+  size_t used = 256;
+  size_t cap;
+  explicit Carve(void* b, size_t c) : base(static_cast<uint8_t*>(b)), cap(c) {}
+  template <typename T>
+  T* take(size_t n) {
+    used = (used + 255) & ~size_t(255);
+    T* p = reinterpret_cast<T*>(base ? base + used : nullptr);
+    used += n * sizeof(T);
+    return p;
+  }
+  bool fits() const { return used <= cap; }
+  int* status() const { return reinterpret_cast<int*>(base); }
+};
+
+// ---- GEMM (tcgen05) --------------------------------------------------------------------------
+enum Epi : int {
+  EPI_F32 = SPD_EPI_F32,
+  EPI_BF16 = SPD_EPI_BF16,
+  EPI_BIAS_BF16 = SPD_EPI_BIAS_BF16,
+  EPI_BIAS_GELU_BF16 = SPD_EPI_BIAS_GELU_BF16,
+  EPI_ADD_F32 = SPD_EPI_ADD_F32,
+  EPI_ROPE_BF16 = 16,  // rotary embedding on weight rows [0, rope_rows) laid out in rotary pairs
+  EPI_SWIGLU_BF16 = 17 // SiLU(gate) * up from weight rows interleaved in gate/up half-warps
+};
+
+struct GemmProblem {
+  const CUtensorMap* map_w;  // weights [n_out][k] bf16, box 64 x 128
+  const void* w;             // (for map creation when map_w is null)
+  const void* x;             // activations [n_tok][k] bf16
+  int n_out, n_tok, k;
+  int epi;
+  void* out;
+  int ldo;
+  const int32_t* rows;       // output row of token t (null = t)
+  const uint16_t* bias;      // [n_out] bf16
+  const int32_t* pos;        // rotary position of token t
+  const float* inv_freq;     // [head_dim / 2]
+  int rope_rows, head_dim;
+  int out_cols;              // valid output columns (SwiGLU: d_ffn)
+};
+
+// Scratch of split-K partial sums and per-tile arrival counters.
+struct GemmScratch {
+  float* partial;
+  size_t partial_floats;
+  int* counters;
+  int n_counters;
+  int* status;
+};
+
+size_t gemm_scratch_bytes();                           // fixed-capacity scratch for any problem
+int make_weight_map(CUtensorMap* map, const void* w, int n_out, int k);
+int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream);
+
+}  // namespace spd

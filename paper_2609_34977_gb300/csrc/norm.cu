@@ -1,0 +1,111 @@
+// Memory-bound row kernels of the prefill: RMSNorm of the fp32 residual stream into bf16 GEMM
+// operands (optionally gathering/scattering rows), bf16 -> fp32 residual initialisation, and bf16
+// row scatter for sequence assembly.
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "internal.h"
+
+namespace spd {
+namespace {
+
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = 0.0f;
+#pragma unroll
+  for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+  return t;
+}
+
+// out[orow(i)] = bf16(gain * h[irow(i)] / sqrt(mean(h^2) + eps)); out2[map2[irow]] gets the same
+// row when map2 is given and map2[irow] >= 0 (compact copy of the attention-active rows).
+__global__ void __launch_bounds__(kThreads)
+    rmsnorm_kernel(const float* __restrict__ h, int D, const uint16_t* __restrict__ gain, float eps,
+                   const int32_t* __restrict__ in_rows, __nv_bfloat16* __restrict__ out,
+                   const int32_t* __restrict__ map2, __nv_bfloat16* __restrict__ out2) {
+  __shared__ float red[kThreads / 32];
+  const int i = blockIdx.x;
+  const int r = in_rows ? in_rows[i] : i;
+  const float4* src = reinterpret_cast<const float4*>(h + size_t(r) * D);
+  const int n4 = D / 4;
+  float ss = 0.0f;
+  for (int c = threadIdx.x; c < n4; c += kThreads) {
+    const float4 v = src[c];
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  const float tot = block_sum(ss, red);
+  const float inv = rsqrtf(tot / float(D) + eps);
+  const int r2 = map2 ? map2[r] : -1;
+  const ushort4* g4 = reinterpret_cast<const ushort4*>(gain);
+  for (int c = threadIdx.x; c < n4; c += kThreads) {
+    const float4 v = src[c];
+    const ushort4 gg = g4[c];
+    __nv_bfloat162 lo = __floats2bfloat162_rn(
+        v.x * inv * __bfloat162float(__ushort_as_bfloat16(gg.x)),
+        v.y * inv * __bfloat162float(__ushort_as_bfloat16(gg.y)));
+    __nv_bfloat162 hi = __floats2bfloat162_rn(
+        v.z * inv * __bfloat162float(__ushort_as_bfloat16(gg.z)),
+        v.w * inv * __bfloat162float(__ushort_as_bfloat16(gg.w)));
+    uint2 pk;
+    pk.x = *reinterpret_cast<uint32_t*>(&lo);
+    pk.y = *reinterpret_cast<uint32_t*>(&hi);
+    reinterpret_cast<uint2*>(out + size_t(i) * D)[c] = pk;
+    if (r2 >= 0) reinterpret_cast<uint2*>(out2 + size_t(r2) * D)[c] = pk;
+  }
+}
+
+__global__ void bf16_to_f32_kernel(const uint16_t* __restrict__ x, float* __restrict__ h, size_t n4) {
+  for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < n4;
+       i += size_t(gridDim.x) * blockDim.x) {
+    const ushort4 v = reinterpret_cast<const ushort4*>(x)[i];
+    reinterpret_cast<float4*>(h)[i] =
+        make_float4(__uint_as_float(uint32_t(v.x) << 16), __uint_as_float(uint32_t(v.y) << 16),
+                    __uint_as_float(uint32_t(v.z) << 16), __uint_as_float(uint32_t(v.w) << 16));
+  }
+}
+
+__global__ void scatter_rows_kernel(const uint16_t* __restrict__ src, int D,
+                                    const int32_t* __restrict__ rows, uint16_t* __restrict__ dst) {
+  const int i = blockIdx.x;
+  const uint4* s = reinterpret_cast<const uint4*>(src + size_t(i) * D);
+  uint4* d = reinterpret_cast<uint4*>(dst + size_t(rows[i]) * D);
+  for (int c = threadIdx.x; c < D / 8; c += blockDim.x) d[c] = s[c];
+}
+
+}  // namespace
+
+int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float eps,
+                const int32_t* in_rows, void* out, const int32_t* map2, void* out2,
+                cudaStream_t stream) {
+  if (n_rows <= 0) return SPD_OK;
+  rmsnorm_kernel<<<n_rows, kThreads, 0, stream>>>(h, D, gain, eps, in_rows,
+                                                  static_cast<__nv_bfloat16*>(out), map2,
+                                                  static_cast<__nv_bfloat16*>(out2));
+  SPD_CUDA_TRY(cudaGetLastError());
+  return SPD_OK;
+}
+
+int bf16_to_f32_run(const uint16_t* x, float* h, size_t n, cudaStream_t stream) {
+  if (n == 0) return SPD_OK;
+  const size_t n4 = n / 4;
+  const int blocks = int((n4 + 255) / 256 < 4096 ? (n4 + 255) / 256 : 4096);
+  bf16_to_f32_kernel<<<blocks, 256, 0, stream>>>(x, h, n4);
+  SPD_CUDA_TRY(cudaGetLastError());
+  return SPD_OK;
+}
+
+int scatter_rows_run(const uint16_t* src, int n_rows, int D, const int32_t* rows, uint16_t* dst,
+                     cudaStream_t stream) {
+  if (n_rows <= 0) return SPD_OK;
+  scatter_rows_kernel<<<n_rows, 128, 0, stream>>>(src, D, rows, dst);
+  SPD_CUDA_TRY(cudaGetLastError());
+  return SPD_OK;
+}
+
+}  // namespace spd

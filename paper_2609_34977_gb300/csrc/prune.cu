@@ -1,0 +1,624 @@
+// MSV-Prune (Sec. 4.1, Eq. 1-3; Alg. 1 stage 1) on the GPU, every tile independently.
+//
+//   rowstats     a_v = head-mean of the attention (Sec. 4.1.1); 1/||F_l,i|| for every tapped layer
+//   anchors      top-N_anc of a_v by a bitonic sort of (a_v desc, index asc) keys (Eq. 1);
+//                stable lists of anchor and non-anchor tokens by block prefix sums
+//   anchor_sim   a_i = max_p cos(F^L_i, F^L_p) over anchors: a tiled fp32 product, max via atomicMax
+//                on order-preserving integer keys (exact, order independent)
+//   kmeans       Lloyd on raw F^L of the non-anchor tokens, fixed-order fp32 sums; Eq. 2 quotas
+//   cluster_sums per cluster and layer, sum_j F_l,j / ||F_l,j|| in token order
+//   scores       s_i = [sum_l w_l f_i . (S_l,k - f_i)] / (|C_k| - 1) + a_i + (A_k - a_i) / (|C_k| - 1),
+//                the per-token mean of Eq. 3's S_ij over the other members of its cluster
+//   select       per cluster the N_k lowest (score, index) keys; kept = anchors + selected, compacted
+//                in ascending index order
+// All reductions run in a fixed order, so repeated runs give identical bits.
+#include <cuda_bf16.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace spd {
+
+struct PruneDims {
+  int n_tiles, n_tok, off, n, d, L, fin, H, form, n_att, keep, K, iters, n_anc, n_cmp, m;
+  float w[SPD_MAX_FEAT_LAYERS];
+  const float* feat[SPD_MAX_FEAT_LAYERS];
+};
+
+struct PruneWs {
+  float* a_v;       // [T][n]
+  float* inv;       // [L][T][n]
+  int8_t* role;     // [T][n] 1 anchor
+  int32_t* alist;   // [T][n_anc]
+  int32_t* ulist;   // [T][m]
+  uint32_t* asim;   // [T][n] ordered keys of a_i
+  int32_t* assign;  // [T][m]
+  int32_t* counts;  // [T][16]
+  int32_t* quotas;  // [T][16]
+  float* asum;      // [T][16]
+  float* csum;      // [T][L][K][d]
+  float* score;     // [T][m]
+  int* status;
+};
+
+namespace {
+
+__device__ __forceinline__ uint32_t ordered_key(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float ordered_val(uint32_t u) {
+  return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+
+// Ascending bitonic sort of N (power of two) keys in shared memory by the whole block.
+__device__ void bitonic_sort(uint64_t* keys, int N) {
+  for (int k = 2; k <= N; k <<= 1) {
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = threadIdx.x; i < N; i += blockDim.x) {
+        const int ixj = i ^ j;
+        if (ixj > i) {
+          const bool up = (i & k) == 0;
+          const uint64_t a = keys[i], b = keys[ixj];
+          if ((a > b) == up) {
+            keys[i] = b;
+            keys[ixj] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
+// Exclusive prefix sum of one int per thread over a block of 1024 threads.
+__device__ int block_scan_excl(int v, int* tmp, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, off);
+    if (lane >= off) x += y;
+  }
+  if (lane == 31) tmp[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = (lane < (int)(blockDim.x >> 5)) ? tmp[lane] : 0;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, off);
+      if (lane >= off) w += y;
+    }
+    tmp[lane] = w;  // inclusive totals of warps
+  }
+  __syncthreads();
+  const int before = (warp ? tmp[warp - 1] : 0) + x - v;
+  if (total) *total = tmp[(blockDim.x >> 5) - 1];
+  __syncthreads();
+  return before;
+}
+
+__device__ __forceinline__ const float* feat_row(const PruneDims& p, int l, int t, int i) {
+  return p.feat[l] + (size_t(t) * p.n_tok + p.off + i) * p.d;
+}
+
+// ---- 1. a_v and inverse norms ---------------------------------------------------------------
+__global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float* __restrict__ attn,
+                                                       PruneWs w) {
+  const int t = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int i = blockIdx.x * 8 + warp;
+  if (i >= p.n) return;
+  for (int l = 0; l < p.L; ++l) {
+    const float4* r = reinterpret_cast<const float4*>(feat_row(p, l, t, i));
+    float ss = 0.0f;
+    for (int c = lane; c < p.d / 4; c += 32) {
+      const float4 v = r[c];
+      ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+    }
+    ss = warp_sum(ss);
+    if (lane == 0) w.inv[(size_t(l) * p.n_tiles + t) * p.n + i] = 1.0f / sqrtf(ss);
+  }
+  if (lane == 0) {
+    const int col = (p.form == 0) ? 1 + i : i;
+    float s = 0.0f;
+    for (int h = 0; h < p.H; ++h) s += attn[(size_t(t) * p.H + h) * p.n_att + col];
+    w.a_v[size_t(t) * p.n + i] = s / float(p.H);
+  }
+}
+
+// ---- 2. anchors (Eq. 1) and stable token lists ------------------------------------------------
+__global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
+  __shared__ uint64_t keys[4096];
+  __shared__ int tmp[32];
+  const int t = blockIdx.x;
+  int N = 1;
+  while (N < p.n) N <<= 1;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    uint64_t k = ~0ull;
+    if (i < p.n)
+      k = (uint64_t(~ordered_key(w.a_v[size_t(t) * p.n + i])) << 32) | uint32_t(i);
+    keys[i] = k;
+  }
+  __syncthreads();
+  bitonic_sort(keys, N);
+  int8_t* role = w.role + size_t(t) * p.n;
+  for (int i = threadIdx.x; i < p.n; i += blockDim.x) role[i] = 0;
+  __syncthreads();
+  for (int r = threadIdx.x; r < p.n_anc; r += blockDim.x) role[keys[r] & 0xffffffffu] = 1;
+  __syncthreads();
+  // stable lists: each thread owns 4 consecutive tokens
+  const int base = threadIdx.x * 4;
+  int na = 0;
+  for (int q = 0; q < 4; ++q)
+    if (base + q < p.n) na += role[base + q];
+  const int nu = ((base < p.n) ? min(4, p.n - base) : 0) - na;
+  const int a0 = block_scan_excl(na, tmp, nullptr);
+  const int u0 = block_scan_excl(nu, tmp, nullptr);
+  int ai = a0, ui = u0;
+  const uint32_t init = (p.n_anc == 0) ? ordered_key(0.0f) : 0u;
+  for (int q = 0; q < 4; ++q) {
+    const int i = base + q;
+    if (i >= p.n) break;
+    if (role[i]) w.alist[size_t(t) * p.n_anc + ai++] = i;
+    else w.ulist[size_t(t) * p.m + ui++] = i;
+    w.asim[size_t(t) * p.n + i] = init;
+  }
+}
+
+// ---- 3. a_i = max over anchors of cos(F^L_i, F^L_p) -------------------------------------------
+__global__ void __launch_bounds__(256) anchor_sim_kernel(PruneDims p, PruneWs w) {
+  __shared__ float Us[32][33], As[32][33];
+  __shared__ float red[8][32];
+  const int t = blockIdx.z, tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const int u0 = blockIdx.x * 32, p0 = blockIdx.y * 32;
+  const int* ul = w.ulist + size_t(t) * p.m;
+  const int* al = w.alist + size_t(t) * p.n_anc;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int d0 = 0; d0 < p.d; d0 += 32) {
+    for (int e = threadIdx.x; e < 1024; e += 256) {
+      const int r = e >> 5, c = e & 31;
+      const bool dc = d0 + c < p.d;
+      Us[r][c] = (u0 + r < p.m && dc) ? feat_row(p, p.fin, t, ul[u0 + r])[d0 + c] : 0.0f;
+      As[r][c] = (p0 + r < p.n_anc && dc) ? feat_row(p, p.fin, t, al[p0 + r])[d0 + c] : 0.0f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int c = 0; c < 32; ++c) {
+      const float u = Us[tx][c];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[q] += u * As[ty + 8 * q][c];
+    }
+    __syncthreads();
+  }
+  float best = -INFINITY;
+  if (u0 + tx < p.m) {
+    const float iu = w.inv[(size_t(p.fin) * p.n_tiles + t) * p.n + ul[u0 + tx]];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int pa = p0 + ty + 8 * q;
+      if (pa < p.n_anc) {
+        const float ia = w.inv[(size_t(p.fin) * p.n_tiles + t) * p.n + al[pa]];
+        best = fmaxf(best, acc[q] * iu * ia);
+      }
+    }
+  }
+  red[ty][tx] = best;
+  __syncthreads();
+  if (ty == 0 && u0 + tx < p.m) {
+    for (int q = 1; q < 8; ++q) best = fmaxf(best, red[q][tx]);
+    atomicMax(&w.asim[size_t(t) * p.n + ul[u0 + tx]], ordered_key(best));
+  }
+}
+
+// ---- 4. K-means (Lloyd) and Eq. 2 quotas ------------------------------------------------------
+__device__ void compute_quotas(const int* sizes, int K, int n_cmp, int* quota) {
+  int total = 0, nonempty = 0;
+  for (int k = 0; k < K; ++k) {
+    quota[k] = 0;
+    total += sizes[k];
+    nonempty += sizes[k] > 0;
+  }
+  if (n_cmp <= 0 || total == 0) return;
+  int order[SPD_MAX_CLUSTERS];
+  if (n_cmp < nonempty) {  // one each to the largest clusters, ties to the lower k
+    for (int k = 0; k < K; ++k) order[k] = k;
+    for (int a = 1; a < K; ++a)
+      for (int b = a; b > 0 && (sizes[order[b]] > sizes[order[b - 1]]); --b) {
+        const int x = order[b]; order[b] = order[b - 1]; order[b - 1] = x;
+      }
+    for (int r = 0; r < n_cmp; ++r) quota[order[r]] = 1;
+    return;
+  }
+  long long rem[SPD_MAX_CLUSTERS];
+  int sum = 0;
+  for (int k = 0; k < K; ++k) {
+    const long long num = (long long)n_cmp * sizes[k];
+    rem[k] = num % total;
+    if (sizes[k] > 0) {
+      int q = int((2 * num + total) / (2LL * total));  // round half away from zero
+      if (q < 1) q = 1;
+      if (q > sizes[k]) q = sizes[k];
+      quota[k] = q;
+    }
+    sum += quota[k];
+  }
+  if (sum < n_cmp) {  // descending fractional part, ties to the lower k
+    for (int k = 0; k < K; ++k) order[k] = k;
+    for (int a = 1; a < K; ++a)
+      for (int b = a; b > 0 && rem[order[b]] > rem[order[b - 1]]; --b) {
+        const int x = order[b]; order[b] = order[b - 1]; order[b - 1] = x;
+      }
+    while (sum < n_cmp)
+      for (int r = 0; r < K && sum < n_cmp; ++r)
+        if (quota[order[r]] < sizes[order[r]]) { ++quota[order[r]]; ++sum; }
+  } else if (sum > n_cmp) {  // ascending fractional part, ties to the higher k
+    for (int k = 0; k < K; ++k) order[k] = K - 1 - k;
+    for (int a = 1; a < K; ++a)
+      for (int b = a; b > 0 && rem[order[b]] < rem[order[b - 1]]; --b) {
+        const int x = order[b]; order[b] = order[b - 1]; order[b - 1] = x;
+      }
+    while (sum > n_cmp)
+      for (int r = 0; r < K && sum > n_cmp; ++r)
+        if (quota[order[r]] > 1) { --quota[order[r]]; --sum; }
+  }
+}
+
+__global__ void __launch_bounds__(1024) kmeans_kernel(PruneDims p, PruneWs w) {
+  extern __shared__ float ksm[];
+  float* cent = ksm;                     // [K][d]
+  float* sums = ksm + size_t(p.K) * p.d; // [K][d]
+  int8_t* asg = reinterpret_cast<int8_t*>(sums + size_t(p.K) * p.d);  // [m]
+  __shared__ int counts[SPD_MAX_CLUSTERS];
+  __shared__ int changed;
+  const int t = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m = p.m, K = p.K, D = p.d;
+  const int* ul = w.ulist + size_t(t) * m;
+  if (m > 0) {
+    for (int e = threadIdx.x; e < K * D; e += blockDim.x) {
+      const int k = e / D, c = e % D;
+      cent[e] = feat_row(p, p.fin, t, ul[(k * m) / K])[c];
+    }
+    __syncthreads();
+    for (int it = 0; it < p.iters; ++it) {
+      if (threadIdx.x == 0) changed = 0;
+      __syncthreads();
+      for (int j = warp; j < m; j += 32) {
+        const float* x = feat_row(p, p.fin, t, ul[j]);
+        float part[SPD_MAX_CLUSTERS];
+#pragma unroll
+        for (int k = 0; k < SPD_MAX_CLUSTERS; ++k) part[k] = 0.0f;
+        for (int c = lane; c < D; c += 32) {
+          const float xv = x[c];
+#pragma unroll
+          for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
+            if (k < K) {
+              const float df = xv - cent[k * D + c];
+              part[k] += df * df;
+            }
+        }
+        int best = 0;
+        float bd = 0.0f;
+#pragma unroll
+        for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
+          if (k < K) {
+            const float dk = warp_sum(part[k]);
+            if (k == 0 || dk < bd) { bd = dk; best = k; }
+          }
+        if (lane == 0) {
+          if (it == 0 || asg[j] != best) changed = 1;
+          asg[j] = int8_t(best);
+        }
+      }
+      __syncthreads();
+      if (it > 0 && !changed) break;
+      if (threadIdx.x < K) counts[threadIdx.x] = 0;
+      __syncthreads();
+      for (int j = threadIdx.x; j < m; j += blockDim.x) atomicAdd(&counts[asg[j]], 1);
+      for (int e = threadIdx.x; e < K * D; e += blockDim.x) sums[e] = 0.0f;
+      __syncthreads();
+      for (int c = threadIdx.x; c < D; c += blockDim.x)
+        for (int j = 0; j < m; ++j) sums[asg[j] * D + c] += feat_row(p, p.fin, t, ul[j])[c];
+      __syncthreads();
+      for (int e = threadIdx.x; e < K * D; e += blockDim.x) {
+        const int k = e / D;
+        if (counts[k] > 0) cent[e] = sums[e] / float(counts[k]);
+      }
+      __syncthreads();
+    }
+  }
+  // final sizes, quotas, and per-cluster sums of a_j
+  if (threadIdx.x < K) counts[threadIdx.x] = 0;
+  __syncthreads();
+  for (int j = threadIdx.x; j < m; j += blockDim.x) {
+    atomicAdd(&counts[asg[j]], 1);
+    w.assign[size_t(t) * m + j] = asg[j];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int q[SPD_MAX_CLUSTERS];
+    compute_quotas(counts, K, p.n_cmp, q);
+    for (int k = 0; k < K; ++k) {
+      w.counts[t * 16 + k] = counts[k];
+      w.quotas[t * 16 + k] = q[k];
+    }
+  }
+  if (warp < K) {
+    float s = 0.0f;
+    for (int j = lane; j < m; j += 32)
+      if (asg[j] == warp) s += ordered_val(w.asim[size_t(t) * p.n + ul[j]]);
+    s = warp_sum(s);
+    if (lane == 0) w.asum[t * 16 + warp] = s;
+  }
+}
+
+// ---- 5. per-cluster sums of unit feature rows ----------------------------------------------
+__global__ void __launch_bounds__(128) cluster_sum_kernel(PruneDims p, PruneWs w) {
+  extern __shared__ int csm[];
+  int* ul = csm;                                       // [m]
+  int8_t* asg = reinterpret_cast<int8_t*>(csm + p.m);  // [m]
+  const int t = blockIdx.y, c = blockIdx.x * 128 + threadIdx.x;
+  for (int j = threadIdx.x; j < p.m; j += 128) {
+    ul[j] = w.ulist[size_t(t) * p.m + j];
+    asg[j] = int8_t(w.assign[size_t(t) * p.m + j]);
+  }
+  __syncthreads();
+  if (c >= p.d) return;
+  for (int k = 0; k < p.K; ++k) {
+    float acc[SPD_MAX_FEAT_LAYERS] = {0.f, 0.f, 0.f, 0.f};
+    for (int j = 0; j < p.m; ++j) {
+      if (asg[j] != k) continue;
+#pragma unroll
+      for (int l = 0; l < SPD_MAX_FEAT_LAYERS; ++l)
+        if (l < p.L)
+          acc[l] += feat_row(p, l, t, ul[j])[c] * w.inv[(size_t(l) * p.n_tiles + t) * p.n + ul[j]];
+    }
+#pragma unroll
+    for (int l = 0; l < SPD_MAX_FEAT_LAYERS; ++l)
+      if (l < p.L) w.csum[((size_t(t) * p.L + l) * p.K + k) * p.d + c] = acc[l];
+  }
+}
+
+// ---- 6. per-token Eq. 3 scores ----------------------------------------------------------------
+__global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
+  const int t = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j = blockIdx.x * 8 + warp;
+  if (j >= p.m) return;
+  const int i = w.ulist[size_t(t) * p.m + j];
+  const int k = w.assign[size_t(t) * p.m + j];
+  const int cnt = w.counts[t * 16 + k];
+  const float ai = ordered_val(w.asim[size_t(t) * p.n + i]);
+  float s;
+  if (cnt <= 1) {
+    s = 2.0f * ai;
+  } else {
+    float acc = 0.0f;
+    for (int l = 0; l < p.L; ++l) {
+      const float wl = (l == p.fin) ? 1.0f : p.w[l];
+      if (wl == 0.0f) continue;
+      const float* x = feat_row(p, l, t, i);
+      const float iv = w.inv[(size_t(l) * p.n_tiles + t) * p.n + i];
+      const float* cs = w.csum + ((size_t(t) * p.L + l) * p.K + k) * p.d;
+      float dot = 0.0f;
+      for (int c = lane; c < p.d; c += 32) {
+        const float u = x[c] * iv;
+        dot += u * (cs[c] - u);
+      }
+      acc += wl * warp_sum(dot);
+    }
+    const float inv_c = 1.0f / float(cnt - 1);
+    s = acc * inv_c + ai + (w.asum[t * 16 + k] - ai) * inv_c;
+  }
+  if (lane == 0) w.score[size_t(t) * p.m + j] = s;
+}
+
+// ---- 7. per-cluster bottom-N_k, compaction, outputs -------------------------------------------
+__global__ void __launch_bounds__(1024) select_kernel(PruneDims p, PruneWs w, int32_t* keep_idx,
+                                                      uint8_t* kind, int8_t* cluster, float* scores) {
+  __shared__ uint64_t keys[4096];
+  __shared__ uint8_t kept[4096];
+  __shared__ int tmp[32];
+  __shared__ int seg[SPD_MAX_CLUSTERS + 1];
+  __shared__ int quota[SPD_MAX_CLUSTERS];
+  const int t = blockIdx.x, m = p.m;
+  const int* ul = w.ulist + size_t(t) * m;
+  int N = 1;
+  while (N < max(m, 1)) N <<= 1;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) {
+    uint64_t key = ~0ull;
+    if (j < m)
+      key = (uint64_t(w.assign[size_t(t) * m + j]) << 45) |
+            (uint64_t(ordered_key(w.score[size_t(t) * m + j])) << 13) | uint64_t(ul[j]);
+    keys[j] = key;
+  }
+  for (int i = threadIdx.x; i < p.n; i += blockDim.x) kept[i] = uint8_t(w.role[size_t(t) * p.n + i]);
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int k = 0; k < p.K; ++k) {
+      seg[k] = acc;
+      acc += w.counts[t * 16 + k];
+      quota[k] = w.quotas[t * 16 + k];
+    }
+    seg[p.K] = acc;
+  }
+  __syncthreads();
+  bitonic_sort(keys, N);
+  for (int r = threadIdx.x; r < m; r += blockDim.x) {
+    const int k = int(keys[r] >> 45);
+    if (r - seg[k] < quota[k]) kept[keys[r] & 0x1fffu] = 2;
+  }
+  __syncthreads();
+  const int base = threadIdx.x * 4;
+  int nk = 0;
+  for (int q = 0; q < 4; ++q)
+    if (base + q < p.n) nk += kept[base + q] != 0;
+  int pos = block_scan_excl(nk, tmp, nullptr);
+  for (int q = 0; q < 4; ++q) {
+    const int i = base + q;
+    if (i >= p.n) break;
+    if (kept[i]) {
+      if (pos < p.keep) keep_idx[size_t(t) * p.keep + pos] = i;
+      else set_status(w.status, SPD_EINVAL);
+      ++pos;
+    }
+    if (kind) kind[size_t(t) * p.n + i] = kept[i];
+    if (kept[i] == 1) {
+      if (cluster) cluster[size_t(t) * p.n + i] = -1;
+      if (scores) scores[size_t(t) * p.n + i] = INFINITY;
+    }
+  }
+  for (int j = threadIdx.x; j < m; j += blockDim.x) {
+    if (cluster) cluster[size_t(t) * p.n + ul[j]] = int8_t(w.assign[size_t(t) * m + j]);
+    if (scores) scores[size_t(t) * p.n + ul[j]] = w.score[size_t(t) * m + j];
+  }
+}
+
+__global__ void gather_bf16_kernel(const float* __restrict__ src, int n_tok, int d, int off,
+                                   const int32_t* __restrict__ idx, int keep,
+                                   __nv_bfloat16* __restrict__ dst, int* status) {
+  const int j = blockIdx.x, t = blockIdx.y;
+  const int i = idx[size_t(t) * keep + j];
+  if (i < 0 || i >= n_tok - off) {
+    if (threadIdx.x == 0) set_status(status, SPD_EINVAL);
+    return;
+  }
+  const float4* s = reinterpret_cast<const float4*>(src + (size_t(t) * n_tok + off + i) * d);
+  uint2* o = reinterpret_cast<uint2*>(dst + (size_t(t) * keep + j) * d);
+  for (int c = threadIdx.x; c < d / 4; c += blockDim.x) {
+    const float4 v = s[c];
+    __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+    o[c] = make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+  }
+}
+
+int validate(const spd_prune_cfg* c, PruneDims* p) {
+  if (!c) return fail(SPD_EINVAL, "null prune config");
+  if (c->n_tiles < 1 || c->n_layers < 1 || c->n_layers > SPD_MAX_FEAT_LAYERS)
+    return fail(SPD_EINVAL, "n_tiles >= 1 and n_layers in [1, %d] required", SPD_MAX_FEAT_LAYERS);
+  if (c->final_layer < 0 || c->final_layer >= c->n_layers) return fail(SPD_EINVAL, "bad final_layer");
+  const int off = c->has_cls ? 1 : 0;
+  const int n = c->n_tok - off;
+  if (n < 1 || n > 4096) return fail(SPD_EINVAL, "patch count must lie in [1, 4096]");
+  if (c->d_feat < 4 || c->d_feat % 4 || c->d_feat > 4096)
+    return fail(SPD_EINVAL, "d_feat must be a multiple of 4 in [4, 4096]");
+  if (c->n_heads < 1) return fail(SPD_EINVAL, "n_heads >= 1 required");
+  if (c->attn_form != 0 && c->attn_form != 1) return fail(SPD_EINVAL, "attn_form must be 0 or 1");
+  if (c->attn_form == 0 && !c->has_cls) return fail(SPD_EINVAL, "CLS-row attention needs has_cls");
+  if (c->keep < 1 || c->keep > n) return fail(SPD_EINVAL, "keep must lie in [1, n_patch]");
+  if (c->n_clusters < 1 || c->n_clusters > SPD_MAX_CLUSTERS) return fail(SPD_EINVAL, "bad n_clusters");
+  if (size_t(c->n_clusters) * c->d_feat > 24576)
+    return fail(SPD_EINVAL, "n_clusters * d_feat must not exceed 24576");
+  if (c->kmeans_iters < 1) return fail(SPD_EINVAL, "kmeans_iters >= 1 required");
+  if (!(c->anchor_ratio >= 0.0 && c->anchor_ratio <= 1.0))
+    return fail(SPD_EINVAL, "anchor_ratio must lie in [0, 1]");
+  p->n_tiles = c->n_tiles;
+  p->n_tok = c->n_tok;
+  p->off = off;
+  p->n = n;
+  p->d = c->d_feat;
+  p->L = c->n_layers;
+  p->fin = c->final_layer;
+  p->H = c->n_heads;
+  p->form = c->attn_form;
+  p->n_att = c->attn_form == 0 ? c->n_tok : n;
+  p->keep = c->keep;
+  p->K = c->n_clusters;
+  p->iters = c->kmeans_iters;
+  p->n_anc = int(floor(double(c->keep) * c->anchor_ratio + 0.5));
+  if (p->n_anc > c->keep) p->n_anc = c->keep;
+  p->n_cmp = c->keep - p->n_anc;
+  p->m = n - p->n_anc;
+  for (int l = 0; l < SPD_MAX_FEAT_LAYERS; ++l) {
+    p->w[l] = c->layer_weight[l];
+    p->feat[l] = nullptr;
+  }
+  return SPD_OK;
+}
+
+PruneWs carve(const PruneDims& p, Carve& cv) {
+  PruneWs w;
+  const size_t T = p.n_tiles;
+  w.status = cv.status();
+  w.a_v = cv.take<float>(T * p.n);
+  w.inv = cv.take<float>(T * p.n * p.L);
+  w.role = cv.take<int8_t>(T * p.n);
+  w.alist = cv.take<int32_t>(T * (p.n_anc + 1));
+  w.ulist = cv.take<int32_t>(T * (p.m + 1));
+  w.asim = cv.take<uint32_t>(T * p.n);
+  w.assign = cv.take<int32_t>(T * (p.m + 1));
+  w.counts = cv.take<int32_t>(T * 16);
+  w.quotas = cv.take<int32_t>(T * 16);
+  w.asum = cv.take<float>(T * 16);
+  w.csum = cv.take<float>(T * p.L * p.K * p.d);
+  w.score = cv.take<float>(T * (p.m + 1));
+  return w;
+}
+
+}  // namespace
+}  // namespace spd
+
+using namespace spd;
+
+extern "C" size_t spd_prune_workspace_size(const spd_prune_cfg* cfg) {
+  PruneDims p;
+  if (validate(cfg, &p)) return 0;
+  Carve cv(nullptr, ~size_t(0));
+  carve(p, cv);
+  return cv.used;
+}
+
+extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, const float* attn,
+                         int32_t* keep_idx, uint8_t* kind, int8_t* cluster, float* scores, void* ws,
+                         size_t ws_bytes, void* stream_) {
+  PruneDims p;
+  if (int rc = validate(cfg, &p)) return rc;
+  if (!feats || !attn || !keep_idx || !ws) return fail(SPD_EINVAL, "null buffer");
+  for (int l = 0; l < p.L; ++l) {
+    if (!feats[l] || (reinterpret_cast<uintptr_t>(feats[l]) & 15))
+      return fail(SPD_EINVAL, "feature pointer %d null or not 16-byte aligned", l);
+    p.feat[l] = feats[l];
+  }
+  Carve cv(ws, ws_bytes);
+  PruneWs w = carve(p, cv);
+  if (!cv.fits()) return fail(SPD_ENOSPC, "prune workspace too small (%zu < %zu)", ws_bytes, cv.used);
+  cudaStream_t st = static_cast<cudaStream_t>(stream_);
+  const int T = p.n_tiles;
+  rowstats_kernel<<<dim3((p.n + 7) / 8, T), 256, 0, st>>>(p, attn, w);
+  anchor_kernel<<<T, 1024, 0, st>>>(p, w);
+  if (p.n_anc > 0 && p.m > 0)
+    anchor_sim_kernel<<<dim3((p.m + 31) / 32, (p.n_anc + 31) / 32, T), 256, 0, st>>>(p, w);
+  const size_t ksmem = size_t(2) * p.K * p.d * sizeof(float) + p.m + 16;
+  static bool attr = false;
+  if (!attr) {
+    SPD_CUDA_TRY(cudaFuncSetAttribute(kmeans_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      2 * 24576 * 4 + 4096 + 16));
+    attr = true;
+  }
+  kmeans_kernel<<<T, 1024, ksmem, st>>>(p, w);
+  if (p.m > 0) {
+    cluster_sum_kernel<<<dim3((p.d + 127) / 128, T), 128, size_t(p.m) * 5 + 16, st>>>(p, w);
+    score_kernel<<<dim3((p.m + 7) / 8, T), 256, 0, st>>>(p, w);
+  }
+  select_kernel<<<T, 1024, 0, st>>>(p, w, keep_idx, kind, cluster, scores);
+  SPD_CUDA_TRY(cudaGetLastError());
+  return SPD_OK;
+}
+
+extern "C" int spd_gather_rows_bf16(const float* src, int n_tiles, int n_tok, int d, int row_offset,
+                                    const int32_t* idx, int keep, uint16_t* dst, void* ws,
+                                    void* stream_) {
+  if (!src || !idx || !dst || n_tiles < 1 || keep < 1 || d < 4 || d % 4 || row_offset < 0 ||
+      row_offset >= n_tok)
+    return fail(SPD_EINVAL, "bad gather arguments");
+  gather_bf16_kernel<<<dim3(keep, n_tiles), 128, 0, static_cast<cudaStream_t>(stream_)>>>(
+      src, n_tok, d, row_offset, idx, keep, reinterpret_cast<__nv_bfloat16*>(dst),
+      ws ? static_cast<int*>(ws) : nullptr);
+  SPD_CUDA_TRY(cudaGetLastError());
+  return SPD_OK;
+}

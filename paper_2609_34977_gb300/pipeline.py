@@ -1,0 +1,108 @@
+"""One SPIDER prefill step (Alg. 1) over a batch of requests, as a sequence of libspider.so calls.
+
+This module only owns buffers and workspaces and calls the C ABI in order. Every computation runs
+in the CUDA library:
+
+    spd_prune              MSV-Prune of every tile (Sec. 4.1)
+    spd_gather_rows_bf16   kept final-layer rows -> bf16
+    spd_project            LLaVA projector into the decoder input rows (or a row copy when the
+                           vision width equals the decoder width and no projector is configured)
+    spd_scatter_rows       text embeddings into their rows
+    spd_prefill            decoder prefill with the per-layer, per-token skip mask (Sec. 4.2-4.3)
+
+Sequence layout per request: [kept visual tokens of its tiles, in tile order and spatial order;
+text tokens]. Alg. 1 writes the text first; the order is a layout choice of the caller and the
+decoder treats both the same way.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import _native as N
+
+
+class SpiderPrefill:
+    """Buffers and workspaces for a fixed batch layout.
+
+    tiles_per_req[b] tiles and text_lens[b] text tokens for request b; `keep` tokens kept per tile
+    (keep = n_patch: no pruning, the dense baseline). skip_mask [L][T] host uint8 or None.
+    """
+
+    def __init__(self, model: N.SpdModel, *, n_patch: int, has_cls: bool, d_vis: int,
+                 n_feat_layers: int, final_layer: int, n_heads_vis: int, attn_form: int,
+                 keep: int, tiles_per_req, text_lens, n_clusters: int = 4, kmeans_iters: int = 10,
+                 anchor_ratio: float = 0.7, layer_weight=None, device: str = "cuda"):
+        self.model = model
+        cfg = model.cfg
+        self.D = cfg["d_model"]
+        self.tiles_per_req = list(tiles_per_req)
+        self.text_lens = list(text_lens)
+        self.n_tiles = int(sum(self.tiles_per_req))
+        self.keep = keep
+        self.n_patch = n_patch
+        self.n_tok = n_patch + (1 if has_cls else 0)
+        self.d_vis = d_vis
+        self.B = len(self.text_lens)
+        self.prune_cfg = N.prune_cfg(self.n_tiles, self.n_tok, d_vis, n_feat_layers, final_layer,
+                                     n_heads_vis, keep, has_cls=has_cls, attn_form=attn_form,
+                                     n_clusters=n_clusters, kmeans_iters=kmeans_iters,
+                                     anchor_ratio=anchor_ratio, layer_weight=layer_weight)
+        self.has_projector = bool(cfg.get("d_proj"))
+        if not self.has_projector and d_vis != self.D:
+            raise ValueError("without a projector the vision width must equal d_model")
+        # sequence layout
+        vis_rows, text_rows, cu = [], [], [0]
+        row = 0
+        for b in range(self.B):
+            nv = self.tiles_per_req[b] * keep
+            vis_rows.extend(range(row, row + nv))
+            row += nv
+            text_rows.extend(range(row, row + self.text_lens[b]))
+            row += self.text_lens[b]
+            cu.append(row)
+        self.T = row
+        self.cu = np.array(cu, dtype=np.int32)
+        self.token_is_visual = np.zeros(self.T, dtype=bool)
+        self.token_is_visual[vis_rows] = True
+        dev = torch.device(device)
+        self.vis_rows = torch.tensor(vis_rows, dtype=torch.int32, device=dev)
+        self.text_rows = torch.tensor(text_rows, dtype=torch.int32, device=dev)
+        # buffers
+        self.keep_idx = torch.empty(self.n_tiles, keep, dtype=torch.int32, device=dev)
+        self.vis = torch.empty(self.n_tiles * keep, d_vis, dtype=torch.bfloat16, device=dev)
+        self.x = torch.empty(self.T, self.D, dtype=torch.bfloat16, device=dev)
+        self.h = torch.empty(self.T, self.D, dtype=torch.float32, device=dev)
+        self.logits = torch.empty(self.B, cfg["vocab"], dtype=torch.float32, device=dev)
+        self.ws_prune = torch.zeros(N.spd_prune_workspace_size(self.prune_cfg), dtype=torch.uint8,
+                                    device=dev)
+        self.ws_proj = (torch.zeros(N.spd_project_workspace_size(model, self.n_tiles * keep),
+                                    dtype=torch.uint8, device=dev) if self.has_projector else None)
+        self.ws_prefill = torch.zeros(N.spd_prefill_workspace_size(model, self.T, self.B),
+                                      dtype=torch.uint8, device=dev)
+
+    def run(self, feats, attn, text, skip_mask, stream=None):
+        """Enqueue one step on device inputs: feats (list of [n_tiles][n_tok][d_vis] fp32), attn,
+        text [sum(text_lens)][D] bf16. Returns the logits tensor [B][vocab] (device)."""
+        N.spd_prune(self.prune_cfg, feats, attn, self.keep_idx, ws=self.ws_prune, stream=stream)
+        fin = int(self.prune_cfg.final_layer)
+        N.spd_gather_rows_bf16(feats[fin], self.n_tiles, self.n_tok, self.d_vis,
+                               1 if self.prune_cfg.has_cls else 0, self.keep_idx, self.keep, self.vis,
+                               ws=self.ws_prune, stream=stream)
+        nv = self.n_tiles * self.keep
+        if self.has_projector:
+            N.spd_project(self.model, self.vis, nv, self.vis_rows, self.x, self.ws_proj, stream=stream)
+        else:
+            N.spd_scatter_rows(self.model, self.vis, nv, self.vis_rows, self.x, stream=stream)
+        if len(self.text_rows):
+            N.spd_scatter_rows(self.model, text, len(self.text_rows), self.text_rows, self.x,
+                               stream=stream)
+        N.spd_prefill(self.model, self.x, self.T, self.cu, skip_mask, self.h, self.logits,
+                      self.ws_prefill, stream=stream)
+        return self.logits
+
+    def status(self) -> int:
+        """First device-side failure recorded by any call of this pipeline (0 = none)."""
+        codes = [N.spd_workspace_status(w) for w in (self.ws_prune, self.ws_proj, self.ws_prefill)
+                 if w is not None]
+        return next((c for c in codes if c), 0)

@@ -1,0 +1,77 @@
+"""Host-side checks of libspider.so (no GPU needed): the library loads, exports every entry point
+include/spider.h declares, and its host-only logic (plan expansion, argument validation) matches
+the oracle."""
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import decoder as od
+from paper_2609_34977_gb300 import _native as N
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(N.LIB_PATH):
+        from paper_2609_34977_gb300 import build
+        build.build()
+    return N.lib()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "spider.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(spd_\w+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 15
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(N.EXPORTS)
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_adaptive_plan_matches_oracle(lib, seed):
+    r = np.random.default_rng(seed)
+    T, L = 50, 7
+    admit = r.integers(-1, L, size=T).astype(np.int16)
+    target = r.integers(1, 3, size=T).astype(np.uint8)
+    np.testing.assert_array_equal(N.spd_plan_adaptive(L, admit, target),
+                                  od.expand_adaptive_plan(admit, target, L))
+
+
+def test_static_plan_matches_oracle(lib):
+    lm = np.array([0, 2, 1, 3], dtype=np.uint8)
+    sel = np.array([1, 0, 1, 1, 0], dtype=np.uint8)
+    np.testing.assert_array_equal(N.spd_plan_static(lm, sel), od.expand_static_plan(lm, sel))
+
+
+def test_plan_rejects_bad_target(lib):
+    with pytest.raises(N.SpiderError) as e:
+        N.spd_plan_adaptive(3, np.array([0], np.int16), np.array([5], np.uint8))
+    assert e.value.code == N.SPD_EINVAL
+
+
+def test_prune_config_validation(lib):
+    good = N.prune_cfg(1, 577, 256, 3, 2, 8, 64)
+    assert N.spd_prune_workspace_size(good) > 0
+    for bad in (N.prune_cfg(1, 577, 256, 3, 3, 8, 64),      # final layer out of range
+                N.prune_cfg(1, 577, 250, 3, 2, 8, 64),      # d not a multiple of 4
+                N.prune_cfg(1, 577, 256, 3, 2, 8, 577),     # keep > n_patch
+                N.prune_cfg(1, 577, 256, 3, 2, 8, 64, n_clusters=17),
+                N.prune_cfg(1, 577, 256, 3, 2, 8, 64, anchor_ratio=1.5),
+                N.prune_cfg(1, 576, 256, 3, 2, 8, 64, has_cls=False, attn_form=0)):
+        assert N.spd_prune_workspace_size(bad) == 0
+
+
+def test_workspace_sizes_grow_with_problem(lib):
+    a = N.spd_prune_workspace_size(N.prune_cfg(1, 577, 1024, 2, 1, 16, 192))
+    b = N.spd_prune_workspace_size(N.prune_cfg(5, 577, 1024, 2, 1, 16, 64))
+    assert b > a > 0
+    assert N.spd_linear_workspace_size(256, 4096) > 0

@@ -1,0 +1,140 @@
+"""Decoder prefill with sub-layer skipping on the GPU (spd_prefill, spd_project) against the CPU
+oracle (Sec. 3.2 VSkip-Attn / VSkip-FFN, Alg. 1 stage 2).
+
+Tolerance (bf16 weights and activations, fp32 accumulation): hidden states and logits within 2e-2,
+measured normwise per row, max_j |gpu - oracle| / max_j |oracle|. Rows whose every sub-layer is
+skipped must come back bit-identical to the input (the fp32 residual is never touched)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import decoder as od
+from paper_2609_34977_gb300 import _native as N
+from paper_2609_34977_gb300 import synth
+from tests.gpu_util import bf16_np, rowwise_rel
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-2
+
+
+def build(cfg, seed, std=0.05):
+    w = synth.decoder_weights(seed, cfg, std=std)
+    wd = {k: v for k, v in w.items() if k != "layers"}
+    wd = {k: v.cuda() for k, v in wd.items()}
+    wd["layers"] = [{k: v.cuda() for k, v in lw.items()} for lw in w["layers"]]
+    return N.SpdModel(cfg, wd), od.model_from_torch(w, cfg)
+
+
+def run(model, x, cu, mask):
+    T = x.shape[0]
+    B = len(cu) - 1
+    ws = torch.zeros(N.spd_prefill_workspace_size(model, T, B), dtype=torch.uint8, device="cuda")
+    h = torch.full((T, model.cfg["d_model"]), float("nan"), device="cuda")
+    logits = torch.full((B, model.cfg["vocab"]), float("nan"), device="cuda")
+    N.spd_prefill(model, x, T, cu, mask, h, logits, ws)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    return h.cpu().numpy(), logits.cpu().numpy()
+
+
+def inputs(T, D, seed):
+    g = torch.Generator().manual_seed(seed)
+    return torch.randn(T, D, generator=g).to(torch.bfloat16)
+
+
+def check(model, om, x, cu, mask):
+    h, lg = run(model, x.cuda(), cu, mask)
+    ho, lo = od.prefill(om, bf16_np(x), cu, mask if mask is not None else
+                        np.zeros((om["cfg"]["n_layers"], x.shape[0]), np.uint8))
+    assert np.isfinite(h).all() and np.isfinite(lg).all()
+    eh, el = rowwise_rel(h, ho), rowwise_rel(lg, lo)
+    assert eh < TOL and el < TOL, (eh, el)
+    return h, lg
+
+
+def test_tiny_config_static_plan():
+    # 2-layer decoder, 64 visual + 32 text tokens, plan {L0: none, L1: skip FFN} on visual tokens.
+    model, om = build(synth.TINY_DECODER, 1)
+    x = inputs(96, 256, 2)
+    vis = np.r_[np.ones(64), np.zeros(32)].astype(np.uint8)
+    mask = N.spd_plan_static(np.array([0, 2], np.uint8), vis)
+    h, _ = check(model, om, x, [0, 96], mask)
+
+
+def test_tiny_no_skipping_and_null_mask():
+    model, om = build(synth.TINY_DECODER, 3)
+    x = inputs(96, 256, 4)
+    h1, l1 = check(model, om, x, [0, 96], None)
+    h2, l2 = run(model, x.cuda(), [0, 96], np.zeros((2, 96), np.uint8))
+    np.testing.assert_array_equal(h1, h2)
+
+
+@pytest.mark.parametrize("seed", [5, 6])
+def test_adaptive_plan_mixed_targets(seed):
+    cfg = dict(synth.TINY_DECODER, n_layers=4)
+    model, om = build(cfg, seed)
+    T = 150
+    x = inputs(T, 256, seed + 10)
+    vis = np.r_[np.ones(110, bool), np.zeros(40, bool)]
+    admit, target = synth.adaptive_plan(seed, 4, vis, 0.6, np.array([1, 2, 1, 2], np.uint8), 0, 3)
+    mask = N.spd_plan_adaptive(4, admit, target)
+    assert (mask & 1).any() and (mask & 2).any()
+    check(model, om, x, [0, T], mask)
+
+
+def test_packed_ragged_sequences_and_bypass_is_bit_exact():
+    cfg = dict(synth.TINY_DECODER, n_layers=3)
+    model, om = build(cfg, 7)
+    cu = [0, 70, 71, 200, 333]          # a 1-token sequence, tiles of 64 with ragged tails
+    T = cu[-1]
+    x = inputs(T, 256, 8)
+    r = np.random.default_rng(9)
+    mask = r.integers(0, 4, size=(3, T)).astype(np.uint8)
+    mask[:, [5, 100, 250]] = 3           # these rows skip every sub-layer of every layer
+    mask[:, [69, 70, 199, 332]] = 0      # last tokens of each sequence stay fully active
+    h, _ = check(model, om, x, cu, mask)
+    for row in (5, 100, 250):
+        np.testing.assert_array_equal(h[row], bf16_np(x[row]).astype(np.float32))
+
+
+def test_gqa_head_dim_128_long_sequence():
+    cfg = dict(n_layers=2, d_model=512, n_heads=8, n_kv_heads=2, head_dim=128, d_ffn=1024,
+               vocab=1000, rope_theta=1e6, rms_eps=1e-6, d_vis=0, d_proj=0)
+    model, om = build(cfg, 11, std=0.03)
+    T = 330
+    x = inputs(T, 512, 12)
+    vis = np.r_[np.ones(250, bool), np.zeros(80, bool)]
+    admit, target = synth.adaptive_plan(13, 2, vis, 0.5, np.array([1, 2], np.uint8), 0, 1)
+    check(model, om, x, [0, T], N.spd_plan_adaptive(2, admit, target))
+
+
+def test_skip_attn_row_is_still_a_key_and_value():
+    cfg = dict(synth.TINY_DECODER, n_layers=1)
+    model, om = build(cfg, 14)
+    T, j = 40, 10
+    x = inputs(T, 256, 15)
+    mask = np.zeros((1, T), np.uint8)
+    mask[0, j] = 1
+    h1, _ = run(model, x.cuda(), [0, T], mask)
+    x2 = x.clone()
+    x2[j] = (x2[j].float() + torch.randn(256)).to(torch.bfloat16)
+    h2, _ = run(model, x2.cuda(), [0, T], mask)
+    np.testing.assert_array_equal(h1[:j], h2[:j])
+    assert np.abs(h1[j + 1:] - h2[j + 1:]).max() > 1e-3
+
+
+def test_projector():
+    cfg = dict(synth.TINY_DECODER, d_vis=128, d_proj=384)
+    model, om = build(cfg, 16)
+    R = 70
+    vis = torch.randn(R, 128).to(torch.bfloat16)
+    rows = torch.arange(R, dtype=torch.int32) * 2 + 1
+    x = torch.zeros(2 * R + 1, 256, dtype=torch.bfloat16, device="cuda")
+    ws = torch.zeros(N.spd_project_workspace_size(model, R), dtype=torch.uint8, device="cuda")
+    N.spd_project(model, vis.cuda(), R, rows.cuda(), x, ws)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    ref = od.project(om, bf16_np(vis))
+    got = bf16_np(x)
+    assert rowwise_rel(got[rows.numpy()], ref) < TOL
+    assert not got[0::2].any()

@@ -1,0 +1,82 @@
+"""MSV-Prune on the GPU (spd_prune) against the CPU oracle (Sec. 4.1, Eq. 1-3).
+
+Kept indices, kinds and cluster ids bit-exact; scores within 1e-5 relative (floor 1e-2) in fp32.
+Inputs are seeded planted-structure tiles on which every discrete decision of the oracle has a
+margin above 1e-3 (anchor cut, K-means assignments, per-cluster cuts)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import prune as op
+from paper_2609_34977_gb300 import _native as N
+from paper_2609_34977_gb300 import synth
+from tests.gpu_util import assert_prune_parity, bf16_np, conditioned_vision, gpu_prune
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("layer_weight", [[1.0, 1.0, 1.0], [0.0, 1.0, 1.0]])
+def test_tiny_config(layer_weight):
+    # 3 tapped layers (early, middle, final), 1 CLS + 576 patches x 256, 8 heads, keep 64.
+    _, v, res = conditioned_vision(20260001, 1, 576, 256, 3, 8, 64, 2, layer_weight=layer_weight)
+    g = gpu_prune(v, 64, 2, layer_weight=layer_weight)
+    assert_prune_parity(g, res)
+
+
+@pytest.mark.parametrize("keep", [192, 128, 64])
+def test_llava15_shape(keep):
+    # ViT-L/14-336: 576 patches x 1024 at the middle (12) and final (24) layers, 16 heads.
+    _, v, res = conditioned_vision(20260101, 1, 576, 1024, 2, 16, keep, 1)
+    assert_prune_parity(gpu_prune(v, keep, 1), res)
+
+
+@pytest.mark.parametrize("keep", [64, 32])
+def test_llava_next_anyres_tiles(keep):
+    # AnyRes: 5 tiles pruned independently with the same budget (320 or 160 kept in total).
+    _, v, res = conditioned_vision(20260201, 5, 576, 1024, 2, 16, keep, 1)
+    assert_prune_parity(gpu_prune(v, keep, 1), res)
+
+
+def test_clsless_received_attention_form():
+    # Qwen-style post-merger tokens: no CLS, received-attention importance, keep ratio 0.25.
+    _, v, res = conditioned_vision(20260301, 1, 1024, 1280, 2, 16, 256, 1, has_cls=False,
+                                   attn_form=1)
+    assert_prune_parity(gpu_prune(v, 256, 1, has_cls=False, attn_form=1), res)
+
+
+@pytest.mark.parametrize("keep,K,r", [(1, 4, 0.7), (576, 4, 0.7), (40, 1, 0.0), (30, 4, 1.0),
+                                      (50, 8, 0.5), (100, 2, 0.3)])
+def test_edge_budgets_and_cluster_counts(keep, K, r):
+    _, v, res = conditioned_vision(20260401, 1, 576, 256, 2, 8, keep, 1, n_clusters=K,
+                                   anchor_ratio=r)
+    g = gpu_prune(v, keep, 1, n_clusters=K, anchor_ratio=r)
+    assert_prune_parity(g, res)
+    idx = g["keep_idx"][0]
+    assert len(idx) == keep and np.all(np.diff(idx) > 0)
+
+
+def test_ragged_patch_count():
+    # a patch count that is not a power of two nor a multiple of 32
+    _, v, res = conditioned_vision(20260501, 2, 333, 128, 2, 4, 50, 1)
+    assert_prune_parity(gpu_prune(v, 50, 1), res)
+
+
+def test_repeat_runs_are_bitwise_identical():
+    v = synth.vision_tiles(7, 2, 576, 1024, 2, 16)
+    a = gpu_prune(v, 128, 1)
+    b = gpu_prune(v, 128, 1)
+    for k in ("keep_idx", "kind", "cluster"):
+        np.testing.assert_array_equal(a[k], b[k])
+    np.testing.assert_array_equal(a["scores"].view(np.uint32), b["scores"].view(np.uint32))
+
+
+def test_gather_rows_bf16():
+    v = synth.vision_tiles(8, 3, 576, 1024, 2, 16)
+    g = gpu_prune(v, 64, 1)
+    dst = torch.empty(3 * 64, 1024, dtype=torch.bfloat16, device="cuda")
+    idx = torch.from_numpy(g["keep_idx"]).cuda()
+    N.spd_gather_rows_bf16(g["feats"][1], 3, 577, 1024, 1, idx, 64, dst, ws=g["ws"])
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(g["ws"]) == 0
+    ref = np.concatenate([v["feats"][1][t, 1 + g["keep_idx"][t]] for t in range(3)])
+    np.testing.assert_array_equal(bf16_np(dst), torch.from_numpy(ref).to(torch.bfloat16).double().numpy())
