@@ -1,0 +1,351 @@
+#!/usr/bin/env python3
+"""Throughput of SPIDER's accelerated multimodal prefill on one GB300 (Alg. 1, both stages).
+
+One step = MSV-Prune of the request's tile(s) + gather + LLaVA projector + sequence assembly +
+32-layer decoder prefill with the adaptive skip plan + LM head, all in libspider.so. Workload: the
+LLaVA-1.5-7B shape (ViT-L/14-336 features at layers 12 and 24, 576 patches x 1024, 16-head CLS
+attention; keep 192 of 576 with r = 0.7, K = 4; projector 1024 -> 4096 -> 4096; decoder 32 x
+(4096 hidden, 32 heads, FFN 11008), vocab 32000, bf16 random init; 64 text tokens; batch 1). The
+tokens counted per request are the ORIGINAL visual tokens plus the text tokens (576 + 64), for the
+SPIDER step and for the dense step (no pruning, no skipping, same kernels) alike.
+
+python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+Multi-GPU (torchrun): every rank runs its own independent requests (weak scaling, no collective on
+the data path); rank 0 prints the max-over-ranks timing.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "pruned+skipped prefill tokens/s on 1 GB300 vs dense; % of HBM/tensor roofline"
+SEED = 20260001
+N_PATCH, D_VIS, H_VIS, TEXT = 576, 1024, 16, 64
+SKIP_FRAC, ADMIT_LO = 0.9, 2     # 90 % of visual tokens enter skip mode at layer U[2, 16)
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--keep", type=int, default=192)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p["hbm_gbs"], p["bf16_tflops"], p["bf16_tflops_sustained"], "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def workload_config(keep, mask, T):
+    skipped = float(mask.astype(bool).sum() + (mask == 3).sum()) / (2.0 * mask.size)
+    return {"workload": (f"llava-1.5-7b shape: 1 tile 1+576 x 1024 (ViT layers 12, 24), 16-head CLS "
+                         f"attention, keep {keep} (r=0.7, K=4), projector 1024->4096->4096, "
+                         f"32-layer decoder 4096/32h/11008, vocab 32000, 64 text tokens, batch 1, "
+                         f"adaptive skip plan (Table 9 targets)"),
+            "keep": keep, "tokens_per_request": N_PATCH + TEXT, "decoder_tokens": T,
+            "skipped_sublayer_fraction": round(skipped, 4),
+            "l2": "inputs larger than L2: 13.5 GB of weights streamed every step (L2 129 MB)"}
+
+
+class Clocks:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    def __init__(self, gpu):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(gpu), f"--query-gpu={q}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return None
+        self.p.terminate()
+        self.p.wait()
+        rows = []
+        with open(self.f.name) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) == 7:
+                    rows.append(parts)
+        os.unlink(self.f.name)
+        if not rows:
+            return None
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[3 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": float(rows[0][1]) if rows[0][1].replace(".", "").isdigit() else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def build_model(torch, N, synth, device):
+    cfg = dict(synth.LLAVA_7B_DECODER)
+    w = synth.decoder_weights(SEED, cfg, device=device)
+    model = N.SpdModel(cfg, w)
+    del w
+    torch.cuda.empty_cache()
+    return model, cfg
+
+
+def count_launches(pipe, mask, dense):
+    L = mask.shape[0] if mask is not None else pipe.model.cfg["n_layers"]
+    n = (0 if dense else 7) + 1 + 2 + 1 + 1 + 2      # prune, gather, projector, text, embed, head
+    for l in range(L):
+        bits = mask[l] if mask is not None else np.zeros(pipe.T, np.uint8)
+        n += 2 + (3 if ((bits & 1) == 0).any() else 0) + (3 if ((bits & 2) == 0).any() else 0)
+    return n
+
+
+def cpu_baseline_sample(keep, v, mask_fn, reps=1):
+    """The oracle as it stands on the host cores: MSV-Prune of the tile, the projector, and 1- and
+    2-layer decoder prefills of the same token count; the step time is extrapolated to 32 layers."""
+    import torch
+
+    from oracle import decoder as od
+    from oracle import prune as op
+    from paper_2609_34977_gb300 import synth
+    cfg = dict(synth.LLAVA_7B_DECODER)
+    t0 = time.perf_counter()
+    res = op.prune(v["feats"], v["attn"], keep=keep, final_layer=1)[0]
+    t_prune = time.perf_counter() - t0
+    w = synth.decoder_weights(SEED + 1, dict(cfg, n_layers=2), device="cpu")
+    m2 = od.model_from_torch(w, dict(cfg, n_layers=2))
+    m1 = dict(m2, layers=m2["layers"][:1], cfg=dict(m2["cfg"], n_layers=1))
+    vis = od.bf16_round(v["feats"][1][0, 1 + res["keep_idx"]])
+    t0 = time.perf_counter()
+    xv = od.project(m2, vis)
+    t_proj = time.perf_counter() - t0
+    T = keep + TEXT
+    x = np.concatenate([xv, od.bf16_round(np.random.default_rng(0).standard_normal((TEXT, 4096)))])
+    mask = mask_fn(T)
+    t0 = time.perf_counter()
+    od.prefill(m1, x, [0, T], mask[:1])
+    t1 = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    od.prefill(m2, x, [0, T], mask[:2])
+    t2 = time.perf_counter() - t0
+    t_layer = max(t2 - t1, 1e-9)
+    t_step = t_prune + t_proj + (t1 - t_layer) + 32 * t_layer
+    cores = torch.get_num_threads()
+    try:
+        from threadpoolctl import threadpool_info
+        cores = max([i.get("num_threads", 0) for i in threadpool_info()] + [cores])
+    except Exception:
+        pass
+    return {"value": (N_PATCH + TEXT) / t_step, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": (f"fp64 numpy oracle: MSV-Prune of 1 tile ({t_prune:.2f} s), projector of "
+                       f"{keep} rows ({t_proj:.2f} s), 1- and 2-layer decoder prefills of {T} tokens "
+                       f"({t1:.2f} s, {t2:.2f} s); step extrapolated as prune + projector + head + "
+                       f"32 x layer = {t_step:.1f} s"),
+            "cpu_seconds": round(t_prune + t_proj + t1 + t2, 1)}
+
+
+def run_reference(a):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2609_34977_gb300 import synth
+    v = synth.vision_tiles(SEED, 1, N_PATCH, D_VIS, 2, H_VIS)
+    m_llava = synth.skip_targets("llava-1.5-7b")
+
+    def mask_fn(T):
+        from oracle import decoder as od
+        vis = np.r_[np.ones(T - TEXT, bool), np.zeros(TEXT, bool)]
+        admit, target = synth.adaptive_plan(SEED, 32, vis, SKIP_FRAC, m_llava, ADMIT_LO, 16)
+        return od.expand_adaptive_plan(admit, target, 32)
+
+    times = []
+    sample = None
+    for i in range(a.warmup + a.steps):
+        s = cpu_baseline_sample(a.keep, v, mask_fn)
+        if i >= a.warmup:
+            times.append((N_PATCH + TEXT) / s["value"])
+            sample = s
+    ms = 1000.0 * statistics.mean(times)
+    val = (N_PATCH + TEXT) / (ms / 1000.0)
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": a.gpus,
+            "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": "the CPU oracle on the llava-1.5-7b shape (see cpu_baseline)",
+                       "keep": a.keep},
+            "cpu_baseline": {k: sample[k] for k in ("kind", "cores", "sample")} | {"value": val,
+                                                                                 "unit": "tokens/s"},
+            "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    a = parse()
+    if a.impl == "reference":
+        return run_reference(a)
+    import torch
+
+    from paper_2609_34977_gb300 import _native as N
+    from paper_2609_34977_gb300 import synth
+    from paper_2609_34977_gb300.pipeline import SpiderPrefill
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    dev = "cuda"
+    model, cfg = build_model(torch, N, synth, dev)
+    m_llava = synth.skip_targets("llava-1.5-7b")
+
+    def make(keep, dense):
+        pipe = SpiderPrefill(model, n_patch=N_PATCH, has_cls=True, d_vis=D_VIS, n_feat_layers=2,
+                             final_layer=1, n_heads_vis=H_VIS, attn_form=0, keep=keep,
+                             tiles_per_req=[1], text_lens=[TEXT], dense=dense)
+        if dense:
+            return pipe, None
+        admit, target = synth.adaptive_plan(SEED + rank, 32, pipe.token_is_visual, SKIP_FRAC, m_llava,
+                                            ADMIT_LO, 16)
+        return pipe, N.spd_plan_adaptive(32, admit, target)
+
+    v = synth.vision_tiles(SEED + rank, 1, N_PATCH, D_VIS, 2, H_VIS)
+    feats = [torch.from_numpy(f).to(dev) for f in v["feats"]]
+    attn = torch.from_numpy(v["attn"]).to(dev)
+    text = torch.from_numpy(synth.text_embeddings(SEED + rank, TEXT, 4096).view(np.int16)).view(
+        torch.bfloat16).to(dev)
+
+    def timed(pipe, mask, steps, warmup, trace=False):
+        for _ in range(warmup):
+            pipe.run(feats, attn, text, mask)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        if trace:
+            N.spd_trace_enable(steps * 400)
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s.record()
+        for _ in range(steps):
+            pipe.run(feats, attn, text, mask)
+        e.record()
+        torch.cuda.synchronize()
+        ms = s.elapsed_time(e) / steps
+        if dist:
+            t = torch.tensor([ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms = float(t.item())
+        return ms
+
+    hbm, tf_burst, tf_sust, src = peaks()
+    spider, mask = make(a.keep, False)
+    dense, _ = make(N_PATCH, True)
+    clocks = Clocks(local)
+    ms = timed(spider, mask, a.steps, a.warmup)
+    clk = clocks.stop()
+    assert spider.status() == 0, "device-side failure recorded"
+    ms_dense = timed(dense, None, a.steps, a.warmup)
+    tokens = (N_PATCH + TEXT) * world
+    value = tokens / (ms / 1000.0)
+
+    # traced pass: per-kernel-class device time and algorithmic work over K steps
+    timed(spider, mask, a.steps, 1, trace=True)
+    cls = {name: N.spd_trace_read(c) for name, c in (("gemm", N.TRACE_GEMM), ("attention", N.TRACE_ATTN),
+                                                     ("rows", N.TRACE_ROWS), ("prune", N.TRACE_PRUNE))}
+    N.spd_trace_enable(0)
+    g = cls["gemm"]
+    ridge = tf_sust * 1e12 / (hbm * 1e9)
+    ai = g["flops"] / max(g["bytes"], 1.0)
+    gbs = g["bytes"] / (g["ms"] / 1000.0) / 1e9
+    tfs = g["flops"] / (g["ms"] / 1000.0) / 1e12
+    if ai < ridge:
+        roof = {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm}
+    else:
+        roof = {"bound": "tensor", "achieved": tfs, "peak": tf_sust, "unit": "TFLOP/s",
+                "frac": tfs / tf_sust}
+    roof.update({"traffic": None, "kernel": "gemm_tc_kernel (tcgen05, all decoder/projector/LM-head GEMMs)",
+                 "peak_source": f"{src} (MEASURED_PEAKS.json)", "launches_per_step": g["launches"] / a.steps,
+                 "avg_launch_us": 1000.0 * g["ms"] / max(g["launches"], 1),
+                 "arith_intensity_flop_per_byte": ai, "tensor_tflops": tfs,
+                 "tensor_frac_of_sustained": tfs / tf_sust, "hbm_frac": gbs / hbm,
+                 "share_of_step": g["ms"] / a.steps / ms})
+    kernels = {k: {"launches_per_step": c["launches"] / a.steps, "ms_per_step": c["ms"] / a.steps,
+                   "GB/s": c["bytes"] / max(c["ms"], 1e-9) / 1e6,
+                   "TFLOP/s": c["flops"] / max(c["ms"], 1e-9) / 1e9} for k, c in cls.items()}
+
+    # end to end through the public API: pinned host inputs -> device, step, logits -> host
+    hf = [f.cpu().pin_memory() for f in feats]
+    ha, ht = attn.cpu().pin_memory(), text.cpu().pin_memory()
+    hl = torch.empty_like(spider.logits, device="cpu").pin_memory()
+    for _ in range(a.warmup):
+        for d_, h_ in zip(feats + [attn, text], hf + [ha, ht]):
+            d_.copy_(h_, non_blocking=True)
+        spider.run(feats, attn, text, mask)
+        hl.copy_(spider.logits, non_blocking=True)
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(a.steps):
+        for d_, h_ in zip(feats + [attn, text], hf + [ha, ht]):
+            d_.copy_(h_, non_blocking=True)
+        spider.run(feats, attn, text, mask)
+        hl.copy_(spider.logits, non_blocking=True)
+    e.record()
+    torch.cuda.synchronize()
+    ms_e2e = s.elapsed_time(e) / a.steps
+    h2d = sum(t.numel() * t.element_size() for t in hf + [ha, ht])
+
+    cpu = None
+    if rank == 0 and not a.no_cpu_baseline:
+        from oracle import decoder as od
+
+        def mask_fn(T):
+            vis = np.r_[np.ones(T - TEXT, bool), np.zeros(TEXT, bool)]
+            ad, tg = synth.adaptive_plan(SEED, 32, vis, SKIP_FRAC, m_llava, ADMIT_LO, 16)
+            return od.expand_adaptive_plan(ad, tg, 32)
+        cpu = cpu_baseline_sample(a.keep, v, mask_fn)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+                "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                "config": workload_config(a.keep, mask, spider.T),
+                "dense": {"value": tokens / (ms_dense / 1000.0), "ms_per_step": ms_dense,
+                          "decoder_tokens": dense.T, "speedup_spider_vs_dense": ms_dense / ms},
+                "roofline": roof, "kernels": kernels, "cpu_baseline": cpu,
+                "e2e": {"value": tokens / (ms_e2e / 1000.0), "unit": "tokens/s",
+                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": hl.numel() * 4,
+                        "ms_per_step": ms_e2e},
+                "gpu_launches": count_launches(spider, mask, False) * a.steps,
+                "clocks": clk,
+                "paper_context": "paper: LLaVA-1.5-7B prefill 67.4 ms (576 tokens) -> 48.2 ms (128), "
+                                 "hardware not stated"}
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

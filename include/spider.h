@@ -11,9 +11,9 @@
  *     bf16 data is passed as uint16_t bit patterns. Matrices are row-major.
  *   - The caller owns every buffer. Work is enqueued on `stream` (a cudaStream_t, NULL = legacy
  *     default stream) and is asynchronous unless stated otherwise.
- *   - spd_prune, spd_project and spd_prefill allocate nothing: they run in a caller-provided
- *     workspace whose size the matching *_workspace_size call returns. A workspace must not be
- *     shared by calls that may overlap on the GPU.
+ *   - spd_prune, spd_project, spd_prefill and spd_linear allocate nothing: they run in a
+ *     caller-provided workspace whose size the matching *_workspace_size call returns. A workspace
+ *     must not be shared by calls that may overlap on the GPU.
  *   - Every call returns SPD_OK (0) or a negative spd_status. Argument errors are detected on the
  *     host before any launch and leave the device untouched; spd_last_error() describes the last
  *     failure of the calling thread. Device-side failures (a bounded wait that gave up) are
@@ -54,6 +54,19 @@ int spd_workspace_status(void* ws, void* stream, int* status);
  * the status word of `ws` (at least 4 bytes of device memory). No fault, trap or hang: the
  * context stays usable. Asynchronous; read the result with spd_workspace_status. */
 int spd_selftest_bounded_wait(void* ws, long long budget_cycles, void* stream);
+
+/* Kernel-class tracing (no counterpart in the paper; measurement support). spd_trace_enable(n)
+ * starts recording up to n launches: every launch of the library is bracketed by a CUDA event pair
+ * on its stream and tagged with its class and algorithmic work; n <= 0 stops recording.
+ * spd_trace_read synchronises on the recorded events and returns, for one class
+ * (SPD_TRACE_GEMM, _ATTN, _ROWS, _PRUNE), the launch count, summed device milliseconds, and summed
+ * algorithmic flops and HBM bytes (the operation's own: operands read once, results written once). */
+#define SPD_TRACE_GEMM 0
+#define SPD_TRACE_ATTN 1
+#define SPD_TRACE_ROWS 2
+#define SPD_TRACE_PRUNE 3
+int spd_trace_enable(int capacity);
+int spd_trace_read(int cls, long long* launches, double* ms, double* flops, double* bytes);
 
 /* ------------------------------------------------------------------------------------------ */
 /* Stage 1: MSV-Prune (Sec. 4.1)                                                                */
@@ -202,6 +215,9 @@ int spd_prefill(const spd_model* m, const uint16_t* x, int n_tokens, const int32
 /* Single kernels, exposed for composition and per-kernel tests                                 */
 /* ------------------------------------------------------------------------------------------ */
 
+/* Epilogues of spd_linear. All but SPD_EPI_ADD_F32 give bit-identical results run to run; the
+ * residual update adds with fire-and-forget atomics, so where K is split across CTAs the fp32
+ * additions land in no fixed order (results agree to rounding). */
 typedef enum {
   SPD_EPI_F32 = 0,       /* out fp32 [M][N] = acc */
   SPD_EPI_BF16 = 1,      /* out bf16 [M][N] = bf16(acc) */

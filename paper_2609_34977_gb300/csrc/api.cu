@@ -16,7 +16,7 @@ namespace spd {
 
 int attention_run(const void* q, int ldq, const void* kv, int ldkv, int v_off, void* o, int ldo,
                   const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads,
-                  int head_dim, cudaStream_t stream);
+                  int head_dim, cudaStream_t stream, double ctx_sum, int n_q, int n_kv_rows);
 int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float eps,
                 const int32_t* in_rows, void* out, const int32_t* map2, void* out2,
                 cudaStream_t stream);
@@ -52,6 +52,18 @@ __global__ void copy_rows_kernel(const uint16_t* __restrict__ src, uint16_t* __r
   const uint16_t* s = src + size_t(src_rows[i]) * cols;
   uint16_t* d = dst + size_t(dst_rows[i]) * cols;
   for (int c = threadIdx.x; c < cols; c += blockDim.x) d[c] = s[c];
+}
+
+// (cos, sin) of position p times frequency j, evaluated in double and stored as float2.
+__global__ void rope_table_kernel(const double* __restrict__ inv_freq, int half, int n_pos,
+                                  float2* __restrict__ tab) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n_pos * half) return;
+  double s, c;
+  sincos(double(i / half) * inv_freq[i % half], &s, &c);
+  tab[i] = make_float2(float(c), float(s));
 }
 
 // Bounded wait on a barrier that nothing arrives on: exercises the timeout path.
@@ -105,7 +117,7 @@ struct spd_model {
   uint16_t *final_norm = nullptr, *lm_head = nullptr;
   uint16_t *pw1 = nullptr, *pb1 = nullptr, *pw2 = nullptr, *pb2 = nullptr;
   CUtensorMap m_lm, m_p1, m_p2;
-  float* inv_freq = nullptr;
+  double* inv_freq = nullptr;  // [head_dim / 2] theta^(-2j / head_dim)
   int gu_rows = 0;
   void* pool = nullptr;
 };
@@ -149,7 +161,7 @@ extern "C" int spd_model_create(const spd_model_cfg* c, const spd_model_weights*
   auto al = [](size_t b) { return (b + 255) & ~size_t(255); };
   const size_t per_layer = al(D * 2) * 2 + al(q_rows * D * 2) + al(2 * kv_rows * D * 2) +
                            al(D * q_rows * 2) + al(size_t(gu_rows) * D * 2) + al(D * F * 2);
-  size_t total = per_layer * c->n_layers + al(D * 2) + al(size_t(c->vocab) * D * 2) + al(hd * 4);
+  size_t total = per_layer * c->n_layers + al(D * 2) + al(size_t(c->vocab) * D * 2) + al(hd * 8);
   if (c->d_vis)
     total += al(size_t(c->d_proj) * c->d_vis * 2) + al(size_t(c->d_proj) * 2) +
              al(D * c->d_proj * 2) + al(D * 2);
@@ -236,11 +248,10 @@ extern "C" int spd_model_create(const spd_model_cfg* c, const spd_model_weights*
   cudaMemcpy(m->final_norm, w->final_norm, D * 2, cudaMemcpyDeviceToDevice);
   cudaMemcpy(m->lm_head, w->lm_head, size_t(c->vocab) * D * 2, cudaMemcpyDeviceToDevice);
   if ((rc = make_weight_map(&m->m_lm, m->lm_head, c->vocab, int(D)))) return fin(rc);
-  m->inv_freq = reinterpret_cast<float*>(take(hd * 4));
-  std::vector<float> inv(hd / 2);
-  for (size_t j = 0; j < hd / 2; ++j)
-    inv[j] = float(pow(double(c->rope_theta), -2.0 * double(j) / double(hd)));
-  cudaMemcpy(m->inv_freq, inv.data(), inv.size() * 4, cudaMemcpyHostToDevice);
+  m->inv_freq = reinterpret_cast<double*>(take(hd * 8));
+  std::vector<double> inv(hd / 2);
+  for (size_t j = 0; j < hd / 2; ++j) inv[j] = pow(double(c->rope_theta), -2.0 * double(j) / double(hd));
+  cudaMemcpy(m->inv_freq, inv.data(), inv.size() * 8, cudaMemcpyHostToDevice);
   if (c->d_vis) {
     if (!w->proj_w1 || !w->proj_b1 || !w->proj_w2 || !w->proj_b2)
       return fin(fail(SPD_EINVAL, "null projector weight"));
@@ -297,7 +308,7 @@ extern "C" size_t spd_linear_workspace_size(int, int) { return 256 + gemm_scratc
 
 static GemmScratch scratch_from(Carve& cv) {
   GemmScratch s;
-  s.partial_floats = size_t(16) << 20;
+  s.partial_floats = kGemmSlotFloats;
   s.partial = cv.take<float>(s.partial_floats);
   s.n_counters = 1 << 16;
   s.counters = cv.take<int>(s.n_counters);
@@ -386,15 +397,18 @@ namespace {
 
 struct PrefillBufs {
   uint16_t *xa, *xq, *q, *kv, *o, *y, *act, *z;
+  float2* rope;
   int32_t* lists;
   size_t list_ints;
   GemmScratch gs;
 };
 
+// Every list starts on a multiple of 4 ints (16 bytes): the attention tiles are read as int4.
+size_t pad4(size_t n) { return (n + 3) & ~size_t(3); }
 size_t list_ints_for(int L, int T, int B) {
   // per layer: arows[T], amap[T], apos[T], frows[T], tiles[(T / 64 + B + 1) * 4]
   // plus pos_all[T], last[B]
-  return size_t(L) * (4 * size_t(T) + 4 * (size_t(T) / 64 + B + 1)) + T + B + 16;
+  return size_t(L) * (4 * pad4(T) + 4 * (size_t(T) / 64 + B + 1)) + pad4(T) + pad4(B) + 16;
 }
 
 PrefillBufs carve_prefill(const spd_model_cfg& c, int T, int B, Carve& cv) {
@@ -409,6 +423,7 @@ PrefillBufs carve_prefill(const spd_model_cfg& c, int T, int B, Carve& cv) {
   b.y = cv.take<uint16_t>(size_t(T) * D);
   b.act = cv.take<uint16_t>(size_t(T) * c.d_ffn);
   b.z = cv.take<uint16_t>(size_t(B) * D);
+  b.rope = cv.take<float2>(size_t(T) * (c.head_dim / 2));
   b.list_ints = list_ints_for(c.n_layers, T, B);
   b.lists = cv.take<int32_t>(b.list_ints);
   return b;
@@ -450,29 +465,31 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
       pos_all[t] = t - cu[b];
       seq_of[t] = b;
     }
-  struct LayerLists { size_t arows, amap, apos, frows, tiles; int na, nf, ntiles; };
+  struct LayerLists { size_t arows, amap, apos, frows, tiles; int na, nf, ntiles; double ctx; };
   std::vector<LayerLists> ll(L);
   size_t off = 0;
   const size_t pos_off = off;
   for (int t = 0; t < T; ++t) hl[off + t] = pos_all[t];
-  off += T;
+  off += pad4(T);
   const size_t last_off = off;
   for (int b = 0; b < B; ++b) hl[off + b] = cu[b + 1] - 1;
-  off += B;
+  off += pad4(B);
   for (int l = 0; l < L; ++l) {
     LayerLists& q = ll[l];
     const uint8_t* mk = mask ? mask + size_t(l) * T : nullptr;
-    q.arows = off; off += T;
-    q.amap = off; off += T;
-    q.apos = off; off += T;
-    q.frows = off; off += T;
+    q.arows = off; off += pad4(T);
+    q.amap = off; off += pad4(T);
+    q.apos = off; off += pad4(T);
+    q.frows = off; off += pad4(T);
     q.tiles = off;
     q.na = q.nf = q.ntiles = 0;
+    q.ctx = 0.0;
     for (int t = 0; t < T; ++t) {
       const int bits = mk ? mk[t] : 0;
       if (!(bits & 1)) {
         hl[q.amap + t] = q.na;
         hl[q.apos + q.na] = pos_all[t];
+        q.ctx += pos_all[t] + 1;
         hl[q.arows + q.na++] = t;
       } else {
         hl[q.amap + t] = -1;
@@ -499,6 +516,10 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
   SPD_CUDA_TRY(cudaMemcpyAsync(dl, hl.data(), off * sizeof(int32_t), cudaMemcpyHostToDevice, st));
   SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
   if (int rc = bf16_to_f32_run(x, h, size_t(T) * D, st)) return rc;
+  int max_len = 0;
+  for (int b = 0; b < B; ++b) max_len = cu[b + 1] - cu[b] > max_len ? cu[b + 1] - cu[b] : max_len;
+  SPD_CUDA_TRY(launch_pdl(rope_table_kernel, dim3((max_len * (hd / 2) + 255) / 256), dim3(256), 0, st,
+                          static_cast<const double*>(m->inv_freq), hd / 2, max_len, bf.rope));
 
   int rc = SPD_OK;
   for (int l = 0; l < L && !rc; ++l) {
@@ -518,7 +539,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
     kvp.out = bf.kv;
     kvp.ldo = 2 * kvd;
     kvp.pos = dl + pos_off;
-    kvp.inv_freq = m->inv_freq;
+    kvp.rope = bf.rope;
     kvp.rope_rows = kvd;
     kvp.head_dim = hd;
     if ((rc = gemm_run(kvp, bf.gs, st))) break;
@@ -535,7 +556,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
       if ((rc = gemm_run(qp, bf.gs, st))) break;
       if ((rc = attention_run(bf.q, qd, bf.kv, 2 * kvd, kvd, bf.o, qd,
                               reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
-                              c.n_heads, c.n_kv_heads, hd, st)))
+                              c.n_heads, c.n_kv_heads, hd, st, q.ctx, q.na, T)))
         break;
       GemmProblem op{};
       op.map_w = &W.m_o;

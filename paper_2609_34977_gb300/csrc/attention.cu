@@ -10,6 +10,8 @@
 #include <stdint.h>
 
 #include "internal.h"
+#include "ptx.cuh"
+#include "trace.h"
 
 namespace spd {
 namespace {
@@ -63,6 +65,8 @@ __global__ void __launch_bounds__(128)
   __nv_bfloat16* Ks = Qs + kQ * LD;
   __nv_bfloat16* Vs = Ks + 2 * kKB * LD;
   int* pos_s = reinterpret_cast<int*>(Vs + 2 * kKB * LD);
+  pdl_launch_dependents();
+  pdl_wait();
 
   const int4 tl = tiles[blockIdx.x];
   const int q0 = tl.x, nq = tl.y, kv0 = tl.z;
@@ -223,10 +227,11 @@ int launch(const void* q, int ldq, const void* kv, int ldkv, int v_off, void* o,
     attr = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf(float(HD));
-  attn_kernel<HD><<<dim3(n_tiles, n_heads), 128, smem, stream>>>(
-      static_cast<const __nv_bfloat16*>(q), ldq, static_cast<const __nv_bfloat16*>(kv), ldkv, v_off,
-      static_cast<__nv_bfloat16*>(o), ldo, tiles, q_pos, n_heads, n_kv_heads, scale_log2);
-  SPD_CUDA_TRY(cudaGetLastError());
+  SPD_CUDA_TRY(launch_pdl(attn_kernel<HD>, dim3(n_tiles, n_heads), dim3(128), smem, stream,
+                          static_cast<const __nv_bfloat16*>(q), ldq,
+                          static_cast<const __nv_bfloat16*>(kv), ldkv, v_off,
+                          static_cast<__nv_bfloat16*>(o), ldo, tiles, q_pos, n_heads, n_kv_heads,
+                          scale_log2));
   return SPD_OK;
 }
 
@@ -234,15 +239,20 @@ int launch(const void* q, int ldq, const void* kv, int ldkv, int v_off, void* o,
 
 int attention_run(const void* q, int ldq, const void* kv, int ldkv, int v_off, void* o, int ldo,
                   const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads,
-                  int head_dim, cudaStream_t stream) {
+                  int head_dim, cudaStream_t stream, double ctx_sum, int n_q, int n_kv_rows) {
   if (n_tiles <= 0) return SPD_OK;
-  if (head_dim == 128)
-    return launch<128>(q, ldq, kv, ldkv, v_off, o, ldo, tiles, n_tiles, q_pos, n_heads, n_kv_heads,
-                       stream);
-  if (head_dim == 64)
-    return launch<64>(q, ldq, kv, ldkv, v_off, o, ldo, tiles, n_tiles, q_pos, n_heads, n_kv_heads,
-                      stream);
-  return fail(SPD_EUNSUPPORTED, "attention supports head_dim 64 and 128");
+  if (head_dim != 128 && head_dim != 64)
+    return fail(SPD_EUNSUPPORTED, "attention supports head_dim 64 and 128");
+  const int slot = trace_begin(stream);
+  const int rc = (head_dim == 128)
+                     ? launch<128>(q, ldq, kv, ldkv, v_off, o, ldo, tiles, n_tiles, q_pos, n_heads,
+                                   n_kv_heads, stream)
+                     : launch<64>(q, ldq, kv, ldkv, v_off, o, ldo, tiles, n_tiles, q_pos, n_heads,
+                                  n_kv_heads, stream);
+  // QK^T and PV over each active query's causal context; Q, K, V read once and O written once
+  trace_end(slot, stream, TR_ATTN, 4.0 * head_dim * n_heads * ctx_sum,
+            2.0 * (2.0 * n_q * n_heads * head_dim + 2.0 * n_kv_rows * n_kv_heads * head_dim));
+  return rc;
 }
 
 }  // namespace spd

@@ -5,6 +5,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "spider.h"
 
 namespace spd {
@@ -23,6 +25,24 @@ int fail(int code, const char* fmt, ...);  // records the thread's message, retu
 constexpr long long kWaitBudget = 1ll << 30;
 
 int num_sms();  // SM count of the current device
+
+// Launches a kernel with programmatic stream serialization: it may be scheduled while the previous
+// kernel of the stream is still running, and orders itself after it with griddepcontrol.wait.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // Bump allocator over a caller-provided workspace. The first 256 bytes hold the status word.
 struct Carve {
@@ -63,12 +83,14 @@ struct GemmProblem {
   const int32_t* rows;       // output row of token t (null = t)
   const uint16_t* bias;      // [n_out] bf16
   const int32_t* pos;        // rotary position of token t
-  const float* inv_freq;     // [head_dim / 2]
+  const void* rope;          // float2 [position][head_dim / 2]: (cos, sin) of position * freq_j
   int rope_rows, head_dim;
   int out_cols;              // valid output columns (SwiGLU: d_ffn)
 };
 
-// Scratch of split-K partial sums and per-tile arrival counters.
+// Scratch of stream-K partial slots (fp32, two per CTA) and per-tile arrival counters. The counters
+// must be zero before a GEMM runs; every GEMM leaves them zero again when it completes.
+constexpr size_t kGemmSlotFloats = size_t(10) << 20;
 struct GemmScratch {
   float* partial;
   size_t partial_floats;

@@ -5,6 +5,8 @@
 #include <stdint.h>
 
 #include "internal.h"
+#include "ptx.cuh"
+#include "trace.h"
 
 namespace spd {
 namespace {
@@ -30,6 +32,8 @@ __global__ void __launch_bounds__(kThreads)
                    const int32_t* __restrict__ in_rows, __nv_bfloat16* __restrict__ out,
                    const int32_t* __restrict__ map2, __nv_bfloat16* __restrict__ out2) {
   __shared__ float red[kThreads / 32];
+  pdl_launch_dependents();
+  pdl_wait();
   const int i = blockIdx.x;
   const int r = in_rows ? in_rows[i] : i;
   const float4* src = reinterpret_cast<const float4*>(h + size_t(r) * D);
@@ -61,6 +65,8 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 __global__ void bf16_to_f32_kernel(const uint16_t* __restrict__ x, float* __restrict__ h, size_t n4) {
+  pdl_launch_dependents();
+  pdl_wait();
   for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < n4;
        i += size_t(gridDim.x) * blockDim.x) {
     const ushort4 v = reinterpret_cast<const ushort4*>(x)[i];
@@ -72,6 +78,8 @@ __global__ void bf16_to_f32_kernel(const uint16_t* __restrict__ x, float* __rest
 
 __global__ void scatter_rows_kernel(const uint16_t* __restrict__ src, int D,
                                     const int32_t* __restrict__ rows, uint16_t* __restrict__ dst) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int i = blockIdx.x;
   const uint4* s = reinterpret_cast<const uint4*>(src + size_t(i) * D);
   uint4* d = reinterpret_cast<uint4*>(dst + size_t(rows[i]) * D);
@@ -84,10 +92,11 @@ int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float e
                 const int32_t* in_rows, void* out, const int32_t* map2, void* out2,
                 cudaStream_t stream) {
   if (n_rows <= 0) return SPD_OK;
-  rmsnorm_kernel<<<n_rows, kThreads, 0, stream>>>(h, D, gain, eps, in_rows,
-                                                  static_cast<__nv_bfloat16*>(out), map2,
-                                                  static_cast<__nv_bfloat16*>(out2));
-  SPD_CUDA_TRY(cudaGetLastError());
+  const int slot = trace_begin(stream);
+  SPD_CUDA_TRY(launch_pdl(rmsnorm_kernel, dim3(n_rows), dim3(kThreads), 0, stream, h, D, gain, eps,
+                          in_rows, static_cast<__nv_bfloat16*>(out), map2,
+                          static_cast<__nv_bfloat16*>(out2)));
+  trace_end(slot, stream, TR_ROWS, 4.0 * n_rows * D, double(n_rows) * D * (4.0 + 2.0));
   return SPD_OK;
 }
 
@@ -95,16 +104,18 @@ int bf16_to_f32_run(const uint16_t* x, float* h, size_t n, cudaStream_t stream) 
   if (n == 0) return SPD_OK;
   const size_t n4 = n / 4;
   const int blocks = int((n4 + 255) / 256 < 4096 ? (n4 + 255) / 256 : 4096);
-  bf16_to_f32_kernel<<<blocks, 256, 0, stream>>>(x, h, n4);
-  SPD_CUDA_TRY(cudaGetLastError());
+  const int slot = trace_begin(stream);
+  SPD_CUDA_TRY(launch_pdl(bf16_to_f32_kernel, dim3(blocks), dim3(256), 0, stream, x, h, n4));
+  trace_end(slot, stream, TR_ROWS, 0.0, 6.0 * double(n));
   return SPD_OK;
 }
 
 int scatter_rows_run(const uint16_t* src, int n_rows, int D, const int32_t* rows, uint16_t* dst,
                      cudaStream_t stream) {
   if (n_rows <= 0) return SPD_OK;
-  scatter_rows_kernel<<<n_rows, 128, 0, stream>>>(src, D, rows, dst);
-  SPD_CUDA_TRY(cudaGetLastError());
+  const int slot = trace_begin(stream);
+  SPD_CUDA_TRY(launch_pdl(scatter_rows_kernel, dim3(n_rows), dim3(128), 0, stream, src, D, rows, dst));
+  trace_end(slot, stream, TR_ROWS, 0.0, 4.0 * double(n_rows) * D);
   return SPD_OK;
 }
 

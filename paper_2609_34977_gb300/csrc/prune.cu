@@ -18,6 +18,7 @@
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "trace.h"
 
 namespace spd {
 
@@ -112,6 +113,8 @@ __device__ __forceinline__ const float* feat_row(const PruneDims& p, int l, int 
 // ---- 1. a_v and inverse norms ---------------------------------------------------------------
 __global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float* __restrict__ attn,
                                                        PruneWs w) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int t = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * 8 + warp;
   if (i >= p.n) return;
@@ -135,6 +138,8 @@ __global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float*
 
 // ---- 2. anchors (Eq. 1) and stable token lists ------------------------------------------------
 __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
+  pdl_launch_dependents();
+  pdl_wait();
   __shared__ uint64_t keys[4096];
   __shared__ int tmp[32];
   const int t = blockIdx.x;
@@ -174,6 +179,8 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
 
 // ---- 3. a_i = max over anchors of cos(F^L_i, F^L_p) -------------------------------------------
 __global__ void __launch_bounds__(256) anchor_sim_kernel(PruneDims p, PruneWs w) {
+  pdl_launch_dependents();
+  pdl_wait();
   __shared__ float Us[32][33], As[32][33];
   __shared__ float red[8][32];
   const int t = blockIdx.z, tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
@@ -271,6 +278,8 @@ __device__ void compute_quotas(const int* sizes, int K, int n_cmp, int* quota) {
 }
 
 __global__ void __launch_bounds__(1024) kmeans_kernel(PruneDims p, PruneWs w) {
+  pdl_launch_dependents();
+  pdl_wait();
   extern __shared__ float ksm[];
   float* cent = ksm;                     // [K][d]
   float* sums = ksm + size_t(p.K) * p.d; // [K][d]
@@ -360,6 +369,8 @@ __global__ void __launch_bounds__(1024) kmeans_kernel(PruneDims p, PruneWs w) {
 
 // ---- 5. per-cluster sums of unit feature rows ----------------------------------------------
 __global__ void __launch_bounds__(128) cluster_sum_kernel(PruneDims p, PruneWs w) {
+  pdl_launch_dependents();
+  pdl_wait();
   extern __shared__ int csm[];
   int* ul = csm;                                       // [m]
   int8_t* asg = reinterpret_cast<int8_t*>(csm + p.m);  // [m]
@@ -387,6 +398,8 @@ __global__ void __launch_bounds__(128) cluster_sum_kernel(PruneDims p, PruneWs w
 
 // ---- 6. per-token Eq. 3 scores ----------------------------------------------------------------
 __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int t = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int j = blockIdx.x * 8 + warp;
   if (j >= p.m) return;
@@ -421,6 +434,8 @@ __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
 // ---- 7. per-cluster bottom-N_k, compaction, outputs -------------------------------------------
 __global__ void __launch_bounds__(1024) select_kernel(PruneDims p, PruneWs w, int32_t* keep_idx,
                                                       uint8_t* kind, int8_t* cluster, float* scores) {
+  pdl_launch_dependents();
+  pdl_wait();
   __shared__ uint64_t keys[4096];
   __shared__ uint8_t kept[4096];
   __shared__ int tmp[32];
@@ -482,6 +497,8 @@ __global__ void __launch_bounds__(1024) select_kernel(PruneDims p, PruneWs w, in
 __global__ void gather_bf16_kernel(const float* __restrict__ src, int n_tok, int d, int off,
                                    const int32_t* __restrict__ idx, int keep,
                                    __nv_bfloat16* __restrict__ dst, int* status) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int j = blockIdx.x, t = blockIdx.y;
   const int i = idx[size_t(t) * keep + j];
   if (i < 0 || i >= n_tok - off) {
@@ -589,10 +606,12 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
   if (!cv.fits()) return fail(SPD_ENOSPC, "prune workspace too small (%zu < %zu)", ws_bytes, cv.used);
   cudaStream_t st = static_cast<cudaStream_t>(stream_);
   const int T = p.n_tiles;
-  rowstats_kernel<<<dim3((p.n + 7) / 8, T), 256, 0, st>>>(p, attn, w);
-  anchor_kernel<<<T, 1024, 0, st>>>(p, w);
+  const int slot = trace_begin(st);
+  SPD_CUDA_TRY(launch_pdl(rowstats_kernel, dim3((p.n + 7) / 8, T), dim3(256), 0, st, p, attn, w));
+  SPD_CUDA_TRY(launch_pdl(anchor_kernel, dim3(T), dim3(1024), 0, st, p, w));
   if (p.n_anc > 0 && p.m > 0)
-    anchor_sim_kernel<<<dim3((p.m + 31) / 32, (p.n_anc + 31) / 32, T), 256, 0, st>>>(p, w);
+    SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel, dim3((p.m + 31) / 32, (p.n_anc + 31) / 32, T),
+                            dim3(256), 0, st, p, w));
   const size_t ksmem = size_t(2) * p.K * p.d * sizeof(float) + p.m + 16;
   static bool attr = false;
   if (!attr) {
@@ -600,13 +619,18 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
                                       2 * 24576 * 4 + 4096 + 16));
     attr = true;
   }
-  kmeans_kernel<<<T, 1024, ksmem, st>>>(p, w);
+  SPD_CUDA_TRY(launch_pdl(kmeans_kernel, dim3(T), dim3(1024), ksmem, st, p, w));
   if (p.m > 0) {
-    cluster_sum_kernel<<<dim3((p.d + 127) / 128, T), 128, size_t(p.m) * 5 + 16, st>>>(p, w);
-    score_kernel<<<dim3((p.m + 7) / 8, T), 256, 0, st>>>(p, w);
+    SPD_CUDA_TRY(launch_pdl(cluster_sum_kernel, dim3((p.d + 127) / 128, T), dim3(128),
+                            size_t(p.m) * 5 + 16, st, p, w));
+    SPD_CUDA_TRY(launch_pdl(score_kernel, dim3((p.m + 7) / 8, T), dim3(256), 0, st, p, w));
   }
-  select_kernel<<<T, 1024, 0, st>>>(p, w, keep_idx, kind, cluster, scores);
-  SPD_CUDA_TRY(cudaGetLastError());
+  SPD_CUDA_TRY(launch_pdl(select_kernel, dim3(T), dim3(1024), 0, st, p, w, keep_idx, kind, cluster,
+                          scores));
+  // algorithmic work per tile: every tapped layer's features and the attention read once, the
+  // kept indices written; anchor similarities (n - N_anc) N_anc d multiply-adds
+  trace_end(slot, st, TR_PRUNE, 2.0 * T * double(p.m) * p.n_anc * p.d,
+            T * (4.0 * p.L * double(p.n_tok) * p.d + 4.0 * p.H * p.n_att + 4.0 * p.keep + 6.0 * p.n));
   return SPD_OK;
 }
 
@@ -616,9 +640,8 @@ extern "C" int spd_gather_rows_bf16(const float* src, int n_tiles, int n_tok, in
   if (!src || !idx || !dst || n_tiles < 1 || keep < 1 || d < 4 || d % 4 || row_offset < 0 ||
       row_offset >= n_tok)
     return fail(SPD_EINVAL, "bad gather arguments");
-  gather_bf16_kernel<<<dim3(keep, n_tiles), 128, 0, static_cast<cudaStream_t>(stream_)>>>(
-      src, n_tok, d, row_offset, idx, keep, reinterpret_cast<__nv_bfloat16*>(dst),
-      ws ? static_cast<int*>(ws) : nullptr);
-  SPD_CUDA_TRY(cudaGetLastError());
+  SPD_CUDA_TRY(launch_pdl(gather_bf16_kernel, dim3(keep, n_tiles), dim3(128), 0,
+                          static_cast<cudaStream_t>(stream_), src, n_tok, d, row_offset, idx, keep,
+                          reinterpret_cast<__nv_bfloat16*>(dst), ws ? static_cast<int*>(ws) : nullptr));
   return SPD_OK;
 }

@@ -159,6 +159,16 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
 }
 
+// ---- programmatic dependent launch ------------------------------------------------------------
+// Lets the next kernel of the stream be scheduled (it still waits for this grid's completion
+// before it reads anything this grid wrote).
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+// Waits until the previous kernel of the stream has completed and its writes are visible. A no-op
+// when the kernel was launched without programmatic serialization.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Records the first device-side failure in a status word (0 = OK).
 __device__ __forceinline__ void set_status(int* status, int code) {
   if (status) atomicCAS(status, 0, code);

@@ -26,19 +26,24 @@ class SpiderPrefill:
     """Buffers and workspaces for a fixed batch layout.
 
     tiles_per_req[b] tiles and text_lens[b] text tokens for request b; `keep` tokens kept per tile
-    (keep = n_patch: no pruning, the dense baseline). skip_mask [L][T] host uint8 or None.
+    skip_mask [L][T] host uint8 or None. dense=True is the un-pruned baseline: every patch is kept
+    in order (no MSV-Prune call) and the same gather/projector/decoder kernels run.
     """
 
     def __init__(self, model: N.SpdModel, *, n_patch: int, has_cls: bool, d_vis: int,
                  n_feat_layers: int, final_layer: int, n_heads_vis: int, attn_form: int,
                  keep: int, tiles_per_req, text_lens, n_clusters: int = 4, kmeans_iters: int = 10,
-                 anchor_ratio: float = 0.7, layer_weight=None, device: str = "cuda"):
+                 anchor_ratio: float = 0.7, layer_weight=None, dense: bool = False,
+                 device: str = "cuda"):
         self.model = model
         cfg = model.cfg
         self.D = cfg["d_model"]
         self.tiles_per_req = list(tiles_per_req)
         self.text_lens = list(text_lens)
         self.n_tiles = int(sum(self.tiles_per_req))
+        self.dense = dense
+        if dense:
+            keep = n_patch
         self.keep = keep
         self.n_patch = n_patch
         self.n_tok = n_patch + (1 if has_cls else 0)
@@ -70,6 +75,8 @@ class SpiderPrefill:
         self.text_rows = torch.tensor(text_rows, dtype=torch.int32, device=dev)
         # buffers
         self.keep_idx = torch.empty(self.n_tiles, keep, dtype=torch.int32, device=dev)
+        if dense:
+            self.keep_idx.copy_(torch.arange(keep, dtype=torch.int32, device=dev).expand(self.n_tiles, keep))
         self.vis = torch.empty(self.n_tiles * keep, d_vis, dtype=torch.bfloat16, device=dev)
         self.x = torch.empty(self.T, self.D, dtype=torch.bfloat16, device=dev)
         self.h = torch.empty(self.T, self.D, dtype=torch.float32, device=dev)
@@ -84,7 +91,8 @@ class SpiderPrefill:
     def run(self, feats, attn, text, skip_mask, stream=None):
         """Enqueue one step on device inputs: feats (list of [n_tiles][n_tok][d_vis] fp32), attn,
         text [sum(text_lens)][D] bf16. Returns the logits tensor [B][vocab] (device)."""
-        N.spd_prune(self.prune_cfg, feats, attn, self.keep_idx, ws=self.ws_prune, stream=stream)
+        if not self.dense:
+            N.spd_prune(self.prune_cfg, feats, attn, self.keep_idx, ws=self.ws_prune, stream=stream)
         fin = int(self.prune_cfg.final_layer)
         N.spd_gather_rows_bf16(feats[fin], self.n_tiles, self.n_tok, self.d_vis,
                                1 if self.prune_cfg.has_cls else 0, self.keep_idx, self.keep, self.vis,

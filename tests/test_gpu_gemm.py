@@ -62,7 +62,8 @@ def test_linear_bias_gelu_bf16_and_scatter_add():
     assert N.spd_workspace_status(ws) == 0
 
 
-def test_linear_is_deterministic_across_runs():
+def test_linear_split_tiles_are_deterministic():
+    # K split across CTAs (32 weight tiles on every SM): partials summed in CTA order
     M, K, N_ = 256, 4096, 4096
     X, W = operands(M, K, N_, seed=2)
     ws = torch.zeros(N.spd_linear_workspace_size(M, N_), dtype=torch.uint8, device="cuda")
