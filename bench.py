@@ -43,6 +43,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--keep", type=int, default=192)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=32,
+                    help="decoder layers (profiling captures only; the benchmark is 32)")
     return ap.parse_args()
 
 
@@ -53,6 +55,20 @@ def peaks():
         return p["hbm_gbs"], p["bf16_tflops"], p["bf16_tflops_sustained"], "measured"
     except Exception:
         return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def gemm_traffic():
+    """DRAM bytes per GEMM launch from the committed ncu summary, if the GEMM source is unchanged."""
+    import hashlib
+    try:
+        txt = open(os.path.join(ROOT, "profiles", "gemm_sk_llava15_layer.md")).read()
+        kv = dict(l.split(": ", 1) for l in txt.splitlines() if l.startswith(("traffic_bytes", "source_sha")))
+        src = os.path.join(ROOT, "paper_2609_34977_gb300", "csrc", "gemm.cu")
+        if hashlib.sha256(open(src, "rb").read()).hexdigest() == kv["source_sha256"].strip():
+            return float(kv["traffic_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
 
 
 def workload_config(keep, mask, T):
@@ -103,8 +119,8 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
-def build_model(torch, N, synth, device):
-    cfg = dict(synth.LLAVA_7B_DECODER)
+def build_model(torch, N, synth, device, layers=32):
+    cfg = dict(synth.LLAVA_7B_DECODER, n_layers=layers)
     w = synth.decoder_weights(SEED, cfg, device=device)
     model = N.SpdModel(cfg, w)
     del w
@@ -219,7 +235,8 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl")
     dev = "cuda"
-    model, cfg = build_model(torch, N, synth, dev)
+    model, cfg = build_model(torch, N, synth, dev, a.layers)
+    L = cfg["n_layers"]
     m_llava = synth.skip_targets("llava-1.5-7b")
 
     def make(keep, dense):
@@ -228,9 +245,10 @@ def main():
                              tiles_per_req=[1], text_lens=[TEXT], dense=dense)
         if dense:
             return pipe, None
-        admit, target = synth.adaptive_plan(SEED + rank, 32, pipe.token_is_visual, SKIP_FRAC, m_llava,
-                                            ADMIT_LO, 16)
-        return pipe, N.spd_plan_adaptive(32, admit, target)
+        admit, target = synth.adaptive_plan(SEED + rank, L, pipe.token_is_visual, SKIP_FRAC,
+                                            m_llava[:L], min(ADMIT_LO, max(L // 2 - 1, 0)),
+                                            max(L // 2, min(ADMIT_LO, max(L // 2 - 1, 0)) + 1))
+        return pipe, N.spd_plan_adaptive(L, admit, target)
 
     v = synth.vision_tiles(SEED + rank, 1, N_PATCH, D_VIS, 2, H_VIS)
     feats = [torch.from_numpy(f).to(dev) for f in v["feats"]]
@@ -285,7 +303,7 @@ def main():
     else:
         roof = {"bound": "tensor", "achieved": tfs, "peak": tf_sust, "unit": "TFLOP/s",
                 "frac": tfs / tf_sust}
-    roof.update({"traffic": None, "kernel": "gemm_tc_kernel (tcgen05, all decoder/projector/LM-head GEMMs)",
+    roof.update({"traffic": gemm_traffic(), "traffic_unit": "bytes per launch (ncu, profiles/)", "kernel": "gemm_tc_kernel (tcgen05, all decoder/projector/LM-head GEMMs)",
                  "peak_source": f"{src} (MEASURED_PEAKS.json)", "launches_per_step": g["launches"] / a.steps,
                  "avg_launch_us": 1000.0 * g["ms"] / max(g["launches"], 1),
                  "arith_intensity_flop_per_byte": ai, "tensor_tflops": tfs,
@@ -331,7 +349,8 @@ def main():
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
                 "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-                "config": workload_config(a.keep, mask, spider.T),
+                "config": dict(workload_config(a.keep, mask, spider.T),
+                               **({} if L == 32 else {"profiling_only_layers": L})),
                 "dense": {"value": tokens / (ms_dense / 1000.0), "ms_per_step": ms_dense,
                           "decoder_tokens": dense.T, "speedup_spider_vs_dense": ms_dense / ms},
                 "roofline": roof, "kernels": kernels, "cpu_baseline": cpu,
