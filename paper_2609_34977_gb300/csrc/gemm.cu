@@ -5,6 +5,16 @@
 // tile) and the tokens on its N side (up to 256 per tile): every weight tile is streamed from HBM
 // once per token tile.
 //
+// Two schedules share the kernel:
+//  * cluster split-K, when the output has at most half as many tiles as there are SMs: a cluster of
+//    C (2, 4 or 8) CTAs owns one output tile, each CTA a contiguous K range. Once every CTA of the
+//    cluster has finished its MMAs (its stage ring is idle), each CTA pushes its TMEM accumulator,
+//    32-column chunk by chunk, into the ring of the chunk's owner CTA (chunk mod C) with posted
+//    distributed-shared-memory stores; after a cluster barrier each owner sums the C copies in rank
+//    order from its own shared memory and runs the fused epilogue. No global partials, no remote
+//    loads, deterministic.
+//  * persistent stream-K otherwise, below.
+//
 // Persistent stream-K: one CTA per SM. The work is the list of (tile, k-block) units in tile-major
 // order; CTA c takes the contiguous units [c U / G, (c+1) U / G). A run of units inside one tile is
 // a segment. A segment that covers the whole K range goes straight to the epilogue. Residual (ADD)
@@ -31,11 +41,15 @@
 #include <math.h>
 #include <stdio.h>
 
+#include <cooperative_groups.h>
+
 #include <mutex>
 
 #include "internal.h"
 #include "ptx.cuh"
 #include "trace.h"
+
+namespace cg = cooperative_groups;
 
 namespace spd {
 namespace {
@@ -52,7 +66,7 @@ constexpr int kCounters = 1 << 16;
 
 struct KArgs {
   int n_out, n_tok, k, tt, n_kb, n_ttiles, units, grid, stages, epi, ldo, rope_rows, head_dim,
-      out_cols, kbox;  // kbox: 64-wide boxes per stage (1 or 2); a k-block is kbox * 64 wide
+      out_cols, kbox, csplit;  // csplit: CTAs per output tile in cluster split-K (1 = stream-K)  // kbox: 64-wide boxes per stage (1 or 2); a k-block is kbox * 64 wide
   void* out;
   const int32_t* rows;
   const uint16_t* bias;
@@ -260,7 +274,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x;
-  const int u0 = unit_lo(c, a), u1 = unit_lo(c + 1, a);
+  int u0, u1;
+  if (a.csplit > 1) {  // cluster split-K: rank r of tile c / C owns k-blocks [r n_kb / C, (r+1) n_kb / C)
+    const int tile = c / a.csplit, r = c - tile * a.csplit;
+    u0 = tile * a.n_kb + r * a.n_kb / a.csplit;
+    u1 = tile * a.n_kb + (r + 1) * a.n_kb / a.csplit;
+  } else {
+    u0 = unit_lo(c, a);
+    u1 = unit_lo(c + 1, a);
+  }
   const SegPlan plan = seg_plan(u0, u1, a.n_kb);
 
   if (threadIdx.x == 0) {
@@ -424,6 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int valid = min(a.tt, a.n_tok - tok0);
       const int n = wt * kBM + row;
       const uint32_t tq = tmem + b * kAccCols + (static_cast<uint32_t>(q * 32) << 16);
+      if (a.csplit > 1) break;  // cluster split-K: the accumulator is pushed after the role loops
       // token metadata of this tile, staged once per segment
       const int et = threadIdx.x - 64;
       if (et < valid) {
@@ -522,6 +545,64 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   __syncthreads();
+  if (a.csplit > 1) {
+    // cluster reduction: every thread of every CTA of the cluster takes part in both barriers.
+    // Receive layout in each owner's ring: [sender][owned chunk][128 rows][36] fp32 (32 columns
+    // + 4 of padding: conflict-free 16-byte accesses).
+    cg::cluster_group cl = cg::this_cluster();
+    const int C = a.csplit, tile = c / C, r = c - tile * C;
+    const int wt = tile / a.n_ttiles, tt_i = tile - wt * a.n_ttiles;
+    const int tok0 = tt_i * a.tt;
+    const int valid = min(a.tt, a.n_tok - tok0);
+    const int cpo = (a.tt / 32 + C - 1) / C;  // chunks owned per CTA
+    float* recv = reinterpret_cast<float*>(smem);
+    const int et = threadIdx.x - 64;
+    if (et >= 0 && et < valid) {
+      trow[et] = a.rows ? a.rows[tok0 + et] : tok0 + et;
+      tpos[et] = a.pos ? a.pos[tok0 + et] : 0;
+    }
+    cl.sync();  // every ring of the cluster is idle
+    if (warp >= 2 && !flags[0]) {
+      const int q = warp & 3, half = (warp - 2) >> 2, row = q * 32 + lane;
+      tc_fence_after();
+      const uint32_t tq = tmem + (static_cast<uint32_t>(q * 32) << 16);
+      for (int ci = half; ci * 32 < valid; ci += 2) {
+        float v[32];
+        tmem_ld32(tq + ci * 32, v);
+        const int owner = ci % C, lc = ci / C;
+        const uint32_t dst =
+            dsmem_addr(recv + (size_t(r * cpo + lc) * kBM + row) * 36, uint32_t(owner));
+#pragma unroll
+        for (int g = 0; g < 8; ++g)
+          st_dsmem_v4(dst + g * 16, make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]));
+      }
+    }
+    cl.sync();  // all pushes have landed
+    if (warp >= 2 && !flags[0]) {
+      const int q = warp & 3, half = (warp - 2) >> 2, row = q * 32 + lane;
+      const int n = wt * kBM + row;
+      for (int lc = half; lc < cpo; lc += 2) {
+        const int ci = r + lc * C;
+        if (ci * 32 >= valid) break;
+        float acc[32];
+#pragma unroll
+        for (int jj = 0; jj < 32; ++jj) acc[jj] = 0.0f;
+        for (int sdr = 0; sdr < C; ++sdr) {
+          const float4* src =
+              reinterpret_cast<const float4*>(recv + (size_t(sdr * cpo + lc) * kBM + row) * 36);
+#pragma unroll
+          for (int g = 0; g < 8; ++g) {
+            const float4 x = src[g];
+            acc[4 * g] += x.x;
+            acc[4 * g + 1] += x.y;
+            acc[4 * g + 2] += x.z;
+            acc[4 * g + 3] += x.w;
+          }
+        }
+        epilogue_chunk(a, n, q, lane, wt, tok0 + ci * 32, acc, trow, tpos, tok0);
+      }
+    }
+  }
   if (threadIdx.x == 0 && flags[0]) {
     // drain: TMA loads issued but never consumed must land before the CTA exits
     for (int i = counts[1]; i < counts[0]; ++i) {
@@ -604,17 +685,29 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   const long long units = tiles * a.n_kb;
   if (units > 0x3fffffffLL) return fail(SPD_EUNSUPPORTED, "GEMM too large");
   a.units = int(units);
+  const int sms = num_sms();
+  const int stage_bytes = a.kbox * (kWBytes + a.tt * 128);
+  a.stages = kSmemPipe / stage_bytes;
+  if (a.stages > kMaxStages) a.stages = kMaxStages;
+  // cluster split-K when the tiles fill at most half the SMs: C CTAs per tile (each >= 1 k-block)
+  a.csplit = 1;
+  if (tiles * 2 <= sms) {
+    int C = 2;
+    while (C < 8 && tiles * C * 2 <= sms && C * 2 <= a.n_kb) C *= 2;
+    // the ring receives C copies of each CTA's share of 32-column chunks ([128][36] fp32 each)
+    const int chunks = a.tt / 32, cpo = (chunks + C - 1) / C;
+    const size_t recv = size_t(C) * cpo * kBM * 36 * sizeof(float);
+    if (C <= a.n_kb && recv <= size_t(a.stages) * stage_bytes) a.csplit = C;
+  }
   // one CTA per SM with at least 2 units each; every CTA owns two partial slots (head, tail)
-  long long grid = num_sms();
+  long long grid = sms;
   if (grid > (units + 1) / 2) grid = (units + 1) / 2;
   const size_t per_slot = size_t(a.tt) * kBM;
   if (size_t(2 * grid) * per_slot > s.partial_floats) grid = s.partial_floats / (2 * per_slot);
   if (grid < 1) grid = 1;
   if (units * (grid + 1) >= (1LL << 31)) return fail(SPD_EUNSUPPORTED, "GEMM too large");
+  if (a.csplit > 1) grid = tiles * a.csplit;
   a.grid = int(grid);
-  const int stage_bytes = a.kbox * (kWBytes + a.tt * 128);
-  a.stages = kSmemPipe / stage_bytes;
-  if (a.stages > kMaxStages) a.stages = kMaxStages;
   a.epi = p.epi;
   a.out = p.out;
   a.ldo = p.ldo;
@@ -640,7 +733,23 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   if (attr_err != cudaSuccess)
     return fail(SPD_ECUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
   const int slot = trace_begin(stream);
-  SPD_CUDA_TRY(launch_pdl(gemm_sk_kernel, dim3(a.grid), dim3(kThreads), smem, stream, map_w, map_x, a));
+  {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = a.csplit;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    SPD_CUDA_TRY(cudaLaunchKernelEx(&cfg, gemm_sk_kernel, map_w, map_x, a));
+  }
   if (slot >= 0) {
     // algorithmic work: valid output columns only; weights, activations and results move once
     const double cols = (p.epi == EPI_SWIGLU_BF16) ? 2.0 * p.out_cols : double(p.n_out);

@@ -3,10 +3,13 @@
 //   rowstats     a_v = head-mean of the attention (Sec. 4.1.1); 1/||F_l,i|| for every tapped layer
 //   anchors      top-N_anc of a_v by a bitonic sort of (a_v desc, index asc) keys (Eq. 1);
 //                stable lists of anchor and non-anchor tokens by block prefix sums
-//   anchor_sim   a_i = max_p cos(F^L_i, F^L_p) over anchors: a tiled fp32 product, max via atomicMax
-//                on order-preserving integer keys (exact, order independent)
-//   kmeans       Lloyd on raw F^L of the non-anchor tokens, fixed-order fp32 sums; Eq. 2 quotas
-//   cluster_sums per cluster and layer, sum_j F_l,j / ||F_l,j|| in token order
+//   anchor_sim   a_i = max_p cos(F^L_i, F^L_p) over anchors: a 64 x 64 register-tiled fp32 product,
+//                max via atomicMax on order-preserving integer keys (exact, order independent)
+//   kmeans       one thread-block cluster of 8 CTAs per tile, each owning a contiguous slice of the
+//                non-anchor tokens: Lloyd on raw F^L (assignment in each CTA, per-CTA sums in token
+//                order, cross-CTA sums in rank order through distributed shared memory), then the
+//                per-cluster, per-layer sums of unit feature rows, the sums of a_j, sizes and Eq. 2
+//                quotas
 //   scores       s_i = [sum_l w_l f_i . (S_l,k - f_i)] / (|C_k| - 1) + a_i + (A_k - a_i) / (|C_k| - 1),
 //                the per-token mean of Eq. 3's S_ij over the other members of its cluster
 //   select       per cluster the N_k lowest (score, index) keys; kept = anchors + selected, compacted
@@ -16,9 +19,13 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <cooperative_groups.h>
+
 #include "internal.h"
 #include "ptx.cuh"
 #include "trace.h"
+
+namespace cg = cooperative_groups;
 
 namespace spd {
 
@@ -178,49 +185,59 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
 }
 
 // ---- 3. a_i = max over anchors of cos(F^L_i, F^L_p) -------------------------------------------
+// CTA tile: 64 non-anchor tokens x 64 anchors, d in chunks of 32 through shared memory (stored
+// transposed), 4 x 4 dot products per thread.
 __global__ void __launch_bounds__(256) anchor_sim_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
-  __shared__ float Us[32][33], As[32][33];
-  __shared__ float red[8][32];
-  const int t = blockIdx.z, tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-  const int u0 = blockIdx.x * 32, p0 = blockIdx.y * 32;
+  __shared__ float Us[32][68], As[32][68];
+  const int t = blockIdx.z, tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  const int u0 = blockIdx.x * 64, p0 = blockIdx.y * 64;
   const int* ul = w.ulist + size_t(t) * p.m;
   const int* al = w.alist + size_t(t) * p.n_anc;
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
   for (int d0 = 0; d0 < p.d; d0 += 32) {
-    for (int e = threadIdx.x; e < 1024; e += 256) {
-      const int r = e >> 5, c = e & 31;
-      const bool dc = d0 + c < p.d;
-      Us[r][c] = (u0 + r < p.m && dc) ? feat_row(p, p.fin, t, ul[u0 + r])[d0 + c] : 0.0f;
-      As[r][c] = (p0 + r < p.n_anc && dc) ? feat_row(p, p.fin, t, al[p0 + r])[d0 + c] : 0.0f;
+    for (int e = threadIdx.x; e < 64 * 32; e += 256) {
+      const int r = e >> 5, dd = e & 31;
+      const bool dc = d0 + dd < p.d;
+      Us[dd][r] = (u0 + r < p.m && dc) ? feat_row(p, p.fin, t, ul[u0 + r])[d0 + dd] : 0.0f;
+      As[dd][r] = (p0 + r < p.n_anc && dc) ? feat_row(p, p.fin, t, al[p0 + r])[d0 + dd] : 0.0f;
     }
     __syncthreads();
 #pragma unroll 8
-    for (int c = 0; c < 32; ++c) {
-      const float u = Us[tx][c];
+    for (int dd = 0; dd < 32; ++dd) {
+      float a[4], b[4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) acc[q] += u * As[ty + 8 * q][c];
+      for (int i = 0; i < 4; ++i) a[i] = Us[dd][ty + 16 * i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) b[j] = As[dd][tx + 16 * j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] += a[i] * b[j];
     }
     __syncthreads();
   }
-  float best = -INFINITY;
-  if (u0 + tx < p.m) {
-    const float iu = w.inv[(size_t(p.fin) * p.n_tiles + t) * p.n + ul[u0 + tx]];
+  const float* inv = w.inv + size_t(p.fin) * p.n_tiles * p.n + size_t(t) * p.n;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int pa = p0 + ty + 8 * q;
-      if (pa < p.n_anc) {
-        const float ia = w.inv[(size_t(p.fin) * p.n_tiles + t) * p.n + al[pa]];
-        best = fmaxf(best, acc[q] * iu * ia);
+  for (int i = 0; i < 4; ++i) {
+    const int ur = u0 + ty + 16 * i;
+    float best = -INFINITY;
+    if (ur < p.m) {
+      const float iu = inv[ul[ur]];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int pa = p0 + tx + 16 * j;
+        if (pa < p.n_anc) best = fmaxf(best, acc[i][j] * iu * inv[al[pa]]);
       }
     }
-  }
-  red[ty][tx] = best;
-  __syncthreads();
-  if (ty == 0 && u0 + tx < p.m) {
-    for (int q = 1; q < 8; ++q) best = fmaxf(best, red[q][tx]);
-    atomicMax(&w.asim[size_t(t) * p.n + ul[u0 + tx]], ordered_key(best));
+#pragma unroll
+    for (int off = 8; off; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
+    if (tx == 0 && ur < p.m) atomicMax(&w.asim[size_t(t) * p.n + ul[ur]], ordered_key(best));
   }
 }
 
@@ -277,122 +294,145 @@ __device__ void compute_quotas(const int* sizes, int K, int n_cmp, int* quota) {
   }
 }
 
-__global__ void __launch_bounds__(1024) kmeans_kernel(PruneDims p, PruneWs w) {
+constexpr int kKC = 8;  // CTAs per tile in the K-means cluster
+
+// Sums over the CTAs of the cluster, in rank order, of the per-CTA column sums `part` (K x D in
+// every CTA's shared memory), for this CTA's slice of columns; `emit(k, c, value)` consumes them.
+template <typename F>
+__device__ __forceinline__ void cluster_column_reduce(cg::cluster_group& cl, float* part, int K, int D,
+                                                      int rank, F emit) {
+  const int c0 = rank * D / kKC, c1 = (rank + 1) * D / kKC, width = c1 - c0;
+  for (int e = threadIdx.x; e < K * width; e += blockDim.x) {
+    const int k = e / width, c = c0 + e % width;
+    float sum = 0.0f;
+    for (int rr = 0; rr < kKC; ++rr) sum += cl.map_shared_rank(part, rr)[k * D + c];
+    emit(k, c, sum);
+  }
+}
+
+__global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
+    kmeans_cluster_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
   extern __shared__ float ksm[];
-  float* cent = ksm;                     // [K][d]
-  float* sums = ksm + size_t(p.K) * p.d; // [K][d]
-  int8_t* asg = reinterpret_cast<int8_t*>(sums + size_t(p.K) * p.d);  // [m]
-  __shared__ int counts[SPD_MAX_CLUSTERS];
+  const int K = p.K, D = p.d, m = p.m;
+  float* cent = ksm;                      // [K][D] centroids (same in every CTA)
+  float* part = ksm + size_t(K) * D;      // [K][D] this CTA's column sums
+  __shared__ int cnt[SPD_MAX_CLUSTERS];   // this CTA's cluster sizes
+  __shared__ float asum_part[SPD_MAX_CLUSTERS];
   __shared__ int changed;
-  const int t = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m = p.m, K = p.K, D = p.d;
+  __shared__ int8_t asg[4096 / kKC + 1];
+  cg::cluster_group cl = cg::this_cluster();
+  const int rank = int(cl.block_rank());
+  const int t = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nw = blockDim.x >> 5;
+  const int j0 = rank * m / kKC, j1 = (rank + 1) * m / kKC, nl = j1 - j0;
   const int* ul = w.ulist + size_t(t) * m;
   if (m > 0) {
     for (int e = threadIdx.x; e < K * D; e += blockDim.x) {
       const int k = e / D, c = e % D;
       cent[e] = feat_row(p, p.fin, t, ul[(k * m) / K])[c];
     }
+  }
+  __syncthreads();
+  for (int it = 0; it < p.iters && m > 0; ++it) {
+    // assignment of this CTA's points
+    if (threadIdx.x == 0) changed = 0;
     __syncthreads();
-    for (int it = 0; it < p.iters; ++it) {
-      if (threadIdx.x == 0) changed = 0;
-      __syncthreads();
-      for (int j = warp; j < m; j += 32) {
-        const float* x = feat_row(p, p.fin, t, ul[j]);
-        float part[SPD_MAX_CLUSTERS];
+    for (int jj = warp; jj < nl; jj += nw) {
+      const float* x = feat_row(p, p.fin, t, ul[j0 + jj]);
+      float part_d[SPD_MAX_CLUSTERS];
 #pragma unroll
-        for (int k = 0; k < SPD_MAX_CLUSTERS; ++k) part[k] = 0.0f;
-        for (int c = lane; c < D; c += 32) {
-          const float xv = x[c];
-#pragma unroll
-          for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
-            if (k < K) {
-              const float df = xv - cent[k * D + c];
-              part[k] += df * df;
-            }
-        }
-        int best = 0;
-        float bd = 0.0f;
+      for (int k = 0; k < SPD_MAX_CLUSTERS; ++k) part_d[k] = 0.0f;
+      for (int c = lane; c < D; c += 32) {
+        const float xv = x[c];
 #pragma unroll
         for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
           if (k < K) {
-            const float dk = warp_sum(part[k]);
-            if (k == 0 || dk < bd) { bd = dk; best = k; }
+            const float df = xv - cent[k * D + c];
+            part_d[k] += df * df;
           }
-        if (lane == 0) {
-          if (it == 0 || asg[j] != best) changed = 1;
-          asg[j] = int8_t(best);
+      }
+      int best = 0;
+      float bd = 0.0f;
+#pragma unroll
+      for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
+        if (k < K) {
+          const float dk = warp_sum(part_d[k]);
+          if (k == 0 || dk < bd) {
+            bd = dk;
+            best = k;
+          }
         }
+      if (lane == 0) {
+        if (it == 0 || asg[jj] != best) changed = 1;
+        asg[jj] = int8_t(best);
       }
-      __syncthreads();
-      if (it > 0 && !changed) break;
-      if (threadIdx.x < K) counts[threadIdx.x] = 0;
-      __syncthreads();
-      for (int j = threadIdx.x; j < m; j += blockDim.x) atomicAdd(&counts[asg[j]], 1);
-      for (int e = threadIdx.x; e < K * D; e += blockDim.x) sums[e] = 0.0f;
-      __syncthreads();
-      for (int c = threadIdx.x; c < D; c += blockDim.x)
-        for (int j = 0; j < m; ++j) sums[asg[j] * D + c] += feat_row(p, p.fin, t, ul[j])[c];
-      __syncthreads();
-      for (int e = threadIdx.x; e < K * D; e += blockDim.x) {
-        const int k = e / D;
-        if (counts[k] > 0) cent[e] = sums[e] / float(counts[k]);
+    }
+    __syncthreads();
+    // this CTA's column sums and sizes
+    if (threadIdx.x < K) cnt[threadIdx.x] = 0;
+    for (int e = threadIdx.x; e < K * D; e += blockDim.x) part[e] = 0.0f;
+    __syncthreads();
+    for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) atomicAdd(&cnt[asg[jj]], 1);
+    for (int c = threadIdx.x; c < D; c += blockDim.x)
+      for (int jj = 0; jj < nl; ++jj) part[asg[jj] * D + c] += feat_row(p, p.fin, t, ul[j0 + jj])[c];
+    cl.sync();
+    int total_changed = 0;
+    for (int rr = 0; rr < kKC; ++rr) total_changed += *cl.map_shared_rank(&changed, rr);
+    if (it > 0 && total_changed == 0) break;  // cluster-uniform decision
+    // new centroids for this CTA's column slice, written into every CTA
+    cluster_column_reduce(cl, part, K, D, rank, [&](int k, int c, float sum) {
+      int n = 0;
+      for (int rr = 0; rr < kKC; ++rr) n += cl.map_shared_rank(cnt, rr)[k];
+      const float v = n > 0 ? sum / float(n) : cent[k * D + c];
+      for (int rr = 0; rr < kKC; ++rr) cl.map_shared_rank(cent, rr)[k * D + c] = v;
+    });
+    cl.sync();
+  }
+  // final assignment: sizes, the per-cluster sums of a_j, and the assignment itself
+  if (threadIdx.x < K) {
+    cnt[threadIdx.x] = 0;
+    asum_part[threadIdx.x] = 0.0f;
+  }
+  __syncthreads();
+  for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) {
+    atomicAdd(&cnt[asg[jj]], 1);
+    w.assign[size_t(t) * m + j0 + jj] = asg[jj];
+  }
+  if (threadIdx.x == 0)
+    for (int jj = 0; jj < nl; ++jj) asum_part[asg[jj]] += ordered_val(w.asim[size_t(t) * p.n + ul[j0 + jj]]);
+  // per layer: sums over each cluster of unit feature rows (F_l,j / ||F_l,j||)
+  for (int l = 0; l < p.L; ++l) {
+    const float* inv = w.inv + (size_t(l) * p.n_tiles + t) * p.n;
+    __syncthreads();
+    for (int e = threadIdx.x; e < K * D; e += blockDim.x) part[e] = 0.0f;
+    __syncthreads();
+    for (int c = threadIdx.x; c < D; c += blockDim.x)
+      for (int jj = 0; jj < nl; ++jj) {
+        const int i = ul[j0 + jj];
+        part[asg[jj] * D + c] += feat_row(p, l, t, i)[c] * inv[i];
       }
-      __syncthreads();
+    cl.sync();
+    float* csum = w.csum + (size_t(t) * p.L + l) * K * D;
+    cluster_column_reduce(cl, part, K, D, rank, [&](int k, int c, float sum) { csum[k * D + c] = sum; });
+    if (l == p.L - 1 && rank == 0 && threadIdx.x == 0) {
+      int sizes[SPD_MAX_CLUSTERS], q[SPD_MAX_CLUSTERS];
+      for (int k = 0; k < K; ++k) {
+        int n = 0;
+        float a = 0.0f;
+        for (int rr = 0; rr < kKC; ++rr) {
+          n += cl.map_shared_rank(cnt, rr)[k];
+          a += cl.map_shared_rank(asum_part, rr)[k];
+        }
+        sizes[k] = n;
+        w.counts[t * 16 + k] = n;
+        w.asum[t * 16 + k] = a;
+      }
+      compute_quotas(sizes, K, p.n_cmp, q);
+      for (int k = 0; k < K; ++k) w.quotas[t * 16 + k] = q[k];
     }
-  }
-  // final sizes, quotas, and per-cluster sums of a_j
-  if (threadIdx.x < K) counts[threadIdx.x] = 0;
-  __syncthreads();
-  for (int j = threadIdx.x; j < m; j += blockDim.x) {
-    atomicAdd(&counts[asg[j]], 1);
-    w.assign[size_t(t) * m + j] = asg[j];
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int q[SPD_MAX_CLUSTERS];
-    compute_quotas(counts, K, p.n_cmp, q);
-    for (int k = 0; k < K; ++k) {
-      w.counts[t * 16 + k] = counts[k];
-      w.quotas[t * 16 + k] = q[k];
-    }
-  }
-  if (warp < K) {
-    float s = 0.0f;
-    for (int j = lane; j < m; j += 32)
-      if (asg[j] == warp) s += ordered_val(w.asim[size_t(t) * p.n + ul[j]]);
-    s = warp_sum(s);
-    if (lane == 0) w.asum[t * 16 + warp] = s;
-  }
-}
-
-// ---- 5. per-cluster sums of unit feature rows ----------------------------------------------
-__global__ void __launch_bounds__(128) cluster_sum_kernel(PruneDims p, PruneWs w) {
-  pdl_launch_dependents();
-  pdl_wait();
-  extern __shared__ int csm[];
-  int* ul = csm;                                       // [m]
-  int8_t* asg = reinterpret_cast<int8_t*>(csm + p.m);  // [m]
-  const int t = blockIdx.y, c = blockIdx.x * 128 + threadIdx.x;
-  for (int j = threadIdx.x; j < p.m; j += 128) {
-    ul[j] = w.ulist[size_t(t) * p.m + j];
-    asg[j] = int8_t(w.assign[size_t(t) * p.m + j]);
-  }
-  __syncthreads();
-  if (c >= p.d) return;
-  for (int k = 0; k < p.K; ++k) {
-    float acc[SPD_MAX_FEAT_LAYERS] = {0.f, 0.f, 0.f, 0.f};
-    for (int j = 0; j < p.m; ++j) {
-      if (asg[j] != k) continue;
-#pragma unroll
-      for (int l = 0; l < SPD_MAX_FEAT_LAYERS; ++l)
-        if (l < p.L)
-          acc[l] += feat_row(p, l, t, ul[j])[c] * w.inv[(size_t(l) * p.n_tiles + t) * p.n + ul[j]];
-    }
-#pragma unroll
-    for (int l = 0; l < SPD_MAX_FEAT_LAYERS; ++l)
-      if (l < p.L) w.csum[((size_t(t) * p.L + l) * p.K + k) * p.d + c] = acc[l];
+    cl.sync();  // peers' shared memory is read above; keep it alive and unchanged until here
   }
 }
 
@@ -610,21 +650,18 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
   SPD_CUDA_TRY(launch_pdl(rowstats_kernel, dim3((p.n + 7) / 8, T), dim3(256), 0, st, p, attn, w));
   SPD_CUDA_TRY(launch_pdl(anchor_kernel, dim3(T), dim3(1024), 0, st, p, w));
   if (p.n_anc > 0 && p.m > 0)
-    SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel, dim3((p.m + 31) / 32, (p.n_anc + 31) / 32, T),
+    SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel, dim3((p.m + 63) / 64, (p.n_anc + 63) / 64, T),
                             dim3(256), 0, st, p, w));
-  const size_t ksmem = size_t(2) * p.K * p.d * sizeof(float) + p.m + 16;
+  const size_t ksmem = size_t(2) * p.K * p.d * sizeof(float);
   static bool attr = false;
   if (!attr) {
-    SPD_CUDA_TRY(cudaFuncSetAttribute(kmeans_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      2 * 24576 * 4 + 4096 + 16));
+    SPD_CUDA_TRY(cudaFuncSetAttribute(kmeans_cluster_kernel,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * 24576 * 4));
     attr = true;
   }
-  SPD_CUDA_TRY(launch_pdl(kmeans_kernel, dim3(T), dim3(1024), ksmem, st, p, w));
-  if (p.m > 0) {
-    SPD_CUDA_TRY(launch_pdl(cluster_sum_kernel, dim3((p.d + 127) / 128, T), dim3(128),
-                            size_t(p.m) * 5 + 16, st, p, w));
+  SPD_CUDA_TRY(launch_pdl(kmeans_cluster_kernel, dim3(kKC, T), dim3(512), ksmem, st, p, w));
+  if (p.m > 0)
     SPD_CUDA_TRY(launch_pdl(score_kernel, dim3((p.m + 7) / 8, T), dim3(256), 0, st, p, w));
-  }
   SPD_CUDA_TRY(launch_pdl(select_kernel, dim3(T), dim3(1024), 0, st, p, w, keep_idx, kind, cluster,
                           scores));
   // algorithmic work per tile: every tapped layer's features and the attention read once, the
