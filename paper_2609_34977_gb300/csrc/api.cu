@@ -365,6 +365,7 @@ extern "C" int spd_project(const spd_model* m, const uint16_t* vis, int rows, co
   SPD_CUDA_TRY(cudaMemsetAsync(s.counters, 0, s.n_counters * sizeof(int), st));
   GemmProblem p{};
   p.map_w = &m->m_p1;
+  p.w = m->pw1;
   p.x = vis;
   p.n_out = m->cfg.d_proj;
   p.n_tok = rows;
@@ -375,6 +376,7 @@ extern "C" int spd_project(const spd_model* m, const uint16_t* vis, int rows, co
   p.bias = m->pb1;
   if (int rc = gemm_run(p, s, st)) return rc;
   p.map_w = &m->m_p2;
+  p.w = m->pw2;
   p.x = hid;
   p.n_out = m->cfg.d_model;
   p.k = m->cfg.d_proj;
@@ -531,6 +533,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
     if (rc) break;
     GemmProblem kvp{};
     kvp.map_w = &W.m_kv;
+    kvp.w = W.wkv;
     kvp.x = bf.xa;
     kvp.n_out = 2 * kvd;
     kvp.n_tok = T;
@@ -546,6 +549,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
     if (q.na > 0) {
       GemmProblem qp = kvp;
       qp.map_w = &W.m_q;
+      qp.w = W.wq;
       qp.x = bf.xq;
       qp.n_out = qd;
       qp.n_tok = q.na;
@@ -560,6 +564,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
         break;
       GemmProblem op{};
       op.map_w = &W.m_o;
+      op.w = W.wo;
       op.x = bf.o;
       op.n_out = D;
       op.n_tok = q.na;
@@ -576,6 +581,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
         break;
       GemmProblem gp{};
       gp.map_w = &W.m_gu;
+      gp.w = W.wgu;
       gp.x = bf.y;
       gp.n_out = m->gu_rows;
       gp.n_tok = q.nf;
@@ -587,6 +593,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
       if ((rc = gemm_run(gp, bf.gs, st))) break;
       GemmProblem dp{};
       dp.map_w = &W.m_d;
+      dp.w = W.wd;
       dp.x = bf.act;
       dp.n_out = D;
       dp.n_tok = q.nf;
@@ -604,6 +611,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
       return rc;
     GemmProblem lp{};
     lp.map_w = &m->m_lm;
+    lp.w = m->lm_head;
     lp.x = bf.z;
     lp.n_out = c.vocab;
     lp.n_tok = B;

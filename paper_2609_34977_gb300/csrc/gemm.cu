@@ -1,18 +1,19 @@
 // tcgen05 bf16 GEMM for the decoder's dense contractions: out = epilogue(X W^T).
 //
 // Prefill after pruning has few token rows (a few hundred) against large weight matrices, so the
-// contraction is weight-stream bound. The WEIGHTS sit on the MMA's M side (128 weight rows per
-// tile) and the tokens on its N side (up to 256 per tile): every weight tile is streamed from HBM
-// once per token tile.
+// contraction is weight-stream bound. The WEIGHTS sit on the MMA's M side and the tokens on its N
+// side (up to 256 per tile): every weight tile is streamed from HBM once per token tile. A tile is
+// 128 weight rows, or 256 (two M = 128 MMAs sharing each token box) when the token tile is at most
+// 64 wide and the stages would otherwise carry few weight bytes.
 //
 // Two schedules share the kernel:
 //  * cluster split-K, when the output has at most half as many tiles as there are SMs: a cluster of
 //    C (2, 4 or 8) CTAs owns one output tile, each CTA a contiguous K range. Once every CTA of the
-//    cluster has finished its MMAs (its stage ring is idle), each CTA pushes its TMEM accumulator,
-//    32-column chunk by chunk, into the ring of the chunk's owner CTA (chunk mod C) with posted
-//    distributed-shared-memory stores; after a cluster barrier each owner sums the C copies in rank
-//    order from its own shared memory and runs the fused epilogue. No global partials, no remote
-//    loads, deterministic.
+//    cluster has finished its MMAs (its stage ring is idle), each CTA pushes one 128-row half of its
+//    TMEM accumulator, 32-column chunk by chunk, into the ring of the chunk's owner CTA (chunk mod
+//    C) with posted distributed-shared-memory stores; after a cluster barrier each owner sums the C
+//    copies in rank order from its own shared memory and runs the fused epilogue; then the second
+//    half. No global partials, no remote loads, deterministic.
 //  * persistent stream-K otherwise, below.
 //
 // Persistent stream-K: one CTA per SM. The work is the list of (tile, k-block) units in tile-major
@@ -25,24 +26,32 @@
 // the tile's k-block count sums the partials in CTA order and runs the epilogue. No CTA ever waits
 // on another.
 //
-// Stages hold BK = 64 or 128 K elements: one or two weight boxes of 128 rows x 64 (128 B per row
-// each, so a 128-wide stage reads 256 contiguous bytes of every weight row) and one or two token
-// boxes of the whole token tile x 64. Few large boxes matter: the TMA box rate, not bytes, caps the
-// stream when the token tile is cut into small boxes.
+// Stages hold BK = 64 or 128 K elements: one or two weight boxes of 128 nh rows x 64 (a 128-wide
+// stage reads 256 contiguous bytes of every weight row) and one or two token boxes of the whole
+// token tile x 64. Few large boxes matter: the TMA box rate, not bytes, caps the stream when a tile
+// is cut into small boxes.
+//
+// The kernel is instantiated once per epilogue, and every epilogue works on 8 accumulator columns
+// at a time (tcgen05.ld x8, a rolled loop around an 8-wide body): with all epilogues inlined and
+// unrolled over 32 columns the code outgrew the instruction cache and the epilogue ran several
+// times slower than its arithmetic and stores.
 //
 // Warp roles (320 threads):
 //   warp 0 lane 0 : TMA producer  - fills the ring of stages
-//   warp 1 lane 0 : MMA issuer    - BK / 16 x tcgen05.mma (K = 16) per stage into one of two TMEM
-//                                   accumulators (2 x 256 columns), commit per stage and segment
-//   warps 2..9    : epilogue      - two warps per TMEM lane quarter, alternating 32-column chunks;
-//                                   tcgen05.ld, fused epilogue; runs on one accumulator while the
-//                                   MMA fills the other
+//   warp 1 lane 0 : MMA issuer    - nh x BK / 16 tcgen05.mma (M = 128, K = 16) per stage into the
+//                                   128-row halves of a TMEM accumulator; commit per stage and per
+//                                   segment. Two accumulators fit in the 512 TMEM columns unless
+//                                   nh = 2 with a token tile wider than 128 (the epilogue drains
+//                                   one while the MMA fills the other).
+//   warps 2..9    : epilogue      - two warps per TMEM lane quarter, alternating 8-column groups;
+//                                   tcgen05.ld, fused epilogue
 #include <cuda_bf16.h>
 #include <math.h>
 #include <stdio.h>
 
 #include <cooperative_groups.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "internal.h"
@@ -54,19 +63,24 @@ namespace cg = cooperative_groups;
 namespace spd {
 namespace {
 
-constexpr int kBM = 128;            // weight rows per tile (MMA M)
-constexpr int kBK = 64;             // K elements per TMA box (one 128-byte swizzle row)
-constexpr int kWBytes = kBM * 128;  // weight box bytes
+constexpr int kBM = 128;            // weight rows per MMA (M) and per TMEM lane set
+constexpr int kBK = 64;             // K elements per box (one 128-byte swizzle row)
+constexpr int kHalfW = kBM * 128;   // bytes of 128 weight rows x 64
 constexpr int kMaxStages = 8;
 constexpr int kSmemPipe = 196608;   // bytes of the stage ring
-constexpr int kAccCols = 256;       // TMEM columns per accumulator
+constexpr int kAccCols = 256;       // TMEM columns per accumulator buffer (double-buffered tiles)
 constexpr int kThreads = 320;
 constexpr int kEpiThreads = 256;
 constexpr int kCounters = 1 << 16;
+constexpr int kRecvPitch = 36;      // fp32 per row of a received 32-column chunk (conflict-free)
 
 struct KArgs {
-  int n_out, n_tok, k, tt, n_kb, n_ttiles, units, grid, stages, epi, ldo, rope_rows, head_dim,
-      out_cols, kbox, csplit;  // csplit: CTAs per output tile in cluster split-K (1 = stream-K)  // kbox: 64-wide boxes per stage (1 or 2); a k-block is kbox * 64 wide
+  int n_out, n_tok, k, tt, n_kb, n_ttiles, units, grid, stages, ldo, rope_rows, head_dim,
+      out_cols, kbox, csplit, nbuf, hoff, nh;
+  // kbox: 64-wide boxes per stage (1 or 2); a k-block is kbox * 64 wide
+  // csplit: CTAs per output tile in cluster split-K (1 = stream-K)
+  // nbuf: TMEM accumulator buffers; hoff: TMEM column offset of the second 128-row half
+  // nh: 128-row halves per tile (1 or 2)
   void* out;
   const int32_t* rows;
   const uint16_t* bias;
@@ -150,89 +164,82 @@ __device__ __forceinline__ void seg_get(const SegPlan& p, int j, int& s, int& e)
   e = s + p.n_kb;
 }
 
-// Applies the epilogue to 32 consecutive tokens t0..t0+31 of weight row n (TMEM lane quarter q).
-// trow / tpos: output row and rotary position of each token of the token tile (shared memory,
-// indexed from the tile's first token tb).
-__device__ __forceinline__ void epilogue_chunk(const KArgs& a, int n, int q, int lane, int w_tile,
-                                               int t0, const float (&v)[32], const int* trow,
-                                               const int* tpos, int tb) {
+// Applies epilogue EPI to 8 consecutive tokens t0..t0+7 of weight row n (TMEM lane quarter q;
+// w_tile = the 128-row block n / 128). trow / tpos: output row and rotary position of each token
+// of the token tile (shared memory, indexed from the tile's first token tb). Warp-uniform calls.
+template <int EPI>
+__device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane, int w_tile,
+                                          int t0, const float (&v)[8], const int* trow,
+                                          const int* tpos, int tb) {
   const int nt = a.n_tok;
-  switch (a.epi) {
-    case EPI_F32:
-    case EPI_ADD_F32: {
-      if (n >= a.n_out) return;
-      float* o = static_cast<float*>(a.out);
+  if constexpr (EPI == EPI_F32 || EPI == EPI_ADD_F32) {
+    if (n >= a.n_out) return;
+    float* o = static_cast<float*>(a.out);
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
+    for (int j = 0; j < 8; ++j) {
+      const int t = t0 + j;
+      if (t < nt) {
+        float* p = o + size_t(trow[t - tb]) * a.ldo + n;
+        if constexpr (EPI == EPI_ADD_F32) atomicAdd(p, v[j]);  // fire-and-forget red.add
+        else *p = v[j];
+      }
+    }
+  } else if constexpr (EPI == EPI_BF16 || EPI == EPI_BIAS_BF16 || EPI == EPI_BIAS_GELU_BF16) {
+    if (n >= a.n_out) return;
+    __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out);
+    const float b =
+        (EPI == EPI_BF16) ? 0.0f : __bfloat162float(__ushort_as_bfloat16(a.bias[n]));
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int t = t0 + j;
+      if (t < nt) {
+        float x = v[j] + b;
+        if constexpr (EPI == EPI_BIAS_GELU_BF16) x = gelu_erf(x);
+        o[size_t(trow[t - tb]) * a.ldo + n] = __float2bfloat16_rn(x);
+      }
+    }
+  } else if constexpr (EPI == EPI_ROPE_BF16) {
+    __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out);
+    if (n < a.rope_rows) {  // warp-uniform: rope_rows is a multiple of 32
+      const int hd = a.head_dim, half = hd >> 1;
+      const int head = n / hd, g = (n % hd) >> 5;
+      const int jf = 16 * g + (lane & 15);
+      const int col = head * hd + ((lane < 16) ? jf : half + jf);
+      float2 cs[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {  // the table loads first, all in flight together
+        const int t = min(t0 + j, nt - 1);
+        cs[j] = a.rope[size_t(tpos[t - tb]) * half + jf];
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float p = __shfl_xor_sync(0xffffffffu, v[j], 16);
         const int t = t0 + j;
         if (t < nt) {
-          float* p = o + size_t(trow[t - tb]) * a.ldo + n;
-          if (a.epi == EPI_ADD_F32) atomicAdd(p, v[j]);  // fire-and-forget red.add
-          else *p = v[j];
+          const float y = (lane < 16) ? v[j] * cs[j].x - p * cs[j].y : v[j] * cs[j].x + p * cs[j].y;
+          o[size_t(trow[t - tb]) * a.ldo + col] = __float2bfloat16_rn(y);
         }
       }
-      return;
-    }
-    case EPI_BF16:
-    case EPI_BIAS_BF16:
-    case EPI_BIAS_GELU_BF16: {
-      if (n >= a.n_out) return;
-      __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out);
-      const float b = (a.epi == EPI_BF16) ? 0.0f
-                                          : __bfloat162float(__ushort_as_bfloat16(a.bias[n]));
+    } else if (n < a.n_out) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
+      for (int j = 0; j < 8; ++j) {
         const int t = t0 + j;
-        if (t < nt) {
-          float x = v[j] + b;
-          if (a.epi == EPI_BIAS_GELU_BF16) x = gelu_erf(x);
-          o[size_t(trow[t - tb]) * a.ldo + n] = __float2bfloat16_rn(x);
-        }
+        if (t < nt) o[size_t(trow[t - tb]) * a.ldo + n] = __float2bfloat16_rn(v[j]);
       }
-      return;
     }
-    case EPI_ROPE_BF16: {
-      __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out);
-      if (n < a.rope_rows) {  // tile-uniform: rope_rows is a multiple of 128
-        const int hd = a.head_dim, half = hd >> 1;
-        const int head = n / hd, g = (n % hd) >> 5;
-        const int jf = 16 * g + (lane & 15);
-        const int col = head * hd + ((lane < 16) ? jf : half + jf);
+  } else if constexpr (EPI == EPI_SWIGLU_BF16) {
+    __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out);
+    const int f = w_tile * 64 + q * 16 + (lane & 15);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const float p = __shfl_xor_sync(0xffffffffu, v[j], 16);
-          const int t = t0 + j;
-          if (t < nt) {
-            const float2 cs = a.rope[size_t(tpos[t - tb]) * half + jf];
-            const float y = (lane < 16) ? v[j] * cs.x - p * cs.y : v[j] * cs.x + p * cs.y;
-            o[size_t(trow[t - tb]) * a.ldo + col] = __float2bfloat16_rn(y);
-          }
-        }
-      } else {
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const int t = t0 + j;
-          if (t < nt) o[size_t(trow[t - tb]) * a.ldo + n] = __float2bfloat16_rn(v[j]);
-        }
+    for (int j = 0; j < 8; ++j) {
+      const float u = __shfl_xor_sync(0xffffffffu, v[j], 16);
+      const int t = t0 + j;
+      if (lane < 16 && t < nt && f < a.out_cols) {
+        const float g = v[j];
+        // SiLU(g) u; __fdividef gives 0 once 1 + e^-g passes 2^126, the limit of g / (1 + e^-g)
+        o[size_t(trow[t - tb]) * a.ldo + f] = __float2bfloat16_rn(__fdividef(g, 1.0f + __expf(-g)) * u);
       }
-      return;
     }
-    case EPI_SWIGLU_BF16: {
-      __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out);
-      const int f = w_tile * 64 + q * 16 + (lane & 15);
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const float u = __shfl_xor_sync(0xffffffffu, v[j], 16);
-        const int t = t0 + j;
-        if (lane < 16 && t < nt && f < a.out_cols) {
-          const float g = v[j];
-          o[size_t(trow[t - tb]) * a.ldo + f] = __float2bfloat16_rn(g / (1.0f + expf(-g)) * u);
-        }
-      }
-      return;
-    }
-    default:
-      return;
   }
 }
 
@@ -253,6 +260,14 @@ __device__ __forceinline__ bool epi_any(bool v) {
   return r != 0;
 }
 
+__device__ __forceinline__ void add4(float (&acc)[8], int o, const float4& x) {
+  acc[o] += x.x;
+  acc[o + 1] += x.y;
+  acc[o + 2] += x.z;
+  acc[o + 3] += x.w;
+}
+
+template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_sk_kernel(const __grid_constant__ CUtensorMap map_w,
                    const __grid_constant__ CUtensorMap map_x, const KArgs a) {
@@ -260,7 +275,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   const uint32_t xbox_bytes = a.tt * 128;
-  const uint32_t stage_bytes = a.kbox * (kWBytes + xbox_bytes);
+  const uint32_t wbox_bytes = a.nh * kHalfW;
+  const uint32_t stage_bytes = a.kbox * (wbox_bytes + xbox_bytes);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.stages * stage_bytes);
   uint64_t* empty = full + kMaxStages;
   uint64_t* accf = empty + kMaxStages;  // [2] accumulator ready (MMA -> epilogue)
@@ -331,8 +347,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t* st = smem + n_pre * stage_bytes;
           mbar_arrive_expect_tx(&full[n_pre], stage_bytes);
           for (int bx = 0; bx < a.kbox; ++bx)
-            tma_load_2d(st + bx * kWBytes, &map_w, &full[n_pre], (pre_kb[n_pre] * a.kbox + bx) * kBK,
-                        wt * kBM, pol_w);
+            tma_load_2d(st + bx * wbox_bytes, &map_w, &full[n_pre],
+                        (pre_kb[n_pre] * a.kbox + bx) * kBK, wt * a.nh * kBM, pol_w);
         }
       }
       pdl_wait();
@@ -340,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int tt_i = pre_tile[i] - (pre_tile[i] / a.n_ttiles) * a.n_ttiles;
         uint8_t* st = smem + i * stage_bytes;
         for (int bx = 0; bx < a.kbox; ++bx)
-          tma_load_2d(st + a.kbox * kWBytes + bx * xbox_bytes, &map_x, &full[i],
+          tma_load_2d(st + a.kbox * wbox_bytes + bx * xbox_bytes, &map_x, &full[i],
                       (pre_kb[i] * a.kbox + bx) * kBK, tt_i * a.tt, pol_x);
       }
       counts[0] = n_pre;
@@ -364,10 +380,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t* st = smem + s * stage_bytes;
           mbar_arrive_expect_tx(&full[s], stage_bytes);
           for (int bx = 0; bx < a.kbox; ++bx) {
-            const int kx = (kb * a.kbox + bx) * kBK;
-            tma_load_2d(st + bx * kWBytes, &map_w, &full[s], kx, wt * kBM, pol_w);
-            tma_load_2d(st + a.kbox * kWBytes + bx * xbox_bytes, &map_x, &full[s], kx, tt_i * a.tt,
-                        pol_x);
+            const int ks = kb * a.kbox + bx;
+            tma_load_2d(st + bx * wbox_bytes, &map_w, &full[s], ks * kBK, wt * a.nh * kBM, pol_w);
+            tma_load_2d(st + a.kbox * wbox_bytes + bx * xbox_bytes, &map_x, &full[s], ks * kBK,
+                        tt_i * a.tt, pol_x);
           }
           counts[0] = i + 1;
         }
@@ -384,8 +400,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < plan.count && ok; ++j) {
         int u, seg_end;
         seg_get(plan, j, u, seg_end);
-        const int b = j & 1;
-        if (!mbar_wait(&acce[b], ((j >> 1) & 1) ^ 1, flags, a.budget)) {
+        const int b = j % a.nbuf;
+        if (!mbar_wait(&acce[b], ((j / a.nbuf) & 1) ^ 1, flags, a.budget)) {
           ok = false;
           break;
         }
@@ -400,12 +416,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
           const uint32_t sw = smem_u32(smem + s * stage_bytes);
-          const uint32_t sx = sw + a.kbox * kWBytes;
+          const uint32_t sx = sw + a.kbox * wbox_bytes;
           for (int kk = 0; kk < ksub; ++kk) {
             const uint32_t off = (kk & 3) * 32;
-            mma_bf16(d, sdesc_k128(sw + (kk >> 2) * kWBytes + off),
-                     sdesc_k128(sx + (kk >> 2) * xbox_bytes + off), idesc,
-                     (uu != u || kk != 0) ? 1u : 0u);
+            const uint64_t bdesc = sdesc_k128(sx + (kk >> 2) * xbox_bytes + off);
+            const uint32_t accum = (uu != u || kk != 0) ? 1u : 0u;
+            for (int h = 0; h < a.nh; ++h)
+              mma_bf16(d + h * a.hoff, sdesc_k128(sw + (kk >> 2) * wbox_bytes + h * kHalfW + off),
+                       bdesc, idesc, accum);
           }
           mma_commit(&empty[s]);
           counts[1] = i + 1;
@@ -423,7 +441,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     pdl_wait();
-    // ---- epilogue (warps 2..9; warp w reads TMEM lane quarter w % 4, chunk parity (w - 2) / 4) ----
+    // ---- epilogue (warps 2..9; warp w reads TMEM lane quarter w % 4 and the 8-column groups of
+    // parity (w - 2) / 4) ----
     const int q = warp & 3;
     const int half = (warp - 2) >> 2;
     const int row = q * 32 + lane;
@@ -433,20 +452,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int tile = u / a.n_kb;
       const int kb_lo = u - tile * a.n_kb;
       const int seg_len = seg_end - u;
-      const int b = j & 1;
-      const bool got = mbar_wait(&accf[b], (j >> 1) & 1, flags, a.budget);
+      const int b = j % a.nbuf;
+      const bool got = mbar_wait(&accf[b], (j / a.nbuf) & 1, flags, a.budget);
       if (epi_any(!got)) {  // every epilogue thread leaves together
         flags[0] = 1;
         set_status(a.status, SPD_ETIMEOUT);
         break;
       }
       tc_fence_after();
+      if (a.csplit > 1) break;  // cluster split-K: the accumulator is pushed after the role loops
       const int wt = tile / a.n_ttiles, tt_i = tile - wt * a.n_ttiles;
       const int tok0 = tt_i * a.tt;
       const int valid = min(a.tt, a.n_tok - tok0);
-      const int n = wt * kBM + row;
       const uint32_t tq = tmem + b * kAccCols + (static_cast<uint32_t>(q * 32) << 16);
-      if (a.csplit > 1) break;  // cluster split-K: the accumulator is pushed after the role loops
       // token metadata of this tile, staged once per segment
       const int et = threadIdx.x - 64;
       if (et < valid) {
@@ -454,26 +472,33 @@ __global__ void __launch_bounds__(kThreads, 1)
         tpos[et] = a.pos ? a.pos[tok0 + et] : 0;
       }
       epi_bar();
-      if ((kb_lo == 0 && seg_len == a.n_kb) || a.epi == EPI_ADD_F32) {
-        for (int cc = half * 32; cc < valid; cc += 64) {
-          float v[32];
-          tmem_ld32(tq + cc, v);
-          epilogue_chunk(a, n, q, lane, wt, tok0 + cc, v, trow, tpos, tok0);
+      if ((kb_lo == 0 && seg_len == a.n_kb) || EPI == EPI_ADD_F32) {
+        for (int h = 0; h < a.nh; ++h) {
+#pragma unroll 1
+          for (int cc = half * 8; cc < valid; cc += 16) {
+            float v[8];
+            tmem_ld8(tq + h * a.hoff + cc, v);
+            epilogue8<EPI>(a, (a.nh * wt + h) * kBM + row, q, lane, a.nh * wt + h, tok0 + cc, v,
+                           trow, tpos, tok0);
+          }
         }
       } else {
         // deterministic split tile: partial into this CTA's head (0) or tail (1) slot, laid out
-        // [32-column chunk][4-column group][128 rows] of float4 (512 contiguous bytes per warp
+        // [row half][4-column group][128 rows] of float4 (512 contiguous bytes per warp
         // instruction); the last arriver sums the partials in CTA order
-        const size_t slot_len = size_t(a.tt / 4) * kBM;
+        const size_t half_len = size_t(a.tt / 4) * kBM;
+        const size_t slot_len = a.nh * half_len;
         float4* part = reinterpret_cast<float4*>(a.partial);
         float4* mine = part + size_t(2 * c + (tile == u0 / a.n_kb ? 0 : 1)) * slot_len;
-        for (int cc = half * 32; cc < valid; cc += 64) {
-          float v[32];
-          tmem_ld32(tq + cc, v);
-          float4* dst = mine + size_t(cc / 4) * kBM + row;
-#pragma unroll
-          for (int g = 0; g < 8; ++g)
-            __stcg(dst + g * kBM, make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]));
+        for (int h = 0; h < a.nh; ++h) {
+#pragma unroll 1
+          for (int cc = half * 8; cc < valid; cc += 16) {
+            float v[8];
+            tmem_ld8(tq + h * a.hoff + cc, v);
+            float4* dst = mine + h * half_len + size_t(cc / 4) * kBM + row;
+            __stcg(dst, make_float4(v[0], v[1], v[2], v[3]));
+            __stcg(dst + kBM, make_float4(v[4], v[5], v[6], v[7]));
+          }
         }
         __threadfence();
         epi_bar();
@@ -486,55 +511,52 @@ __global__ void __launch_bounds__(kThreads, 1)
           __threadfence();
           const int c_first = cta_of_unit(tile * a.n_kb, a);
           const int c_last = cta_of_unit((tile + 1) * a.n_kb - 1, a);
-          for (int cc = half * 32; cc < valid; cc += 64) {
-            float v[32], acc[32];
-            tmem_ld32(tq + cc, v);
+          for (int h = 0; h < a.nh; ++h) {
+#pragma unroll 1
+            for (int cc = half * 8; cc < valid; cc += 16) {
+              float v[8], acc[8];
+              tmem_ld8(tq + h * a.hoff + cc, v);
 #pragma unroll
-            for (int jj = 0; jj < 32; ++jj) acc[jj] = 0.0f;
-            // contributors in CTA order, two partial tiles in flight at a time
-            for (int o = c_first; o <= c_last; o += 2) {
-              float4 x0[8], x1[8];
-              const bool l0 = (o != c), l1 = (o + 1 <= c_last) && (o + 1 != c);
-              if (l0) {
-                const int os = 2 * o + (tile == unit_lo(o, a) / a.n_kb ? 0 : 1);
-                const float4* src = part + size_t(os) * slot_len + size_t(cc / 4) * kBM + row;
-#pragma unroll
-                for (int g = 0; g < 8; ++g) x0[g] = __ldcg(src + g * kBM);
-              }
-              if (l1) {
-                const int os = 2 * (o + 1) + (tile == unit_lo(o + 1, a) / a.n_kb ? 0 : 1);
-                const float4* src = part + size_t(os) * slot_len + size_t(cc / 4) * kBM + row;
-#pragma unroll
-                for (int g = 0; g < 8; ++g) x1[g] = __ldcg(src + g * kBM);
-              }
-              if (l0) {
-#pragma unroll
-                for (int g = 0; g < 8; ++g) {
-                  acc[4 * g] += x0[g].x;
-                  acc[4 * g + 1] += x0[g].y;
-                  acc[4 * g + 2] += x0[g].z;
-                  acc[4 * g + 3] += x0[g].w;
+              for (int jj = 0; jj < 8; ++jj) acc[jj] = 0.0f;
+              // contributors in CTA order, two partial tiles in flight at a time
+#pragma unroll 1
+              for (int o = c_first; o <= c_last; o += 2) {
+                float4 x[4];
+                const bool l0 = (o != c), l1 = (o + 1 <= c_last) && (o + 1 != c);
+                if (l0) {
+                  const int os = 2 * o + (tile == unit_lo(o, a) / a.n_kb ? 0 : 1);
+                  const float4* src =
+                      part + size_t(os) * slot_len + h * half_len + size_t(cc / 4) * kBM + row;
+                  x[0] = __ldcg(src);
+                  x[1] = __ldcg(src + kBM);
                 }
-              } else {
-#pragma unroll
-                for (int jj = 0; jj < 32; ++jj) acc[jj] += v[jj];
-              }
-              if (o + 1 <= c_last) {
                 if (l1) {
-#pragma unroll
-                  for (int g = 0; g < 8; ++g) {
-                    acc[4 * g] += x1[g].x;
-                    acc[4 * g + 1] += x1[g].y;
-                    acc[4 * g + 2] += x1[g].z;
-                    acc[4 * g + 3] += x1[g].w;
-                  }
+                  const int os = 2 * (o + 1) + (tile == unit_lo(o + 1, a) / a.n_kb ? 0 : 1);
+                  const float4* src =
+                      part + size_t(os) * slot_len + h * half_len + size_t(cc / 4) * kBM + row;
+                  x[2] = __ldcg(src);
+                  x[3] = __ldcg(src + kBM);
+                }
+                if (l0) {
+                  add4(acc, 0, x[0]);
+                  add4(acc, 4, x[1]);
                 } else {
 #pragma unroll
-                  for (int jj = 0; jj < 32; ++jj) acc[jj] += v[jj];
+                  for (int jj = 0; jj < 8; ++jj) acc[jj] += v[jj];
+                }
+                if (o + 1 <= c_last) {
+                  if (l1) {
+                    add4(acc, 0, x[2]);
+                    add4(acc, 4, x[3]);
+                  } else {
+#pragma unroll
+                    for (int jj = 0; jj < 8; ++jj) acc[jj] += v[jj];
+                  }
                 }
               }
+              epilogue8<EPI>(a, (a.nh * wt + h) * kBM + row, q, lane, a.nh * wt + h, tok0 + cc,
+                             acc, trow, tpos, tok0);
             }
-            epilogue_chunk(a, n, q, lane, wt, tok0 + cc, acc, trow, tpos, tok0);
           }
           if (threadIdx.x == 64) a.counters[tile] = 0;  // ready for the next launch
         }
@@ -546,9 +568,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncthreads();
   if (a.csplit > 1) {
-    // cluster reduction: every thread of every CTA of the cluster takes part in both barriers.
-    // Receive layout in each owner's ring: [sender][owned chunk][128 rows][36] fp32 (32 columns
-    // + 4 of padding: conflict-free 16-byte accesses).
+    // cluster reduction, one 128-row half at a time; every thread of every CTA of the cluster
+    // takes part in every barrier. Receive layout in each owner's ring: [sender][owned chunk][128
+    // rows][kRecvPitch] fp32 (32 columns + 4 of padding: conflict-free 16-byte accesses).
     cg::cluster_group cl = cg::this_cluster();
     const int C = a.csplit, tile = c / C, r = c - tile * C;
     const int wt = tile / a.n_ttiles, tt_i = tile - wt * a.n_ttiles;
@@ -561,45 +583,48 @@ __global__ void __launch_bounds__(kThreads, 1)
       trow[et] = a.rows ? a.rows[tok0 + et] : tok0 + et;
       tpos[et] = a.pos ? a.pos[tok0 + et] : 0;
     }
-    cl.sync();  // every ring of the cluster is idle
-    if (warp >= 2 && !flags[0]) {
-      const int q = warp & 3, half = (warp - 2) >> 2, row = q * 32 + lane;
-      tc_fence_after();
-      const uint32_t tq = tmem + (static_cast<uint32_t>(q * 32) << 16);
-      for (int ci = half; ci * 32 < valid; ci += 2) {
-        float v[32];
-        tmem_ld32(tq + ci * 32, v);
-        const int owner = ci % C, lc = ci / C;
-        const uint32_t dst =
-            dsmem_addr(recv + (size_t(r * cpo + lc) * kBM + row) * 36, uint32_t(owner));
+    const bool epi = warp >= 2 && !flags[0];
+    const int q = warp & 3, half = (warp - 2) >> 2, row = q * 32 + lane;
+    for (int h = 0; h < a.nh; ++h) {
+      cl.sync();  // every ring of the cluster is idle (h = 0) / its previous half consumed (h = 1)
+      if (epi) {
+        tc_fence_after();
+        const uint32_t tq = tmem + h * a.hoff + (static_cast<uint32_t>(q * 32) << 16);
+#pragma unroll 1
+        for (int ci = half; ci * 32 < valid; ci += 2) {
+          float v[32];
+          tmem_ld32(tq + ci * 32, v);
+          const int owner = ci % C, lc = ci / C;
+          const uint32_t dst = dsmem_addr(
+              recv + (size_t(r * cpo + lc) * kBM + row) * kRecvPitch, uint32_t(owner));
 #pragma unroll
-        for (int g = 0; g < 8; ++g)
-          st_dsmem_v4(dst + g * 16, make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]));
-      }
-    }
-    cl.sync();  // all pushes have landed
-    if (warp >= 2 && !flags[0]) {
-      const int q = warp & 3, half = (warp - 2) >> 2, row = q * 32 + lane;
-      const int n = wt * kBM + row;
-      for (int lc = half; lc < cpo; lc += 2) {
-        const int ci = r + lc * C;
-        if (ci * 32 >= valid) break;
-        float acc[32];
-#pragma unroll
-        for (int jj = 0; jj < 32; ++jj) acc[jj] = 0.0f;
-        for (int sdr = 0; sdr < C; ++sdr) {
-          const float4* src =
-              reinterpret_cast<const float4*>(recv + (size_t(sdr * cpo + lc) * kBM + row) * 36);
-#pragma unroll
-          for (int g = 0; g < 8; ++g) {
-            const float4 x = src[g];
-            acc[4 * g] += x.x;
-            acc[4 * g + 1] += x.y;
-            acc[4 * g + 2] += x.z;
-            acc[4 * g + 3] += x.w;
-          }
+          for (int g = 0; g < 8; ++g)
+            st_dsmem_v4(dst + g * 16,
+                        make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]));
         }
-        epilogue_chunk(a, n, q, lane, wt, tok0 + ci * 32, acc, trow, tpos, tok0);
+      }
+      cl.sync();  // all pushes of this half have landed
+      if (epi) {
+        const int n = (a.nh * wt + h) * kBM + row;
+        // owned chunk lc covers columns (r + lc C) 32 .. +31; 8-column groups alternate between
+        // the two warps of a lane quarter
+#pragma unroll 1
+        for (int gi = half; gi < 4 * cpo; gi += 2) {
+          const int lc = gi >> 2, g8 = (gi & 3) * 8;
+          const int col = (r + lc * C) * 32 + g8;
+          if (col >= valid) continue;
+          float acc[8];
+#pragma unroll
+          for (int jj = 0; jj < 8; ++jj) acc[jj] = 0.0f;
+#pragma unroll 1
+          for (int sdr = 0; sdr < C; ++sdr) {
+            const float4* src = reinterpret_cast<const float4*>(
+                recv + (size_t(sdr * cpo + lc) * kBM + row) * kRecvPitch + g8);
+            add4(acc, 0, src[0]);
+            add4(acc, 4, src[1]);
+          }
+          epilogue8<EPI>(a, n, q, lane, a.nh * wt + h, tok0 + col, acc, trow, tpos, tok0);
+        }
       }
     }
   }
@@ -660,55 +685,141 @@ int make_weight_map(CUtensorMap* map, const void* w, int n_out, int k) {
   return make_map(map, w, k, n_out, kBM);
 }
 
+namespace {
+
+using KernelFn = void (*)(CUtensorMap, CUtensorMap, KArgs);
+
+KernelFn kernel_for(int epi) {
+  switch (epi) {
+    case EPI_F32: return gemm_sk_kernel<EPI_F32>;
+    case EPI_BF16: return gemm_sk_kernel<EPI_BF16>;
+    case EPI_BIAS_BF16: return gemm_sk_kernel<EPI_BIAS_BF16>;
+    case EPI_BIAS_GELU_BF16: return gemm_sk_kernel<EPI_BIAS_GELU_BF16>;
+    case EPI_ADD_F32: return gemm_sk_kernel<EPI_ADD_F32>;
+    case EPI_ROPE_BF16: return gemm_sk_kernel<EPI_ROPE_BF16>;
+    case EPI_SWIGLU_BF16: return gemm_sk_kernel<EPI_SWIGLU_BF16>;
+    default: return nullptr;
+  }
+}
+
+// Sets the shared-memory limit of every instance once; returns the first error.
+cudaError_t set_kernel_attributes() {
+  static std::once_flag once;
+  static cudaError_t err = cudaSuccess;
+  std::call_once(once, [] {
+    for (int e : {int(EPI_F32), int(EPI_BF16), int(EPI_BIAS_BF16), int(EPI_BIAS_GELU_BF16),
+                  int(EPI_ADD_F32), int(EPI_ROPE_BF16), int(EPI_SWIGLU_BF16)}) {
+      const cudaError_t r =
+          cudaFuncSetAttribute(reinterpret_cast<const void*>(kernel_for(e)),
+                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               kSmemPipe + 1024 + 256 + 16384);
+      if (r != cudaSuccess && err == cudaSuccess) err = r;
+    }
+  });
+  return err;
+}
+
+// Clusters of C CTAs (at the largest shared-memory size) that the GPU holds at once. Not every
+// GPC holds the same number of them, so 152 SMs need not hold 152 / C clusters.
+int max_active_clusters(int C) {
+  static int cache[9] = {0};
+  static std::once_flag once;
+  std::call_once(once, [] {
+    for (int cs = 2; cs <= 8; cs *= 2) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(cs);
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = kSmemPipe + 1024 + 256 + 2048;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = cs;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kernel_for(EPI_F32)),
+                                         &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+      }
+      cache[cs] = n;
+    }
+  });
+  return cache[C];
+}
+
+}  // namespace
+
 int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   if (p.n_tok <= 0 || p.n_out <= 0) return SPD_OK;
   if (p.k <= 0) return fail(SPD_EINVAL, "GEMM K must be positive");
-  CUtensorMap map_w, map_x;
-  if (p.map_w) {
-    map_w = *p.map_w;
-  } else if (int rc = make_map(&map_w, p.w, p.k, p.n_out, kBM)) {
-    return rc;
-  }
+  const KernelFn kern = kernel_for(p.epi);
+  if (!kern) return fail(SPD_EINVAL, "unknown GEMM epilogue %d", p.epi);
+  if (!p.map_w && !p.w) return fail(SPD_EINVAL, "GEMM without weights");
+  if (cudaError_t e = set_kernel_attributes())
+    return fail(SPD_ECUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(e));
   KArgs a{};
   a.n_out = p.n_out;
   a.n_tok = p.n_tok;
   a.k = p.k;
   a.n_ttiles = (p.n_tok + 255) / 256;
   a.tt = ((p.n_tok + a.n_ttiles - 1) / a.n_ttiles + 31) / 32 * 32;
-  if (int rc = make_map(&map_x, p.x, p.k, p.n_tok, a.tt)) return rc;
-  // 128-wide k-blocks when at least two fit in the ring (two 128-byte runs per weight row)
-  a.kbox = (2 * 2 * (kWBytes + a.tt * 128) <= kSmemPipe && p.k > kBK) ? 2 : 1;
+  // 256-row tiles for token tiles of at most 64: their stages are mostly weights, and two MMAs
+  // per token box double the weight bytes per stage (needs the row-major pointer for the map)
+  a.nh = (a.tt <= 64 && p.w) ? 2 : 1;
+  const int tile_rows = a.nh * kBM;
+  const int wbox = a.nh * kHalfW;
+  auto stages_for = [&](int kb) {
+    return std::min(kMaxStages, kSmemPipe / (kb * (wbox + a.tt * 128)));
+  };
+  // 128-wide k-blocks (256 contiguous bytes of every weight row per stage) when two stages fit
+  a.kbox = (p.k > kBK && stages_for(2) >= 2) ? 2 : 1;
   a.n_kb = (p.k + a.kbox * kBK - 1) / (a.kbox * kBK);
-  const int n_wtiles = (p.n_out + kBM - 1) / kBM;
+  a.stages = stages_for(a.kbox);
+  const int stage_bytes = a.kbox * (wbox + a.tt * 128);
+  // TMEM (512 columns): two accumulator buffers of 256 columns unless a 256-row tile is wider than
+  // 128 tokens; the second 128-row half sits 128 or 256 columns after the first
+  a.nbuf = (a.nh * a.tt <= 256) ? 2 : 1;
+  a.hoff = a.tt <= 128 ? 128 : 256;
+  CUtensorMap map_w, map_x;
+  if (a.nh == 1 && p.map_w) {
+    map_w = *p.map_w;
+  } else if (int rc = make_map(&map_w, p.w, p.k, p.n_out, tile_rows)) {
+    return rc;
+  }
+  if (int rc = make_map(&map_x, p.x, p.k, p.n_tok, a.tt)) return rc;
+  const int n_wtiles = (p.n_out + tile_rows - 1) / tile_rows;
   const long long tiles = (long long)n_wtiles * a.n_ttiles;
   if (tiles > s.n_counters) return fail(SPD_EUNSUPPORTED, "GEMM has too many output tiles");
   const long long units = tiles * a.n_kb;
   if (units > 0x3fffffffLL) return fail(SPD_EUNSUPPORTED, "GEMM too large");
   a.units = int(units);
   const int sms = num_sms();
-  const int stage_bytes = a.kbox * (kWBytes + a.tt * 128);
-  a.stages = kSmemPipe / stage_bytes;
-  if (a.stages > kMaxStages) a.stages = kMaxStages;
-  // cluster split-K when the tiles fill at most half the SMs: C CTAs per tile (each >= 1 k-block)
+  // cluster split-K when the tiles fill at most half the SMs: the largest C in {2, 4, 8} with at
+  // least one k-block per CTA whose clusters all fit on the GPU at once
   a.csplit = 1;
   if (tiles * 2 <= sms) {
-    int C = 2;
-    while (C < 8 && tiles * C * 2 <= sms && C * 2 <= a.n_kb) C *= 2;
-    // the ring receives C copies of each CTA's share of 32-column chunks ([128][36] fp32 each)
-    const int chunks = a.tt / 32, cpo = (chunks + C - 1) / C;
-    const size_t recv = size_t(C) * cpo * kBM * 36 * sizeof(float);
-    if (C <= a.n_kb && recv <= size_t(a.stages) * stage_bytes) a.csplit = C;
+    for (int C = 8; C >= 2; C /= 2) {
+      // the ring receives C copies of each CTA's share of 32-column chunks ([128][36] fp32 each)
+      const int chunks = a.tt / 32, cpo = (chunks + C - 1) / C;
+      const size_t recv = size_t(C) * cpo * kBM * kRecvPitch * sizeof(float);
+      if (C <= a.n_kb && tiles * C <= sms && tiles <= max_active_clusters(C) &&
+          recv <= size_t(a.stages) * stage_bytes) {
+        a.csplit = C;
+        break;
+      }
+    }
   }
   // one CTA per SM with at least 2 units each; every CTA owns two partial slots (head, tail)
   long long grid = sms;
   if (grid > (units + 1) / 2) grid = (units + 1) / 2;
-  const size_t per_slot = size_t(a.tt) * kBM;
+  const size_t per_slot = size_t(a.tt) * tile_rows;
   if (size_t(2 * grid) * per_slot > s.partial_floats) grid = s.partial_floats / (2 * per_slot);
   if (grid < 1) grid = 1;
   if (units * (grid + 1) >= (1LL << 31)) return fail(SPD_EUNSUPPORTED, "GEMM too large");
   if (a.csplit > 1) grid = tiles * a.csplit;
   a.grid = int(grid);
-  a.epi = p.epi;
   a.out = p.out;
   a.ldo = p.ldo;
   a.rows = p.rows;
@@ -724,14 +835,6 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.budget = kWaitBudget;
 
   const size_t smem = size_t(a.stages) * stage_bytes + 1024 + 256 + 2048;
-  static std::once_flag attr_once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(attr_once, [] {
-    attr_err = cudaFuncSetAttribute(gemm_sk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    kSmemPipe + 1024 + 256 + 16384);
-  });
-  if (attr_err != cudaSuccess)
-    return fail(SPD_ECUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
   const int slot = trace_begin(stream);
   {
     cudaLaunchConfig_t cfg = {};
@@ -748,7 +851,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    SPD_CUDA_TRY(cudaLaunchKernelEx(&cfg, gemm_sk_kernel, map_w, map_x, a));
+    SPD_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, map_w, map_x, a));
   }
   if (slot >= 0) {
     // algorithmic work: valid output columns only; weights, activations and results move once

@@ -73,8 +73,8 @@ enum Epi : int {
 };
 
 struct GemmProblem {
-  const CUtensorMap* map_w;  // weights [n_out][k] bf16, box 64 x 128
-  const void* w;             // (for map creation when map_w is null)
+  const CUtensorMap* map_w;  // weights [n_out][k] bf16, box 64 x 128 (optional)
+  const void* w;             // the same weights (maps of other box heights are made from it)
   const void* x;             // activations [n_tok][k] bf16
   int n_out, n_tok, k;
   int epi;
