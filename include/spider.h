@@ -237,6 +237,30 @@ int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, int N, int ep
                const uint16_t* bias, const int32_t* rows, void* out, int ldo, void* ws,
                size_t ws_bytes, void* stream);
 
+/* Capacity of the scratch that spd_linear_noalloc keeps inside the library. */
+#define SPD_LINEAR_NOALLOC_SCRATCH_BYTES (8u << 20) /* 8 MiB of device memory */
+#define SPD_LINEAR_NOALLOC_MAX_TILES 4096           /* output tiles: ceil(N / 128) x ceil(M / 256) */
+
+/* spd_linear without a workspace argument. The paper has no counterpart: this is a convenience of
+ * the library, for callers that have no device buffer to lend at the point of the call and must
+ * not allocate one there - e.g. a plain C host without a device memory pool, or a latency-bound
+ * loop where cudaMalloc would stall the device and its memory budget is already handed out.
+ * Same operation, arguments, layouts and results as spd_linear (within the same rounding: the
+ * partial-sum scratch is smaller, so a large problem may be split over fewer CTAs).
+ * Its scratch is one file-scope device array of SPD_LINEAR_NOALLOC_SCRATCH_BYTES in this library,
+ * shared by all callers of a device: calls that may overlap on the GPU (other streams, other host
+ * threads) race on it and must be serialized by the caller. The call allocates and frees nothing:
+ * it clears the scratch's status word and tile counters on `stream`, then launches the GEMM.
+ * The first call on a device (the device current at the call) looks up the scratch's address on
+ * that device (cudaGetSymbolAddress) and caches it; make that first call before any stream capture.
+ * status (dev, may be NULL): int32 receiving this call's device-side status (0 = OK, else an
+ * spd_status, e.g. SPD_ETIMEOUT) once the work completes.
+ * Errors: SPD_EINVAL; SPD_ENOSPC when the output has more than SPD_LINEAR_NOALLOC_MAX_TILES tiles
+ * (detected on the host, nothing is launched); SPD_ECUDA. */
+int spd_linear_noalloc(const uint16_t* X, int M, int K, const uint16_t* W, int N, int epilogue,
+                       const uint16_t* bias, const int32_t* rows, void* out, int ldo, int* status,
+                       void* stream);
+
 #ifdef __cplusplus
 }
 #endif

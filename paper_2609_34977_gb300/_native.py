@@ -23,7 +23,8 @@ EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait"
            "spd_prune_workspace_size", "spd_prune", "spd_gather_rows_bf16", "spd_model_create",
            "spd_model_destroy", "spd_plan_adaptive", "spd_plan_static", "spd_project_workspace_size",
            "spd_project", "spd_scatter_rows", "spd_prefill_workspace_size", "spd_prefill",
-           "spd_linear_workspace_size", "spd_linear", "spd_trace_enable", "spd_trace_read")
+           "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
+           "spd_trace_read")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
 
 
@@ -87,6 +88,7 @@ def lib():
             "spd_prefill": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, sz, vp]),
             "spd_linear_workspace_size": (sz, [i, i]),
             "spd_linear": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, sz, vp]),
+            "spd_linear_noalloc": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, vp]),
             "spd_trace_enable": (i, [i]),
             "spd_trace_read": (i, [i, C.POINTER(ll), C.POINTER(C.c_double), C.POINTER(C.c_double),
                                    C.POINTER(C.c_double)]),
@@ -241,6 +243,13 @@ def spd_linear_workspace_size(M: int, N: int) -> int:
 def spd_linear(X, M, K, W, N, epilogue, out, ldo, ws, bias=None, rows=None, stream=None):
     _check(lib().spd_linear(_p(X), M, K, _p(W), N, epilogue, _p(bias), _p(rows), _p(out), ldo, _p(ws),
                             ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def spd_linear_noalloc(X, M, K, W, N, epilogue, out, ldo, bias=None, rows=None, status=None,
+                       stream=None):
+    """spd_linear with the library's own static scratch instead of a caller workspace."""
+    _check(lib().spd_linear_noalloc(_p(X), M, K, _p(W), N, epilogue, _p(bias), _p(rows), _p(out),
+                                    ldo, _p(status), _stream(stream)))
 
 
 def spd_trace_enable(capacity: int):

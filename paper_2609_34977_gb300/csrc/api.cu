@@ -344,6 +344,74 @@ extern "C" int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, in
   return gemm_run(p, s, st);
 }
 
+// ---- allocation-free variant of spd_linear ---------------------------------------------------
+// Scratch of spd_linear_noalloc: status word, per-tile counters, then partial-sum slots.
+static __device__ __align__(256) uint8_t g_linear_scratch[SPD_LINEAR_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_linear_scratch_mu;
+void* g_linear_scratch_ptr[kMaxDevices] = {};  // per device, set by the first call on it
+
+// Address of g_linear_scratch on the current device, looked up once per device.
+int linear_scratch(void** out) {
+  int dev = 0;
+  SPD_CUDA_TRY(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return fail(SPD_EUNSUPPORTED, "device ordinal %d", dev);
+  std::lock_guard<std::mutex> lock(g_linear_scratch_mu);
+  if (!g_linear_scratch_ptr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_linear_scratch);
+    if (e != cudaSuccess) return fail(SPD_ECUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+    g_linear_scratch_ptr[dev] = p;
+  }
+  *out = g_linear_scratch_ptr[dev];
+  return SPD_OK;
+}
+}  // namespace
+
+extern "C" int spd_linear_noalloc(const uint16_t* X, int M, int K, const uint16_t* W, int N,
+                                  int epilogue, const uint16_t* bias, const int32_t* rows, void* out,
+                                  int ldo, int* status, void* stream) {
+  if (!X || !W || !out || M < 0 || K < 8 || N < 1 || ldo < N)
+    return fail(SPD_EINVAL, "bad linear arguments");
+  if (epilogue < SPD_EPI_F32 || epilogue > SPD_EPI_ADD_F32) return fail(SPD_EINVAL, "bad epilogue");
+  if ((epilogue == SPD_EPI_BIAS_BF16 || epilogue == SPD_EPI_BIAS_GELU_BF16) && !bias)
+    return fail(SPD_EINVAL, "epilogue needs a bias");
+  const long long tiles = (long long)((N + 127) / 128) * ((M + 255) / 256);
+  if (tiles > SPD_LINEAR_NOALLOC_MAX_TILES)
+    return fail(SPD_ENOSPC, "spd_linear_noalloc: %lld output tiles exceed the static scratch (%d)",
+                tiles, SPD_LINEAR_NOALLOC_MAX_TILES);
+  void* base = nullptr;
+  if (int rc = linear_scratch(&base)) return rc;
+  Carve cv(base, SPD_LINEAR_NOALLOC_SCRATCH_BYTES);
+  GemmScratch s;
+  s.status = cv.status();
+  s.n_counters = SPD_LINEAR_NOALLOC_MAX_TILES;
+  s.counters = cv.take<int>(s.n_counters);
+  s.partial = cv.take<float>(0);
+  s.partial_floats = (SPD_LINEAR_NOALLOC_SCRATCH_BYTES - cv.used) / sizeof(float);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // the status word and the counters start at zero (a failed earlier call may have left them set)
+  SPD_CUDA_TRY(cudaMemsetAsync(base, 0, 256, st));
+  SPD_CUDA_TRY(cudaMemsetAsync(s.counters, 0, s.n_counters * sizeof(int), st));
+  GemmProblem p{};
+  p.w = W;
+  p.x = X;
+  p.n_out = N;
+  p.n_tok = M;
+  p.k = K;
+  p.epi = epilogue;
+  p.out = out;
+  p.ldo = ldo;
+  p.rows = rows;
+  p.bias = bias;
+  p.out_cols = N;
+  if (int rc = gemm_run(p, s, st)) return rc;
+  if (status) SPD_CUDA_TRY(cudaMemcpyAsync(status, s.status, sizeof(int), cudaMemcpyDeviceToDevice, st));
+  return SPD_OK;
+}
+
 // ---- projector and sequence assembly --------------------------------------------------------
 extern "C" size_t spd_project_workspace_size(const spd_model* m, int rows) {
   if (!m || rows < 0) return 0;
