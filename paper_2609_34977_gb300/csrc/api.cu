@@ -54,18 +54,6 @@ __global__ void copy_rows_kernel(const uint16_t* __restrict__ src, uint16_t* __r
   for (int c = threadIdx.x; c < cols; c += blockDim.x) d[c] = s[c];
 }
 
-// (cos, sin) of position p times frequency j, evaluated in double and stored as float2.
-__global__ void rope_table_kernel(const double* __restrict__ inv_freq, int half, int n_pos,
-                                  float2* __restrict__ tab) {
-  pdl_launch_dependents();
-  pdl_wait();
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n_pos * half) return;
-  double s, c;
-  sincos(double(i / half) * inv_freq[i % half], &s, &c);
-  tab[i] = make_float2(float(c), float(s));
-}
-
 // Bounded wait on a barrier that nothing arrives on: exercises the timeout path.
 __global__ void bounded_wait_probe_kernel(int* status, long long budget) {
   __shared__ uint64_t bar;
@@ -111,13 +99,13 @@ struct spd_model {
   spd_model_cfg cfg;
   struct Layer {
     uint16_t *attn_norm, *ffn_norm, *wq, *wkv, *wo, *wgu, *wd;
-    CUtensorMap m_q, m_kv, m_o, m_gu, m_d;
+    CUtensorMap m_qkv, m_kv, m_o, m_gu, m_d;
   };
   std::vector<Layer> layers;
   uint16_t *final_norm = nullptr, *lm_head = nullptr;
   uint16_t *pw1 = nullptr, *pb1 = nullptr, *pw2 = nullptr, *pb2 = nullptr;
   CUtensorMap m_lm, m_p1, m_p2;
-  double* inv_freq = nullptr;  // [head_dim / 2] theta^(-2j / head_dim)
+  float2* freq = nullptr;  // [head_dim / 2] theta^(-2j / head_dim) in double, split into fp32 (hi, lo)
   int gu_rows = 0;
   void* pool = nullptr;
 };
@@ -235,7 +223,11 @@ extern "C" int spd_model_create(const spd_model_cfg* c, const spd_model_weights*
     }
     if ((rc = copy_rows(s.w_gate, L.wgu, int(D), gs, gd))) break;
     if ((rc = copy_rows(s.w_up, L.wgu, int(D), us, ud))) break;
-    if ((rc = make_weight_map(&L.m_q, L.wq, int(q_rows), int(D)))) break;
+    if (L.wkv != L.wq + q_rows * D) {  // the pool keeps them adjacent (sizes multiples of 256 B)
+      rc = fail(SPD_EUNSUPPORTED, "Wq and Wk|Wv are not adjacent");
+      break;
+    }
+    if ((rc = make_weight_map(&L.m_qkv, L.wq, int(q_rows + 2 * kv_rows), int(D)))) break;
     if ((rc = make_weight_map(&L.m_kv, L.wkv, int(2 * kv_rows), int(D)))) break;
     if ((rc = make_weight_map(&L.m_o, L.wo, int(D), int(q_rows)))) break;
     if ((rc = make_weight_map(&L.m_gu, L.wgu, gu_rows, int(D)))) break;
@@ -248,10 +240,14 @@ extern "C" int spd_model_create(const spd_model_cfg* c, const spd_model_weights*
   cudaMemcpy(m->final_norm, w->final_norm, D * 2, cudaMemcpyDeviceToDevice);
   cudaMemcpy(m->lm_head, w->lm_head, size_t(c->vocab) * D * 2, cudaMemcpyDeviceToDevice);
   if ((rc = make_weight_map(&m->m_lm, m->lm_head, c->vocab, int(D)))) return fin(rc);
-  m->inv_freq = reinterpret_cast<double*>(take(hd * 8));
-  std::vector<double> inv(hd / 2);
-  for (size_t j = 0; j < hd / 2; ++j) inv[j] = pow(double(c->rope_theta), -2.0 * double(j) / double(hd));
-  cudaMemcpy(m->inv_freq, inv.data(), inv.size() * 8, cudaMemcpyHostToDevice);
+  m->freq = reinterpret_cast<float2*>(take(hd / 2 * sizeof(float2)));
+  std::vector<float2> fr(hd / 2);
+  for (size_t j = 0; j < hd / 2; ++j) {
+    const double f = pow(double(c->rope_theta), -2.0 * double(j) / double(hd));
+    const float hi = float(f);
+    fr[j] = make_float2(hi, float(f - double(hi)));
+  }
+  cudaMemcpy(m->freq, fr.data(), fr.size() * sizeof(float2), cudaMemcpyHostToDevice);
   if (c->d_vis) {
     if (!w->proj_w1 || !w->proj_b1 || !w->proj_w2 || !w->proj_b2)
       return fin(fail(SPD_EINVAL, "null projector weight"));
@@ -466,8 +462,7 @@ extern "C" int spd_scatter_rows(const spd_model* m, const uint16_t* src, int row
 namespace {
 
 struct PrefillBufs {
-  uint16_t *xa, *xq, *q, *kv, *o, *y, *act, *z;
-  float2* rope;
+  uint16_t *xa, *q, *kv, *o, *y, *act, *z;
   int32_t* lists;
   size_t list_ints;
   GemmScratch gs;
@@ -486,14 +481,12 @@ PrefillBufs carve_prefill(const spd_model_cfg& c, int T, int B, Carve& cv) {
   const size_t D = c.d_model, qd = size_t(c.n_heads) * c.head_dim, kvd = size_t(c.n_kv_heads) * c.head_dim;
   b.gs = scratch_from(cv);
   b.xa = cv.take<uint16_t>(size_t(T) * D);
-  b.xq = cv.take<uint16_t>(size_t(T) * D);
   b.q = cv.take<uint16_t>(size_t(T) * qd);
   b.kv = cv.take<uint16_t>(size_t(T) * 2 * kvd);
   b.o = cv.take<uint16_t>(size_t(T) * qd);
   b.y = cv.take<uint16_t>(size_t(T) * D);
   b.act = cv.take<uint16_t>(size_t(T) * c.d_ffn);
   b.z = cv.take<uint16_t>(size_t(B) * D);
-  b.rope = cv.take<float2>(size_t(T) * (c.head_dim / 2));
   b.list_ints = list_ints_for(c.n_layers, T, B);
   b.lists = cv.take<int32_t>(b.list_ints);
   return b;
@@ -586,18 +579,15 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
   SPD_CUDA_TRY(cudaMemcpyAsync(dl, hl.data(), off * sizeof(int32_t), cudaMemcpyHostToDevice, st));
   SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
   if (int rc = bf16_to_f32_run(x, h, size_t(T) * D, st)) return rc;
-  int max_len = 0;
-  for (int b = 0; b < B; ++b) max_len = cu[b + 1] - cu[b] > max_len ? cu[b + 1] - cu[b] : max_len;
-  SPD_CUDA_TRY(launch_pdl(rope_table_kernel, dim3((max_len * (hd / 2) + 255) / 256), dim3(256), 0, st,
-                          static_cast<const double*>(m->inv_freq), hd / 2, max_len, bf.rope));
 
   int rc = SPD_OK;
   for (int l = 0; l < L && !rc; ++l) {
     const spd_model::Layer& W = m->layers[l];
     const LayerLists& q = ll[l];
-    // attention sub-layer: norm of every row (K/V need all tokens) + compact copy of query rows
-    rc = rmsnorm_run(h, T, D, W.attn_norm, c.rms_eps, nullptr, bf.xa, q.na ? dl + q.amap : nullptr,
-                     bf.xq, st);
+    // attention sub-layer: norm of every row (K/V need all tokens); one GEMM gives K, V of every
+    // token and Q of the query tokens (rows of skipped tokens computed but not stored: the
+    // contraction is weight-bound, one pass over Wq|Wk|Wv beats two launches)
+    rc = rmsnorm_run(h, T, D, W.attn_norm, c.rms_eps, nullptr, bf.xa, nullptr, nullptr, st);
     if (rc) break;
     GemmProblem kvp{};
     kvp.map_w = &W.m_kv;
@@ -610,22 +600,27 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
     kvp.out = bf.kv;
     kvp.ldo = 2 * kvd;
     kvp.pos = dl + pos_off;
-    kvp.rope = bf.rope;
+    kvp.rope = m->freq;
     kvp.rope_rows = kvd;
     kvp.head_dim = hd;
-    if ((rc = gemm_run(kvp, bf.gs, st))) break;
     if (q.na > 0) {
       GemmProblem qp = kvp;
-      qp.map_w = &W.m_q;
-      qp.w = W.wq;
-      qp.x = bf.xq;
-      qp.n_out = qd;
-      qp.n_tok = q.na;
+      qp.map_w = &W.m_qkv;
+      qp.w = W.wq;  // Wq rows, then Wk and Wv rows, contiguous
+      qp.n_out = qd + 2 * kvd;
+      qp.epi = EPI_QKV_BF16;
       qp.out = bf.q;
       qp.ldo = qd;
-      qp.pos = dl + q.apos;
-      qp.rope_rows = qd;
+      qp.rows = dl + q.amap;
+      qp.out2 = bf.kv;
+      qp.ldo2 = 2 * kvd;
+      qp.split = qd;
+      qp.n_tok_out = q.na;
       if ((rc = gemm_run(qp, bf.gs, st))) break;
+    } else if ((rc = gemm_run(kvp, bf.gs, st))) {
+      break;
+    }
+    if (q.na > 0) {
       if ((rc = attention_run(bf.q, qd, bf.kv, 2 * kvd, kvd, bf.o, qd,
                               reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
                               c.n_heads, c.n_kv_heads, hd, st, q.ctx, q.na, T)))

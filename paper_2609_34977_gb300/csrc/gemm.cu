@@ -14,6 +14,8 @@
 //    C) with posted distributed-shared-memory stores; after a cluster barrier each owner sums the C
 //    copies in rank order from its own shared memory and runs the fused epilogue; then the second
 //    half. No global partials, no remote loads, deterministic.
+//    Residual (ADD) epilogues split K the same way without a cluster: each CTA adds its partial
+//    into the destination rows with red.add, which the residual update does anyway.
 //  * persistent stream-K otherwise, below.
 //
 // Persistent stream-K: one CTA per SM. The work is the list of (tile, k-block) units in tile-major
@@ -76,16 +78,18 @@ constexpr int kRecvPitch = 36;      // fp32 per row of a received 32-column chun
 
 struct KArgs {
   int n_out, n_tok, k, tt, n_kb, n_ttiles, units, grid, stages, ldo, rope_rows, head_dim,
-      out_cols, kbox, csplit, nbuf, hoff, nh;
+      out_cols, kbox, csplit, cluster, nbuf, hoff, nh, ldo2, split;
   // kbox: 64-wide boxes per stage (1 or 2); a k-block is kbox * 64 wide
-  // csplit: CTAs per output tile in cluster split-K (1 = stream-K)
+  // csplit: CTAs per output tile in split-K (1 = stream-K); cluster: split-K CTAs reduce through
+  // distributed shared memory (0: ADD epilogue, every CTA adds its own partial)
   // nbuf: TMEM accumulator buffers; hoff: TMEM column offset of the second 128-row half
   // nh: 128-row halves per tile (1 or 2)
   void* out;
+  void* out2;
   const int32_t* rows;
   const uint16_t* bias;
   const int32_t* pos;
-  const float2* rope;  // [position][head_dim / 2] (cos, sin)
+  const float2* rope;  // [head_dim / 2] rotary frequency theta^(-2j / head_dim) as fp32 (hi, lo)
   float* partial;
   int* counters;
   int* status;
@@ -164,6 +168,68 @@ __device__ __forceinline__ void seg_get(const SegPlan& p, int j, int& s, int& e)
   e = s + p.n_kb;
 }
 
+// 2 pi = kTwoPiHi + kTwoPiLo; kTwoPiHi = 6.28125 has 8 significant bits, so k kTwoPiHi is exact
+// in fp32 for |k| < 2^16 (two-constant Cody-Waite reduction).
+constexpr float kTwoPiHi = 6.28125f;
+constexpr float kTwoPiLo = 1.9353071795864769e-3f;
+constexpr float kInvTwoPi = 0.15915494309189535f;
+
+// cos and sin of position p times frequency (f.x + f.y). The product is formed exactly (two-product)
+// and reduced to about [-pi, pi] with the split 2 pi above, so the angle is within ~2e-7 of exact
+// for angles below 2^16 x 2 pi; __sincosf then adds at most 2^-21.4.
+__device__ __forceinline__ void rope_cos_sin(int p, float2 f, float& c, float& sn) {
+  const float pf = float(p);  // exact for p < 2^24
+  const float x_hi = pf * f.x;
+  const float x_lo = fmaf(pf, f.x, -x_hi) + pf * f.y;
+  const float k = rintf(x_hi * kInvTwoPi);
+  float r = fmaf(-k, kTwoPiHi, x_hi);  // exact
+  r = fmaf(-k, kTwoPiLo, r) + x_lo;
+  __sincosf(r, &sn, &c);
+}
+
+// Rotary embedding of weight row nn (rows laid out in rotary pairs: lane l < 16 of a 32-row group
+// holds pair element j, lane l + 16 element j + head_dim / 2) for 8 tokens, stored as bf16 to row
+// row_of(t) (skipped when negative), column head * head_dim + rotated index. The angles are
+// computed in registers: a per-position table would cost an L2 round trip per 8 tokens.
+template <typename RowOf>
+__device__ __forceinline__ void rope_store8(const KArgs& a, __nv_bfloat16* o, int ldo, int nn,
+                                            int lane, int t0, const float (&v)[8], const int* tpos,
+                                            int tb, RowOf row_of) {
+  const int nt = a.n_tok;
+  const int hd = a.head_dim, half = hd >> 1;
+  const int head = nn / hd, g = (nn % hd) >> 5;
+  const int jf = 16 * g + (lane & 15);
+  const int col = head * hd + ((lane < 16) ? jf : half + jf);
+  const float2 fr = a.rope[jf];
+  const float sgn = (lane < 16) ? -1.0f : 1.0f;
+  // lanes l and l + 16 rotate by the same angles: each evaluates four tokens' and they trade
+  const int hi = lane >> 4;
+  float cm[4], sm[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int t = min(t0 + 4 * hi + i, nt - 1);
+    rope_cos_sin(tpos[t - tb], fr, cm[i], sm[i]);
+  }
+  float y[8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {  // branch-free math, then the stores
+    const float co = __shfl_xor_sync(0xffffffffu, cm[i], 16);
+    const float so = __shfl_xor_sync(0xffffffffu, sm[i], 16);
+    const float c_lo = hi ? co : cm[i], s_lo = hi ? so : sm[i];  // token i
+    const float c_hi = hi ? cm[i] : co, s_hi = hi ? sm[i] : so;  // token i + 4
+    const float p_lo = __shfl_xor_sync(0xffffffffu, v[i], 16);
+    const float p_hi = __shfl_xor_sync(0xffffffffu, v[i + 4], 16);
+    y[i] = fmaf(sgn * p_lo, s_lo, v[i] * c_lo);
+    y[i + 4] = fmaf(sgn * p_hi, s_hi, v[i + 4] * c_hi);
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int t = t0 + j;
+    const int r = (t < nt) ? row_of(t) : -1;
+    if (r >= 0) o[size_t(r) * ldo + col] = __float2bfloat16_rn(y[j]);
+  }
+}
+
 // Applies epilogue EPI to 8 consecutive tokens t0..t0+7 of weight row n (TMEM lane quarter q;
 // w_tile = the 128-row block n / 128). trow / tpos: output row and rotary position of each token
 // of the token tile (shared memory, indexed from the tile's first token tb). Warp-uniform calls.
@@ -201,25 +267,7 @@ __device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane
   } else if constexpr (EPI == EPI_ROPE_BF16) {
     __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out);
     if (n < a.rope_rows) {  // warp-uniform: rope_rows is a multiple of 32
-      const int hd = a.head_dim, half = hd >> 1;
-      const int head = n / hd, g = (n % hd) >> 5;
-      const int jf = 16 * g + (lane & 15);
-      const int col = head * hd + ((lane < 16) ? jf : half + jf);
-      float2 cs[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {  // the table loads first, all in flight together
-        const int t = min(t0 + j, nt - 1);
-        cs[j] = a.rope[size_t(tpos[t - tb]) * half + jf];
-      }
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float p = __shfl_xor_sync(0xffffffffu, v[j], 16);
-        const int t = t0 + j;
-        if (t < nt) {
-          const float y = (lane < 16) ? v[j] * cs[j].x - p * cs[j].y : v[j] * cs[j].x + p * cs[j].y;
-          o[size_t(trow[t - tb]) * a.ldo + col] = __float2bfloat16_rn(y);
-        }
-      }
+      rope_store8(a, o, a.ldo, n, lane, t0, v, tpos, tb, [&](int t) { return trow[t - tb]; });
     } else if (n < a.n_out) {
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -227,17 +275,44 @@ __device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane
         if (t < nt) o[size_t(trow[t - tb]) * a.ldo + n] = __float2bfloat16_rn(v[j]);
       }
     }
+  } else if constexpr (EPI == EPI_QKV_BF16) {
+    if (n < a.split) {  // query rows (warp-uniform: split is a multiple of 128)
+      rope_store8(a, static_cast<__nv_bfloat16*>(a.out), a.ldo, n, lane, t0, v, tpos, tb,
+                  [&](int t) { return trow[t - tb]; });
+    } else {
+      __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out2);
+      const int nn = n - a.split;
+      if (nn < a.rope_rows) {
+        rope_store8(a, o, a.ldo2, nn, lane, t0, v, tpos, tb, [](int t) { return t; });
+      } else if (n < a.n_out) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int t = t0 + j;
+          if (t < nt) o[size_t(t) * a.ldo2 + nn] = __float2bfloat16_rn(v[j]);
+        }
+      }
+    }
   } else if constexpr (EPI == EPI_SWIGLU_BF16) {
+    // lanes l and l + 16 hold gate and up of the same FFN channel f: after one exchange lane l
+    // finishes the even tokens of the group and lane l + 16 the odd ones
     __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out);
     const int f = w_tile * 64 + q * 16 + (lane & 15);
+    const int odd = lane >> 4;
+    float y[4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float u = __shfl_xor_sync(0xffffffffu, v[j], 16);
-      const int t = t0 + j;
-      if (lane < 16 && t < nt && f < a.out_cols) {
-        const float g = v[j];
-        // SiLU(g) u; __fdividef gives 0 once 1 + e^-g passes 2^126, the limit of g / (1 + e^-g)
-        o[size_t(trow[t - tb]) * a.ldo + f] = __float2bfloat16_rn(__fdividef(g, 1.0f + __expf(-g)) * u);
+    for (int i = 0; i < 4; ++i) {
+      // lane < 16 sends v[2i + 1] (its gate of the odd token) and receives the up of the even one
+      const float e0 = v[2 * i], e1 = v[2 * i + 1];
+      const float mine = odd ? e1 : e0, other = odd ? e0 : e1;
+      const float recv = __shfl_xor_sync(0xffffffffu, other, 16);
+      const float g = odd ? recv : mine, u = odd ? mine : recv;
+      y[i] = __fdividef(g, 1.0f + __expf(-g)) * u;  // SiLU(g) u; 0 once 1 + e^-g passes 2^126
+    }
+    if (f < a.out_cols) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int t = t0 + 2 * i + odd;
+        if (t < nt) o[size_t(trow[t - tb]) * a.ldo + f] = __float2bfloat16_rn(y[i]);
       }
     }
   }
@@ -267,6 +342,7 @@ __device__ __forceinline__ void add4(float (&acc)[8], int o, const float4& x) {
   acc[o + 3] += x.w;
 }
 
+// 10 warps: three share an SM sub-partition's 16K registers, so at most 168 registers a thread.
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_sk_kernel(const __grid_constant__ CUtensorMap map_w,
@@ -291,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x;
   int u0, u1;
-  if (a.csplit > 1) {  // cluster split-K: rank r of tile c / C owns k-blocks [r n_kb / C, (r+1) n_kb / C)
+  if (a.csplit > 1) {  // split-K: rank r of tile c / C owns k-blocks [r n_kb / C, (r+1) n_kb / C)
     const int tile = c / a.csplit, r = c - tile * a.csplit;
     u0 = tile * a.n_kb + r * a.n_kb / a.csplit;
     u1 = tile * a.n_kb + (r + 1) * a.n_kb / a.csplit;
@@ -460,7 +536,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after();
-      if (a.csplit > 1) break;  // cluster split-K: the accumulator is pushed after the role loops
+      if (a.cluster) break;  // cluster split-K: the accumulator is pushed after the role loops
       const int wt = tile / a.n_ttiles, tt_i = tile - wt * a.n_ttiles;
       const int tok0 = tt_i * a.tt;
       const int valid = min(a.tt, a.n_tok - tok0);
@@ -511,6 +587,93 @@ __global__ void __launch_bounds__(kThreads, 1)
           __threadfence();
           const int c_first = cta_of_unit(tile * a.n_kb, a);
           const int c_last = cta_of_unit((tile + 1) * a.n_kb - 1, a);
+          if (c_last - c_first == 1) {
+            // one other contributor (the usual case): its partial for eight 8-column groups in
+            // flight at a time; a + b is exact in either order, so this matches the loop below
+            const int o = (c == c_first) ? c_last : c_first;
+            const int os = 2 * o + (tile == unit_lo(o, a) / a.n_kb ? 0 : 1);
+            for (int h = 0; h < a.nh; ++h) {
+              const float4* src = part + size_t(os) * slot_len + h * half_len + row;
+#pragma unroll 1
+              for (int cc0 = half * 8; cc0 < valid; cc0 += 128) {
+                float4 x[16];
+#pragma unroll
+                for (int g = 0; g < 8; ++g) {
+                  const int cc = cc0 + 16 * g;
+                  if (cc < valid) {
+                    x[2 * g] = __ldcg(src + size_t(cc / 4) * kBM);
+                    x[2 * g + 1] = __ldcg(src + size_t(cc / 4 + 1) * kBM);
+                  }
+                }
+#pragma unroll 1
+                for (int g = 0; g < 8; ++g) {
+                  const int cc = cc0 + 16 * g;
+                  if (cc < valid) {
+                    float v[8];
+                    tmem_ld8(tq + h * a.hoff + cc, v);
+                    add4(v, 0, x[0]);
+                    add4(v, 4, x[1]);
+                    epilogue8<EPI>(a, (a.nh * wt + h) * kBM + row, q, lane, a.nh * wt + h,
+                                   tok0 + cc, v, trow, tpos, tok0);
+                  }
+                  // next group's data into the fixed slots (static register indices)
+#pragma unroll
+                  for (int k = 0; k < 14; ++k) x[k] = x[k + 2];
+                }
+              }
+            }
+          } else if (c_last - c_first == 2) {
+            // two other contributors: two groups in flight, summed in CTA order
+            // ((first + second) + third, this CTA's own partial in its place), as below
+            const int own = c - c_first;
+            const int oa = (own == 0) ? c_first + 1 : c_first;  // first other contributor
+            const int ob = (own == 2) ? c_first + 1 : c_last;   // second
+            const int sa = 2 * oa + (tile == unit_lo(oa, a) / a.n_kb ? 0 : 1);
+            const int sb = 2 * ob + (tile == unit_lo(ob, a) / a.n_kb ? 0 : 1);
+            for (int h = 0; h < a.nh; ++h) {
+              const float4* pa = part + size_t(sa) * slot_len + h * half_len + row;
+              const float4* pb = part + size_t(sb) * slot_len + h * half_len + row;
+#pragma unroll 1
+              for (int cc0 = half * 8; cc0 < valid; cc0 += 32) {
+                float4 xa[4], xb[4];
+#pragma unroll
+                for (int g = 0; g < 2; ++g) {
+                  const int cc = cc0 + 16 * g;
+                  if (cc < valid) {
+                    xa[2 * g] = __ldcg(pa + size_t(cc / 4) * kBM);
+                    xa[2 * g + 1] = __ldcg(pa + size_t(cc / 4 + 1) * kBM);
+                    xb[2 * g] = __ldcg(pb + size_t(cc / 4) * kBM);
+                    xb[2 * g + 1] = __ldcg(pb + size_t(cc / 4 + 1) * kBM);
+                  }
+                }
+#pragma unroll 1
+                for (int g = 0; g < 2; ++g) {
+                  const int cc = cc0 + 16 * g;
+                  if (cc < valid) {
+                    float v[8];
+                    tmem_ld8(tq + h * a.hoff + cc, v);
+                    const float x1[8] = {xa[0].x, xa[0].y, xa[0].z, xa[0].w,
+                                         xa[1].x, xa[1].y, xa[1].z, xa[1].w};
+                    const float x2[8] = {xb[0].x, xb[0].y, xb[0].z, xb[0].w,
+                                         xb[1].x, xb[1].y, xb[1].z, xb[1].w};
+                    float acc[8];
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                      if (own == 0) acc[k] = (v[k] + x1[k]) + x2[k];
+                      else if (own == 1) acc[k] = (x1[k] + v[k]) + x2[k];
+                      else acc[k] = (x1[k] + x2[k]) + v[k];
+                    }
+                    epilogue8<EPI>(a, (a.nh * wt + h) * kBM + row, q, lane, a.nh * wt + h,
+                                   tok0 + cc, acc, trow, tpos, tok0);
+                  }
+                  xa[0] = xa[2];
+                  xa[1] = xa[3];
+                  xb[0] = xb[2];
+                  xb[1] = xb[3];
+                }
+              }
+            }
+          } else {
           for (int h = 0; h < a.nh; ++h) {
 #pragma unroll 1
             for (int cc = half * 8; cc < valid; cc += 16) {
@@ -558,6 +721,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                              acc, trow, tpos, tok0);
             }
           }
+          }
           if (threadIdx.x == 64) a.counters[tile] = 0;  // ready for the next launch
         }
       }
@@ -567,7 +731,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   __syncthreads();
-  if (a.csplit > 1) {
+  if (a.cluster) {
     // cluster reduction, one 128-row half at a time; every thread of every CTA of the cluster
     // takes part in every barrier. Receive layout in each owner's ring: [sender][owned chunk][128
     // rows][kRecvPitch] fp32 (32 columns + 4 of padding: conflict-free 16-byte accesses).
@@ -698,6 +862,7 @@ KernelFn kernel_for(int epi) {
     case EPI_ADD_F32: return gemm_sk_kernel<EPI_ADD_F32>;
     case EPI_ROPE_BF16: return gemm_sk_kernel<EPI_ROPE_BF16>;
     case EPI_SWIGLU_BF16: return gemm_sk_kernel<EPI_SWIGLU_BF16>;
+    case EPI_QKV_BF16: return gemm_sk_kernel<EPI_QKV_BF16>;
     default: return nullptr;
   }
 }
@@ -708,7 +873,8 @@ cudaError_t set_kernel_attributes() {
   static cudaError_t err = cudaSuccess;
   std::call_once(once, [] {
     for (int e : {int(EPI_F32), int(EPI_BF16), int(EPI_BIAS_BF16), int(EPI_BIAS_GELU_BF16),
-                  int(EPI_ADD_F32), int(EPI_ROPE_BF16), int(EPI_SWIGLU_BF16)}) {
+                  int(EPI_ADD_F32), int(EPI_ROPE_BF16), int(EPI_SWIGLU_BF16),
+                  int(EPI_QKV_BF16)}) {
       const cudaError_t r =
           cudaFuncSetAttribute(reinterpret_cast<const void*>(kernel_for(e)),
                                cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -796,10 +962,16 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   if (units > 0x3fffffffLL) return fail(SPD_EUNSUPPORTED, "GEMM too large");
   a.units = int(units);
   const int sms = num_sms();
-  // cluster split-K when the tiles fill at most half the SMs: the largest C in {2, 4, 8} with at
-  // least one k-block per CTA whose clusters all fit on the GPU at once
+  // split-K when the tiles fill at most half the SMs. ADD epilogues: the most CTAs per tile (a
+  // power of two, at least two k-blocks each) that still fit one per SM. Others: the largest C in
+  // {2, 4, 8} with at least one k-block per CTA whose clusters all fit on the GPU at once.
   a.csplit = 1;
-  if (tiles * 2 <= sms) {
+  a.cluster = 0;
+  if (tiles * 2 <= sms && p.epi == EPI_ADD_F32) {
+    int C = 2;
+    while (tiles * C * 2 <= sms && C * 4 <= a.n_kb) C *= 2;
+    if (C * 2 <= a.n_kb) a.csplit = C;
+  } else if (tiles * 2 <= sms) {
     for (int C = 8; C >= 2; C /= 2) {
       // the ring receives C copies of each CTA's share of 32-column chunks ([128][36] fp32 each)
       const int chunks = a.tt / 32, cpo = (chunks + C - 1) / C;
@@ -807,6 +979,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
       if (C <= a.n_kb && tiles * C <= sms && tiles <= max_active_clusters(C) &&
           recv <= size_t(a.stages) * stage_bytes) {
         a.csplit = C;
+        a.cluster = 1;
         break;
       }
     }
@@ -818,10 +991,20 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   if (size_t(2 * grid) * per_slot > s.partial_floats) grid = s.partial_floats / (2 * per_slot);
   if (grid < 1) grid = 1;
   if (units * (grid + 1) >= (1LL << 31)) return fail(SPD_EUNSUPPORTED, "GEMM too large");
-  if (a.csplit > 1) grid = tiles * a.csplit;
+  if (a.csplit > 1) {
+    grid = tiles * a.csplit;
+  } else if (tiles <= sms && tiles * 2 > sms && a.tt >= 128) {
+    // between half and all of the SMs' worth of wide tiles: one whole tile per CTA. Stream-K's
+    // balance would split most tiles two or three ways, and the fixups of wide token tiles cost
+    // more than the idle SMs do.
+    grid = tiles;
+  }
   a.grid = int(grid);
   a.out = p.out;
   a.ldo = p.ldo;
+  a.out2 = p.out2;
+  a.ldo2 = p.ldo2;
+  a.split = p.split;
   a.rows = p.rows;
   a.bias = p.bias;
   a.pos = p.pos;
@@ -846,7 +1029,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = a.csplit;
+    attr[1].val.clusterDim.x = a.cluster ? a.csplit : 1;
     attr[1].val.clusterDim.y = 1;
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
@@ -855,11 +1038,17 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   }
   if (slot >= 0) {
     // algorithmic work: valid output columns only; weights, activations and results move once
+    // (fused QKV: query rows count for the query tokens only)
     const double cols = (p.epi == EPI_SWIGLU_BF16) ? 2.0 * p.out_cols : double(p.n_out);
     const double out_cols = (p.epi == EPI_SWIGLU_BF16) ? double(p.out_cols) : double(p.n_out);
     const double ob = (p.epi == EPI_F32) ? 4.0 : (p.epi == EPI_ADD_F32) ? 8.0 : 2.0;
-    trace_end(slot, stream, TR_GEMM, 2.0 * p.n_tok * cols * p.k,
-              2.0 * cols * p.k + 2.0 * p.n_tok * p.k + ob * p.n_tok * out_cols);
+    double tok_cols = double(p.n_tok) * cols, tok_out = double(p.n_tok) * out_cols;
+    if (p.epi == EPI_QKV_BF16) {
+      tok_cols = double(p.n_tok_out) * p.split + double(p.n_tok) * (p.n_out - p.split);
+      tok_out = tok_cols;
+    }
+    trace_end(slot, stream, TR_GEMM, 2.0 * tok_cols * p.k,
+              2.0 * cols * p.k + 2.0 * p.n_tok * p.k + ob * tok_out);
   }
   return SPD_OK;
 }

@@ -69,7 +69,9 @@ enum Epi : int {
   EPI_BIAS_GELU_BF16 = SPD_EPI_BIAS_GELU_BF16,
   EPI_ADD_F32 = SPD_EPI_ADD_F32,
   EPI_ROPE_BF16 = 16,  // rotary embedding on weight rows [0, rope_rows) laid out in rotary pairs
-  EPI_SWIGLU_BF16 = 17 // SiLU(gate) * up from weight rows interleaved in gate/up half-warps
+  EPI_SWIGLU_BF16 = 17, // SiLU(gate) * up from weight rows interleaved in gate/up half-warps
+  EPI_QKV_BF16 = 18     // rows [0, split): rotary, to out at row rows[t] (skipped when < 0);
+                        // rows [split, n_out): to out2 at row t, rotary on the first rope_rows
 };
 
 struct GemmProblem {
@@ -83,9 +85,12 @@ struct GemmProblem {
   const int32_t* rows;       // output row of token t (null = t)
   const uint16_t* bias;      // [n_out] bf16
   const int32_t* pos;        // rotary position of token t
-  const void* rope;          // float2 [position][head_dim / 2]: (cos, sin) of position * freq_j
+  const void* rope;          // float2 [head_dim / 2]: freq_j = theta^(-2j / head_dim) as (hi, lo)
   int rope_rows, head_dim;
   int out_cols;              // valid output columns (SwiGLU: d_ffn)
+  void* out2;                // EPI_QKV_BF16: second output, row stride ldo2, from weight row split
+  int ldo2, split;
+  int n_tok_out;             // EPI_QKV_BF16: tokens whose first-output rows are stored (tracing)
 };
 
 // Scratch of stream-K partial slots (fp32, two per CTA) and per-tile arrival counters. The counters
