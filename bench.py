@@ -61,7 +61,7 @@ def gemm_traffic():
     """DRAM bytes per GEMM launch from the committed ncu summary, if the GEMM source is unchanged."""
     import hashlib
     try:
-        txt = open(os.path.join(ROOT, "profiles", "gemm_sk_llava15_layer.md")).read()
+        txt = open(os.path.join(ROOT, "profiles", "gemm_llava15_layer.md")).read()
         kv = dict(l.split(": ", 1) for l in txt.splitlines() if l.startswith(("traffic_bytes", "source_sha")))
         src = os.path.join(ROOT, "paper_2609_34977_gb300", "csrc", "gemm.cu")
         if hashlib.sha256(open(src, "rb").read()).hexdigest() == kv["source_sha256"].strip():
