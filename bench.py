@@ -303,7 +303,7 @@ def main():
     else:
         roof = {"bound": "tensor", "achieved": tfs, "peak": tf_sust, "unit": "TFLOP/s",
                 "frac": tfs / tf_sust}
-    roof.update({"traffic": gemm_traffic(), "traffic_unit": "bytes per launch (ncu, profiles/)", "kernel": "gemm_tc_kernel (tcgen05, all decoder/projector/LM-head GEMMs)",
+    roof.update({"traffic": gemm_traffic(), "traffic_unit": "bytes per launch (ncu, profiles/)", "kernel": "gemm_sk_kernel (tcgen05, all decoder/projector/LM-head GEMMs)",
                  "peak_source": f"{src} (MEASURED_PEAKS.json)", "launches_per_step": g["launches"] / a.steps,
                  "avg_launch_us": 1000.0 * g["ms"] / max(g["launches"], 1),
                  "arith_intensity_flop_per_byte": ai, "tensor_tflops": tfs,
