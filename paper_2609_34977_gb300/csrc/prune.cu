@@ -3,8 +3,10 @@
 //   rowstats     a_v = head-mean of the attention (Sec. 4.1.1); 1/||F_l,i|| for every tapped layer
 //   anchors      top-N_anc of a_v by a bitonic sort of (a_v desc, index asc) keys (Eq. 1);
 //                stable lists of anchor and non-anchor tokens by block prefix sums
-//   anchor_sim   a_i = max_p cos(F^L_i, F^L_p) over anchors: a 64 x 64 register-tiled fp32 product,
-//                max via atomicMax on order-preserving integer keys (exact, order independent)
+//   anchor_sim   a_i = max_p cos(F^L_i, F^L_p) over anchors: 64 x 64 register-tiled fp32 products,
+//                the feature dimension split over a cluster of 4 CTAs whose partial tiles are summed
+//                in rank order through distributed shared memory; max via atomicMax on
+//                order-preserving integer keys (exact, order independent)
 //   kmeans       one thread-block cluster of 8 CTAs per tile, each owning a contiguous slice of the
 //                non-anchor tokens: Lloyd on raw F^L (assignment in each CTA, per-CTA sums in token
 //                order, cross-CTA sums in rank order through distributed shared memory), then the
@@ -185,36 +187,66 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
 }
 
 // ---- 3. a_i = max over anchors of cos(F^L_i, F^L_p) -------------------------------------------
-// CTA tile: 64 non-anchor tokens x 64 anchors, d in chunks of 32 through shared memory (stored
-// transposed), 4 x 4 dot products per thread.
-__global__ void __launch_bounds__(256) anchor_sim_kernel(PruneDims p, PruneWs w) {
+// A cluster of kAS CTAs per 64 non-anchor tokens x 64 anchors tile, each CTA one slice of the
+// feature dimension: 32-wide chunks through shared memory (stored transposed; the next chunk is
+// fetched into registers while the current one is multiplied), 4 x 4 dot products per thread.
+// The partial tiles are summed in rank order through distributed shared memory, each CTA
+// finishing 16 rows.
+constexpr int kAS = 4;
+
+__global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
+    anchor_sim_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
   __shared__ float Us[32][68], As[32][68];
+  __shared__ float P[64][65];  // this CTA's partial dot products
+  cg::cluster_group cl = cg::this_cluster();
+  const int rank = int(cl.block_rank());
   const int t = blockIdx.z, tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  const int u0 = blockIdx.x * 64, p0 = blockIdx.y * 64;
+  const int u0 = (blockIdx.x / kAS) * 64, p0 = blockIdx.y * 64;
   const int* ul = w.ulist + size_t(t) * p.m;
   const int* al = w.alist + size_t(t) * p.n_anc;
+  // staging: thread loads column dd of rows r0 + 8 i (i < 8) of both operands
+  const int dd = threadIdx.x & 31, r0 = threadIdx.x >> 5;
+  const float* urow[8];
+  const float* arow[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int r = r0 + 8 * i;
+    urow[i] = (u0 + r < p.m) ? feat_row(p, p.fin, t, ul[u0 + r]) : nullptr;
+    arow[i] = (p0 + r < p.n_anc) ? feat_row(p, p.fin, t, al[p0 + r]) : nullptr;
+  }
+  const int nch = (p.d + 31) / 32, c0 = rank * nch / kAS, c1 = (rank + 1) * nch / kAS;
+  float ru[8], ra[8];
+  auto fetch = [&](int ch) {
+    const int dcol = ch * 32 + dd;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      ru[i] = (urow[i] && dcol < p.d) ? urow[i][dcol] : 0.0f;
+      ra[i] = (arow[i] && dcol < p.d) ? arow[i][dcol] : 0.0f;
+    }
+  };
   float acc[4][4];
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
     for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
-  for (int d0 = 0; d0 < p.d; d0 += 32) {
-    for (int e = threadIdx.x; e < 64 * 32; e += 256) {
-      const int r = e >> 5, dd = e & 31;
-      const bool dc = d0 + dd < p.d;
-      Us[dd][r] = (u0 + r < p.m && dc) ? feat_row(p, p.fin, t, ul[u0 + r])[d0 + dd] : 0.0f;
-      As[dd][r] = (p0 + r < p.n_anc && dc) ? feat_row(p, p.fin, t, al[p0 + r])[d0 + dd] : 0.0f;
+  if (c0 < c1) fetch(c0);
+  for (int ch = c0; ch < c1; ++ch) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      Us[dd][r0 + 8 * i] = ru[i];
+      As[dd][r0 + 8 * i] = ra[i];
     }
     __syncthreads();
+    if (ch + 1 < c1) fetch(ch + 1);  // in flight during the products below
 #pragma unroll 8
-    for (int dd = 0; dd < 32; ++dd) {
+    for (int e = 0; e < 32; ++e) {
       float a[4], b[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = Us[dd][ty + 16 * i];
+      for (int i = 0; i < 4; ++i) a[i] = Us[e][ty + 16 * i];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) b[j] = As[dd][tx + 16 * j];
+      for (int j = 0; j < 4; ++j) b[j] = As[e][tx + 16 * j];
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -222,23 +254,38 @@ __global__ void __launch_bounds__(256) anchor_sim_kernel(PruneDims p, PruneWs w)
     }
     __syncthreads();
   }
-  const float* inv = w.inv + size_t(p.fin) * p.n_tiles * p.n + size_t(t) * p.n;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int ur = u0 + ty + 16 * i;
-    float best = -INFINITY;
-    if (ur < p.m) {
-      const float iu = inv[ul[ur]];
+  for (int i = 0; i < 4; ++i)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int pa = p0 + tx + 16 * j;
-        if (pa < p.n_anc) best = fmaxf(best, acc[i][j] * iu * inv[al[pa]]);
-      }
-    }
+    for (int j = 0; j < 4; ++j) P[ty + 16 * i][tx + 16 * j] = acc[i][j];
+  cl.sync();
+  // rows 16 rank .. 16 rank + 15 of the tile: all kAS partials loaded first, summed in rank order
+  const int lr = 16 * rank + ty;
+  float x[kAS][4];
 #pragma unroll
-    for (int off = 8; off; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
-    if (tx == 0 && ur < p.m) atomicMax(&w.asim[size_t(t) * p.n + ul[ur]], ordered_key(best));
+  for (int src = 0; src < kAS; ++src) {
+    const float* pp = cl.map_shared_rank(&P[0][0], src) + lr * 65;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) x[src][j] = pp[tx + 16 * j];
   }
+  const float* inv = w.inv + size_t(p.fin) * p.n_tiles * p.n + size_t(t) * p.n;
+  const int ur = u0 + lr;
+  float best = -INFINITY;
+  if (ur < p.m) {
+    const float iu = inv[ul[ur]];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      float sdot = 0.0f;
+#pragma unroll
+      for (int src = 0; src < kAS; ++src) sdot += x[src][j];
+      const int pa = p0 + tx + 16 * j;
+      if (pa < p.n_anc) best = fmaxf(best, sdot * iu * inv[al[pa]]);
+    }
+  }
+#pragma unroll
+  for (int off = 8; off; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
+  if (tx == 0 && ur < p.m) atomicMax(&w.asim[size_t(t) * p.n + ul[ur]], ordered_key(best));
+  cl.sync();  // peers read this CTA's partial tile above
 }
 
 // ---- 4. K-means (Lloyd) and Eq. 2 quotas ------------------------------------------------------
@@ -304,8 +351,12 @@ __device__ __forceinline__ void cluster_column_reduce(cg::cluster_group& cl, flo
   const int c0 = rank * D / kKC, c1 = (rank + 1) * D / kKC, width = c1 - c0;
   for (int e = threadIdx.x; e < K * width; e += blockDim.x) {
     const int k = e / width, c = c0 + e % width;
+    float x[kKC];
+#pragma unroll
+    for (int rr = 0; rr < kKC; ++rr) x[rr] = cl.map_shared_rank(part, rr)[k * D + c];  // in flight
     float sum = 0.0f;
-    for (int rr = 0; rr < kKC; ++rr) sum += cl.map_shared_rank(part, rr)[k * D + c];
+#pragma unroll
+    for (int rr = 0; rr < kKC; ++rr) sum += x[rr];
     emit(k, c, sum);
   }
 }
@@ -322,36 +373,60 @@ __global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
   __shared__ float asum_part[SPD_MAX_CLUSTERS];
   __shared__ int changed;
   __shared__ int8_t asg[4096 / kKC + 1];
+  __shared__ int idx[4096 / kKC + 1];    // patch index of each of this CTA's tokens
+  __shared__ float av[4096 / kKC + 1];   // their a_j
+  __shared__ int ncl[SPD_MAX_CLUSTERS];  // cluster sizes over the whole cluster of CTAs
   cg::cluster_group cl = cg::this_cluster();
   const int rank = int(cl.block_rank());
   const int t = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nw = blockDim.x >> 5;
   const int j0 = rank * m / kKC, j1 = (rank + 1) * m / kKC, nl = j1 - j0;
   const int* ul = w.ulist + size_t(t) * m;
+  const size_t row0 = size_t(t) * p.n_tok + p.off;  // feature row of patch 0 of this tile
+  for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) {
+    idx[jj] = ul[j0 + jj];
+    av[jj] = ordered_val(w.asim[size_t(t) * p.n + ul[j0 + jj]]);
+  }
   if (m > 0) {
+#pragma unroll 4
     for (int e = threadIdx.x; e < K * D; e += blockDim.x) {
       const int k = e / D, c = e % D;
       cent[e] = feat_row(p, p.fin, t, ul[(k * m) / K])[c];
     }
   }
   __syncthreads();
+  const float* fin = p.feat[p.fin];
   for (int it = 0; it < p.iters && m > 0; ++it) {
     // assignment of this CTA's points
     if (threadIdx.x == 0) changed = 0;
     __syncthreads();
     for (int jj = warp; jj < nl; jj += nw) {
-      const float* x = feat_row(p, p.fin, t, ul[j0 + jj]);
+      const float* x = fin + (row0 + idx[jj]) * D;
       float part_d[SPD_MAX_CLUSTERS];
 #pragma unroll
       for (int k = 0; k < SPD_MAX_CLUSTERS; ++k) part_d[k] = 0.0f;
-      for (int c = lane; c < D; c += 32) {
-        const float xv = x[c];
+      // 16-byte loads, four in flight per lane (D is a multiple of 4)
+      for (int cb = 4 * lane; cb < D; cb += 512) {
+        float4 xv[4];
 #pragma unroll
-        for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
-          if (k < K) {
-            const float df = xv - cent[k * D + c];
-            part_d[k] += df * df;
+        for (int u = 0; u < 4; ++u) {
+          const int c = cb + 128 * u;
+          xv[u] = c < D ? *reinterpret_cast<const float4*>(x + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int c = cb + 128 * u;
+          if (c < D) {
+#pragma unroll
+            for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
+              if (k < K) {
+                const float4 ce = *reinterpret_cast<const float4*>(cent + k * D + c);
+                const float d0 = xv[u].x - ce.x, d1 = xv[u].y - ce.y, d2 = xv[u].z - ce.z,
+                            d3 = xv[u].w - ce.w;
+                part_d[k] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+              }
           }
+        }
       }
       int best = 0;
       float bd = 0.0f;
@@ -376,15 +451,28 @@ __global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
     __syncthreads();
     for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) atomicAdd(&cnt[asg[jj]], 1);
     for (int c = threadIdx.x; c < D; c += blockDim.x)
-      for (int jj = 0; jj < nl; ++jj) part[asg[jj] * D + c] += feat_row(p, p.fin, t, ul[j0 + jj])[c];
+      for (int jb = 0; jb < nl; jb += 8) {  // token order; eight loads in flight
+        float xv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          xv[u] = jb + u < nl ? fin[(row0 + idx[jb + u]) * D + c] : 0.0f;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (jb + u < nl) part[asg[jb + u] * D + c] += xv[u];
+      }
     cl.sync();
     int total_changed = 0;
     for (int rr = 0; rr < kKC; ++rr) total_changed += *cl.map_shared_rank(&changed, rr);
     if (it > 0 && total_changed == 0) break;  // cluster-uniform decision
     // new centroids for this CTA's column slice, written into every CTA
-    cluster_column_reduce(cl, part, K, D, rank, [&](int k, int c, float sum) {
+    if (threadIdx.x < K) {
       int n = 0;
-      for (int rr = 0; rr < kKC; ++rr) n += cl.map_shared_rank(cnt, rr)[k];
+      for (int rr = 0; rr < kKC; ++rr) n += cl.map_shared_rank(cnt, rr)[threadIdx.x];
+      ncl[threadIdx.x] = n;
+    }
+    __syncthreads();
+    cluster_column_reduce(cl, part, K, D, rank, [&](int k, int c, float sum) {
+      const int n = ncl[k];
       const float v = n > 0 ? sum / float(n) : cent[k * D + c];
       for (int rr = 0; rr < kKC; ++rr) cl.map_shared_rank(cent, rr)[k * D + c] = v;
     });
@@ -400,18 +488,26 @@ __global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
     atomicAdd(&cnt[asg[jj]], 1);
     w.assign[size_t(t) * m + j0 + jj] = asg[jj];
   }
-  if (threadIdx.x == 0)
-    for (int jj = 0; jj < nl; ++jj) asum_part[asg[jj]] += ordered_val(w.asim[size_t(t) * p.n + ul[j0 + jj]]);
+  if (threadIdx.x == 0)  // token order
+    for (int jj = 0; jj < nl; ++jj) asum_part[asg[jj]] += av[jj];
   // per layer: sums over each cluster of unit feature rows (F_l,j / ||F_l,j||)
   for (int l = 0; l < p.L; ++l) {
     const float* inv = w.inv + (size_t(l) * p.n_tiles + t) * p.n;
     __syncthreads();
     for (int e = threadIdx.x; e < K * D; e += blockDim.x) part[e] = 0.0f;
     __syncthreads();
+    const float* fl = p.feat[l];
     for (int c = threadIdx.x; c < D; c += blockDim.x)
-      for (int jj = 0; jj < nl; ++jj) {
-        const int i = ul[j0 + jj];
-        part[asg[jj] * D + c] += feat_row(p, l, t, i)[c] * inv[i];
+      for (int jb = 0; jb < nl; jb += 8) {  // token order; eight loads in flight
+        float xv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int i = jb + u < nl ? idx[jb + u] : 0;
+          xv[u] = jb + u < nl ? fl[(row0 + i) * D + c] * inv[i] : 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (jb + u < nl) part[asg[jb + u] * D + c] += xv[u];
       }
     cl.sync();
     float* csum = w.csum + (size_t(t) * p.L + l) * K * D;
@@ -650,8 +746,9 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
   SPD_CUDA_TRY(launch_pdl(rowstats_kernel, dim3((p.n + 7) / 8, T), dim3(256), 0, st, p, attn, w));
   SPD_CUDA_TRY(launch_pdl(anchor_kernel, dim3(T), dim3(1024), 0, st, p, w));
   if (p.n_anc > 0 && p.m > 0)
-    SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel, dim3((p.m + 63) / 64, (p.n_anc + 63) / 64, T),
-                            dim3(256), 0, st, p, w));
+    SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel,
+                            dim3((p.m + 63) / 64 * kAS, (p.n_anc + 63) / 64, T), dim3(256), 0, st,
+                            p, w));
   const size_t ksmem = size_t(2) * p.K * p.d * sizeof(float);
   static bool attr = false;
   if (!attr) {
