@@ -78,12 +78,13 @@ constexpr int kRecvPitch = 36;      // fp32 per row of a received 32-column chun
 
 struct KArgs {
   int n_out, n_tok, k, tt, n_kb, n_ttiles, units, grid, stages, ldo, rope_rows, head_dim,
-      out_cols, kbox, csplit, cluster, nbuf, hoff, nh, ldo2, split;
+      out_cols, kbox, csplit, cluster, nbuf, hoff, nh, ldo2, split, accs;
   // kbox: 64-wide boxes per stage (1 or 2); a k-block is kbox * 64 wide
   // csplit: CTAs per output tile in split-K (1 = stream-K); cluster: split-K CTAs reduce through
   // distributed shared memory (0: ADD epilogue, every CTA adds its own partial)
   // nbuf: TMEM accumulator buffers; hoff: TMEM column offset of the second 128-row half
-  // nh: 128-row halves per tile (1 or 2)
+  // nh: 128-row halves per tile (1 or 2); accs: TMEM columns between accumulator buffers
+  // CTA-pair kernels: a work item (grid entry) is a pair of CTAs sharing one M = 256 tile
   void* out;
   void* out2;
   const int32_t* rows;
@@ -343,14 +344,19 @@ __device__ __forceinline__ void add4(float (&acc)[8], int o, const float4& x) {
 }
 
 // 10 warps: three share an SM sub-partition's 16K registers, so at most 168 registers a thread.
-template <int EPI>
+// PAIR: a cluster of two CTAs computes 256 weight rows x the token tile with M = 256 MMAs
+// (tcgen05 cta_group::2): each CTA loads its own 128 weight rows and half of the tokens, the
+// even CTA issues the MMAs, each CTA's TMEM holds its 128 rows. Per weight byte that moves 5
+// bytes through shared memory instead of 6 (the token half is read by both tensor cores but
+// written once), the limit of the single-CTA main loop.
+template <int EPI, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_sk_kernel(const __grid_constant__ CUtensorMap map_w,
                    const __grid_constant__ CUtensorMap map_x, const KArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  const uint32_t xbox_bytes = a.tt * 128;
+  const uint32_t xbox_bytes = (PAIR ? a.tt / 2 : a.tt) * 128;
   const uint32_t wbox_bytes = a.nh * kHalfW;
   const uint32_t stage_bytes = a.kbox * (wbox_bytes + xbox_bytes);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.stages * stage_bytes);
@@ -365,15 +371,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   int* tpos = trow + 256;                     // [256] rotary position of each token
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int c = blockIdx.x;
+  const int c = blockIdx.x;              // CTA index (partial slots)
+  const int wc = PAIR ? c >> 1 : c;      // work item
+  const int prank = PAIR ? c & 1 : 0;    // CTA within the pair (cluster rank); 0 issues the MMAs
   int u0, u1;
-  if (a.csplit > 1) {  // split-K: rank r of tile c / C owns k-blocks [r n_kb / C, (r+1) n_kb / C)
-    const int tile = c / a.csplit, r = c - tile * a.csplit;
+  if (a.csplit > 1) {  // split-K: rank r of tile wc / C owns k-blocks [r n_kb / C, (r+1) n_kb / C)
+    const int tile = wc / a.csplit, r = wc - tile * a.csplit;
     u0 = tile * a.n_kb + r * a.n_kb / a.csplit;
     u1 = tile * a.n_kb + (r + 1) * a.n_kb / a.csplit;
   } else {
-    u0 = unit_lo(c, a);
-    u1 = unit_lo(c + 1, a);
+    u0 = unit_lo(wc, a);
+    u1 = unit_lo(wc + 1, a);
   }
   const SegPlan plan = seg_plan(u0, u1, a.n_kb);
 
@@ -384,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
-      mbar_init(&acce[b], kEpiThreads);
+      mbar_init(&acce[b], PAIR ? 2 : kEpiThreads);  // PAIR: one arrive per CTA
     }
     mbar_init(done, 1);
     flags[0] = 0;
@@ -396,13 +404,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&map_x);
   }
   if (warp == 0) {
-    tmem_alloc(tmem_slot, 2 * kAccCols);
-    tmem_relinquish();
+    if constexpr (PAIR) {
+      tmem_alloc_pair(tmem_slot, kAccCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, 2 * kAccCols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
+  uint32_t tmem;
+  if constexpr (PAIR) {
+    // barriers initialised and TMEM allocated in both CTAs before either signals the other; both
+    // use the even CTA's TMEM address (the one its MMAs write)
+    cg::this_cluster().sync();
+    tc_fence_after();
+    tmem = ld_dsmem_u32(dsmem_addr(tmem_slot, 0));
+  } else {
+    tc_fence_after();
+    tmem = *tmem_slot;
+  }
 
   pdl_launch_dependents();
   if (warp == 0) {
@@ -421,19 +443,30 @@ __global__ void __launch_bounds__(kThreads, 1)
           pre_kb[n_pre] = u - pre_tile[n_pre] * a.n_kb;
           const int wt = pre_tile[n_pre] / a.n_ttiles;
           uint8_t* st = smem + n_pre * stage_bytes;
-          mbar_arrive_expect_tx(&full[n_pre], stage_bytes);
-          for (int bx = 0; bx < a.kbox; ++bx)
-            tma_load_2d(st + bx * wbox_bytes, &map_w, &full[n_pre],
-                        (pre_kb[n_pre] * a.kbox + bx) * kBK, wt * a.nh * kBM, pol_w);
+          if (prank == 0) mbar_arrive_expect_tx(&full[n_pre], PAIR ? 2 * stage_bytes : stage_bytes);
+          for (int bx = 0; bx < a.kbox; ++bx) {
+            const int kx = (pre_kb[n_pre] * a.kbox + bx) * kBK;
+            if constexpr (PAIR)
+              tma_load_2d_pair(st + bx * wbox_bytes, &map_w, dsmem_addr(&full[n_pre], 0), kx,
+                               (2 * wt + prank) * kBM, pol_w);
+            else
+              tma_load_2d(st + bx * wbox_bytes, &map_w, &full[n_pre], kx, wt * a.nh * kBM, pol_w);
+          }
         }
       }
       pdl_wait();
       for (int i = 0; i < n_pre; ++i) {
         const int tt_i = pre_tile[i] - (pre_tile[i] / a.n_ttiles) * a.n_ttiles;
         uint8_t* st = smem + i * stage_bytes;
-        for (int bx = 0; bx < a.kbox; ++bx)
-          tma_load_2d(st + a.kbox * wbox_bytes + bx * xbox_bytes, &map_x, &full[i],
-                      (pre_kb[i] * a.kbox + bx) * kBK, tt_i * a.tt, pol_x);
+        for (int bx = 0; bx < a.kbox; ++bx) {
+          const int kx = (pre_kb[i] * a.kbox + bx) * kBK;
+          if constexpr (PAIR)
+            tma_load_2d_pair(st + a.kbox * wbox_bytes + bx * xbox_bytes, &map_x,
+                             dsmem_addr(&full[i], 0), kx, tt_i * a.tt + prank * (a.tt / 2), pol_x);
+          else
+            tma_load_2d(st + a.kbox * wbox_bytes + bx * xbox_bytes, &map_x, &full[i], kx,
+                        tt_i * a.tt, pol_x);
+        }
       }
       counts[0] = n_pre;
       int i = 0;
@@ -454,12 +487,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           uint8_t* st = smem + s * stage_bytes;
-          mbar_arrive_expect_tx(&full[s], stage_bytes);
+          if (prank == 0) mbar_arrive_expect_tx(&full[s], PAIR ? 2 * stage_bytes : stage_bytes);
           for (int bx = 0; bx < a.kbox; ++bx) {
             const int ks = kb * a.kbox + bx;
-            tma_load_2d(st + bx * wbox_bytes, &map_w, &full[s], ks * kBK, wt * a.nh * kBM, pol_w);
-            tma_load_2d(st + a.kbox * wbox_bytes + bx * xbox_bytes, &map_x, &full[s], ks * kBK,
-                        tt_i * a.tt, pol_x);
+            if constexpr (PAIR) {
+              const uint32_t fb = dsmem_addr(&full[s], 0);
+              tma_load_2d_pair(st + bx * wbox_bytes, &map_w, fb, ks * kBK, (2 * wt + prank) * kBM,
+                               pol_w);
+              tma_load_2d_pair(st + a.kbox * wbox_bytes + bx * xbox_bytes, &map_x, fb, ks * kBK,
+                               tt_i * a.tt + prank * (a.tt / 2), pol_x);
+            } else {
+              tma_load_2d(st + bx * wbox_bytes, &map_w, &full[s], ks * kBK, wt * a.nh * kBM, pol_w);
+              tma_load_2d(st + a.kbox * wbox_bytes + bx * xbox_bytes, &map_x, &full[s], ks * kBK,
+                          tt_i * a.tt, pol_x);
+            }
           }
           counts[0] = i + 1;
         }
@@ -467,9 +508,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     pdl_wait();
-    if (lane == 0) {
-      // ---- MMA issuer ----
-      const uint32_t idesc = idesc_bf16_f32(kBM, a.tt);
+    if (lane == 0 && prank == 0) {
+      // ---- MMA issuer (PAIR: the even CTA, for both) ----
+      const uint32_t idesc = idesc_bf16_f32(PAIR ? 2 * kBM : kBM, a.tt);
       const int ksub = a.kbox * (kBK / 16);
       int i = 0;
       bool ok = true;
@@ -482,7 +523,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t d = tmem + b * kAccCols;
+        const uint32_t d = tmem + b * a.accs;
         for (int uu = u; uu < seg_end; ++uu, ++i) {
           const int s = i % a.stages;
           const uint32_t ph = (i / a.stages) & 1;
@@ -497,21 +538,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t off = (kk & 3) * 32;
             const uint64_t bdesc = sdesc_k128(sx + (kk >> 2) * xbox_bytes + off);
             const uint32_t accum = (uu != u || kk != 0) ? 1u : 0u;
-            for (int h = 0; h < a.nh; ++h)
-              mma_bf16(d + h * a.hoff, sdesc_k128(sw + (kk >> 2) * wbox_bytes + h * kHalfW + off),
-                       bdesc, idesc, accum);
+            if constexpr (PAIR) {
+              mma_bf16_pair(d, sdesc_k128(sw + (kk >> 2) * wbox_bytes + off), bdesc, idesc, accum);
+            } else {
+              for (int h = 0; h < a.nh; ++h)
+                mma_bf16(d + h * a.hoff,
+                         sdesc_k128(sw + (kk >> 2) * wbox_bytes + h * kHalfW + off), bdesc, idesc,
+                         accum);
+            }
           }
-          mma_commit(&empty[s]);
+          if constexpr (PAIR) mma_commit_pair(&empty[s], 3);  // both CTAs' stage s is free
+          else mma_commit(&empty[s]);
           counts[1] = i + 1;
         }
         if (!ok) break;
-        mma_commit(&accf[b]);
+        if constexpr (PAIR) mma_commit_pair(&accf[b], 3);
+        else mma_commit(&accf[b]);
       }
       if (!ok) {
         flags[0] = 1;
         set_status(a.status, SPD_ETIMEOUT);
       }
-      mma_commit(done);  // arrives once every MMA issued above has completed
+      // arrives once every MMA issued above has completed
+      if constexpr (PAIR) mma_commit_pair(done, 1);
+      else mma_commit(done);
       volatile int no_abort = 0;
       if (!mbar_wait(done, 0, &no_abort, a.budget)) set_status(a.status, SPD_ETIMEOUT);
     }
@@ -540,7 +590,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int wt = tile / a.n_ttiles, tt_i = tile - wt * a.n_ttiles;
       const int tok0 = tt_i * a.tt;
       const int valid = min(a.tt, a.n_tok - tok0);
-      const uint32_t tq = tmem + b * kAccCols + (static_cast<uint32_t>(q * 32) << 16);
+      const uint32_t tq = tmem + b * a.accs + (static_cast<uint32_t>(q * 32) << 16);
+      const int blk0 = PAIR ? 2 * wt + prank : a.nh * wt;  // first 128-row block of this CTA
       // token metadata of this tile, staged once per segment
       const int et = threadIdx.x - 64;
       if (et < valid) {
@@ -554,8 +605,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int cc = half * 8; cc < valid; cc += 16) {
             float v[8];
             tmem_ld8(tq + h * a.hoff + cc, v);
-            epilogue8<EPI>(a, (a.nh * wt + h) * kBM + row, q, lane, a.nh * wt + h, tok0 + cc, v,
-                           trow, tpos, tok0);
+            epilogue8<EPI>(a, (blk0 + h) * kBM + row, q, lane, blk0 + h, tok0 + cc, v, trow, tpos,
+                           tok0);
           }
         }
       } else {
@@ -578,20 +629,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         __threadfence();
         epi_bar();
+        const int ctr = PAIR ? 2 * tile + prank : tile;  // PAIR: each CTA's rows fix up alone
         if (threadIdx.x == 64) {
-          const int old = atomicAdd(&a.counters[tile], seg_len);
+          const int old = atomicAdd(&a.counters[ctr], seg_len);
           flags[1] = (old + seg_len == a.n_kb);
         }
         epi_bar();
         if (flags[1]) {
           __threadfence();
+          // contributors are work items c_first..c_last (this one: wc); the partial of item o
+          // sits in the head or tail slot of its CTA (PAIR: the CTA holding these rows)
           const int c_first = cta_of_unit(tile * a.n_kb, a);
           const int c_last = cta_of_unit((tile + 1) * a.n_kb - 1, a);
+          auto slot_of = [&](int o) {
+            return 2 * (PAIR ? 2 * o + prank : o) + (tile == unit_lo(o, a) / a.n_kb ? 0 : 1);
+          };
           if (c_last - c_first == 1) {
             // one other contributor (the usual case): its partial for eight 8-column groups in
             // flight at a time; a + b is exact in either order, so this matches the loop below
-            const int o = (c == c_first) ? c_last : c_first;
-            const int os = 2 * o + (tile == unit_lo(o, a) / a.n_kb ? 0 : 1);
+            const int o = (wc == c_first) ? c_last : c_first;
+            const int os = slot_of(o);
             for (int h = 0; h < a.nh; ++h) {
               const float4* src = part + size_t(os) * slot_len + h * half_len + row;
 #pragma unroll 1
@@ -613,7 +670,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tmem_ld8(tq + h * a.hoff + cc, v);
                     add4(v, 0, x[0]);
                     add4(v, 4, x[1]);
-                    epilogue8<EPI>(a, (a.nh * wt + h) * kBM + row, q, lane, a.nh * wt + h,
+                    epilogue8<EPI>(a, (blk0 + h) * kBM + row, q, lane, blk0 + h,
                                    tok0 + cc, v, trow, tpos, tok0);
                   }
                   // next group's data into the fixed slots (static register indices)
@@ -625,11 +682,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           } else if (c_last - c_first == 2) {
             // two other contributors: two groups in flight, summed in CTA order
             // ((first + second) + third, this CTA's own partial in its place), as below
-            const int own = c - c_first;
+            const int own = wc - c_first;
             const int oa = (own == 0) ? c_first + 1 : c_first;  // first other contributor
             const int ob = (own == 2) ? c_first + 1 : c_last;   // second
-            const int sa = 2 * oa + (tile == unit_lo(oa, a) / a.n_kb ? 0 : 1);
-            const int sb = 2 * ob + (tile == unit_lo(ob, a) / a.n_kb ? 0 : 1);
+            const int sa = slot_of(oa);
+            const int sb = slot_of(ob);
             for (int h = 0; h < a.nh; ++h) {
               const float4* pa = part + size_t(sa) * slot_len + h * half_len + row;
               const float4* pb = part + size_t(sb) * slot_len + h * half_len + row;
@@ -663,7 +720,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                       else if (own == 1) acc[k] = (x1[k] + v[k]) + x2[k];
                       else acc[k] = (x1[k] + x2[k]) + v[k];
                     }
-                    epilogue8<EPI>(a, (a.nh * wt + h) * kBM + row, q, lane, a.nh * wt + h,
+                    epilogue8<EPI>(a, (blk0 + h) * kBM + row, q, lane, blk0 + h,
                                    tok0 + cc, acc, trow, tpos, tok0);
                   }
                   xa[0] = xa[2];
@@ -685,16 +742,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
               for (int o = c_first; o <= c_last; o += 2) {
                 float4 x[4];
-                const bool l0 = (o != c), l1 = (o + 1 <= c_last) && (o + 1 != c);
+                const bool l0 = (o != wc), l1 = (o + 1 <= c_last) && (o + 1 != wc);
                 if (l0) {
-                  const int os = 2 * o + (tile == unit_lo(o, a) / a.n_kb ? 0 : 1);
+                  const int os = slot_of(o);
                   const float4* src =
                       part + size_t(os) * slot_len + h * half_len + size_t(cc / 4) * kBM + row;
                   x[0] = __ldcg(src);
                   x[1] = __ldcg(src + kBM);
                 }
                 if (l1) {
-                  const int os = 2 * (o + 1) + (tile == unit_lo(o + 1, a) / a.n_kb ? 0 : 1);
+                  const int os = slot_of(o + 1);
                   const float4* src =
                       part + size_t(os) * slot_len + h * half_len + size_t(cc / 4) * kBM + row;
                   x[2] = __ldcg(src);
@@ -717,21 +774,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                   }
                 }
               }
-              epilogue8<EPI>(a, (a.nh * wt + h) * kBM + row, q, lane, a.nh * wt + h, tok0 + cc,
+              epilogue8<EPI>(a, (blk0 + h) * kBM + row, q, lane, blk0 + h, tok0 + cc,
                              acc, trow, tpos, tok0);
             }
           }
           }
-          if (threadIdx.x == 64) a.counters[tile] = 0;  // ready for the next launch
+          if (threadIdx.x == 64) a.counters[ctr] = 0;  // ready for the next launch
         }
       }
-      epi_bar();  // trow / tpos / flags[1] are reused by the next segment
       tc_fence_before();
-      mbar_arrive(&acce[b]);
+      epi_bar();  // trow / tpos / flags[1] are reused by the next segment
+      if constexpr (PAIR) {  // one arrive per CTA on the even CTA's barrier
+        if (threadIdx.x == 64) {
+          if (prank == 0) mbar_arrive(&acce[b]);
+          else mbar_arrive_cluster(dsmem_addr(&acce[b], 0));
+        }
+      } else {
+        mbar_arrive(&acce[b]);
+      }
     }
   }
   __syncthreads();
-  if (a.cluster) {
+  if (!PAIR && a.cluster) {
     // cluster reduction, one 128-row half at a time; every thread of every CTA of the cluster
     // takes part in every barrier. Receive layout in each owner's ring: [sender][owned chunk][128
     // rows][kRecvPitch] fp32 (32 columns + 4 of padding: conflict-free 16-byte accesses).
@@ -792,8 +856,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
-  if (threadIdx.x == 0 && flags[0]) {
-    // drain: TMA loads issued but never consumed must land before the CTA exits
+  if (threadIdx.x == 0 && flags[0] && prank == 0) {
+    // drain: TMA loads issued but never consumed must land before the CTA exits (PAIR: the even
+    // CTA's stage barriers count both CTAs' loads)
     for (int i = counts[1]; i < counts[0]; ++i) {
       volatile int no_abort = 0;
       mbar_wait(&full[i % a.stages], (i / a.stages) & 1, &no_abort, a.budget);
@@ -801,8 +866,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
-  tc_fence_after();
-  if (warp == 0) tmem_dealloc(tmem, 2 * kAccCols);
+  if constexpr (PAIR) {
+    // the even CTA's MMAs have completed (its MMA thread waited above) and both CTAs' epilogues
+    // are done before either CTA frees its TMEM or leaves (its shared memory feeds the MMAs)
+    cg::this_cluster().sync();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc_pair(*tmem_slot, kAccCols);
+  } else {
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, 2 * kAccCols);
+  }
 }
 
 // ---- host side -------------------------------------------------------------------------------
@@ -853,19 +926,21 @@ namespace {
 
 using KernelFn = void (*)(CUtensorMap, CUtensorMap, KArgs);
 
+template <bool PAIR>
 KernelFn kernel_for(int epi) {
   switch (epi) {
-    case EPI_F32: return gemm_sk_kernel<EPI_F32>;
-    case EPI_BF16: return gemm_sk_kernel<EPI_BF16>;
-    case EPI_BIAS_BF16: return gemm_sk_kernel<EPI_BIAS_BF16>;
-    case EPI_BIAS_GELU_BF16: return gemm_sk_kernel<EPI_BIAS_GELU_BF16>;
-    case EPI_ADD_F32: return gemm_sk_kernel<EPI_ADD_F32>;
-    case EPI_ROPE_BF16: return gemm_sk_kernel<EPI_ROPE_BF16>;
-    case EPI_SWIGLU_BF16: return gemm_sk_kernel<EPI_SWIGLU_BF16>;
-    case EPI_QKV_BF16: return gemm_sk_kernel<EPI_QKV_BF16>;
+    case EPI_F32: return gemm_sk_kernel<EPI_F32, PAIR>;
+    case EPI_BF16: return gemm_sk_kernel<EPI_BF16, PAIR>;
+    case EPI_BIAS_BF16: return gemm_sk_kernel<EPI_BIAS_BF16, PAIR>;
+    case EPI_BIAS_GELU_BF16: return gemm_sk_kernel<EPI_BIAS_GELU_BF16, PAIR>;
+    case EPI_ADD_F32: return gemm_sk_kernel<EPI_ADD_F32, PAIR>;
+    case EPI_ROPE_BF16: return gemm_sk_kernel<EPI_ROPE_BF16, PAIR>;
+    case EPI_SWIGLU_BF16: return gemm_sk_kernel<EPI_SWIGLU_BF16, PAIR>;
+    case EPI_QKV_BF16: return gemm_sk_kernel<EPI_QKV_BF16, PAIR>;
     default: return nullptr;
   }
 }
+KernelFn kernel_for(int epi, bool pair) { return pair ? kernel_for<true>(epi) : kernel_for<false>(epi); }
 
 // Sets the shared-memory limit of every instance once; returns the first error.
 cudaError_t set_kernel_attributes() {
@@ -875,11 +950,13 @@ cudaError_t set_kernel_attributes() {
     for (int e : {int(EPI_F32), int(EPI_BF16), int(EPI_BIAS_BF16), int(EPI_BIAS_GELU_BF16),
                   int(EPI_ADD_F32), int(EPI_ROPE_BF16), int(EPI_SWIGLU_BF16),
                   int(EPI_QKV_BF16)}) {
-      const cudaError_t r =
-          cudaFuncSetAttribute(reinterpret_cast<const void*>(kernel_for(e)),
-                               cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               kSmemPipe + 1024 + 256 + 16384);
-      if (r != cudaSuccess && err == cudaSuccess) err = r;
+      for (bool pair : {false, true}) {
+        const cudaError_t r =
+            cudaFuncSetAttribute(reinterpret_cast<const void*>(kernel_for(e, pair)),
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kSmemPipe + 1024 + 256 + 16384);
+        if (r != cudaSuccess && err == cudaSuccess) err = r;
+      }
     }
   });
   return err;
@@ -904,7 +981,8 @@ int max_active_clusters(int C) {
       cfg.attrs = attr;
       cfg.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kernel_for(EPI_F32)),
+      if (cudaOccupancyMaxActiveClusters(&n,
+                                         reinterpret_cast<const void*>(kernel_for(EPI_F32, false)),
                                          &cfg) != cudaSuccess) {
         cudaGetLastError();
         n = 0;
@@ -920,8 +998,7 @@ int max_active_clusters(int C) {
 int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   if (p.n_tok <= 0 || p.n_out <= 0) return SPD_OK;
   if (p.k <= 0) return fail(SPD_EINVAL, "GEMM K must be positive");
-  const KernelFn kern = kernel_for(p.epi);
-  if (!kern) return fail(SPD_EINVAL, "unknown GEMM epilogue %d", p.epi);
+  if (!kernel_for(p.epi, false)) return fail(SPD_EINVAL, "unknown GEMM epilogue %d", p.epi);
   if (!p.map_w && !p.w) return fail(SPD_EINVAL, "GEMM without weights");
   if (cudaError_t e = set_kernel_attributes())
     return fail(SPD_ECUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(e));
@@ -931,47 +1008,66 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.k = p.k;
   a.n_ttiles = (p.n_tok + 255) / 256;
   a.tt = ((p.n_tok + a.n_ttiles - 1) / a.n_ttiles + 31) / 32 * 32;
-  // 256-row tiles for token tiles of at most 64: their stages are mostly weights, and two MMAs
-  // per token box double the weight bytes per stage (needs the row-major pointer for the map)
-  a.nh = (a.tt <= 64 && p.w) ? 2 : 1;
-  const int tile_rows = a.nh * kBM;
-  const int wbox = a.nh * kHalfW;
+  const int sms = num_sms();
+  // CTA pairs (M = 256 over two SMs) for token tiles of at least 128, except where the tiles are
+  // so few that only the cluster reduction of split-K partials fills the GPU (non-residual
+  // epilogues): there the single-CTA kernel runs.
+  const int slots = sms / 2;  // pairs the GPU holds at once
+  const long long pair_tiles = (long long)((p.n_out + 2 * kBM - 1) / (2 * kBM)) * a.n_ttiles;
+  const bool pair = a.tt >= 128 && !(p.epi != EPI_ADD_F32 && pair_tiles * 2 <= slots);
+  // 256-row tiles in one CTA for token tiles of at most 64: their stages are mostly weights, and
+  // two MMAs per token box double the weight bytes per stage (needs the row-major pointer)
+  a.nh = (!pair && a.tt <= 64 && p.w) ? 2 : 1;
+  const int tile_rows = pair ? 2 * kBM : a.nh * kBM;  // weight rows per work item
+  const int cta_rows = pair ? kBM : tile_rows;          // ... per CTA
+  const int wbox = (pair ? 1 : a.nh) * kHalfW;
+  const int xrows = pair ? a.tt / 2 : a.tt;            // token rows per CTA
   auto stages_for = [&](int kb) {
-    return std::min(kMaxStages, kSmemPipe / (kb * (wbox + a.tt * 128)));
+    return std::min(kMaxStages, kSmemPipe / (kb * (wbox + xrows * 128)));
   };
   // 128-wide k-blocks (256 contiguous bytes of every weight row per stage) when two stages fit
   a.kbox = (p.k > kBK && stages_for(2) >= 2) ? 2 : 1;
   a.n_kb = (p.k + a.kbox * kBK - 1) / (a.kbox * kBK);
   a.stages = stages_for(a.kbox);
-  const int stage_bytes = a.kbox * (wbox + a.tt * 128);
-  // TMEM (512 columns): two accumulator buffers of 256 columns unless a 256-row tile is wider than
-  // 128 tokens; the second 128-row half sits 128 or 256 columns after the first
-  a.nbuf = (a.nh * a.tt <= 256) ? 2 : 1;
-  a.hoff = a.tt <= 128 ? 128 : 256;
+  const int stage_bytes = a.kbox * (wbox + xrows * 128);
+  // TMEM. Single CTA: 512 columns, two accumulator buffers of 256 unless a 256-row tile is wider
+  // than 128 tokens; the second 128-row half sits 128 or 256 columns after the first. Pair: 256
+  // columns, two buffers of 128 for token tiles up to 128, else one.
+  if (pair) {
+    a.nbuf = a.tt <= 128 ? 2 : 1;
+    a.accs = 128;
+    a.hoff = 0;
+  } else {
+    a.nbuf = (a.nh * a.tt <= 256) ? 2 : 1;
+    a.accs = kAccCols;
+    a.hoff = a.tt <= 128 ? 128 : 256;
+  }
   CUtensorMap map_w, map_x;
-  if (a.nh == 1 && p.map_w) {
+  if (cta_rows == kBM && p.map_w) {
     map_w = *p.map_w;
-  } else if (int rc = make_map(&map_w, p.w, p.k, p.n_out, tile_rows)) {
+  } else if (int rc = make_map(&map_w, p.w, p.k, p.n_out, cta_rows)) {
     return rc;
   }
-  if (int rc = make_map(&map_x, p.x, p.k, p.n_tok, a.tt)) return rc;
+  if (int rc = make_map(&map_x, p.x, p.k, p.n_tok, xrows)) return rc;
   const int n_wtiles = (p.n_out + tile_rows - 1) / tile_rows;
   const long long tiles = (long long)n_wtiles * a.n_ttiles;
-  if (tiles > s.n_counters) return fail(SPD_EUNSUPPORTED, "GEMM has too many output tiles");
+  if (tiles * (pair ? 2 : 1) > s.n_counters)
+    return fail(SPD_EUNSUPPORTED, "GEMM has too many output tiles");
   const long long units = tiles * a.n_kb;
   if (units > 0x3fffffffLL) return fail(SPD_EUNSUPPORTED, "GEMM too large");
   a.units = int(units);
-  const int sms = num_sms();
-  // split-K when the tiles fill at most half the SMs. ADD epilogues: the most CTAs per tile (a
-  // power of two, at least two k-blocks each) that still fit one per SM. Others: the largest C in
-  // {2, 4, 8} with at least one k-block per CTA whose clusters all fit on the GPU at once.
+  const int work_slots = pair ? slots : sms;  // work items the GPU holds at once
+  // split-K when the tiles fill at most half the work slots. ADD epilogues: the most work items
+  // per tile (a power of two, at least two k-blocks each) that still fit. Others (single CTA):
+  // the largest C in {2, 4, 8} with at least one k-block per CTA whose clusters all fit on the
+  // GPU at once.
   a.csplit = 1;
   a.cluster = 0;
-  if (tiles * 2 <= sms && p.epi == EPI_ADD_F32) {
+  if (tiles * 2 <= work_slots && p.epi == EPI_ADD_F32) {
     int C = 2;
-    while (tiles * C * 2 <= sms && C * 4 <= a.n_kb) C *= 2;
+    while (tiles * C * 2 <= work_slots && C * 4 <= a.n_kb) C *= 2;
     if (C * 2 <= a.n_kb) a.csplit = C;
-  } else if (tiles * 2 <= sms) {
+  } else if (!pair && tiles * 2 <= sms) {
     for (int C = 8; C >= 2; C /= 2) {
       // the ring receives C copies of each CTA's share of 32-column chunks ([128][36] fp32 each)
       const int chunks = a.tt / 32, cpo = (chunks + C - 1) / C;
@@ -984,22 +1080,24 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
       }
     }
   }
-  // one CTA per SM with at least 2 units each; every CTA owns two partial slots (head, tail)
-  long long grid = sms;
+  // stream-K: one work item per slot with at least 2 units each; every CTA owns two partial
+  // slots (head, tail) of its rows x the token tile
+  long long grid = work_slots;
   if (grid > (units + 1) / 2) grid = (units + 1) / 2;
-  const size_t per_slot = size_t(a.tt) * tile_rows;
-  if (size_t(2 * grid) * per_slot > s.partial_floats) grid = s.partial_floats / (2 * per_slot);
+  const size_t per_item = size_t(2) * a.tt * tile_rows;  // both slots of every CTA of the item
+  if (size_t(grid) * per_item > s.partial_floats) grid = s.partial_floats / per_item;
   if (grid < 1) grid = 1;
   if (units * (grid + 1) >= (1LL << 31)) return fail(SPD_EUNSUPPORTED, "GEMM too large");
   if (a.csplit > 1) {
     grid = tiles * a.csplit;
-  } else if (tiles <= sms && tiles * 2 > sms && a.tt >= 128) {
-    // between half and all of the SMs' worth of wide tiles: one whole tile per CTA. Stream-K's
-    // balance would split most tiles two or three ways, and the fixups of wide token tiles cost
-    // more than the idle SMs do.
+  } else if (tiles <= work_slots && tiles * 2 > work_slots && a.tt >= 128) {
+    // between half and all of the work slots' worth of wide tiles: one whole tile per work item.
+    // Stream-K's balance would split most tiles two or three ways, and the fixups of wide token
+    // tiles cost more than the idle SMs do.
     grid = tiles;
   }
   a.grid = int(grid);
+  const KernelFn kern = kernel_for(p.epi, pair);
   a.out = p.out;
   a.ldo = p.ldo;
   a.out2 = p.out2;
@@ -1021,7 +1119,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   const int slot = trace_begin(stream);
   {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(a.grid);
+    cfg.gridDim = dim3(pair ? 2 * a.grid : a.grid);
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
@@ -1029,7 +1127,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = a.cluster ? a.csplit : 1;
+    attr[1].val.clusterDim.x = pair ? 2 : (a.cluster ? a.csplit : 1);
     attr[1].val.clusterDim.y = 1;
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;

@@ -73,3 +73,31 @@ def test_linear_split_tiles_are_deterministic():
         N.spd_linear(X.cuda(), M, K, W.cuda(), N_, N.EPI_F32, out, N_, ws)
         outs.append(out)
     assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
+@pytest.mark.parametrize("M,K,N_,epi", [
+    (256, 1024, 22016, N.EPI_F32),      # CTA pairs, stream-K (86 pair tiles > 76 pair slots)
+    (256, 4096, 12288, N.EPI_F32),      # CTA pairs, one tile per pair (48 pair tiles)
+    (230, 2048, 11008, N.EPI_F32),      # CTA pairs, stream-K, ragged token tile halves
+    (200, 4096, 4096, N.EPI_ADD_F32),   # CTA pairs, split-K with red.add
+    (160, 11008, 4096, N.EPI_ADD_F32),  # CTA pairs, split-K, long K
+])
+def test_linear_cta_pairs(M, K, N_, epi):
+    X, W = operands(M, K, N_, seed=M + K)
+    ref = bf16_np(X) @ bf16_np(W).T
+    ws = torch.zeros(N.spd_linear_workspace_size(M, N_), dtype=torch.uint8, device="cuda")
+    h0 = torch.randn(M, N_, device="cuda") if epi == N.EPI_ADD_F32 else torch.zeros(M, N_, device="cuda")
+    outs = []
+    for _ in range(2):
+        out = h0.clone() if epi == N.EPI_ADD_F32 else torch.full((M, N_), float("nan"), device="cuda")
+        N.spd_linear(X.cuda(), M, K, W.cuda(), N_, epi, out, N_, ws)
+        torch.cuda.synchronize()
+        assert N.spd_workspace_status(ws) == 0
+        outs.append(out)
+    want = ref + (h0.cpu().double().numpy() if epi == N.EPI_ADD_F32 else 0.0)
+    for out in outs:
+        got = out.cpu().numpy()
+        assert np.isfinite(got).all()
+        assert rowwise_rel(got, want) < 1e-4
+    if epi == N.EPI_F32:  # split tiles are summed in CTA order: bit-identical runs
+        assert torch.equal(outs[0], outs[1])

@@ -140,3 +140,18 @@ def test_projector():
     got = bf16_np(x)
     assert rowwise_rel(got[rows.numpy()], ref) < TOL
     assert not got[0::2].any()
+
+
+def test_llava_width_layer_with_cta_pairs():
+    # one decoder layer at the LLaVA-1.5-7B width (the benchmark's GEMM shapes: fused QKV over
+    # 256 tokens, gate-up, down, O on query/FFN rows), a skip plan on the visual tokens
+    cfg = dict(n_layers=1, d_model=4096, n_heads=32, n_kv_heads=32, head_dim=128, d_ffn=11008,
+               vocab=1000, rope_theta=1e4, rms_eps=1e-5, d_vis=0, d_proj=0)
+    model, om = build(cfg, 21, std=0.02)
+    T = 256
+    x = inputs(T, 4096, 22)
+    vis = np.r_[np.ones(192, bool), np.zeros(64, bool)]
+    r = np.random.default_rng(23)
+    mask = np.zeros((1, T), np.uint8)
+    mask[0, vis] = r.integers(0, 3, size=192)  # some tokens skip attention, some the FFN
+    check(model, om, x, [0, T], mask)
