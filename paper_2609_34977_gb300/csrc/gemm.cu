@@ -404,8 +404,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&map_x);
   }
   if (warp == 0) {
-    if constexpr (PAIR) {
-      tmem_alloc_pair(tmem_slot, kAccCols);
+    if constexpr (PAIR) {  // collective: both CTAs receive the same columns
+      tmem_alloc_pair(tmem_slot, 2 * kAccCols);
       tmem_relinquish_pair();
     } else {
       tmem_alloc(tmem_slot, 2 * kAccCols);
@@ -871,7 +871,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // are done before either CTA frees its TMEM or leaves (its shared memory feeds the MMAs)
     cg::this_cluster().sync();
     tc_fence_after();
-    if (warp == 0) tmem_dealloc_pair(*tmem_slot, kAccCols);
+    if (warp == 0) tmem_dealloc_pair(*tmem_slot, 2 * kAccCols);
   } else {
     tc_fence_after();
     if (warp == 0) tmem_dealloc(tmem, 2 * kAccCols);
@@ -1030,12 +1030,12 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.n_kb = (p.k + a.kbox * kBK - 1) / (a.kbox * kBK);
   a.stages = stages_for(a.kbox);
   const int stage_bytes = a.kbox * (wbox + xrows * 128);
-  // TMEM. Single CTA: 512 columns, two accumulator buffers of 256 unless a 256-row tile is wider
-  // than 128 tokens; the second 128-row half sits 128 or 256 columns after the first. Pair: 256
-  // columns, two buffers of 128 for token tiles up to 128, else one.
+  // TMEM: 512 columns. Single CTA: two accumulator buffers of 256 unless a 256-row tile is wider
+  // than 128 tokens; the second 128-row half sits 128 or 256 columns after the first. Pair: two
+  // buffers of 256 (each CTA's TMEM holds its 128 rows).
   if (pair) {
-    a.nbuf = a.tt <= 128 ? 2 : 1;
-    a.accs = 128;
+    a.nbuf = 2;
+    a.accs = kAccCols;
     a.hoff = 0;
   } else {
     a.nbuf = (a.nh * a.tt <= 256) ? 2 : 1;
