@@ -189,6 +189,25 @@ int spd_project(const spd_model* m, const uint16_t* vis, int rows, const int32_t
 int spd_scatter_rows(const spd_model* m, const uint16_t* src, int rows, const int32_t* rows_map,
                      uint16_t* dst, void* stream);
 
+/* Workspace bytes of spd_attention for n_q queries in n_seqs sequences. */
+size_t spd_attention_workspace_size(int n_q, int n_seqs);
+
+/* The attention step of a decoder layer on its own (Sec. 3.2 VSkip-Attn: only the active tokens
+ * are queries; every token of a sequence is a key and a value of that sequence):
+ *   o_i = softmax_{t <= pos_i} (q_i . k_t / sqrt(head_dim)) v_t   per head, head h reading K/V head
+ *   h / (n_heads / n_kv_heads), keys t of the query's own sequence.
+ * q (dev) bf16 [n_q][n_heads * head_dim]: the queries of sequence b are rows [q_cu[b], q_cu[b+1]),
+ * positions q_pos (dev int32 [n_q]) strictly ascending within a sequence and in [0, its length).
+ * kv (dev) bf16 [n_kv][2 * n_kv_heads * head_dim]: per token K (rotated) then V; the tokens of
+ * sequence b are rows [cu_seqlens[b], cu_seqlens[b+1]). q_cu and cu_seqlens are HOST int32 [n_seqs+1]
+ * from 0 to n_q and n_kv. o (dev) bf16 [n_q][n_heads * head_dim]. head_dim 64 or 128.
+ * Positions that break the precondition give wrong values, never an out-of-bounds access.
+ * Errors: SPD_EINVAL, SPD_EUNSUPPORTED (head_dim), SPD_ENOSPC; device timeouts in the workspace's
+ * status word. */
+int spd_attention(const uint16_t* q, int n_q, const int32_t* q_pos, const int32_t* q_cu,
+                  const uint16_t* kv, int n_kv, const int32_t* cu_seqlens, int n_seqs, int n_heads,
+                  int n_kv_heads, int head_dim, uint16_t* o, void* ws, size_t ws_bytes, void* stream);
+
 /* Workspace bytes of spd_prefill for up to `max_tokens` packed tokens in up to `max_seqs` sequences. */
 size_t spd_prefill_workspace_size(const spd_model* m, int max_tokens, int max_seqs);
 

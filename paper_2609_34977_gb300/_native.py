@@ -22,7 +22,8 @@ EPI_F32, EPI_BF16, EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_ADD_F32 = 0, 1, 2, 3, 
 EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait",
            "spd_prune_workspace_size", "spd_prune", "spd_gather_rows_bf16", "spd_model_create",
            "spd_model_destroy", "spd_plan_adaptive", "spd_plan_static", "spd_project_workspace_size",
-           "spd_project", "spd_scatter_rows", "spd_prefill_workspace_size", "spd_prefill",
+           "spd_project", "spd_scatter_rows", "spd_attention_workspace_size", "spd_attention",
+           "spd_prefill_workspace_size", "spd_prefill",
            "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
            "spd_trace_read")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
@@ -84,6 +85,8 @@ def lib():
             "spd_project_workspace_size": (sz, [vp, i]),
             "spd_project": (i, [vp, vp, i, vp, vp, vp, sz, vp]),
             "spd_scatter_rows": (i, [vp, vp, i, vp, vp, vp]),
+            "spd_attention_workspace_size": (sz, [i, i]),
+            "spd_attention": (i, [vp, i, vp, vp, vp, i, vp, i, i, i, i, vp, vp, sz, vp]),
             "spd_prefill_workspace_size": (sz, [vp, i, i]),
             "spd_prefill": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, sz, vp]),
             "spd_linear_workspace_size": (sz, [i, i]),
@@ -219,6 +222,20 @@ def spd_project_workspace_size(model: SpdModel, rows: int) -> int:
 def spd_project(model: SpdModel, vis, rows, out_rows, x, ws, stream=None):
     _check(lib().spd_project(model.handle, _p(vis), rows, _p(out_rows), _p(x), _p(ws),
                              ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def spd_attention_workspace_size(n_q: int, n_seqs: int) -> int:
+    return int(lib().spd_attention_workspace_size(n_q, n_seqs))
+
+
+def spd_attention(q, q_pos, q_cu, kv, cu_seqlens, n_heads, n_kv_heads, head_dim, o, ws, stream=None):
+    """Causal attention of the query rows q (positions q_pos, sequences delimited by the host
+    array q_cu) over the K/V rows kv of their sequences (host cu_seqlens); writes o."""
+    q_cu = np.ascontiguousarray(q_cu, dtype=np.int32)
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    _check(lib().spd_attention(_p(q), int(q_cu[-1]), _p(q_pos), _p(q_cu), _p(kv), int(cu[-1]), _p(cu),
+                               len(cu) - 1, n_heads, n_kv_heads, head_dim, _p(o), _p(ws),
+                               ws.numel() * ws.element_size(), _stream(stream)))
 
 
 def spd_scatter_rows(model: SpdModel, src, rows, rows_map, dst, stream=None):

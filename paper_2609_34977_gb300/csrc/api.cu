@@ -6,6 +6,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
 #include <mutex>
 #include <vector>
 
@@ -14,9 +15,6 @@
 
 namespace spd {
 
-int attention_run(const void* q, int ldq, const void* kv, int ldkv, int v_off, void* o, int ldo,
-                  const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads,
-                  int head_dim, cudaStream_t stream, double ctx_sum, int n_q, int n_kv_rows);
 int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float eps,
                 const int32_t* in_rows, void* out, const int32_t* map2, void* out2,
                 cudaStream_t stream);
@@ -458,6 +456,46 @@ extern "C" int spd_scatter_rows(const spd_model* m, const uint16_t* src, int row
   return scatter_rows_run(src, rows, m->cfg.d_model, rows_map, dst, static_cast<cudaStream_t>(stream));
 }
 
+// ---- attention on its own ---------------------------------------------------------------------
+namespace {
+size_t attention_tiles(int n_q, int n_seqs) { return size_t(n_q) / kAttnTileQ + n_seqs + 1; }
+}  // namespace
+
+extern "C" size_t spd_attention_workspace_size(int n_q, int n_seqs) {
+  if (n_q < 1 || n_seqs < 1) return 0;
+  Carve cv(nullptr, ~size_t(0));
+  cv.take<int4>(attention_tiles(n_q, n_seqs));
+  return cv.used;
+}
+
+extern "C" int spd_attention(const uint16_t* q, int n_q, const int32_t* q_pos, const int32_t* q_cu,
+                             const uint16_t* kv, int n_kv, const int32_t* cu, int B, int n_heads,
+                             int n_kv_heads, int head_dim, uint16_t* o, void* ws, size_t ws_bytes,
+                             void* stream) {
+  if (!q || !q_pos || !q_cu || !kv || !cu || !o || !ws || n_q < 1 || n_kv < 1 || B < 1 ||
+      n_heads < 1 || n_kv_heads < 1 || n_heads % n_kv_heads)
+    return fail(SPD_EINVAL, "bad attention arguments");
+  if (q_cu[0] != 0 || q_cu[B] != n_q || cu[0] != 0 || cu[B] != n_kv)
+    return fail(SPD_EINVAL, "q_cu and cu_seqlens must run from 0 to n_q and n_kv");
+  for (int b = 0; b < B; ++b)
+    if (q_cu[b + 1] < q_cu[b] || cu[b + 1] <= cu[b] || q_cu[b + 1] - q_cu[b] > cu[b + 1] - cu[b])
+      return fail(SPD_EINVAL, "sequence %d: empty, decreasing, or more queries than tokens", b);
+  Carve cv(ws, ws_bytes);
+  int4* tiles = cv.take<int4>(attention_tiles(n_q, B));
+  if (!cv.fits()) return fail(SPD_ENOSPC, "attention workspace too small");
+  std::vector<int4> ht;
+  for (int b = 0; b < B; ++b)
+    for (int s0 = q_cu[b]; s0 < q_cu[b + 1]; s0 += kAttnTileQ)
+      ht.push_back(make_int4(s0, std::min(kAttnTileQ, q_cu[b + 1] - s0), cu[b], cu[b + 1] - cu[b]));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SPD_CUDA_TRY(cudaMemcpyAsync(tiles, ht.data(), ht.size() * sizeof(int4), cudaMemcpyHostToDevice, st));
+  const int kvd = n_kv_heads * head_dim;
+  double ctx = 0.0;  // for the trace only: an upper bound (every key of the sequence)
+  for (int b = 0; b < B; ++b) ctx += double(q_cu[b + 1] - q_cu[b]) * (cu[b + 1] - cu[b]);
+  return attention_run(q, n_q, kv, n_kv, 2 * kvd, kvd, o, n_heads * head_dim, tiles, int(ht.size()),
+                       q_pos, n_heads, n_kv_heads, head_dim, cv.status(), st, ctx);
+}
+
 // ---- prefill executor ------------------------------------------------------------------------
 namespace {
 
@@ -559,15 +597,15 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
       }
       if (!(bits & 2)) hl[q.frows + q.nf++] = t;
     }
-    // attention tiles: 64 active queries of one sequence each
+    // attention tiles: up to kAttnTileQ active queries of one sequence each
     int a = 0;
     for (int b = 0; b < B; ++b) {
       int a_end = a;
       while (a_end < q.na && seq_of[hl[q.arows + a_end]] == b) ++a_end;
-      for (int s0 = a; s0 < a_end; s0 += 64) {
+      for (int s0 = a; s0 < a_end; s0 += kAttnTileQ) {
         int32_t* tl = &hl[q.tiles + 4 * size_t(q.ntiles++)];
         tl[0] = s0;
-        tl[1] = (a_end - s0 < 64) ? a_end - s0 : 64;
+        tl[1] = (a_end - s0 < kAttnTileQ) ? a_end - s0 : kAttnTileQ;
         tl[2] = cu[b];
         tl[3] = cu[b + 1] - cu[b];
       }
@@ -621,9 +659,9 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
       break;
     }
     if (q.na > 0) {
-      if ((rc = attention_run(bf.q, qd, bf.kv, 2 * kvd, kvd, bf.o, qd,
+      if ((rc = attention_run(bf.q, q.na, bf.kv, T, 2 * kvd, kvd, bf.o, qd,
                               reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
-                              c.n_heads, c.n_kv_heads, hd, st, q.ctx, q.na, T)))
+                              c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx)))
         break;
       GemmProblem op{};
       op.map_w = &W.m_o;

@@ -1,12 +1,19 @@
-// Variable-length causal attention over packed sequences, queries restricted to the
-// attention-active tokens (VSkip-Attn, Sec. 3.2: a skipped token is not a query, but it still
-// serves as a key and a value for every other token of its sequence).
+// Variable-length causal attention over packed sequences on the tcgen05 tensor cores, queries
+// restricted to the attention-active tokens (VSkip-Attn, Sec. 3.2: a skipped token is not a
+// query, but it stays a key and a value for every other token of its sequence).
 //
-// One CTA = 64 active queries of one sequence x one head. Four warps own 16 query rows each.
-// K/V blocks of 64 keys stream through shared memory (cp.async double buffer). Scores use
-// bf16 mma.sync with fp32 accumulation. The softmax is online, in fp32 with exp2, and P is
-// rounded to bf16 for the PV product. A query at position p sees keys 0..p of its own sequence.
+// One CTA = up to 128 active queries of one sequence x one head (the MMA's M = 128 rows):
+//   warp 4     TMA producer: the Q tile once, then blocks of 128 keys of K and V into a two-stage
+//              ring (128-byte swizzle, boxes of 64 head-dim columns)
+//   warp 5     MMA issuer: S = Q K^T into TMEM (kind::f16, fp32), then O += P V with P from shared
+//              memory and V read in place as an MN-major operand (the layout its TMA box has)
+//   warps 0-3  softmax: thread r owns query row r (TMEM lane r); online softmax in fp32 with exp2;
+//              P rounded to bf16 into shared memory as a K-major swizzled operand; O rescaled in
+//              TMEM when a row's running maximum grows; at the end O / l goes to HBM in bf16
+// S of block j + 1 is computed while the softmax of block j runs. A query at position p sees keys
+// 0..p of its own sequence. Every wait is bounded (status SPD_ETIMEOUT, no hang).
 #include <cuda_bf16.h>
+#include <math.h>
 #include <stdint.h>
 
 #include "internal.h"
@@ -16,242 +23,303 @@
 namespace spd {
 namespace {
 
-constexpr int kQ = 64;   // queries per CTA
-constexpr int kKB = 64;  // keys per block
+constexpr int kTK = 128;              // keys per block (S columns, K of the PV product)
+constexpr uint32_t kBox = 128 * 128;  // one TMA box: 128 rows x 64 bf16
+constexpr int kThreads = 192;
 
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
-                   static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
-               "l"(gmem)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))));
-}
-__device__ __forceinline__ void mma16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
+template <int HD>
+struct AttnSmem {
+  static constexpr int kChunks = HD / 64;                       // 64-column boxes per row
+  static constexpr uint32_t q = 0;                              // Q tile
+  static constexpr uint32_t k = q + kChunks * kBox;             // K stages
+  static constexpr uint32_t v = k + 2 * kChunks * kBox;         // V stages
+  static constexpr uint32_t p = v + 2 * kChunks * kBox;         // P: two 64-key halves
+  static constexpr uint32_t bars = p + 2 * kBox;
+  static constexpr uint32_t bytes = bars + 128 + 1024;          // + alignment slack
+};
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
 template <int HD>
-__global__ void __launch_bounds__(128)
-    attn_kernel(const __nv_bfloat16* __restrict__ q, int ldq, const __nv_bfloat16* __restrict__ kv,
-                int ldkv, int v_off, __nv_bfloat16* __restrict__ o, int ldo,
-                const int4* __restrict__ tiles, const int32_t* __restrict__ q_pos, int n_heads,
-                int n_kv_heads, float scale_log2) {
-  constexpr int LD = HD + 8;  // padded row (elements): conflict-free ldmatrix
-  extern __shared__ __align__(16) uint8_t smem_raw[];
-  __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem_raw);
-  __nv_bfloat16* Ks = Qs + kQ * LD;
-  __nv_bfloat16* Vs = Ks + 2 * kKB * LD;
-  int* pos_s = reinterpret_cast<int*>(Vs + 2 * kKB * LD);
-  pdl_launch_dependents();
-  pdl_wait();
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
+                   const __grid_constant__ CUtensorMap map_kv, __nv_bfloat16* __restrict__ o,
+                   int ldo, const int4* __restrict__ tiles, const int32_t* __restrict__ q_pos,
+                   int n_heads, int n_kv_heads, int v_off, float scale_log2, int* status,
+                   long long budget) {
+  using L = AttnSmem<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + L::bars);
+  uint64_t* kv_full = q_full + 1;   // [2] K and V block landed
+  uint64_t* kv_empty = q_full + 3;  // [2] its PV product has completed
+  uint64_t* s_full = q_full + 5;    // S of the current block is in TMEM
+  uint64_t* s_free = q_full + 6;    // the softmax warps have read S
+  uint64_t* p_full = q_full + 7;    // P written and O rescaled
+  uint64_t* o_done = q_full + 8;    // PV product of the current block completed
+  uint64_t* drain = q_full + 9;     // every MMA completed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 10);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
-  const int4 tl = tiles[blockIdx.x];
-  const int q0 = tl.x, nq = tl.y, kv0 = tl.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
   const int hk = h / (n_heads / n_kv_heads);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int g = lane >> 2, t4 = lane & 3;
-
-  if (tid < kQ) pos_s[tid] = q_pos[q0 + min(tid, nq - 1)];
-  constexpr int CH = HD / 8;  // 16-byte chunks per row
-  for (int i = tid; i < kQ * CH; i += 128) {
-    const int r = i / CH, c = i % CH;
-    const int qr = q0 + min(r, nq - 1);
-    cp_async16(Qs + r * LD + c * 8, q + size_t(qr) * ldq + h * HD + c * 8);
-  }
-  cp_async_commit();
-  __syncthreads();
-  const int kmax = pos_s[kQ - 1 < nq - 1 ? kQ - 1 : nq - 1] + 1;  // positions ascend in a tile
-  const int nkb = (kmax + kKB - 1) / kKB;
-
-  auto load_kv = [&](int kb, int buf) {
-    __nv_bfloat16* ks = Ks + buf * kKB * LD;
-    __nv_bfloat16* vs = Vs + buf * kKB * LD;
-    for (int i = tid; i < kKB * CH; i += 128) {
-      const int r = i / CH, c = i % CH;
-      const int key = min(kb * kKB + r, kmax - 1);
-      const __nv_bfloat16* src = kv + size_t(kv0 + key) * ldkv + hk * HD + c * 8;
-      cp_async16(ks + r * LD + c * 8, src);
-      cp_async16(vs + r * LD + c * 8, src + v_off);
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
     }
-    cp_async_commit();
-  };
-  load_kv(0, 0);
-  cp_async_wait<1>();
+    mbar_init(s_full, 1);
+    mbar_init(s_free, 4);  // one arrival per softmax warp
+    mbar_init(p_full, 4);
+    mbar_init(o_done, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&map_q);
+    prefetch_tmap(&map_kv);
+  }
+  if (warp == 4) {
+    tmem_alloc(tmem_slot, 256);  // S: columns [0, 128); O: [128, 128 + HD)
+    tmem_relinquish();
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_s = tmem, t_o = tmem + 128;
 
-  uint32_t qa[HD / 16][4];
+  pdl_launch_dependents();
+  pdl_wait();  // Q, K and V come from the previous kernel
+  const int4 tl = tiles[blockIdx.x];
+  const int q0 = tl.x, nq = tl.y, kv0 = tl.z, len = tl.w;
+  const int p_last = q_pos[q0 + nq - 1];  // positions ascend within a tile
+  const int nkb = max(1, min((p_last + kTK) / kTK, (len + kTK - 1) / kTK));
+
+  int issued = 0;  // K/V blocks whose loads the producer issued
+  if (warp == 4) {
+    if (lane == 0) {
+      // ---- TMA producer ----
+      const uint64_t pol_q = policy_evict_first(), pol_kv = policy_evict_last();
+      mbar_arrive_expect_tx(q_full, L::kChunks * kBox);
+      for (int c = 0; c < L::kChunks; ++c)
+        tma_load_2d(smem + L::q + c * kBox, &map_q, q_full, h * HD + c * 64, q0, pol_q);
+      for (int j = 0; j < nkb; ++j) {
+        const int s = j & 1;
+        if (j >= 2 && !mbar_wait(&kv_empty[s], ((j >> 1) - 1) & 1, abort_flag, budget)) {
+          *abort_flag = 1;
+          set_status(status, SPD_ETIMEOUT);
+          break;
+        }
+        mbar_arrive_expect_tx(&kv_full[s], 2 * L::kChunks * kBox);
+        for (int c = 0; c < L::kChunks; ++c) {
+          const int x = hk * HD + c * 64, y = kv0 + j * kTK;
+          tma_load_2d(smem + L::k + (s * L::kChunks + c) * kBox, &map_kv, &kv_full[s], x, y, pol_kv);
+          tma_load_2d(smem + L::v + (s * L::kChunks + c) * kBox, &map_kv, &kv_full[s], v_off + x, y,
+                      pol_kv);
+        }
+        issued = j + 1;
+      }
+    }
+  } else if (warp == 5) {
+    if (lane == 0) {
+      // ---- MMA issuer ----
+      const uint32_t id_s = idesc_bf16_f32(128, kTK);
+      const uint32_t id_o = idesc_bf16_f32(128, HD) | (1u << 16);  // V is MN-major
+      const uint32_t sq = smem_u32(smem + L::q), sp = smem_u32(smem + L::p);
+      bool ok = mbar_wait(q_full, 0, abort_flag, budget);
+      auto issue_s = [&](int j) -> bool {
+        const int s = j & 1;
+        if (!mbar_wait(&kv_full[s], (j >> 1) & 1, abort_flag, budget)) return false;
+        if (j > 0 && !mbar_wait(s_free, (j - 1) & 1, abort_flag, budget)) return false;
+        tc_fence_after();
+        const uint32_t sk = smem_u32(smem + L::k + s * L::kChunks * kBox);
 #pragma unroll
-  for (int ks = 0; ks < HD / 16; ++ks)
-    ldsm_x4(qa[ks], Qs + (warp * 16 + (lane & 15)) * LD + ks * 16 + 8 * (lane >> 4));
-
-  const int p0 = pos_s[warp * 16 + g], p1 = pos_s[warp * 16 + g + 8];
-  float oacc[HD / 8][4];
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
+          mma_bf16(t_s, sdesc_k128(sq + off), sdesc_k128(sk + off), id_s, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(s_full);
+        return true;
+      };
+      if (ok) ok = issue_s(0);
+      for (int j = 0; j < nkb && ok; ++j) {
+        if (j + 1 < nkb && !(ok = issue_s(j + 1))) break;
+        if (!(ok = mbar_wait(p_full, j & 1, abort_flag, budget))) break;
+        tc_fence_after();
+        const uint32_t sv = smem_u32(smem + L::v + (j & 1) * L::kChunks * kBox);
 #pragma unroll
-  for (int i = 0; i < HD / 8; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.0f;
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.0f, l1 = 0.0f;
-
-  for (int kb = 0; kb < nkb; ++kb) {
-    const int buf = kb & 1;
-    if (kb + 1 < nkb) {
-      load_kv(kb + 1, buf ^ 1);
-      cp_async_wait<1>();
+        for (int kk = 0; kk < kTK / 16; ++kk) {
+          const uint64_t ad = sdesc_k128(sp + (kk >> 2) * kBox + (kk & 3) * 32);
+          const uint64_t bd = sdesc_mn128(sv + kk * 2048, kBox);
+          mma_bf16(t_o, ad, bd, id_o, (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        mma_commit(o_done);
+        mma_commit(&kv_empty[j & 1]);
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        set_status(status, SPD_ETIMEOUT);
+      }
+      mma_commit(drain);  // arrives once every MMA issued above has completed
+      volatile int no_abort = 0;
+      if (!mbar_wait(drain, 0, &no_abort, budget)) set_status(status, SPD_ETIMEOUT);
+    }
+  } else {
+    // ---- softmax and epilogue: warp w reads TMEM lanes [32 w, 32 w + 32) ----
+    const int r = warp * 32 + lane;  // query row of the tile
+    const int my_pos = q_pos[q0 + min(r, nq - 1)];
+    const uint32_t lanes = static_cast<uint32_t>(warp * 32) << 16;
+    uint8_t* prow = smem + L::p + r * 128;
+    float m_run = -INFINITY, l_run = 0.0f;
+    bool ok = true;
+    for (int j = 0; j < nkb; ++j) {
+      if (!(ok = __all_sync(0xffffffffu, mbar_wait(s_full, j & 1, abort_flag, budget)))) break;
+      tc_fence_after();
+      float s[kTK];
+#pragma unroll
+      for (int c = 0; c < kTK / 32; ++c) {
+        float v[32];
+        tmem_ld32(t_s + lanes + c * 32, v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) s[c * 32 + i] = v[i];
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(s_free);
+      const int kb = j * kTK;
+      float mx = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < kTK; ++i) {
+        s[i] = (kb + i <= my_pos) ? s[i] * scale_log2 : -INFINITY;
+        mx = fmaxf(mx, s[i]);
+      }
+      const float m_new = fmaxf(m_run, mx);  // finite: block 0 holds key 0 <= every position
+      const float corr = exp2f(m_run - m_new);  // 0 on the first block
+      float rs = 0.0f;
+#pragma unroll
+      for (int i = 0; i < kTK; ++i) {
+        s[i] = exp2f(s[i] - m_new);
+        rs += s[i];
+      }
+      l_run = l_run * corr + rs;
+      m_run = m_new;
+      if (j > 0) {
+        // the previous PV product has completed: P's buffer is free and O can be rescaled
+        if (!(ok = __all_sync(0xffffffffu, mbar_wait(o_done, (j - 1) & 1, abort_flag, budget))))
+          break;
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, corr != 1.0f)) {
+#pragma unroll 1
+          for (int c = 0; c < HD / 32; ++c) {
+            float v[32];
+            tmem_ld32(t_o + lanes + c * 32, v);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= corr;
+            tmem_st32(t_o + lanes + c * 32, v);
+          }
+        }
+      }
+      // P in bf16: row r of a K-major operand in the 128-byte swizzle layout (16-byte unit u of
+      // the row at position u ^ (r % 8)), keys [0, 64) and [64, 128) in two boxes
+#pragma unroll
+      for (int u = 0; u < kTK / 8; ++u) {
+        const uint4 w = make_uint4(pack_bf16(s[8 * u], s[8 * u + 1]), pack_bf16(s[8 * u + 2], s[8 * u + 3]),
+                                   pack_bf16(s[8 * u + 4], s[8 * u + 5]),
+                                   pack_bf16(s[8 * u + 6], s[8 * u + 7]));
+        *reinterpret_cast<uint4*>(prow + (u >> 3) * kBox + (((u & 7) ^ (r & 7)) << 4)) = w;
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+    }
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_done, (nkb - 1) & 1, abort_flag, budget));
+    if (!ok) {
+      *abort_flag = 1;
+      set_status(status, SPD_ETIMEOUT);
     } else {
-      cp_async_wait<0>();
-    }
-    __syncthreads();
-    const __nv_bfloat16* ks = Ks + buf * kKB * LD;
-    const __nv_bfloat16* vs = Vs + buf * kKB * LD;
-
-    float s[kKB / 8][4];
+      tc_fence_after();
+      const float inv = 1.0f / l_run;
+      __nv_bfloat16* orow = o + size_t(q0 + r) * ldo + h * HD;
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        float v[32];
+        tmem_ld32(t_o + lanes + c * 32, v);
+        if (r < nq) {
 #pragma unroll
-    for (int nt = 0; nt < kKB / 8; ++nt) {
-      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.0f;
-#pragma unroll
-      for (int ks2 = 0; ks2 < HD / 16; ks2 += 2) {
-        uint32_t b[4];
-        ldsm_x4(b, ks + (nt * 8 + (lane & 7)) * LD + ks2 * 16 + 8 * (lane >> 3));
-        mma16816(s[nt], qa[ks2], b[0], b[1]);
-        mma16816(s[nt], qa[ks2 + 1], b[2], b[3]);
+          for (int u = 0; u < 4; ++u)
+            reinterpret_cast<uint4*>(orow + c * 32)[u] =
+                make_uint4(pack_bf16(v[8 * u] * inv, v[8 * u + 1] * inv),
+                           pack_bf16(v[8 * u + 2] * inv, v[8 * u + 3] * inv),
+                           pack_bf16(v[8 * u + 4] * inv, v[8 * u + 5] * inv),
+                           pack_bf16(v[8 * u + 6] * inv, v[8 * u + 7] * inv));
+        }
       }
     }
-    float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-    for (int nt = 0; nt < kKB / 8; ++nt) {
-      const int key = kb * kKB + nt * 8 + 2 * t4;
-      s[nt][0] = (key <= p0) ? s[nt][0] * scale_log2 : -INFINITY;
-      s[nt][1] = (key + 1 <= p0) ? s[nt][1] * scale_log2 : -INFINITY;
-      s[nt][2] = (key <= p1) ? s[nt][2] * scale_log2 : -INFINITY;
-      s[nt][3] = (key + 1 <= p1) ? s[nt][3] * scale_log2 : -INFINITY;
-      mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
-      mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
-    }
-#pragma unroll
-    for (int off = 1; off <= 2; off <<= 1) {
-      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
-      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
-    }
-    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-    const float c0 = exp2f(m0 - mn0), c1 = exp2f(m1 - mn1);  // 0 on the first block (m = -inf)
-    m0 = mn0;
-    m1 = mn1;
-    float rs0 = 0.0f, rs1 = 0.0f;
-#pragma unroll
-    for (int nt = 0; nt < kKB / 8; ++nt) {
-      s[nt][0] = exp2f(s[nt][0] - mn0);
-      s[nt][1] = exp2f(s[nt][1] - mn0);
-      s[nt][2] = exp2f(s[nt][2] - mn1);
-      s[nt][3] = exp2f(s[nt][3] - mn1);
-      rs0 += s[nt][0] + s[nt][1];
-      rs1 += s[nt][2] + s[nt][3];
-    }
-    l0 = l0 * c0 + rs0;
-    l1 = l1 * c1 + rs1;
-#pragma unroll
-    for (int i = 0; i < HD / 8; ++i) {
-      oacc[i][0] *= c0;
-      oacc[i][1] *= c0;
-      oacc[i][2] *= c1;
-      oacc[i][3] *= c1;
-    }
-#pragma unroll
-    for (int kc = 0; kc < kKB / 16; ++kc) {
-      uint32_t pa[4];
-      pa[0] = pack_bf16(s[2 * kc][0], s[2 * kc][1]);
-      pa[1] = pack_bf16(s[2 * kc][2], s[2 * kc][3]);
-      pa[2] = pack_bf16(s[2 * kc + 1][0], s[2 * kc + 1][1]);
-      pa[3] = pack_bf16(s[2 * kc + 1][2], s[2 * kc + 1][3]);
-#pragma unroll
-      for (int nt2 = 0; nt2 < HD / 16; ++nt2) {
-        uint32_t b[4];
-        ldsm_x4_t(b, vs + (kc * 16 + (lane & 7) + 8 * ((lane >> 3) & 1)) * LD + nt2 * 16 +
-                         8 * (lane >> 4));
-        mma16816(oacc[2 * nt2], pa, b[0], b[1]);
-        mma16816(oacc[2 * nt2 + 1], pa, b[2], b[3]);
-      }
-    }
-    __syncthreads();  // buffer `buf` is refilled by the next iteration's prefetch
   }
-#pragma unroll
-  for (int off = 1; off <= 2; off <<= 1) {
-    l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 128 && *abort_flag) {
+    // loads issued but never consumed land before the CTA exits (without an abort the last PV
+    // product consumed every issued block)
+    volatile int no_abort = 0;
+    mbar_wait(q_full, 0, &no_abort, budget);
+    for (int j = max(0, issued - 2); j < issued; ++j)
+      mbar_wait(&kv_full[j & 1], (j >> 1) & 1, &no_abort, budget);
   }
-  const float i0 = 1.0f / l0, i1 = 1.0f / l1;
-  const int r0 = warp * 16 + g, r1 = r0 + 8;
-#pragma unroll
-  for (int nt = 0; nt < HD / 8; ++nt) {
-    const int col = h * HD + nt * 8 + 2 * t4;
-    if (r0 < nq)
-      *reinterpret_cast<uint32_t*>(o + size_t(q0 + r0) * ldo + col) =
-          pack_bf16(oacc[nt][0] * i0, oacc[nt][1] * i0);
-    if (r1 < nq)
-      *reinterpret_cast<uint32_t*>(o + size_t(q0 + r1) * ldo + col) =
-          pack_bf16(oacc[nt][2] * i1, oacc[nt][3] * i1);
-  }
+  __syncwarp();
+  tc_fence_after();
+  if (warp == 4) tmem_dealloc(tmem, 256);
 }
 
 template <int HD>
-int launch(const void* q, int ldq, const void* kv, int ldkv, int v_off, void* o, int ldo,
-           const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads,
+int launch(const CUtensorMap& mq, const CUtensorMap& mkv, void* o, int ldo, const int4* tiles,
+           int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads, int v_off, int* status,
            cudaStream_t stream) {
-  constexpr int LD = HD + 8;
-  const size_t smem = size_t(kQ + 4 * kKB) * LD * 2 + kQ * sizeof(int);
+  using L = AttnSmem<HD>;
   static bool attr = false;
   if (!attr) {
-    SPD_CUDA_TRY(cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      int(smem)));
+    SPD_CUDA_TRY(cudaFuncSetAttribute(attn_tc_kernel<HD>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, int(L::bytes)));
     attr = true;
   }
   const float scale_log2 = 1.4426950408889634f / sqrtf(float(HD));
-  SPD_CUDA_TRY(launch_pdl(attn_kernel<HD>, dim3(n_tiles, n_heads), dim3(128), smem, stream,
-                          static_cast<const __nv_bfloat16*>(q), ldq,
-                          static_cast<const __nv_bfloat16*>(kv), ldkv, v_off,
-                          static_cast<__nv_bfloat16*>(o), ldo, tiles, q_pos, n_heads, n_kv_heads,
-                          scale_log2));
+  SPD_CUDA_TRY(launch_pdl(attn_tc_kernel<HD>, dim3(n_tiles, n_heads), dim3(kThreads), L::bytes,
+                          stream, mq, mkv, static_cast<__nv_bfloat16*>(o), ldo, tiles, q_pos,
+                          n_heads, n_kv_heads, v_off, scale_log2, status, kWaitBudget));
   return SPD_OK;
 }
 
 }  // namespace
 
-int attention_run(const void* q, int ldq, const void* kv, int ldkv, int v_off, void* o, int ldo,
-                  const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads,
-                  int head_dim, cudaStream_t stream, double ctx_sum, int n_q, int n_kv_rows) {
+int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, int v_off, void* o,
+                  int ldo, const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads,
+                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum) {
   if (n_tiles <= 0) return SPD_OK;
   if (head_dim != 128 && head_dim != 64)
     return fail(SPD_EUNSUPPORTED, "attention supports head_dim 64 and 128");
+  if (n_kv_heads < 1 || n_heads % n_kv_heads)
+    return fail(SPD_EINVAL, "n_heads must be a multiple of n_kv_heads");
+  if (v_off % 64 || ldkv < v_off + n_kv_heads * head_dim)
+    return fail(SPD_EINVAL, "V must start at a multiple of 64 columns inside each K/V row");
+  CUtensorMap mq, mkv;
+  if (int rc = make_operand_map(&mq, q, n_heads * head_dim, n_q, 128)) return rc;
+  if (int rc = make_operand_map(&mkv, kv, ldkv, n_kv, kTK)) return rc;
   const int slot = trace_begin(stream);
   const int rc = (head_dim == 128)
-                     ? launch<128>(q, ldq, kv, ldkv, v_off, o, ldo, tiles, n_tiles, q_pos, n_heads,
-                                   n_kv_heads, stream)
-                     : launch<64>(q, ldq, kv, ldkv, v_off, o, ldo, tiles, n_tiles, q_pos, n_heads,
-                                  n_kv_heads, stream);
+                     ? launch<128>(mq, mkv, o, ldo, tiles, n_tiles, q_pos, n_heads, n_kv_heads,
+                                   v_off, status, stream)
+                     : launch<64>(mq, mkv, o, ldo, tiles, n_tiles, q_pos, n_heads, n_kv_heads,
+                                  v_off, status, stream);
   // QK^T and PV over each active query's causal context; Q, K, V read once and O written once
   trace_end(slot, stream, TR_ATTN, 4.0 * head_dim * n_heads * ctx_sum,
-            2.0 * (2.0 * n_q * n_heads * head_dim + 2.0 * n_kv_rows * n_kv_heads * head_dim));
+            2.0 * (2.0 * n_q * n_heads * head_dim + 2.0 * n_kv * n_kv_heads * head_dim));
   return rc;
 }
 

@@ -922,6 +922,10 @@ int make_weight_map(CUtensorMap* map, const void* w, int n_out, int k) {
   return make_map(map, w, k, n_out, kBM);
 }
 
+int make_operand_map(CUtensorMap* map, const void* ptr, int inner, int outer, int box_outer) {
+  return make_map(map, ptr, inner, outer, box_outer);
+}
+
 namespace {
 
 using KernelFn = void (*)(CUtensorMap, CUtensorMap, KArgs);

@@ -106,6 +106,19 @@ struct GemmScratch {
 
 size_t gemm_scratch_bytes();                           // fixed-capacity scratch for any problem
 int make_weight_map(CUtensorMap* map, const void* w, int n_out, int k);
+// Tensor map of a dense bf16 matrix [outer][inner] (row stride inner elements) read in boxes of
+// 64 columns x box_outer rows with the 128-byte swizzle; rows past `outer` read as zeros.
+int make_operand_map(CUtensorMap* map, const void* ptr, int inner, int outer, int box_outer);
+
+// ---- attention (tcgen05) ---------------------------------------------------------------------
+// Causal attention of n_q active queries (q [n_q][n_heads * head_dim], rows grouped by sequence,
+// positions ascending within a sequence) over the keys and values of their sequences (kv
+// [n_kv][ldkv]: K of head g at column g * head_dim, V at v_off + g * head_dim). `tiles` (device
+// int4 [n_tiles]): first query row, query count (<= 128), first key row, sequence length.
+int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, int v_off, void* o,
+                  int ldo, const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads,
+                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum);
+constexpr int kAttnTileQ = 128;  // queries per attention tile
 int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream);
 
 }  // namespace spd

@@ -138,7 +138,22 @@ __device__ __forceinline__ uint64_t sdesc_k128(uint32_t saddr) {
   return d;
 }
 
+// Shared-memory matrix descriptor of an MN-major operand tile in the 128-byte swizzle layout TMA
+// writes for boxes whose rows are 64 bf16 along MN and one K index each: 8 consecutive K indices
+// form a 1024-byte atom (groups of 8 K indices 1024 bytes apart) and consecutive 64-element MN
+// blocks lie `lbo` bytes apart. A K slice of 16 starts at an atom boundary (2048-byte steps).
+__device__ __forceinline__ uint64_t sdesc_mn128(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);  // bits 0-13: start address >> 4
+  d |= static_cast<uint64_t>(lbo >> 4) << 16;           // bits 16-29: MN-block stride >> 4
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;          // bits 32-45: 8-K-group stride >> 4
+  d |= static_cast<uint64_t>(1) << 46;                  // bits 46-47: descriptor version 1
+  d |= static_cast<uint64_t>(2) << 61;                  // bits 61-63: 128-byte swizzle
+  return d;
+}
+
 // Instruction descriptor of tcgen05.mma kind::f16: bf16 A and B (both K-major), fp32 D.
+// (Bit 16 set: B is MN-major.)
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int m, int n) {
   return (1u << 4)                                    // D format: f32
          | (1u << 7)                                  // A format: bf16
@@ -219,6 +234,27 @@ __device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int j = 0; j < 8; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+// Stores 32 consecutive fp32 columns of this warp's 32 TMEM lanes (the layout of tmem_ld32) and
+// waits until the stores have completed.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]),
+      "f"(v[8]), "f"(v[9]), "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15]),
+      "f"(v[16]), "f"(v[17]), "f"(v[18]), "f"(v[19]), "f"(v[20]), "f"(v[21]), "f"(v[22]),
+      "f"(v[23]), "f"(v[24]), "f"(v[25]), "f"(v[26]), "f"(v[27]), "f"(v[28]), "f"(v[29]),
+      "f"(v[30]), "f"(v[31])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Makes this thread's generic-proxy shared-memory writes visible to the async proxy (TMA, MMA).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // ---- distributed shared memory (thread-block clusters) -------------------------------------
