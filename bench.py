@@ -137,6 +137,45 @@ def count_launches(pipe, mask, dense):
     return n
 
 
+def prune_batch(torch, N, synth, dev, steps, warmup, hbm, tiles=64, keep=64):
+    """Scoring + compaction at serving batch: MSV-Prune of `tiles` LLaVA tiles in one call plus the
+    gather of the kept rows to bf16 (the projector's input). Algorithmic bytes per tile: both tapped
+    layers' features and the attention row read once, the kept indices written, the kept rows read
+    and written in bf16. The features (2 x 4.7 MB per tile) exceed L2 at this batch."""
+    v = synth.vision_tiles(SEED + 7, tiles, N_PATCH, D_VIS, 2, H_VIS)
+    feats = [torch.from_numpy(f).to(dev) for f in v["feats"]]
+    attn = torch.from_numpy(v["attn"]).to(dev)
+    del v
+    cfg = N.prune_cfg(tiles, N_PATCH + 1, D_VIS, 2, 1, H_VIS, keep, has_cls=True, attn_form=0)
+    ws = torch.zeros(N.spd_prune_workspace_size(cfg), dtype=torch.uint8, device=dev)
+    idx = torch.empty((tiles, keep), dtype=torch.int32, device=dev)
+    out = torch.empty((tiles * keep, D_VIS), dtype=torch.bfloat16, device=dev)
+
+    def run():
+        N.spd_prune(cfg, feats, attn, idx, ws=ws)
+        N.spd_gather_rows_bf16(feats[1], tiles, N_PATCH + 1, D_VIS, 1, idx, keep, out, ws=ws)
+
+    for _ in range(warmup):
+        run()
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        run()
+    e.record()
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0, "device-side failure recorded"
+    us = 1000.0 * s.elapsed_time(e) / steps
+    per_tile = (2 * (N_PATCH + 1) * D_VIS * 4 + H_VIS * (N_PATCH + 1) * 4
+                + keep * (4 + D_VIS * 4 + D_VIS * 2))
+    gbs = tiles * per_tile / (us * 1e-6) / 1e9
+    return {"tiles": tiles, "keep_per_tile": keep, "us_per_call": us,
+            "tiles_per_s": tiles / (us * 1e-6), "GB/s": gbs, "hbm_frac": gbs / hbm,
+            "bytes_per_tile": per_tile,
+            "what": "spd_prune + spd_gather_rows_bf16 of 64 llava tiles (576 patches x 1024, "
+                    "layers 12/24, keep 64 per tile), features larger than L2"}
+
+
 def cpu_baseline_sample(keep, v, mask_fn, reps=1):
     """The oracle as it stands on the host cores: MSV-Prune of the tile, the projector, and 1- and
     2-layer decoder prefills of the same token count; the step time is extrapolated to 32 layers."""
@@ -313,6 +352,16 @@ def main():
                    "GB/s": c["bytes"] / max(c["ms"], 1e-9) / 1e6,
                    "TFLOP/s": c["flops"] / max(c["ms"], 1e-9) / 1e9} for k, c in cls.items()}
 
+    # the dense step's GEMMs (640 token rows, above the ridge) against the tensor roofline
+    timed(dense, None, a.steps, 1, trace=True)
+    dg = N.spd_trace_read(N.TRACE_GEMM)
+    N.spd_trace_enable(0)
+    dense_tfs = dg["flops"] / (dg["ms"] / 1000.0) / 1e12
+    dense_gemm = {"ms_per_step": dg["ms"] / a.steps, "TFLOP/s": dense_tfs,
+                  "tensor_frac_of_sustained": dense_tfs / tf_sust,
+                  "GB/s": dg["bytes"] / (dg["ms"] / 1000.0) / 1e9}
+    pb = prune_batch(torch, N, synth, dev, a.steps, a.warmup, hbm)
+
     # end to end through the public API: pinned host inputs -> device, step, logits -> host
     hf = [f.cpu().pin_memory() for f in feats]
     ha, ht = attn.cpu().pin_memory(), text.cpu().pin_memory()
@@ -353,7 +402,8 @@ def main():
                                **({} if L == 32 else {"profiling_only_layers": L})),
                 "dense": {"value": tokens / (ms_dense / 1000.0), "ms_per_step": ms_dense,
                           "decoder_tokens": dense.T, "speedup_spider_vs_dense": ms_dense / ms},
-                "roofline": roof, "kernels": kernels, "cpu_baseline": cpu,
+                "roofline": roof, "kernels": kernels, "dense_gemm": dense_gemm,
+                "prune_batch": pb, "cpu_baseline": cpu,
                 "e2e": {"value": tokens / (ms_e2e / 1000.0), "unit": "tokens/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": hl.numel() * 4,
                         "ms_per_step": ms_e2e},

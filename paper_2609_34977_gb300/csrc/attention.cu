@@ -94,12 +94,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   const uint32_t t_s = tmem, t_o = tmem + 128;
 
-  pdl_launch_dependents();
-  pdl_wait();  // Q, K and V come from the previous kernel
+  // the tile list and the positions are written before the stream's previous kernels ran (host
+  // copies), so they are read before the wait; Q, K and V come from the previous kernel
   const int4 tl = tiles[blockIdx.x];
   const int q0 = tl.x, nq = tl.y, kv0 = tl.z, len = tl.w;
   const int p_last = q_pos[q0 + nq - 1];  // positions ascend within a tile
   const int nkb = max(1, min((p_last + kTK) / kTK, (len + kTK - 1) / kTK));
+  const int my_pos = threadIdx.x < 128 ? q_pos[q0 + min(int(threadIdx.x), nq - 1)] : 0;
+  pdl_launch_dependents();
+  pdl_wait();
 
   int issued = 0;  // K/V blocks whose loads the producer issued
   if (warp == 4) {
@@ -173,7 +176,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ---- softmax and epilogue: warp w reads TMEM lanes [32 w, 32 w + 32) ----
     const int r = warp * 32 + lane;  // query row of the tile
-    const int my_pos = q_pos[q0 + min(r, nq - 1)];
     const uint32_t lanes = static_cast<uint32_t>(warp * 32) << 16;
     uint8_t* prow = smem + L::p + r * 128;
     float m_run = -INFINITY, l_run = 0.0f;
@@ -193,20 +195,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(s_free);
       const int kb = j * kTK;
-      float mx = -INFINITY;
+      // eight independent max / sum chains (one warp per sub-partition: latency, not throughput)
+      float mx8[8], rs8[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) mx8[c] = -INFINITY;
 #pragma unroll
       for (int i = 0; i < kTK; ++i) {
         s[i] = (kb + i <= my_pos) ? s[i] * scale_log2 : -INFINITY;
-        mx = fmaxf(mx, s[i]);
+        mx8[i & 7] = fmaxf(mx8[i & 7], s[i]);
       }
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
       const float m_new = fmaxf(m_run, mx);  // finite: block 0 holds key 0 <= every position
       const float corr = exp2f(m_run - m_new);  // 0 on the first block
-      float rs = 0.0f;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) rs8[c] = 0.0f;
 #pragma unroll
       for (int i = 0; i < kTK; ++i) {
         s[i] = exp2f(s[i] - m_new);
-        rs += s[i];
+        rs8[i & 7] += s[i];
       }
+      const float rs = ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
       l_run = l_run * corr + rs;
       m_run = m_new;
       if (j > 0) {
