@@ -7,9 +7,11 @@
 //                the feature dimension split over a cluster of 4 CTAs whose partial tiles are summed
 //                in rank order through distributed shared memory; max via atomicMax on
 //                order-preserving integer keys (exact, order independent)
-//   kmeans       one thread-block cluster of 8 CTAs per tile, each owning a contiguous slice of the
-//                non-anchor tokens: Lloyd on raw F^L (assignment in each CTA, per-CTA sums in token
-//                order, cross-CTA sums in rank order through distributed shared memory), then the
+//   kmeans       one thread-block cluster of 16 CTAs per tile, each owning a contiguous slice of the
+//                non-anchor tokens whose F^L rows it keeps in shared memory for every iteration (8
+//                CTAs re-reading them from L2 where they do not fit): Lloyd on raw F^L (assignment
+//                in each CTA, per-CTA sums in token order, cross-CTA sums in rank order through
+//                distributed shared memory), then the
 //                per-cluster, per-layer sums of unit feature rows, the sums of a_j, sizes and Eq. 2
 //                quotas
 //   scores       s_i = [sum_l w_l f_i . (S_l,k - f_i)] / (|C_k| - 1) + a_i + (A_k - a_i) / (|C_k| - 1),
@@ -22,6 +24,8 @@
 #include <stdint.h>
 
 #include <cooperative_groups.h>
+
+#include <mutex>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -341,51 +345,98 @@ __device__ void compute_quotas(const int* sizes, int K, int n_cmp, int* quota) {
   }
 }
 
-constexpr int kKC = 8;  // CTAs per tile in the K-means cluster
+// part[k][c] = sum over this CTA's tokens jj of cluster k, in token order, of value(jj, c): one
+// thread per column, KN accumulators in registers, eight values in flight.
+template <int KN, typename F>
+__device__ __forceinline__ void column_sums(float* part, int K, int D, int nl, const int8_t* asg,
+                                            F value) {
+  for (int c = threadIdx.x; c < D; c += blockDim.x) {
+    float acc[KN];
+#pragma unroll
+    for (int k = 0; k < KN; ++k) acc[k] = 0.0f;
+    for (int jb = 0; jb < nl; jb += 8) {
+      float xv[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) xv[u] = jb + u < nl ? value(jb + u, c) : 0.0f;
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (jb + u < nl) {
+          const int a = asg[jb + u];
+#pragma unroll
+          for (int k = 0; k < KN; ++k)
+            if (k == a) acc[k] += xv[u];
+        }
+    }
+#pragma unroll
+    for (int k = 0; k < KN; ++k)
+      if (k < K) part[k * D + c] = acc[k];
+  }
+}
 
-// Sums over the CTAs of the cluster, in rank order, of the per-CTA column sums `part` (K x D in
+// Sums over the KC CTAs of the cluster, in rank order, of the per-CTA column sums `part` (K x D in
 // every CTA's shared memory), for this CTA's slice of columns; `emit(k, c, value)` consumes them.
-template <typename F>
+template <int KC, typename F>
 __device__ __forceinline__ void cluster_column_reduce(cg::cluster_group& cl, float* part, int K, int D,
                                                       int rank, F emit) {
-  const int c0 = rank * D / kKC, c1 = (rank + 1) * D / kKC, width = c1 - c0;
+  const int c0 = rank * D / KC, c1 = (rank + 1) * D / KC, width = c1 - c0;
   for (int e = threadIdx.x; e < K * width; e += blockDim.x) {
     const int k = e / width, c = c0 + e % width;
-    float x[kKC];
+    float x[KC];
 #pragma unroll
-    for (int rr = 0; rr < kKC; ++rr) x[rr] = cl.map_shared_rank(part, rr)[k * D + c];  // in flight
+    for (int rr = 0; rr < KC; ++rr) x[rr] = cl.map_shared_rank(part, rr)[k * D + c];  // in flight
     float sum = 0.0f;
 #pragma unroll
-    for (int rr = 0; rr < kKC; ++rr) sum += x[rr];
+    for (int rr = 0; rr < KC; ++rr) sum += x[rr];
     emit(k, c, sum);
   }
 }
 
-__global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
-    kmeans_cluster_kernel(PruneDims p, PruneWs w) {
+// K-means over one tile per cluster of KC CTAs, CTA r owning the non-anchor tokens
+// [r m / KC, (r+1) m / KC). RES: those tokens' F^L rows are copied into the CTA's shared memory
+// once (one bulk copy per row) and every Lloyd iteration reads them there; otherwise each
+// iteration re-reads them from global memory (L2). KN: an upper bound of K known at compile time
+// (K itself for the paper's K = 4), sizing the per-thread accumulators.
+template <int KC, bool RES, int KN>
+__global__ void __launch_bounds__(512) kmeans_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
-  extern __shared__ float ksm[];
+  extern __shared__ __align__(16) float ksm[];
   const int K = p.K, D = p.d, m = p.m;
-  float* cent = ksm;                      // [K][D] centroids (same in every CTA)
-  float* part = ksm + size_t(K) * D;      // [K][D] this CTA's column sums
+  const int nl_max = (m + KC - 1) / KC;
+  float* rows = ksm;                                          // RES: [nl_max][D]
+  float* cent = ksm + (RES ? size_t(nl_max) * D : size_t(0));  // [K][D] centroids (every CTA)
+  float* part = cent + size_t(K) * D;                         // [K][D] this CTA's column sums
   __shared__ int cnt[SPD_MAX_CLUSTERS];   // this CTA's cluster sizes
   __shared__ float asum_part[SPD_MAX_CLUSTERS];
-  __shared__ int changed;
-  __shared__ int8_t asg[4096 / kKC + 1];
-  __shared__ int idx[4096 / kKC + 1];    // patch index of each of this CTA's tokens
-  __shared__ float av[4096 / kKC + 1];   // their a_j
+  __shared__ int changed;      // this CTA's assignment changed in the current iteration
+  __shared__ int any_changed;  // ... some CTA's of the cluster
+  __shared__ int8_t asg[4096 / KC + 1];
+  __shared__ int idx[4096 / KC + 1];     // patch index of each of this CTA's tokens
+  __shared__ float av[4096 / KC + 1];    // their a_j
+  __shared__ float rinv[4096 / KC + 1];  // their 1 / ||F_l,j|| for the layer being summed
   __shared__ int ncl[SPD_MAX_CLUSTERS];  // cluster sizes over the whole cluster of CTAs
+  __shared__ uint64_t rows_bar;
   cg::cluster_group cl = cg::this_cluster();
   const int rank = int(cl.block_rank());
   const int t = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nw = blockDim.x >> 5;
-  const int j0 = rank * m / kKC, j1 = (rank + 1) * m / kKC, nl = j1 - j0;
+  const int j0 = rank * m / KC, j1 = (rank + 1) * m / KC, nl = j1 - j0;
   const int* ul = w.ulist + size_t(t) * m;
   const size_t row0 = size_t(t) * p.n_tok + p.off;  // feature row of patch 0 of this tile
+  const float* fin = p.feat[p.fin];
   for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) {
     idx[jj] = ul[j0 + jj];
     av[jj] = ordered_val(w.asim[size_t(t) * p.n + ul[j0 + jj]]);
+  }
+  if (RES && threadIdx.x == 0) {
+    mbar_init(&rows_bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (RES && threadIdx.x == 0 && nl > 0) {
+    mbar_arrive_expect_tx(&rows_bar, uint32_t(nl) * D * 4);
+    for (int jj = 0; jj < nl; ++jj)
+      bulk_load(rows + size_t(jj) * D, fin + (row0 + idx[jj]) * D, uint32_t(D) * 4, &rows_bar);
   }
   if (m > 0) {
 #pragma unroll 4
@@ -394,17 +445,27 @@ __global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
       cent[e] = feat_row(p, p.fin, t, ul[(k * m) / K])[c];
     }
   }
+  if (RES && nl > 0) {
+    volatile int no_abort = 0;
+    if (!mbar_wait(&rows_bar, 0, &no_abort, kWaitBudget)) {
+      set_status(w.status, SPD_ETIMEOUT);
+      mbar_wait(&rows_bar, 0, &no_abort, kWaitBudget);  // the copies land before anything reuses it
+    }
+  }
   __syncthreads();
-  const float* fin = p.feat[p.fin];
+  // this CTA's token jj of the tile's non-anchor list, row of F^L
+  auto xrow = [&](int jj) -> const float* {
+    return RES ? rows + size_t(jj) * D : fin + (row0 + idx[jj]) * D;
+  };
   for (int it = 0; it < p.iters && m > 0; ++it) {
     // assignment of this CTA's points
     if (threadIdx.x == 0) changed = 0;
     __syncthreads();
     for (int jj = warp; jj < nl; jj += nw) {
-      const float* x = fin + (row0 + idx[jj]) * D;
-      float part_d[SPD_MAX_CLUSTERS];
+      const float* x = xrow(jj);
+      float part_d[KN];
 #pragma unroll
-      for (int k = 0; k < SPD_MAX_CLUSTERS; ++k) part_d[k] = 0.0f;
+      for (int k = 0; k < KN; ++k) part_d[k] = 0.0f;
       // 16-byte loads, four in flight per lane (D is a multiple of 4)
       for (int cb = 4 * lane; cb < D; cb += 512) {
         float4 xv[4];
@@ -418,7 +479,7 @@ __global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
           const int c = cb + 128 * u;
           if (c < D) {
 #pragma unroll
-            for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
+            for (int k = 0; k < KN; ++k)
               if (k < K) {
                 const float4 ce = *reinterpret_cast<const float4*>(cent + k * D + c);
                 const float d0 = xv[u].x - ce.x, d1 = xv[u].y - ce.y, d2 = xv[u].z - ce.z,
@@ -431,7 +492,7 @@ __global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
       int best = 0;
       float bd = 0.0f;
 #pragma unroll
-      for (int k = 0; k < SPD_MAX_CLUSTERS; ++k)
+      for (int k = 0; k < KN; ++k)
         if (k < K) {
           const float dk = warp_sum(part_d[k]);
           if (k == 0 || dk < bd) {
@@ -445,36 +506,31 @@ __global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
       }
     }
     __syncthreads();
-    // this CTA's column sums and sizes
+    // this CTA's column sums (token order, in registers) and sizes
     if (threadIdx.x < K) cnt[threadIdx.x] = 0;
-    for (int e = threadIdx.x; e < K * D; e += blockDim.x) part[e] = 0.0f;
     __syncthreads();
     for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) atomicAdd(&cnt[asg[jj]], 1);
-    for (int c = threadIdx.x; c < D; c += blockDim.x)
-      for (int jb = 0; jb < nl; jb += 8) {  // token order; eight loads in flight
-        float xv[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u)
-          xv[u] = jb + u < nl ? fin[(row0 + idx[jb + u]) * D + c] : 0.0f;
-#pragma unroll
-        for (int u = 0; u < 8; ++u)
-          if (jb + u < nl) part[asg[jb + u] * D + c] += xv[u];
-      }
+    column_sums<KN>(part, K, D, nl, asg, [&](int jj, int c) { return xrow(jj)[c]; });
     cl.sync();
-    int total_changed = 0;
-    for (int rr = 0; rr < kKC; ++rr) total_changed += *cl.map_shared_rank(&changed, rr);
-    if (it > 0 && total_changed == 0) break;  // cluster-uniform decision
-    // new centroids for this CTA's column slice, written into every CTA
-    if (threadIdx.x < K) {
-      int n = 0;
-      for (int rr = 0; rr < kKC; ++rr) n += cl.map_shared_rank(cnt, rr)[threadIdx.x];
-      ncl[threadIdx.x] = n;
+    // one warp reads the peers' flags and sizes (lane r: CTA r) and publishes them in this CTA
+    if (warp == 0) {
+      const int f = lane < KC ? *cl.map_shared_rank(&changed, lane) : 0;
+      const int any = __any_sync(0xffffffffu, f != 0);
+      for (int k = 0; k < K; ++k) {
+        int n = lane < KC ? cl.map_shared_rank(cnt, lane)[k] : 0;
+#pragma unroll
+        for (int off = 16; off; off >>= 1) n += __shfl_xor_sync(0xffffffffu, n, off);
+        if (lane == 0) ncl[k] = n;
+      }
+      if (lane == 0) any_changed = any;
     }
     __syncthreads();
-    cluster_column_reduce(cl, part, K, D, rank, [&](int k, int c, float sum) {
+    if (it > 0 && !any_changed) break;  // cluster-uniform decision
+    // new centroids for this CTA's column slice, written into every CTA
+    cluster_column_reduce<KC>(cl, part, K, D, rank, [&](int k, int c, float sum) {
       const int n = ncl[k];
       const float v = n > 0 ? sum / float(n) : cent[k * D + c];
-      for (int rr = 0; rr < kKC; ++rr) cl.map_shared_rank(cent, rr)[k * D + c] = v;
+      for (int rr = 0; rr < KC; ++rr) cl.map_shared_rank(cent, rr)[k * D + c] = v;
     });
     cl.sync();
   }
@@ -491,42 +547,58 @@ __global__ void __cluster_dims__(kKC, 1, 1) __launch_bounds__(512)
   if (threadIdx.x == 0)  // token order
     for (int jj = 0; jj < nl; ++jj) asum_part[asg[jj]] += av[jj];
   // per layer: sums over each cluster of unit feature rows (F_l,j / ||F_l,j||)
-  for (int l = 0; l < p.L; ++l) {
+  // (RES: the final layer first, from the resident rows; then each other layer's rows are copied
+  // into the same buffer)
+  for (int li = 0; li < p.L; ++li) {
+    const int l = RES ? (li == 0 ? p.fin : (li <= p.fin ? li - 1 : li)) : li;
     const float* inv = w.inv + (size_t(l) * p.n_tiles + t) * p.n;
-    __syncthreads();
-    for (int e = threadIdx.x; e < K * D; e += blockDim.x) part[e] = 0.0f;
-    __syncthreads();
     const float* fl = p.feat[l];
-    for (int c = threadIdx.x; c < D; c += blockDim.x)
-      for (int jb = 0; jb < nl; jb += 8) {  // token order; eight loads in flight
-        float xv[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int i = jb + u < nl ? idx[jb + u] : 0;
-          xv[u] = jb + u < nl ? fl[(row0 + i) * D + c] * inv[i] : 0.0f;
-        }
-#pragma unroll
-        for (int u = 0; u < 8; ++u)
-          if (jb + u < nl) part[asg[jb + u] * D + c] += xv[u];
+    __syncthreads();  // the previous layer's rows are no longer read
+    for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) rinv[jj] = inv[idx[jj]];
+    if (RES && l != p.fin && threadIdx.x == 0 && nl > 0) {
+      mbar_arrive_expect_tx(&rows_bar, uint32_t(nl) * D * 4);
+      for (int jj = 0; jj < nl; ++jj)
+        bulk_load(rows + size_t(jj) * D, fl + (row0 + idx[jj]) * D, uint32_t(D) * 4, &rows_bar);
+    }
+    if (RES && l != p.fin && nl > 0) {
+      volatile int no_abort = 0;
+      if (!mbar_wait(&rows_bar, li & 1, &no_abort, kWaitBudget)) {
+        set_status(w.status, SPD_ETIMEOUT);
+        mbar_wait(&rows_bar, li & 1, &no_abort, kWaitBudget);
       }
+    }
+    __syncthreads();
+    if (RES)
+      column_sums<KN>(part, K, D, nl, asg,
+                      [&](int jj, int c) { return rows[size_t(jj) * D + c] * rinv[jj]; });
+    else
+      column_sums<KN>(part, K, D, nl, asg,
+                      [&](int jj, int c) { return fl[(row0 + idx[jj]) * D + c] * rinv[jj]; });
     cl.sync();
     float* csum = w.csum + (size_t(t) * p.L + l) * K * D;
-    cluster_column_reduce(cl, part, K, D, rank, [&](int k, int c, float sum) { csum[k * D + c] = sum; });
-    if (l == p.L - 1 && rank == 0 && threadIdx.x == 0) {
+    cluster_column_reduce<KC>(cl, part, K, D, rank,
+                              [&](int k, int c, float sum) { csum[k * D + c] = sum; });
+    if (li == p.L - 1 && rank == 0 && warp == 0) {
+      // sizes and a_j sums over the CTAs (lane r reads CTA r; the a_j sums added in rank order)
       int sizes[SPD_MAX_CLUSTERS], q[SPD_MAX_CLUSTERS];
       for (int k = 0; k < K; ++k) {
-        int n = 0;
+        const int nr = lane < KC ? cl.map_shared_rank(cnt, lane)[k] : 0;
+        const float ar = lane < KC ? cl.map_shared_rank(asum_part, lane)[k] : 0.0f;
+        int n = nr;
+#pragma unroll
+        for (int off = 16; off; off >>= 1) n += __shfl_xor_sync(0xffffffffu, n, off);
         float a = 0.0f;
-        for (int rr = 0; rr < kKC; ++rr) {
-          n += cl.map_shared_rank(cnt, rr)[k];
-          a += cl.map_shared_rank(asum_part, rr)[k];
-        }
+        for (int rr = 0; rr < KC; ++rr) a += __shfl_sync(0xffffffffu, ar, rr);
         sizes[k] = n;
-        w.counts[t * 16 + k] = n;
-        w.asum[t * 16 + k] = a;
+        if (lane == 0) {
+          w.counts[t * 16 + k] = n;
+          w.asum[t * 16 + k] = a;
+        }
       }
-      compute_quotas(sizes, K, p.n_cmp, q);
-      for (int k = 0; k < K; ++k) w.quotas[t * 16 + k] = q[k];
+      if (lane == 0) {
+        compute_quotas(sizes, K, p.n_cmp, q);
+        for (int k = 0; k < K; ++k) w.quotas[t * 16 + k] = q[k];
+      }
     }
     cl.sync();  // peers' shared memory is read above; keep it alive and unchanged until here
   }
@@ -713,6 +785,72 @@ PruneWs carve(const PruneDims& p, Carve& cv) {
   return w;
 }
 
+constexpr size_t kResSmem = 200 * 1024;  // dynamic shared memory of the resident K-means
+int g_res_clusters = -1;                 // 16-CTA clusters of it the GPU holds at once
+
+template <int KC, bool RES, int KN>
+cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, size_t smem, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(KC, p.n_tiles);
+  cfg.blockDim = dim3(512);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = KC;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kmeans_kernel<KC, RES, KN>, p, w);
+}
+
+// Kernel attributes (once per process) and whether 16-CTA clusters of the resident kernel fit.
+int kmeans_setup() {
+  static std::once_flag once;
+  static cudaError_t err = cudaSuccess;
+  std::call_once(once, [] {
+    auto streamed = [](auto kern) {
+      return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * 24576 * 4);
+    };
+    auto resident = [](auto kern) {
+      cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kResSmem));
+      return e;
+    };
+    err = streamed(kmeans_kernel<8, false, 4>);
+    if (err == cudaSuccess) err = streamed(kmeans_kernel<8, false, SPD_MAX_CLUSTERS>);
+    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, 4>);
+    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, SPD_MAX_CLUSTERS>);
+    g_res_clusters = 0;
+    if (err == cudaSuccess) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(16);
+      cfg.blockDim = dim3(512);
+      cfg.dynamicSmemBytes = kResSmem;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 16;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, kmeans_kernel<16, true, SPD_MAX_CLUSTERS>, &cfg) !=
+          cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+      }
+      g_res_clusters = n;
+    }
+  });
+  if (err != cudaSuccess) return fail(SPD_ECUDA, "K-means attributes: %s", cudaGetErrorString(err));
+  return SPD_OK;
+}
+
 }  // namespace
 }  // namespace spd
 
@@ -749,14 +887,20 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
     SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel,
                             dim3((p.m + 63) / 64 * kAS, (p.n_anc + 63) / 64, T), dim3(256), 0, st,
                             p, w));
-  const size_t ksmem = size_t(2) * p.K * p.d * sizeof(float);
-  static bool attr = false;
-  if (!attr) {
-    SPD_CUDA_TRY(cudaFuncSetAttribute(kmeans_cluster_kernel,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * 24576 * 4));
-    attr = true;
-  }
-  SPD_CUDA_TRY(launch_pdl(kmeans_cluster_kernel, dim3(kKC, T), dim3(512), ksmem, st, p, w));
+  // K-means: the rows resident in shared memory over 16 CTAs per tile where they fit, else
+  // re-read from L2 each iteration by 8 CTAs per tile
+  if (int rc = kmeans_setup()) return rc;
+  const size_t cent_bytes = size_t(2) * p.K * p.d * sizeof(float);
+  const size_t res_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float) + cent_bytes;
+  const bool res = p.m > 0 && res_bytes <= kResSmem && g_res_clusters > 0;
+  if (res && p.K == 4)
+    SPD_CUDA_TRY((launch_kmeans<16, true, 4>(p, w, res_bytes, st)));
+  else if (res)
+    SPD_CUDA_TRY((launch_kmeans<16, true, SPD_MAX_CLUSTERS>(p, w, res_bytes, st)));
+  else if (p.K == 4)
+    SPD_CUDA_TRY((launch_kmeans<8, false, 4>(p, w, cent_bytes, st)));
+  else
+    SPD_CUDA_TRY((launch_kmeans<8, false, SPD_MAX_CLUSTERS>(p, w, cent_bytes, st)));
   if (p.m > 0)
     SPD_CUDA_TRY(launch_pdl(score_kernel, dim3((p.m + 7) / 8, T), dim3(256), 0, st, p, w));
   SPD_CUDA_TRY(launch_pdl(select_kernel, dim3(T), dim3(1024), 0, st, p, w, keep_idx, kind, cluster,
