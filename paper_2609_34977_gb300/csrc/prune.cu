@@ -92,6 +92,27 @@ __device__ void bitonic_sort(uint64_t* keys, int N) {
   }
 }
 
+// Position of every key in the ascending order of keys[0..N) (distinct keys): the number of smaller
+// keys, counted by each thread for its keys (broadcast shared-memory reads, no barriers). rank_of
+// is called with (i, rank) for i < N.
+template <typename F>
+__device__ __forceinline__ void rank_keys(const uint64_t* keys, int N, F rank_of) {
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    const uint64_t ki = keys[i];
+    int r0 = 0, r1 = 0, r2 = 0, r3 = 0;
+    int j = 0;
+    for (; j + 4 <= N; j += 4) {
+      r0 += keys[j] < ki;
+      r1 += keys[j + 1] < ki;
+      r2 += keys[j + 2] < ki;
+      r3 += keys[j + 3] < ki;
+    }
+    for (; j < N; ++j) r0 += keys[j] < ki;
+    rank_of(i, r0 + r1 + r2 + r3);
+  }
+}
+constexpr int kRankMax = 2048;  // longest list ranked by counting; longer ones are sorted
+
 // Exclusive prefix sum of one int per thread over a block of 1024 threads.
 __device__ int block_scan_excl(int v, int* tmp, int* total) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -158,6 +179,7 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
   const int t = blockIdx.x;
   int N = 1;
   while (N < p.n) N <<= 1;
+  // (a_v descending, index ascending) as ascending 64-bit keys
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
     uint64_t k = ~0ull;
     if (i < p.n)
@@ -165,11 +187,16 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
     keys[i] = k;
   }
   __syncthreads();
-  bitonic_sort(keys, N);
   int8_t* role = w.role + size_t(t) * p.n;
-  for (int i = threadIdx.x; i < p.n; i += blockDim.x) role[i] = 0;
-  __syncthreads();
-  for (int r = threadIdx.x; r < p.n_anc; r += blockDim.x) role[keys[r] & 0xffffffffu] = 1;
+  if (p.n <= kRankMax) {
+    // anchor iff its key is among the n_anc smallest
+    rank_keys(keys, p.n, [&](int i, int r) { role[i] = r < p.n_anc ? 1 : 0; });
+  } else {
+    bitonic_sort(keys, N);
+    for (int i = threadIdx.x; i < p.n; i += blockDim.x) role[i] = 0;
+    __syncthreads();
+    for (int r = threadIdx.x; r < p.n_anc; r += blockDim.x) role[keys[r] & 0xffffffffu] = 1;
+  }
   __syncthreads();
   // stable lists: each thread owns 4 consecutive tokens
   const int base = threadIdx.x * 4;
@@ -623,15 +650,31 @@ __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
     for (int l = 0; l < p.L; ++l) {
       const float wl = (l == p.fin) ? 1.0f : p.w[l];
       if (wl == 0.0f) continue;
-      const float* x = feat_row(p, l, t, i);
+      const float4* x4 = reinterpret_cast<const float4*>(feat_row(p, l, t, i));
       const float iv = w.inv[(size_t(l) * p.n_tiles + t) * p.n + i];
-      const float* cs = w.csum + ((size_t(t) * p.L + l) * p.K + k) * p.d;
-      float dot = 0.0f;
-      for (int c = lane; c < p.d; c += 32) {
-        const float u = x[c] * iv;
-        dot += u * (cs[c] - u);
+      const float4* c4 =
+          reinterpret_cast<const float4*>(w.csum + ((size_t(t) * p.L + l) * p.K + k) * p.d);
+      // 16-byte loads, sixteen in flight per lane, two independent chains
+      const int d4 = p.d / 4;
+      float dot0 = 0.0f, dot1 = 0.0f;
+      for (int cb = lane; cb < d4; cb += 256) {
+        float4 xv[8], cv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int c = cb + 32 * u;
+          xv[u] = c < d4 ? x4[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+          cv[u] = c < d4 ? c4[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const float a0 = xv[u].x * iv, a1 = xv[u].y * iv, a2 = xv[u].z * iv, a3 = xv[u].w * iv;
+          const float part = a0 * (cv[u].x - a0) + a1 * (cv[u].y - a1) + a2 * (cv[u].z - a2) +
+                             a3 * (cv[u].w - a3);
+          if (u & 1) dot1 += part;
+          else dot0 += part;
+        }
       }
-      acc += wl * warp_sum(dot);
+      acc += wl * warp_sum(dot0 + dot1);
     }
     const float inv_c = 1.0f / float(cnt - 1);
     s = acc * inv_c + ai + (w.asum[t * 16 + k] - ai) * inv_c;
@@ -671,10 +714,18 @@ __global__ void __launch_bounds__(1024) select_kernel(PruneDims p, PruneWs w, in
     seg[p.K] = acc;
   }
   __syncthreads();
-  bitonic_sort(keys, N);
-  for (int r = threadIdx.x; r < m; r += blockDim.x) {
-    const int k = int(keys[r] >> 45);
-    if (r - seg[k] < quota[k]) kept[keys[r] & 0x1fffu] = 2;
+  if (m <= kRankMax) {
+    // the key at sorted position r of cluster k's segment is kept iff r - seg[k] < quota[k]
+    rank_keys(keys, m, [&](int j, int r) {
+      const int k = int(keys[j] >> 45);
+      if (r - seg[k] < quota[k]) kept[keys[j] & 0x1fffu] = 2;
+    });
+  } else {
+    bitonic_sort(keys, N);
+    for (int r = threadIdx.x; r < m; r += blockDim.x) {
+      const int k = int(keys[r] >> 45);
+      if (r - seg[k] < quota[k]) kept[keys[r] & 0x1fffu] = 2;
+    }
   }
   __syncthreads();
   const int base = threadIdx.x * 4;
