@@ -372,31 +372,91 @@ __device__ void compute_quotas(const int* sizes, int K, int n_cmp, int* quota) {
   }
 }
 
+// Row jj of this CTA's tokens: resident in shared memory (rows + jj D) or in global memory
+// (g + (row0 + idx[jj]) D), optionally scaled by scale[jj].
+struct RowAccess {
+  const float* rows;  // resident rows, or null
+  const float* g;
+  size_t row0;
+  const int* idx;
+  int D;
+  const float* scale;  // or null
+  __device__ __forceinline__ const float* row(int jj) const {
+    return rows ? rows + size_t(jj) * D : g + (row0 + idx[jj]) * D;
+  }
+  __device__ __forceinline__ float operator()(int jj, int c) const {
+    const float v = row(jj)[c];
+    return scale ? v * scale[jj] : v;
+  }
+  __device__ __forceinline__ float4 v4(int jj, int c) const {
+    float4 v = *reinterpret_cast<const float4*>(row(jj) + c);
+    if (scale) {
+      const float sc = scale[jj];
+      v.x *= sc;
+      v.y *= sc;
+      v.z *= sc;
+      v.w *= sc;
+    }
+    return v;
+  }
+};
+
 // part[k][c] = sum over this CTA's tokens jj of cluster k, in token order, of value(jj, c): one
 // thread per column, KN accumulators in registers, eight values in flight.
 template <int KN, typename F>
 __device__ __forceinline__ void column_sums(float* part, int K, int D, int nl, const int8_t* asg,
                                             F value) {
-  for (int c = threadIdx.x; c < D; c += blockDim.x) {
-    float acc[KN];
+  if constexpr (KN == 4) {
+    // four adjacent columns per thread (float4), same token-order sums per column
+    for (int c = 4 * threadIdx.x; c < D; c += 4 * blockDim.x) {
+      float4 acc[KN];
 #pragma unroll
-    for (int k = 0; k < KN; ++k) acc[k] = 0.0f;
-    for (int jb = 0; jb < nl; jb += 8) {
-      float xv[8];
+      for (int k = 0; k < KN; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int jb = 0; jb < nl; jb += 8) {
+        float4 xv[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) xv[u] = jb + u < nl ? value(jb + u, c) : 0.0f;
+        for (int u = 0; u < 8; ++u)
+          xv[u] = jb + u < nl ? value.v4(jb + u, c) : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
-        if (jb + u < nl) {
-          const int a = asg[jb + u];
+        for (int u = 0; u < 8; ++u)
+          if (jb + u < nl) {
+            const int a = asg[jb + u];
 #pragma unroll
-          for (int k = 0; k < KN; ++k)
-            if (k == a) acc[k] += xv[u];
-        }
+            for (int k = 0; k < KN; ++k)
+              if (k == a) {
+                acc[k].x += xv[u].x;
+                acc[k].y += xv[u].y;
+                acc[k].z += xv[u].z;
+                acc[k].w += xv[u].w;
+              }
+          }
+      }
+#pragma unroll
+      for (int k = 0; k < KN; ++k)
+        if (k < K) *reinterpret_cast<float4*>(part + k * D + c) = acc[k];
     }
+  } else {
+    for (int c = threadIdx.x; c < D; c += blockDim.x) {
+      float acc[KN];
 #pragma unroll
-    for (int k = 0; k < KN; ++k)
-      if (k < K) part[k * D + c] = acc[k];
+      for (int k = 0; k < KN; ++k) acc[k] = 0.0f;
+      for (int jb = 0; jb < nl; jb += 8) {
+        float xv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) xv[u] = jb + u < nl ? value(jb + u, c) : 0.0f;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (jb + u < nl) {
+            const int a = asg[jb + u];
+#pragma unroll
+            for (int k = 0; k < KN; ++k)
+              if (k == a) acc[k] += xv[u];
+          }
+      }
+#pragma unroll
+      for (int k = 0; k < KN; ++k)
+        if (k < K) part[k * D + c] = acc[k];
+    }
   }
 }
 
@@ -423,8 +483,11 @@ __device__ __forceinline__ void cluster_column_reduce(cg::cluster_group& cl, flo
 // once (one bulk copy per row) and every Lloyd iteration reads them there; otherwise each
 // iteration re-reads them from global memory (L2). KN: an upper bound of K known at compile time
 // (K itself for the paper's K = 4), sizing the per-thread accumulators.
+template <int KN>
+constexpr int kmeans_threads() { return KN == 4 ? 256 : 512; }
+
 template <int KC, bool RES, int KN>
-__global__ void __launch_bounds__(512) kmeans_kernel(PruneDims p, PruneWs w) {
+__global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
   extern __shared__ __align__(16) float ksm[];
@@ -488,7 +551,56 @@ __global__ void __launch_bounds__(512) kmeans_kernel(PruneDims p, PruneWs w) {
     // assignment of this CTA's points
     if (threadIdx.x == 0) changed = 0;
     __syncthreads();
-    for (int jj = warp; jj < nl; jj += nw) {
+    bool done_assign = false;
+    if constexpr (KN == 4) {
+      if (D <= 1024) {
+        done_assign = true;
+        // lane's columns 4 lane + 128 j (j < 8) of the four centroids in registers
+        float4 cr[4][8];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int c = 4 * lane + 128 * j;
+            cr[k][j] = (k < K && c < D) ? *reinterpret_cast<const float4*>(cent + k * D + c)
+                                        : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+        for (int jj = warp; jj < nl; jj += nw) {
+          const float* x = xrow(jj);
+          float4 xv[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int c = 4 * lane + 128 * j;
+            xv[j] = c < D ? *reinterpret_cast<const float4*>(x + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+          float pd[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float d0 = xv[j].x - cr[k][j].x, d1 = xv[j].y - cr[k][j].y,
+                          d2 = xv[j].z - cr[k][j].z, d3 = xv[j].w - cr[k][j].w;
+              pd[k] += d0 * d0 + d1 * d1 + d2 * d2 + d3 * d3;
+            }
+          int best = 0;
+          float bd = 0.0f;
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            if (k < K) {
+              const float dk = warp_sum(pd[k]);
+              if (k == 0 || dk < bd) {
+                bd = dk;
+                best = k;
+              }
+            }
+          if (lane == 0) {
+            if (it == 0 || asg[jj] != best) changed = 1;
+            asg[jj] = int8_t(best);
+          }
+        }
+      }
+    }
+    for (int jj = done_assign ? nl : warp; jj < nl; jj += nw) {
       const float* x = xrow(jj);
       float part_d[KN];
 #pragma unroll
@@ -537,7 +649,8 @@ __global__ void __launch_bounds__(512) kmeans_kernel(PruneDims p, PruneWs w) {
     if (threadIdx.x < K) cnt[threadIdx.x] = 0;
     __syncthreads();
     for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) atomicAdd(&cnt[asg[jj]], 1);
-    column_sums<KN>(part, K, D, nl, asg, [&](int jj, int c) { return xrow(jj)[c]; });
+    column_sums<KN>(part, K, D, nl, asg,
+                    RowAccess{RES ? rows : nullptr, fin, row0, idx, D, nullptr});
     cl.sync();
     // one warp reads the peers' flags and sizes (lane r: CTA r) and publishes them in this CTA
     if (warp == 0) {
@@ -595,12 +708,7 @@ __global__ void __launch_bounds__(512) kmeans_kernel(PruneDims p, PruneWs w) {
       }
     }
     __syncthreads();
-    if (RES)
-      column_sums<KN>(part, K, D, nl, asg,
-                      [&](int jj, int c) { return rows[size_t(jj) * D + c] * rinv[jj]; });
-    else
-      column_sums<KN>(part, K, D, nl, asg,
-                      [&](int jj, int c) { return fl[(row0 + idx[jj]) * D + c] * rinv[jj]; });
+    column_sums<KN>(part, K, D, nl, asg, RowAccess{RES ? rows : nullptr, fl, row0, idx, D, rinv});
     cl.sync();
     float* csum = w.csum + (size_t(t) * p.L + l) * K * D;
     cluster_column_reduce<KC>(cl, part, K, D, rank,
@@ -843,7 +951,7 @@ template <int KC, bool RES, int KN>
 cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, size_t smem, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(KC, p.n_tiles);
-  cfg.blockDim = dim3(512);
+  cfg.blockDim = dim3(kmeans_threads<KN>());
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute attr[2];
@@ -938,12 +1046,13 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
     SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel,
                             dim3((p.m + 63) / 64 * kAS, (p.n_anc + 63) / 64, T), dim3(256), 0, st,
                             p, w));
-  // K-means: the rows resident in shared memory over 16 CTAs per tile where they fit, else
-  // re-read from L2 each iteration by 8 CTAs per tile
+  // K-means: the rows resident in shared memory over 16 CTAs per tile where they fit and all
+  // tiles run in one wave of such clusters (latency); else re-read from L2 each pass by 8 CTAs per
+  // tile, twice as many tiles at once (throughput)
   if (int rc = kmeans_setup()) return rc;
   const size_t cent_bytes = size_t(2) * p.K * p.d * sizeof(float);
   const size_t res_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float) + cent_bytes;
-  const bool res = p.m > 0 && res_bytes <= kResSmem && g_res_clusters > 0;
+  const bool res = p.m > 0 && res_bytes <= kResSmem && g_res_clusters > 0 && T <= g_res_clusters;
   if (res && p.K == 4)
     SPD_CUDA_TRY((launch_kmeans<16, true, 4>(p, w, res_bytes, st)));
   else if (res)

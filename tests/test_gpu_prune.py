@@ -37,6 +37,20 @@ def test_llava_next_anyres_tiles(keep):
     assert_prune_parity(gpu_prune(v, keep, 1), res)
 
 
+def test_many_tiles_streamed_kmeans():
+    # more tiles than one wave of resident 16-CTA K-means clusters: the form that re-reads the rows
+    # from L2 with 8 CTAs per tile runs (serving batches)
+    # (tiles conditioned one by one: a seed whose 24 tiles all have margins above 1e-3 is rare)
+    vs, res = [], []
+    for i in range(24):
+        _, v1, r1 = conditioned_vision(20260601 + 97 * i, 1, 576, 1024, 2, 16, 64, 1)
+        vs.append(v1)
+        res += r1
+    v = {"feats": [np.concatenate([x["feats"][l] for x in vs]) for l in range(2)],
+         "attn": np.concatenate([x["attn"] for x in vs])}
+    assert_prune_parity(gpu_prune(v, 64, 1), res)
+
+
 def test_clsless_received_attention_form():
     # Qwen-style post-merger tokens: no CLS, received-attention importance, keep ratio 0.25.
     _, v, res = conditioned_vision(20260301, 1, 1024, 1280, 2, 16, 256, 1, has_cls=False,
