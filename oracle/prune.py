@@ -29,6 +29,44 @@ def attention_importance(attn_tile: np.ndarray, form: int) -> np.ndarray:
     return a.mean(axis=0)
 
 
+def received_attention(maps: np.ndarray, groups=None) -> np.ndarray:
+    """Received-attention form [H][n_out] from full self-attention maps [H][n_q][n_k] (§4.1.1:
+    without a [CLS] token, the importance of a patch is the mean attention it receives).
+
+    R[h, i] = (1 / n_q) * sum over query rows q of maps[h, q, i].
+
+    groups (optional): for encoders with a patch merger (§Implementation details: Qwen's
+    PatchMerger), a list over post-merger tokens of the pre-merger token indices each one merges.
+    The post-merger token receives the attention its members receive, summed: merging keys merges
+    their probability mass (reading: the paper states that importance is computed on post-merger
+    tokens but not how attention is carried through the merger). Without groups, n_out = n_k.
+    """
+    a = np.asarray(maps, dtype=np.float64)
+    h, n_q, n_k = a.shape
+    r = np.zeros((h, n_k))
+    for q in range(n_q):  # explicit sum over the query rows
+        r += a[:, q, :]
+    r /= n_q
+    if groups is None:
+        return r
+    out = np.zeros((h, len(groups)))
+    for j, members in enumerate(groups):
+        for i in members:
+            out[:, j] += r[:, i]
+    return out
+
+
+def merge_groups_2x2(rows: int, cols: int):
+    """Pre-merger token indices of each post-merger token for a 2 x 2 spatial merger over a
+    rows x cols patch grid (row-major, both even): post token (y, x) merges patches (2y + dy,
+    2x + dx), dy, dx in {0, 1}, listed in ascending index order."""
+    groups = []
+    for y in range(rows // 2):
+        for x in range(cols // 2):
+            groups.append(sorted((2 * y + dy) * cols + 2 * x + dx for dy in (0, 1) for dx in (0, 1)))
+    return groups
+
+
 def n_anchor_tokens(keep: int, anchor_ratio: float) -> int:
     """N_anc = round(keep * r), half away from zero, evaluated in double (§4.1, Eq. 1 budget n R r).
 

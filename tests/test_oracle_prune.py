@@ -210,3 +210,54 @@ def test_planted_inputs_are_well_conditioned_for_some_seeds():
         res = op.prune(v["feats"], v["attn"], keep=64, final_layer=2)[0]
         ok += op.well_conditioned(res)
     assert ok >= 2
+
+
+# ---- received attention from full maps (§4.1.1 without [CLS]; the Qwen PatchMerger reading) ----
+def _softmax_maps(rng, h, n_q, n_k):
+    z = rng.standard_normal((h, n_q, n_k)) * 2.0
+    e = np.exp(z - z.max(axis=2, keepdims=True))
+    return e / e.sum(axis=2, keepdims=True)
+
+
+def test_received_attention_conserves_mass_on_non_square_maps():
+    # every query row of a softmax map sums to one, so the mean over queries of the attention each
+    # key receives sums to one per head (a reduction over the key axis instead would sum to
+    # n_q / n_k here)
+    rng = np.random.default_rng(1)
+    a = _softmax_maps(rng, 3, 7, 12)
+    r = op.received_attention(a)
+    assert r.shape == (3, 12)
+    np.testing.assert_allclose(r.sum(axis=1), 1.0, rtol=0, atol=1e-12)
+    g = op.merge_groups_2x2(2, 6)  # the 12 keys as a 2 x 6 grid: three merged tokens
+    np.testing.assert_allclose(op.received_attention(a, g).sum(axis=1), 1.0, rtol=0, atol=1e-12)
+
+
+def test_received_attention_closed_forms():
+    n = 24
+    uniform = np.full((2, 10, n), 1.0 / n)
+    np.testing.assert_allclose(op.received_attention(uniform), 1.0 / n, rtol=1e-15)
+    g = op.merge_groups_2x2(4, 6)
+    np.testing.assert_allclose(op.received_attention(uniform, g), 4.0 / n, rtol=1e-15)
+    one_hot = np.zeros((1, 5, n))
+    one_hot[0, :, 13] = 1.0  # every query attends to key 13 only
+    r = op.received_attention(one_hot, g)[0]
+    owner = [j for j, members in enumerate(g) if 13 in members]
+    assert owner == [3]  # key 13 = grid (2, 1): post-merger token (1, 0) of a 2 x 3 post grid
+    expect = np.zeros(len(g))
+    expect[3] = 1.0
+    np.testing.assert_array_equal(r, expect)
+
+
+def test_received_attention_ignores_query_order():
+    rng = np.random.default_rng(2)
+    a = _softmax_maps(rng, 2, 9, 9)
+    perm = rng.permutation(9)
+    np.testing.assert_allclose(op.received_attention(a[:, perm, :]), op.received_attention(a),
+                               rtol=1e-13)
+
+
+def test_merge_groups_2x2_partition_the_grid_into_blocks():
+    g = op.merge_groups_2x2(4, 6)
+    assert g[0] == [0, 1, 6, 7] and g[1] == [2, 3, 8, 9] and g[3] == [12, 13, 18, 19]
+    flat = sorted(i for members in g for i in members)
+    assert flat == list(range(24))
