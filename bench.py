@@ -179,6 +179,39 @@ def prune_batch(torch, N, synth, dev, steps, warmup, hbm, tiles=64, keep=64):
                     "layers 12/24, keep 64 per tile), features larger than L2"}
 
 
+def received_batch(torch, N, dev, steps, warmup, hbm, images=4, heads=16, grid=64):
+    """The received-attention form from full maps (encoders without [CLS], Qwen-style): 4 images x
+    16 heads of 4096 x 4096 pre-merger attention (a 64 x 64 patch grid) reduced to 1024
+    post-merger tokens through a 2 x 2 merger. Algorithmic bytes: every map entry read once, the
+    result written once; the maps (1.07 GB) exceed L2. Timed with CUDA events."""
+    n = grid * grid
+    maps = torch.rand((images * heads, n, n), device=dev)
+    post = [(2 * y + dy) * grid + 2 * x + dx for y in range(grid // 2) for x in range(grid // 2)
+            for dy in (0, 1) for dx in (0, 1)]
+    start = torch.arange(0, len(post) + 1, 4, dtype=torch.int32, device=dev)
+    members = torch.tensor(post, dtype=torch.int32, device=dev)
+    out = torch.empty((images * heads, n // 4), device=dev)
+    ws = torch.zeros(N.spd_received_attention_workspace_size(images * heads, n, n), dtype=torch.uint8,
+                     device=dev)
+    for _ in range(warmup):
+        N.spd_received_attention(maps, out, ws, start, members)
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        N.spd_received_attention(maps, out, ws, start, members)
+    e.record()
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0, "device-side failure recorded"
+    us = 1000.0 * s.elapsed_time(e) / steps
+    nbytes = 4.0 * images * heads * n * n + 4.0 * images * heads * (n // 4)
+    gbs = nbytes / (us * 1e-6) / 1e9
+    del maps
+    return {"us_per_call": us, "GB/s": gbs, "hbm_frac": gbs / hbm, "bytes": nbytes,
+            "what": f"spd_received_attention: {images} images x {heads} heads of {n} x {n} fp32 "
+                    f"attention -> {n // 4} post-merger tokens (2 x 2 merger)"}
+
+
 def cpu_baseline_sample(keep, v, mask_fn, reps=1):
     """The oracle as it stands on the host cores: MSV-Prune of the tile, the projector, and 1- and
     2-layer decoder prefills of the same token count; the step time is extrapolated to 32 layers."""
@@ -364,6 +397,7 @@ def main():
                   "tensor_frac_of_sustained": dense_tfs / tf_sust,
                   "GB/s": dg["bytes"] / (dg["ms"] / 1000.0) / 1e9}
     pb = prune_batch(torch, N, synth, dev, a.steps, a.warmup, hbm)
+    ra = received_batch(torch, N, dev, a.steps, a.warmup, hbm)
 
     # end to end through the public API: pinned host inputs -> device, step, logits -> host
     hf = [f.cpu().pin_memory() for f in feats]
@@ -406,7 +440,7 @@ def main():
                 "dense": {"value": tokens / (ms_dense / 1000.0), "ms_per_step": ms_dense,
                           "decoder_tokens": dense.T, "speedup_spider_vs_dense": ms_dense / ms},
                 "roofline": roof, "kernels": kernels, "dense_gemm": dense_gemm,
-                "prune_batch": pb, "cpu_baseline": cpu,
+                "prune_batch": pb, "received_attention": ra, "cpu_baseline": cpu,
                 "e2e": {"value": tokens / (ms_e2e / 1000.0), "unit": "tokens/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": hl.numel() * 4,
                         "ms_per_step": ms_e2e},

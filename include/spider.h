@@ -111,6 +111,26 @@ int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, const float* 
               int32_t* keep_idx, uint8_t* kind, int8_t* cluster, float* scores,
               void* ws, size_t ws_bytes, void* stream);
 
+/* Workspace bytes of spd_received_attention. */
+size_t spd_received_attention_workspace_size(int n_maps, int n_q, int n_k);
+
+/* The received-attention input form of spd_prune (attn_form 1) from full self-attention maps
+ * (Sec. 4.1.1: for an encoder without a [CLS] token a patch's importance is the mean attention it
+ * receives), per map m (tile x head):
+ *   R[m][i] = (1 / n_q) sum over query rows q of maps[m][q][i],
+ * optionally carried through a patch merger whose post-merger token j merges pre-merger tokens
+ * group_members[group_start[j] .. group_start[j+1]) (ascending): out[m][j] = sum of R[m][i] over
+ * the members (merging keys merges their attention mass; the paper computes importance on the
+ * post-merger tokens but does not state the aggregation - this is the library's reading).
+ * maps (dev) fp32 [n_maps][n_q][n_k], 16-byte aligned, n_k a multiple of 4; group_start (dev)
+ * int32 [n_out + 1] and group_members (dev) int32, both NULL for no merger (then n_out = n_k);
+ * out (dev) fp32 [n_maps][n_out]. Sums run in a fixed order (bit-identical run to run).
+ * Errors: SPD_EINVAL (arguments; a member index outside [0, n_k) is reported through the
+ * workspace's status word), SPD_ENOSPC. */
+int spd_received_attention(const float* maps, int n_maps, int n_q, int n_k, const int32_t* group_start,
+                           const int32_t* group_members, int n_out, float* out, void* ws,
+                           size_t ws_bytes, void* stream);
+
 /* Gathers the kept rows of a per-tile payload (e.g. F^L) into packed bf16 rows for the projector:
  * dst[t * keep + j][:] = bf16(src[t][row_offset + idx[t][j]][:]), round to nearest even.
  * src (dev) fp32 [n_tiles][n_tok][d]; idx (dev) int32 [n_tiles][keep]; dst (dev) bf16

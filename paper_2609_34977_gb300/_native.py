@@ -20,7 +20,8 @@ EPI_F32, EPI_BF16, EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_ADD_F32 = 0, 1, 2, 3, 
 
 # every symbol include/spider.h declares
 EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait",
-           "spd_prune_workspace_size", "spd_prune", "spd_gather_rows_bf16", "spd_model_create",
+           "spd_prune_workspace_size", "spd_prune", "spd_received_attention_workspace_size",
+           "spd_received_attention", "spd_gather_rows_bf16", "spd_model_create",
            "spd_model_destroy", "spd_plan_adaptive", "spd_plan_static", "spd_project_workspace_size",
            "spd_project", "spd_scatter_rows", "spd_attention_workspace_size", "spd_attention",
            "spd_prefill_workspace_size", "spd_prefill",
@@ -77,6 +78,8 @@ def lib():
             "spd_selftest_bounded_wait": (i, [vp, ll, vp]),
             "spd_prune_workspace_size": (sz, [C.POINTER(PruneCfg)]),
             "spd_prune": (i, [C.POINTER(PruneCfg), C.POINTER(vp), vp, vp, vp, vp, vp, vp, sz, vp]),
+            "spd_received_attention_workspace_size": (sz, [i, i, i]),
+            "spd_received_attention": (i, [vp, i, i, i, vp, vp, i, vp, vp, sz, vp]),
             "spd_gather_rows_bf16": (i, [vp, i, i, i, i, vp, i, vp, vp, vp]),
             "spd_model_create": (i, [C.POINTER(ModelCfg), C.POINTER(ModelWeights), C.POINTER(vp)]),
             "spd_model_destroy": (None, [vp]),
@@ -158,6 +161,20 @@ def spd_prune(cfg, feats, attn, keep_idx, kind=None, cluster=None, scores=None, 
     arr = (C.c_void_p * len(feats))(*[_p(f) for f in feats])
     _check(lib().spd_prune(C.byref(cfg), arr, _p(attn), _p(keep_idx), _p(kind), _p(cluster),
                            _p(scores), _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def spd_received_attention_workspace_size(n_maps: int, n_q: int, n_k: int) -> int:
+    return int(lib().spd_received_attention_workspace_size(n_maps, n_q, n_k))
+
+
+def spd_received_attention(maps, out, ws, group_start=None, group_members=None, stream=None):
+    """Received-attention form out [n_maps][n_out] from full maps [n_maps][n_q][n_k] (optionally
+    through a patch merger given as CSR groups)."""
+    n_maps, n_q, n_k = maps.shape
+    n_out = out.shape[-1]
+    _check(lib().spd_received_attention(_p(maps), n_maps, n_q, n_k, _p(group_start), _p(group_members),
+                                        n_out, _p(out), _p(ws), ws.numel() * ws.element_size(),
+                                        _stream(stream)))
 
 
 def spd_gather_rows_bf16(src, n_tiles, n_tok, d, row_offset, idx, keep, dst, ws=None, stream=None):

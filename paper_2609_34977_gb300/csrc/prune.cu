@@ -25,6 +25,7 @@
 
 #include <cooperative_groups.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "internal.h"
@@ -790,6 +791,71 @@ __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
   if (lane == 0) w.score[size_t(t) * p.m + j] = s;
 }
 
+// ---- received attention from full maps (Sec. 4.1.1 without [CLS]) ------------------------------
+// Column sums of attention maps: CTA (column block, map, row split) adds rows [q0, q1) of its 1024
+// columns (thread: four adjacent columns, float4 loads, eight rows in flight) in row order.
+__global__ void __launch_bounds__(256) received_colsum_kernel(const float* __restrict__ maps, int n_q,
+                                                              int n_k, int rows_per_split,
+                                                              float* __restrict__ partial) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int c4 = blockIdx.x * 256 + threadIdx.x;  // float4 column group
+  const int mp = blockIdx.y, sp = blockIdx.z, n_maps = gridDim.y;
+  if (4 * c4 >= n_k) return;
+  const int q0 = sp * rows_per_split, q1 = min(n_q, q0 + rows_per_split);
+  const float4* src = reinterpret_cast<const float4*>(maps + size_t(mp) * n_q * n_k) + c4;
+  const size_t ld4 = n_k / 4;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int q = q0; q < q1; q += 8) {
+    float4 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      v[u] = q + u < q1 ? __ldcs(src + size_t(q + u) * ld4) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      acc.x += v[u].x;
+      acc.y += v[u].y;
+      acc.z += v[u].z;
+      acc.w += v[u].w;
+    }
+  }
+  reinterpret_cast<float4*>(partial + (size_t(sp) * n_maps + mp) * n_k)[c4] = acc;
+}
+
+// out[m][j] = sum over the members i of group j (ascending) of (sum over splits, in order, of the
+// partial column sums) / n_q; without groups j = i.
+__global__ void __launch_bounds__(256) received_finish_kernel(const float* __restrict__ partial,
+                                                              int n_maps, int n_k, int n_splits,
+                                                              float inv_nq,
+                                                              const int32_t* __restrict__ gstart,
+                                                              const int32_t* __restrict__ gmem,
+                                                              int n_out, float* __restrict__ out,
+                                                              int* status) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int j = blockIdx.x * 256 + threadIdx.x, mp = blockIdx.y;
+  if (j >= n_out) return;
+  auto col = [&](int i) {
+    float s = 0.0f;
+    for (int sp = 0; sp < n_splits; ++sp) s += partial[(size_t(sp) * n_maps + mp) * n_k + i];
+    return s * inv_nq;
+  };
+  float v = 0.0f;
+  if (gstart) {
+    for (int e = gstart[j]; e < gstart[j + 1]; ++e) {
+      const int i = gmem[e];
+      if (i < 0 || i >= n_k) {
+        set_status(status, SPD_EINVAL);
+        continue;
+      }
+      v += col(i);
+    }
+  } else {
+    v = col(j);
+  }
+  out[size_t(mp) * n_out + j] = v;
+}
+
 // ---- 7. per-cluster bottom-N_k, compaction, outputs -------------------------------------------
 __global__ void __launch_bounds__(1024) select_kernel(PruneDims p, PruneWs w, int32_t* keep_idx,
                                                       uint8_t* kind, int8_t* cluster, float* scores) {
@@ -1069,6 +1135,51 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
   // kept indices written; anchor similarities (n - N_anc) N_anc d multiply-adds
   trace_end(slot, st, TR_PRUNE, 2.0 * T * double(p.m) * p.n_anc * p.d,
             T * (4.0 * p.L * double(p.n_tok) * p.d + 4.0 * p.H * p.n_att + 4.0 * p.keep + 6.0 * p.n));
+  return SPD_OK;
+}
+
+namespace {
+int received_splits(int n_maps, int n_q, int n_k) {
+  const int blocks = (n_k / 4 + 255) / 256;
+  int sp = (2 * num_sms() + blocks * n_maps - 1) / (blocks * n_maps);  // about two CTAs per SM
+  sp = std::max(1, std::min(sp, (n_q + 63) / 64));                    // at least 64 rows each
+  return sp;
+}
+}  // namespace
+
+extern "C" size_t spd_received_attention_workspace_size(int n_maps, int n_q, int n_k) {
+  if (n_maps < 1 || n_q < 1 || n_k < 4) return 0;
+  Carve cv(nullptr, ~size_t(0));
+  cv.take<float>(size_t(received_splits(n_maps, n_q, n_k)) * n_maps * n_k);
+  return cv.used;
+}
+
+extern "C" int spd_received_attention(const float* maps, int n_maps, int n_q, int n_k,
+                                      const int32_t* group_start, const int32_t* group_members,
+                                      int n_out, float* out, void* ws, size_t ws_bytes,
+                                      void* stream_) {
+  if (!maps || !out || !ws || n_maps < 1 || n_q < 1 || n_k < 4 || n_k % 4 ||
+      (reinterpret_cast<uintptr_t>(maps) & 15))
+    return fail(SPD_EINVAL, "bad received-attention arguments (n_k a multiple of 4, maps 16-byte aligned)");
+  if ((group_start == nullptr) != (group_members == nullptr))
+    return fail(SPD_EINVAL, "group_start and group_members go together");
+  if (!group_start && n_out != n_k) return fail(SPD_EINVAL, "without groups n_out must equal n_k");
+  if (n_out < 1) return fail(SPD_EINVAL, "n_out >= 1 required");
+  const int sp = received_splits(n_maps, n_q, n_k);
+  Carve cv(ws, ws_bytes);
+  float* partial = cv.take<float>(size_t(sp) * n_maps * n_k);
+  if (!cv.fits()) return fail(SPD_ENOSPC, "received-attention workspace too small");
+  cudaStream_t st = static_cast<cudaStream_t>(stream_);
+  const int rows = (n_q + sp - 1) / sp;
+  const int slot = trace_begin(st);
+  SPD_CUDA_TRY(launch_pdl(received_colsum_kernel, dim3((n_k / 4 + 255) / 256, n_maps, sp), dim3(256),
+                          0, st, maps, n_q, n_k, rows, partial));
+  SPD_CUDA_TRY(launch_pdl(received_finish_kernel, dim3((n_out + 255) / 256, n_maps), dim3(256), 0, st,
+                          static_cast<const float*>(partial), n_maps, n_k, sp, float(1.0 / n_q),
+                          group_start, group_members, n_out, out, cv.status()));
+  // algorithmic work: every map entry read once, the result written once
+  trace_end(slot, st, TR_PRUNE, double(n_maps) * n_q * n_k,
+            4.0 * double(n_maps) * n_q * n_k + 4.0 * double(n_maps) * n_out);
   return SPD_OK;
 }
 

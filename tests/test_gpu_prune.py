@@ -94,3 +94,62 @@ def test_gather_rows_bf16():
     assert N.spd_workspace_status(g["ws"]) == 0
     ref = np.concatenate([v["feats"][1][t, 1 + g["keep_idx"][t]] for t in range(3)])
     np.testing.assert_array_equal(bf16_np(dst), torch.from_numpy(ref).to(torch.bfloat16).double().numpy())
+
+
+# ---- received attention from full maps (Sec. 4.1.1 without [CLS]) --------------------------------
+def _maps(seed, n_maps, n_q, n_k):
+    g = torch.Generator().manual_seed(seed)
+    z = torch.randn(n_maps, n_q, n_k, generator=g, dtype=torch.float64) * 2.0
+    return torch.softmax(z, dim=2)
+
+
+def _gpu_received(maps, groups=None):
+    m = maps.float().cuda()
+    n_maps, n_q, n_k = m.shape
+    ws = torch.zeros(N.spd_received_attention_workspace_size(n_maps, n_q, n_k), dtype=torch.uint8,
+                     device="cuda")
+    if groups is None:
+        out = torch.full((n_maps, n_k), float("nan"), device="cuda")
+        N.spd_received_attention(m, out, ws)
+    else:
+        start = np.cumsum([0] + [len(g) for g in groups]).astype(np.int32)
+        members = np.concatenate([np.asarray(g, np.int32) for g in groups])
+        out = torch.full((n_maps, len(groups)), float("nan"), device="cuda")
+        N.spd_received_attention(m, out, ws, torch.from_numpy(start).cuda(),
+                                 torch.from_numpy(members).cuda())
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    return out.cpu().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("n_maps,n_q,n_k", [(16, 1024, 1024), (3, 777, 1100), (1, 64, 4)])
+def test_received_attention_matches_oracle(n_maps, n_q, n_k):
+    maps = _maps(n_maps + n_q, n_maps, n_q, n_k)
+    got = _gpu_received(maps)
+    ref = op.received_attention(maps.float().double().numpy())
+    np.testing.assert_allclose(got, ref, rtol=1e-5, atol=1e-9)
+    np.testing.assert_allclose(got.sum(axis=1), 1.0, rtol=0, atol=1e-4)  # mass conservation
+
+
+def test_received_attention_through_a_2x2_merger_feeds_prune():
+    # Qwen-style: pre-merger maps over a 32 x 40 patch grid, 2 x 2 merger -> 320 post tokens,
+    # then MSV-Prune on the received form (attn_form 1) of those post-merger tokens
+    rows, cols, H = 32, 40, 4
+    groups = op.merge_groups_2x2(rows, cols)
+    maps = _maps(7, H, rows * cols, rows * cols)
+    got = _gpu_received(maps, groups)
+    ref = op.received_attention(maps.float().double().numpy(), groups)
+    np.testing.assert_allclose(got, ref, rtol=1e-5, atol=1e-9)
+    a = torch.from_numpy(got.astype(np.float32))[None]  # [1 tile][H][320]
+    _, v, _ = conditioned_vision(20260701, 1, len(groups), 128, 2, H, 80, 1, has_cls=False,
+                                 attn_form=1)
+    v["attn"] = a.numpy()
+    res = op.prune(v["feats"], v["attn"], has_cls=False, attn_form=1, final_layer=1, keep=80)
+    if all(op.well_conditioned(r) for r in res):
+        assert_prune_parity(gpu_prune(v, 80, 1, has_cls=False, attn_form=1), res)
+
+
+def test_received_attention_repeat_runs_are_bitwise_identical():
+    maps = _maps(3, 8, 512, 512)
+    a, b = _gpu_received(maps), _gpu_received(maps)
+    np.testing.assert_array_equal(a, b)
