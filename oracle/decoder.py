@@ -118,6 +118,35 @@ def expand_static_plan(layer_mask, token_sel):
     return (layer_mask[:, None] * token_sel[None, :]).astype(np.uint8)
 
 
+def forward_layer(cfg, w, h, mask_l, cu, pos, round_fn=bf16_round, trace=None):
+    """One decoder layer in place on the residual stream h [T][D]: tokens with bit 0 of mask_l
+    bypass attention (not queries; still keys and values), tokens with bit 1 bypass the FFN."""
+    H, Hkv, hd, eps = cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"], cfg["rms_eps"]
+    xa = round_fn(rmsnorm(h, w["attn_norm"], eps))
+    k = round_fn(rope(xa @ w["wk"].T, pos, Hkv, hd, cfg["rope_theta"]))
+    v = round_fn(xa @ w["wv"].T)
+    act = np.flatnonzero((mask_l & 1) == 0)
+    if len(act):
+        q = round_fn(rope(xa[act] @ w["wq"].T, pos[act], H, hd, cfg["rope_theta"]))
+        o = np.zeros((len(act), H * hd))
+        for b in range(len(cu) - 1):
+            rows = np.flatnonzero((act >= cu[b]) & (act < cu[b + 1]))
+            if len(rows):
+                sl = slice(cu[b], cu[b + 1])
+                o[rows] = causal_attention(q[rows], k[sl], v[sl], pos[act[rows]], pos[sl],
+                                           H, Hkv, hd)
+        h[act] += round_fn(o) @ w["wo"].T
+    if trace is not None:
+        trace.append(h.copy())
+    actf = np.flatnonzero((mask_l & 2) == 0)
+    if len(actf):
+        y = round_fn(rmsnorm(h[actf], w["ffn_norm"], eps))
+        a = round_fn(silu(y @ w["w_gate"].T) * (y @ w["w_up"].T))
+        h[actf] += a @ w["w_down"].T
+    if trace is not None:
+        trace.append(h.copy())
+
+
 def prefill(model, x, cu_seqlens, skip_mask, round_fn=bf16_round, trace=None):
     """Decoder prefill over packed sequences with per-layer, per-token sub-layer bypass.
 
@@ -126,38 +155,85 @@ def prefill(model, x, cu_seqlens, skip_mask, round_fn=bf16_round, trace=None):
     If `trace` is a list, the residual stream after every sub-layer is appended to it.
     """
     cfg = model["cfg"]
-    H, Hkv, hd, eps = cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"], cfg["rms_eps"]
+    h = np.array(x, dtype=np.float64)
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    pos = np.concatenate([np.arange(cu[b + 1] - cu[b]) for b in range(len(cu) - 1)])
+    for l, w in enumerate(model["layers"]):
+        forward_layer(cfg, w, h, skip_mask[l], cu, pos, round_fn, trace)
+    last = cu[1:] - 1
+    z = round_fn(rmsnorm(h[last], model["final_norm"], cfg["rms_eps"]))
+    return h, z @ model["lm_head"].T
+
+
+def normalized_entropy(logits):
+    """Shannon entropy of softmax(logits) per row divided by log V (§4.2.1 E_ii in [0, 1])."""
+    z = np.asarray(logits, dtype=np.float64)
+    z = z - z.max(axis=-1, keepdims=True)
+    p = np.exp(z)
+    p /= p.sum(axis=-1, keepdims=True)
+    plogp = np.where(p > 0, p * np.log(np.where(p > 0, p, 1.0)), 0.0)
+    return -plogp.sum(axis=-1) / np.log(z.shape[-1])
+
+
+def skippability(model, h, cand, seq_of, text_rows, round_fn=bf16_round):
+    """S_sa(i, l) = ReLU(1 - E_ii - F_itc) for the candidate tokens (§4.2.1).
+
+    E_ii: normalized entropy of the vocabulary distribution of the token's hidden state, read
+    through the unembedding after the final RMSNorm (the logit-lens reading; the operand rounded to
+    bf16 as every GEMM input). F_itc = (cos(h_i, q_t) + 1) / 2 with q_t the mean hidden state of the
+    text tokens of the token's sequence (cos = 0 when that sequence has no text tokens).
+    """
+    cfg = model["cfg"]
+    z = round_fn(rmsnorm(h[cand], model["final_norm"], cfg["rms_eps"]))
+    e = normalized_entropy(z @ model["lm_head"].T)
+    f = np.empty(len(cand))
+    for n, i in enumerate(cand):
+        t = text_rows[seq_of[i]]
+        if len(t) == 0:
+            f[n] = 0.5
+            continue
+        q = h[t].mean(axis=0)
+        den = np.linalg.norm(h[i]) * np.linalg.norm(q)
+        f[n] = ((h[i] @ q) / den if den > 0 else 0.0) * 0.5 + 0.5
+    return np.maximum(0.0, 1.0 - e - f), e, f
+
+
+def prefill_adaptive(model, x, cu_seqlens, is_visual, slc_norm, layer_target, t_skip, w1, w2,
+                     window, round_fn=bf16_round):
+    """Alg. 1 stage 2 with the online plan: at each layer l < window, every visual token not yet
+    in skip mode accumulates S_skip += w1 S_sa(i, l) + w2 SLC^Norm(l) (Eq. 6); once S_skip >= T_skip
+    it enters skip mode with target m(l) = layer_target[l], frozen, and bypasses that sub-layer
+    from layer l on. Returns (h, logits, admit [T] (-1 never), target [T], margin), margin = the
+    smallest |S_skip - T_skip| over every comparison made (for choosing well-conditioned tests).
+    """
+    cfg = model["cfg"]
+    L = cfg["n_layers"]
     h = np.array(x, dtype=np.float64)
     T = len(h)
     cu = np.asarray(cu_seqlens, dtype=np.int64)
     pos = np.concatenate([np.arange(cu[b + 1] - cu[b]) for b in range(len(cu) - 1)])
-    for l, w in enumerate(model["layers"]):
-        xa = round_fn(rmsnorm(h, w["attn_norm"], eps))
-        k = round_fn(rope(xa @ w["wk"].T, pos, Hkv, hd, cfg["rope_theta"]))
-        v = round_fn(xa @ w["wv"].T)
-        act = np.flatnonzero((skip_mask[l] & 1) == 0)
-        if len(act):
-            q = round_fn(rope(xa[act] @ w["wq"].T, pos[act], H, hd, cfg["rope_theta"]))
-            o = np.zeros((len(act), H * hd))
-            for b in range(len(cu) - 1):
-                rows = np.flatnonzero((act >= cu[b]) & (act < cu[b + 1]))
-                if len(rows):
-                    sl = slice(cu[b], cu[b + 1])
-                    o[rows] = causal_attention(q[rows], k[sl], v[sl], pos[act[rows]], pos[sl],
-                                               H, Hkv, hd)
-            h[act] += round_fn(o) @ w["wo"].T
-        if trace is not None:
-            trace.append(h.copy())
-        actf = np.flatnonzero((skip_mask[l] & 2) == 0)
-        if len(actf):
-            y = round_fn(rmsnorm(h[actf], w["ffn_norm"], eps))
-            a = round_fn(silu(y @ w["w_gate"].T) * (y @ w["w_up"].T))
-            h[actf] += a @ w["w_down"].T
-        if trace is not None:
-            trace.append(h.copy())
+    seq_of = np.concatenate([np.full(cu[b + 1] - cu[b], b) for b in range(len(cu) - 1)])
+    vis = np.asarray(is_visual, dtype=bool)
+    text_rows = [np.flatnonzero((seq_of == b) & ~vis) for b in range(len(cu) - 1)]
+    admit = np.full(T, -1, dtype=np.int64)
+    target = np.zeros(T, dtype=np.uint8)
+    s_skip = np.zeros(T)
+    margin = np.inf
+    for l in range(L):
+        if l < window:
+            cand = np.flatnonzero(vis & (admit < 0))
+            if len(cand):
+                s_sa, _, _ = skippability(model, h, cand, seq_of, text_rows, round_fn)
+                s_skip[cand] += w1 * s_sa + w2 * slc_norm[l]
+                margin = min(margin, float(np.abs(s_skip[cand] - t_skip).min()))
+                new = cand[s_skip[cand] >= t_skip]
+                admit[new] = l
+                target[new] = layer_target[l]
+        mask_l = np.where((admit >= 0) & (admit <= l), target, 0).astype(np.uint8)
+        forward_layer(cfg, model["layers"][l], h, mask_l, cu, pos, round_fn)
     last = cu[1:] - 1
-    z = round_fn(rmsnorm(h[last], model["final_norm"], eps))
-    return h, z @ model["lm_head"].T
+    z = round_fn(rmsnorm(h[last], model["final_norm"], cfg["rms_eps"]))
+    return h, z @ model["lm_head"].T, admit, target, margin
 
 
 def dense_forward(model, x, round_fn=bf16_round):

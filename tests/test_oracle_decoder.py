@@ -192,3 +192,77 @@ def test_table9_covers_every_layer_once():
         assert sorted(t["attn"] + t["ffn"]) == list(range(32))
     assert (synth.skip_targets("llava-1.5-7b") == 2).sum() == 5
     assert (synth.skip_targets("llava-next-7b") == 2).sum() == 7
+
+
+# ---- ASL-Skip online plan (§4.2, Eq. 6, Alg. 1 stage 2) -------------------------------------------
+def test_normalized_entropy_closed_forms():
+    np.testing.assert_allclose(od.normalized_entropy(np.zeros((2, 512))), 1.0, rtol=1e-14)
+    one_hot = np.full((1, 100), -1e4)
+    one_hot[0, 7] = 0.0
+    assert od.normalized_entropy(one_hot)[0] < 1e-12
+    two = np.full((1, 64), -1e4)
+    two[0, :2] = 0.0  # two equally likely words: log 2 / log 64 = 1/6
+    np.testing.assert_allclose(od.normalized_entropy(two), 1.0 / 6.0, rtol=1e-12)
+
+
+def test_skippability_factors_and_clamp():
+    model, _ = tiny_model(std=0.05)
+    D = model["cfg"]["d_model"]
+    rng = np.random.default_rng(3)
+    q = rng.standard_normal(D)
+    h = np.stack([q, -q, 2.0 * q, rng.standard_normal(D), q])  # rows 0-3 visual, 4 text
+    seq_of = np.zeros(5, dtype=np.int64)
+    s_sa, e, f = od.skippability(model, h, np.arange(4), seq_of, [np.array([4])])
+    np.testing.assert_allclose(f[[0, 2]], 1.0, rtol=1e-12)  # parallel to the text mean
+    np.testing.assert_allclose(f[1], 0.0, atol=1e-12)       # antiparallel
+    assert np.all((e >= 0) & (e <= 1))
+    np.testing.assert_allclose(s_sa, np.maximum(0.0, 1.0 - e - f), rtol=1e-15)
+    assert s_sa[0] == 0.0 and s_sa[2] == 0.0  # F_itc = 1 leaves nothing to skip
+    s0, _, f0 = od.skippability(model, h, np.arange(4), seq_of, [np.array([], dtype=np.int64)])
+    np.testing.assert_allclose(f0, 0.5)  # no text in the sequence: cosine taken as 0
+
+
+def _adaptive_case(n_layers=4, T=24, n_text=8):
+    cfg = dict(synth.TINY_DECODER, n_layers=n_layers)
+    model, _ = tiny_model(seed=9, cfg=cfg)
+    x = od.bf16_round(np.random.default_rng(4).standard_normal((T, cfg["d_model"])))
+    vis = np.r_[np.ones(T - n_text, bool), np.zeros(n_text, bool)]
+    return model, x, vis
+
+
+def test_adaptive_plan_with_w1_zero_admits_by_cumulative_slc():
+    # without the online score every visual token is admitted at the first layer whose cumulative
+    # w2 SLC^Norm reaches T_skip, with that layer's target; text tokens never
+    model, x, vis = _adaptive_case()
+    slc = np.array([0.3, 0.5, 0.4, 0.9])
+    tgt = np.array([1, 2, 1, 2], np.uint8)
+    _, _, admit, target, _ = od.prefill_adaptive(model, x, [0, len(x)], vis, slc, tgt, t_skip=0.75,
+                                                 w1=0.0, w2=1.0, window=4)
+    assert np.all(admit[vis] == 1) and np.all(target[vis] == 2)  # 0.3 + 0.5 >= 0.75 at layer 1
+    assert np.all(admit[~vis] == -1)
+
+
+def test_adaptive_plan_never_admitting_is_the_plain_prefill():
+    model, x, vis = _adaptive_case()
+    h, lg, admit, _, _ = od.prefill_adaptive(model, x, [0, len(x)], vis, np.ones(4), np.ones(4, np.uint8),
+                                             t_skip=1e9, w1=3.0, w2=1.0, window=2)
+    h0, lg0 = od.prefill(model, x, [0, len(x)], np.zeros((4, len(x)), np.uint8))
+    assert np.all(admit == -1)
+    np.testing.assert_array_equal(h, h0)
+    np.testing.assert_array_equal(lg, lg0)
+
+
+def test_adaptive_plan_equals_prefill_with_its_own_frozen_plan():
+    # re-running the plain prefill with the plan the online rule produced gives the same stream:
+    # the admission happens before the layer's forward and the target stays frozen
+    model, x, vis = _adaptive_case(n_layers=6)
+    slc = np.array([0.2, 0.9, 0.1, 0.6, 0.8, 0.3])
+    tgt = np.array([1, 2, 2, 1, 1, 2], np.uint8)
+    h, lg, admit, target, _ = od.prefill_adaptive(model, x, [0, len(x)], vis, slc, tgt, t_skip=1.0,
+                                                  w1=3.0, w2=1.0, window=3)
+    assert (admit >= 0).any()
+    plan = od.expand_adaptive_plan(admit, target, 6)
+    h0, lg0 = od.prefill(model, x, [0, len(x)], plan)
+    np.testing.assert_array_equal(h, h0)
+    np.testing.assert_array_equal(lg, lg0)
+    assert np.all(admit < 3)  # decisions only inside the window
