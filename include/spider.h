@@ -250,6 +250,34 @@ int spd_prefill(const spd_model* m, const uint16_t* x, int n_tokens, const int32
                 int n_seqs, const uint8_t* skip_mask, float* h, float* logits, void* ws,
                 size_t ws_bytes, void* stream);
 
+/* ASL-Skip's online plan (Sec. 4.2, Eq. 6, Alg. 1 stage 2). */
+typedef struct {
+  float t_skip;                /* T_skip: a token enters skip mode once its accumulated score reaches it */
+  float w1, w2;                /* weights of the online score S_sa and of SLC^Norm (Eq. 6) */
+  int window;                  /* decision layers 0 .. window-1 (Alg. 1: l <= L/2) */
+  const float* slc_norm;       /* host [n_layers]: SLC^Norm of layer l's designated sub-layer (Eq. 5) */
+  const uint8_t* layer_target; /* host [n_layers]: m(l), 1 = attention, 2 = FFN */
+  const uint8_t* is_visual;    /* host [n_tokens]: 1 for the visual tokens (the skip candidates) */
+} spd_skip_policy;
+
+/* Workspace bytes of spd_prefill_adaptive for up to `max_tokens` tokens in `max_seqs` sequences. */
+size_t spd_prefill_adaptive_workspace_size(const spd_model* m, int max_tokens, int max_seqs);
+
+/* spd_prefill with the skip plan computed online instead of given. Before each layer l < window,
+ * every visual token i not yet in skip mode gets
+ *   E_ii  = entropy of softmax(W_unembed . RMSNorm_final(h_i)) / log V (the logit-lens reading),
+ *   F_itc = (cos(h_i, q_t) + 1) / 2, q_t the mean hidden state of the text tokens of i's sequence
+ *           (F_itc = 1/2 when it has none),
+ *   S_sa  = ReLU(1 - E_ii - F_itc),  S_skip(i) += w1 S_sa + w2 SLC^Norm(l),
+ * and enters skip mode when S_skip(i) >= T_skip, bypassing sub-layer m(l) (frozen) from layer l
+ * on. Arguments as spd_prefill; admit_layer (HOST int16 [n_tokens]) receives each token's
+ * admission layer (-1 = never). The call reads each window layer's admissions back to the host
+ * (one stream synchronisation per window layer) to build that layer's row lists.
+ * Errors as spd_prefill. */
+int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int n_tokens, const int32_t* cu_seqlens,
+                         int n_seqs, const spd_skip_policy* policy, int16_t* admit_layer, float* h,
+                         float* logits, void* ws, size_t ws_bytes, void* stream);
+
 /* ------------------------------------------------------------------------------------------ */
 /* Single kernels, exposed for composition and per-kernel tests                                 */
 /* ------------------------------------------------------------------------------------------ */

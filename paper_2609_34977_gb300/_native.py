@@ -24,7 +24,8 @@ EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait"
            "spd_received_attention", "spd_gather_rows_bf16", "spd_model_create",
            "spd_model_destroy", "spd_plan_adaptive", "spd_plan_static", "spd_project_workspace_size",
            "spd_project", "spd_scatter_rows", "spd_attention_workspace_size", "spd_attention",
-           "spd_prefill_workspace_size", "spd_prefill",
+           "spd_prefill_workspace_size", "spd_prefill", "spd_prefill_adaptive_workspace_size",
+           "spd_prefill_adaptive",
            "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
            "spd_trace_read")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
@@ -49,6 +50,11 @@ class ModelCfg(C.Structure):
                 ("n_kv_heads", C.c_int), ("head_dim", C.c_int), ("d_ffn", C.c_int),
                 ("vocab", C.c_int), ("rope_theta", C.c_float), ("rms_eps", C.c_float),
                 ("d_vis", C.c_int), ("d_proj", C.c_int)]
+
+
+class SkipPolicy(C.Structure):
+    _fields_ = [("t_skip", C.c_float), ("w1", C.c_float), ("w2", C.c_float), ("window", C.c_int),
+                ("slc_norm", C.c_void_p), ("layer_target", C.c_void_p), ("is_visual", C.c_void_p)]
 
 
 class LayerWeights(C.Structure):
@@ -92,6 +98,9 @@ def lib():
             "spd_attention": (i, [vp, i, vp, vp, vp, i, vp, i, i, i, i, vp, vp, sz, vp]),
             "spd_prefill_workspace_size": (sz, [vp, i, i]),
             "spd_prefill": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, sz, vp]),
+            "spd_prefill_adaptive_workspace_size": (sz, [vp, i, i]),
+            "spd_prefill_adaptive": (i, [vp, vp, i, vp, i, C.POINTER(SkipPolicy), vp, vp, vp, vp, sz,
+                                         vp]),
             "spd_linear_workspace_size": (sz, [i, i]),
             "spd_linear": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, sz, vp]),
             "spd_linear_noalloc": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, vp]),
@@ -261,6 +270,27 @@ def spd_scatter_rows(model: SpdModel, src, rows, rows_map, dst, stream=None):
 
 def spd_prefill_workspace_size(model: SpdModel, max_tokens: int, max_seqs: int) -> int:
     return int(lib().spd_prefill_workspace_size(model.handle, max_tokens, max_seqs))
+
+
+def spd_prefill_adaptive_workspace_size(model: SpdModel, max_tokens: int, max_seqs: int) -> int:
+    return int(lib().spd_prefill_adaptive_workspace_size(model.handle, max_tokens, max_seqs))
+
+
+def spd_prefill_adaptive(model: SpdModel, x, n_tokens, cu_seqlens, is_visual, slc_norm, layer_target,
+                         t_skip, w1, w2, window, h, logits, ws, stream=None):
+    """Prefill with the online ASL-Skip plan; returns the admission layer of every token (host
+    int16, -1 = never)."""
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    slc = np.ascontiguousarray(slc_norm, dtype=np.float32)
+    tgt = np.ascontiguousarray(layer_target, dtype=np.uint8)
+    vis = np.ascontiguousarray(is_visual, dtype=np.uint8)
+    admit = np.full(n_tokens, -9, dtype=np.int16)
+    pol = SkipPolicy(float(t_skip), float(w1), float(w2), int(window), slc.ctypes.data, tgt.ctypes.data,
+                     vis.ctypes.data)
+    _check(lib().spd_prefill_adaptive(model.handle, _p(x), n_tokens, cu.ctypes.data, len(cu) - 1,
+                                      C.byref(pol), admit.ctypes.data, _p(h), _p(logits), _p(ws),
+                                      ws.numel() * ws.element_size(), _stream(stream)))
+    return admit
 
 
 def spd_prefill(model: SpdModel, x, n_tokens, cu_seqlens, skip_mask, h, logits, ws, stream=None):

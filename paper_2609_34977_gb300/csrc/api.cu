@@ -539,13 +539,215 @@ extern "C" size_t spd_prefill_workspace_size(const spd_model* m, int max_tokens,
   return cv.used;
 }
 
-extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const int32_t* cu, int B,
-                           const uint8_t* mask, float* h, float* logits, void* ws, size_t ws_bytes,
-                           void* stream) {
+namespace {
+
+// Host side of one prefill call: the per-layer row lists (the plan is control data: it decides
+// which launches happen), in one int32 buffer whose layout the device copy shares.
+struct LayerLists {
+  size_t arows, amap, apos, frows, tiles;  // offsets into the buffer
+  int na, nf, ntiles;
+  double ctx;
+};
+struct HostPlan {
+  std::vector<int32_t> hl;
+  std::vector<int> pos_all, seq_of;
+  std::vector<LayerLists> ll;
+  size_t pos_off = 0, last_off = 0, end = 0;
+};
+
+void plan_init(HostPlan& P, const spd_model_cfg& c, const int32_t* cu, int B, int T, size_t list_ints) {
+  P.hl.assign(list_ints, 0);
+  P.pos_all.assign(T, 0);
+  P.seq_of.assign(T, 0);
+  for (int b = 0; b < B; ++b)
+    for (int t = cu[b]; t < cu[b + 1]; ++t) {
+      P.pos_all[t] = t - cu[b];
+      P.seq_of[t] = b;
+    }
+  P.ll.assign(c.n_layers, LayerLists{});
+  size_t off = 0;
+  P.pos_off = off;
+  for (int t = 0; t < T; ++t) P.hl[off + t] = P.pos_all[t];
+  off += pad4(T);
+  P.last_off = off;
+  for (int b = 0; b < B; ++b) P.hl[off + b] = cu[b + 1] - 1;
+  off += pad4(B);
+  for (int l = 0; l < c.n_layers; ++l) {
+    LayerLists& q = P.ll[l];
+    q.arows = off; off += pad4(T);
+    q.amap = off; off += pad4(T);
+    q.apos = off; off += pad4(T);
+    q.frows = off; off += pad4(T);
+    q.tiles = off;
+    off += 4 * (size_t(T) / 64 + B + 1);
+  }
+  P.end = off;
+}
+
+// Layer l's lists from its skip bits (bit 0 skip attention, bit 1 skip FFN; null = none).
+void plan_layer(HostPlan& P, int l, const uint8_t* mk, const int32_t* cu, int B, int T) {
+  LayerLists& q = P.ll[l];
+  std::vector<int32_t>& hl = P.hl;
+  q.na = q.nf = q.ntiles = 0;
+  q.ctx = 0.0;
+  for (int t = 0; t < T; ++t) {
+    const int bits = mk ? mk[t] : 0;
+    if (!(bits & 1)) {
+      hl[q.amap + t] = q.na;
+      hl[q.apos + q.na] = P.pos_all[t];
+      q.ctx += P.pos_all[t] + 1;
+      hl[q.arows + q.na++] = t;
+    } else {
+      hl[q.amap + t] = -1;
+    }
+    if (!(bits & 2)) hl[q.frows + q.nf++] = t;
+  }
+  // attention tiles: up to kAttnTileQ active queries of one sequence each
+  int a = 0;
+  for (int b = 0; b < B; ++b) {
+    int a_end = a;
+    while (a_end < q.na && P.seq_of[hl[q.arows + a_end]] == b) ++a_end;
+    for (int s0 = a; s0 < a_end; s0 += kAttnTileQ) {
+      int32_t* tl = &hl[q.tiles + 4 * size_t(q.ntiles++)];
+      tl[0] = s0;
+      tl[1] = (a_end - s0 < kAttnTileQ) ? a_end - s0 : kAttnTileQ;
+      tl[2] = cu[b];
+      tl[3] = cu[b + 1] - cu[b];
+    }
+    a = a_end;
+  }
+}
+
+int validate_prefill(const spd_model* m, const uint16_t* x, int T, const int32_t* cu, int B,
+                     const float* h, const void* ws) {
   if (!m || !x || !cu || !h || !ws || T < 1 || B < 1) return fail(SPD_EINVAL, "bad prefill arguments");
   if (cu[0] != 0 || cu[B] != T) return fail(SPD_EINVAL, "cu_seqlens must run from 0 to n_tokens");
   for (int b = 0; b < B; ++b)
     if (cu[b + 1] <= cu[b]) return fail(SPD_EINVAL, "sequence %d is empty or cu_seqlens decreases", b);
+  return SPD_OK;
+}
+
+// Decoder layer l on the residual stream h with its lists at dl (device copy of the plan).
+int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P, const PrefillBufs& bf,
+              const int32_t* dl, float* h, int T, cudaStream_t st) {
+  const spd_model_cfg& c = m->cfg;
+  const int D = c.d_model, hd = c.head_dim;
+  const int qd = c.n_heads * hd, kvd = c.n_kv_heads * hd;
+  const spd_model::Layer& W = m->layers[l];
+  int rc;
+  // attention sub-layer: norm of every row (K/V need all tokens); one GEMM gives K, V of every
+  // token and Q of the query tokens (rows of skipped tokens computed but not stored: the
+  // contraction is weight-bound, one pass over Wq|Wk|Wv beats two launches)
+  if ((rc = rmsnorm_run(h, T, D, W.attn_norm, c.rms_eps, nullptr, bf.xa, nullptr, nullptr, st)))
+    return rc;
+  GemmProblem kvp{};
+  kvp.map_w = &W.m_kv;
+  kvp.w = W.wkv;
+  kvp.x = bf.xa;
+  kvp.n_out = 2 * kvd;
+  kvp.n_tok = T;
+  kvp.k = D;
+  kvp.epi = EPI_ROPE_BF16;
+  kvp.out = bf.kv;
+  kvp.ldo = 2 * kvd;
+  kvp.pos = dl + P.pos_off;
+  kvp.rope = m->freq;
+  kvp.rope_rows = kvd;
+  kvp.head_dim = hd;
+  if (q.na > 0) {
+    GemmProblem qp = kvp;
+    qp.map_w = &W.m_qkv;
+    qp.w = W.wq;  // Wq rows, then Wk and Wv rows, contiguous
+    qp.n_out = qd + 2 * kvd;
+    qp.epi = EPI_QKV_BF16;
+    qp.out = bf.q;
+    qp.ldo = qd;
+    qp.rows = dl + q.amap;
+    qp.out2 = bf.kv;
+    qp.ldo2 = 2 * kvd;
+    qp.split = qd;
+    qp.n_tok_out = q.na;
+    if ((rc = gemm_run(qp, bf.gs, st))) return rc;
+  } else if ((rc = gemm_run(kvp, bf.gs, st))) {
+    return rc;
+  }
+  if (q.na > 0) {
+    if ((rc = attention_run(bf.q, q.na, bf.kv, T, 2 * kvd, kvd, bf.o, qd,
+                            reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
+                            c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx)))
+      return rc;
+    GemmProblem op{};
+    op.map_w = &W.m_o;
+    op.w = W.wo;
+    op.x = bf.o;
+    op.n_out = D;
+    op.n_tok = q.na;
+    op.k = qd;
+    op.epi = EPI_ADD_F32;
+    op.out = h;
+    op.ldo = D;
+    op.rows = dl + q.arows;
+    if ((rc = gemm_run(op, bf.gs, st))) return rc;
+  }
+  if (q.nf > 0) {
+    if ((rc = rmsnorm_run(h, q.nf, D, W.ffn_norm, c.rms_eps, dl + q.frows, bf.y, nullptr, nullptr,
+                          st)))
+      return rc;
+    GemmProblem gp{};
+    gp.map_w = &W.m_gu;
+    gp.w = W.wgu;
+    gp.x = bf.y;
+    gp.n_out = m->gu_rows;
+    gp.n_tok = q.nf;
+    gp.k = D;
+    gp.epi = EPI_SWIGLU_BF16;
+    gp.out = bf.act;
+    gp.ldo = c.d_ffn;
+    gp.out_cols = c.d_ffn;
+    if ((rc = gemm_run(gp, bf.gs, st))) return rc;
+    GemmProblem dp{};
+    dp.map_w = &W.m_d;
+    dp.w = W.wd;
+    dp.x = bf.act;
+    dp.n_out = D;
+    dp.n_tok = q.nf;
+    dp.k = c.d_ffn;
+    dp.epi = EPI_ADD_F32;
+    dp.out = h;
+    dp.ldo = D;
+    dp.rows = dl + q.frows;
+    if ((rc = gemm_run(dp, bf.gs, st))) return rc;
+  }
+  return SPD_OK;
+}
+
+// Final norm and LM head of each sequence's last token.
+int run_head(const spd_model* m, const HostPlan& P, const PrefillBufs& bf, const int32_t* dl,
+             float* h, int B, float* logits, cudaStream_t st) {
+  if (!logits) return SPD_OK;
+  const spd_model_cfg& c = m->cfg;
+  if (int rc = rmsnorm_run(h, B, c.d_model, m->final_norm, c.rms_eps, dl + P.last_off, bf.z, nullptr,
+                           nullptr, st))
+    return rc;
+  GemmProblem lp{};
+  lp.map_w = &m->m_lm;
+  lp.w = m->lm_head;
+  lp.x = bf.z;
+  lp.n_out = c.vocab;
+  lp.n_tok = B;
+  lp.k = c.d_model;
+  lp.epi = EPI_F32;
+  lp.out = logits;
+  lp.ldo = c.vocab;
+  return gemm_run(lp, bf.gs, st);
+}
+
+}  // namespace
+
+extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const int32_t* cu, int B,
+                           const uint8_t* mask, float* h, float* logits, void* ws, size_t ws_bytes,
+                           void* stream) {
+  if (int rc = validate_prefill(m, x, T, cu, B, h, ws)) return rc;
   if (mask)
     for (size_t i = 0; i < size_t(m->cfg.n_layers) * T; ++i)
       if (mask[i] > 3) return fail(SPD_EINVAL, "skip mask entries must be in 0..3");
@@ -554,173 +756,140 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
   PrefillBufs bf = carve_prefill(c, T, B, cv);
   if (!cv.fits()) return fail(SPD_ENOSPC, "prefill workspace too small (%zu < %zu)", ws_bytes, cv.used);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  const int L = c.n_layers, D = c.d_model, hd = c.head_dim;
-  const int qd = c.n_heads * hd, kvd = c.n_kv_heads * hd;
-
-  // Host: per-layer row lists (the plan is control data: it decides which launches happen).
-  static thread_local std::vector<int32_t> hl;
-  hl.assign(bf.list_ints, 0);
-  std::vector<int> pos_all(T), seq_of(T);
-  for (int b = 0; b < B; ++b)
-    for (int t = cu[b]; t < cu[b + 1]; ++t) {
-      pos_all[t] = t - cu[b];
-      seq_of[t] = b;
-    }
-  struct LayerLists { size_t arows, amap, apos, frows, tiles; int na, nf, ntiles; double ctx; };
-  std::vector<LayerLists> ll(L);
-  size_t off = 0;
-  const size_t pos_off = off;
-  for (int t = 0; t < T; ++t) hl[off + t] = pos_all[t];
-  off += pad4(T);
-  const size_t last_off = off;
-  for (int b = 0; b < B; ++b) hl[off + b] = cu[b + 1] - 1;
-  off += pad4(B);
-  for (int l = 0; l < L; ++l) {
-    LayerLists& q = ll[l];
-    const uint8_t* mk = mask ? mask + size_t(l) * T : nullptr;
-    q.arows = off; off += pad4(T);
-    q.amap = off; off += pad4(T);
-    q.apos = off; off += pad4(T);
-    q.frows = off; off += pad4(T);
-    q.tiles = off;
-    q.na = q.nf = q.ntiles = 0;
-    q.ctx = 0.0;
-    for (int t = 0; t < T; ++t) {
-      const int bits = mk ? mk[t] : 0;
-      if (!(bits & 1)) {
-        hl[q.amap + t] = q.na;
-        hl[q.apos + q.na] = pos_all[t];
-        q.ctx += pos_all[t] + 1;
-        hl[q.arows + q.na++] = t;
-      } else {
-        hl[q.amap + t] = -1;
-      }
-      if (!(bits & 2)) hl[q.frows + q.nf++] = t;
-    }
-    // attention tiles: up to kAttnTileQ active queries of one sequence each
-    int a = 0;
-    for (int b = 0; b < B; ++b) {
-      int a_end = a;
-      while (a_end < q.na && seq_of[hl[q.arows + a_end]] == b) ++a_end;
-      for (int s0 = a; s0 < a_end; s0 += kAttnTileQ) {
-        int32_t* tl = &hl[q.tiles + 4 * size_t(q.ntiles++)];
-        tl[0] = s0;
-        tl[1] = (a_end - s0 < kAttnTileQ) ? a_end - s0 : kAttnTileQ;
-        tl[2] = cu[b];
-        tl[3] = cu[b + 1] - cu[b];
-      }
-      a = a_end;
-    }
-    off += 4 * (size_t(T) / 64 + B + 1);
-  }
+  static thread_local HostPlan P;
+  plan_init(P, c, cu, B, T, bf.list_ints);
+  for (int l = 0; l < c.n_layers; ++l) plan_layer(P, l, mask ? mask + size_t(l) * T : nullptr, cu, B, T);
   int32_t* dl = bf.lists;
-  SPD_CUDA_TRY(cudaMemcpyAsync(dl, hl.data(), off * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  SPD_CUDA_TRY(cudaMemcpyAsync(dl, P.hl.data(), P.end * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
+  if (int rc = bf16_to_f32_run(x, h, size_t(T) * c.d_model, st)) return rc;
+  for (int l = 0; l < c.n_layers; ++l)
+    if (int rc = run_layer(m, l, P.ll[l], P, bf, dl, h, T, st)) return rc;
+  return run_head(m, P, bf, dl, h, B, logits, st);
+}
+
+// ---- prefill with the online ASL-Skip plan (Alg. 1 stage 2) -----------------------------------
+namespace {
+struct AdaptiveBufs {
+  float* logits;  // [T][V] vocabulary logits of the candidates
+  float* tmean;   // [B][D] mean text hidden state per sequence
+  float* s_skip;  // [T] accumulated skippability
+  uint8_t* flag;  // [T] admitted at this layer (per candidate)
+  int32_t* cand;  // [T] candidate token indices
+  int32_t* seq;   // [T] sequence of every token
+  int32_t* ts;    // [B + 1] text-token ranges
+  int32_t* text;  // [T] text-token indices
+};
+AdaptiveBufs carve_adaptive(const spd_model_cfg& c, int T, int B, Carve& cv) {
+  AdaptiveBufs a;
+  a.logits = cv.take<float>(size_t(T) * c.vocab);
+  a.tmean = cv.take<float>(size_t(B) * c.d_model);
+  a.s_skip = cv.take<float>(T);
+  a.flag = cv.take<uint8_t>(T);
+  a.cand = cv.take<int32_t>(T);
+  a.seq = cv.take<int32_t>(T);
+  a.ts = cv.take<int32_t>(B + 1);
+  a.text = cv.take<int32_t>(T);
+  return a;
+}
+}  // namespace
+
+extern "C" size_t spd_prefill_adaptive_workspace_size(const spd_model* m, int max_tokens, int max_seqs) {
+  if (!m || max_tokens < 1 || max_seqs < 1) return 0;
+  Carve cv(nullptr, ~size_t(0));
+  carve_prefill(m->cfg, max_tokens, max_seqs, cv);
+  carve_adaptive(m->cfg, max_tokens, max_seqs, cv);
+  return cv.used;
+}
+
+extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T, const int32_t* cu,
+                                    int B, const spd_skip_policy* pol, int16_t* admit_layer,
+                                    float* h, float* logits, void* ws, size_t ws_bytes,
+                                    void* stream) {
+  if (int rc = validate_prefill(m, x, T, cu, B, h, ws)) return rc;
+  if (!pol || !pol->slc_norm || !pol->layer_target || !pol->is_visual || !admit_layer)
+    return fail(SPD_EINVAL, "adaptive prefill needs a policy (SLC^Norm, targets, visual tokens)");
+  const spd_model_cfg& c = m->cfg;
+  const int L = c.n_layers, D = c.d_model;
+  if (pol->window < 0 || pol->window > L) return fail(SPD_EINVAL, "window must lie in [0, n_layers]");
+  for (int l = 0; l < L; ++l)
+    if (pol->layer_target[l] != 1 && pol->layer_target[l] != 2)
+      return fail(SPD_EINVAL, "layer targets must be 1 (attention) or 2 (FFN)");
+  Carve cv(ws, ws_bytes);
+  PrefillBufs bf = carve_prefill(c, T, B, cv);
+  AdaptiveBufs ab = carve_adaptive(c, T, B, cv);
+  if (!cv.fits()) return fail(SPD_ENOSPC, "adaptive prefill workspace too small (%zu < %zu)", ws_bytes, cv.used);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  static thread_local HostPlan P;
+  plan_init(P, c, cu, B, T, bf.list_ints);
+  int32_t* dl = bf.lists;
+  // positions and last tokens; sequences and text tokens of the scores
+  SPD_CUDA_TRY(cudaMemcpyAsync(dl, P.hl.data(), (P.ll.empty() ? P.end : P.ll[0].arows) * sizeof(int32_t),
+                               cudaMemcpyHostToDevice, st));
+  std::vector<int32_t> seq(P.seq_of.begin(), P.seq_of.end()), ts(B + 1, 0), text;
+  for (int b = 0; b < B; ++b) {
+    for (int t = cu[b]; t < cu[b + 1]; ++t)
+      if (!pol->is_visual[t]) text.push_back(t);
+    ts[b + 1] = int32_t(text.size());
+  }
+  SPD_CUDA_TRY(cudaMemcpyAsync(ab.seq, seq.data(), T * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  SPD_CUDA_TRY(cudaMemcpyAsync(ab.ts, ts.data(), (B + 1) * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  if (!text.empty())
+    SPD_CUDA_TRY(cudaMemcpyAsync(ab.text, text.data(), text.size() * sizeof(int32_t),
+                                 cudaMemcpyHostToDevice, st));
+  SPD_CUDA_TRY(cudaMemsetAsync(ab.s_skip, 0, T * sizeof(float), st));
   SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
   if (int rc = bf16_to_f32_run(x, h, size_t(T) * D, st)) return rc;
 
-  int rc = SPD_OK;
-  for (int l = 0; l < L && !rc; ++l) {
-    const spd_model::Layer& W = m->layers[l];
-    const LayerLists& q = ll[l];
-    // attention sub-layer: norm of every row (K/V need all tokens); one GEMM gives K, V of every
-    // token and Q of the query tokens (rows of skipped tokens computed but not stored: the
-    // contraction is weight-bound, one pass over Wq|Wk|Wv beats two launches)
-    rc = rmsnorm_run(h, T, D, W.attn_norm, c.rms_eps, nullptr, bf.xa, nullptr, nullptr, st);
-    if (rc) break;
-    GemmProblem kvp{};
-    kvp.map_w = &W.m_kv;
-    kvp.w = W.wkv;
-    kvp.x = bf.xa;
-    kvp.n_out = 2 * kvd;
-    kvp.n_tok = T;
-    kvp.k = D;
-    kvp.epi = EPI_ROPE_BF16;
-    kvp.out = bf.kv;
-    kvp.ldo = 2 * kvd;
-    kvp.pos = dl + pos_off;
-    kvp.rope = m->freq;
-    kvp.rope_rows = kvd;
-    kvp.head_dim = hd;
-    if (q.na > 0) {
-      GemmProblem qp = kvp;
-      qp.map_w = &W.m_qkv;
-      qp.w = W.wq;  // Wq rows, then Wk and Wv rows, contiguous
-      qp.n_out = qd + 2 * kvd;
-      qp.epi = EPI_QKV_BF16;
-      qp.out = bf.q;
-      qp.ldo = qd;
-      qp.rows = dl + q.amap;
-      qp.out2 = bf.kv;
-      qp.ldo2 = 2 * kvd;
-      qp.split = qd;
-      qp.n_tok_out = q.na;
-      if ((rc = gemm_run(qp, bf.gs, st))) break;
-    } else if ((rc = gemm_run(kvp, bf.gs, st))) {
-      break;
+  std::vector<int> admit(T, -1);
+  std::vector<uint8_t> target(T, 0), row(T, 0), flags(T);
+  std::vector<int32_t> cand;
+  for (int l = 0; l < L; ++l) {
+    if (l < pol->window) {
+      // the decision before layer l's forward, on its input hidden states (Alg. 1)
+      cand.clear();
+      for (int t = 0; t < T; ++t)
+        if (pol->is_visual[t] && admit[t] < 0) cand.push_back(t);
+      const int nc = int(cand.size());
+      if (nc > 0) {
+        SPD_CUDA_TRY(cudaMemcpyAsync(ab.cand, cand.data(), nc * sizeof(int32_t),
+                                     cudaMemcpyHostToDevice, st));
+        // logit lens: final RMSNorm, then the unembedding (LM head) in fp32
+        if (int rc = rmsnorm_run(h, nc, D, m->final_norm, c.rms_eps, ab.cand, bf.xa, nullptr, nullptr, st))
+          return rc;
+        GemmProblem up{};
+        up.map_w = &m->m_lm;
+        up.w = m->lm_head;
+        up.x = bf.xa;
+        up.n_out = c.vocab;
+        up.n_tok = nc;
+        up.k = D;
+        up.epi = EPI_F32;
+        up.out = ab.logits;
+        up.ldo = c.vocab;
+        if (int rc = gemm_run(up, bf.gs, st)) return rc;
+        if (int rc = skip_scores_run(ab.logits, c.vocab, nc, h, D, ab.cand, ab.ts, ab.text, ab.seq, B,
+                                     ab.tmean, pol->w1, pol->w2 * pol->slc_norm[l], pol->t_skip,
+                                     ab.s_skip, ab.flag, st))
+          return rc;
+        SPD_CUDA_TRY(cudaMemcpyAsync(flags.data(), ab.flag, nc, cudaMemcpyDeviceToHost, st));
+        SPD_CUDA_TRY(cudaStreamSynchronize(st));
+        for (int n = 0; n < nc; ++n)
+          if (flags[n]) {
+            admit[cand[n]] = l;
+            target[cand[n]] = pol->layer_target[l];  // frozen at admission
+          }
+      }
     }
-    if (q.na > 0) {
-      if ((rc = attention_run(bf.q, q.na, bf.kv, T, 2 * kvd, kvd, bf.o, qd,
-                              reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
-                              c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx)))
-        break;
-      GemmProblem op{};
-      op.map_w = &W.m_o;
-      op.w = W.wo;
-      op.x = bf.o;
-      op.n_out = D;
-      op.n_tok = q.na;
-      op.k = qd;
-      op.epi = EPI_ADD_F32;
-      op.out = h;
-      op.ldo = D;
-      op.rows = dl + q.arows;
-      if ((rc = gemm_run(op, bf.gs, st))) break;
-    }
-    if (q.nf > 0) {
-      if ((rc = rmsnorm_run(h, q.nf, D, W.ffn_norm, c.rms_eps, dl + q.frows, bf.y, nullptr, nullptr,
-                            st)))
-        break;
-      GemmProblem gp{};
-      gp.map_w = &W.m_gu;
-      gp.w = W.wgu;
-      gp.x = bf.y;
-      gp.n_out = m->gu_rows;
-      gp.n_tok = q.nf;
-      gp.k = D;
-      gp.epi = EPI_SWIGLU_BF16;
-      gp.out = bf.act;
-      gp.ldo = c.d_ffn;
-      gp.out_cols = c.d_ffn;
-      if ((rc = gemm_run(gp, bf.gs, st))) break;
-      GemmProblem dp{};
-      dp.map_w = &W.m_d;
-      dp.w = W.wd;
-      dp.x = bf.act;
-      dp.n_out = D;
-      dp.n_tok = q.nf;
-      dp.k = c.d_ffn;
-      dp.epi = EPI_ADD_F32;
-      dp.out = h;
-      dp.ldo = D;
-      dp.rows = dl + q.frows;
-      if ((rc = gemm_run(dp, bf.gs, st))) break;
-    }
+    for (int t = 0; t < T; ++t) row[t] = (admit[t] >= 0 && admit[t] <= l) ? target[t] : 0;
+    plan_layer(P, l, row.data(), cu, B, T);
+    const LayerLists& q = P.ll[l];
+    const size_t blk_end = q.tiles + 4 * (size_t(T) / 64 + B + 1);
+    SPD_CUDA_TRY(cudaMemcpyAsync(dl + q.arows, P.hl.data() + q.arows, (blk_end - q.arows) * sizeof(int32_t),
+                                 cudaMemcpyHostToDevice, st));
+    if (int rc = run_layer(m, l, q, P, bf, dl, h, T, st)) return rc;
   }
-  if (rc) return rc;
-  if (logits) {
-    if ((rc = rmsnorm_run(h, B, D, m->final_norm, c.rms_eps, dl + last_off, bf.z, nullptr, nullptr, st)))
-      return rc;
-    GemmProblem lp{};
-    lp.map_w = &m->m_lm;
-    lp.w = m->lm_head;
-    lp.x = bf.z;
-    lp.n_out = c.vocab;
-    lp.n_tok = B;
-    lp.k = D;
-    lp.epi = EPI_F32;
-    lp.out = logits;
-    lp.ldo = c.vocab;
-    if ((rc = gemm_run(lp, bf.gs, st))) return rc;
-  }
-  return SPD_OK;
+  for (int t = 0; t < T; ++t) admit_layer[t] = int16_t(admit[t]);
+  return run_head(m, P, bf, dl, h, B, logits, st);
 }
+

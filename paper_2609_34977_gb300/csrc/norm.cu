@@ -2,6 +2,7 @@
 // operands (optionally gathering/scattering rows), bf16 -> fp32 residual initialisation, and bf16
 // row scatter for sequence assembly.
 #include <cuda_bf16.h>
+#include <math.h>
 #include <stdint.h>
 
 #include "internal.h"
@@ -86,7 +87,100 @@ __global__ void scatter_rows_kernel(const uint16_t* __restrict__ src, int D,
   for (int c = threadIdx.x; c < D / 8; c += blockDim.x) d[c] = s[c];
 }
 
+// q_t of sequence b (ASL-Skip's text context, Sec. 4.2.1): the mean of h over the text tokens
+// text[ts[b] .. ts[b+1]), one thread per column, tokens in order (zero when there are none).
+__global__ void __launch_bounds__(kThreads) text_mean_kernel(const float* __restrict__ h, int D,
+                                                             const int32_t* __restrict__ ts,
+                                                             const int32_t* __restrict__ text,
+                                                             float* __restrict__ tmean) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int c = blockIdx.x * kThreads + threadIdx.x, b = blockIdx.y;
+  if (c >= D) return;
+  const int t0 = ts[b], t1 = ts[b + 1];
+  float s = 0.0f;
+  for (int e = t0; e < t1; ++e) s += h[size_t(text[e]) * D + c];
+  tmean[size_t(b) * D + c] = t1 > t0 ? s / float(t1 - t0) : 0.0f;
+}
+
+__device__ __forceinline__ float block_max(float v, float* red) {
+#pragma unroll
+  for (int off = 16; off; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = red[0];
+#pragma unroll
+  for (int w = 1; w < kThreads / 32; ++w) t = fmaxf(t, red[w]);
+  return t;
+}
+
+// One candidate visual token per CTA (Sec. 4.2.1 and Eq. 6): E_ii = entropy of softmax(logits
+// row) / log V, F_itc = (cos(h_i, q_t) + 1) / 2 (0.5 without text), S_sa = ReLU(1 - E - F);
+// s_skip[i] += w1 S_sa + w2 SLC^Norm(l), flag[n] = s_skip[i] >= T_skip.
+__global__ void __launch_bounds__(kThreads)
+    skip_score_kernel(const float* __restrict__ logits, int V, const float* __restrict__ h, int D,
+                      const int32_t* __restrict__ cand, const int32_t* __restrict__ ts,
+                      const int32_t* __restrict__ seq_of, const float* __restrict__ tmean,
+                      float inv_log_v, float w1, float add_slc, float t_skip,
+                      float* __restrict__ s_skip, uint8_t* __restrict__ flag) {
+  __shared__ float red[kThreads / 32];
+  pdl_launch_dependents();
+  pdl_wait();
+  const int n = blockIdx.x, i = cand[n], b = seq_of[i];
+  const float* z = logits + size_t(n) * V;
+  float mx = -INFINITY;
+  for (int v = threadIdx.x; v < V; v += kThreads) mx = fmaxf(mx, z[v]);
+  mx = block_max(mx, red);
+  float se = 0.0f, te = 0.0f;  // sum e^(z - m) and sum e^(z - m) (z - m)
+  for (int v = threadIdx.x; v < V; v += kThreads) {
+    const float d = z[v] - mx, e = expf(d);
+    se += e;
+    te += e * d;
+  }
+  __syncthreads();
+  se = block_sum(se, red);
+  __syncthreads();
+  te = block_sum(te, red);
+  const float ent = (logf(se) - te / se) * inv_log_v;
+  const float* hi = h + size_t(i) * D;
+  const float* q = tmean + size_t(b) * D;
+  float dot = 0.0f, hh = 0.0f, qq = 0.0f;
+  for (int c = threadIdx.x; c < D; c += kThreads) {
+    dot += hi[c] * q[c];
+    hh += hi[c] * hi[c];
+    qq += q[c] * q[c];
+  }
+  __syncthreads();
+  dot = block_sum(dot, red);
+  __syncthreads();
+  hh = block_sum(hh, red);
+  __syncthreads();
+  qq = block_sum(qq, red);
+  if (threadIdx.x == 0) {
+    const bool has_text = ts[b + 1] > ts[b] && hh > 0.0f && qq > 0.0f;
+    const float f = has_text ? 0.5f + 0.5f * dot / (sqrtf(hh) * sqrtf(qq)) : 0.5f;
+    const float s_sa = fmaxf(0.0f, 1.0f - ent - f);
+    const float acc = s_skip[i] + (w1 * s_sa + add_slc);
+    s_skip[i] = acc;
+    flag[n] = acc >= t_skip ? 1 : 0;
+  }
+}
+
 }  // namespace
+
+int skip_scores_run(const float* logits, int V, int n_cand, const float* h, int D, const int32_t* cand,
+                    const int32_t* ts, const int32_t* text, const int32_t* seq_of, int B, float* tmean,
+                    float w1, float add_slc, float t_skip, float* s_skip, uint8_t* flag,
+                    cudaStream_t stream) {
+  SPD_CUDA_TRY(launch_pdl(text_mean_kernel, dim3((D + kThreads - 1) / kThreads, B), dim3(kThreads), 0,
+                          stream, h, D, ts, text, tmean));
+  SPD_CUDA_TRY(launch_pdl(skip_score_kernel, dim3(n_cand), dim3(kThreads), 0, stream,
+                          logits, V, h, D, cand, ts, seq_of, static_cast<const float*>(tmean),
+                          float(1.0 / log(double(V))), w1, add_slc, t_skip, s_skip, flag));
+  return SPD_OK;
+}
 
 int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float eps,
                 const int32_t* in_rows, void* out, const int32_t* map2, void* out2,

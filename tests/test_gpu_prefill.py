@@ -155,3 +155,68 @@ def test_llava_width_layer_with_cta_pairs():
     mask = np.zeros((1, T), np.uint8)
     mask[0, vis] = r.integers(0, 3, size=192)  # some tokens skip attention, some the FFN
     check(model, om, x, [0, T], mask)
+
+
+# ---- ASL-Skip online plan (Sec. 4.2, Eq. 6, Alg. 1 stage 2) ----------------------------------------
+def _adaptive_inputs(seed, lens, n_text):
+    cfg = dict(synth.TINY_DECODER, n_layers=6)
+    w = synth.decoder_weights(seed, cfg, std=0.05)
+    w["lm_head"] = (w["lm_head"].float() * 12.0).to(torch.bfloat16)  # peaked vocabularies: E_ii varies
+    om = od.model_from_torch(w, cfg)
+    wd = {k: v.cuda() for k, v in w.items() if k != "layers"}
+    wd["layers"] = [{k: v.cuda() for k, v in lw.items()} for lw in w["layers"]]
+    model = N.SpdModel(cfg, wd)
+    T = sum(lens)
+    x = inputs(T, cfg["d_model"], seed + 1)
+    vis = np.concatenate([np.r_[np.ones(n - t, bool), np.zeros(t, bool)] for n, t in zip(lens, n_text)])
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    return model, om, x, vis, cu
+
+
+def test_adaptive_plan_matches_oracle():
+    model, om, x, vis, cu = _adaptive_inputs(31, [64, 40], [16, 8])
+    slc = np.array([0.2, 0.5, 0.1, 0.7, 0.3, 0.9])
+    tgt = np.array([1, 2, 1, 1, 2, 2], np.uint8)
+    xn = bf16_np(x)
+    chosen = None
+    for t_skip in np.linspace(0.6, 2.6, 41):  # a threshold every decision clears by a margin
+        h0, lg0, admit0, target0, margin = od.prefill_adaptive(om, xn, cu, vis, slc, tgt, t_skip,
+                                                               3.0, 1.0, 3)
+        if margin > 0.05 and len(set(admit0[vis])) >= 2:
+            chosen = (t_skip, h0, lg0, admit0)
+            break
+    assert chosen is not None, "no well-separated threshold in the grid"
+    t_skip, h0, lg0, admit0 = chosen
+    T = x.shape[0]
+    ws = torch.zeros(N.spd_prefill_adaptive_workspace_size(model, T, len(cu) - 1), dtype=torch.uint8,
+                     device="cuda")
+    h = torch.full((T, 256), float("nan"), device="cuda")
+    logits = torch.full((len(cu) - 1, 512), float("nan"), device="cuda")
+    admit = N.spd_prefill_adaptive(model, x.cuda(), T, cu, vis, slc, tgt, t_skip, 3.0, 1.0, 3, h,
+                                   logits, ws)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    np.testing.assert_array_equal(admit.astype(np.int64), admit0)
+    assert np.all(admit[~vis] == -1) and np.all(admit < 3)
+    assert rowwise_rel(h.cpu().numpy(), h0) < TOL
+    assert rowwise_rel(logits.cpu().numpy(), lg0) < TOL
+
+
+def test_adaptive_plan_with_given_plan_is_the_plain_prefill():
+    # the same tokens, the plan the online rule chose, run through spd_prefill: the same result up
+    # to the order of the residual adds (split-K red.add), i.e. to fp32 rounding
+    model, om, x, vis, cu = _adaptive_inputs(33, [48], [16])
+    slc = np.full(6, 0.4)
+    tgt = np.array([2, 1, 2, 1, 2, 1], np.uint8)
+    T = x.shape[0]
+    ws = torch.zeros(N.spd_prefill_adaptive_workspace_size(model, T, 1), dtype=torch.uint8, device="cuda")
+    h1 = torch.zeros((T, 256), device="cuda")
+    lg1 = torch.zeros((1, 512), device="cuda")
+    admit = N.spd_prefill_adaptive(model, x.cuda(), T, cu, vis, slc, tgt, 0.9, 3.0, 1.0, 3, h1, lg1, ws)
+    torch.cuda.synchronize()
+    target = np.where(admit >= 0, tgt[np.maximum(admit, 0)], 0).astype(np.uint8)
+    plan = od.expand_adaptive_plan(admit.astype(np.int64), target, 6)
+    h2, lg2 = run(model, x.cuda(), cu, plan)
+    assert (admit >= 0).any()
+    assert rowwise_rel(h1.cpu().numpy(), h2) < 1e-5
+    assert rowwise_rel(lg1.cpu().numpy(), lg2) < 1e-5
