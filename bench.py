@@ -71,6 +71,17 @@ def gemm_traffic():
     return None
 
 
+def od_expand(admit, layer_target, n_layers):
+    """Per-layer skip bits of a frozen-target plan (token i bypasses layer_target[admit[i]] from
+    layer admit[i] on; -1 = never)."""
+    admit = np.asarray(admit, dtype=np.int64)
+    tgt = np.asarray(layer_target, dtype=np.uint8)
+    mask = np.zeros((n_layers, len(admit)), dtype=np.uint8)
+    for i in np.flatnonzero(admit >= 0):
+        mask[admit[i]:, i] = tgt[admit[i]]
+    return mask
+
+
 def workload_config(keep, mask, T):
     skipped = float(mask.astype(bool).sum() + (mask == 3).sum()) / (2.0 * mask.size)
     return {"workload": (f"llava-1.5-7b shape: 1 tile 1+576 x 1024 (ViT layers 12, 24), 16-head CLS "
@@ -396,6 +407,35 @@ def main():
     dense_gemm = {"ms_per_step": dg["ms"] / a.steps, "TFLOP/s": dense_tfs,
                   "tensor_frac_of_sustained": dense_tfs / tf_sust,
                   "GB/s": dg["bytes"] / (dg["ms"] / 1000.0) / 1e9}
+    # the same step with the skip plan computed online (Alg. 1 stage 2) at the paper's operating
+    # point: T_skip = 20, w1 / w2 = 3, decision window L / 2, targets m(l) of Table 9, SLC^Norm
+    # seeded in [0, 1] (the paper plots it but prints no values)
+    slc = np.random.default_rng(SEED).uniform(0.0, 1.0, L).astype(np.float32)
+    policy = {"slc_norm": slc, "layer_target": np.asarray(m_llava[:L], np.uint8), "t_skip": 20.0,
+              "w1": 3.0, "w2": 1.0, "window": L // 2}
+
+    def timed_policy(steps, warmup):
+        for _ in range(warmup):
+            spider.run(feats, attn, text, None, policy=policy)
+        torch.cuda.synchronize()
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0 = time.perf_counter()
+        s.record()
+        for _ in range(steps):
+            spider.run(feats, attn, text, None, policy=policy)
+        e.record()
+        torch.cuda.synchronize()
+        return s.elapsed_time(e) / steps, 1000.0 * (time.perf_counter() - t0) / steps
+
+    ms_ad, _ = timed_policy(a.steps, a.warmup)
+    admitted = float((spider.admit[spider.token_is_visual] >= 0).mean())
+    realized = od_expand(spider.admit, m_llava[:L], L)
+    ms_given = timed(spider, realized, a.steps, a.warmup)
+    adaptive = {"ms_per_step": ms_ad, "tokens_per_s": tokens / (ms_ad / 1000.0),
+                "admitted_visual_fraction": admitted,
+                "ms_per_step_same_plan_given": ms_given,
+                "online_plan_overhead_ms": ms_ad - ms_given,
+                "policy": "T_skip 20, w1 3, w2 1, window 16 (L/2), Table 9 targets, SLC^Norm seeded"}
     pb = prune_batch(torch, N, synth, dev, a.steps, a.warmup, hbm)
     ra = received_batch(torch, N, dev, a.steps, a.warmup, hbm)
 
@@ -440,7 +480,8 @@ def main():
                 "dense": {"value": tokens / (ms_dense / 1000.0), "ms_per_step": ms_dense,
                           "decoder_tokens": dense.T, "speedup_spider_vs_dense": ms_dense / ms},
                 "roofline": roof, "kernels": kernels, "dense_gemm": dense_gemm,
-                "prune_batch": pb, "received_attention": ra, "cpu_baseline": cpu,
+                "prune_batch": pb, "received_attention": ra, "adaptive_plan": adaptive,
+                "cpu_baseline": cpu,
                 "e2e": {"value": tokens / (ms_e2e / 1000.0), "unit": "tokens/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": hl.numel() * 4,
                         "ms_per_step": ms_e2e},

@@ -9,6 +9,7 @@ in the CUDA library:
                            vision width equals the decoder width and no projector is configured)
     spd_scatter_rows       text embeddings into their rows
     spd_prefill            decoder prefill with the per-layer, per-token skip mask (Sec. 4.2-4.3)
+    spd_prefill_adaptive   ... or with the skip plan computed online (Alg. 1 stage 2)
 
 Sequence layout per request: [kept visual tokens of its tiles, in tile order and spatial order;
 text tokens]. Alg. 1 writes the text first; the order is a layout choice of the caller and the
@@ -87,10 +88,15 @@ class SpiderPrefill:
                                     dtype=torch.uint8, device=dev) if self.has_projector else None)
         self.ws_prefill = torch.zeros(N.spd_prefill_workspace_size(model, self.T, self.B),
                                       dtype=torch.uint8, device=dev)
+        self.ws_adaptive = None
+        self.admit = None
 
-    def run(self, feats, attn, text, skip_mask, stream=None):
+    def run(self, feats, attn, text, skip_mask, stream=None, policy=None):
         """Enqueue one step on device inputs: feats (list of [n_tiles][n_tok][d_vis] fp32), attn,
-        text [sum(text_lens)][D] bf16. Returns the logits tensor [B][vocab] (device)."""
+        text [sum(text_lens)][D] bf16. Returns the logits tensor [B][vocab] (device).
+
+        policy (dict: slc_norm, layer_target, t_skip, w1, w2, window) replaces skip_mask by the
+        online ASL-Skip plan; the admission layer of every token is then left in self.admit."""
         if not self.dense:
             N.spd_prune(self.prune_cfg, feats, attn, self.keep_idx, ws=self.ws_prune, stream=stream)
         fin = int(self.prune_cfg.final_layer)
@@ -105,12 +111,21 @@ class SpiderPrefill:
         if len(self.text_rows):
             N.spd_scatter_rows(self.model, text, len(self.text_rows), self.text_rows, self.x,
                                stream=stream)
-        N.spd_prefill(self.model, self.x, self.T, self.cu, skip_mask, self.h, self.logits,
-                      self.ws_prefill, stream=stream)
+        if policy is None:
+            N.spd_prefill(self.model, self.x, self.T, self.cu, skip_mask, self.h, self.logits,
+                          self.ws_prefill, stream=stream)
+            return self.logits
+        if self.ws_adaptive is None:
+            self.ws_adaptive = torch.zeros(N.spd_prefill_adaptive_workspace_size(self.model, self.T, self.B),
+                                           dtype=torch.uint8, device=self.h.device)
+        self.admit = N.spd_prefill_adaptive(self.model, self.x, self.T, self.cu, self.token_is_visual,
+                                            policy["slc_norm"], policy["layer_target"], policy["t_skip"],
+                                            policy["w1"], policy["w2"], policy["window"], self.h,
+                                            self.logits, self.ws_adaptive, stream=stream)
         return self.logits
 
     def status(self) -> int:
         """First device-side failure recorded by any call of this pipeline (0 = none)."""
-        codes = [N.spd_workspace_status(w) for w in (self.ws_prune, self.ws_proj, self.ws_prefill)
-                 if w is not None]
+        codes = [N.spd_workspace_status(w) for w in (self.ws_prune, self.ws_proj, self.ws_prefill,
+                                                     self.ws_adaptive) if w is not None]
         return next((c for c in codes if c), 0)
