@@ -278,6 +278,33 @@ int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int n_tokens, co
                          int n_seqs, const spd_skip_policy* policy, int16_t* admit_layer, float* h,
                          float* logits, void* ws, size_t ws_bytes, void* stream);
 
+/* Bytes of a KV cache for n_seqs sequences of up to max_len tokens: per layer l, per sequence b,
+ * per position p, the row [K (rotated) | V] bf16 of 2 * n_kv_heads * head_dim values, at row
+ * (l * n_seqs + b) * max_len + p. The caller allocates it ZERO-FILLED: the attention reads key
+ * blocks past a sequence's length with zero weight, and unwritten rows must hold finite values. */
+size_t spd_kv_cache_bytes(const spd_model* m, int n_seqs, int max_len);
+
+/* spd_prefill that also leaves every layer's K and V of every token in kv_cache (sequence b's
+ * position p -> row b * max_len + p of each layer's block), for later decode steps. Tokens that
+ * bypass attention at a layer still write their K and V (they are keys and values of the others).
+ * The workspace is spd_prefill's. Errors as spd_prefill; SPD_EINVAL if a sequence exceeds max_len. */
+int spd_prefill_kv(const spd_model* m, const uint16_t* x, int n_tokens, const int32_t* cu_seqlens,
+                   int n_seqs, const uint8_t* skip_mask, float* h, float* logits, uint16_t* kv_cache,
+                   int max_len, void* ws, size_t ws_bytes, void* stream);
+
+/* Workspace bytes of spd_decode for n_seqs sequences. */
+size_t spd_decode_workspace_size(const spd_model* m, int n_seqs);
+
+/* One generation step after spd_prefill_kv: x (dev bf16 [n_seqs][d_model]) holds the embedding of
+ * each sequence's next token, at position pos[b] (HOST int32 [n_seqs], in [0, max_len)). Every
+ * layer appends the token's K and V to the cache and attends over positions 0..pos[b] of its
+ * sequence; a generated token is a text token and runs every sub-layer (the visual tokens' skip
+ * targets were applied when their cache rows were written). logits (dev fp32 [n_seqs][vocab]).
+ * Errors: SPD_EINVAL, SPD_ENOSPC, SPD_ECUDA. */
+int spd_decode(const spd_model* m, const uint16_t* x, int n_seqs, const int32_t* pos,
+               uint16_t* kv_cache, int max_len, float* logits, void* ws, size_t ws_bytes,
+               void* stream);
+
 /* ------------------------------------------------------------------------------------------ */
 /* Single kernels, exposed for composition and per-kernel tests                                 */
 /* ------------------------------------------------------------------------------------------ */

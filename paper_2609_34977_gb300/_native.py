@@ -25,7 +25,8 @@ EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait"
            "spd_model_destroy", "spd_plan_adaptive", "spd_plan_static", "spd_project_workspace_size",
            "spd_project", "spd_scatter_rows", "spd_attention_workspace_size", "spd_attention",
            "spd_prefill_workspace_size", "spd_prefill", "spd_prefill_adaptive_workspace_size",
-           "spd_prefill_adaptive",
+           "spd_prefill_adaptive", "spd_kv_cache_bytes", "spd_prefill_kv", "spd_decode_workspace_size",
+           "spd_decode",
            "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
            "spd_trace_read")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
@@ -99,6 +100,10 @@ def lib():
             "spd_prefill_workspace_size": (sz, [vp, i, i]),
             "spd_prefill": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, sz, vp]),
             "spd_prefill_adaptive_workspace_size": (sz, [vp, i, i]),
+            "spd_kv_cache_bytes": (sz, [vp, i, i]),
+            "spd_prefill_kv": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, i, vp, sz, vp]),
+            "spd_decode_workspace_size": (sz, [vp, i]),
+            "spd_decode": (i, [vp, vp, i, vp, vp, i, vp, vp, sz, vp]),
             "spd_prefill_adaptive": (i, [vp, vp, i, vp, i, C.POINTER(SkipPolicy), vp, vp, vp, vp, sz,
                                          vp]),
             "spd_linear_workspace_size": (sz, [i, i]),
@@ -291,6 +296,29 @@ def spd_prefill_adaptive(model: SpdModel, x, n_tokens, cu_seqlens, is_visual, sl
                                       C.byref(pol), admit.ctypes.data, _p(h), _p(logits), _p(ws),
                                       ws.numel() * ws.element_size(), _stream(stream)))
     return admit
+
+
+def spd_kv_cache_bytes(model: SpdModel, n_seqs: int, max_len: int) -> int:
+    return int(lib().spd_kv_cache_bytes(model.handle, n_seqs, max_len))
+
+
+def spd_prefill_kv(model: SpdModel, x, n_tokens, cu_seqlens, skip_mask, h, logits, kv_cache, max_len, ws,
+                   stream=None):
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    mk = None if skip_mask is None else np.ascontiguousarray(skip_mask, dtype=np.uint8)
+    _check(lib().spd_prefill_kv(model.handle, _p(x), n_tokens, cu.ctypes.data, len(cu) - 1,
+                                None if mk is None else mk.ctypes.data, _p(h), _p(logits), _p(kv_cache),
+                                max_len, _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def spd_decode_workspace_size(model: SpdModel, n_seqs: int) -> int:
+    return int(lib().spd_decode_workspace_size(model.handle, n_seqs))
+
+
+def spd_decode(model: SpdModel, x, pos, kv_cache, max_len, logits, ws, stream=None):
+    p = np.ascontiguousarray(pos, dtype=np.int32)
+    _check(lib().spd_decode(model.handle, _p(x), len(p), p.ctypes.data, _p(kv_cache), max_len,
+                            _p(logits), _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
 
 
 def spd_prefill(model: SpdModel, x, n_tokens, cu_seqlens, skip_mask, h, logits, ws, stream=None):

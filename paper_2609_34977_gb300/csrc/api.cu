@@ -510,8 +510,8 @@ struct PrefillBufs {
 size_t pad4(size_t n) { return (n + 3) & ~size_t(3); }
 size_t list_ints_for(int L, int T, int B) {
   // per layer: arows[T], amap[T], apos[T], frows[T], tiles[(T / 64 + B + 1) * 4]
-  // plus pos_all[T], last[B]
-  return size_t(L) * (4 * pad4(T) + 4 * (size_t(T) / 64 + B + 1)) + pad4(T) + pad4(B) + 16;
+  // plus pos_all[T], kvrow[T], last[B]
+  return size_t(L) * (4 * pad4(T) + 4 * (size_t(T) / 64 + B + 1)) + 2 * pad4(T) + pad4(B) + 16;
 }
 
 PrefillBufs carve_prefill(const spd_model_cfg& c, int T, int B, Carve& cv) {
@@ -551,23 +551,35 @@ struct LayerLists {
 struct HostPlan {
   std::vector<int32_t> hl;
   std::vector<int> pos_all, seq_of;
+  std::vector<int> kv0, kvlen;  // per sequence: first key row and key count of its attention
   std::vector<LayerLists> ll;
-  size_t pos_off = 0, last_off = 0, end = 0;
+  size_t pos_off = 0, kvrow_off = 0, last_off = 0, end = 0;
 };
 
-void plan_init(HostPlan& P, const spd_model_cfg& c, const int32_t* cu, int B, int T, size_t list_ints) {
+// Token t of sequence b = seq_of at position pos_all; its K/V row is kvrow (cache modes) or t.
+// Sequence b attends over key rows [kv0[b], kv0[b] + kvlen[b]).
+void plan_init(HostPlan& P, const spd_model_cfg& c, const int32_t* cu, int B, int T, size_t list_ints,
+               const int* pos = nullptr, int max_len = 0) {
   P.hl.assign(list_ints, 0);
   P.pos_all.assign(T, 0);
   P.seq_of.assign(T, 0);
-  for (int b = 0; b < B; ++b)
+  P.kv0.assign(B, 0);
+  P.kvlen.assign(B, 0);
+  for (int b = 0; b < B; ++b) {
     for (int t = cu[b]; t < cu[b + 1]; ++t) {
-      P.pos_all[t] = t - cu[b];
+      P.pos_all[t] = (pos ? pos[b] : 0) + t - cu[b];
       P.seq_of[t] = b;
     }
+    P.kv0[b] = max_len ? b * max_len : cu[b];
+    P.kvlen[b] = (pos ? pos[b] : 0) + cu[b + 1] - cu[b];
+  }
   P.ll.assign(c.n_layers, LayerLists{});
   size_t off = 0;
   P.pos_off = off;
   for (int t = 0; t < T; ++t) P.hl[off + t] = P.pos_all[t];
+  off += pad4(T);
+  P.kvrow_off = off;
+  for (int t = 0; t < T; ++t) P.hl[off + t] = max_len ? P.seq_of[t] * max_len + P.pos_all[t] : t;
   off += pad4(T);
   P.last_off = off;
   for (int b = 0; b < B; ++b) P.hl[off + b] = cu[b + 1] - 1;
@@ -611,8 +623,8 @@ void plan_layer(HostPlan& P, int l, const uint8_t* mk, const int32_t* cu, int B,
       int32_t* tl = &hl[q.tiles + 4 * size_t(q.ntiles++)];
       tl[0] = s0;
       tl[1] = (a_end - s0 < kAttnTileQ) ? a_end - s0 : kAttnTileQ;
-      tl[2] = cu[b];
-      tl[3] = cu[b + 1] - cu[b];
+      tl[2] = P.kv0[b];
+      tl[3] = P.kvlen[b];
     }
     a = a_end;
   }
@@ -627,9 +639,16 @@ int validate_prefill(const spd_model* m, const uint16_t* x, int T, const int32_t
   return SPD_OK;
 }
 
+// Where layer l's K and V go: the prefill's scratch (rows = tokens) or a cache block.
+struct KVDest {
+  uint16_t* kv;  // [n_rows][2 kvd]
+  int n_rows;
+  bool cache;    // rows from the plan's kvrow list
+};
+
 // Decoder layer l on the residual stream h with its lists at dl (device copy of the plan).
 int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P, const PrefillBufs& bf,
-              const int32_t* dl, float* h, int T, cudaStream_t st) {
+              const int32_t* dl, float* h, int T, cudaStream_t st, const KVDest* kvd_dest = nullptr) {
   const spd_model_cfg& c = m->cfg;
   const int D = c.d_model, hd = c.head_dim;
   const int qd = c.n_heads * hd, kvd = c.n_kv_heads * hd;
@@ -640,6 +659,8 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
   // contraction is weight-bound, one pass over Wq|Wk|Wv beats two launches)
   if ((rc = rmsnorm_run(h, T, D, W.attn_norm, c.rms_eps, nullptr, bf.xa, nullptr, nullptr, st)))
     return rc;
+  const KVDest dest = kvd_dest ? *kvd_dest : KVDest{bf.kv, T, false};
+  const int32_t* kvrow = dest.cache ? dl + P.kvrow_off : nullptr;
   GemmProblem kvp{};
   kvp.map_w = &W.m_kv;
   kvp.w = W.wkv;
@@ -648,8 +669,9 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
   kvp.n_tok = T;
   kvp.k = D;
   kvp.epi = EPI_ROPE_BF16;
-  kvp.out = bf.kv;
+  kvp.out = dest.kv;
   kvp.ldo = 2 * kvd;
+  kvp.rows = kvrow;
   kvp.pos = dl + P.pos_off;
   kvp.rope = m->freq;
   kvp.rope_rows = kvd;
@@ -663,7 +685,8 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
     qp.out = bf.q;
     qp.ldo = qd;
     qp.rows = dl + q.amap;
-    qp.out2 = bf.kv;
+    qp.out2 = dest.kv;
+    qp.rows2 = kvrow;
     qp.ldo2 = 2 * kvd;
     qp.split = qd;
     qp.n_tok_out = q.na;
@@ -672,7 +695,7 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
     return rc;
   }
   if (q.na > 0) {
-    if ((rc = attention_run(bf.q, q.na, bf.kv, T, 2 * kvd, kvd, bf.o, qd,
+    if ((rc = attention_run(bf.q, q.na, dest.kv, dest.n_rows, 2 * kvd, kvd, bf.o, qd,
                             reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
                             c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx)))
       return rc;
@@ -890,6 +913,90 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
     if (int rc = run_layer(m, l, q, P, bf, dl, h, T, st)) return rc;
   }
   for (int t = 0; t < T; ++t) admit_layer[t] = int16_t(admit[t]);
+  return run_head(m, P, bf, dl, h, B, logits, st);
+}
+
+// ---- KV cache and decode (the cache a prefill leaves for generation) --------------------------
+extern "C" size_t spd_kv_cache_bytes(const spd_model* m, int n_seqs, int max_len) {
+  if (!m || n_seqs < 1 || max_len < 1) return 0;
+  return size_t(m->cfg.n_layers) * n_seqs * max_len * 2 * m->cfg.n_kv_heads * m->cfg.head_dim *
+         sizeof(uint16_t);
+}
+
+extern "C" int spd_prefill_kv(const spd_model* m, const uint16_t* x, int T, const int32_t* cu, int B,
+                              const uint8_t* mask, float* h, float* logits, uint16_t* kv_cache,
+                              int max_len, void* ws, size_t ws_bytes, void* stream) {
+  if (int rc = validate_prefill(m, x, T, cu, B, h, ws)) return rc;
+  if (!kv_cache || max_len < 1) return fail(SPD_EINVAL, "null KV cache or max_len < 1");
+  for (int b = 0; b < B; ++b)
+    if (cu[b + 1] - cu[b] > max_len) return fail(SPD_EINVAL, "sequence %d is longer than max_len", b);
+  if (mask)
+    for (size_t i = 0; i < size_t(m->cfg.n_layers) * T; ++i)
+      if (mask[i] > 3) return fail(SPD_EINVAL, "skip mask entries must be in 0..3");
+  const spd_model_cfg& c = m->cfg;
+  Carve cv(ws, ws_bytes);
+  PrefillBufs bf = carve_prefill(c, T, B, cv);
+  if (!cv.fits()) return fail(SPD_ENOSPC, "prefill workspace too small (%zu < %zu)", ws_bytes, cv.used);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  static thread_local HostPlan P;
+  plan_init(P, c, cu, B, T, bf.list_ints, nullptr, max_len);
+  for (int l = 0; l < c.n_layers; ++l) plan_layer(P, l, mask ? mask + size_t(l) * T : nullptr, cu, B, T);
+  int32_t* dl = bf.lists;
+  SPD_CUDA_TRY(cudaMemcpyAsync(dl, P.hl.data(), P.end * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
+  if (int rc = bf16_to_f32_run(x, h, size_t(T) * c.d_model, st)) return rc;
+  const size_t layer_rows = size_t(B) * max_len, row = 2 * size_t(c.n_kv_heads) * c.head_dim;
+  for (int l = 0; l < c.n_layers; ++l) {
+    const KVDest dest{kv_cache + l * layer_rows * row, int(layer_rows), true};
+    if (int rc = run_layer(m, l, P.ll[l], P, bf, dl, h, T, st, &dest)) return rc;
+  }
+  return run_head(m, P, bf, dl, h, B, logits, st);
+}
+
+namespace {
+size_t carve_decode(const spd_model_cfg& c, int B, Carve& cv, PrefillBufs* bf, float** h) {
+  *bf = carve_prefill(c, B, B, cv);
+  *h = cv.take<float>(size_t(B) * c.d_model);
+  return cv.used;
+}
+}  // namespace
+
+extern "C" size_t spd_decode_workspace_size(const spd_model* m, int n_seqs) {
+  if (!m || n_seqs < 1) return 0;
+  Carve cv(nullptr, ~size_t(0));
+  PrefillBufs bf;
+  float* h;
+  return carve_decode(m->cfg, n_seqs, cv, &bf, &h);
+}
+
+extern "C" int spd_decode(const spd_model* m, const uint16_t* x, int B, const int32_t* pos,
+                          uint16_t* kv_cache, int max_len, float* logits, void* ws, size_t ws_bytes,
+                          void* stream) {
+  if (!m || !x || !pos || !kv_cache || !logits || !ws || B < 1 || max_len < 1)
+    return fail(SPD_EINVAL, "bad decode arguments");
+  for (int b = 0; b < B; ++b)
+    if (pos[b] < 0 || pos[b] >= max_len) return fail(SPD_EINVAL, "position of sequence %d outside [0, max_len)", b);
+  const spd_model_cfg& c = m->cfg;
+  Carve cv(ws, ws_bytes);
+  PrefillBufs bf;
+  float* h;
+  carve_decode(c, B, cv, &bf, &h);
+  if (!cv.fits()) return fail(SPD_ENOSPC, "decode workspace too small (%zu < %zu)", ws_bytes, cv.used);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  std::vector<int32_t> cu(B + 1);
+  for (int b = 0; b <= B; ++b) cu[b] = b;
+  static thread_local HostPlan P;
+  plan_init(P, c, cu.data(), B, B, bf.list_ints, pos, max_len);
+  for (int l = 0; l < c.n_layers; ++l) plan_layer(P, l, nullptr, cu.data(), B, B);
+  int32_t* dl = bf.lists;
+  SPD_CUDA_TRY(cudaMemcpyAsync(dl, P.hl.data(), P.end * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
+  if (int rc = bf16_to_f32_run(x, h, size_t(B) * c.d_model, st)) return rc;
+  const size_t layer_rows = size_t(B) * max_len, row = 2 * size_t(c.n_kv_heads) * c.head_dim;
+  for (int l = 0; l < c.n_layers; ++l) {
+    const KVDest dest{kv_cache + l * layer_rows * row, int(layer_rows), true};
+    if (int rc = run_layer(m, l, P.ll[l], P, bf, dl, h, B, st, &dest)) return rc;
+  }
   return run_head(m, P, bf, dl, h, B, logits, st);
 }
 

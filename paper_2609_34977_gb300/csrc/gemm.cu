@@ -88,6 +88,7 @@ struct KArgs {
   void* out;
   void* out2;
   const int32_t* rows;
+  const int32_t* rows2;  // EPI_QKV_BF16: row of token t in out2 (null = t)
   const uint16_t* bias;
   const int32_t* pos;
   const float2* rope;  // [head_dim / 2] rotary frequency theta^(-2j / head_dim) as fp32 (hi, lo)
@@ -284,12 +285,13 @@ __device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane
       __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out2);
       const int nn = n - a.split;
       if (nn < a.rope_rows) {
-        rope_store8(a, o, a.ldo2, nn, lane, t0, v, tpos, tb, [](int t) { return t; });
+        rope_store8(a, o, a.ldo2, nn, lane, t0, v, tpos, tb,
+                    [&](int t) { return a.rows2 ? a.rows2[t] : t; });
       } else if (n < a.n_out) {
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const int t = t0 + j;
-          if (t < nt) o[size_t(t) * a.ldo2 + nn] = __float2bfloat16_rn(v[j]);
+          if (t < nt) o[size_t(a.rows2 ? a.rows2[t] : t) * a.ldo2 + nn] = __float2bfloat16_rn(v[j]);
         }
       }
     }
@@ -1108,6 +1110,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.ldo2 = p.ldo2;
   a.split = p.split;
   a.rows = p.rows;
+  a.rows2 = p.rows2;
   a.bias = p.bias;
   a.pos = p.pos;
   a.rope = reinterpret_cast<const float2*>(p.rope);

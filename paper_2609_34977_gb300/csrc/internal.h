@@ -89,6 +89,7 @@ struct GemmProblem {
   int rope_rows, head_dim;
   int out_cols;              // valid output columns (SwiGLU: d_ffn)
   void* out2;                // EPI_QKV_BF16: second output, row stride ldo2, from weight row split
+  const int32_t* rows2;      // EPI_QKV_BF16: row of token t in out2 (null = t)
   int ldo2, split;
   int n_tok_out;             // EPI_QKV_BF16: tokens whose first-output rows are stored (tracing)
 };

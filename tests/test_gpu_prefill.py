@@ -220,3 +220,69 @@ def test_adaptive_plan_with_given_plan_is_the_plain_prefill():
     assert (admit >= 0).any()
     assert rowwise_rel(h1.cpu().numpy(), h2) < 1e-5
     assert rowwise_rel(lg1.cpu().numpy(), lg2) < 1e-5
+
+
+# ---- KV cache and decode steps ---------------------------------------------------------------------
+def _decode_case(seed, lens, n_vis, n_layers=3):
+    cfg = dict(synth.TINY_DECODER, n_layers=n_layers)
+    model, om = build(cfg, seed)
+    T = sum(lens)
+    x = inputs(T, cfg["d_model"], seed + 1)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    vis = np.concatenate([np.r_[np.ones(v, bool), np.zeros(n - v, bool)] for n, v in zip(lens, n_vis)])
+    r = np.random.default_rng(seed)
+    mask = np.zeros((n_layers, T), np.uint8)
+    mask[:, vis] = r.integers(0, 3, size=(n_layers, int(vis.sum())))
+    return cfg, model, om, x, cu, mask
+
+
+def test_prefill_kv_equals_prefill_and_fills_the_cache():
+    cfg, model, om, x, cu, mask = _decode_case(41, [30, 45], [20, 30])
+    T, B, max_len = x.shape[0], 2, 64
+    h0, lg0 = run(model, x.cuda(), cu, mask)
+    cache = torch.zeros(N.spd_kv_cache_bytes(model, B, max_len) // 2, dtype=torch.bfloat16, device="cuda")
+    ws = torch.zeros(N.spd_prefill_workspace_size(model, T, B), dtype=torch.uint8, device="cuda")
+    h = torch.zeros((T, cfg["d_model"]), device="cuda")
+    lg = torch.zeros((B, cfg["vocab"]), device="cuda")
+    N.spd_prefill_kv(model, x.cuda(), T, cu, mask, h, lg, cache, max_len, ws)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    # the cache layout moves each sequence's keys to its own slot, which changes how the attention
+    # groups keys into blocks (and so where P is rounded to bf16): equal within the tolerance
+    assert rowwise_rel(h.cpu().numpy(), h0) < TOL and rowwise_rel(lg.cpu().numpy(), lg0) < TOL
+    ho, lo = od.prefill(om, bf16_np(x), cu, mask)
+    assert rowwise_rel(h.cpu().numpy(), ho) < TOL and rowwise_rel(lg.cpu().numpy(), lo) < TOL
+    kvd = 2 * cfg["n_kv_heads"] * cfg["head_dim"]
+    c = bf16_np(cache).reshape(cfg["n_layers"], B, max_len, kvd)
+    for b, n in enumerate([30, 45]):
+        assert np.abs(c[:, b, :n]).max() > 0 and not c[:, b, n:].any()  # written rows only
+
+
+@pytest.mark.parametrize("steps", [1, 2])
+def test_decode_steps_equal_prefill_of_the_extended_sequences(steps):
+    lens, n_vis = [30, 45], [20, 30]
+    cfg, model, om, x, cu, mask = _decode_case(43, lens, n_vis)
+    T, B, max_len, D = x.shape[0], 2, 64, cfg["d_model"]
+    cache = torch.zeros(N.spd_kv_cache_bytes(model, B, max_len) // 2, dtype=torch.bfloat16, device="cuda")
+    ws = torch.zeros(N.spd_prefill_workspace_size(model, T, B), dtype=torch.uint8, device="cuda")
+    h = torch.zeros((T, D), device="cuda")
+    lg = torch.zeros((B, cfg["vocab"]), device="cuda")
+    N.spd_prefill_kv(model, x.cuda(), T, cu, mask, h, lg, cache, max_len, ws)
+    new = inputs(B * steps, D, 44).reshape(steps, B, D)  # generated-token embeddings
+    wsd = torch.zeros(N.spd_decode_workspace_size(model, B), dtype=torch.uint8, device="cuda")
+    out = torch.full((B, cfg["vocab"]), float("nan"), device="cuda")
+    for s in range(steps):
+        N.spd_decode(model, new[s].contiguous().cuda(), np.array(lens) + s, cache, max_len, out, wsd)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(wsd) == 0
+    # oracle: each sequence extended by its generated tokens (text tokens: no skipping)
+    xs, masks, cu_e = [], [], [0]
+    for b in range(B):
+        xb = bf16_np(x[cu[b]:cu[b + 1]])
+        xs.append(np.concatenate([xb] + [bf16_np(new[s, b:b + 1]) for s in range(steps)]))
+        masks.append(np.concatenate([mask[:, cu[b]:cu[b + 1]], np.zeros((cfg["n_layers"], steps), np.uint8)], 1))
+        cu_e.append(cu_e[-1] + lens[b] + steps)
+    _, lo = od.prefill(om, np.concatenate(xs), cu_e, np.concatenate(masks, 1))
+    got = out.cpu().numpy()
+    assert np.isfinite(got).all()
+    assert rowwise_rel(got, lo) < TOL
