@@ -223,6 +223,41 @@ def received_batch(torch, N, dev, steps, warmup, hbm, images=4, heads=16, grid=6
                     f"attention -> {n // 4} post-merger tokens (2 x 2 merger)"}
 
 
+def decode_steps(torch, N, spider, mask, dev, steps, warmup, hbm, max_len=512):
+    """Generation after the SPIDER prefill (batch 1): spd_prefill_kv leaves the K/V of the pruned,
+    skip-planned sequence in a cache, then spd_decode steps one token at a time. Algorithmic bytes
+    per step: every weight of the decoder and the LM head once, plus the cache rows read."""
+    model = spider.model
+    cfg = model.cfg
+    cache = torch.zeros(N.spd_kv_cache_bytes(model, 1, max_len) // 2, dtype=torch.bfloat16, device=dev)
+    N.spd_prefill_kv(model, spider.x, spider.T, spider.cu, mask, spider.h, spider.logits, cache, max_len,
+                     spider.ws_prefill)
+    ws = torch.zeros(N.spd_decode_workspace_size(model, 1), dtype=torch.uint8, device=dev)
+    x = torch.randn(1, cfg["d_model"], device=dev).to(torch.bfloat16)
+    out = torch.empty(1, cfg["vocab"], device=dev)
+    pos = spider.T
+    for _ in range(warmup):
+        N.spd_decode(model, x, [pos], cache, max_len, out, ws)
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for k in range(steps):
+        N.spd_decode(model, x, [pos + k], cache, max_len, out, ws)
+    e.record()
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0, "device-side failure recorded"
+    ms = s.elapsed_time(e) / steps
+    L, D, F, V = cfg["n_layers"], cfg["d_model"], cfg["d_ffn"], cfg["vocab"]
+    kvd = cfg["n_kv_heads"] * cfg["head_dim"]
+    qd = cfg["n_heads"] * cfg["head_dim"]
+    wbytes = 2.0 * (L * (D * (qd + 2 * kvd) + qd * D + 3 * D * F) + V * D)
+    cbytes = 2.0 * L * (pos + steps / 2) * 2 * kvd
+    gbs = (wbytes + cbytes) / (ms / 1000.0) / 1e9
+    return {"ms_per_token": ms, "tokens_per_s": 1000.0 / ms, "context": pos, "GB/s": gbs,
+            "hbm_frac": gbs / hbm,
+            "what": "spd_decode, batch 1, after spd_prefill_kv of the SPIDER sequence (pruned, skip plan)"}
+
+
 def cpu_baseline_sample(keep, v, mask_fn, reps=1):
     """The oracle as it stands on the host cores: MSV-Prune of the tile, the projector, and 1- and
     2-layer decoder prefills of the same token count; the step time is extrapolated to 32 layers."""
@@ -438,6 +473,7 @@ def main():
                 "policy": "T_skip 20, w1 3, w2 1, window 16 (L/2), Table 9 targets, SLC^Norm seeded"}
     pb = prune_batch(torch, N, synth, dev, a.steps, a.warmup, hbm)
     ra = received_batch(torch, N, dev, a.steps, a.warmup, hbm)
+    dec = decode_steps(torch, N, spider, mask, dev, a.steps, a.warmup, hbm)
 
     # end to end through the public API: pinned host inputs -> device, step, logits -> host
     hf = [f.cpu().pin_memory() for f in feats]
@@ -480,7 +516,7 @@ def main():
                 "dense": {"value": tokens / (ms_dense / 1000.0), "ms_per_step": ms_dense,
                           "decoder_tokens": dense.T, "speedup_spider_vs_dense": ms_dense / ms},
                 "roofline": roof, "kernels": kernels, "dense_gemm": dense_gemm,
-                "prune_batch": pb, "received_attention": ra, "adaptive_plan": adaptive,
+                "prune_batch": pb, "received_attention": ra, "adaptive_plan": adaptive, "decode": dec,
                 "cpu_baseline": cpu,
                 "e2e": {"value": tokens / (ms_e2e / 1000.0), "unit": "tokens/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": hl.numel() * 4,
