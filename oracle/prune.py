@@ -92,14 +92,55 @@ def unit_rows(f: np.ndarray) -> np.ndarray:
     return f / np.sqrt((f * f).sum(axis=1, keepdims=True))
 
 
-def anchor_similarity(fl_unit: np.ndarray, anchors: np.ndarray) -> np.ndarray:
+SIM_KINDS = ("cos", "mse", "kl")
+
+
+def log_softmax_rows(f: np.ndarray) -> np.ndarray:
+    """log of the softmax of every row over the feature dimension (shifted by the row maximum)."""
+    f = np.asarray(f, dtype=np.float64)
+    z = f - f.max(axis=1, keepdims=True)
+    return z - np.log(np.exp(z).sum(axis=1, keepdims=True))
+
+
+def similarity(a: np.ndarray, b: np.ndarray, kind: str = "cos") -> np.ndarray:
+    """sim(F_i, F_j) of Eq. 3 for every row i of a and row j of b, as an [len(a)][len(b)] matrix.
+
+    cos: the cosine similarity, the paper's choice.
+    mse, kl: the ablation of the MSV-Prune table, part (c), that puts the mean squared error or the
+    Kullback-Leibler divergence in place of the cosine. Both measure dissimilarity, so they enter
+    Eq. 3 negated: a larger value still means more alike, and the N_k lowest-scoring tokens of a
+    cluster are still its least redundant ones (reading: the paper names only the replacement).
+      mse: -(1/d) sum_k (a_ik - b_jk)^2
+      kl:  -KL(P_i || Q_j) = -sum_k P_ik (log P_ik - log Q_jk), with P_i and Q_j the softmax of the
+           rows over the feature dimension (reading: features are not distributions, and the
+           softmax is what makes them ones).
+    """
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    if kind == "cos":
+        return unit_rows(a) @ unit_rows(b).T
+    out = np.empty((len(a), len(b)))
+    if kind == "mse":
+        for i in range(len(a)):  # one row of the matrix at a time (bounded memory)
+            out[i] = -((b - a[i]) ** 2).mean(axis=1)
+        return out
+    if kind == "kl":
+        la, lb = log_softmax_rows(a), log_softmax_rows(b)
+        for i in range(len(a)):
+            out[i] = -(np.exp(la[i]) * (la[i] - lb)).sum(axis=1)
+        return out
+    raise ValueError(f"unknown similarity kind {kind!r}")
+
+
+def anchor_similarity(f_final: np.ndarray, anchors: np.ndarray, kind: str = "cos") -> np.ndarray:
     """max over anchors p of sim(F^L_i, F^L_p), for every token i (Eq. 3, second bracket).
 
     With no anchors (r = 0) the term is absent and 0 is returned.
     """
     if len(anchors) == 0:
-        return np.zeros(len(fl_unit))
-    return (fl_unit @ fl_unit[anchors].T).max(axis=1)
+        return np.zeros(len(f_final))
+    f_final = np.asarray(f_final, dtype=np.float64)
+    return similarity(f_final, f_final[anchors], kind).max(axis=1)
 
 
 def kmeans(x: np.ndarray, k: int, iters: int):
@@ -182,27 +223,35 @@ def cluster_quotas(sizes, n_cmp: int):
     return quota
 
 
-def pairwise_scores(members, units_final, units_other, other_weights, a_anchor):
+def pairwise_scores(members, feats_final, feats_other, other_weights, a_anchor, *, kind="cos",
+                    use_final_sim=True, use_anchor_sim=True):
     """Eq. 3 for the tokens of one cluster, reduced to one score per token.
 
     S_ij = sim(F^L_i, F^L_j) + sim(F^M_i, F^M_j) + max_p sim(F^L_i, F^L_p) + max_p sim(F^L_j, F^L_p).
-    The paper selects "the N_k lowest-scoring tokens" of each cluster from this pairwise score; the
+    The paper selects the N_k lowest-scoring tokens of each cluster from this pairwise score; the
     per-token score read here is the mean of S_ij over the other members j != i of the cluster. The
     intra-cluster term sums every tapped non-final layer with its weight (one middle layer with
     weight 1 in the paper). A singleton cluster has no pair; its token scores 2 * a_i.
+
+    Ablations of the MSV-Prune table: `kind` replaces the cosine (see similarity); without the
+    final-layer term (use_final_sim False: "only middle layer tokens" in the intra-cluster part)
+    and without the anchor bracket (use_anchor_sim False). A zero weight of the middle layer gives
+    "without middle layer tokens".
 
     Computed literally: the full |C| x |C| matrix of S_ij, diagonal excluded.
     """
     members = np.asarray(members)
     c = len(members)
-    a = a_anchor[members]
+    a = a_anchor[members] if use_anchor_sim else np.zeros(c)
     if c == 1:
         return 2.0 * a
-    u = units_final[members]
-    s = u @ u.T
-    for w, uo in zip(other_weights, units_other):
-        v = uo[members]
-        s = s + w * (v @ v.T)
+    s = np.zeros((c, c))
+    if use_final_sim:
+        f = feats_final[members]
+        s = s + similarity(f, f, kind)
+    for w, fo in zip(other_weights, feats_other):
+        v = fo[members]
+        s = s + w * similarity(v, v, kind)
     s = s + a[:, None] + a[None, :]
     np.fill_diagonal(s, 0.0)
     return s.sum(axis=1) / (c - 1)
@@ -210,8 +259,12 @@ def pairwise_scores(members, units_final, units_other, other_weights, a_anchor):
 
 def prune_tile(feats, attn_tile, *, has_cls: bool, attn_form: int, final_layer: int, keep: int,
                n_clusters: int = 4, kmeans_iters: int = 10, anchor_ratio: float = 0.7,
-               layer_weight=None):
+               layer_weight=None, sim: str = "cos", use_final_sim: bool = True,
+               use_anchor_sim: bool = True):
     """MSV-Prune of one tile (Alg. 1 stage 1): anchors, clustering, scoring, per-cluster selection.
+
+    sim, use_final_sim, use_anchor_sim: the ablations of pairwise_scores (the paper's method is
+    cos, True, True); n_clusters = 1 is the ablation without semantic clustering.
 
     feats: list over tapped layers of [n_tok][d] arrays (row 0 is [CLS] when has_cls, never kept).
     Returns a dict with keep_idx (ascending patch indices, length keep), kind (0 dropped, 1 anchor,
@@ -237,9 +290,11 @@ def prune_tile(feats, attn_tile, *, has_cls: bool, attn_form: int, final_layer: 
     is_anchor[anchors] = True
     rest = np.flatnonzero(~is_anchor)
 
-    units_final = unit_rows(patch[final_layer])
-    units_other = [unit_rows(patch[l]) for l in others]
-    a_sim = anchor_similarity(units_final, anchors)
+    if sim not in SIM_KINDS:
+        raise ValueError(f"unknown similarity kind {sim!r}")
+    feats_final = patch[final_layer]
+    feats_other = [patch[l] for l in others]
+    a_sim = anchor_similarity(feats_final, anchors, sim) if use_anchor_sim else np.zeros(n)
 
     assign, km_margin = kmeans(patch[final_layer][rest], n_clusters, kmeans_iters)
     sizes = [int((assign == k).sum()) for k in range(n_clusters)]
@@ -254,8 +309,9 @@ def prune_tile(feats, attn_tile, *, has_cls: bool, attn_form: int, final_layer: 
         members = rest[assign == k]
         if len(members) == 0:
             continue
-        s = pairwise_scores(members, units_final, units_other,
-                            [layer_weight[l] for l in others], a_sim)
+        s = pairwise_scores(members, feats_final, feats_other, [layer_weight[l] for l in others],
+                            a_sim, kind=sim, use_final_sim=use_final_sim,
+                            use_anchor_sim=use_anchor_sim)
         scores[members] = s
         order = sorted(range(len(members)), key=lambda j: (s[j], members[j]))
         selected.extend(members[order[:quotas[k]]].tolist())
@@ -274,7 +330,8 @@ def prune_tile(feats, attn_tile, *, has_cls: bool, attn_form: int, final_layer: 
 
 
 def prune(feats, attn, *, has_cls=True, attn_form=0, final_layer=-1, keep=64, n_clusters=4,
-          kmeans_iters=10, anchor_ratio=0.7, layer_weight=None):
+          kmeans_iters=10, anchor_ratio=0.7, layer_weight=None, sim="cos", use_final_sim=True,
+          use_anchor_sim=True):
     """MSV-Prune of every tile independently (AnyRes: same rule and budget per tile, §5.1).
 
     feats: list over tapped layers of [n_tiles][n_tok][d]; attn: [n_tiles][H][n_att].
@@ -285,7 +342,8 @@ def prune(feats, attn, *, has_cls=True, attn_form=0, final_layer=-1, keep=64, n_
         out.append(prune_tile([f[t] for f in feats], attn[t], has_cls=has_cls, attn_form=attn_form,
                               final_layer=final_layer, keep=keep, n_clusters=n_clusters,
                               kmeans_iters=kmeans_iters, anchor_ratio=anchor_ratio,
-                              layer_weight=layer_weight))
+                              layer_weight=layer_weight, sim=sim, use_final_sim=use_final_sim,
+                              use_anchor_sim=use_anchor_sim))
     return out
 
 

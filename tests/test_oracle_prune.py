@@ -261,3 +261,129 @@ def test_merge_groups_2x2_partition_the_grid_into_blocks():
     assert g[0] == [0, 1, 6, 7] and g[1] == [2, 3, 8, 9] and g[3] == [12, 13, 18, 19]
     flat = sorted(i for members in g for i in members)
     assert flat == list(range(24))
+
+
+# ---- ablation variants of the MSV-Prune table (K, middle-layer and anchor terms, sim kinds) ----
+def _sim_brute(x, y, kind):
+    """One pair's similarity computed through library routines, not the oracle's formulas."""
+    from scipy.spatial.distance import sqeuclidean
+    from scipy.special import softmax
+    from scipy.stats import entropy
+    if kind == "cos":
+        return _cos(x, y)
+    if kind == "mse":
+        return -sqeuclidean(x, y) / len(x)
+    return -float(entropy(softmax(x), softmax(y)))
+
+
+@pytest.mark.parametrize("kind", ["cos", "mse", "kl"])
+def test_similarity_kinds_against_library_routines(kind):
+    r = np.random.default_rng(21)
+    a, b = r.standard_normal((5, 9)), 2.0 * r.standard_normal((4, 9))
+    expect = [[_sim_brute(a[i], b[j], kind) for j in range(4)] for i in range(5)]
+    np.testing.assert_allclose(op.similarity(a, b, kind), expect, rtol=0, atol=1e-12)
+
+
+def test_similarity_kinds_invariances():
+    r = np.random.default_rng(22)
+    a, b = r.standard_normal((6, 8)), r.standard_normal((5, 8))
+    base = {k: op.similarity(a, b, k) for k in op.SIM_KINDS}
+    # cosine: positive scaling of any row; MSE: one translation of all rows; KL (of softmaxes): a
+    # constant added to any row
+    s = r.uniform(0.5, 3.0, (6, 1))
+    np.testing.assert_allclose(op.similarity(a * s, b, "cos"), base["cos"], atol=1e-12)
+    t = r.standard_normal(8)
+    np.testing.assert_allclose(op.similarity(a + t, b + t, "mse"), base["mse"], atol=1e-12)
+    c = r.standard_normal((6, 1))
+    np.testing.assert_allclose(op.similarity(a + c, b, "kl"), base["kl"], atol=1e-12)
+    # a row compared with itself: cosine 1, no distance, no divergence; others never exceed that
+    for k, top in (("cos", 1.0), ("mse", 0.0), ("kl", 0.0)):
+        g = op.similarity(a, a, k)
+        np.testing.assert_allclose(np.diag(g), top, atol=1e-12)
+        assert (g <= top + 1e-12).all()
+
+
+@pytest.mark.parametrize("kind,use_final,use_anchor", [
+    ("cos", False, True), ("cos", True, False), ("mse", True, True), ("kl", True, True),
+    ("mse", False, False), ("kl", True, False)])
+def test_ablated_pairwise_scores_against_explicit_pair_loop(kind, use_final, use_anchor):
+    r = np.random.default_rng(23)
+    n, d = 8, 6
+    fl, fm = r.standard_normal((n, d)), r.standard_normal((n, d))
+    anchors = [2, 6]
+    members = [0, 1, 3, 4, 7]
+    a = {i: max(_sim_brute(fl[i], fl[p], kind) for p in anchors) for i in range(n)}
+    expect = []
+    for i in members:
+        tot = 0.0
+        for j in members:
+            if j != i:
+                tot += ((_sim_brute(fl[i], fl[j], kind) if use_final else 0.0)
+                        + 0.75 * _sim_brute(fm[i], fm[j], kind)
+                        + ((a[i] + a[j]) if use_anchor else 0.0))
+        expect.append(tot / (len(members) - 1))
+    a_arr = op.anchor_similarity(fl, np.array(anchors), kind)
+    got = op.pairwise_scores(np.array(members), fl, [fm], [0.75], a_arr, kind=kind,
+                             use_final_sim=use_final, use_anchor_sim=use_anchor)
+    np.testing.assert_allclose(got, expect, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("kind", ["cos", "mse", "kl"])
+def test_outlier_is_kept_over_near_duplicates(kind):
+    # ten near-copies of one row and one unrelated row, one cluster, no anchors, keep 1: the
+    # unrelated row is the least redundant under every similarity kind
+    r = np.random.default_rng(24)
+    d = 16
+    base = r.standard_normal(d)
+    rows = [base + 0.05 * r.standard_normal(d) for _ in range(10)]
+    rows.insert(7, -base + 0.5 * r.standard_normal(d))
+    f = np.vstack([np.zeros(d), np.array(rows)])  # row 0 is [CLS]
+    attn = r.uniform(size=(1, 12))
+    res = op.prune_tile([f, f], attn, has_cls=True, attn_form=0, final_layer=1, keep=1, n_clusters=1,
+                        anchor_ratio=0.0, sim=kind)
+    np.testing.assert_array_equal(res["keep_idx"], [7])
+
+
+def test_without_anchor_term_anchor_features_do_not_matter():
+    v = synth.vision_tiles(25, 1, 144, 32, 2, 4)
+    feats = [f[0].copy() for f in v["feats"]]
+    kw = dict(has_cls=True, attn_form=0, final_layer=1, keep=40, anchor_ratio=0.5)
+    ref = op.prune_tile(feats, v["attn"][0], use_anchor_sim=False, **kw)
+    anchors = np.flatnonzero(ref["kind"] == 1)
+    moved = [f.copy() for f in feats]
+    for f in moved:
+        f[1 + anchors] = np.random.default_rng(26).standard_normal((len(anchors), f.shape[1]))
+    got = op.prune_tile(moved, v["attn"][0], use_anchor_sim=False, **kw)
+    np.testing.assert_array_equal(got["keep_idx"], ref["keep_idx"])
+    np.testing.assert_array_equal(got["scores"], ref["scores"])
+    # with the anchor term the same move changes the scores
+    with_term = op.prune_tile(feats, v["attn"][0], **kw)
+    moved_term = op.prune_tile(moved, v["attn"][0], **kw)
+    assert not np.allclose(with_term["scores"][ref["kind"] != 1], moved_term["scores"][ref["kind"] != 1])
+
+
+def test_only_middle_layer_scores_ignore_final_layer_beyond_clustering():
+    # without the final-layer term, F^L enters only through K = 1 clustering (trivial) and the
+    # anchor bracket (dropped too): the scores are those of the middle layer alone
+    r = np.random.default_rng(27)
+    n, d = 20, 8
+    fm, fl = r.standard_normal((n + 1, d)), r.standard_normal((n + 1, d))
+    attn = r.uniform(size=(1, n + 1))
+    kw = dict(has_cls=True, attn_form=0, final_layer=1, keep=6, n_clusters=1, anchor_ratio=0.0,
+              use_final_sim=False)
+    a = op.prune_tile([fm, fl], attn, **kw)
+    b = op.prune_tile([fm, r.standard_normal((n + 1, d))], attn, **kw)
+    np.testing.assert_array_equal(a["scores"], b["scores"])
+    g = np.array([[_cos(fm[1 + i], fm[1 + j]) for j in range(n)] for i in range(n)])
+    np.testing.assert_allclose(a["scores"], (g.sum(1) - 1.0) / (n - 1), atol=1e-12)
+
+
+@pytest.mark.parametrize("K", [1, 2, 8])
+def test_cluster_count_variants_keep_the_budget(K):
+    v = synth.vision_tiles(28, 1, 576, 32, 2, 4)
+    res = op.prune(v["feats"], v["attn"], keep=64, final_layer=1, n_clusters=K)[0]
+    assert len(res["keep_idx"]) == 64
+    assert sum(res["quotas"]) == 64 - op.n_anchor_tokens(64, 0.7)
+    c = res["cluster"][res["kind"] != 1]
+    assert c.min() >= 0 and c.max() < K
+    assert all(q >= 1 for q, sz in zip(res["quotas"], res["sizes"]) if sz > 0)
