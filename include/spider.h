@@ -87,8 +87,26 @@ typedef struct {
   int kmeans_iters; /* maximum Lloyd assignment steps, >= 1 (stops early on a repeated assignment) */
   double anchor_ratio; /* r in [0, 1]; N_anc = floor(keep * r + 0.5), N_cmp = keep - N_anc */
   float layer_weight[SPD_MAX_FEAT_LAYERS]; /* weight of each non-final layer's intra-cluster cosine
-                       term in the score; 1 everywhere reproduces Eq. 3 (entry of final_layer unused) */
+                       term in the score; 1 everywhere reproduces Eq. 3 (entry of final_layer unused);
+                       0 for the middle layer is the ablation without middle-layer tokens */
+  int sim_kind;     /* sim() of Eq. 3: SPD_SIM_COS (the paper's) or an ablation below */
+  int ablate;       /* bit set of SPD_PRUNE_NO_* below; 0 = Eq. 3 as printed */
 } spd_prune_cfg;
+
+/* Similarity kinds of Eq. 3 (the MSV-Prune ablation table, part (c)). The two dissimilarities enter
+ * negated, so that the N_k lowest-scoring tokens stay the least redundant ones:
+ *   SPD_SIM_COS  cos(F_i, F_j)
+ *   SPD_SIM_MSE  -(1/d) sum_c (F_i,c - F_j,c)^2
+ *   SPD_SIM_KL   -KL(softmax(F_i) || softmax(F_j)), softmax over the feature dimension.
+ * Ablation bits: SPD_PRUNE_NO_FINAL_SIM drops sim(F^L_i, F^L_j) from the intra-cluster bracket
+ * (with a middle layer: "only middle layer tokens"; with a zero middle weight as well: no
+ * intra-cluster term); SPD_PRUNE_NO_ANCHOR_SIM drops the bracket of similarities to the anchors.
+ * n_clusters = 1 is the ablation without semantic clustering. */
+#define SPD_SIM_COS 0
+#define SPD_SIM_MSE 1
+#define SPD_SIM_KL 2
+#define SPD_PRUNE_NO_FINAL_SIM 1
+#define SPD_PRUNE_NO_ANCHOR_SIM 2
 
 /* Bytes of device workspace spd_prune needs for `cfg` (0 if cfg is invalid). */
 size_t spd_prune_workspace_size(const spd_prune_cfg* cfg);
@@ -100,6 +118,7 @@ size_t spd_prune_workspace_size(const spd_prune_cfg* cfg);
  *   on F^L of the non-anchor tokens; quotas N_k by Eq. 2 made to sum to N_cmp; per-token score =
  *   mean over the other members j of the cluster of S_ij (Eq. 3); in each cluster the N_k
  *   lowest-scoring tokens (ties to the lower index) join the anchors; kept indices ascending.
+ *   sim_kind and ablate select the ablation variants of Eq. 3 described above.
  * feats    (host array of n_layers dev pointers) each [n_tiles][n_tok][d_feat] fp32.
  * attn     (dev) fp32, [n_tiles][n_heads][n_tok] (form 0) or [n_tiles][n_heads][n_patch] (form 1).
  * keep_idx (dev) int32 [n_tiles][keep]: kept patch indices (0-based, CLS excluded), ascending.
@@ -258,7 +277,20 @@ typedef struct {
   const float* slc_norm;       /* host [n_layers]: SLC^Norm of layer l's designated sub-layer (Eq. 5) */
   const uint8_t* layer_target; /* host [n_layers]: m(l), 1 = attention, 2 = FFN */
   const uint8_t* is_visual;    /* host [n_tokens]: 1 for the visual tokens (the skip candidates) */
+  int ablate;                  /* bit set of SPD_SKIP_NO_* below; 0 = the method as printed */
 } spd_skip_policy;
+
+/* Ablation variants of ASL-Skip (the ASL-Skip ablation table). w1 = 0 is the variant without
+ * S_sa (every visual token follows the offline SLC list; no logit lens runs).
+ *   SPD_SKIP_NO_ENTROPY  S_sa = ReLU(1 - F_itc) (no logit lens runs)
+ *   SPD_SKIP_NO_ITC      S_sa = ReLU(1 - E_ii)
+ *   SPD_SKIP_NO_ACCUM    S_skip(i) = w1 S_sa + w2 SLC^Norm(l) of the current layer only
+ *   SPD_SKIP_NO_SLC      no SLC^Norm term, and an admitted token bypasses both sub-layers from its
+ *                        admission layer on (whole layers instead of m(l)) */
+#define SPD_SKIP_NO_ENTROPY 1
+#define SPD_SKIP_NO_ITC 2
+#define SPD_SKIP_NO_ACCUM 4
+#define SPD_SKIP_NO_SLC 8
 
 /* Workspace bytes of spd_prefill_adaptive for up to `max_tokens` tokens in `max_seqs` sequences. */
 size_t spd_prefill_adaptive_workspace_size(const spd_model* m, int max_tokens, int max_seqs);

@@ -175,19 +175,26 @@ def normalized_entropy(logits):
     return -plogp.sum(axis=-1) / np.log(z.shape[-1])
 
 
-def skippability(model, h, cand, seq_of, text_rows, round_fn=bf16_round):
+def skippability(model, h, cand, seq_of, text_rows, round_fn=bf16_round, use_entropy=True,
+                 use_itc=True):
     """S_sa(i, l) = ReLU(1 - E_ii - F_itc) for the candidate tokens (§4.2.1).
 
     E_ii: normalized entropy of the vocabulary distribution of the token's hidden state, read
     through the unembedding after the final RMSNorm (the logit-lens reading; the operand rounded to
     bf16 as every GEMM input). F_itc = (cos(h_i, q_t) + 1) / 2 with q_t the mean hidden state of the
     text tokens of the token's sequence (cos = 0 when that sequence has no text tokens).
+    use_entropy / use_itc False: the ablations of S_sa's components (ASL-Skip ablation table,
+    part (c)); the dropped term is left out of the sum (reading), and is returned as 0.
     """
     cfg = model["cfg"]
-    z = round_fn(rmsnorm(h[cand], model["final_norm"], cfg["rms_eps"]))
-    e = normalized_entropy(z @ model["lm_head"].T)
-    f = np.empty(len(cand))
+    e = np.zeros(len(cand))
+    if use_entropy:
+        z = round_fn(rmsnorm(h[cand], model["final_norm"], cfg["rms_eps"]))
+        e = normalized_entropy(z @ model["lm_head"].T)
+    f = np.zeros(len(cand))
     for n, i in enumerate(cand):
+        if not use_itc:
+            continue
         t = text_rows[seq_of[i]]
         if len(t) == 0:
             f[n] = 0.5
@@ -199,12 +206,18 @@ def skippability(model, h, cand, seq_of, text_rows, round_fn=bf16_round):
 
 
 def prefill_adaptive(model, x, cu_seqlens, is_visual, slc_norm, layer_target, t_skip, w1, w2,
-                     window, round_fn=bf16_round):
+                     window, round_fn=bf16_round, use_entropy=True, use_itc=True, accumulate=True,
+                     use_slc=True):
     """Alg. 1 stage 2 with the online plan: at each layer l < window, every visual token not yet
     in skip mode accumulates S_skip += w1 S_sa(i, l) + w2 SLC^Norm(l) (Eq. 6); once S_skip >= T_skip
     it enters skip mode with target m(l) = layer_target[l], frozen, and bypasses that sub-layer
     from layer l on. Returns (h, logits, admit [T] (-1 never), target [T], margin), margin = the
     smallest |S_skip - T_skip| over every comparison made (for choosing well-conditioned tests).
+
+    Ablations of the ASL-Skip table: w1 = 0 (without S_sa); use_entropy / use_itc False (without
+    E_ii / F_itc, see skippability); accumulate False (S_skip is the current layer's S_fuse alone);
+    use_slc False (no w2 SLC^Norm term, and an admitted token bypasses both sub-layers: whole
+    layers, the paper's description of that variant).
     """
     cfg = model["cfg"]
     L = cfg["n_layers"]
@@ -223,12 +236,14 @@ def prefill_adaptive(model, x, cu_seqlens, is_visual, slc_norm, layer_target, t_
         if l < window:
             cand = np.flatnonzero(vis & (admit < 0))
             if len(cand):
-                s_sa, _, _ = skippability(model, h, cand, seq_of, text_rows, round_fn)
-                s_skip[cand] += w1 * s_sa + w2 * slc_norm[l]
+                s_sa, _, _ = skippability(model, h, cand, seq_of, text_rows, round_fn,
+                                          use_entropy, use_itc)
+                s_fuse = w1 * s_sa + (w2 * slc_norm[l] if use_slc else 0.0)
+                s_skip[cand] = (s_skip[cand] + s_fuse) if accumulate else s_fuse
                 margin = min(margin, float(np.abs(s_skip[cand] - t_skip).min()))
                 new = cand[s_skip[cand] >= t_skip]
                 admit[new] = l
-                target[new] = layer_target[l]
+                target[new] = layer_target[l] if use_slc else 3
         mask_l = np.where((admit >= 0) & (admit <= l), target, 0).astype(np.uint8)
         forward_layer(cfg, model["layers"][l], h, mask_l, cu, pos, round_fn)
     last = cu[1:] - 1

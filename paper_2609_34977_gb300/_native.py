@@ -43,7 +43,13 @@ class PruneCfg(C.Structure):
                 ("n_layers", C.c_int), ("final_layer", C.c_int), ("n_heads", C.c_int),
                 ("attn_form", C.c_int), ("keep", C.c_int), ("n_clusters", C.c_int),
                 ("kmeans_iters", C.c_int), ("anchor_ratio", C.c_double),
-                ("layer_weight", C.c_float * SPD_MAX_FEAT_LAYERS)]
+                ("layer_weight", C.c_float * SPD_MAX_FEAT_LAYERS), ("sim_kind", C.c_int),
+                ("ablate", C.c_int)]
+
+
+SIM_KINDS = {"cos": 0, "mse": 1, "kl": 2}
+SPD_PRUNE_NO_FINAL_SIM = 1
+SPD_PRUNE_NO_ANCHOR_SIM = 2
 
 
 class ModelCfg(C.Structure):
@@ -55,7 +61,14 @@ class ModelCfg(C.Structure):
 
 class SkipPolicy(C.Structure):
     _fields_ = [("t_skip", C.c_float), ("w1", C.c_float), ("w2", C.c_float), ("window", C.c_int),
-                ("slc_norm", C.c_void_p), ("layer_target", C.c_void_p), ("is_visual", C.c_void_p)]
+                ("slc_norm", C.c_void_p), ("layer_target", C.c_void_p), ("is_visual", C.c_void_p),
+                ("ablate", C.c_int)]
+
+
+SPD_SKIP_NO_ENTROPY = 1
+SPD_SKIP_NO_ITC = 2
+SPD_SKIP_NO_ACCUM = 4
+SPD_SKIP_NO_SLC = 8
 
 
 class LayerWeights(C.Structure):
@@ -159,12 +172,14 @@ def spd_selftest_bounded_wait(ws, budget_cycles: int, stream=None):
 
 
 def prune_cfg(n_tiles, n_tok, d_feat, n_layers, final_layer, n_heads, keep, *, has_cls=True,
-              attn_form=0, n_clusters=4, kmeans_iters=10, anchor_ratio=0.7, layer_weight=None):
+              attn_form=0, n_clusters=4, kmeans_iters=10, anchor_ratio=0.7, layer_weight=None,
+              sim="cos", use_final_sim=True, use_anchor_sim=True):
     w = list(layer_weight) if layer_weight is not None else [1.0] * SPD_MAX_FEAT_LAYERS
     w = w + [1.0] * (SPD_MAX_FEAT_LAYERS - len(w))
+    ablate = (0 if use_final_sim else SPD_PRUNE_NO_FINAL_SIM) | (0 if use_anchor_sim else SPD_PRUNE_NO_ANCHOR_SIM)
     return PruneCfg(n_tiles, n_tok, int(has_cls), d_feat, n_layers, final_layer, n_heads, attn_form,
                     keep, n_clusters, kmeans_iters, float(anchor_ratio),
-                    (C.c_float * SPD_MAX_FEAT_LAYERS)(*w))
+                    (C.c_float * SPD_MAX_FEAT_LAYERS)(*w), SIM_KINDS[sim], ablate)
 
 
 def spd_prune_workspace_size(cfg: PruneCfg) -> int:
@@ -282,16 +297,16 @@ def spd_prefill_adaptive_workspace_size(model: SpdModel, max_tokens: int, max_se
 
 
 def spd_prefill_adaptive(model: SpdModel, x, n_tokens, cu_seqlens, is_visual, slc_norm, layer_target,
-                         t_skip, w1, w2, window, h, logits, ws, stream=None):
+                         t_skip, w1, w2, window, h, logits, ws, stream=None, ablate=0):
     """Prefill with the online ASL-Skip plan; returns the admission layer of every token (host
-    int16, -1 = never)."""
+    int16, -1 = never). ablate: bit set of SPD_SKIP_NO_*."""
     cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
     slc = np.ascontiguousarray(slc_norm, dtype=np.float32)
     tgt = np.ascontiguousarray(layer_target, dtype=np.uint8)
     vis = np.ascontiguousarray(is_visual, dtype=np.uint8)
     admit = np.full(n_tokens, -9, dtype=np.int16)
     pol = SkipPolicy(float(t_skip), float(w1), float(w2), int(window), slc.ctypes.data, tgt.ctypes.data,
-                     vis.ctypes.data)
+                     vis.ctypes.data, int(ablate))
     _check(lib().spd_prefill_adaptive(model.handle, _p(x), n_tokens, cu.ctypes.data, len(cu) - 1,
                                       C.byref(pol), admit.ctypes.data, _p(h), _p(logits), _p(ws),
                                       ws.numel() * ws.element_size(), _stream(stream)))

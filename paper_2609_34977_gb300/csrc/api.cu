@@ -838,6 +838,13 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
   for (int l = 0; l < L; ++l)
     if (pol->layer_target[l] != 1 && pol->layer_target[l] != 2)
       return fail(SPD_EINVAL, "layer targets must be 1 (attention) or 2 (FFN)");
+  const int ab_bits = SPD_SKIP_NO_ENTROPY | SPD_SKIP_NO_ITC | SPD_SKIP_NO_ACCUM | SPD_SKIP_NO_SLC;
+  if (pol->ablate & ~ab_bits) return fail(SPD_EINVAL, "unknown ablate bits");
+  // which parts of Eq. 4-6 run (S_sa's terms are not computed where w1 = 0 makes them irrelevant)
+  const bool no_slc = pol->ablate & SPD_SKIP_NO_SLC;
+  const int mode = ((pol->w1 != 0.0f && !(pol->ablate & SPD_SKIP_NO_ENTROPY)) ? kSkipEntropy : 0) |
+                   ((pol->w1 != 0.0f && !(pol->ablate & SPD_SKIP_NO_ITC)) ? kSkipItc : 0) |
+                   ((pol->ablate & SPD_SKIP_NO_ACCUM) ? 0 : kSkipAccumulate);
   Carve cv(ws, ws_bytes);
   PrefillBufs bf = carve_prefill(c, T, B, cv);
   AdaptiveBufs ab = carve_adaptive(c, T, B, cv);
@@ -877,30 +884,33 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
       if (nc > 0) {
         SPD_CUDA_TRY(cudaMemcpyAsync(ab.cand, cand.data(), nc * sizeof(int32_t),
                                      cudaMemcpyHostToDevice, st));
-        // logit lens: final RMSNorm, then the unembedding (LM head) in fp32
-        if (int rc = rmsnorm_run(h, nc, D, m->final_norm, c.rms_eps, ab.cand, bf.xa, nullptr, nullptr, st))
-          return rc;
-        GemmProblem up{};
-        up.map_w = &m->m_lm;
-        up.w = m->lm_head;
-        up.x = bf.xa;
-        up.n_out = c.vocab;
-        up.n_tok = nc;
-        up.k = D;
-        up.epi = EPI_F32;
-        up.out = ab.logits;
-        up.ldo = c.vocab;
-        if (int rc = gemm_run(up, bf.gs, st)) return rc;
+        if (mode & kSkipEntropy) {
+          // logit lens: final RMSNorm, then the unembedding (LM head) in fp32
+          if (int rc = rmsnorm_run(h, nc, D, m->final_norm, c.rms_eps, ab.cand, bf.xa, nullptr, nullptr, st))
+            return rc;
+          GemmProblem up{};
+          up.map_w = &m->m_lm;
+          up.w = m->lm_head;
+          up.x = bf.xa;
+          up.n_out = c.vocab;
+          up.n_tok = nc;
+          up.k = D;
+          up.epi = EPI_F32;
+          up.out = ab.logits;
+          up.ldo = c.vocab;
+          if (int rc = gemm_run(up, bf.gs, st)) return rc;
+        }
+        const float add_slc = no_slc ? 0.0f : pol->w2 * pol->slc_norm[l];
         if (int rc = skip_scores_run(ab.logits, c.vocab, nc, h, D, ab.cand, ab.ts, ab.text, ab.seq, B,
-                                     ab.tmean, pol->w1, pol->w2 * pol->slc_norm[l], pol->t_skip,
-                                     ab.s_skip, ab.flag, st))
+                                     ab.tmean, pol->w1, add_slc, pol->t_skip, mode, ab.s_skip, ab.flag,
+                                     st))
           return rc;
         SPD_CUDA_TRY(cudaMemcpyAsync(flags.data(), ab.flag, nc, cudaMemcpyDeviceToHost, st));
         SPD_CUDA_TRY(cudaStreamSynchronize(st));
         for (int n = 0; n < nc; ++n)
           if (flags[n]) {
             admit[cand[n]] = l;
-            target[cand[n]] = pol->layer_target[l];  // frozen at admission
+            target[cand[n]] = no_slc ? 3 : pol->layer_target[l];  // frozen at admission
           }
       }
     }

@@ -123,13 +123,15 @@ constexpr int kAttnTileQ = 128;  // queries per attention tile
 int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream);
 
 // ---- ASL-Skip online scores (Sec. 4.2.1, Eq. 6) -------------------------------------------------
-// For candidate n (token cand[n], sequence seq_of[token]): entropy of softmax(logits[n]) / log V,
-// cosine of h[token] to the mean h of its sequence's text tokens text[ts[b] .. ts[b+1]) (computed
-// into tmean [B][D]), S_sa = ReLU(1 - E - F); s_skip[token] += w1 S_sa + add_slc; flag[n] =
-// (s_skip[token] >= t_skip).
+// For candidate n (token cand[n], sequence seq_of[token]): E = entropy of softmax(logits[n]) / log V
+// (mode kSkipEntropy, else 0; logits unread), F = (cos of h[token] to the mean h of its sequence's
+// text tokens text[ts[b] .. ts[b+1]) (computed into tmean [B][D]) + 1) / 2 (mode kSkipItc, else 0),
+// S_sa = ReLU(1 - E - F); s_skip[token] = (kSkipAccumulate ? s_skip[token] : 0) + w1 S_sa + add_slc;
+// flag[n] = (s_skip[token] >= t_skip).
+constexpr int kSkipEntropy = 1, kSkipItc = 2, kSkipAccumulate = 4;
 int skip_scores_run(const float* logits, int V, int n_cand, const float* h, int D, const int32_t* cand,
                     const int32_t* ts, const int32_t* text, const int32_t* seq_of, int B, float* tmean,
-                    float w1, float add_slc, float t_skip, float* s_skip, uint8_t* flag,
+                    float w1, float add_slc, float t_skip, int mode, float* s_skip, uint8_t* flag,
                     cudaStream_t stream);
 
 }  // namespace spd

@@ -123,46 +123,53 @@ __global__ void __launch_bounds__(kThreads)
     skip_score_kernel(const float* __restrict__ logits, int V, const float* __restrict__ h, int D,
                       const int32_t* __restrict__ cand, const int32_t* __restrict__ ts,
                       const int32_t* __restrict__ seq_of, const float* __restrict__ tmean,
-                      float inv_log_v, float w1, float add_slc, float t_skip,
+                      float inv_log_v, float w1, float add_slc, float t_skip, int mode,
                       float* __restrict__ s_skip, uint8_t* __restrict__ flag) {
   __shared__ float red[kThreads / 32];
   pdl_launch_dependents();
   pdl_wait();
   const int n = blockIdx.x, i = cand[n], b = seq_of[i];
-  const float* z = logits + size_t(n) * V;
-  float mx = -INFINITY;
-  for (int v = threadIdx.x; v < V; v += kThreads) mx = fmaxf(mx, z[v]);
-  mx = block_max(mx, red);
-  float se = 0.0f, te = 0.0f;  // sum e^(z - m) and sum e^(z - m) (z - m)
-  for (int v = threadIdx.x; v < V; v += kThreads) {
-    const float d = z[v] - mx, e = expf(d);
-    se += e;
-    te += e * d;
+  float ent = 0.0f;
+  if (mode & kSkipEntropy) {
+    const float* z = logits + size_t(n) * V;
+    float mx = -INFINITY;
+    for (int v = threadIdx.x; v < V; v += kThreads) mx = fmaxf(mx, z[v]);
+    mx = block_max(mx, red);
+    float se = 0.0f, te = 0.0f;  // sum e^(z - m) and sum e^(z - m) (z - m)
+    for (int v = threadIdx.x; v < V; v += kThreads) {
+      const float d = z[v] - mx, e = expf(d);
+      se += e;
+      te += e * d;
+    }
+    __syncthreads();
+    se = block_sum(se, red);
+    __syncthreads();
+    te = block_sum(te, red);
+    ent = (logf(se) - te / se) * inv_log_v;
   }
-  __syncthreads();
-  se = block_sum(se, red);
-  __syncthreads();
-  te = block_sum(te, red);
-  const float ent = (logf(se) - te / se) * inv_log_v;
   const float* hi = h + size_t(i) * D;
   const float* q = tmean + size_t(b) * D;
-  float dot = 0.0f, hh = 0.0f, qq = 0.0f;
-  for (int c = threadIdx.x; c < D; c += kThreads) {
-    dot += hi[c] * q[c];
-    hh += hi[c] * hi[c];
-    qq += q[c] * q[c];
-  }
-  __syncthreads();
-  dot = block_sum(dot, red);
-  __syncthreads();
-  hh = block_sum(hh, red);
-  __syncthreads();
-  qq = block_sum(qq, red);
-  if (threadIdx.x == 0) {
+  float f = 0.0f;
+  if (mode & kSkipItc) {
+    float dot = 0.0f, hh = 0.0f, qq = 0.0f;
+    for (int c = threadIdx.x; c < D; c += kThreads) {
+      dot += hi[c] * q[c];
+      hh += hi[c] * hi[c];
+      qq += q[c] * q[c];
+    }
+    __syncthreads();
+    dot = block_sum(dot, red);
+    __syncthreads();
+    hh = block_sum(hh, red);
+    __syncthreads();
+    qq = block_sum(qq, red);
     const bool has_text = ts[b + 1] > ts[b] && hh > 0.0f && qq > 0.0f;
-    const float f = has_text ? 0.5f + 0.5f * dot / (sqrtf(hh) * sqrtf(qq)) : 0.5f;
+    f = has_text ? 0.5f + 0.5f * dot / (sqrtf(hh) * sqrtf(qq)) : 0.5f;
+  }
+  if (threadIdx.x == 0) {
     const float s_sa = fmaxf(0.0f, 1.0f - ent - f);
-    const float acc = s_skip[i] + (w1 * s_sa + add_slc);
+    const float fuse = w1 * s_sa + add_slc;
+    const float acc = (mode & kSkipAccumulate) ? s_skip[i] + fuse : fuse;
     s_skip[i] = acc;
     flag[n] = acc >= t_skip ? 1 : 0;
   }
@@ -172,13 +179,14 @@ __global__ void __launch_bounds__(kThreads)
 
 int skip_scores_run(const float* logits, int V, int n_cand, const float* h, int D, const int32_t* cand,
                     const int32_t* ts, const int32_t* text, const int32_t* seq_of, int B, float* tmean,
-                    float w1, float add_slc, float t_skip, float* s_skip, uint8_t* flag,
+                    float w1, float add_slc, float t_skip, int mode, float* s_skip, uint8_t* flag,
                     cudaStream_t stream) {
-  SPD_CUDA_TRY(launch_pdl(text_mean_kernel, dim3((D + kThreads - 1) / kThreads, B), dim3(kThreads), 0,
-                          stream, h, D, ts, text, tmean));
+  if (mode & kSkipItc)
+    SPD_CUDA_TRY(launch_pdl(text_mean_kernel, dim3((D + kThreads - 1) / kThreads, B), dim3(kThreads),
+                            0, stream, h, D, ts, text, tmean));
   SPD_CUDA_TRY(launch_pdl(skip_score_kernel, dim3(n_cand), dim3(kThreads), 0, stream,
                           logits, V, h, D, cand, ts, seq_of, static_cast<const float*>(tmean),
-                          float(1.0 / log(double(V))), w1, add_slc, t_skip, s_skip, flag));
+                          float(1.0 / log(double(V))), w1, add_slc, t_skip, mode, s_skip, flag));
   return SPD_OK;
 }
 

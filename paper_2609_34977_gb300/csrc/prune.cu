@@ -1,6 +1,8 @@
 // MSV-Prune (Sec. 4.1, Eq. 1-3; Alg. 1 stage 1) on the GPU, every tile independently.
 //
 //   rowstats     a_v = head-mean of the attention (Sec. 4.1.1); 1/||F_l,i|| for every tapped layer
+//                (and ||F_l,i||^2, or the log-sum-exp and negentropy of softmax(F_l,i), for the
+//                MSE and KL ablations of sim)
 //   anchors      top-N_anc of a_v by a bitonic sort of (a_v desc, index asc) keys (Eq. 1);
 //                stable lists of anchor and non-anchor tokens by block prefix sums
 //   anchor_sim   a_i = max_p cos(F^L_i, F^L_p) over anchors: 64 x 64 register-tiled fp32 products,
@@ -15,7 +17,9 @@
 //                per-cluster, per-layer sums of unit feature rows, the sums of a_j, sizes and Eq. 2
 //                quotas
 //   scores       s_i = [sum_l w_l f_i . (S_l,k - f_i)] / (|C_k| - 1) + a_i + (A_k - a_i) / (|C_k| - 1),
-//                the per-token mean of Eq. 3's S_ij over the other members of its cluster
+//                the per-token mean of Eq. 3's S_ij over the other members of its cluster (for
+//                the MSE and KL ablations the same cluster-sum identity with raw rows, plus the
+//                per-cluster sums of ||F_j||^2 or of the log-sum-exps)
 //   select       per cluster the N_k lowest (score, index) keys; kept = anchors + selected, compacted
 //                in ascending index order
 // All reductions run in a fixed order, so repeated runs give identical bits.
@@ -38,6 +42,8 @@ namespace spd {
 
 struct PruneDims {
   int n_tiles, n_tok, off, n, d, L, fin, H, form, n_att, keep, K, iters, n_anc, n_cmp, m;
+  int sim;        // SPD_SIM_*
+  float wf, wa;   // weights (0 or 1) of the final-layer intra-cluster term and the anchor bracket
   float w[SPD_MAX_FEAT_LAYERS];
   const float* feat[SPD_MAX_FEAT_LAYERS];
 };
@@ -45,6 +51,8 @@ struct PruneDims {
 struct PruneWs {
   float* a_v;       // [T][n]
   float* inv;       // [L][T][n]
+  float* st1;       // [L][T][n] MSE: ||F_l,i||^2; KL: log-sum-exp of F_l,i
+  float* st2;       // [L][T][n] KL: sum_c P_c log P_c of P = softmax(F_l,i)
   int8_t* role;     // [T][n] 1 anchor
   int32_t* alist;   // [T][n_anc]
   int32_t* ulist;   // [T][m]
@@ -54,6 +62,7 @@ struct PruneWs {
   int32_t* quotas;  // [T][16]
   float* asum;      // [T][16]
   float* csum;      // [T][L][K][d]
+  float* ssum;      // [T][L][16] MSE / KL: per-cluster sums of st1
   float* score;     // [T][m]
   int* status;
 };
@@ -161,7 +170,36 @@ __global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float*
       ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
     }
     ss = warp_sum(ss);
-    if (lane == 0) w.inv[(size_t(l) * p.n_tiles + t) * p.n + i] = 1.0f / sqrtf(ss);
+    const size_t o = (size_t(l) * p.n_tiles + t) * p.n + i;
+    if (lane == 0) w.inv[o] = 1.0f / sqrtf(ss);
+    if (p.sim == SPD_SIM_MSE && lane == 0) w.st1[o] = ss;
+    if (p.sim == SPD_SIM_KL) {  // softmax over the row: max, then sum e^z and sum e^z z (z = x - max)
+      float mx = -INFINITY;
+      for (int c = lane; c < p.d / 4; c += 32) {
+        const float4 v = r[c];
+        mx = fmaxf(mx, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)));
+      }
+#pragma unroll
+      for (int off = 16; off; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+      float se = 0.0f, te = 0.0f;
+      for (int c = lane; c < p.d / 4; c += 32) {
+        const float4 v = r[c];
+        const float z[4] = {v.x - mx, v.y - mx, v.z - mx, v.w - mx};
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const float e = expf(z[u]);
+          se += e;
+          te += e * z[u];
+        }
+      }
+      se = warp_sum(se);
+      te = warp_sum(te);
+      if (lane == 0) {
+        const float lse = logf(se);
+        w.st1[o] = mx + lse;        // log sum_c e^x_c
+        w.st2[o] = te / se - lse;   // sum_c P_c log P_c
+      }
+    }
   }
   if (lane == 0) {
     const int col = (p.form == 0) ? 1 + i : i;
@@ -208,7 +246,8 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
   const int a0 = block_scan_excl(na, tmp, nullptr);
   const int u0 = block_scan_excl(nu, tmp, nullptr);
   int ai = a0, ui = u0;
-  const uint32_t init = (p.n_anc == 0) ? ordered_key(0.0f) : 0u;
+  // a_i = 0 where the anchor bracket is absent (no anchors, or the ablation without it)
+  const uint32_t init = (p.n_anc == 0 || p.wa == 0.0f) ? ordered_key(0.0f) : 0u;
   for (int q = 0; q < 4; ++q) {
     const int i = base + q;
     if (i >= p.n) break;
@@ -240,13 +279,18 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
   const int* al = w.alist + size_t(t) * p.n_anc;
   // staging: thread loads column dd of rows r0 + 8 i (i < 8) of both operands
   const int dd = threadIdx.x & 31, r0 = threadIdx.x >> 5;
+  // per-row statistics of the final layer (MSE: squared norms; KL: log-sum-exps, negentropies)
+  const size_t so = (size_t(p.fin) * p.n_tiles + t) * p.n;
+  const bool kl = p.sim == SPD_SIM_KL;
   const float* urow[8];
   const float* arow[8];
+  float ulse[8];  // KL: the non-anchor operand is softmax(F^L_i) = exp(F^L_i - lse_i)
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const int r = r0 + 8 * i;
     urow[i] = (u0 + r < p.m) ? feat_row(p, p.fin, t, ul[u0 + r]) : nullptr;
     arow[i] = (p0 + r < p.n_anc) ? feat_row(p, p.fin, t, al[p0 + r]) : nullptr;
+    ulse[i] = (kl && urow[i]) ? w.st1[so + ul[u0 + r]] : 0.0f;
   }
   const int nch = (p.d + 31) / 32, c0 = rank * nch / kAS, c1 = (rank + 1) * nch / kAS;
   float ru[8], ra[8];
@@ -254,7 +298,8 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
     const int dcol = ch * 32 + dd;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      ru[i] = (urow[i] && dcol < p.d) ? urow[i][dcol] : 0.0f;
+      const float x = (urow[i] && dcol < p.d) ? urow[i][dcol] : 0.0f;
+      ru[i] = (kl && urow[i] && dcol < p.d) ? expf(x - ulse[i]) : x;
       ra[i] = (arow[i] && dcol < p.d) ? arow[i][dcol] : 0.0f;
     }
   };
@@ -303,6 +348,10 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
   const float* inv = w.inv + size_t(p.fin) * p.n_tiles * p.n + size_t(t) * p.n;
   const int ur = u0 + lr;
   float best = -INFINITY;
+  // candidates whose maximum over p gives a_i through an increasing map g:
+  //   cos: F_i.F_p / (|F_i| |F_p|)             (g = identity)
+  //   MSE: 2 F_i.F_p - |F_p|^2                  (g(v) = -(|F_i|^2 - v) / d)
+  //   KL:  P_i.F_p - lse_p = -KL(P_i||P_p) + N_i (g(v) = v - N_i)
   if (ur < p.m) {
     const float iu = inv[ul[ur]];
 #pragma unroll
@@ -311,12 +360,23 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
 #pragma unroll
       for (int src = 0; src < kAS; ++src) sdot += x[src][j];
       const int pa = p0 + tx + 16 * j;
-      if (pa < p.n_anc) best = fmaxf(best, sdot * iu * inv[al[pa]]);
+      if (pa < p.n_anc) {
+        const int ia = al[pa];
+        const float v = p.sim == SPD_SIM_COS ? sdot * iu * inv[ia]
+                        : p.sim == SPD_SIM_MSE ? 2.0f * sdot - w.st1[so + ia]
+                                               : sdot - w.st1[so + ia];
+        best = fmaxf(best, v);
+      }
     }
   }
 #pragma unroll
   for (int off = 8; off; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
-  if (tx == 0 && ur < p.m) atomicMax(&w.asim[size_t(t) * p.n + ul[ur]], ordered_key(best));
+  if (tx == 0 && ur < p.m) {
+    const int iu = ul[ur];
+    if (p.sim == SPD_SIM_MSE) best = -(w.st1[so + iu] - best) / float(p.d);
+    else if (p.sim == SPD_SIM_KL) best = best - w.st2[so + iu];
+    atomicMax(&w.asim[size_t(t) * p.n + iu], ordered_key(best));
+  }
   cl.sync();  // peers read this CTA's partial tile above
 }
 
@@ -499,12 +559,13 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
   float* part = cent + size_t(K) * D;                         // [K][D] this CTA's column sums
   __shared__ int cnt[SPD_MAX_CLUSTERS];   // this CTA's cluster sizes
   __shared__ float asum_part[SPD_MAX_CLUSTERS];
+  __shared__ float ssum_part[SPD_MAX_CLUSTERS];  // MSE / KL: this CTA's sums of st1 per cluster
   __shared__ int changed;      // this CTA's assignment changed in the current iteration
   __shared__ int any_changed;  // ... some CTA's of the cluster
   __shared__ int8_t asg[4096 / KC + 1];
   __shared__ int idx[4096 / KC + 1];     // patch index of each of this CTA's tokens
   __shared__ float av[4096 / KC + 1];    // their a_j
-  __shared__ float rinv[4096 / KC + 1];  // their 1 / ||F_l,j|| for the layer being summed
+  __shared__ float rinv[4096 / KC + 1];  // their 1 / ||F_l,j|| (cos) or st1 (MSE, KL) of the layer
   __shared__ int ncl[SPD_MAX_CLUSTERS];  // cluster sizes over the whole cluster of CTAs
   __shared__ uint64_t rows_bar;
   cg::cluster_group cl = cg::this_cluster();
@@ -687,15 +748,17 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
   }
   if (threadIdx.x == 0)  // token order
     for (int jj = 0; jj < nl; ++jj) asum_part[asg[jj]] += av[jj];
-  // per layer: sums over each cluster of unit feature rows (F_l,j / ||F_l,j||)
+  // per layer: sums over each cluster of unit feature rows (F_l,j / ||F_l,j||), or of raw rows and
+  // of st1 for the MSE and KL similarities
   // (RES: the final layer first, from the resident rows; then each other layer's rows are copied
   // into the same buffer)
+  const bool cos_sim = p.sim == SPD_SIM_COS;
   for (int li = 0; li < p.L; ++li) {
     const int l = RES ? (li == 0 ? p.fin : (li <= p.fin ? li - 1 : li)) : li;
-    const float* inv = w.inv + (size_t(l) * p.n_tiles + t) * p.n;
+    const float* rstat = (cos_sim ? w.inv : w.st1) + (size_t(l) * p.n_tiles + t) * p.n;
     const float* fl = p.feat[l];
     __syncthreads();  // the previous layer's rows are no longer read
-    for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) rinv[jj] = inv[idx[jj]];
+    for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) rinv[jj] = rstat[idx[jj]];
     if (RES && l != p.fin && threadIdx.x == 0 && nl > 0) {
       mbar_arrive_expect_tx(&rows_bar, uint32_t(nl) * D * 4);
       for (int jj = 0; jj < nl; ++jj)
@@ -709,11 +772,24 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
       }
     }
     __syncthreads();
-    column_sums<KN>(part, K, D, nl, asg, RowAccess{RES ? rows : nullptr, fl, row0, idx, D, rinv});
+    if (!cos_sim && threadIdx.x == 0) {  // token order
+      for (int k = 0; k < K; ++k) ssum_part[k] = 0.0f;
+      for (int jj = 0; jj < nl; ++jj) ssum_part[asg[jj]] += rinv[jj];
+    }
+    column_sums<KN>(part, K, D, nl, asg,
+                    RowAccess{RES ? rows : nullptr, fl, row0, idx, D, cos_sim ? rinv : nullptr});
     cl.sync();
     float* csum = w.csum + (size_t(t) * p.L + l) * K * D;
     cluster_column_reduce<KC>(cl, part, K, D, rank,
                               [&](int k, int c, float sum) { csum[k * D + c] = sum; });
+    if (!cos_sim && rank == 0 && warp == 1) {  // CTA sums added in rank order
+      for (int k = 0; k < K; ++k) {
+        const float sr = lane < KC ? cl.map_shared_rank(ssum_part, lane)[k] : 0.0f;
+        float a = 0.0f;
+        for (int rr = 0; rr < KC; ++rr) a += __shfl_sync(0xffffffffu, sr, rr);
+        if (lane == 0) w.ssum[(size_t(t) * p.L + l) * 16 + k] = a;
+      }
+    }
     if (li == p.L - 1 && rank == 0 && warp == 0) {
       // sizes and a_j sums over the CTAs (lane r reads CTA r; the a_j sums added in rank order)
       int sizes[SPD_MAX_CLUSTERS], q[SPD_MAX_CLUSTERS];
@@ -741,6 +817,14 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
 }
 
 // ---- 6. per-token Eq. 3 scores ----------------------------------------------------------------
+// Per layer, with X_k the cluster's column sums and c = |C_k|, the sum over the other members j:
+//   cos: sum_j f_i.f_j = f_i.(X_k - f_i)                                     (f = F / |F|)
+//   MSE: sum_j -|F_i - F_j|^2 / d = -[(c - 1) |F_i|^2 - 2 F_i.(X_k - F_i) + (Q_k - |F_i|^2)] / d
+//   KL:  sum_j -KL(P_i || P_j) = -c sum_c P_i,c (log P_i,c - (X_k,c - S_k) / c)
+//        (the j = i term is 0; (X_k - S_k) / c is the cluster mean of log P_j, so every product
+//        is of a probability and an O(1) difference of logs, with no cancellation of large sums)
+// (Q_k, S_k: the cluster's sums of |F_j|^2 and of lse_j.)
+template <int SIM>
 __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
@@ -753,14 +837,18 @@ __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
   const float ai = ordered_val(w.asim[size_t(t) * p.n + i]);
   float s;
   if (cnt <= 1) {
-    s = 2.0f * ai;
+    s = p.wa * 2.0f * ai;
   } else {
     float acc = 0.0f;
     for (int l = 0; l < p.L; ++l) {
-      const float wl = (l == p.fin) ? 1.0f : p.w[l];
+      const float wl = (l == p.fin) ? p.wf : p.w[l];
       if (wl == 0.0f) continue;
       const float4* x4 = reinterpret_cast<const float4*>(feat_row(p, l, t, i));
-      const float iv = w.inv[(size_t(l) * p.n_tiles + t) * p.n + i];
+      const size_t so = (size_t(l) * p.n_tiles + t) * p.n + i;
+      const float iv = SIM == SPD_SIM_COS ? w.inv[so] : 1.0f;
+      const float lse = SIM == SPD_SIM_KL ? w.st1[so] : 0.0f;
+      const float inv_n = 1.0f / float(cnt);
+      const float sbar = SIM == SPD_SIM_KL ? w.ssum[(size_t(t) * p.L + l) * 16 + k] * inv_n : 0.0f;
       const float4* c4 =
           reinterpret_cast<const float4*>(w.csum + ((size_t(t) * p.L + l) * p.K + k) * p.d);
       // 16-byte loads, sixteen in flight per lane, two independent chains
@@ -776,17 +864,35 @@ __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
         }
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-          const float a0 = xv[u].x * iv, a1 = xv[u].y * iv, a2 = xv[u].z * iv, a3 = xv[u].w * iv;
-          const float part = a0 * (cv[u].x - a0) + a1 * (cv[u].y - a1) + a2 * (cv[u].z - a2) +
-                             a3 * (cv[u].w - a3);
+          // cos: f.(X - f) with f = x |x|^-1; MSE: x.(X - x); KL: P.(log P - mean_j log P_j)
+          const float b0 = xv[u].x * iv, b1 = xv[u].y * iv, b2 = xv[u].z * iv, b3 = xv[u].w * iv;
+          float part;
+          if (SIM == SPD_SIM_KL) {
+            if (cb + 32 * u >= d4) continue;  // a zero-filled slot is no zero term here
+            const float l0 = b0 - lse, l1 = b1 - lse, l2 = b2 - lse, l3 = b3 - lse;
+            part = expf(l0) * (l0 - (cv[u].x * inv_n - sbar)) + expf(l1) * (l1 - (cv[u].y * inv_n - sbar)) +
+                   expf(l2) * (l2 - (cv[u].z * inv_n - sbar)) + expf(l3) * (l3 - (cv[u].w * inv_n - sbar));
+          } else {
+            part = b0 * (cv[u].x - b0) + b1 * (cv[u].y - b1) + b2 * (cv[u].z - b2) + b3 * (cv[u].w - b3);
+          }
           if (u & 1) dot1 += part;
           else dot0 += part;
         }
       }
-      acc += wl * warp_sum(dot0 + dot1);
+      const float dot = warp_sum(dot0 + dot1);
+      float term = dot;
+      if (SIM != SPD_SIM_COS) {
+        if (SIM == SPD_SIM_MSE) {
+          const float sk = w.ssum[(size_t(t) * p.L + l) * 16 + k], st = w.st1[so];
+          term = -(float(cnt - 1) * st - 2.0f * dot + (sk - st)) / float(p.d);
+        } else {
+          term = -float(cnt) * dot;
+        }
+      }
+      acc += wl * term;
     }
     const float inv_c = 1.0f / float(cnt - 1);
-    s = acc * inv_c + ai + (w.asum[t * 16 + k] - ai) * inv_c;
+    s = acc * inv_c + p.wa * (ai + (w.asum[t * 16 + k] - ai) * inv_c);
   }
   if (lane == 0) w.score[size_t(t) * p.m + j] = s;
 }
@@ -967,6 +1073,12 @@ int validate(const spd_prune_cfg* c, PruneDims* p) {
   if (c->kmeans_iters < 1) return fail(SPD_EINVAL, "kmeans_iters >= 1 required");
   if (!(c->anchor_ratio >= 0.0 && c->anchor_ratio <= 1.0))
     return fail(SPD_EINVAL, "anchor_ratio must lie in [0, 1]");
+  if (c->sim_kind < SPD_SIM_COS || c->sim_kind > SPD_SIM_KL) return fail(SPD_EINVAL, "bad sim_kind");
+  if (c->ablate & ~(SPD_PRUNE_NO_FINAL_SIM | SPD_PRUNE_NO_ANCHOR_SIM))
+    return fail(SPD_EINVAL, "unknown ablate bits");
+  p->sim = c->sim_kind;
+  p->wf = (c->ablate & SPD_PRUNE_NO_FINAL_SIM) ? 0.0f : 1.0f;
+  p->wa = (c->ablate & SPD_PRUNE_NO_ANCHOR_SIM) ? 0.0f : 1.0f;
   p->n_tiles = c->n_tiles;
   p->n_tok = c->n_tok;
   p->off = off;
@@ -997,6 +1109,9 @@ PruneWs carve(const PruneDims& p, Carve& cv) {
   w.status = cv.status();
   w.a_v = cv.take<float>(T * p.n);
   w.inv = cv.take<float>(T * p.n * p.L);
+  const size_t nst = p.sim == SPD_SIM_COS ? 0 : T * p.n * p.L;
+  w.st1 = cv.take<float>(nst);
+  w.st2 = cv.take<float>(p.sim == SPD_SIM_KL ? nst : 0);
   w.role = cv.take<int8_t>(T * p.n);
   w.alist = cv.take<int32_t>(T * (p.n_anc + 1));
   w.ulist = cv.take<int32_t>(T * (p.m + 1));
@@ -1006,6 +1121,7 @@ PruneWs carve(const PruneDims& p, Carve& cv) {
   w.quotas = cv.take<int32_t>(T * 16);
   w.asum = cv.take<float>(T * 16);
   w.csum = cv.take<float>(T * p.L * p.K * p.d);
+  w.ssum = cv.take<float>(T * p.L * 16);
   w.score = cv.take<float>(T * (p.m + 1));
   return w;
 }
@@ -1108,7 +1224,7 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
   const int slot = trace_begin(st);
   SPD_CUDA_TRY(launch_pdl(rowstats_kernel, dim3((p.n + 7) / 8, T), dim3(256), 0, st, p, attn, w));
   SPD_CUDA_TRY(launch_pdl(anchor_kernel, dim3(T), dim3(1024), 0, st, p, w));
-  if (p.n_anc > 0 && p.m > 0)
+  if (p.n_anc > 0 && p.m > 0 && p.wa != 0.0f)
     SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel,
                             dim3((p.m + 63) / 64 * kAS, (p.n_anc + 63) / 64, T), dim3(256), 0, st,
                             p, w));
@@ -1127,8 +1243,11 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
     SPD_CUDA_TRY((launch_kmeans<8, false, 4>(p, w, cent_bytes, st)));
   else
     SPD_CUDA_TRY((launch_kmeans<8, false, SPD_MAX_CLUSTERS>(p, w, cent_bytes, st)));
-  if (p.m > 0)
-    SPD_CUDA_TRY(launch_pdl(score_kernel, dim3((p.m + 7) / 8, T), dim3(256), 0, st, p, w));
+  if (p.m > 0) {
+    auto score = p.sim == SPD_SIM_COS ? score_kernel<SPD_SIM_COS>
+                 : p.sim == SPD_SIM_MSE ? score_kernel<SPD_SIM_MSE> : score_kernel<SPD_SIM_KL>;
+    SPD_CUDA_TRY(launch_pdl(score, dim3((p.m + 7) / 8, T), dim3(256), 0, st, p, w));
+  }
   SPD_CUDA_TRY(launch_pdl(select_kernel, dim3(T), dim3(1024), 0, st, p, w, keep_idx, kind, cluster,
                           scores));
   // algorithmic work per tile: every tapped layer's features and the attention read once, the

@@ -95,8 +95,9 @@ class SpiderPrefill:
         """Enqueue one step on device inputs: feats (list of [n_tiles][n_tok][d_vis] fp32), attn,
         text [sum(text_lens)][D] bf16. Returns the logits tensor [B][vocab] (device).
 
-        policy (dict: slc_norm, layer_target, t_skip, w1, w2, window) replaces skip_mask by the
-        online ASL-Skip plan; the admission layer of every token is then left in self.admit."""
+        policy (dict: slc_norm, layer_target, t_skip, w1, w2, window, optional ablate bits
+        SPD_SKIP_NO_*) replaces skip_mask by the online ASL-Skip plan; the admission layer of every
+        token is then left in self.admit."""
         if not self.dense:
             N.spd_prune(self.prune_cfg, feats, attn, self.keep_idx, ws=self.ws_prune, stream=stream)
         fin = int(self.prune_cfg.final_layer)
@@ -121,7 +122,8 @@ class SpiderPrefill:
         self.admit = N.spd_prefill_adaptive(self.model, self.x, self.T, self.cu, self.token_is_visual,
                                             policy["slc_norm"], policy["layer_target"], policy["t_skip"],
                                             policy["w1"], policy["w2"], policy["window"], self.h,
-                                            self.logits, self.ws_adaptive, stream=stream)
+                                            self.logits, self.ws_adaptive, stream=stream,
+                                            ablate=policy.get("ablate", 0))
         return self.logits
 
     def status(self) -> int:

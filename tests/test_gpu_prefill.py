@@ -202,6 +202,43 @@ def test_adaptive_plan_matches_oracle():
     assert rowwise_rel(logits.cpu().numpy(), lg0) < TOL
 
 
+@pytest.mark.parametrize("bits,w1", [
+    (N.SPD_SKIP_NO_ENTROPY, 3.0), (N.SPD_SKIP_NO_ITC, 3.0), (N.SPD_SKIP_NO_ACCUM, 3.0),
+    (N.SPD_SKIP_NO_SLC, 3.0), (0, 0.0), (N.SPD_SKIP_NO_ACCUM | N.SPD_SKIP_NO_SLC, 3.0)],
+    ids=["no_entropy", "no_itc", "no_accum", "no_slc", "no_s_sa", "no_accum_no_slc"])
+def test_adaptive_plan_ablations_match_oracle(bits, w1):
+    # the ablation variants of the ASL-Skip table against the oracle's, on a threshold that every
+    # decision clears by a margin
+    model, om, x, vis, cu = _adaptive_inputs(35, [64, 40], [16, 8])
+    slc = np.array([0.2, 0.5, 0.1, 0.7, 0.3, 0.9])
+    tgt = np.array([1, 2, 1, 1, 2, 2], np.uint8)
+    kw = dict(use_entropy=not bits & N.SPD_SKIP_NO_ENTROPY, use_itc=not bits & N.SPD_SKIP_NO_ITC,
+              accumulate=not bits & N.SPD_SKIP_NO_ACCUM, use_slc=not bits & N.SPD_SKIP_NO_SLC)
+    xn = bf16_np(x)
+    chosen = None
+    for t_skip in np.linspace(0.15, 6.0, 235):
+        h0, lg0, admit0, target0, margin = od.prefill_adaptive(om, xn, cu, vis, slc, tgt, t_skip, w1,
+                                                               1.0, 3, **kw)
+        varied = len(set(admit0[vis])) >= 2 or (w1 == 0.0 and (admit0 >= 0).any())
+        if margin > 0.02 and varied:
+            chosen = (t_skip, h0, lg0, admit0, target0)
+            break
+    assert chosen is not None, "no well-separated threshold in the grid"
+    t_skip, h0, lg0, admit0, target0 = chosen
+    T = x.shape[0]
+    ws = torch.zeros(N.spd_prefill_adaptive_workspace_size(model, T, len(cu) - 1), dtype=torch.uint8,
+                     device="cuda")
+    h = torch.full((T, 256), float("nan"), device="cuda")
+    logits = torch.full((len(cu) - 1, 512), float("nan"), device="cuda")
+    admit = N.spd_prefill_adaptive(model, x.cuda(), T, cu, vis, slc, tgt, t_skip, w1, 1.0, 3, h,
+                                   logits, ws, ablate=bits)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    np.testing.assert_array_equal(admit.astype(np.int64), admit0)
+    assert rowwise_rel(h.cpu().numpy(), h0) < TOL
+    assert rowwise_rel(logits.cpu().numpy(), lg0) < TOL
+
+
 def test_adaptive_plan_with_given_plan_is_the_plain_prefill():
     # the same tokens, the plan the online rule chose, run through spd_prefill: the same result up
     # to the order of the residual adds (split-K red.add), i.e. to fp32 rounding

@@ -153,3 +153,43 @@ def test_received_attention_repeat_runs_are_bitwise_identical():
     maps = _maps(3, 8, 512, 512)
     a, b = _gpu_received(maps), _gpu_received(maps)
     np.testing.assert_array_equal(a, b)
+
+
+# ---- ablation variants of the MSV-Prune table ----
+# Scores of the KL kind within 5e-5 relative (floor 1e-2): the fp32 softmax exp(F - lse) of rows
+# whose entries reach |F| ~ 20 carries a relative error of about eps32 |F - lse| ~ 3e-6 in every
+# probability; times the log-ratios (~ 40) that KL sums, about 1e-4 absolute on scores of a few units.
+def _score_rtol(kw):
+    return 5e-5 if kw.get("sim") == "kl" else 1e-5
+
+
+@pytest.mark.parametrize("kw", [
+    dict(sim="mse"),                                      # cos -> MSE
+    dict(sim="kl"),                                       # cos -> KL
+    dict(use_anchor_sim=False),                           # without similarity to the anchors
+    dict(use_final_sim=False),                            # only middle-layer tokens
+    dict(layer_weight=[0.0, 1.0]),                        # without middle-layer tokens
+    dict(use_final_sim=False, layer_weight=[0.0, 1.0]),   # without the intra-cluster bracket
+    dict(n_clusters=1),                                   # without semantic clustering
+    dict(n_clusters=2), dict(n_clusters=8),
+    dict(sim="kl", n_clusters=8, use_anchor_sim=False),
+    dict(sim="mse", anchor_ratio=0.0),
+], ids=lambda kw: "-".join(f"{k}={v}" for k, v in kw.items()))
+def test_ablation_variants(kw):
+    # the LLaVA-1.5 shape (576 patches x 1024, layers 12 and 24, 16 heads), keep 128
+    _, v, res = conditioned_vision(20260701, 1, 576, 1024, 2, 16, 128, 1, **kw)
+    assert_prune_parity(gpu_prune(v, 128, 1, **kw), res, _score_rtol(kw))
+
+
+@pytest.mark.parametrize("sim", ["mse", "kl"])
+def test_ablation_sims_streamed_kmeans_and_three_layers(sim):
+    # the L2-streaming K-means (more tiles than one wave of resident clusters) with an early,
+    # middle and final layer, for the similarity kinds whose cluster sums are raw rows
+    vs, res = [], []
+    for i in range(20):
+        _, v1, r1 = conditioned_vision(20260801 + 89 * i, 1, 576, 256, 3, 8, 64, 2, sim=sim)
+        vs.append(v1)
+        res += r1
+    v = {"feats": [np.concatenate([x["feats"][l] for x in vs]) for l in range(3)],
+         "attn": np.concatenate([x["attn"] for x in vs])}
+    assert_prune_parity(gpu_prune(v, 64, 2, sim=sim), res, _score_rtol(dict(sim=sim)))

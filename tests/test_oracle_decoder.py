@@ -266,3 +266,52 @@ def test_adaptive_plan_equals_prefill_with_its_own_frozen_plan():
     np.testing.assert_array_equal(h, h0)
     np.testing.assert_array_equal(lg, lg0)
     assert np.all(admit < 3)  # decisions only inside the window
+
+
+# ---- ablation variants of ASL-Skip (the ASL-Skip ablation table) ----------------------------------
+def test_skippability_without_one_term():
+    model, _ = tiny_model(std=0.05)
+    D = model["cfg"]["d_model"]
+    rng = np.random.default_rng(5)
+    q = rng.standard_normal(D)
+    h = np.stack([q, -q, np.zeros(D), q])  # rows 0-2 visual, 3 text
+    seq_of = np.zeros(4, dtype=np.int64)
+    # without E_ii: parallel to the text mean leaves nothing (F = 1), antiparallel everything (F = 0)
+    s_sa, e, _ = od.skippability(model, h, np.arange(2), seq_of, [np.array([3])], use_entropy=False)
+    np.testing.assert_array_equal(e, 0.0)
+    np.testing.assert_allclose(s_sa, [0.0, 1.0], atol=1e-12)
+    # without F_itc: a zero hidden state reads uniform logits through the lens (E = 1): S_sa = 0;
+    # a one-hot vocabulary distribution would give S_sa = 1
+    s_sa, _, f = od.skippability(model, h, np.array([2]), seq_of, [np.array([3])], use_itc=False)
+    np.testing.assert_array_equal(f, 0.0)
+    np.testing.assert_allclose(s_sa, [0.0], atol=1e-12)
+
+
+def test_adaptive_plan_without_accumulation_needs_one_layer_over_threshold():
+    # with w1 = 0, S_skip is w2 SLC^Norm(l) of the layer alone: the first layer whose own score
+    # reaches T_skip (0.9 at layer 3), where accumulation admits at layer 1 (0.3 + 0.5)
+    model, x, vis = _adaptive_case()
+    slc = np.array([0.3, 0.5, 0.4, 0.9])
+    tgt = np.array([1, 2, 1, 2], np.uint8)
+    _, _, admit, target, _ = od.prefill_adaptive(model, x, [0, len(x)], vis, slc, tgt, t_skip=0.75,
+                                                 w1=0.0, w2=1.0, window=4, accumulate=False)
+    assert np.all(admit[vis] == 3) and np.all(target[vis] == 2)
+    assert np.all(admit[~vis] == -1)
+
+
+def test_adaptive_plan_without_slc_freezes_whole_layers():
+    # without SLC an admitted token bypasses both sub-layers: its residual row stops changing at its
+    # admission layer, so it equals the row that a run of only the layers before it leaves
+    model, x, vis = _adaptive_case(n_layers=5)
+    slc = np.full(5, 100.0)  # must have no effect
+    tgt = np.array([1, 2, 1, 2, 1], np.uint8)
+    kw = dict(t_skip=1.0, w1=1.0, w2=1.0, window=4, use_slc=False, use_entropy=False)
+    h, _, admit, target, _ = od.prefill_adaptive(model, x, [0, len(x)], vis, slc, tgt, **kw)
+    assert (admit > 0).any() and np.all(target[admit >= 0] == 3)
+    for a in sorted(set(admit[admit > 0].tolist())):
+        sub = dict(model, layers=model["layers"][:a], cfg=dict(model["cfg"], n_layers=a))
+        h_a, _, admit_a, _, _ = od.prefill_adaptive(sub, x, [0, len(x)], vis, slc[:a], tgt[:a],
+                                                   **dict(kw, window=min(4, a)))
+        rows = np.flatnonzero(admit == a)
+        np.testing.assert_array_equal(h[rows], h_a[rows])
+        assert np.all(admit_a[rows] == -1)
