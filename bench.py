@@ -247,6 +247,17 @@ def decode_steps(torch, N, spider, mask, dev, steps, warmup, hbm, max_len=512):
     torch.cuda.synchronize()
     assert N.spd_workspace_status(ws) == 0, "device-side failure recorded"
     ms = s.elapsed_time(e) / steps
+    # traced pass: device time and algorithmic bytes per kernel class (events around every launch,
+    # so the classes' sum exceeds the untraced step)
+    N.spd_trace_enable(steps * 400)
+    for k in range(steps):
+        N.spd_decode(model, x, [pos + k], cache, max_len, out, ws)
+    per = {}
+    for name, c in (("gemv", N.TRACE_GEMM), ("attention", N.TRACE_ATTN), ("rows", N.TRACE_ROWS)):
+        r = N.spd_trace_read(c)
+        per[name] = {"launches_per_token": r["launches"] / steps, "ms_per_token": r["ms"] / steps,
+                     "GB/s": r["bytes"] / (r["ms"] / 1000.0) / 1e9 if r["ms"] > 0 else None}
+    N.spd_trace_enable(0)
     L, D, F, V = cfg["n_layers"], cfg["d_model"], cfg["d_ffn"], cfg["vocab"]
     kvd = cfg["n_kv_heads"] * cfg["head_dim"]
     qd = cfg["n_heads"] * cfg["head_dim"]
@@ -254,7 +265,7 @@ def decode_steps(torch, N, spider, mask, dev, steps, warmup, hbm, max_len=512):
     cbytes = 2.0 * L * (pos + steps / 2) * 2 * kvd
     gbs = (wbytes + cbytes) / (ms / 1000.0) / 1e9
     return {"ms_per_token": ms, "tokens_per_s": 1000.0 / ms, "context": pos, "GB/s": gbs,
-            "hbm_frac": gbs / hbm,
+            "hbm_frac": gbs / hbm, "kernels": per,
             "what": "spd_decode, batch 1, after spd_prefill_kv of the SPIDER sequence (pruned, skip plan)"}
 
 

@@ -554,6 +554,7 @@ struct HostPlan {
   std::vector<int> kv0, kvlen;  // per sequence: first key row and key count of its attention
   std::vector<LayerLists> ll;
   size_t pos_off = 0, kvrow_off = 0, last_off = 0, end = 0;
+  bool decode = false;  // one query per sequence at its last position (attention_decode_run)
 };
 
 // Token t of sequence b = seq_of at position pos_all; its K/V row is kvrow (cache modes) or t.
@@ -574,6 +575,7 @@ void plan_init(HostPlan& P, const spd_model_cfg& c, const int32_t* cu, int B, in
     P.kvlen[b] = (pos ? pos[b] : 0) + cu[b + 1] - cu[b];
   }
   P.ll.assign(c.n_layers, LayerLists{});
+  P.decode = false;
   size_t off = 0;
   P.pos_off = off;
   for (int t = 0; t < T; ++t) P.hl[off + t] = P.pos_all[t];
@@ -656,9 +658,8 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
   int rc;
   // attention sub-layer: norm of every row (K/V need all tokens); one GEMM gives K, V of every
   // token and Q of the query tokens (rows of skipped tokens computed but not stored: the
-  // contraction is weight-bound, one pass over Wq|Wk|Wv beats two launches)
-  if ((rc = rmsnorm_run(h, T, D, W.attn_norm, c.rms_eps, nullptr, bf.xa, nullptr, nullptr, st)))
-    return rc;
+  // contraction is weight-bound, one pass over Wq|Wk|Wv beats two launches). On the
+  // matrix-vector path (a few tokens) the GEMM applies the norm itself.
   const KVDest dest = kvd_dest ? *kvd_dest : KVDest{bf.kv, T, false};
   const int32_t* kvrow = dest.cache ? dl + P.kvrow_off : nullptr;
   GemmProblem kvp{};
@@ -676,6 +677,17 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
   kvp.rope = m->freq;
   kvp.rope_rows = kvd;
   kvp.head_dim = hd;
+  auto with_norm = [&](GemmProblem& p, const uint16_t* gain, const int32_t* rows, int n,
+                       void* xbuf) -> int {
+    if (gemm_fuses_norm(p)) {
+      p.norm_h = h;
+      p.norm_gain = gain;
+      p.norm_rows = rows;
+      p.norm_eps = c.rms_eps;
+      return SPD_OK;
+    }
+    return rmsnorm_run(h, n, D, gain, c.rms_eps, rows, xbuf, nullptr, nullptr, st);
+  };
   if (q.na > 0) {
     GemmProblem qp = kvp;
     qp.map_w = &W.m_qkv;
@@ -690,15 +702,22 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
     qp.ldo2 = 2 * kvd;
     qp.split = qd;
     qp.n_tok_out = q.na;
+    if ((rc = with_norm(qp, W.attn_norm, nullptr, T, bf.xa))) return rc;
     if ((rc = gemm_run(qp, bf.gs, st))) return rc;
-  } else if ((rc = gemm_run(kvp, bf.gs, st))) {
-    return rc;
+  } else {
+    if ((rc = with_norm(kvp, W.attn_norm, nullptr, T, bf.xa))) return rc;
+    if ((rc = gemm_run(kvp, bf.gs, st))) return rc;
   }
   if (q.na > 0) {
-    if ((rc = attention_run(bf.q, q.na, dest.kv, dest.n_rows, 2 * kvd, kvd, bf.o, qd,
-                            reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
-                            c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx)))
-      return rc;
+    if (P.decode)
+      rc = attention_decode_run(bf.q, dest.kv, 2 * kvd, kvd, bf.o, qd,
+                                reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, c.n_heads,
+                                c.n_kv_heads, hd, st, q.ctx);
+    else
+      rc = attention_run(bf.q, q.na, dest.kv, dest.n_rows, 2 * kvd, kvd, bf.o, qd,
+                         reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
+                         c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx);
+    if (rc) return rc;
     GemmProblem op{};
     op.map_w = &W.m_o;
     op.w = W.wo;
@@ -713,9 +732,6 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
     if ((rc = gemm_run(op, bf.gs, st))) return rc;
   }
   if (q.nf > 0) {
-    if ((rc = rmsnorm_run(h, q.nf, D, W.ffn_norm, c.rms_eps, dl + q.frows, bf.y, nullptr, nullptr,
-                          st)))
-      return rc;
     GemmProblem gp{};
     gp.map_w = &W.m_gu;
     gp.w = W.wgu;
@@ -727,6 +743,7 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
     gp.out = bf.act;
     gp.ldo = c.d_ffn;
     gp.out_cols = c.d_ffn;
+    if ((rc = with_norm(gp, W.ffn_norm, dl + q.frows, q.nf, bf.y))) return rc;
     if ((rc = gemm_run(gp, bf.gs, st))) return rc;
     GemmProblem dp{};
     dp.map_w = &W.m_d;
@@ -749,9 +766,6 @@ int run_head(const spd_model* m, const HostPlan& P, const PrefillBufs& bf, const
              float* h, int B, float* logits, cudaStream_t st) {
   if (!logits) return SPD_OK;
   const spd_model_cfg& c = m->cfg;
-  if (int rc = rmsnorm_run(h, B, c.d_model, m->final_norm, c.rms_eps, dl + P.last_off, bf.z, nullptr,
-                           nullptr, st))
-    return rc;
   GemmProblem lp{};
   lp.map_w = &m->m_lm;
   lp.w = m->lm_head;
@@ -762,6 +776,15 @@ int run_head(const spd_model* m, const HostPlan& P, const PrefillBufs& bf, const
   lp.epi = EPI_F32;
   lp.out = logits;
   lp.ldo = c.vocab;
+  if (gemm_fuses_norm(lp)) {  // the final norm of the last tokens, inside the matrix-vector kernel
+    lp.norm_h = h;
+    lp.norm_gain = m->final_norm;
+    lp.norm_rows = dl + P.last_off;
+    lp.norm_eps = c.rms_eps;
+  } else if (int rc = rmsnorm_run(h, B, c.d_model, m->final_norm, c.rms_eps, dl + P.last_off, bf.z,
+                                  nullptr, nullptr, st)) {
+    return rc;
+  }
   return gemm_run(lp, bf.gs, st);
 }
 
@@ -997,6 +1020,7 @@ extern "C" int spd_decode(const spd_model* m, const uint16_t* x, int B, const in
   for (int b = 0; b <= B; ++b) cu[b] = b;
   static thread_local HostPlan P;
   plan_init(P, c, cu.data(), B, B, bf.list_ints, pos, max_len);
+  P.decode = true;
   for (int l = 0; l < c.n_layers; ++l) plan_layer(P, l, nullptr, cu.data(), B, B);
   int32_t* dl = bf.lists;
   SPD_CUDA_TRY(cudaMemcpyAsync(dl, P.hl.data(), P.end * sizeof(int32_t), cudaMemcpyHostToDevice, st));

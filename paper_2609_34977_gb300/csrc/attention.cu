@@ -16,12 +16,16 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <cooperative_groups.h>
+
 #include "internal.h"
 #include "ptx.cuh"
 #include "trace.h"
 
 namespace spd {
 namespace {
+
+namespace cg = cooperative_groups;
 
 constexpr int kTK = 128;              // keys per block (S columns, K of the PV product)
 constexpr uint32_t kBox = 128 * 128;  // one TMA box: 128 rows x 64 bf16
@@ -305,6 +309,135 @@ int launch(const CUtensorMap& mq, const CUtensorMap& mkv, void* o, int ldo, cons
   return SPD_OK;
 }
 
+// ---- one query per sequence (a decode step) ---------------------------------------------------
+// Cluster of kDecSplit CTAs per (tile, head): the tile's single query (its sequence's last position,
+// so every key of the sequence is visible) against the keys [first key row, + key count), CTA r of
+// the cluster taking the r-th contiguous quarter of them. Within a CTA the 8 warps take keys j with
+// j mod 8 = warp; each lane holds HD / 32 consecutive elements of the head. A warp keeps an online
+// softmax (running maximum m, sum l, output o) over its keys, four keys' K and V loads in flight;
+// the warps' states are merged in warp order, then the CTAs' states in rank order by rank 0
+// through distributed shared memory, which writes the output in bf16. At one query per sequence
+// there is no tile for the tensor cores to fill: the step reads K and V once, over enough CTAs to
+// keep many loads in flight.
+constexpr int kDecWarps = 8;
+constexpr int kDecSplit = 4;
+
+template <int HD>
+__global__ void __launch_bounds__(kDecWarps * 32)
+    attn_decode_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ kv,
+                       int ldkv, int v_off, __nv_bfloat16* __restrict__ o, int ldo,
+                       const int4* __restrict__ tiles, int n_heads, int n_kv_heads, float scale_log2) {
+  constexpr int E = HD / 32;  // elements per lane: 2 or 4
+  __shared__ float wm[kDecWarps], wl[kDecWarps];
+  __shared__ float wo[kDecWarps][HD];
+  __shared__ float cm, cl, co[HD];  // this CTA's merged state
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = int(cluster.block_rank());
+  pdl_launch_dependents();
+  pdl_wait();
+  const int head = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int4 tl = tiles[blockIdx.x];  // (query row, query count = 1, first key row, key count)
+  const int j_lo = rank * tl.w / kDecSplit, j_hi = (rank + 1) * tl.w / kDecSplit;
+  const int g = head / (n_heads / n_kv_heads);
+  float qv[E];
+  {
+    const __nv_bfloat16* qp = q + size_t(tl.x) * (n_heads * HD) + head * HD + lane * E;
+#pragma unroll
+    for (int e = 0; e < E; ++e) qv[e] = __bfloat162float(qp[e]) * scale_log2;
+  }
+  auto load_row = [&](int j, int off, float (&r)[E]) {
+    const __nv_bfloat16* p = kv + size_t(tl.z + j) * ldkv + off + g * HD + lane * E;
+    if constexpr (E == 4) {
+      const uint2 u = *reinterpret_cast<const uint2*>(p);
+      r[0] = __uint_as_float(u.x << 16);
+      r[1] = __uint_as_float(u.x & 0xffff0000u);
+      r[2] = __uint_as_float(u.y << 16);
+      r[3] = __uint_as_float(u.y & 0xffff0000u);
+    } else {
+      const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
+      r[0] = __uint_as_float(u << 16);
+      r[1] = __uint_as_float(u & 0xffff0000u);
+    }
+  };
+  float m = -INFINITY, l = 0.0f, acc[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) acc[e] = 0.0f;
+  for (int j0 = j_lo + warp; j0 < j_hi; j0 += 4 * kDecWarps) {
+    float kr[4][E], vr[4][E];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = j0 + u * kDecWarps;
+      if (j < j_hi) {
+        load_row(j, 0, kr[u]);
+        load_row(j, v_off, vr[u]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = j0 + u * kDecWarps;
+      if (j < j_hi) {  // warp-uniform
+        float sdot = 0.0f;
+#pragma unroll
+        for (int e = 0; e < E; ++e) sdot = fmaf(qv[e], kr[u][e], sdot);
+#pragma unroll
+        for (int off = 16; off; off >>= 1) sdot += __shfl_xor_sync(0xffffffffu, sdot, off);
+        const float mn = fmaxf(m, sdot);
+        const float corr = exp2f(m - mn), pj = exp2f(sdot - mn);
+        l = l * corr + pj;
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[e] = fmaf(pj, vr[u][e], acc[e] * corr);
+        m = mn;
+      }
+    }
+  }
+  if (lane == 0) {
+    wm[warp] = m;
+    wl[warp] = l;
+  }
+#pragma unroll
+  for (int e = 0; e < E; ++e) wo[warp][lane * E + e] = acc[e];
+  __syncthreads();
+  // merge of states (m_i, l_i, o_i): m = max m_i, l = sum l_i 2^(m_i - m), o = sum o_i 2^(m_i - m)
+  // (a state without keys has m = -inf and contributes nothing)
+  if (threadIdx.x < HD) {
+    float mt = -INFINITY;
+    for (int w = 0; w < kDecWarps; ++w) mt = fmaxf(mt, wm[w]);
+    float lt = 0.0f, ot = 0.0f;
+    for (int w = 0; w < kDecWarps; ++w) {
+      const float f = wm[w] == -INFINITY ? 0.0f : exp2f(wm[w] - mt);
+      lt = fmaf(wl[w], f, lt);
+      ot = fmaf(wo[w][threadIdx.x], f, ot);
+    }
+    co[threadIdx.x] = ot;
+    if (threadIdx.x == 0) {
+      cm = mt;
+      cl = lt;
+    }
+  }
+  cluster.sync();
+  if (rank == 0 && threadIdx.x < HD) {
+    float ms[kDecSplit], ls[kDecSplit], os[kDecSplit];
+#pragma unroll
+    for (int r = 0; r < kDecSplit; ++r) {
+      ms[r] = *cluster.map_shared_rank(&cm, r);
+      ls[r] = *cluster.map_shared_rank(&cl, r);
+      os[r] = cluster.map_shared_rank(co, r)[threadIdx.x];
+    }
+    float mt = -INFINITY;
+#pragma unroll
+    for (int r = 0; r < kDecSplit; ++r) mt = fmaxf(mt, ms[r]);
+    float lt = 0.0f, ot = 0.0f;
+#pragma unroll
+    for (int r = 0; r < kDecSplit; ++r) {
+      const float f = ms[r] == -INFINITY ? 0.0f : exp2f(ms[r] - mt);
+      lt = fmaf(ls[r], f, lt);
+      ot = fmaf(os[r], f, ot);
+    }
+    o[size_t(tl.x) * ldo + head * HD + threadIdx.x] = __float2bfloat16_rn(ot / lt);
+  }
+  cluster.sync();  // the peers' shared memory stays alive until rank 0 has read it
+}
+
 }  // namespace
 
 int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, int v_off, void* o,
@@ -330,6 +463,45 @@ int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, in
   trace_end(slot, stream, TR_ATTN, 4.0 * head_dim * n_heads * ctx_sum,
             2.0 * (2.0 * n_q * n_heads * head_dim + 2.0 * n_kv * n_kv_heads * head_dim));
   return rc;
+}
+
+int attention_decode_run(const void* q, const void* kv, int ldkv, int v_off, void* o, int ldo,
+                         const int4* tiles, int n_tiles, int n_heads, int n_kv_heads, int head_dim,
+                         cudaStream_t stream, double ctx_sum) {
+  if (n_tiles <= 0) return SPD_OK;
+  if (head_dim != 128 && head_dim != 64)
+    return fail(SPD_EUNSUPPORTED, "attention supports head_dim 64 and 128");
+  if (n_kv_heads < 1 || n_heads % n_kv_heads)
+    return fail(SPD_EINVAL, "n_heads must be a multiple of n_kv_heads");
+  if ((ldkv | v_off) % 4) return fail(SPD_EINVAL, "K/V rows must be 8-byte aligned");
+  const float scale_log2 = float(1.4426950408889634 / sqrt(double(head_dim)));
+  const int slot = trace_begin(stream);
+  const auto* qb = static_cast<const __nv_bfloat16*>(q);
+  const auto* kb = static_cast<const __nv_bfloat16*>(kv);
+  auto* ob = static_cast<__nv_bfloat16*>(o);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_tiles, n_heads, kDecSplit);
+  cfg.blockDim = dim3(kDecWarps * 32);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = kDecSplit;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (head_dim == 128)
+    SPD_CUDA_TRY(cudaLaunchKernelEx(&cfg, attn_decode_kernel<128>, qb, kb, ldkv, v_off, ob, ldo, tiles,
+                                    n_heads, n_kv_heads, scale_log2));
+  else
+    SPD_CUDA_TRY(cudaLaunchKernelEx(&cfg, attn_decode_kernel<64>, qb, kb, ldkv, v_off, ob, ldo, tiles,
+                                    n_heads, n_kv_heads, scale_log2));
+  // Q read and O written once per query; K and V of every visible key once per KV head
+  trace_end(slot, stream, TR_ATTN, 4.0 * head_dim * n_heads * ctx_sum,
+            2.0 * (2.0 * n_tiles * n_heads * head_dim + 2.0 * ctx_sum * n_kv_heads * head_dim));
+  return SPD_OK;
 }
 
 }  // namespace spd

@@ -96,7 +96,17 @@ struct KArgs {
   int* counters;
   int* status;
   long long budget;
+  const float* norm_h;  // matrix-vector path: input RMSNorm (see GemmProblem)
+  const uint16_t* norm_gain;
+  const int32_t* norm_rows;
+  float norm_eps;
 };
+
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+  for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
 
 __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
@@ -930,6 +940,198 @@ int make_operand_map(CUtensorMap* map, const void* ptr, int inner, int outer, in
 
 namespace {
 
+// ---- matrix-vector path (at most kGemvTok tokens, e.g. a decode step) ----------------------------
+// With a handful of tokens the contraction is a pure weight stream: no tensor-core tile can be
+// filled, and the tiled kernel's fixed costs (TMEM, barriers, a ring sized for wide tiles) and its
+// shared-memory traffic per weight byte cap it well below the HBM roof. Here each CTA owns 32
+// weight rows (warp w: rows 4w .. 4w + 3) over a range of K; every lane streams 16-byte chunks
+// (eight bf16) so that one warp load covers 512 contiguous bytes of a row, with eight loads in
+// flight per lane, and multiplies them with the tokens' chunks staged in shared memory (fp32
+// accumulation, fixed order). The first batch of weight loads is issued before the grid waits
+// on its predecessor (weights do not depend on it). The 32 row sums are then laid out as the
+// tcgen05 accumulator would hold them (lane = row within the 32-row group, eight token columns)
+// and go through the same fused epilogues. Residual (ADD) epilogues may split K over several CTAs
+// (red.add, as in the tiled kernel); the others own whole rows.
+constexpr int kGemvTok = 4;
+constexpr int kGemvThreads = 256;
+constexpr int kGemvChunk = 256;  // K elements per chunk column (32 lanes x 8 bf16)
+
+__device__ __forceinline__ int4 ld_weights(const int4* p) {
+  int4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.s32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+// acc + the dot product of eight bf16 pairs (w, x), element 2i in the low half of word i
+__device__ __forceinline__ float dot8_bf16(const int4& w, const int4& x, float acc) {
+  const uint32_t wu[4] = {uint32_t(w.x), uint32_t(w.y), uint32_t(w.z), uint32_t(w.w)};
+  const uint32_t xu[4] = {uint32_t(x.x), uint32_t(x.y), uint32_t(x.z), uint32_t(x.w)};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    acc = fmaf(__uint_as_float(wu[i] << 16), __uint_as_float(xu[i] << 16), acc);
+    acc = fmaf(__uint_as_float(wu[i] & 0xffff0000u), __uint_as_float(xu[i] & 0xffff0000u), acc);
+  }
+  return acc;
+}
+
+// NT: tokens computed (>= n_tok); CPR: chunks of a row per batch. A warp's work is a sequence of
+// batches (row pair, block of CPR chunk columns). One register buffer per warp: latency is hidden
+// by the number of resident warps (measured faster than double-buffering registers, which lowers
+// occupancy).
+template <int EPI, int NT, int CPR>
+__global__ void __launch_bounds__(kGemvThreads)
+    gemv_kernel(const uint16_t* __restrict__ w, const uint16_t* __restrict__ x, const KArgs a,
+                int ksplit) {
+  extern __shared__ __align__(16) uint8_t gsm[];
+  __shared__ float red[32][NT];
+  __shared__ int trow[kGemvTok], tpos[kGemvTok];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int grp = blockIdx.x / ksplit, ks = blockIdx.x - grp * ksplit;
+  const int n0 = grp * 32;
+  const int C = a.k / kGemvChunk;
+  const int kc0 = ks * C / ksplit, kc1 = (ks + 1) * C / ksplit, nc = kc1 - kc0;
+  const int nblk = (nc + CPR - 1) / CPR;  // chunk blocks per row pair
+  const int nb = 2 * nblk;                // batches of this warp (two row pairs)
+  const int4* xs = reinterpret_cast<const int4*>(gsm);  // [NT][nc * 32] chunks of this K range
+  const size_t wrow = size_t(a.k) / 8;                  // int4 per weight row
+  const int4* wbase = reinterpret_cast<const int4*>(w) + size_t(kc0) * 32 + lane;
+  // batch b: rows n0 + 4 warp + 2 (b / nblk) + {0, 1}, chunk columns (b % nblk) CPR + u
+  auto load = [&](int4 (&buf)[2][CPR], int b) {
+    const int rp = b / nblk, c0 = (b - rp * nblk) * CPR;
+    const int r = n0 + 4 * warp + 2 * rp;
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int u = 0; u < CPR; ++u)
+        buf[h][u] = (c0 + u < nc && r + h < a.n_out)
+                        ? ld_weights(wbase + size_t(r + h) * wrow + 32 * (c0 + u))
+                        : make_int4(0, 0, 0, 0);
+  };
+  float acc[2][NT];
+  auto compute = [&](const int4 (&buf)[2][CPR], int b) {
+    const int rp = b / nblk, blk = b - rp * nblk, c0 = blk * CPR;
+    if (blk == 0) {
+#pragma unroll
+      for (int t = 0; t < NT; ++t) acc[0][t] = acc[1][t] = 0.0f;
+    }
+#pragma unroll
+    for (int u = 0; u < CPR; ++u) {
+      const int c = c0 + u;
+      if (c < nc) {
+#pragma unroll
+        for (int t = 0; t < NT; ++t) {
+          const int4 xv = xs[t * nc * 32 + c * 32 + lane];
+          acc[0][t] = dot8_bf16(buf[0][u], xv, acc[0][t]);
+          acc[1][t] = dot8_bf16(buf[1][u], xv, acc[1][t]);
+        }
+      }
+    }
+    if (blk == nblk - 1) {  // the row pair is complete
+#pragma unroll
+      for (int t = 0; t < NT; ++t) {
+        const float s0 = warp_sum_f(acc[0][t]), s1 = warp_sum_f(acc[1][t]);
+        if (lane == 0) {
+          red[4 * warp + 2 * rp][t] = s0;
+          red[4 * warp + 2 * rp + 1][t] = s1;
+        }
+      }
+    }
+  };
+  pdl_launch_dependents();
+  int4 b0[2][CPR];
+  load(b0, 0);  // weights do not depend on the predecessor: in flight before the wait
+  pdl_wait();
+  if (a.norm_h) {  // the input RMSNorm of each token's fp32 row, computed by every CTA
+    __shared__ float nred[kGemvThreads / 32][NT];
+    __shared__ float ninv[NT];
+#pragma unroll
+    for (int t = 0; t < NT; ++t) {
+      float ss = 0.0f;
+      if (t < a.n_tok) {
+        const float4* hr = reinterpret_cast<const float4*>(
+            a.norm_h + size_t(a.norm_rows ? a.norm_rows[t] : t) * a.k);
+        for (int c = threadIdx.x; c < a.k / 4; c += kGemvThreads) {
+          const float4 v = hr[c];
+          ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        }
+      }
+      ss = warp_sum_f(ss);
+      if (lane == 0) nred[warp][t] = ss;
+    }
+    __syncthreads();
+    if (threadIdx.x < NT) {
+      float tot = 0.0f;
+      for (int i = 0; i < kGemvThreads / 32; ++i) tot += nred[i][threadIdx.x];
+      ninv[threadIdx.x] = rsqrtf(tot / float(a.k) + a.norm_eps);
+    }
+    __syncthreads();
+    int4* xd = reinterpret_cast<int4*>(gsm);
+    for (int e = threadIdx.x; e < NT * nc * 32; e += kGemvThreads) {
+      const int t = e / (nc * 32), c = e - t * (nc * 32);
+      int4 r = make_int4(0, 0, 0, 0);
+      if (t < a.n_tok) {
+        const size_t k0 = size_t(kc0 * 32 + c) * 8;
+        const float* hr = a.norm_h + size_t(a.norm_rows ? a.norm_rows[t] : t) * a.k + k0;
+        const float4 v0 = reinterpret_cast<const float4*>(hr)[0], v1 = reinterpret_cast<const float4*>(hr)[1];
+        const uint4 gg = *reinterpret_cast<const uint4*>(a.norm_gain + k0);
+        const float inv = ninv[t];
+        const float hv[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+        const uint32_t gw[4] = {gg.x, gg.y, gg.z, gg.w};
+        uint32_t pk[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {  // the same products and rounding as the RMSNorm kernel
+          const __nv_bfloat162 b2 = __floats2bfloat162_rn(hv[2 * i] * inv * __uint_as_float(gw[i] << 16),
+                                                          hv[2 * i + 1] * inv * __uint_as_float(gw[i] & 0xffff0000u));
+          pk[i] = *reinterpret_cast<const uint32_t*>(&b2);
+        }
+        r = make_int4(int(pk[0]), int(pk[1]), int(pk[2]), int(pk[3]));
+      }
+      xd[e] = r;
+    }
+    if (threadIdx.x < a.n_tok) {
+      trow[threadIdx.x] = a.rows ? a.rows[threadIdx.x] : threadIdx.x;
+      tpos[threadIdx.x] = a.pos ? a.pos[threadIdx.x] : 0;
+    }
+  } else {  // tokens' chunks of this K range; token rows past n_tok are zeros
+    int4* xd = reinterpret_cast<int4*>(gsm);
+    for (int e = threadIdx.x; e < NT * nc * 32; e += kGemvThreads) {
+      const int t = e / (nc * 32), c = e - t * (nc * 32);
+      xd[e] = t < a.n_tok ? reinterpret_cast<const int4*>(x + size_t(t) * a.k)[kc0 * 32 + c]
+                          : make_int4(0, 0, 0, 0);
+    }
+    if (threadIdx.x < a.n_tok) {
+      trow[threadIdx.x] = a.rows ? a.rows[threadIdx.x] : threadIdx.x;
+      tpos[threadIdx.x] = a.pos ? a.pos[threadIdx.x] : 0;
+    }
+  }
+  __syncthreads();
+#pragma unroll 1
+  for (int b = 0; b < nb; ++b) {
+    if (b > 0) load(b0, b);
+    compute(b0, b);
+  }
+  __syncthreads();
+  if (warp == 0) {
+    float v[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) v[t] = t < NT ? red[lane][t] : 0.0f;
+    epilogue8<EPI>(a, n0 + lane, (n0 >> 5) & 3, lane, n0 >> 7, 0, v, trow, tpos, 0);
+  }
+}
+
+using GemvFn = void (*)(const uint16_t*, const uint16_t*, KArgs, int);
+template <int NT, int CPR>
+GemvFn gemv_for(int epi) {
+  switch (epi) {
+    case EPI_F32: return gemv_kernel<EPI_F32, NT, CPR>;
+    case EPI_ADD_F32: return gemv_kernel<EPI_ADD_F32, NT, CPR>;
+    case EPI_SWIGLU_BF16: return gemv_kernel<EPI_SWIGLU_BF16, NT, CPR>;
+    case EPI_QKV_BF16: return gemv_kernel<EPI_QKV_BF16, NT, CPR>;
+    default: return nullptr;
+  }
+}
+
 using KernelFn = void (*)(CUtensorMap, CUtensorMap, KArgs);
 
 template <bool PAIR>
@@ -1001,11 +1203,95 @@ int max_active_clusters(int C) {
 
 }  // namespace
 
+namespace {
+// Algorithmic work of one GEMM call (valid output columns only; weights, activations and results
+// move once; fused QKV: query rows count for the query tokens only), recorded with its trace slot.
+void trace_gemm(int slot, const GemmProblem& p, cudaStream_t stream) {
+  if (slot < 0) return;
+  const double cols = (p.epi == EPI_SWIGLU_BF16) ? 2.0 * p.out_cols : double(p.n_out);
+  const double out_cols = (p.epi == EPI_SWIGLU_BF16) ? double(p.out_cols) : double(p.n_out);
+  const double ob = (p.epi == EPI_F32) ? 4.0 : (p.epi == EPI_ADD_F32) ? 8.0 : 2.0;
+  double tok_cols = double(p.n_tok) * cols, tok_out = double(p.n_tok) * out_cols;
+  if (p.epi == EPI_QKV_BF16) {
+    tok_cols = double(p.n_tok_out) * p.split + double(p.n_tok) * (p.n_out - p.split);
+    tok_out = tok_cols;
+  }
+  trace_end(slot, stream, TR_GEMM, 2.0 * tok_cols * p.k,
+            2.0 * cols * p.k + 2.0 * p.n_tok * p.k + ob * tok_out);
+}
+
+bool gemv_eligible(const GemmProblem& p) {
+  if (p.norm_h && ((reinterpret_cast<uintptr_t>(p.norm_h) | reinterpret_cast<uintptr_t>(p.norm_gain)) & 15))
+    return false;
+  return p.n_tok <= kGemvTok && p.w && p.k % kGemvChunk == 0 &&
+         (reinterpret_cast<uintptr_t>(p.w) & 15) == 0 && (reinterpret_cast<uintptr_t>(p.x) & 15) == 0 &&
+         gemv_for<1, 4>(p.epi) != nullptr;
+}
+
+int gemv_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
+  KArgs a{};
+  a.n_out = p.n_out;
+  a.n_tok = p.n_tok;
+  a.k = p.k;
+  a.out = p.out;
+  a.ldo = p.ldo;
+  a.out2 = p.out2;
+  a.ldo2 = p.ldo2;
+  a.split = p.split;
+  a.rows = p.rows;
+  a.rows2 = p.rows2;
+  a.bias = p.bias;
+  a.pos = p.pos;
+  a.rope = reinterpret_cast<const float2*>(p.rope);
+  a.rope_rows = p.rope_rows;
+  a.head_dim = p.head_dim;
+  a.out_cols = p.out_cols;
+  a.status = s.status;
+  a.norm_h = p.norm_h;
+  a.norm_gain = p.norm_gain;
+  a.norm_rows = p.norm_rows;
+  a.norm_eps = p.norm_eps;
+  const int groups = (p.n_out + 31) / 32, C = p.k / kGemvChunk;
+  // residual epilogues split K until about two CTAs per SM stream (each at least one chunk column)
+  int ksplit = 1;
+  if (p.epi == EPI_ADD_F32)
+    while (groups * ksplit < 2 * num_sms() && ksplit * 2 <= C && ksplit < 8) ksplit *= 2;
+  const bool one = p.n_tok == 1;
+  const int nt = one ? 1 : kGemvTok;
+  const size_t smem = size_t(nt) * ((C + ksplit - 1) / ksplit) * kGemvChunk * sizeof(uint16_t);
+  const GemvFn kern = one ? gemv_for<1, 4>(p.epi) : gemv_for<kGemvTok, 4>(p.epi);
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [] {
+    for (int e : {int(EPI_F32), int(EPI_ADD_F32), int(EPI_SWIGLU_BF16), int(EPI_QKV_BF16)})
+      for (GemvFn f : {gemv_for<1, 4>(e), gemv_for<kGemvTok, 4>(e)}) {
+        const cudaError_t r = cudaFuncSetAttribute(reinterpret_cast<const void*>(f),
+                                                   cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   200 * 1024);
+        if (r != cudaSuccess && attr_err == cudaSuccess) attr_err = r;
+      }
+  });
+  if (attr_err != cudaSuccess)
+    return fail(SPD_ECUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
+  if (smem > 200 * 1024) return fail(SPD_EUNSUPPORTED, "GEMV K range too long");
+  const int slot = trace_begin(stream);
+  SPD_CUDA_TRY(launch_pdl(kern, dim3(groups * ksplit), dim3(kGemvThreads), smem, stream,
+                          static_cast<const uint16_t*>(p.w), static_cast<const uint16_t*>(p.x), a,
+                          ksplit));
+  trace_gemm(slot, p, stream);
+  return SPD_OK;
+}
+}  // namespace
+
+bool gemm_fuses_norm(const GemmProblem& p) { return p.n_tok > 0 && gemv_eligible(p); }
+
 int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   if (p.n_tok <= 0 || p.n_out <= 0) return SPD_OK;
   if (p.k <= 0) return fail(SPD_EINVAL, "GEMM K must be positive");
   if (!kernel_for(p.epi, false)) return fail(SPD_EINVAL, "unknown GEMM epilogue %d", p.epi);
   if (!p.map_w && !p.w) return fail(SPD_EINVAL, "GEMM without weights");
+  if (gemv_eligible(p)) return gemv_run(p, s, stream);
+  if (p.norm_h) return fail(SPD_EINVAL, "input RMSNorm fusion needs the matrix-vector path");
   if (cudaError_t e = set_kernel_attributes())
     return fail(SPD_ECUDA, "cudaFuncSetAttribute: %s", cudaGetErrorString(e));
   KArgs a{};
@@ -1141,20 +1427,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
     cfg.numAttrs = 2;
     SPD_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, map_w, map_x, a));
   }
-  if (slot >= 0) {
-    // algorithmic work: valid output columns only; weights, activations and results move once
-    // (fused QKV: query rows count for the query tokens only)
-    const double cols = (p.epi == EPI_SWIGLU_BF16) ? 2.0 * p.out_cols : double(p.n_out);
-    const double out_cols = (p.epi == EPI_SWIGLU_BF16) ? double(p.out_cols) : double(p.n_out);
-    const double ob = (p.epi == EPI_F32) ? 4.0 : (p.epi == EPI_ADD_F32) ? 8.0 : 2.0;
-    double tok_cols = double(p.n_tok) * cols, tok_out = double(p.n_tok) * out_cols;
-    if (p.epi == EPI_QKV_BF16) {
-      tok_cols = double(p.n_tok_out) * p.split + double(p.n_tok) * (p.n_out - p.split);
-      tok_out = tok_cols;
-    }
-    trace_end(slot, stream, TR_GEMM, 2.0 * tok_cols * p.k,
-              2.0 * cols * p.k + 2.0 * p.n_tok * p.k + ob * tok_out);
-  }
+  trace_gemm(slot, p, stream);
   return SPD_OK;
 }
 

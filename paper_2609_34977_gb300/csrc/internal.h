@@ -92,7 +92,16 @@ struct GemmProblem {
   const int32_t* rows2;      // EPI_QKV_BF16: row of token t in out2 (null = t)
   int ldo2, split;
   int n_tok_out;             // EPI_QKV_BF16: tokens whose first-output rows are stored (tracing)
+  // Optional RMSNorm of the input, for the matrix-vector path only (gemm_fuses_norm): x is then
+  // bf16(norm_gain * h[r] * rsqrt(mean h[r]^2 + norm_eps)) of fp32 rows r = norm_rows[t] (null = t)
+  // of norm_h [.][k], and `x` is not read.
+  const float* norm_h;
+  const uint16_t* norm_gain;
+  const int32_t* norm_rows;
+  float norm_eps;
 };
+// True when gemm_run will run p on the matrix-vector path, which can apply the input RMSNorm itself.
+bool gemm_fuses_norm(const GemmProblem& p);
 
 // Scratch of stream-K partial slots (fp32, two per CTA) and per-tile arrival counters. The counters
 // must be zero before a GEMM runs; every GEMM leaves them zero again when it completes.
@@ -120,6 +129,11 @@ int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, in
                   int ldo, const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads,
                   int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum);
 constexpr int kAttnTileQ = 128;  // queries per attention tile
+// The same attention when every tile holds ONE query at its sequence's last position (a decode
+// step): tiles as above with query count 1; ctx_sum = the summed key counts.
+int attention_decode_run(const void* q, const void* kv, int ldkv, int v_off, void* o, int ldo,
+                         const int4* tiles, int n_tiles, int n_heads, int n_kv_heads, int head_dim,
+                         cudaStream_t stream, double ctx_sum);
 int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream);
 
 // ---- ASL-Skip online scores (Sec. 4.2.1, Eq. 6) -------------------------------------------------

@@ -101,3 +101,27 @@ def test_linear_cta_pairs(M, K, N_, epi):
         assert rowwise_rel(got, want) < 1e-4
     if epi == N.EPI_F32:  # split tiles are summed in CTA order: bit-identical runs
         assert torch.equal(outs[0], outs[1])
+
+
+@pytest.mark.parametrize("M", [1, 2, 3, 4])
+@pytest.mark.parametrize("K,N_", [(256, 1000), (4096, 4096), (11008, 640)])
+def test_linear_few_tokens_matrix_vector_path(M, K, N_):
+    # at most four tokens with K a multiple of 256: the matrix-vector kernel (F32 output, and the
+    # residual scatter-add, whose K range is split over several CTAs)
+    X, W = operands(M, K, N_, seed=M + K)
+    ref = bf16_np(X) @ bf16_np(W).T
+    ws = torch.zeros(N.spd_linear_workspace_size(M, N_), dtype=torch.uint8, device="cuda")
+    out = torch.full((M, N_), float("nan"), device="cuda")
+    N.spd_linear(X.cuda(), M, K, W.cuda(), N_, N.EPI_F32, out, N_, ws)
+    h0 = torch.randn(9, N_, device="cuda")
+    h = h0.clone()
+    rows = torch.randperm(9)[:M].to(torch.int32)
+    N.spd_linear(X.cuda(), M, K, W.cuda(), N_, N.EPI_ADD_F32, h, N_, ws, rows=rows.cuda())
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    assert rowwise_rel(out.cpu().numpy(), ref) < 1e-4
+    ref_h = h0.cpu().double().numpy()
+    ref_h[rows.numpy()] += ref
+    assert rowwise_rel(h.cpu().numpy(), ref_h) < 1e-4
+    other = np.setdiff1d(np.arange(9), rows.numpy())
+    assert torch.equal(h[other], h0[other])

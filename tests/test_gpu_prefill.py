@@ -260,8 +260,10 @@ def test_adaptive_plan_with_given_plan_is_the_plain_prefill():
 
 
 # ---- KV cache and decode steps ---------------------------------------------------------------------
-def _decode_case(seed, lens, n_vis, n_layers=3):
-    cfg = dict(synth.TINY_DECODER, n_layers=n_layers)
+def _decode_case(seed, lens, n_vis, n_layers=3, d_ffn=None, **over):
+    cfg = dict(synth.TINY_DECODER, n_layers=n_layers, **over)
+    if d_ffn:
+        cfg["d_ffn"] = d_ffn
     model, om = build(cfg, seed)
     T = sum(lens)
     x = inputs(T, cfg["d_model"], seed + 1)
@@ -295,11 +297,17 @@ def test_prefill_kv_equals_prefill_and_fills_the_cache():
         assert np.abs(c[:, b, :n]).max() > 0 and not c[:, b, n:].any()  # written rows only
 
 
-@pytest.mark.parametrize("steps", [1, 2])
-def test_decode_steps_equal_prefill_of_the_extended_sequences(steps):
-    lens, n_vis = [30, 45], [20, 30]
-    cfg, model, om, x, cu, mask = _decode_case(43, lens, n_vis)
-    T, B, max_len, D = x.shape[0], 2, 64, cfg["d_model"]
+@pytest.mark.parametrize("steps,B,d_ffn,over", [
+    (1, 2, None, {}), (2, 2, None, {}),  # d_ffn 688: the down projection on the tiled kernel
+    (2, 1, 768, {}),                     # every contraction on the one-token matrix-vector kernel
+    (1, 3, 768, {}),                     # the few-token matrix-vector kernel (three tokens of four)
+    (1, 5, 768, {}),                     # five tokens: the tiled tcgen05 kernel
+    (2, 2, 768, dict(n_heads=2, n_kv_heads=1, head_dim=128)),  # head_dim 128, grouped KV heads
+])
+def test_decode_steps_equal_prefill_of_the_extended_sequences(steps, B, d_ffn, over):
+    lens, n_vis = [30, 45, 20, 33, 12][:B], [20, 30, 10, 25, 5][:B]
+    cfg, model, om, x, cu, mask = _decode_case(43, lens, n_vis, d_ffn=d_ffn, **over)
+    T, max_len, D = x.shape[0], 64, cfg["d_model"]
     cache = torch.zeros(N.spd_kv_cache_bytes(model, B, max_len) // 2, dtype=torch.bfloat16, device="cuda")
     ws = torch.zeros(N.spd_prefill_workspace_size(model, T, B), dtype=torch.uint8, device="cuda")
     h = torch.zeros((T, D), device="cuda")
