@@ -77,6 +77,8 @@ def test_linear_split_tiles_are_deterministic():
 
 @pytest.mark.parametrize("M,K,N_,epi", [
     (256, 1024, 22016, N.EPI_F32),      # CTA pairs, stream-K (86 pair tiles > 76 pair slots)
+    (300, 1024, 12288, N.EPI_F32),      # stream-K over two token tiles (96 tiles)
+    (256, 1024, 40960, N.EPI_F32),      # CTA pairs, stream-K over 160 pair tiles
     (256, 4096, 12288, N.EPI_F32),      # CTA pairs, one tile per pair (48 pair tiles)
     (230, 2048, 11008, N.EPI_F32),      # CTA pairs, stream-K, ragged token tile halves
     (200, 4096, 4096, N.EPI_ADD_F32),   # CTA pairs, split-K with red.add
