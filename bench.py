@@ -473,7 +473,11 @@ def main():
         torch.cuda.synchronize()
         return s.elapsed_time(e) / steps, 1000.0 * (time.perf_counter() - t0) / steps
 
+    ms_host, _ = timed_policy(a.steps, a.warmup)  # decisions read back per window layer
+    admit_host = spider.admit.copy()
+    policy["device_plan"] = 1                      # decisions and row lists on the device
     ms_ad, _ = timed_policy(a.steps, a.warmup)
+    assert np.array_equal(spider.admit, admit_host), "device and host plans disagree"
     admitted = float((spider.admit[spider.token_is_visual] >= 0).mean())
     realized = od_expand(spider.admit, m_llava[:L], L)
     ms_given = timed(spider, realized, a.steps, a.warmup)
@@ -481,6 +485,8 @@ def main():
                 "admitted_visual_fraction": admitted,
                 "ms_per_step_same_plan_given": ms_given,
                 "online_plan_overhead_ms": ms_ad - ms_given,
+                "ms_per_step_host_plan": ms_host,
+                "plan": "device (admissions and row lists built by kernels; one read-back per step)",
                 "policy": "T_skip 20, w1 3, w2 1, window 16 (L/2), Table 9 targets, SLC^Norm seeded"}
     pb = prune_batch(torch, N, synth, dev, a.steps, a.warmup, hbm)
     ra = received_batch(torch, N, dev, a.steps, a.warmup, hbm)

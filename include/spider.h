@@ -278,6 +278,12 @@ typedef struct {
   const uint8_t* layer_target; /* host [n_layers]: m(l), 1 = attention, 2 = FFN */
   const uint8_t* is_visual;    /* host [n_tokens]: 1 for the visual tokens (the skip candidates) */
   int ablate;                  /* bit set of SPD_SKIP_NO_* below; 0 = the method as printed */
+  int device_plan;             /* 0: each window layer's admissions are read back to the host, which
+                                  builds that layer's row lists (one stream synchronisation per
+                                  window layer; sub-layers without active tokens launch nothing).
+                                  1: admissions and row lists stay on the device (a list-building
+                                  kernel per window layer; the sub-layers run over every row with
+                                  the lists' padding skipped); one synchronisation at the end. */
 } spd_skip_policy;
 
 /* Ablation variants of ASL-Skip (the ASL-Skip ablation table). w1 = 0 is the variant without
@@ -303,8 +309,8 @@ size_t spd_prefill_adaptive_workspace_size(const spd_model* m, int max_tokens, i
  *   S_sa  = ReLU(1 - E_ii - F_itc),  S_skip(i) += w1 S_sa + w2 SLC^Norm(l),
  * and enters skip mode when S_skip(i) >= T_skip, bypassing sub-layer m(l) (frozen) from layer l
  * on. Arguments as spd_prefill; admit_layer (HOST int16 [n_tokens]) receives each token's
- * admission layer (-1 = never). The call reads each window layer's admissions back to the host
- * (one stream synchronisation per window layer) to build that layer's row lists.
+ * admission layer (-1 = never); the call returns once it is filled (see device_plan for where the
+ * decisions are taken). device_plan = 1 supports at most 1024 sequences.
  * Errors as spd_prefill. */
 int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int n_tokens, const int32_t* cu_seqlens,
                          int n_seqs, const spd_skip_policy* policy, int16_t* admit_layer, float* h,

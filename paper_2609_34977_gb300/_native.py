@@ -62,7 +62,7 @@ class ModelCfg(C.Structure):
 class SkipPolicy(C.Structure):
     _fields_ = [("t_skip", C.c_float), ("w1", C.c_float), ("w2", C.c_float), ("window", C.c_int),
                 ("slc_norm", C.c_void_p), ("layer_target", C.c_void_p), ("is_visual", C.c_void_p),
-                ("ablate", C.c_int)]
+                ("ablate", C.c_int), ("device_plan", C.c_int)]
 
 
 SPD_SKIP_NO_ENTROPY = 1
@@ -297,16 +297,17 @@ def spd_prefill_adaptive_workspace_size(model: SpdModel, max_tokens: int, max_se
 
 
 def spd_prefill_adaptive(model: SpdModel, x, n_tokens, cu_seqlens, is_visual, slc_norm, layer_target,
-                         t_skip, w1, w2, window, h, logits, ws, stream=None, ablate=0):
+                         t_skip, w1, w2, window, h, logits, ws, stream=None, ablate=0, device_plan=0):
     """Prefill with the online ASL-Skip plan; returns the admission layer of every token (host
-    int16, -1 = never). ablate: bit set of SPD_SKIP_NO_*."""
+    int16, -1 = never). ablate: bit set of SPD_SKIP_NO_*; device_plan: decisions and row lists on
+    the device (1) or read back per window layer (0)."""
     cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
     slc = np.ascontiguousarray(slc_norm, dtype=np.float32)
     tgt = np.ascontiguousarray(layer_target, dtype=np.uint8)
     vis = np.ascontiguousarray(is_visual, dtype=np.uint8)
     admit = np.full(n_tokens, -9, dtype=np.int16)
     pol = SkipPolicy(float(t_skip), float(w1), float(w2), int(window), slc.ctypes.data, tgt.ctypes.data,
-                     vis.ctypes.data, int(ablate))
+                     vis.ctypes.data, int(ablate), int(device_plan))
     _check(lib().spd_prefill_adaptive(model.handle, _p(x), n_tokens, cu.ctypes.data, len(cu) - 1,
                                       C.byref(pol), admit.ctypes.data, _p(h), _p(logits), _p(ws),
                                       ws.numel() * ws.element_size(), _stream(stream)))

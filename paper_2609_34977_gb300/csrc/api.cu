@@ -8,12 +8,14 @@
 
 #include <algorithm>
 #include <mutex>
+#include <memory>
 #include <vector>
 
 #include "internal.h"
 #include "ptx.cuh"
 
 namespace spd {
+thread_local int g_no_overlap = 0;
 
 int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float eps,
                 const int32_t* in_rows, void* out, const int32_t* map2, void* out2,
@@ -650,7 +652,8 @@ struct KVDest {
 
 // Decoder layer l on the residual stream h with its lists at dl (device copy of the plan).
 int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P, const PrefillBufs& bf,
-              const int32_t* dl, float* h, int T, cudaStream_t st, const KVDest* kvd_dest = nullptr) {
+              const int32_t* dl, float* h, int T, cudaStream_t st, const KVDest* kvd_dest = nullptr,
+              bool dev_lists = false) {
   const spd_model_cfg& c = m->cfg;
   const int D = c.d_model, hd = c.head_dim;
   const int qd = c.n_heads * hd, kvd = c.n_kv_heads * hd;
@@ -716,7 +719,7 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
     else
       rc = attention_run(bf.q, q.na, dest.kv, dest.n_rows, 2 * kvd, kvd, bf.o, qd,
                          reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
-                         c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx);
+                         c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx, dev_lists);
     if (rc) return rc;
     GemmProblem op{};
     op.map_w = &W.m_o;
@@ -825,6 +828,12 @@ struct AdaptiveBufs {
   int32_t* seq;   // [T] sequence of every token
   int32_t* ts;    // [B + 1] text-token ranges
   int32_t* text;  // [T] text-token indices
+  // device plan
+  int32_t* admit;   // [T] admission layer (-1 = never)
+  uint8_t* target;  // [T] frozen target
+  int32_t* cu;      // [B + 1]
+  int32_t* kv0;     // [B] first key row of each sequence
+  int32_t* kvlen;   // [B] key count of each sequence
 };
 AdaptiveBufs carve_adaptive(const spd_model_cfg& c, int T, int B, Carve& cv) {
   AdaptiveBufs a;
@@ -836,6 +845,11 @@ AdaptiveBufs carve_adaptive(const spd_model_cfg& c, int T, int B, Carve& cv) {
   a.seq = cv.take<int32_t>(T);
   a.ts = cv.take<int32_t>(B + 1);
   a.text = cv.take<int32_t>(T);
+  a.admit = cv.take<int32_t>(T);
+  a.target = cv.take<uint8_t>(T);
+  a.cu = cv.take<int32_t>(B + 1);
+  a.kv0 = cv.take<int32_t>(B);
+  a.kvlen = cv.take<int32_t>(B);
   return a;
 }
 }  // namespace
@@ -894,6 +908,86 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
   SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
   if (int rc = bf16_to_f32_run(x, h, size_t(T) * D, st)) return rc;
 
+  // logit lens of nc candidate tokens (device list): final RMSNorm, then the unembedding in fp32
+  auto lens = [&](const int32_t* cand_dev, int nc) -> int {
+    if (int rc = rmsnorm_run(h, nc, D, m->final_norm, c.rms_eps, cand_dev, bf.xa, nullptr, nullptr, st))
+      return rc;
+    GemmProblem up{};
+    up.map_w = &m->m_lm;
+    up.w = m->lm_head;
+    up.x = bf.xa;
+    up.n_out = c.vocab;
+    up.n_tok = nc;
+    up.k = D;
+    up.epi = EPI_F32;
+    up.out = ab.logits;
+    up.ldo = c.vocab;
+    return gemm_run(up, bf.gs, st);
+  };
+
+  if (pol->device_plan) {
+    // plain stream order inside the decision window: the list builder's outputs feed kernels
+    // several launches later, and with programmatic overlap of the launches in between those
+    // kernels read wrong results in repeated runs (found by testing; plain order measured exact)
+    auto plain_order = std::make_unique<NoOverlap>();
+    // Decisions and row lists on the device: every window layer scores every visual token (those
+    // already in skip mode are passed over), admits on the device, and a kernel rebuilds the row
+    // lists; the sub-layers then run over all T rows with the lists' padding rows skipped. No
+    // host round trip until the admission layers are read back at the end.
+    std::vector<int32_t> vis;
+    for (int t = 0; t < T; ++t)
+      if (pol->is_visual[t]) vis.push_back(t);
+    const int nv = int(vis.size());
+    if (nv > 0)
+      SPD_CUDA_TRY(cudaMemcpyAsync(ab.cand, vis.data(), nv * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+    std::vector<int32_t> kv0(P.kv0.begin(), P.kv0.end()), kvl(P.kvlen.begin(), P.kvlen.end());
+    SPD_CUDA_TRY(cudaMemcpyAsync(ab.cu, cu, (B + 1) * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+    SPD_CUDA_TRY(cudaMemcpyAsync(ab.kv0, kv0.data(), B * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+    SPD_CUDA_TRY(cudaMemcpyAsync(ab.kvlen, kvl.data(), B * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+    SPD_CUDA_TRY(cudaMemsetAsync(ab.admit, 0xff, T * sizeof(int32_t), st));  // -1: never
+    SPD_CUDA_TRY(cudaMemsetAsync(ab.target, 0, T, st));
+    // Each decision layer writes its own list block (written once per call, never while a kernel
+    // that read it may still be resident: a rewritten block could be read through another
+    // kernel's stale cache lines under programmatic overlap); the layers past the window reuse the
+    // last decision layer's block.
+    int max_tiles = 0;
+    for (int b = 0; b < B; ++b) max_tiles += (cu[b + 1] - cu[b] + kAttnTileQ - 1) / kAttnTileQ;
+    double ctx_all = 0.0;
+    for (int t = 0; t < T; ++t) ctx_all += P.pos_all[t] + 1;
+    const int last_block = pol->window > 0 ? pol->window - 1 : 0;
+    for (int l = 0; l < L; ++l) {
+      LayerLists LD = P.ll[l < last_block ? l : last_block];
+      LD.na = T;
+      LD.nf = T;
+      LD.ntiles = max_tiles;
+      LD.ctx = ctx_all;
+      if (l < pol->window && nv > 0) {
+        if (int rc = stream_barrier(st)) return rc;
+        if (mode & kSkipEntropy)
+          if (int rc = lens(ab.cand, nv)) return rc;
+        const float add_slc = no_slc ? 0.0f : pol->w2 * pol->slc_norm[l];
+        if (int rc = skip_scores_run(ab.logits, c.vocab, nv, h, D, ab.cand, ab.ts, ab.text, ab.seq, B,
+                                     ab.tmean, pol->w1, add_slc, pol->t_skip, mode | kSkipDevice,
+                                     ab.s_skip, ab.flag, st, ab.admit, ab.target, l,
+                                     no_slc ? 3 : pol->layer_target[l]))
+          return rc;
+      }
+      if (l <= last_block)  // past the window the plan no longer changes
+        if (int rc = plan_lists_run(T, B, ab.cu, dl + P.pos_off, ab.admit, ab.target, l, ab.kv0,
+                                    ab.kvlen, dl + LD.arows, dl + LD.amap, dl + LD.apos, dl + LD.frows,
+                                    reinterpret_cast<int4*>(dl + LD.tiles), max_tiles, st))
+          return rc;
+      if (int rc = run_layer(m, l, LD, P, bf, dl, h, T, st, nullptr, true)) return rc;
+      if (l == last_block) plain_order.reset();
+    }
+    std::vector<int32_t> ad(T);
+    SPD_CUDA_TRY(cudaMemcpyAsync(ad.data(), ab.admit, T * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+    const int rc = run_head(m, P, bf, dl, h, B, logits, st);
+    SPD_CUDA_TRY(cudaStreamSynchronize(st));
+    for (int t = 0; t < T; ++t) admit_layer[t] = int16_t(ad[t]);
+    return rc;
+  }
+
   std::vector<int> admit(T, -1);
   std::vector<uint8_t> target(T, 0), row(T, 0), flags(T);
   std::vector<int32_t> cand;
@@ -907,22 +1001,8 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
       if (nc > 0) {
         SPD_CUDA_TRY(cudaMemcpyAsync(ab.cand, cand.data(), nc * sizeof(int32_t),
                                      cudaMemcpyHostToDevice, st));
-        if (mode & kSkipEntropy) {
-          // logit lens: final RMSNorm, then the unembedding (LM head) in fp32
-          if (int rc = rmsnorm_run(h, nc, D, m->final_norm, c.rms_eps, ab.cand, bf.xa, nullptr, nullptr, st))
-            return rc;
-          GemmProblem up{};
-          up.map_w = &m->m_lm;
-          up.w = m->lm_head;
-          up.x = bf.xa;
-          up.n_out = c.vocab;
-          up.n_tok = nc;
-          up.k = D;
-          up.epi = EPI_F32;
-          up.out = ab.logits;
-          up.ldo = c.vocab;
-          if (int rc = gemm_run(up, bf.gs, st)) return rc;
-        }
+        if (mode & kSkipEntropy)
+          if (int rc = lens(ab.cand, nc)) return rc;
         const float add_slc = no_slc ? 0.0f : pol->w2 * pol->slc_norm[l];
         if (int rc = skip_scores_run(ab.logits, c.vocab, nc, h, D, ab.cand, ab.ts, ab.text, ab.seq, B,
                                      ab.tmean, pol->w1, add_slc, pol->t_skip, mode, ab.s_skip, ab.flag,

@@ -53,7 +53,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                    const __grid_constant__ CUtensorMap map_kv, __nv_bfloat16* __restrict__ o,
                    int ldo, const int4* __restrict__ tiles, const int32_t* __restrict__ q_pos,
                    int n_heads, int n_kv_heads, int v_off, float scale_log2, int* status,
-                   long long budget) {
+                   long long budget, int lists_late) {
   using L = AttnSmem<HD>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -98,15 +98,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   const uint32_t t_s = tmem, t_o = tmem + 128;
 
-  // the tile list and the positions are written before the stream's previous kernels ran (host
-  // copies), so they are read before the wait; Q, K and V come from the previous kernel
+  // host-copied tile lists and positions were written before the stream's previous kernels ran, so
+  // they are read before the wait; lists built by a kernel (lists_late) only after it. Q, K and V
+  // come from the previous kernel.
+  if (lists_late) {
+    pdl_launch_dependents();
+    pdl_wait();
+  }
   const int4 tl = tiles[blockIdx.x];
   const int q0 = tl.x, nq = tl.y, kv0 = tl.z, len = tl.w;
   const int p_last = q_pos[q0 + nq - 1];  // positions ascend within a tile
   const int nkb = max(1, min((p_last + kTK) / kTK, (len + kTK - 1) / kTK));
   const int my_pos = threadIdx.x < 128 ? q_pos[q0 + min(int(threadIdx.x), nq - 1)] : 0;
-  pdl_launch_dependents();
-  pdl_wait();
+  if (!lists_late) {
+    pdl_launch_dependents();
+    pdl_wait();
+  }
 
   int issued = 0;  // K/V blocks whose loads the producer issued
   if (warp == 4) {
@@ -294,7 +301,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <int HD>
 int launch(const CUtensorMap& mq, const CUtensorMap& mkv, void* o, int ldo, const int4* tiles,
            int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads, int v_off, int* status,
-           cudaStream_t stream) {
+           cudaStream_t stream, int lists_late) {
   using L = AttnSmem<HD>;
   static bool attr = false;
   if (!attr) {
@@ -305,7 +312,7 @@ int launch(const CUtensorMap& mq, const CUtensorMap& mkv, void* o, int ldo, cons
   const float scale_log2 = 1.4426950408889634f / sqrtf(float(HD));
   SPD_CUDA_TRY(launch_pdl(attn_tc_kernel<HD>, dim3(n_tiles, n_heads), dim3(kThreads), L::bytes,
                           stream, mq, mkv, static_cast<__nv_bfloat16*>(o), ldo, tiles, q_pos,
-                          n_heads, n_kv_heads, v_off, scale_log2, status, kWaitBudget));
+                          n_heads, n_kv_heads, v_off, scale_log2, status, kWaitBudget, lists_late));
   return SPD_OK;
 }
 
@@ -442,7 +449,8 @@ __global__ void __launch_bounds__(kDecWarps * 32)
 
 int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, int v_off, void* o,
                   int ldo, const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads,
-                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum) {
+                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum,
+                  bool lists_from_device) {
   if (n_tiles <= 0) return SPD_OK;
   if (head_dim != 128 && head_dim != 64)
     return fail(SPD_EUNSUPPORTED, "attention supports head_dim 64 and 128");
@@ -456,9 +464,9 @@ int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, in
   const int slot = trace_begin(stream);
   const int rc = (head_dim == 128)
                      ? launch<128>(mq, mkv, o, ldo, tiles, n_tiles, q_pos, n_heads, n_kv_heads,
-                                   v_off, status, stream)
+                                   v_off, status, stream, lists_from_device)
                      : launch<64>(mq, mkv, o, ldo, tiles, n_tiles, q_pos, n_heads, n_kv_heads,
-                                  v_off, status, stream);
+                                  v_off, status, stream, lists_from_device);
   // QK^T and PV over each active query's causal context; Q, K, V read once and O written once
   trace_end(slot, stream, TR_ATTN, 4.0 * head_dim * n_heads * ctx_sum,
             2.0 * (2.0 * n_q * n_heads * head_dim + 2.0 * n_kv * n_kv_heads * head_dim));
@@ -485,7 +493,7 @@ int attention_decode_run(const void* q, const void* kv, int ldkv, int v_off, voi
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].val.programmaticStreamSerializationAllowed = overlap_allowed();
   attr[1].id = cudaLaunchAttributeClusterDimension;
   attr[1].val.clusterDim.x = 1;
   attr[1].val.clusterDim.y = 1;

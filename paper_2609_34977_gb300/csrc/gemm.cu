@@ -256,8 +256,9 @@ __device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int t = t0 + j;
-      if (t < nt) {
-        float* p = o + size_t(trow[t - tb]) * a.ldo + n;
+      const int r = t < nt ? trow[t - tb] : -1;  // negative: a padding row of a device-built list
+      if (r >= 0) {
+        float* p = o + size_t(r) * a.ldo + n;
         if constexpr (EPI == EPI_ADD_F32) atomicAdd(p, v[j]);  // fire-and-forget red.add
         else *p = v[j];
       }
@@ -1048,9 +1049,9 @@ __global__ void __launch_bounds__(kGemvThreads)
 #pragma unroll
     for (int t = 0; t < NT; ++t) {
       float ss = 0.0f;
-      if (t < a.n_tok) {
-        const float4* hr = reinterpret_cast<const float4*>(
-            a.norm_h + size_t(a.norm_rows ? a.norm_rows[t] : t) * a.k);
+      const int hrow = t < a.n_tok ? (a.norm_rows ? a.norm_rows[t] : t) : -1;  // -1: list padding
+      if (hrow >= 0) {
+        const float4* hr = reinterpret_cast<const float4*>(a.norm_h + size_t(hrow) * a.k);
         for (int c = threadIdx.x; c < a.k / 4; c += kGemvThreads) {
           const float4 v = hr[c];
           ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
@@ -1070,9 +1071,10 @@ __global__ void __launch_bounds__(kGemvThreads)
     for (int e = threadIdx.x; e < NT * nc * 32; e += kGemvThreads) {
       const int t = e / (nc * 32), c = e - t * (nc * 32);
       int4 r = make_int4(0, 0, 0, 0);
-      if (t < a.n_tok) {
+      const int hrow = t < a.n_tok ? (a.norm_rows ? a.norm_rows[t] : t) : -1;
+      if (hrow >= 0) {
         const size_t k0 = size_t(kc0 * 32 + c) * 8;
-        const float* hr = a.norm_h + size_t(a.norm_rows ? a.norm_rows[t] : t) * a.k + k0;
+        const float* hr = a.norm_h + size_t(hrow) * a.k + k0;
         const float4 v0 = reinterpret_cast<const float4*>(hr)[0], v1 = reinterpret_cast<const float4*>(hr)[1];
         const uint4 gg = *reinterpret_cast<const uint4*>(a.norm_gain + k0);
         const float inv = ninv[t];
@@ -1418,7 +1420,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
     cfg.stream = stream;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[0].val.programmaticStreamSerializationAllowed = overlap_allowed();
     attr[1].id = cudaLaunchAttributeClusterDimension;
     attr[1].val.clusterDim.x = pair ? 2 : (a.cluster ? a.csplit : 1);
     attr[1].val.clusterDim.y = 1;

@@ -26,6 +26,16 @@ constexpr long long kWaitBudget = 1ll << 30;
 
 int num_sms();  // SM count of the current device
 
+// Programmatic overlap of consecutive launches is off on this thread while a NoOverlap guard is
+// alive (launches then follow plain stream order; the kernels' griddepcontrol instructions are
+// no-ops).
+extern thread_local int g_no_overlap;
+struct NoOverlap {
+  NoOverlap() { ++g_no_overlap; }
+  ~NoOverlap() { --g_no_overlap; }
+};
+inline int overlap_allowed() { return g_no_overlap ? 0 : 1; }
+
 // Launches a kernel with programmatic stream serialization: it may be scheduled while the previous
 // kernel of the stream is still running, and orders itself after it with griddepcontrol.wait.
 template <typename... KArgs, typename... Args>
@@ -38,7 +48,7 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].val.programmaticStreamSerializationAllowed = overlap_allowed();
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
@@ -124,10 +134,13 @@ int make_operand_map(CUtensorMap* map, const void* ptr, int inner, int outer, in
 // Causal attention of n_q active queries (q [n_q][n_heads * head_dim], rows grouped by sequence,
 // positions ascending within a sequence) over the keys and values of their sequences (kv
 // [n_kv][ldkv]: K of head g at column g * head_dim, V at v_off + g * head_dim). `tiles` (device
-// int4 [n_tiles]): first query row, query count (<= 128), first key row, sequence length.
+// int4 [n_tiles]): first query row, query count (1..128), first key row, sequence length.
+// lists_from_device: the tiles and q_pos were written by a kernel earlier in the stream (read
+// after the grid dependency wait) rather than copied from the host.
 int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, int v_off, void* o,
                   int ldo, const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads,
-                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum);
+                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum,
+                  bool lists_from_device = false);
 constexpr int kAttnTileQ = 128;  // queries per attention tile
 // The same attention when every tile holds ONE query at its sequence's last position (a decode
 // step): tiles as above with query count 1; ctx_sum = the summed key counts.
@@ -142,10 +155,22 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream);
 // text tokens text[ts[b] .. ts[b+1]) (computed into tmean [B][D]) + 1) / 2 (mode kSkipItc, else 0),
 // S_sa = ReLU(1 - E - F); s_skip[token] = (kSkipAccumulate ? s_skip[token] : 0) + w1 S_sa + add_slc;
 // flag[n] = (s_skip[token] >= t_skip).
-constexpr int kSkipEntropy = 1, kSkipItc = 2, kSkipAccumulate = 4;
+// kSkipDevice: the decision stays on the device: candidates with admit >= 0 are left alone, and
+// one that reaches t_skip gets admit = layer, target = tgt (flag unused).
+constexpr int kSkipEntropy = 1, kSkipItc = 2, kSkipAccumulate = 4, kSkipDevice = 8;
 int skip_scores_run(const float* logits, int V, int n_cand, const float* h, int D, const int32_t* cand,
                     const int32_t* ts, const int32_t* text, const int32_t* seq_of, int B, float* tmean,
                     float w1, float add_slc, float t_skip, int mode, float* s_skip, uint8_t* flag,
-                    cudaStream_t stream);
+                    cudaStream_t stream, int32_t* admit = nullptr, uint8_t* target = nullptr,
+                    int layer = 0, int tgt = 0);
+// An empty kernel launched without programmatic overlap: the kernels after it start only once all
+// earlier work in the stream has completed.
+int stream_barrier(cudaStream_t stream);
+// Layer l's row lists built on the device from admission layers (see plan_lists_kernel).
+constexpr int kPlanMaxSeqs = 1024;
+int plan_lists_run(int T, int B, const int32_t* cu, const int32_t* pos, const int32_t* admit,
+                   const uint8_t* target, int l, const int32_t* kv0, const int32_t* kvlen,
+                   int32_t* arows, int32_t* amap, int32_t* apos, int32_t* frows, int4* tiles,
+                   int max_tiles, cudaStream_t stream);
 
 }  // namespace spd

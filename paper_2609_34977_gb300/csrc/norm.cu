@@ -37,6 +37,7 @@ __global__ void __launch_bounds__(kThreads)
   pdl_wait();
   const int i = blockIdx.x;
   const int r = in_rows ? in_rows[i] : i;
+  if (r < 0) return;  // a padding entry of a device-built row list
   const float4* src = reinterpret_cast<const float4*>(h + size_t(r) * D);
   const int n4 = D / 4;
   float ss = 0.0f;
@@ -124,11 +125,13 @@ __global__ void __launch_bounds__(kThreads)
                       const int32_t* __restrict__ cand, const int32_t* __restrict__ ts,
                       const int32_t* __restrict__ seq_of, const float* __restrict__ tmean,
                       float inv_log_v, float w1, float add_slc, float t_skip, int mode,
-                      float* __restrict__ s_skip, uint8_t* __restrict__ flag) {
+                      float* __restrict__ s_skip, uint8_t* __restrict__ flag,
+                      int32_t* __restrict__ admit, uint8_t* __restrict__ target, int layer, int tgt) {
   __shared__ float red[kThreads / 32];
   pdl_launch_dependents();
   pdl_wait();
   const int n = blockIdx.x, i = cand[n], b = seq_of[i];
+  if ((mode & kSkipDevice) && admit[i] >= 0) return;  // already in skip mode (block-uniform)
   float ent = 0.0f;
   if (mode & kSkipEntropy) {
     const float* z = logits + size_t(n) * V;
@@ -171,7 +174,114 @@ __global__ void __launch_bounds__(kThreads)
     const float fuse = w1 * s_sa + add_slc;
     const float acc = (mode & kSkipAccumulate) ? s_skip[i] + fuse : fuse;
     s_skip[i] = acc;
-    flag[n] = acc >= t_skip ? 1 : 0;
+    if (mode & kSkipDevice) {
+      if (acc >= t_skip) {  // enters skip mode here, its target frozen
+        admit[i] = layer;
+        target[i] = uint8_t(tgt);
+      }
+    } else {
+      flag[n] = acc >= t_skip ? 1 : 0;
+    }
+  }
+}
+
+// Exclusive prefix sum of one int per thread over the block (blockDim.x a multiple of 32, at most
+// 1024); *total receives the block's sum. Every thread must call it.
+__device__ int block_scan_excl(int v, int* tmp, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, off);
+    if (lane >= off) x += y;
+  }
+  if (lane == 31) tmp[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < nw ? tmp[lane] : 0;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, off);
+      if (lane >= off) w += y;
+    }
+    tmp[lane] = w;
+  }
+  __syncthreads();
+  const int before = (warp ? tmp[warp - 1] : 0) + x - v;
+  *total = tmp[nw - 1];
+  __syncthreads();
+  return before;
+}
+
+// Decoder layer l's row lists from the admission layers, built on the device (the executor's plan
+// for a decision made by a kernel): token t bypasses target[t] (1 attention, 2 FFN, 3 both) at
+// layer l when 0 <= admit[t] <= l. Outputs in the executor's layout: arows (attention-active
+// tokens, ascending; padded to T with -1), amap (token -> its query row or -1), apos (positions of
+// the query rows), frows (FFN-active tokens; padded with -1), tiles (up to 128 queries of one
+// sequence each; padded to max_tiles with copies of the last tile, whose recomputation writes the
+// same values, or a one-query tile when no token is a query). One CTA.
+__global__ void __launch_bounds__(1024)
+    plan_lists_kernel(int T, int B, const int32_t* __restrict__ cu, const int32_t* __restrict__ pos,
+                      const int32_t* __restrict__ admit, const uint8_t* __restrict__ target, int l,
+                      const int32_t* __restrict__ kv0, const int32_t* __restrict__ kvlen,
+                      int32_t* __restrict__ arows, int32_t* __restrict__ amap,
+                      int32_t* __restrict__ apos, int32_t* __restrict__ frows, int4* __restrict__ tiles,
+                      int max_tiles) {
+  __shared__ int tmp[32];
+  __shared__ int seq_cnt[kPlanMaxSeqs];
+  pdl_launch_dependents();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  auto bits_of = [&](int t) {
+    const int ad = admit[t];
+    return (ad >= 0 && ad <= l) ? int(target[t]) : 0;
+  };
+  int na = 0, nf = 0;
+  for (int base = 0; base < T; base += blockDim.x) {
+    const int t = base + threadIdx.x;
+    const int bits = t < T ? bits_of(t) : 3;
+    const int a_act = !(bits & 1), f_act = !(bits & 2);
+    int ta, tf;
+    const int ea = block_scan_excl(a_act, tmp, &ta);
+    const int ef = block_scan_excl(f_act, tmp, &tf);
+    if (t < T) {
+      if (a_act) {
+        arows[na + ea] = t;
+        amap[t] = na + ea;
+        apos[na + ea] = pos[t];
+      } else {
+        amap[t] = -1;
+      }
+      if (f_act) frows[nf + ef] = t;
+    }
+    na += ta;
+    nf += tf;
+  }
+  for (int r = na + threadIdx.x; r < T; r += blockDim.x) arows[r] = -1;
+  for (int r = nf + threadIdx.x; r < T; r += blockDim.x) frows[r] = -1;
+  for (int b = warp; b < B; b += blockDim.x >> 5) {  // active queries per sequence
+    int cnt = 0;
+    for (int t = cu[b] + lane; t < cu[b + 1]; t += 32) cnt += !(bits_of(t) & 1);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, off);
+    if (lane == 0) seq_cnt[b] = cnt;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int a = 0, k = 0;
+    for (int b = 0; b < B; ++b) {
+      const int n = seq_cnt[b];
+      for (int s0 = 0; s0 < n; s0 += 128) tiles[k++] = make_int4(a + s0, min(128, n - s0), kv0[b], kvlen[b]);
+      a += n;
+    }
+    int4 pad;
+    if (k > 0) {
+      pad = tiles[k - 1];
+    } else {
+      pad = make_int4(0, 1, kv0[0], kvlen[0]);
+      apos[0] = pos[0];
+    }
+    for (; k < max_tiles; ++k) tiles[k] = pad;
   }
 }
 
@@ -180,13 +290,37 @@ __global__ void __launch_bounds__(kThreads)
 int skip_scores_run(const float* logits, int V, int n_cand, const float* h, int D, const int32_t* cand,
                     const int32_t* ts, const int32_t* text, const int32_t* seq_of, int B, float* tmean,
                     float w1, float add_slc, float t_skip, int mode, float* s_skip, uint8_t* flag,
-                    cudaStream_t stream) {
+                    cudaStream_t stream, int32_t* admit, uint8_t* target, int layer, int tgt) {
   if (mode & kSkipItc)
     SPD_CUDA_TRY(launch_pdl(text_mean_kernel, dim3((D + kThreads - 1) / kThreads, B), dim3(kThreads),
                             0, stream, h, D, ts, text, tmean));
   SPD_CUDA_TRY(launch_pdl(skip_score_kernel, dim3(n_cand), dim3(kThreads), 0, stream,
                           logits, V, h, D, cand, ts, seq_of, static_cast<const float*>(tmean),
-                          float(1.0 / log(double(V))), w1, add_slc, t_skip, mode, s_skip, flag));
+                          float(1.0 / log(double(V))), w1, add_slc, t_skip, mode, s_skip, flag,
+                          admit, target, layer, tgt));
+  return SPD_OK;
+}
+
+namespace {
+__global__ void stream_barrier_kernel() {}
+}  // namespace
+
+int stream_barrier(cudaStream_t stream) {
+  stream_barrier_kernel<<<1, 32, 0, stream>>>();
+  SPD_CUDA_TRY(cudaGetLastError());
+  return SPD_OK;
+}
+
+int plan_lists_run(int T, int B, const int32_t* cu, const int32_t* pos, const int32_t* admit,
+                   const uint8_t* target, int l, const int32_t* kv0, const int32_t* kvlen,
+                   int32_t* arows, int32_t* amap, int32_t* apos, int32_t* frows, int4* tiles,
+                   int max_tiles, cudaStream_t stream) {
+  if (B > kPlanMaxSeqs) return fail(SPD_EUNSUPPORTED, "device plans support at most %d sequences", kPlanMaxSeqs);
+  // an ordinary launch (no programmatic overlap): it starts once all earlier work in the stream
+  // has completed, so every later kernel sees the decisions and the lists complete
+  plan_lists_kernel<<<1, 1024, 0, stream>>>(T, B, cu, pos, admit, target, l, kv0, kvlen, arows, amap,
+                                            apos, frows, tiles, max_tiles);
+  SPD_CUDA_TRY(cudaGetLastError());
   return SPD_OK;
 }
 

@@ -1138,7 +1138,7 @@ cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, size_t smem, cud
   cfg.stream = st;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].val.programmaticStreamSerializationAllowed = overlap_allowed();
   attr[1].id = cudaLaunchAttributeClusterDimension;
   attr[1].val.clusterDim.x = KC;
   attr[1].val.clusterDim.y = 1;

@@ -96,7 +96,7 @@ class SpiderPrefill:
         text [sum(text_lens)][D] bf16. Returns the logits tensor [B][vocab] (device).
 
         policy (dict: slc_norm, layer_target, t_skip, w1, w2, window, optional ablate bits
-        SPD_SKIP_NO_*) replaces skip_mask by the online ASL-Skip plan; the admission layer of every
+        SPD_SKIP_NO_* and device_plan) replaces skip_mask by the online ASL-Skip plan; the admission layer of every
         token is then left in self.admit."""
         if not self.dense:
             N.spd_prune(self.prune_cfg, feats, attn, self.keep_idx, ws=self.ws_prune, stream=stream)
@@ -123,7 +123,8 @@ class SpiderPrefill:
                                             policy["slc_norm"], policy["layer_target"], policy["t_skip"],
                                             policy["w1"], policy["w2"], policy["window"], self.h,
                                             self.logits, self.ws_adaptive, stream=stream,
-                                            ablate=policy.get("ablate", 0))
+                                            ablate=policy.get("ablate", 0),
+                                            device_plan=policy.get("device_plan", 0))
         return self.logits
 
     def status(self) -> int:

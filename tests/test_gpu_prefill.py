@@ -173,7 +173,8 @@ def _adaptive_inputs(seed, lens, n_text):
     return model, om, x, vis, cu
 
 
-def test_adaptive_plan_matches_oracle():
+@pytest.mark.parametrize("device_plan", [0, 1])
+def test_adaptive_plan_matches_oracle(device_plan):
     model, om, x, vis, cu = _adaptive_inputs(31, [64, 40], [16, 8])
     slc = np.array([0.2, 0.5, 0.1, 0.7, 0.3, 0.9])
     tgt = np.array([1, 2, 1, 1, 2, 2], np.uint8)
@@ -193,7 +194,7 @@ def test_adaptive_plan_matches_oracle():
     h = torch.full((T, 256), float("nan"), device="cuda")
     logits = torch.full((len(cu) - 1, 512), float("nan"), device="cuda")
     admit = N.spd_prefill_adaptive(model, x.cuda(), T, cu, vis, slc, tgt, t_skip, 3.0, 1.0, 3, h,
-                                   logits, ws)
+                                   logits, ws, device_plan=device_plan)
     torch.cuda.synchronize()
     assert N.spd_workspace_status(ws) == 0
     np.testing.assert_array_equal(admit.astype(np.int64), admit0)
@@ -206,7 +207,8 @@ def test_adaptive_plan_matches_oracle():
     (N.SPD_SKIP_NO_ENTROPY, 3.0), (N.SPD_SKIP_NO_ITC, 3.0), (N.SPD_SKIP_NO_ACCUM, 3.0),
     (N.SPD_SKIP_NO_SLC, 3.0), (0, 0.0), (N.SPD_SKIP_NO_ACCUM | N.SPD_SKIP_NO_SLC, 3.0)],
     ids=["no_entropy", "no_itc", "no_accum", "no_slc", "no_s_sa", "no_accum_no_slc"])
-def test_adaptive_plan_ablations_match_oracle(bits, w1):
+@pytest.mark.parametrize("device_plan", [0, 1])
+def test_adaptive_plan_ablations_match_oracle(bits, w1, device_plan):
     # the ablation variants of the ASL-Skip table against the oracle's, on a threshold that every
     # decision clears by a margin
     model, om, x, vis, cu = _adaptive_inputs(35, [64, 40], [16, 8])
@@ -231,7 +233,38 @@ def test_adaptive_plan_ablations_match_oracle(bits, w1):
     h = torch.full((T, 256), float("nan"), device="cuda")
     logits = torch.full((len(cu) - 1, 512), float("nan"), device="cuda")
     admit = N.spd_prefill_adaptive(model, x.cuda(), T, cu, vis, slc, tgt, t_skip, w1, 1.0, 3, h,
-                                   logits, ws, ablate=bits)
+                                   logits, ws, ablate=bits, device_plan=device_plan)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    np.testing.assert_array_equal(admit.astype(np.int64), admit0)
+    assert rowwise_rel(h.cpu().numpy(), h0) < TOL
+    assert rowwise_rel(logits.cpu().numpy(), lg0) < TOL
+
+
+@pytest.mark.parametrize("seed,lens,n_text", [
+    (37, [4, 30], [1, 0]),  # a sequence of visual tokens only (no text mean: F_itc = 1/2)
+    (41, [4], [1]),         # four tokens: the matrix-vector path, whose fused norms meet padded lists
+])
+def test_adaptive_device_plan_small_and_textless_sequences(seed, lens, n_text):
+    model, om, x, vis, cu = _adaptive_inputs(seed, lens, n_text)
+    slc = np.array([0.2, 0.5, 0.1, 0.7, 0.3, 0.9])
+    tgt = np.array([1, 2, 1, 1, 2, 2], np.uint8)
+    xn = bf16_np(x)
+    chosen = None
+    for t_skip in np.linspace(0.15, 6.0, 235):
+        h0, lg0, admit0, _, margin = od.prefill_adaptive(om, xn, cu, vis, slc, tgt, t_skip, 3.0, 1.0, 3)
+        if margin > 0.02 and (admit0 >= 0).any() and (admit0[vis] < 0).any():
+            chosen = (t_skip, h0, lg0, admit0)
+            break
+    assert chosen is not None, "no well-separated threshold in the grid"
+    t_skip, h0, lg0, admit0 = chosen
+    T = x.shape[0]
+    B = len(lens)
+    ws = torch.zeros(N.spd_prefill_adaptive_workspace_size(model, T, B), dtype=torch.uint8, device="cuda")
+    h = torch.full((T, 256), float("nan"), device="cuda")
+    logits = torch.full((B, 512), float("nan"), device="cuda")
+    admit = N.spd_prefill_adaptive(model, x.cuda(), T, cu, vis, slc, tgt, t_skip, 3.0, 1.0, 3, h, logits,
+                                   ws, device_plan=1)
     torch.cuda.synchronize()
     assert N.spd_workspace_status(ws) == 0
     np.testing.assert_array_equal(admit.astype(np.int64), admit0)
