@@ -141,10 +141,11 @@ def build_model(torch, N, synth, device, layers=32):
 
 def count_launches(pipe, mask, dense):
     """Kernels of one step: MSV-Prune (6) and the gather, projector (2), text scatter, residual
-    initialisation, final norm and LM head; per layer RMSNorm and the QKV GEMM, attention and O
-    when a token attends, RMSNorm, gate/up and down when a token runs the FFN."""
+    initialisation, final norm and LM head (one matrix-vector launch with the norm fused for at most
+    four sequences); per layer RMSNorm and the QKV GEMM, attention and O when a token attends,
+    RMSNorm, gate/up and down when a token runs the FFN."""
     L = mask.shape[0] if mask is not None else pipe.model.cfg["n_layers"]
-    n = (0 if dense else 7) + 2 + 1 + 1 + 2
+    n = (0 if dense else 7) + 2 + 1 + 1 + (1 if pipe.B <= 4 else 2)
     for l in range(L):
         bits = mask[l] if mask is not None else np.zeros(pipe.T, np.uint8)
         n += 2 + (2 if ((bits & 1) == 0).any() else 0) + (3 if ((bits & 2) == 0).any() else 0)

@@ -155,6 +155,7 @@ __device__ __forceinline__ const float* feat_row(const PruneDims& p, int l, int 
 }
 
 // ---- 1. a_v and inverse norms ---------------------------------------------------------------
+template <int SIM>
 __global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float* __restrict__ attn,
                                                        PruneWs w) {
   pdl_launch_dependents();
@@ -172,8 +173,8 @@ __global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float*
     ss = warp_sum(ss);
     const size_t o = (size_t(l) * p.n_tiles + t) * p.n + i;
     if (lane == 0) w.inv[o] = 1.0f / sqrtf(ss);
-    if (p.sim == SPD_SIM_MSE && lane == 0) w.st1[o] = ss;
-    if (p.sim == SPD_SIM_KL) {  // softmax over the row: max, then sum e^z and sum e^z z (z = x - max)
+    if (SIM == SPD_SIM_MSE && lane == 0) w.st1[o] = ss;
+    if (SIM == SPD_SIM_KL) {  // softmax over the row: max, then sum e^z and sum e^z z (z = x - max)
       float mx = -INFINITY;
       for (int c = lane; c < p.d / 4; c += 32) {
         const float4 v = r[c];
@@ -265,6 +266,7 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
 // finishing 16 rows.
 constexpr int kAS = 4;
 
+template <int SIM>
 __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
     anchor_sim_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
@@ -281,7 +283,7 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
   const int dd = threadIdx.x & 31, r0 = threadIdx.x >> 5;
   // per-row statistics of the final layer (MSE: squared norms; KL: log-sum-exps, negentropies)
   const size_t so = (size_t(p.fin) * p.n_tiles + t) * p.n;
-  const bool kl = p.sim == SPD_SIM_KL;
+  constexpr bool kl = SIM == SPD_SIM_KL;
   const float* urow[8];
   const float* arow[8];
   float ulse[8];  // KL: the non-anchor operand is softmax(F^L_i) = exp(F^L_i - lse_i)
@@ -362,9 +364,9 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
       const int pa = p0 + tx + 16 * j;
       if (pa < p.n_anc) {
         const int ia = al[pa];
-        const float v = p.sim == SPD_SIM_COS ? sdot * iu * inv[ia]
-                        : p.sim == SPD_SIM_MSE ? 2.0f * sdot - w.st1[so + ia]
-                                               : sdot - w.st1[so + ia];
+        const float v = SIM == SPD_SIM_COS ? sdot * iu * inv[ia]
+                        : SIM == SPD_SIM_MSE ? 2.0f * sdot - w.st1[so + ia]
+                                             : sdot - w.st1[so + ia];
         best = fmaxf(best, v);
       }
     }
@@ -373,8 +375,8 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
   for (int off = 8; off; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
   if (tx == 0 && ur < p.m) {
     const int iu = ul[ur];
-    if (p.sim == SPD_SIM_MSE) best = -(w.st1[so + iu] - best) / float(p.d);
-    else if (p.sim == SPD_SIM_KL) best = best - w.st2[so + iu];
+    if (SIM == SPD_SIM_MSE) best = -(w.st1[so + iu] - best) / float(p.d);
+    else if (SIM == SPD_SIM_KL) best = best - w.st2[so + iu];
     atomicMax(&w.asim[size_t(t) * p.n + iu], ordered_key(best));
   }
   cl.sync();  // peers read this CTA's partial tile above
@@ -547,7 +549,9 @@ __device__ __forceinline__ void cluster_column_reduce(cg::cluster_group& cl, flo
 template <int KN>
 constexpr int kmeans_threads() { return KN == 4 ? 256 : 512; }
 
-template <int KC, bool RES, int KN>
+// COS: the similarity kind is the cosine (the paper's); the MSE / KL ablations' extra sums are
+// compiled into the other instance only (the Lloyd loop is instruction-bound).
+template <int KC, bool RES, int KN, bool COS>
 __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
@@ -752,7 +756,7 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
   // of st1 for the MSE and KL similarities
   // (RES: the final layer first, from the resident rows; then each other layer's rows are copied
   // into the same buffer)
-  const bool cos_sim = p.sim == SPD_SIM_COS;
+  constexpr bool cos_sim = COS;
   for (int li = 0; li < p.L; ++li) {
     const int l = RES ? (li == 0 ? p.fin : (li <= p.fin ? li - 1 : li)) : li;
     const float* rstat = (cos_sim ? w.inv : w.st1) + (size_t(l) * p.n_tiles + t) * p.n;
@@ -777,7 +781,7 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
       for (int jj = 0; jj < nl; ++jj) ssum_part[asg[jj]] += rinv[jj];
     }
     column_sums<KN>(part, K, D, nl, asg,
-                    RowAccess{RES ? rows : nullptr, fl, row0, idx, D, cos_sim ? rinv : nullptr});
+                    RowAccess{RES ? rows : nullptr, fl, row0, idx, D, cos_sim ? rinv : static_cast<float*>(nullptr)});
     cl.sync();
     float* csum = w.csum + (size_t(t) * p.L + l) * K * D;
     cluster_column_reduce<KC>(cl, part, K, D, rank,
@@ -1131,6 +1135,7 @@ int g_res_clusters = -1;                 // 16-CTA clusters of it the GPU holds 
 
 template <int KC, bool RES, int KN>
 cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, size_t smem, cudaStream_t st) {
+  auto kern = p.sim == SPD_SIM_COS ? kmeans_kernel<KC, RES, KN, true> : kmeans_kernel<KC, RES, KN, false>;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(KC, p.n_tiles);
   cfg.blockDim = dim3(kmeans_threads<KN>());
@@ -1145,7 +1150,7 @@ cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, size_t smem, cud
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, kmeans_kernel<KC, RES, KN>, p, w);
+  return cudaLaunchKernelEx(&cfg, kern, p, w);
 }
 
 // Kernel attributes (once per process) and whether 16-CTA clusters of the resident kernel fit.
@@ -1162,10 +1167,14 @@ int kmeans_setup() {
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kResSmem));
       return e;
     };
-    err = streamed(kmeans_kernel<8, false, 4>);
-    if (err == cudaSuccess) err = streamed(kmeans_kernel<8, false, SPD_MAX_CLUSTERS>);
-    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, 4>);
-    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, SPD_MAX_CLUSTERS>);
+    err = streamed(kmeans_kernel<8, false, 4, true>);
+    if (err == cudaSuccess) err = streamed(kmeans_kernel<8, false, SPD_MAX_CLUSTERS, true>);
+    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, 4, true>);
+    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, SPD_MAX_CLUSTERS, true>);
+    if (err == cudaSuccess) err = streamed(kmeans_kernel<8, false, 4, false>);
+    if (err == cudaSuccess) err = streamed(kmeans_kernel<8, false, SPD_MAX_CLUSTERS, false>);
+    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, 4, false>);
+    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, SPD_MAX_CLUSTERS, false>);
     g_res_clusters = 0;
     if (err == cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
@@ -1180,7 +1189,7 @@ int kmeans_setup() {
       cfg.attrs = attr;
       cfg.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, kmeans_kernel<16, true, SPD_MAX_CLUSTERS>, &cfg) !=
+      if (cudaOccupancyMaxActiveClusters(&n, kmeans_kernel<16, true, SPD_MAX_CLUSTERS, true>, &cfg) !=
           cudaSuccess) {
         cudaGetLastError();
         n = 0;
@@ -1222,10 +1231,14 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
   cudaStream_t st = static_cast<cudaStream_t>(stream_);
   const int T = p.n_tiles;
   const int slot = trace_begin(st);
-  SPD_CUDA_TRY(launch_pdl(rowstats_kernel, dim3((p.n + 7) / 8, T), dim3(256), 0, st, p, attn, w));
+  SPD_CUDA_TRY(launch_pdl(p.sim == SPD_SIM_COS ? rowstats_kernel<SPD_SIM_COS>
+                          : p.sim == SPD_SIM_MSE ? rowstats_kernel<SPD_SIM_MSE> : rowstats_kernel<SPD_SIM_KL>,
+                          dim3((p.n + 7) / 8, T), dim3(256), 0, st, p, attn, w));
   SPD_CUDA_TRY(launch_pdl(anchor_kernel, dim3(T), dim3(1024), 0, st, p, w));
   if (p.n_anc > 0 && p.m > 0 && p.wa != 0.0f)
-    SPD_CUDA_TRY(launch_pdl(anchor_sim_kernel,
+    SPD_CUDA_TRY(launch_pdl(p.sim == SPD_SIM_COS ? anchor_sim_kernel<SPD_SIM_COS>
+                            : p.sim == SPD_SIM_MSE ? anchor_sim_kernel<SPD_SIM_MSE>
+                                                   : anchor_sim_kernel<SPD_SIM_KL>,
                             dim3((p.m + 63) / 64 * kAS, (p.n_anc + 63) / 64, T), dim3(256), 0, st,
                             p, w));
   // K-means: the rows resident in shared memory over 16 CTAs per tile where they fit and all
