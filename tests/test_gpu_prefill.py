@@ -17,8 +17,8 @@ pytestmark = pytest.mark.gpu
 TOL = 2e-2
 
 
-def build(cfg, seed, std=0.05):
-    w = synth.decoder_weights(seed, cfg, std=std)
+def build(cfg, seed, std=0.05, device="cpu"):
+    w = synth.decoder_weights(seed, cfg, std=std, device=device)
     wd = {k: v for k, v in w.items() if k != "layers"}
     wd = {k: v.cuda() for k, v in wd.items()}
     wd["layers"] = [{k: v.cuda() for k, v in lw.items()} for lw in w["layers"]]
@@ -155,6 +155,48 @@ def test_llava_width_layer_with_cta_pairs():
     mask = np.zeros((1, T), np.uint8)
     mask[0, vis] = r.integers(0, 3, size=192)  # some tokens skip attention, some the FFN
     check(model, om, x, [0, T], mask)
+
+
+def _sampled_plan(lens, n_vis, seed, per_seq=6):
+    """Every token bypasses both sub-layers except, per sequence, a few visual and text tokens that
+    run attention, the FFN or both (the oracle then computes K and V for every token but queries,
+    attention and FFN only for the sampled rows, which keeps a full-width layer cheap on the CPU);
+    the last token of each sequence runs both (its logits)."""
+    r = np.random.default_rng(seed)
+    T = sum(lens)
+    mask = np.full((1, T), 3, np.uint8)
+    start = 0
+    for n, v in zip(lens, n_vis):
+        rows = np.r_[r.choice(v, per_seq, replace=False), v + r.choice(n - v, per_seq, replace=False)]
+        mask[0, start + rows] = r.integers(0, 3, size=len(rows))
+        mask[0, start + n - 1] = 0
+        start += n
+    return mask
+
+
+@pytest.mark.parametrize("shape", ["llava-next-7b", "qwen2-gqa"])
+def test_full_width_layer_at_serving_token_counts(shape):
+    # one decoder layer at the full width of the workload with its token counts: LLaVA-NeXT-7B
+    # (8 requests of 320 kept visual + 128 text tokens) and the Qwen2-style GQA decoder (4 requests
+    # of 256-1024 kept visual + 256 text tokens, 28 query / 4 KV heads); K and V of all ~3600
+    # tokens, sampled query and FFN rows (see _sampled_plan), every row and the logits compared
+    if shape == "llava-next-7b":
+        cfg = dict(n_layers=1, d_model=4096, n_heads=32, n_kv_heads=32, head_dim=128, d_ffn=11008,
+                   vocab=1000, rope_theta=1e4, rms_eps=1e-5, d_vis=0, d_proj=0)
+        n_vis, n_text = [320] * 8, [128] * 8
+    else:
+        cfg = dict(n_layers=1, d_model=3584, n_heads=28, n_kv_heads=4, head_dim=128, d_ffn=18944,
+                   vocab=1000, rope_theta=1e6, rms_eps=1e-6, d_vis=0, d_proj=0)
+        n_vis, n_text = [256, 512, 768, 1024], [256] * 4
+    lens = [v + t for v, t in zip(n_vis, n_text)]
+    model, om = build(cfg, 31, std=0.02, device="cuda")  # weights drawn on the GPU (fast)
+    T = sum(lens)
+    x = inputs(T, cfg["d_model"], 32)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    mask = _sampled_plan(lens, n_vis, 33)
+    h, _ = check(model, om, x, cu, mask)
+    bypass = np.flatnonzero(mask[0] == 3)
+    np.testing.assert_array_equal(h[bypass], bf16_np(x)[bypass])  # the residual passes unchanged
 
 
 # ---- ASL-Skip online plan (Sec. 4.2, Eq. 6, Alg. 1 stage 2) ----------------------------------------
