@@ -71,6 +71,28 @@ def gemm_traffic():
     return None
 
 
+def rank_seed(rank):
+    """Seed of a rank's requests: every rank runs its own independent requests (weak scaling; no
+    collective on the data path)."""
+    return SEED + rank
+
+
+def max_over_ranks(ms, dist, device):
+    """The slowest rank's step time (the job's step ends when its last rank's does)."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([float(ms)], device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank, world, ms):
+    """Whole-job tokens/s: the tokens every rank processed in one step over the slowest rank's
+    step time."""
+    return tokens_per_rank * world / (ms / 1000.0)
+
+
 def od_expand(admit, layer_target, n_layers):
     """Per-layer skip bits of a frozen-target plan (token i bypasses layer_target[admit[i]] from
     layer admit[i] on; -1 = never)."""
@@ -94,7 +116,8 @@ def workload_config(keep, mask, T):
 
 
 class Clocks:
-    """nvidia-smi samples every 200 ms while the timed region runs."""
+    """nvidia-smi samples every 25 ms while the timed region runs (a 20-step region lasts about
+    0.1 s)."""
 
     def __init__(self, gpu):
         self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
@@ -103,7 +126,7 @@ class Clocks:
              "clocks_event_reasons.sw_power_cap")
         try:
             self.p = subprocess.Popen(["nvidia-smi", "-i", str(gpu), f"--query-gpu={q}",
-                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                       "--format=csv,noheader,nounits", "-lms", "25"],
                                       stdout=self.f, stderr=subprocess.DEVNULL)
         except Exception:
             self.p = None
@@ -378,15 +401,15 @@ def main():
                              tiles_per_req=[1], text_lens=[TEXT], dense=dense)
         if dense:
             return pipe, None
-        admit, target = synth.adaptive_plan(SEED + rank, L, pipe.token_is_visual, SKIP_FRAC,
+        admit, target = synth.adaptive_plan(rank_seed(rank), L, pipe.token_is_visual, SKIP_FRAC,
                                             m_llava[:L], min(ADMIT_LO, max(L // 2 - 1, 0)),
                                             max(L // 2, min(ADMIT_LO, max(L // 2 - 1, 0)) + 1))
         return pipe, N.spd_plan_adaptive(L, admit, target)
 
-    v = synth.vision_tiles(SEED + rank, 1, N_PATCH, D_VIS, 2, H_VIS)
+    v = synth.vision_tiles(rank_seed(rank), 1, N_PATCH, D_VIS, 2, H_VIS)
     feats = [torch.from_numpy(f).to(dev) for f in v["feats"]]
     attn = torch.from_numpy(v["attn"]).to(dev)
-    text = torch.from_numpy(synth.text_embeddings(SEED + rank, TEXT, 4096).view(np.int16)).view(
+    text = torch.from_numpy(synth.text_embeddings(rank_seed(rank), TEXT, 4096).view(np.int16)).view(
         torch.bfloat16).to(dev)
 
     def timed(pipe, mask, steps, warmup, trace=False):
@@ -403,12 +426,7 @@ def main():
             pipe.run(feats, attn, text, mask)
         e.record()
         torch.cuda.synchronize()
-        ms = s.elapsed_time(e) / steps
-        if dist:
-            t = torch.tensor([ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
-        return ms
+        return max_over_ranks(s.elapsed_time(e) / steps, dist, dev)
 
     hbm, tf_burst, tf_sust, src = peaks()
     spider, mask = make(a.keep, False)
@@ -419,7 +437,7 @@ def main():
     assert spider.status() == 0, "device-side failure recorded"
     ms_dense = timed(dense, None, a.steps, a.warmup)
     tokens = (N_PATCH + TEXT) * world
-    value = tokens / (ms / 1000.0)
+    value = job_throughput(N_PATCH + TEXT, world, ms)
 
     # traced pass: per-kernel-class device time and algorithmic work over K steps
     timed(spider, mask, a.steps, 1, trace=True)
