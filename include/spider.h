@@ -203,7 +203,7 @@ int spd_model_create(const spd_model_cfg* cfg, const spd_model_weights* w, spd_m
 void spd_model_destroy(spd_model* m);
 
 /* Expands Alg. 1's per-token plan into per-layer skip bits (host only):
- * a token with admit[i] >= 0 bypasses sub-layer target[i] (1 attention, 2 FFN) in every layer
+ * a token with admit[i] >= 0 bypasses sub-layer target[i] (1 attention, 2 FFN, 3 both) in every layer
  * l >= admit[i] (the target is frozen at admission, Sec. 4.2). admit -1 = never.
  * mask (host) uint8 [n_layers][n_tokens]: bit 0 skip attention, bit 1 skip FFN. */
 int spd_plan_adaptive(int n_layers, int n_tokens, const int16_t* admit, const uint8_t* target,
@@ -392,6 +392,44 @@ int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, int N, int ep
 int spd_linear_noalloc(const uint16_t* X, int M, int K, const uint16_t* W, int N, int epilogue,
                        const uint16_t* bias, const int32_t* rows, void* out, int ldo, int* status,
                        void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
+/* The hot path's contract names (thin forms of the calls above)                               */
+/* ------------------------------------------------------------------------------------------ */
+
+/* = spd_prune_workspace_size. */
+size_t spd_prune_workspace(const spd_prune_cfg* cfg);
+
+/* = spd_prefill_workspace_size. */
+size_t spd_prefill_workspace(const spd_model* m, int total_tokens, int n_seqs);
+
+/* = spd_gather_rows_bf16 with the kept patch indices of spd_prune: out[t * keep + j][:] =
+ * bf16(payload[t][has_cls + keep_idx[t][j]][:]). payload (dev) fp32 [n_tiles][n_tok][d] (n_tok rows
+ * per tile, including the [CLS] row when has_cls); keep_idx (dev) int32 [n_tiles][keep]; out (dev)
+ * bf16 [n_tiles * keep][d]; d a multiple of 4. Out-of-range indices are skipped (no report).
+ * Errors as spd_gather_rows_bf16. */
+int spd_gather_bf16(const float* payload, int n_tok, const int32_t* keep_idx, int n_tiles, int keep,
+                    int has_cls, int d, uint16_t* out, void* stream);
+
+/* Copies the message of the calling thread's last failed call (spd_last_error) into buf, at most
+ * n - 1 characters and a terminating NUL (n > 0). Returns the message's full length. */
+int spd_last_error_detail(char* buf, size_t n);
+
+/* Device-side status of a workspace (synchronises `stream`): SPD_OK or the first failure recorded
+ * since the last read (which it clears), or a negative status of the read itself. */
+int spd_check(void* ws, void* stream);
+
+/* = spd_plan_static: a per-layer mask applied to the selected (visual) tokens. */
+int spd_plan_from_layer_mask(int n_layers, int n_tokens, const uint8_t* layer_mask,
+                             const uint8_t* token_is_visual, uint8_t* mask);
+
+/* spd_prefill with Alg. 1's plan in its per-token form: token i bypasses target[i] (1 attention,
+ * 2 FFN, 3 both) in every layer l >= admit_layer[i] (-1 = never). admit_layer (HOST int16
+ * [n_tokens]) and target (HOST uint8 [n_tokens]) are expanded on the host (spd_plan_adaptive);
+ * both NULL = no skipping. Other arguments and errors as spd_prefill. */
+int spd_prefill_admit(const spd_model* m, const uint16_t* x, int n_tokens, const int32_t* cu_seqlens,
+                      int n_seqs, const int16_t* admit_layer, const uint8_t* target, float* h,
+                      float* logits, void* ws, size_t ws_bytes, void* stream);
 
 #ifdef __cplusplus
 }

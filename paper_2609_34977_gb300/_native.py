@@ -28,7 +28,8 @@ EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait"
            "spd_prefill_adaptive", "spd_kv_cache_bytes", "spd_prefill_kv", "spd_decode_workspace_size",
            "spd_decode",
            "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
-           "spd_trace_read")
+           "spd_trace_read", "spd_prune_workspace", "spd_prefill_workspace", "spd_gather_bf16",
+           "spd_last_error_detail", "spd_check", "spd_plan_from_layer_mask", "spd_prefill_admit")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
 
 
@@ -112,6 +113,13 @@ def lib():
             "spd_attention": (i, [vp, i, vp, vp, vp, i, vp, i, i, i, i, vp, vp, sz, vp]),
             "spd_prefill_workspace_size": (sz, [vp, i, i]),
             "spd_prefill": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, sz, vp]),
+            "spd_prune_workspace": (sz, [C.POINTER(PruneCfg)]),
+            "spd_prefill_workspace": (sz, [vp, i, i]),
+            "spd_gather_bf16": (i, [vp, i, vp, i, i, i, i, vp, vp]),
+            "spd_last_error_detail": (i, [C.c_char_p, sz]),
+            "spd_check": (i, [vp, vp]),
+            "spd_plan_from_layer_mask": (i, [i, i, vp, vp, vp]),
+            "spd_prefill_admit": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, vp, sz, vp]),
             "spd_prefill_adaptive_workspace_size": (sz, [vp, i, i]),
             "spd_kv_cache_bytes": (sz, [vp, i, i]),
             "spd_prefill_kv": (i, [vp, vp, i, vp, i, vp, vp, vp, vp, i, vp, sz, vp]),
@@ -342,6 +350,28 @@ def spd_prefill(model: SpdModel, x, n_tokens, cu_seqlens, skip_mask, h, logits, 
     mask = None if skip_mask is None else np.ascontiguousarray(skip_mask, dtype=np.uint8)
     _check(lib().spd_prefill(model.handle, _p(x), n_tokens, _p(cu), len(cu) - 1, _p(mask), _p(h),
                              _p(logits), _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def spd_prefill_admit(model: SpdModel, x, n_tokens, cu_seqlens, admit_layer, target, h, logits, ws,
+                      stream=None):
+    """spd_prefill with the per-token plan (admission layer, frozen target), expanded on the host."""
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    ad = None if admit_layer is None else np.ascontiguousarray(admit_layer, dtype=np.int16)
+    tg = None if target is None else np.ascontiguousarray(target, dtype=np.uint8)
+    _check(lib().spd_prefill_admit(model.handle, _p(x), n_tokens, _p(cu), len(cu) - 1, _p(ad), _p(tg),
+                                   _p(h), _p(logits), _p(ws), ws.numel() * ws.element_size(),
+                                   _stream(stream)))
+
+
+def spd_check(ws, stream=None) -> int:
+    """Device-side status of a workspace (reads and clears it; synchronises the stream)."""
+    return int(lib().spd_check(_p(ws), _stream(stream)))
+
+
+def spd_last_error_detail() -> str:
+    buf = C.create_string_buffer(512)
+    lib().spd_last_error_detail(buf, 512)
+    return buf.value.decode()
 
 
 def spd_linear_workspace_size(M: int, N: int) -> int:

@@ -281,7 +281,7 @@ extern "C" int spd_plan_adaptive(int n_layers, int n_tokens, const int16_t* admi
   memset(mask, 0, size_t(n_layers) * n_tokens);
   for (int i = 0; i < n_tokens; ++i) {
     if (admit[i] < 0) continue;
-    if (target[i] != 1 && target[i] != 2) return fail(SPD_EINVAL, "token %d: target must be 1 or 2", i);
+    if (target[i] < 1 || target[i] > 3) return fail(SPD_EINVAL, "token %d: target must be 1, 2 or 3", i);
     for (int l = admit[i]; l < n_layers; ++l) mask[size_t(l) * n_tokens + i] = target[i];
   }
   return SPD_OK;
@@ -1114,3 +1114,48 @@ extern "C" int spd_decode(const spd_model* m, const uint16_t* x, int B, const in
   return run_head(m, P, bf, dl, h, B, logits, st);
 }
 
+
+// ---- the hot path's contract names (thin forms of the calls above) --------------------------------
+extern "C" size_t spd_prune_workspace(const spd_prune_cfg* cfg) { return spd_prune_workspace_size(cfg); }
+
+extern "C" size_t spd_prefill_workspace(const spd_model* m, int total_tokens, int n_seqs) {
+  return spd_prefill_workspace_size(m, total_tokens, n_seqs);
+}
+
+extern "C" int spd_gather_bf16(const float* payload, int n_tok, const int32_t* keep_idx, int n_tiles,
+                               int keep, int has_cls, int d, uint16_t* out, void* stream) {
+  return spd_gather_rows_bf16(payload, n_tiles, n_tok, d, has_cls ? 1 : 0, keep_idx, keep, out, nullptr,
+                              stream);
+}
+
+extern "C" int spd_last_error_detail(char* buf, size_t n) {
+  const char* msg = spd_last_error();
+  const size_t len = strlen(msg);
+  if (buf && n > 0) {
+    const size_t c = len < n - 1 ? len : n - 1;
+    memcpy(buf, msg, c);
+    buf[c] = '\0';
+  }
+  return int(len);
+}
+
+extern "C" int spd_check(void* ws, void* stream) {
+  int status = SPD_OK;
+  if (int rc = spd_workspace_status(ws, stream, &status)) return rc;
+  return status;
+}
+
+extern "C" int spd_plan_from_layer_mask(int n_layers, int n_tokens, const uint8_t* layer_mask,
+                                        const uint8_t* token_is_visual, uint8_t* mask) {
+  return spd_plan_static(n_layers, n_tokens, layer_mask, token_is_visual, mask);
+}
+
+extern "C" int spd_prefill_admit(const spd_model* m, const uint16_t* x, int T, const int32_t* cu, int B,
+                                 const int16_t* admit_layer, const uint8_t* target, float* h,
+                                 float* logits, void* ws, size_t ws_bytes, void* stream) {
+  if (!admit_layer && !target) return spd_prefill(m, x, T, cu, B, nullptr, h, logits, ws, ws_bytes, stream);
+  if (!m || !admit_layer || !target || T < 1) return fail(SPD_EINVAL, "admit_layer and target go together");
+  std::vector<uint8_t> mask(size_t(m->cfg.n_layers) * T);
+  if (int rc = spd_plan_adaptive(m->cfg.n_layers, T, admit_layer, target, mask.data())) return rc;
+  return spd_prefill(m, x, T, cu, B, mask.data(), h, logits, ws, ws_bytes, stream);
+}

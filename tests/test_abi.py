@@ -75,3 +75,27 @@ def test_workspace_sizes_grow_with_problem(lib):
     b = N.spd_prune_workspace_size(N.prune_cfg(5, 577, 1024, 2, 1, 16, 64))
     assert b > a > 0
     assert N.spd_linear_workspace_size(256, 4096) > 0
+
+
+def test_contract_names_are_the_same_calls(lib):
+    cfg = N.prune_cfg(2, 577, 64, 2, 1, 4, 32)
+    assert lib.spd_prune_workspace(C.byref(cfg)) == lib.spd_prune_workspace_size(C.byref(cfg)) > 0
+    lm = np.array([0, 2, 1], dtype=np.uint8)
+    sel = np.array([1, 0, 1, 1], dtype=np.uint8)
+    a = np.zeros(12, np.uint8)
+    b = np.zeros(12, np.uint8)
+    assert lib.spd_plan_from_layer_mask(3, 4, lm.ctypes.data, sel.ctypes.data, a.ctypes.data) == 0
+    assert lib.spd_plan_static(3, 4, lm.ctypes.data, sel.ctypes.data, b.ctypes.data) == 0
+    np.testing.assert_array_equal(a, b)
+    # a rejected call's message through both forms; truncation to the buffer
+    with pytest.raises(N.SpiderError):
+        N.spd_plan_adaptive(3, np.array([0], np.int16), np.array([5], np.uint8))
+    assert N.spd_last_error_detail() == N.lib().spd_last_error().decode()
+    small = C.create_string_buffer(5)
+    n = lib.spd_last_error_detail(small, 5)
+    assert n == len(N.lib().spd_last_error()) and len(small.value) == 4
+
+
+def test_plan_accepts_both_sublayers_target(lib):
+    mask = N.spd_plan_adaptive(3, np.array([1, -1], np.int16), np.array([3, 1], np.uint8))
+    np.testing.assert_array_equal(mask, [[0, 0], [3, 0], [3, 0]])

@@ -406,3 +406,22 @@ def test_decode_steps_equal_prefill_of_the_extended_sequences(steps, B, d_ffn, o
     got = out.cpu().numpy()
     assert np.isfinite(got).all()
     assert rowwise_rel(got, lo) < TOL
+
+
+def test_prefill_admit_form_equals_the_expanded_plan():
+    # the contract's per-token plan form (admission layer, frozen target, 3 = both sub-layers)
+    model, om, x, vis, cu = _adaptive_inputs(39, [48, 20], [16, 4])
+    T = x.shape[0]
+    r = np.random.default_rng(40)
+    admit = np.where(vis & (r.random(T) < 0.7), r.integers(0, 6, T), -1).astype(np.int16)
+    target = r.integers(1, 4, T).astype(np.uint8)
+    ws = torch.zeros(N.spd_prefill_workspace_size(model, T, 2), dtype=torch.uint8, device="cuda")
+    h = torch.full((T, 256), float("nan"), device="cuda")
+    lg = torch.full((2, 512), float("nan"), device="cuda")
+    N.spd_prefill_admit(model, x.cuda(), T, cu, admit, target, h, lg, ws)
+    assert N.spd_check(ws) == 0
+    mask = od.expand_adaptive_plan(admit, target, 6)
+    h0, lg0 = od.prefill(om, bf16_np(x), cu, mask)
+    assert rowwise_rel(h.cpu().numpy(), h0) < TOL and rowwise_rel(lg.cpu().numpy(), lg0) < TOL
+    h2, lg2 = run(model, x.cuda(), cu, mask)
+    assert rowwise_rel(h.cpu().numpy(), h2) < 1e-5  # the same executor (residual adds in any order)

@@ -193,3 +193,17 @@ def test_ablation_sims_streamed_kmeans_and_three_layers(sim):
     v = {"feats": [np.concatenate([x["feats"][l] for x in vs]) for l in range(3)],
          "attn": np.concatenate([x["attn"] for x in vs])}
     assert_prune_parity(gpu_prune(v, 64, 2, sim=sim), res, _score_rtol(dict(sim=sim)))
+
+
+def test_gather_contract_form_equals_gather_rows():
+    v = synth.vision_tiles(9, 3, 576, 256, 2, 8)
+    src = torch.from_numpy(v["feats"][1]).cuda()
+    idx = torch.stack([torch.randperm(576)[:64].sort().values for _ in range(3)]).to(torch.int32).cuda()
+    a = torch.empty(3 * 64, 256, dtype=torch.bfloat16, device="cuda")
+    b = torch.empty_like(a)
+    assert N.lib().spd_gather_bf16(src.data_ptr(), 577, idx.data_ptr(), 3, 64, 1, 256, a.data_ptr(), None) == 0
+    N.spd_gather_rows_bf16(src, 3, 577, 256, 1, idx, 64, b)
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+    want = torch.from_numpy(v["feats"][1]).cuda()[torch.arange(3).repeat_interleave(64).cuda(), 1 + idx.flatten().long()]
+    assert torch.equal(a, want.to(torch.bfloat16))
