@@ -319,7 +319,7 @@ int launch(const CUtensorMap& mq, const CUtensorMap& mkv, void* o, int ldo, cons
 // ---- one query per sequence (a decode step) ---------------------------------------------------
 // Cluster of kDecSplit CTAs per (tile, head): the tile's single query (its sequence's last position,
 // so every key of the sequence is visible) against the keys [first key row, + key count), CTA r of
-// the cluster taking the r-th contiguous quarter of them. Within a CTA the 8 warps take keys j with
+// the cluster taking the r-th contiguous eighth of them. Within a CTA the 8 warps take keys j with
 // j mod 8 = warp; each lane holds HD / 32 consecutive elements of the head. A warp keeps an online
 // softmax (running maximum m, sum l, output o) over its keys, four keys' K and V loads in flight;
 // the warps' states are merged in warp order, then the CTAs' states in rank order by rank 0
@@ -327,7 +327,7 @@ int launch(const CUtensorMap& mq, const CUtensorMap& mkv, void* o, int ldo, cons
 // there is no tile for the tensor cores to fill: the step reads K and V once, over enough CTAs to
 // keep many loads in flight.
 constexpr int kDecWarps = 8;
-constexpr int kDecSplit = 4;
+constexpr int kDecSplit = 8;
 
 template <int HD>
 __global__ void __launch_bounds__(kDecWarps * 32)
