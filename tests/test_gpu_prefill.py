@@ -15,6 +15,22 @@ from tests.gpu_util import bf16_np, rowwise_rel
 
 pytestmark = pytest.mark.gpu
 TOL = 2e-2
+# Two runs of the same executor on the same plan: the split-K residual adds (red.add) land in any
+# order, so the fp32 sums differ in the last bits, and where such a sum sits at a bf16 rounding
+# boundary the rounded activation moves by one bf16 unit (2^-8 relative), which moves an output
+# row by at most about 2^-7 of its largest entry. Two units bound it; one wrong plan bit moves some
+# row by far more (each test checks that with the oracle).
+SAME_EXECUTOR = 2.0**-6
+
+
+def wrong_bit_moves(om, xn, cu, mask, h_ref, rng):
+    """The smallest row-relative move of the oracle's output under one flipped plan bit (5 tries)."""
+    moves = []
+    for _ in range(5):
+        m2 = mask.copy()
+        m2[rng.integers(0, m2.shape[0]), rng.integers(0, m2.shape[1])] ^= 1 << rng.integers(0, 2)
+        moves.append(rowwise_rel(od.prefill(om, xn, cu, m2)[0], h_ref))
+    return min(moves)
 
 
 def build(cfg, seed, std=0.05, device="cpu"):
@@ -316,7 +332,7 @@ def test_adaptive_device_plan_small_and_textless_sequences(seed, lens, n_text):
 
 def test_adaptive_plan_with_given_plan_is_the_plain_prefill():
     # the same tokens, the plan the online rule chose, run through spd_prefill: the same result up
-    # to the order of the residual adds (split-K red.add), i.e. to fp32 rounding
+    # to the order of the residual adds (split-K red.add) and the bf16 roundings that order decides
     model, om, x, vis, cu = _adaptive_inputs(33, [48], [16])
     slc = np.full(6, 0.4)
     tgt = np.array([2, 1, 2, 1, 2, 1], np.uint8)
@@ -330,8 +346,10 @@ def test_adaptive_plan_with_given_plan_is_the_plain_prefill():
     plan = od.expand_adaptive_plan(admit.astype(np.int64), target, 6)
     h2, lg2 = run(model, x.cuda(), cu, plan)
     assert (admit >= 0).any()
-    assert rowwise_rel(h1.cpu().numpy(), h2) < 1e-5
-    assert rowwise_rel(lg1.cpu().numpy(), lg2) < 1e-5
+    assert rowwise_rel(h1.cpu().numpy(), h2) < SAME_EXECUTOR
+    assert rowwise_rel(lg1.cpu().numpy(), lg2) < SAME_EXECUTOR
+    h0, _ = od.prefill(om, bf16_np(x), cu, plan)
+    assert wrong_bit_moves(om, bf16_np(x), cu, plan, h0, np.random.default_rng(34)) > 3 * SAME_EXECUTOR
 
 
 # ---- KV cache and decode steps ---------------------------------------------------------------------
@@ -424,4 +442,5 @@ def test_prefill_admit_form_equals_the_expanded_plan():
     h0, lg0 = od.prefill(om, bf16_np(x), cu, mask)
     assert rowwise_rel(h.cpu().numpy(), h0) < TOL and rowwise_rel(lg.cpu().numpy(), lg0) < TOL
     h2, lg2 = run(model, x.cuda(), cu, mask)
-    assert rowwise_rel(h.cpu().numpy(), h2) < 1e-5  # the same executor (residual adds in any order)
+    assert rowwise_rel(h.cpu().numpy(), h2) < SAME_EXECUTOR
+    assert wrong_bit_moves(om, bf16_np(x), cu, mask, h0, r) > 3 * SAME_EXECUTOR
