@@ -82,9 +82,8 @@ def test_tiny_no_skipping_and_null_mask():
     x = inputs(96, 256, 4)
     h1, l1 = check(model, om, x, [0, 96], None)
     h2, l2 = run(model, x.cuda(), [0, 96], np.zeros((2, 96), np.uint8))
-    # same computation. Residual updates of K-split GEMM tiles add in no fixed order; a last-bit
-    # difference in the fp32 residual can flip a bf16 rounding downstream, so runs agree to ~1e-3.
-    assert rowwise_rel(h2, h1) < 5e-3 and rowwise_rel(l2, l1) < 5e-3
+    # the same computation, up to the order of the residual adds (SAME_EXECUTOR)
+    assert rowwise_rel(h2, h1) < SAME_EXECUTOR and rowwise_rel(l2, l1) < SAME_EXECUTOR
 
 
 @pytest.mark.parametrize("seed", [5, 6])
@@ -133,11 +132,11 @@ def test_skip_attn_row_is_still_a_key_and_value():
     x = inputs(T, 256, 15)
     mask = np.zeros((1, T), np.uint8)
     mask[0, j] = 1
-    h1, _ = run(model, x.cuda(), [0, T], mask)
+    h1, _ = check(model, om, x, [0, T], mask)
     x2 = x.clone()
-    x2[j] = (x2[j].float() + torch.randn(256)).to(torch.bfloat16)
-    h2, _ = run(model, x2.cuda(), [0, T], mask)
-    assert rowwise_rel(h1[:j], h2[:j]) < 5e-3            # causal: earlier tokens do not see j
+    x2[j] = (x2[j].float() + torch.randn(256, generator=torch.Generator().manual_seed(16))).to(torch.bfloat16)
+    h2, _ = check(model, om, x2, [0, T], mask)           # the oracle's attention is causal
+    assert rowwise_rel(h1[:j], h2[:j]) < SAME_EXECUTOR   # earlier tokens do not see j
     assert np.abs(h1[j + 1:] - h2[j + 1:]).max() > 1e-3  # later tokens read j's K/V
 
 
