@@ -553,6 +553,8 @@ def main():
                                **({} if L == 32 else {"profiling_only_layers": L})),
                 "dense": {"value": tokens / (ms_dense / 1000.0), "ms_per_step": ms_dense,
                           "decoder_tokens": dense.T, "speedup_spider_vs_dense": ms_dense / ms},
+                "compacted": {"decoder_tokens_per_request": spider.T,
+                              "tokens_per_s": spider.T * world / (ms / 1000.0)},
                 "roofline": roof, "kernels": kernels, "dense_gemm": dense_gemm,
                 "prune_batch": pb, "received_attention": ra, "adaptive_plan": adaptive, "decode": dec,
                 "cpu_baseline": cpu,
