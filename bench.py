@@ -363,8 +363,7 @@ def run_reference(a):
     line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": a.gpus,
             "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": "the CPU oracle on the llava-1.5-7b shape (see cpu_baseline)",
-                       "keep": a.keep},
+            "config": workload_config(a.keep, mask_fn(a.keep + TEXT), a.keep + TEXT),
             "cpu_baseline": {k: sample[k] for k in ("kind", "cores", "sample")} | {"value": val,
                                                                                  "unit": "tokens/s"},
             "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
