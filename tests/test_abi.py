@@ -99,3 +99,13 @@ def test_contract_names_are_the_same_calls(lib):
 def test_plan_accepts_both_sublayers_target(lib):
     mask = N.spd_plan_adaptive(3, np.array([1, -1], np.int16), np.array([3, 1], np.uint8))
     np.testing.assert_array_equal(mask, [[0, 0], [3, 0], [3, 0]])
+
+
+def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
+    # the product path has no CPU fallback: without the built library every call raises
+    monkeypatch.setattr(N, "_lib", None)
+    monkeypatch.setattr(N, "LIB_PATH", str(tmp_path / "libspider.so"))
+    with pytest.raises(RuntimeError, match="is missing"):
+        N.lib()
+    with pytest.raises(RuntimeError, match="is missing"):
+        N.spd_plan_adaptive(2, np.array([0, -1], np.int16), np.array([1, 0], np.uint8))
