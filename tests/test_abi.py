@@ -109,3 +109,27 @@ def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
         N.lib()
     with pytest.raises(RuntimeError, match="is missing"):
         N.spd_plan_adaptive(2, np.array([0, -1], np.int16), np.array([1, 0], np.uint8))
+
+
+def test_plan_expansions_match_oracle_over_random_shapes(lib):
+    # per-token (admission layer, target in 1..3) and per-layer masks, 1..40 layers, 1..300 tokens
+    r = np.random.default_rng(77)
+    for _ in range(60):
+        L, T = int(r.integers(1, 41)), int(r.integers(1, 301))
+        admit = r.integers(-1, L, size=T).astype(np.int16)
+        target = r.integers(1, 4, size=T).astype(np.uint8)
+        np.testing.assert_array_equal(N.spd_plan_adaptive(L, admit, target),
+                                      od.expand_adaptive_plan(admit, target, L))
+        lm = r.integers(0, 4, size=L).astype(np.uint8)
+        sel = (r.random(T) < 0.6).astype(np.uint8)
+        np.testing.assert_array_equal(N.spd_plan_static(lm, sel), od.expand_static_plan(lm, sel))
+
+
+def test_plan_admission_edges(lib):
+    # an admission at or past the last layer never takes effect; a token never admitted may carry
+    # any target; an admitted token's target must name a sub-layer
+    mask = N.spd_plan_adaptive(3, np.array([3, -1, -5, 2], np.int16), np.array([1, 0, 9, 2], np.uint8))
+    np.testing.assert_array_equal(mask, [[0, 0, 0, 0], [0, 0, 0, 0], [0, 0, 0, 2]])
+    with pytest.raises(N.SpiderError) as e:
+        N.spd_plan_adaptive(3, np.array([0], np.int16), np.array([0], np.uint8))
+    assert e.value.code == N.SPD_EINVAL
