@@ -148,13 +148,20 @@ def _check(rc: int):
 
 
 def _p(t):
-    """Device (torch) or host (numpy) pointer, or NULL for None."""
+    """Pointer for an argument: NULL for None, the host address of a numpy array (the wrappers
+    below convert every host argument to one), the device address of a CUDA tensor. A tensor in
+    host memory is refused: its address would reach a kernel as an invalid device pointer."""
     if t is None:
         return None
     if isinstance(t, np.ndarray):
-        assert t.flags["C_CONTIGUOUS"]
+        if not t.flags["C_CONTIGUOUS"]:
+            raise ValueError("host arrays passed to libspider must be C-contiguous")
         return t.ctypes.data
-    assert t.is_contiguous(), "tensors passed to libspider must be contiguous"
+    if not getattr(t, "is_cuda", False):
+        raise TypeError(f"device arguments of libspider must be CUDA tensors, got "
+                        f"{type(t).__name__} on {getattr(t, 'device', 'the host')}")
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to libspider must be contiguous")
     return t.data_ptr()
 
 

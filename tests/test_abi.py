@@ -133,3 +133,10 @@ def test_plan_admission_edges(lib):
     with pytest.raises(N.SpiderError) as e:
         N.spd_plan_adaptive(3, np.array([0], np.int16), np.array([0], np.uint8))
     assert e.value.code == N.SPD_EINVAL
+
+
+def test_host_tensor_for_a_device_argument_is_refused(lib):
+    # refused in the binding, before the library is called: no kernel sees a host address
+    import torch
+    with pytest.raises(TypeError, match="CUDA tensors"):
+        N.spd_workspace_status(torch.zeros(16, dtype=torch.uint8))
