@@ -112,6 +112,7 @@ def workload_config(keep, mask, T):
                          f"adaptive skip plan (Table 9 targets)"),
             "keep": keep, "tokens_per_request": N_PATCH + TEXT, "decoder_tokens": T,
             "skipped_sublayer_fraction": round(skipped, 4),
+            "seed": SEED, "seed_of_rank_r": "seed + r",
             "l2": "inputs larger than L2: 13.5 GB of weights streamed every step (L2 129 MB)"}
 
 
