@@ -315,3 +315,71 @@ def test_adaptive_plan_without_slc_freezes_whole_layers():
         rows = np.flatnonzero(admit == a)
         np.testing.assert_array_equal(h[rows], h_a[rows])
         assert np.all(admit_a[rows] == -1)
+
+
+def _torch_llama_forward(w, cfg, x):
+    """One causal sequence through a LLaMA-style decoder written with torch.nn.functional in fp64:
+    RMSNorm (F.rms_norm), rotate-half RoPE, scaled-dot-product attention with the causal mask and
+    grouped K/V heads repeated per query group, SwiGLU as F.silu(y W_gate^T) * (y W_up^T). Shares
+    nothing with the oracle but the weights."""
+    F = torch.nn.functional
+    H, Hkv, hd, eps, theta = (cfg[k] for k in ("n_heads", "n_kv_heads", "head_dim", "rms_eps",
+                                                "rope_theta"))
+    D = cfg["d_model"]
+    f64 = lambda t: t.to(torch.float64)  # noqa: E731
+    h = torch.as_tensor(x, dtype=torch.float64)
+    T = h.shape[0]
+    inv_freq = theta ** (-torch.arange(0, hd, 2, dtype=torch.float64) / hd)
+    ang = torch.arange(T, dtype=torch.float64)[:, None] * inv_freq[None, :]
+    cos, sin = torch.cat([ang.cos(), ang.cos()], -1), torch.cat([ang.sin(), ang.sin()], -1)
+
+    def rotate_half(t):
+        return torch.cat([-t[..., hd // 2:], t[..., :hd // 2]], -1)
+
+    for lw in w["layers"]:
+        xa = F.rms_norm(h, (D,), weight=f64(lw["attn_norm"]), eps=eps)
+        q = (xa @ f64(lw["wq"]).T).view(T, H, hd).transpose(0, 1)
+        k = (xa @ f64(lw["wk"]).T).view(T, Hkv, hd).transpose(0, 1)
+        v = (xa @ f64(lw["wv"]).T).view(T, Hkv, hd).transpose(0, 1)
+        q, k = q * cos + rotate_half(q) * sin, k * cos + rotate_half(k) * sin
+        k, v = k.repeat_interleave(H // Hkv, dim=0), v.repeat_interleave(H // Hkv, dim=0)
+        o = F.scaled_dot_product_attention(q[None], k[None], v[None], is_causal=True)[0]
+        h = h + o.transpose(0, 1).reshape(T, H * hd) @ f64(lw["wo"]).T
+        y = F.rms_norm(h, (D,), weight=f64(lw["ffn_norm"]), eps=eps)
+        h = h + (F.silu(y @ f64(lw["w_gate"]).T) * (y @ f64(lw["w_up"]).T)) @ f64(lw["w_down"]).T
+    z = F.rms_norm(h[-1:], (D,), weight=f64(w["final_norm"]), eps=eps)
+    return h.numpy(), (z @ f64(w["lm_head"]).T)[0].numpy()
+
+
+@pytest.mark.parametrize("kv_heads", [4, 2])
+def test_prefill_equals_torch_functional_llama(kv_heads):
+    # the oracle's decoder with an empty plan and no bf16 rounding against an independent torch
+    # formulation of the same LLaMA-style layers (MHA and GQA), two packed sequences
+    cfg = dict(n_layers=2, d_model=128, n_heads=4, n_kv_heads=kv_heads, head_dim=32, d_ffn=160,
+               vocab=50, rope_theta=1e4, rms_eps=1e-5, d_vis=0, d_proj=0)
+    w = synth.decoder_weights(17, cfg, std=0.08)
+    om = od.model_from_torch(w, cfg)
+    x = np.random.default_rng(18).standard_normal((11, 128))
+    cu = [0, 7, 11]
+    h, lg = od.prefill(om, x, cu, np.zeros((2, 11), np.uint8), round_fn=od.identity)
+    for b in range(2):
+        h_t, lg_t = _torch_llama_forward(w, cfg, x[cu[b]:cu[b + 1]])
+        np.testing.assert_allclose(h[cu[b]:cu[b + 1]], h_t, rtol=1e-10, atol=1e-10)
+        np.testing.assert_allclose(lg[b], lg_t, rtol=1e-10, atol=1e-10)
+
+
+def test_swiglu_gate_is_the_silu_operand():
+    # swapping W_gate and W_up changes the layer (SiLU is not symmetric in its two factors), so the
+    # comparison above fixes which weight the oracle gates
+    cfg = dict(n_layers=1, d_model=64, n_heads=2, n_kv_heads=2, head_dim=32, d_ffn=96, vocab=10,
+               rope_theta=1e4, rms_eps=1e-5, d_vis=0, d_proj=0)
+    w = synth.decoder_weights(19, cfg, std=0.2)
+    om = od.model_from_torch(w, cfg)
+    sw = od.model_from_torch(w, cfg)
+    sw["layers"][0]["w_gate"], sw["layers"][0]["w_up"] = sw["layers"][0]["w_up"], sw["layers"][0]["w_gate"]
+    x = np.random.default_rng(20).standard_normal((5, 64))
+    h, _ = od.prefill(om, x, [0, 5], np.zeros((1, 5), np.uint8), round_fn=od.identity)
+    hs, _ = od.prefill(sw, x, [0, 5], np.zeros((1, 5), np.uint8), round_fn=od.identity)
+    h_t, _ = _torch_llama_forward(w, cfg, x)
+    np.testing.assert_allclose(h, h_t, rtol=1e-10, atol=1e-10)
+    assert np.abs(hs - h_t).max() > 1e-3
