@@ -29,7 +29,8 @@ EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait"
            "spd_decode",
            "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
            "spd_trace_read", "spd_prune_workspace", "spd_prefill_workspace", "spd_gather_bf16",
-           "spd_last_error_detail", "spd_check", "spd_plan_from_layer_mask", "spd_prefill_admit")
+           "spd_last_error_detail", "spd_check", "spd_plan_from_layer_mask", "spd_prefill_admit",
+           "spd_stamp_enable", "spd_stamp_read")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
 
 
@@ -131,6 +132,9 @@ def lib():
             "spd_linear": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, sz, vp]),
             "spd_linear_noalloc": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, vp]),
             "spd_trace_enable": (i, [i]),
+            "spd_stamp_enable": (i, [i]),
+            "spd_stamp_read": (i, [i, C.POINTER(ll), C.POINTER(C.c_double), C.POINTER(C.c_double),
+                                   C.POINTER(C.c_double)]),
             "spd_trace_read": (i, [i, C.POINTER(ll), C.POINTER(C.c_double), C.POINTER(C.c_double),
                                    C.POINTER(C.c_double)]),
         }
@@ -163,6 +167,43 @@ def _p(t):
     if not t.is_contiguous():
         raise ValueError("tensors passed to libspider must be contiguous")
     return t.data_ptr()
+
+
+_DT = {"f32": "float32", "bf16": "bfloat16", "i32": "int32", "u8": "uint8", "i8": "int8"}
+
+
+def _dev(t, dt, n, name, optional=False):
+    """Device pointer of argument `name` after checking it: a contiguous CUDA tensor of element
+    type dt ('f32', 'bf16', 'i32', 'u8', 'i8') holding at least n elements (the elements the call
+    reads or writes). Raises before the library is called, so no kernel is handed a buffer that is
+    too small, of the wrong type, or in host memory."""
+    if t is None:
+        if optional:
+            return None
+        raise ValueError(f"{name}: a device tensor is required")
+    if isinstance(t, np.ndarray) or not getattr(t, "is_cuda", False):
+        raise TypeError(f"{name}: device arguments of libspider must be CUDA tensors, got "
+                        f"{type(t).__name__} on {getattr(t, 'device', 'the host')}")
+    if str(t.dtype) != "torch." + _DT[dt]:
+        raise ValueError(f"{name}: expected {_DT[dt]}, got {t.dtype}")
+    if t.numel() < n:
+        raise ValueError(f"{name}: {t.numel()} elements, the call touches {int(n)}")
+    return _p(t)
+
+
+def _host(a, dtype, n, name):
+    """C-contiguous host copy of a host array argument with at least n elements."""
+    a = np.ascontiguousarray(a, dtype=dtype)
+    if a.size < n:
+        raise ValueError(f"{name}: {a.size} elements, the call reads {int(n)}")
+    return a
+
+
+def _ws(ws):
+    """Pointer and byte size of a workspace (a CUDA tensor of any element type)."""
+    if ws is None:
+        raise ValueError("ws: a device workspace is required")
+    return _p(ws), ws.numel() * ws.element_size()
 
 
 def _stream(stream):
@@ -202,9 +243,18 @@ def spd_prune_workspace_size(cfg: PruneCfg) -> int:
 
 
 def spd_prune(cfg, feats, attn, keep_idx, kind=None, cluster=None, scores=None, ws=None, stream=None):
-    arr = (C.c_void_p * len(feats))(*[_p(f) for f in feats])
-    _check(lib().spd_prune(C.byref(cfg), arr, _p(attn), _p(keep_idx), _p(kind), _p(cluster),
-                           _p(scores), _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+    T, n_tok, d = cfg.n_tiles, cfg.n_tok, cfg.d_feat
+    n = n_tok - (1 if cfg.has_cls else 0)
+    if len(feats) != cfg.n_layers:
+        raise ValueError(f"feats: {len(feats)} layers, cfg.n_layers = {cfg.n_layers}")
+    arr = (C.c_void_p * len(feats))(*[_dev(f, "f32", T * n_tok * d, f"feats[{i}]")
+                                      for i, f in enumerate(feats)])
+    n_att = n_tok if cfg.attn_form == 0 else n
+    wp, wb = _ws(ws)
+    _check(lib().spd_prune(C.byref(cfg), arr, _dev(attn, "f32", T * cfg.n_heads * n_att, "attn"),
+                           _dev(keep_idx, "i32", T * cfg.keep, "keep_idx"),
+                           _dev(kind, "u8", T * n, "kind", True), _dev(cluster, "i8", T * n, "cluster", True),
+                           _dev(scores, "f32", T * n, "scores", True), wp, wb, _stream(stream)))
 
 
 def spd_received_attention_workspace_size(n_maps: int, n_q: int, n_k: int) -> int:
@@ -216,14 +266,21 @@ def spd_received_attention(maps, out, ws, group_start=None, group_members=None, 
     through a patch merger given as CSR groups)."""
     n_maps, n_q, n_k = maps.shape
     n_out = out.shape[-1]
-    _check(lib().spd_received_attention(_p(maps), n_maps, n_q, n_k, _p(group_start), _p(group_members),
-                                        n_out, _p(out), _p(ws), ws.numel() * ws.element_size(),
+    if (group_start is None) != (group_members is None):
+        raise ValueError("group_start and group_members go together")
+    wp, wb = _ws(ws)
+    _check(lib().spd_received_attention(_dev(maps, "f32", n_maps * n_q * n_k, "maps"), n_maps, n_q, n_k,
+                                        _dev(group_start, "i32", n_out + 1, "group_start", True),
+                                        _dev(group_members, "i32", 1, "group_members", True),
+                                        n_out, _dev(out, "f32", n_maps * n_out, "out"), wp, wb,
                                         _stream(stream)))
 
 
 def spd_gather_rows_bf16(src, n_tiles, n_tok, d, row_offset, idx, keep, dst, ws=None, stream=None):
-    _check(lib().spd_gather_rows_bf16(_p(src), n_tiles, n_tok, d, row_offset, _p(idx), keep, _p(dst),
-                                      _p(ws), _stream(stream)))
+    _check(lib().spd_gather_rows_bf16(_dev(src, "f32", n_tiles * n_tok * d, "src"), n_tiles, n_tok, d,
+                                      row_offset, _dev(idx, "i32", n_tiles * keep, "idx"), keep,
+                                      _dev(dst, "bf16", n_tiles * keep * d, "dst"), _p(ws),
+                                      _stream(stream)))
 
 
 class SpdModel:
@@ -235,12 +292,20 @@ class SpdModel:
                       cfg["head_dim"], cfg["d_ffn"], cfg["vocab"], float(cfg["rope_theta"]),
                       float(cfg["rms_eps"]), cfg.get("d_vis", 0) if cfg.get("d_proj") else 0,
                       cfg.get("d_proj", 0))
+        D, H, Hkv, hd, F = (cfg[k] for k in ("d_model", "n_heads", "n_kv_heads", "head_dim", "d_ffn"))
+        shapes = dict(attn_norm=D, wq=H * hd * D, wk=Hkv * hd * D, wv=Hkv * hd * D, wo=D * H * hd,
+                      ffn_norm=D, w_gate=F * D, w_up=F * D, w_down=D * F)
+        if len(weights["layers"]) != cfg["n_layers"]:
+            raise ValueError(f"weights: {len(weights['layers'])} layers, n_layers = {cfg['n_layers']}")
         layers = (LayerWeights * cfg["n_layers"])()
         for l, lw in enumerate(weights["layers"]):
             for k, _ in LayerWeights._fields_:
-                setattr(layers[l], k, _p(lw[k]))
-        mw = ModelWeights(layers, _p(weights["final_norm"]), _p(weights["lm_head"]),
-                          *[_p(weights.get(k)) for k in ("proj_w1", "proj_b1", "proj_w2", "proj_b2")])
+                setattr(layers[l], k, _dev(lw[k], "bf16", shapes[k], f"layers[{l}].{k}"))
+        dv, dp = mc.d_vis, mc.d_proj
+        proj = [_dev(weights.get(k), "bf16", n, k, optional=not dp)
+                for k, n in (("proj_w1", dp * dv), ("proj_b1", dp), ("proj_w2", D * dp), ("proj_b2", D))]
+        mw = ModelWeights(layers, _dev(weights["final_norm"], "bf16", D, "final_norm"),
+                          _dev(weights["lm_head"], "bf16", cfg["vocab"] * D, "lm_head"), *proj)
         h = C.c_void_p()
         import torch
         torch.cuda.synchronize()
@@ -261,7 +326,7 @@ class SpdModel:
 
 def spd_plan_adaptive(n_layers: int, admit: np.ndarray, target: np.ndarray) -> np.ndarray:
     admit = np.ascontiguousarray(admit, dtype=np.int16)
-    target = np.ascontiguousarray(target, dtype=np.uint8)
+    target = _host(target, np.uint8, len(admit), "target")
     mask = np.zeros((n_layers, len(admit)), dtype=np.uint8)
     _check(lib().spd_plan_adaptive(n_layers, len(admit), _p(admit), _p(target), _p(mask)))
     return mask
@@ -281,8 +346,13 @@ def spd_project_workspace_size(model: SpdModel, rows: int) -> int:
 
 
 def spd_project(model: SpdModel, vis, rows, out_rows, x, ws, stream=None):
-    _check(lib().spd_project(model.handle, _p(vis), rows, _p(out_rows), _p(x), _p(ws),
-                             ws.numel() * ws.element_size(), _stream(stream)))
+    """Projector of `rows` bf16 vision rows into rows out_rows[i] of x (row indices must lie inside
+    x: device values, not read back here)."""
+    D = model.cfg["d_model"]
+    wp, wb = _ws(ws)
+    _check(lib().spd_project(model.handle, _dev(vis, "bf16", rows * model.cfg.get("d_vis", 0), "vis"),
+                             rows, _dev(out_rows, "i32", rows, "out_rows"),
+                             _dev(x, "bf16", min(rows, 1) * D, "x"), wp, wb, _stream(stream)))
 
 
 def spd_attention_workspace_size(n_q: int, n_seqs: int) -> int:
@@ -293,14 +363,23 @@ def spd_attention(q, q_pos, q_cu, kv, cu_seqlens, n_heads, n_kv_heads, head_dim,
     """Causal attention of the query rows q (positions q_pos, sequences delimited by the host
     array q_cu) over the K/V rows kv of their sequences (host cu_seqlens); writes o."""
     q_cu = np.ascontiguousarray(q_cu, dtype=np.int32)
-    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
-    _check(lib().spd_attention(_p(q), int(q_cu[-1]), _p(q_pos), _p(q_cu), _p(kv), int(cu[-1]), _p(cu),
-                               len(cu) - 1, n_heads, n_kv_heads, head_dim, _p(o), _p(ws),
-                               ws.numel() * ws.element_size(), _stream(stream)))
+    cu = _host(cu_seqlens, np.int32, len(q_cu), "cu_seqlens")
+    n_q, n_kv = int(q_cu[-1]), int(cu[-1])
+    qd, kvd = n_heads * head_dim, n_kv_heads * head_dim
+    wp, wb = _ws(ws)
+    _check(lib().spd_attention(_dev(q, "bf16", n_q * qd, "q"), n_q, _dev(q_pos, "i32", n_q, "q_pos"),
+                               _p(q_cu), _dev(kv, "bf16", n_kv * 2 * kvd, "kv"), n_kv, _p(cu),
+                               len(q_cu) - 1, n_heads, n_kv_heads, head_dim,
+                               _dev(o, "bf16", n_q * qd, "o"), wp, wb, _stream(stream)))
 
 
 def spd_scatter_rows(model: SpdModel, src, rows, rows_map, dst, stream=None):
-    _check(lib().spd_scatter_rows(model.handle, _p(src), rows, _p(rows_map), _p(dst), _stream(stream)))
+    """dst[rows_map[i]] = src[i] for `rows` bf16 rows of d_model (row indices must lie inside dst:
+    device values, not read back here)."""
+    D = model.cfg["d_model"]
+    _check(lib().spd_scatter_rows(model.handle, _dev(src, "bf16", rows * D, "src"), rows,
+                                  _dev(rows_map, "i32", rows, "rows_map"),
+                                  _dev(dst, "bf16", min(rows, 1) * D, "dst"), _stream(stream)))
 
 
 def spd_prefill_workspace_size(model: SpdModel, max_tokens: int, max_seqs: int) -> int:
@@ -317,15 +396,19 @@ def spd_prefill_adaptive(model: SpdModel, x, n_tokens, cu_seqlens, is_visual, sl
     int16, -1 = never). ablate: bit set of SPD_SKIP_NO_*; device_plan: decisions and row lists on
     the device (1) or read back per window layer (0)."""
     cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
-    slc = np.ascontiguousarray(slc_norm, dtype=np.float32)
-    tgt = np.ascontiguousarray(layer_target, dtype=np.uint8)
-    vis = np.ascontiguousarray(is_visual, dtype=np.uint8)
+    L, D, B = model.cfg["n_layers"], model.cfg["d_model"], len(cu) - 1
+    slc = _host(slc_norm, np.float32, L, "slc_norm")
+    tgt = _host(layer_target, np.uint8, L, "layer_target")
+    vis = _host(is_visual, np.uint8, n_tokens, "is_visual")
     admit = np.full(n_tokens, -9, dtype=np.int16)
     pol = SkipPolicy(float(t_skip), float(w1), float(w2), int(window), slc.ctypes.data, tgt.ctypes.data,
                      vis.ctypes.data, int(ablate), int(device_plan))
-    _check(lib().spd_prefill_adaptive(model.handle, _p(x), n_tokens, cu.ctypes.data, len(cu) - 1,
-                                      C.byref(pol), admit.ctypes.data, _p(h), _p(logits), _p(ws),
-                                      ws.numel() * ws.element_size(), _stream(stream)))
+    wp, wb = _ws(ws)
+    _check(lib().spd_prefill_adaptive(model.handle, _dev(x, "bf16", n_tokens * D, "x"), n_tokens,
+                                      cu.ctypes.data, B, C.byref(pol), admit.ctypes.data,
+                                      _dev(h, "f32", n_tokens * D, "h"),
+                                      _dev(logits, "f32", B * model.cfg["vocab"], "logits", True), wp, wb,
+                                      _stream(stream)))
     return admit
 
 
@@ -336,10 +419,14 @@ def spd_kv_cache_bytes(model: SpdModel, n_seqs: int, max_len: int) -> int:
 def spd_prefill_kv(model: SpdModel, x, n_tokens, cu_seqlens, skip_mask, h, logits, kv_cache, max_len, ws,
                    stream=None):
     cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
-    mk = None if skip_mask is None else np.ascontiguousarray(skip_mask, dtype=np.uint8)
-    _check(lib().spd_prefill_kv(model.handle, _p(x), n_tokens, cu.ctypes.data, len(cu) - 1,
-                                None if mk is None else mk.ctypes.data, _p(h), _p(logits), _p(kv_cache),
-                                max_len, _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+    L, D, B = model.cfg["n_layers"], model.cfg["d_model"], len(cu) - 1
+    mk = None if skip_mask is None else _host(skip_mask, np.uint8, L * n_tokens, "skip_mask")
+    wp, wb = _ws(ws)
+    _check(lib().spd_prefill_kv(model.handle, _dev(x, "bf16", n_tokens * D, "x"), n_tokens, cu.ctypes.data,
+                                B, None if mk is None else mk.ctypes.data, _dev(h, "f32", n_tokens * D, "h"),
+                                _dev(logits, "f32", B * model.cfg["vocab"], "logits", True),
+                                _dev(kv_cache, "bf16", spd_kv_cache_bytes(model, B, max_len) // 2, "kv_cache"),
+                                max_len, wp, wb, _stream(stream)))
 
 
 def spd_decode_workspace_size(model: SpdModel, n_seqs: int) -> int:
@@ -348,25 +435,36 @@ def spd_decode_workspace_size(model: SpdModel, n_seqs: int) -> int:
 
 def spd_decode(model: SpdModel, x, pos, kv_cache, max_len, logits, ws, stream=None):
     p = np.ascontiguousarray(pos, dtype=np.int32)
-    _check(lib().spd_decode(model.handle, _p(x), len(p), p.ctypes.data, _p(kv_cache), max_len,
-                            _p(logits), _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+    B, D = len(p), model.cfg["d_model"]
+    wp, wb = _ws(ws)
+    _check(lib().spd_decode(model.handle, _dev(x, "bf16", B * D, "x"), B, p.ctypes.data,
+                            _dev(kv_cache, "bf16", spd_kv_cache_bytes(model, B, max_len) // 2, "kv_cache"),
+                            max_len, _dev(logits, "f32", B * model.cfg["vocab"], "logits"), wp, wb,
+                            _stream(stream)))
 
 
 def spd_prefill(model: SpdModel, x, n_tokens, cu_seqlens, skip_mask, h, logits, ws, stream=None):
     cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
-    mask = None if skip_mask is None else np.ascontiguousarray(skip_mask, dtype=np.uint8)
-    _check(lib().spd_prefill(model.handle, _p(x), n_tokens, _p(cu), len(cu) - 1, _p(mask), _p(h),
-                             _p(logits), _p(ws), ws.numel() * ws.element_size(), _stream(stream)))
+    L, D, B = model.cfg["n_layers"], model.cfg["d_model"], len(cu) - 1
+    mask = None if skip_mask is None else _host(skip_mask, np.uint8, L * n_tokens, "skip_mask")
+    wp, wb = _ws(ws)
+    _check(lib().spd_prefill(model.handle, _dev(x, "bf16", n_tokens * D, "x"), n_tokens, _p(cu), B,
+                             _p(mask), _dev(h, "f32", n_tokens * D, "h"),
+                             _dev(logits, "f32", B * model.cfg["vocab"], "logits", True), wp, wb,
+                             _stream(stream)))
 
 
 def spd_prefill_admit(model: SpdModel, x, n_tokens, cu_seqlens, admit_layer, target, h, logits, ws,
                       stream=None):
     """spd_prefill with the per-token plan (admission layer, frozen target), expanded on the host."""
     cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
-    ad = None if admit_layer is None else np.ascontiguousarray(admit_layer, dtype=np.int16)
-    tg = None if target is None else np.ascontiguousarray(target, dtype=np.uint8)
-    _check(lib().spd_prefill_admit(model.handle, _p(x), n_tokens, _p(cu), len(cu) - 1, _p(ad), _p(tg),
-                                   _p(h), _p(logits), _p(ws), ws.numel() * ws.element_size(),
+    D, B = model.cfg["d_model"], len(cu) - 1
+    ad = None if admit_layer is None else _host(admit_layer, np.int16, n_tokens, "admit_layer")
+    tg = None if target is None else _host(target, np.uint8, n_tokens, "target")
+    wp, wb = _ws(ws)
+    _check(lib().spd_prefill_admit(model.handle, _dev(x, "bf16", n_tokens * D, "x"), n_tokens, _p(cu), B,
+                                   _p(ad), _p(tg), _dev(h, "f32", n_tokens * D, "h"),
+                                   _dev(logits, "f32", B * model.cfg["vocab"], "logits", True), wp, wb,
                                    _stream(stream)))
 
 
@@ -385,16 +483,28 @@ def spd_linear_workspace_size(M: int, N: int) -> int:
     return int(lib().spd_linear_workspace_size(M, N))
 
 
+def _linear_args(X, M, K, W, N, epilogue, out, ldo, bias, rows):
+    """Checked pointers of a linear call: out holds M rows of ldo (or, with a row map, at least one
+    row: the map's device values must lie inside out and are not read back here)."""
+    out_dt = "f32" if epilogue in (EPI_F32, EPI_ADD_F32) else "bf16"
+    out_n = (ldo if rows is not None else M * ldo) if M > 0 else 0
+    return (_dev(X, "bf16", M * K, "X"), _dev(W, "bf16", N * K, "W"),
+            _dev(bias, "bf16", N, "bias", True), _dev(rows, "i32", M, "rows", True),
+            _dev(out, out_dt, out_n, "out"))
+
+
 def spd_linear(X, M, K, W, N, epilogue, out, ldo, ws, bias=None, rows=None, stream=None):
-    _check(lib().spd_linear(_p(X), M, K, _p(W), N, epilogue, _p(bias), _p(rows), _p(out), ldo, _p(ws),
-                            ws.numel() * ws.element_size(), _stream(stream)))
+    x, w, b, r, o = _linear_args(X, M, K, W, N, epilogue, out, ldo, bias, rows)
+    wp, wb = _ws(ws)
+    _check(lib().spd_linear(x, M, K, w, N, epilogue, b, r, o, ldo, wp, wb, _stream(stream)))
 
 
 def spd_linear_noalloc(X, M, K, W, N, epilogue, out, ldo, bias=None, rows=None, status=None,
                        stream=None):
     """spd_linear with the library's own static scratch instead of a caller workspace."""
-    _check(lib().spd_linear_noalloc(_p(X), M, K, _p(W), N, epilogue, _p(bias), _p(rows), _p(out),
-                                    ldo, _p(status), _stream(stream)))
+    x, w, b, r, o = _linear_args(X, M, K, W, N, epilogue, out, ldo, bias, rows)
+    _check(lib().spd_linear_noalloc(x, M, K, w, N, epilogue, b, r, o, ldo,
+                                    _dev(status, "i32", 1, "status", True), _stream(stream)))
 
 
 def spd_trace_enable(capacity: int):
@@ -405,4 +515,16 @@ def spd_trace_read(cls: int) -> dict:
     """Launch count, device ms, algorithmic flops and bytes of one kernel class (synchronises)."""
     n, ms, fl, by = C.c_longlong(), C.c_double(), C.c_double(), C.c_double()
     _check(lib().spd_trace_read(cls, C.byref(n), C.byref(ms), C.byref(fl), C.byref(by)))
+    return dict(launches=n.value, ms=ms.value, flops=fl.value, bytes=by.value)
+
+
+def spd_stamp_enable(capacity: int):
+    _check(lib().spd_stamp_enable(int(capacity)))
+
+
+def spd_stamp_read(cls: int) -> dict:
+    """Launch count, stamped device ms, algorithmic flops and bytes of one kernel class (device
+    globaltimer stamps; synchronises)."""
+    n, ms, fl, by = C.c_longlong(), C.c_double(), C.c_double(), C.c_double()
+    _check(lib().spd_stamp_read(cls, C.byref(n), C.byref(ms), C.byref(fl), C.byref(by)))
     return dict(launches=n.value, ms=ms.value, flops=fl.value, bytes=by.value)

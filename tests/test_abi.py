@@ -140,3 +140,80 @@ def test_host_tensor_for_a_device_argument_is_refused(lib):
     import torch
     with pytest.raises(TypeError, match="CUDA tensors"):
         N.spd_workspace_status(torch.zeros(16, dtype=torch.uint8))
+
+
+class _FakeCuda:
+    """Stands in for a CUDA tensor in the binding's argument checks (no GPU here): the checks must
+    refuse it before the library is called, so its pointer is never used."""
+
+    def __init__(self, dtype, numel):
+        import torch
+        self.dtype = getattr(torch, dtype)
+        self.is_cuda = True
+        self._n = numel
+
+    def numel(self):
+        return self._n
+
+    def element_size(self):
+        return 1
+
+    def is_contiguous(self):
+        return True
+
+    def data_ptr(self):
+        return 0
+
+
+def test_binding_refuses_undersized_or_mistyped_device_arguments(lib):
+    M, K, Nw = 64, 256, 128
+    ok = dict(X=_FakeCuda("bfloat16", M * K), W=_FakeCuda("bfloat16", Nw * K),
+              out=_FakeCuda("float32", M * Nw))
+    bad = [dict(X=_FakeCuda("bfloat16", M * K - 1)),            # X one element short
+           dict(W=_FakeCuda("float32", Nw * K)),                 # fp32 weights where bf16 is read
+           dict(out=_FakeCuda("float32", M * Nw - 8)),           # output rows past the end
+           dict(out=_FakeCuda("bfloat16", M * Nw)),              # bf16 output for an fp32 epilogue
+           dict(X=np.zeros((M, K), np.float32))]                 # a host array for a device pointer
+    for b in bad:
+        a = dict(ok, **b)
+        with pytest.raises((ValueError, TypeError)):
+            N.spd_linear(a["X"], M, K, a["W"], Nw, N.EPI_F32, a["out"], Nw, _FakeCuda("uint8", 1 << 30))
+        with pytest.raises((ValueError, TypeError)):
+            N.spd_linear_noalloc(a["X"], M, K, a["W"], Nw, N.EPI_F32, a["out"], Nw)
+    with pytest.raises(ValueError):  # a residual status word of the wrong type
+        N.spd_linear_noalloc(ok["X"], M, K, ok["W"], Nw, N.EPI_F32, ok["out"], Nw,
+                             status=_FakeCuda("float32", 1))
+
+
+def test_binding_refuses_short_host_arrays_and_buffers_of_prune_and_gather(lib):
+    cfg = N.prune_cfg(2, 577, 64, 2, 1, 4, 32)
+    feats = [_FakeCuda("float32", 2 * 577 * 64)] * 2
+    attn = _FakeCuda("float32", 2 * 4 * 577)
+    idx = _FakeCuda("int32", 2 * 32)
+    ws = _FakeCuda("uint8", 1 << 20)
+    for kw in (dict(feats=[feats[0]]),                                  # one layer missing
+               dict(attn=_FakeCuda("float32", 2 * 4 * 576)),            # the CLS rows are 577 wide
+               dict(idx=_FakeCuda("int32", 63)),
+               dict(kind=_FakeCuda("uint8", 2 * 576 - 1))):
+        a = dict(feats=feats, attn=attn, idx=idx, kind=None) | kw
+        with pytest.raises(ValueError):
+            N.spd_prune(cfg, a["feats"], a["attn"], a["idx"], kind=a["kind"], ws=ws)
+    with pytest.raises(ValueError):
+        N.spd_gather_rows_bf16(feats[0], 2, 577, 64, 1, idx, 32, _FakeCuda("bfloat16", 2 * 32 * 64 - 1))
+
+
+def test_binding_refuses_short_plans_and_residual_buffers(lib):
+    class M:  # a model handle is never reached: the checks come first
+        cfg = dict(n_layers=3, d_model=64, vocab=10)
+        handle = None
+    T = 20
+    x, h = _FakeCuda("bfloat16", T * 64), _FakeCuda("float32", T * 64)
+    ws = _FakeCuda("uint8", 1 << 20)
+    with pytest.raises(ValueError):  # skip mask of 2 layers for a 3-layer model
+        N.spd_prefill(M, x, T, [0, T], np.zeros((2, T), np.uint8), h, None, ws)
+    with pytest.raises(ValueError):  # residual stream one row short
+        N.spd_prefill(M, x, T, [0, T], None, _FakeCuda("float32", (T - 1) * 64), None, ws)
+    with pytest.raises(ValueError):  # logits of one sequence for two
+        N.spd_prefill(M, x, T, [0, 5, T], None, h, _FakeCuda("float32", 10), ws)
+    with pytest.raises(ValueError):  # per-token plan shorter than the tokens
+        N.spd_prefill_admit(M, x, T, [0, T], np.zeros(T - 1, np.int16), np.ones(T, np.uint8), h, None, ws)
