@@ -68,6 +68,24 @@ int spd_selftest_bounded_wait(void* ws, long long budget_cycles, void* stream);
 int spd_trace_enable(int capacity);
 int spd_trace_read(int cls, long long* launches, double* ms, double* flops, double* bytes);
 
+/* Launch stamps (measurement support, no counterpart in the paper): spd_stamp_enable(n) starts
+ * stamping up to n launches of the GEMM, attention and RMSNorm kernels without adding any stream
+ * operation between launches: each stamped kernel records, in device memory, the globaltimer time
+ * of its first CTA past the grid dependency wait and of its last CTA's end. n <= 0 stops. The
+ * intervals of successive kernels of a stream do not overlap (a kernel passes its wait only after
+ * its predecessor completed), so a class's summed time never exceeds the wall time of the work.
+ * spd_stamp_read synchronises the device and returns for one class (SPD_TRACE_*) the launch count,
+ * summed milliseconds and summed algorithmic flops and bytes, as spd_trace_read. Not thread-safe
+ * with respect to concurrent library calls from other threads (the slots are taken in call
+ * order). Errors: SPD_ECUDA. */
+int spd_stamp_enable(int capacity);
+int spd_stamp_read(int cls, long long* launches, double* ms, double* flops, double* bytes);
+/* Stamp k (0-based, in launch order since spd_stamp_enable): class, start and end (globaltimer ns;
+ * end < start when the launch did not run), algorithmic flops and bytes. Synchronises the device.
+ * Errors: SPD_EINVAL when fewer than k + 1 launches were stamped; SPD_ECUDA. */
+int spd_stamp_launch(int k, int* cls, unsigned long long* start_ns, unsigned long long* end_ns,
+                     double* flops, double* bytes);
+
 /* ------------------------------------------------------------------------------------------ */
 /* Stage 1: MSV-Prune (Sec. 4.1)                                                                */
 /* ------------------------------------------------------------------------------------------ */
@@ -371,7 +389,7 @@ int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, int N, int ep
 
 /* Capacity of the scratch that spd_linear_noalloc keeps inside the library. */
 #define SPD_LINEAR_NOALLOC_SCRATCH_BYTES (8u << 20) /* 8 MiB of device memory */
-#define SPD_LINEAR_NOALLOC_MAX_TILES 4096           /* output tiles: ceil(N / 128) x ceil(M / 256) */
+#define SPD_LINEAR_NOALLOC_MAX_TILES 4096           /* tile counters: 2 ceil(N / 256) x ceil(M / 256) */
 
 /* spd_linear without a workspace argument. The paper has no counterpart: this is a convenience of
  * the library, for callers that have no device buffer to lend at the point of the call and must
@@ -386,9 +404,12 @@ int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, int N, int ep
  * The first call on a device (the device current at the call) looks up the scratch's address on
  * that device (cudaGetSymbolAddress) and caches it; make that first call before any stream capture.
  * status (dev, may be NULL): int32 receiving this call's device-side status (0 = OK, else an
- * spd_status, e.g. SPD_ETIMEOUT) once the work completes.
- * Errors: SPD_EINVAL; SPD_ENOSPC when the output has more than SPD_LINEAR_NOALLOC_MAX_TILES tiles
- * (detected on the host, nothing is launched); SPD_ECUDA. */
+ * spd_status, e.g. SPD_ETIMEOUT) once the work completes. With NULL a device-side failure of the
+ * call is not reported anywhere: the scratch's own status word is cleared by the next call and no
+ * entry point reads it.
+ * Errors: SPD_EINVAL; SPD_ENOSPC when the problem needs more than SPD_LINEAR_NOALLOC_MAX_TILES tile
+ * counters, counted as 2 ceil(N / 256) x ceil(M / 256) (the most any tiling of the GEMM uses;
+ * detected on the host before anything is enqueued); SPD_ECUDA. */
 int spd_linear_noalloc(const uint16_t* X, int M, int K, const uint16_t* W, int N, int epilogue,
                        const uint16_t* bias, const int32_t* rows, void* out, int ldo, int* status,
                        void* stream);

@@ -30,7 +30,7 @@ EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait"
            "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
            "spd_trace_read", "spd_prune_workspace", "spd_prefill_workspace", "spd_gather_bf16",
            "spd_last_error_detail", "spd_check", "spd_plan_from_layer_mask", "spd_prefill_admit",
-           "spd_stamp_enable", "spd_stamp_read")
+           "spd_stamp_enable", "spd_stamp_read", "spd_stamp_launch")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
 
 
@@ -133,6 +133,8 @@ def lib():
             "spd_linear_noalloc": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, vp]),
             "spd_trace_enable": (i, [i]),
             "spd_stamp_enable": (i, [i]),
+            "spd_stamp_launch": (i, [i, C.POINTER(i), C.POINTER(C.c_ulonglong), C.POINTER(C.c_ulonglong),
+                                     C.POINTER(C.c_double), C.POINTER(C.c_double)]),
             "spd_stamp_read": (i, [i, C.POINTER(ll), C.POINTER(C.c_double), C.POINTER(C.c_double),
                                    C.POINTER(C.c_double)]),
             "spd_trace_read": (i, [i, C.POINTER(ll), C.POINTER(C.c_double), C.POINTER(C.c_double),
@@ -528,3 +530,16 @@ def spd_stamp_read(cls: int) -> dict:
     n, ms, fl, by = C.c_longlong(), C.c_double(), C.c_double(), C.c_double()
     _check(lib().spd_stamp_read(cls, C.byref(n), C.byref(ms), C.byref(fl), C.byref(by)))
     return dict(launches=n.value, ms=ms.value, flops=fl.value, bytes=by.value)
+
+
+def spd_stamp_launches() -> list:
+    """Every stamped launch since spd_stamp_enable, in launch order: (class, start ns, end ns,
+    flops, bytes)."""
+    out = []
+    k = 0
+    cls, s0, s1 = C.c_int(), C.c_ulonglong(), C.c_ulonglong()
+    fl, by = C.c_double(), C.c_double()
+    while lib().spd_stamp_launch(k, C.byref(cls), C.byref(s0), C.byref(s1), C.byref(fl), C.byref(by)) == SPD_OK:
+        out.append((cls.value, s0.value, s1.value, fl.value, by.value))
+        k += 1
+    return out

@@ -15,7 +15,6 @@
 #include "ptx.cuh"
 
 namespace spd {
-thread_local int g_no_overlap = 0;
 
 int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float eps,
                 const int32_t* in_rows, void* out, const int32_t* map2, void* out2,
@@ -374,9 +373,11 @@ extern "C" int spd_linear_noalloc(const uint16_t* X, int M, int K, const uint16_
   if (epilogue < SPD_EPI_F32 || epilogue > SPD_EPI_ADD_F32) return fail(SPD_EINVAL, "bad epilogue");
   if ((epilogue == SPD_EPI_BIAS_BF16 || epilogue == SPD_EPI_BIAS_GELU_BF16) && !bias)
     return fail(SPD_EINVAL, "epilogue needs a bias");
-  const long long tiles = (long long)((N + 127) / 128) * ((M + 255) / 256);
+  // tile counters of the worst tiling gemm_run may choose: CTA pairs count each 128-row half of a
+  // 256-row tile (2 ceil(N / 256) >= ceil(N / 128) per token tile of 256)
+  const long long tiles = 2LL * ((N + 255) / 256) * ((M + 255) / 256);
   if (tiles > SPD_LINEAR_NOALLOC_MAX_TILES)
-    return fail(SPD_ENOSPC, "spd_linear_noalloc: %lld output tiles exceed the static scratch (%d)",
+    return fail(SPD_ENOSPC, "spd_linear_noalloc: %lld tile counters exceed the static scratch (%d)",
                 tiles, SPD_LINEAR_NOALLOC_MAX_TILES);
   void* base = nullptr;
   if (int rc = linear_scratch(&base)) return rc;
@@ -652,8 +653,7 @@ struct KVDest {
 
 // Decoder layer l on the residual stream h with its lists at dl (device copy of the plan).
 int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P, const PrefillBufs& bf,
-              const int32_t* dl, float* h, int T, cudaStream_t st, const KVDest* kvd_dest = nullptr,
-              bool dev_lists = false) {
+              const int32_t* dl, float* h, int T, cudaStream_t st, const KVDest* kvd_dest = nullptr) {
   const spd_model_cfg& c = m->cfg;
   const int D = c.d_model, hd = c.head_dim;
   const int qd = c.n_heads * hd, kvd = c.n_kv_heads * hd;
@@ -719,7 +719,7 @@ int run_layer(const spd_model* m, int l, const LayerLists& q, const HostPlan& P,
     else
       rc = attention_run(bf.q, q.na, dest.kv, dest.n_rows, 2 * kvd, kvd, bf.o, qd,
                          reinterpret_cast<const int4*>(dl + q.tiles), q.ntiles, dl + q.apos,
-                         c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx, dev_lists);
+                         c.n_heads, c.n_kv_heads, hd, bf.gs.status, st, q.ctx);
     if (rc) return rc;
     GemmProblem op{};
     op.map_w = &W.m_o;
@@ -926,10 +926,6 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
   };
 
   if (pol->device_plan) {
-    // plain stream order inside the decision window: the list builder's outputs feed kernels
-    // several launches later, and with programmatic overlap of the launches in between those
-    // kernels read wrong results in repeated runs (found by testing; plain order measured exact)
-    auto plain_order = std::make_unique<NoOverlap>();
     // Decisions and row lists on the device: every window layer scores every visual token (those
     // already in skip mode are passed over), admits on the device, and a kernel rebuilds the row
     // lists; the sub-layers then run over all T rows with the lists' padding rows skipped. No
@@ -946,10 +942,8 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
     SPD_CUDA_TRY(cudaMemcpyAsync(ab.kvlen, kvl.data(), B * sizeof(int32_t), cudaMemcpyHostToDevice, st));
     SPD_CUDA_TRY(cudaMemsetAsync(ab.admit, 0xff, T * sizeof(int32_t), st));  // -1: never
     SPD_CUDA_TRY(cudaMemsetAsync(ab.target, 0, T, st));
-    // Each decision layer writes its own list block (written once per call, never while a kernel
-    // that read it may still be resident: a rewritten block could be read through another
-    // kernel's stale cache lines under programmatic overlap); the layers past the window reuse the
-    // last decision layer's block.
+    // Each decision layer writes its own list block; the layers past the window reuse the last
+    // decision layer's block.
     int max_tiles = 0;
     for (int b = 0; b < B; ++b) max_tiles += (cu[b + 1] - cu[b] + kAttnTileQ - 1) / kAttnTileQ;
     double ctx_all = 0.0;
@@ -962,7 +956,6 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
       LD.ntiles = max_tiles;
       LD.ctx = ctx_all;
       if (l < pol->window && nv > 0) {
-        if (int rc = stream_barrier(st)) return rc;
         if (mode & kSkipEntropy)
           if (int rc = lens(ab.cand, nv)) return rc;
         const float add_slc = no_slc ? 0.0f : pol->w2 * pol->slc_norm[l];
@@ -977,8 +970,7 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
                                     ab.kvlen, dl + LD.arows, dl + LD.amap, dl + LD.apos, dl + LD.frows,
                                     reinterpret_cast<int4*>(dl + LD.tiles), max_tiles, st))
           return rc;
-      if (int rc = run_layer(m, l, LD, P, bf, dl, h, T, st, nullptr, true)) return rc;
-      if (l == last_block) plain_order.reset();
+      if (int rc = run_layer(m, l, LD, P, bf, dl, h, T, st)) return rc;
     }
     std::vector<int32_t> ad(T);
     SPD_CUDA_TRY(cudaMemcpyAsync(ad.data(), ab.admit, T * sizeof(int32_t), cudaMemcpyDeviceToHost, st));

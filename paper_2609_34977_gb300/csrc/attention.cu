@@ -51,9 +51,9 @@ template <int HD>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                    const __grid_constant__ CUtensorMap map_kv, __nv_bfloat16* __restrict__ o,
-                   int ldo, const int4* __restrict__ tiles, const int32_t* __restrict__ q_pos,
-                   int n_heads, int n_kv_heads, int v_off, float scale_log2, int* status,
-                   long long budget, int lists_late) {
+                   int ldo, const int4* tiles, const int32_t* q_pos, int n_heads, int n_kv_heads,
+                   int v_off, float scale_log2, int* status, long long budget,
+                   unsigned long long* stamp) {
   using L = AttnSmem<HD>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -98,22 +98,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   const uint32_t t_s = tmem, t_o = tmem + 128;
 
-  // host-copied tile lists and positions were written before the stream's previous kernels ran, so
-  // they are read before the wait; lists built by a kernel (lists_late) only after it. Q, K and V
-  // come from the previous kernel.
-  if (lists_late) {
-    pdl_launch_dependents();
-    pdl_wait();
-  }
+  // Nothing written by an earlier kernel of the stream is read before the grid dependency wait:
+  // under programmatic overlap this kernel's prologue may run while several earlier kernels are
+  // still resident, so the tile list and the positions (copied or built by a kernel) are read
+  // after it, with coherent loads. Q, K and V come from the previous kernels too.
+  pdl_launch_dependents();
+  pdl_wait();
+  if (threadIdx.x == 0) stamp_start(stamp);
   const int4 tl = tiles[blockIdx.x];
   const int q0 = tl.x, nq = tl.y, kv0 = tl.z, len = tl.w;
   const int p_last = q_pos[q0 + nq - 1];  // positions ascend within a tile
   const int nkb = max(1, min((p_last + kTK) / kTK, (len + kTK - 1) / kTK));
   const int my_pos = threadIdx.x < 128 ? q_pos[q0 + min(int(threadIdx.x), nq - 1)] : 0;
-  if (!lists_late) {
-    pdl_launch_dependents();
-    pdl_wait();
-  }
 
   int issued = 0;  // K/V blocks whose loads the producer issued
   if (warp == 4) {
@@ -296,12 +292,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncwarp();
   tc_fence_after();
   if (warp == 4) tmem_dealloc(tmem, 256);
+  if (threadIdx.x == 0) stamp_end(stamp);
 }
 
 template <int HD>
 int launch(const CUtensorMap& mq, const CUtensorMap& mkv, void* o, int ldo, const int4* tiles,
            int n_tiles, const int32_t* q_pos, int n_heads, int n_kv_heads, int v_off, int* status,
-           cudaStream_t stream, int lists_late) {
+           cudaStream_t stream, unsigned long long* stamp) {
   using L = AttnSmem<HD>;
   static bool attr = false;
   if (!attr) {
@@ -312,7 +309,7 @@ int launch(const CUtensorMap& mq, const CUtensorMap& mkv, void* o, int ldo, cons
   const float scale_log2 = 1.4426950408889634f / sqrtf(float(HD));
   SPD_CUDA_TRY(launch_pdl(attn_tc_kernel<HD>, dim3(n_tiles, n_heads), dim3(kThreads), L::bytes,
                           stream, mq, mkv, static_cast<__nv_bfloat16*>(o), ldo, tiles, q_pos,
-                          n_heads, n_kv_heads, v_off, scale_log2, status, kWaitBudget, lists_late));
+                          n_heads, n_kv_heads, v_off, scale_log2, status, kWaitBudget, stamp));
   return SPD_OK;
 }
 
@@ -331,9 +328,9 @@ constexpr int kDecSplit = 8;
 
 template <int HD>
 __global__ void __launch_bounds__(kDecWarps * 32)
-    attn_decode_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ kv,
-                       int ldkv, int v_off, __nv_bfloat16* __restrict__ o, int ldo,
-                       const int4* __restrict__ tiles, int n_heads, int n_kv_heads, float scale_log2) {
+    attn_decode_kernel(const __nv_bfloat16* q, const __nv_bfloat16* kv, int ldkv, int v_off,
+                       __nv_bfloat16* __restrict__ o, int ldo, const int4* tiles, int n_heads,
+                       int n_kv_heads, float scale_log2, unsigned long long* stamp) {
   constexpr int E = HD / 32;  // elements per lane: 2 or 4
   __shared__ float wm[kDecWarps], wl[kDecWarps];
   __shared__ float wo[kDecWarps][HD];
@@ -342,6 +339,7 @@ __global__ void __launch_bounds__(kDecWarps * 32)
   const int rank = int(cluster.block_rank());
   pdl_launch_dependents();
   pdl_wait();
+  if (threadIdx.x == 0) stamp_start(stamp);
   const int head = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int4 tl = tiles[blockIdx.x];  // (query row, query count = 1, first key row, key count)
   const int j_lo = rank * tl.w / kDecSplit, j_hi = (rank + 1) * tl.w / kDecSplit;
@@ -443,14 +441,14 @@ __global__ void __launch_bounds__(kDecWarps * 32)
     o[size_t(tl.x) * ldo + head * HD + threadIdx.x] = __float2bfloat16_rn(ot / lt);
   }
   cluster.sync();  // the peers' shared memory stays alive until rank 0 has read it
+  if (threadIdx.x == 0) stamp_end(stamp);
 }
 
 }  // namespace
 
 int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, int v_off, void* o,
                   int ldo, const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads,
-                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum,
-                  bool lists_from_device) {
+                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum) {
   if (n_tiles <= 0) return SPD_OK;
   if (head_dim != 128 && head_dim != 64)
     return fail(SPD_EUNSUPPORTED, "attention supports head_dim 64 and 128");
@@ -461,15 +459,17 @@ int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, in
   CUtensorMap mq, mkv;
   if (int rc = make_operand_map(&mq, q, n_heads * head_dim, n_q, 128)) return rc;
   if (int rc = make_operand_map(&mkv, kv, ldkv, n_kv, kTK)) return rc;
+  // QK^T and PV over each active query's causal context; Q, K, V read once and O written once
+  const double fl = 4.0 * head_dim * n_heads * ctx_sum;
+  const double by = 2.0 * (2.0 * n_q * n_heads * head_dim + 2.0 * n_kv * n_kv_heads * head_dim);
+  unsigned long long* stamp = stamp_slot(TR_ATTN, fl, by);
   const int slot = trace_begin(stream);
   const int rc = (head_dim == 128)
                      ? launch<128>(mq, mkv, o, ldo, tiles, n_tiles, q_pos, n_heads, n_kv_heads,
-                                   v_off, status, stream, lists_from_device)
+                                   v_off, status, stream, stamp)
                      : launch<64>(mq, mkv, o, ldo, tiles, n_tiles, q_pos, n_heads, n_kv_heads,
-                                  v_off, status, stream, lists_from_device);
-  // QK^T and PV over each active query's causal context; Q, K, V read once and O written once
-  trace_end(slot, stream, TR_ATTN, 4.0 * head_dim * n_heads * ctx_sum,
-            2.0 * (2.0 * n_q * n_heads * head_dim + 2.0 * n_kv * n_kv_heads * head_dim));
+                                  v_off, status, stream, stamp);
+  trace_end(slot, stream, TR_ATTN, fl, by);
   return rc;
 }
 
@@ -483,6 +483,10 @@ int attention_decode_run(const void* q, const void* kv, int ldkv, int v_off, voi
     return fail(SPD_EINVAL, "n_heads must be a multiple of n_kv_heads");
   if ((ldkv | v_off) % 4) return fail(SPD_EINVAL, "K/V rows must be 8-byte aligned");
   const float scale_log2 = float(1.4426950408889634 / sqrt(double(head_dim)));
+  // Q read and O written once per query; K and V of every visible key once per KV head
+  const double fl = 4.0 * head_dim * n_heads * ctx_sum;
+  const double by = 2.0 * (2.0 * n_tiles * n_heads * head_dim + 2.0 * ctx_sum * n_kv_heads * head_dim);
+  unsigned long long* stamp = stamp_slot(TR_ATTN, fl, by);
   const int slot = trace_begin(stream);
   const auto* qb = static_cast<const __nv_bfloat16*>(q);
   const auto* kb = static_cast<const __nv_bfloat16*>(kv);
@@ -493,7 +497,7 @@ int attention_decode_run(const void* q, const void* kv, int ldkv, int v_off, voi
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = overlap_allowed();
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   attr[1].id = cudaLaunchAttributeClusterDimension;
   attr[1].val.clusterDim.x = 1;
   attr[1].val.clusterDim.y = 1;
@@ -502,13 +506,11 @@ int attention_decode_run(const void* q, const void* kv, int ldkv, int v_off, voi
   cfg.numAttrs = 2;
   if (head_dim == 128)
     SPD_CUDA_TRY(cudaLaunchKernelEx(&cfg, attn_decode_kernel<128>, qb, kb, ldkv, v_off, ob, ldo, tiles,
-                                    n_heads, n_kv_heads, scale_log2));
+                                    n_heads, n_kv_heads, scale_log2, stamp));
   else
     SPD_CUDA_TRY(cudaLaunchKernelEx(&cfg, attn_decode_kernel<64>, qb, kb, ldkv, v_off, ob, ldo, tiles,
-                                    n_heads, n_kv_heads, scale_log2));
-  // Q read and O written once per query; K and V of every visible key once per KV head
-  trace_end(slot, stream, TR_ATTN, 4.0 * head_dim * n_heads * ctx_sum,
-            2.0 * (2.0 * n_tiles * n_heads * head_dim + 2.0 * ctx_sum * n_kv_heads * head_dim));
+                                    n_heads, n_kv_heads, scale_log2, stamp));
+  trace_end(slot, stream, TR_ATTN, fl, by);
   return SPD_OK;
 }
 

@@ -100,6 +100,7 @@ struct KArgs {
   const uint16_t* norm_gain;
   const int32_t* norm_rows;
   float norm_eps;
+  unsigned long long* stamp;  // launch stamp [start, end] (measurement; null = off)
 };
 
 __device__ __forceinline__ float warp_sum_f(float v) {
@@ -521,6 +522,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     pdl_wait();
+    if (lane == 0) stamp_start(a.stamp);
     if (lane == 0 && prank == 0) {
       // ---- MMA issuer (PAIR: the even CTA, for both) ----
       const uint32_t idesc = idesc_bf16_f32(PAIR ? 2 * kBM : kBM, a.tt);
@@ -879,6 +881,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if (threadIdx.x == 0) stamp_end(a.stamp);
   if constexpr (PAIR) {
     // the even CTA's MMAs have completed (its MMA thread waited above) and both CTAs' epilogues
     // are done before either CTA frees its TMEM or leaves (its shared memory feeds the MMAs)
@@ -982,7 +985,7 @@ __device__ __forceinline__ float dot8_bf16(const int4& w, const int4& x, float a
 // occupancy).
 template <int EPI, int NT, int CPR>
 __global__ void __launch_bounds__(kGemvThreads)
-    gemv_kernel(const uint16_t* __restrict__ w, const uint16_t* __restrict__ x, const KArgs a,
+    gemv_kernel(const uint16_t* __restrict__ w, const uint16_t* x, const KArgs a,
                 int ksplit) {
   extern __shared__ __align__(16) uint8_t gsm[];
   __shared__ float red[32][NT];
@@ -1043,6 +1046,7 @@ __global__ void __launch_bounds__(kGemvThreads)
   int4 b0[2][CPR];
   load(b0, 0);  // weights do not depend on the predecessor: in flight before the wait
   pdl_wait();
+  if (threadIdx.x == 0) stamp_start(a.stamp);
   if (a.norm_h) {  // the input RMSNorm of each token's fp32 row, computed by every CTA
     __shared__ float nred[kGemvThreads / 32][NT];
     __shared__ float ninv[NT];
@@ -1119,6 +1123,7 @@ __global__ void __launch_bounds__(kGemvThreads)
 #pragma unroll
     for (int t = 0; t < 8; ++t) v[t] = t < NT ? red[lane][t] : 0.0f;
     epilogue8<EPI>(a, n0 + lane, (n0 >> 5) & 3, lane, n0 >> 7, 0, v, trow, tpos, 0);
+    if (lane == 0) stamp_end(a.stamp);
   }
 }
 
@@ -1207,9 +1212,8 @@ int max_active_clusters(int C) {
 
 namespace {
 // Algorithmic work of one GEMM call (valid output columns only; weights, activations and results
-// move once; fused QKV: query rows count for the query tokens only), recorded with its trace slot.
-void trace_gemm(int slot, const GemmProblem& p, cudaStream_t stream) {
-  if (slot < 0) return;
+// move once; fused QKV: query rows count for the query tokens only).
+void gemm_work(const GemmProblem& p, double* flops, double* bytes) {
   const double cols = (p.epi == EPI_SWIGLU_BF16) ? 2.0 * p.out_cols : double(p.n_out);
   const double out_cols = (p.epi == EPI_SWIGLU_BF16) ? double(p.out_cols) : double(p.n_out);
   const double ob = (p.epi == EPI_F32) ? 4.0 : (p.epi == EPI_ADD_F32) ? 8.0 : 2.0;
@@ -1218,8 +1222,19 @@ void trace_gemm(int slot, const GemmProblem& p, cudaStream_t stream) {
     tok_cols = double(p.n_tok_out) * p.split + double(p.n_tok) * (p.n_out - p.split);
     tok_out = tok_cols;
   }
-  trace_end(slot, stream, TR_GEMM, 2.0 * tok_cols * p.k,
-            2.0 * cols * p.k + 2.0 * p.n_tok * p.k + ob * tok_out);
+  *flops = 2.0 * tok_cols * p.k;
+  *bytes = 2.0 * cols * p.k + 2.0 * p.n_tok * p.k + ob * tok_out;
+}
+void trace_gemm(int slot, const GemmProblem& p, cudaStream_t stream) {
+  if (slot < 0) return;
+  double fl, by;
+  gemm_work(p, &fl, &by);
+  trace_end(slot, stream, TR_GEMM, fl, by);
+}
+unsigned long long* gemm_stamp(const GemmProblem& p) {
+  double fl, by;
+  gemm_work(p, &fl, &by);
+  return stamp_slot(TR_GEMM, fl, by);
 }
 
 bool gemv_eligible(const GemmProblem& p) {
@@ -1253,6 +1268,7 @@ int gemv_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.norm_gain = p.norm_gain;
   a.norm_rows = p.norm_rows;
   a.norm_eps = p.norm_eps;
+  a.stamp = gemm_stamp(p);
   const int groups = (p.n_out + 31) / 32, C = p.k / kGemvChunk;
   // residual epilogues split K until about two CTAs per SM stream (each at least one chunk column)
   int ksplit = 1;
@@ -1409,6 +1425,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.counters = s.counters;
   a.status = s.status;
   a.budget = kWaitBudget;
+  a.stamp = gemm_stamp(p);
 
   const size_t smem = size_t(a.stages) * stage_bytes + 1024 + 256 + 2048;
   const int slot = trace_begin(stream);
@@ -1420,7 +1437,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
     cfg.stream = stream;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = overlap_allowed();
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     attr[1].id = cudaLaunchAttributeClusterDimension;
     attr[1].val.clusterDim.x = pair ? 2 : (a.cluster ? a.csplit : 1);
     attr[1].val.clusterDim.y = 1;

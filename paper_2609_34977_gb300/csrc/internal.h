@@ -26,18 +26,21 @@ constexpr long long kWaitBudget = 1ll << 30;
 
 int num_sms();  // SM count of the current device
 
-// Programmatic overlap of consecutive launches is off on this thread while a NoOverlap guard is
-// alive (launches then follow plain stream order; the kernels' griddepcontrol instructions are
-// no-ops).
-extern thread_local int g_no_overlap;
-struct NoOverlap {
-  NoOverlap() { ++g_no_overlap; }
-  ~NoOverlap() { --g_no_overlap; }
-};
-inline int overlap_allowed() { return g_no_overlap ? 0 : 1; }
 
 // Launches a kernel with programmatic stream serialization: it may be scheduled while the previous
 // kernel of the stream is still running, and orders itself after it with griddepcontrol.wait.
+//
+// Rules every kernel of the library keeps under this overlap (the chain of launches in a stream
+// can have several kernels resident at once, each waiting on its predecessor):
+//  * before griddepcontrol.wait a kernel reads only data that no launch of the library writes
+//    (weights, tensor maps, its own arguments) and writes nothing but its own shared memory;
+//  * data that an earlier kernel of the stream wrote is read after the wait, and never through
+//    the non-coherent path (no const __restrict__ pointers or ld.global.nc on it: PTX allows that
+//    path only for data that stays unchanged while the kernel runs, and here the predecessor
+//    writes it during this kernel's prologue);
+//  * every kernel executes griddepcontrol.wait in at least one thread before it can complete, so
+//    completion orders transitively: when kernel N passes its wait, every earlier kernel of the
+//    stream has completed.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
                        cudaStream_t stream, Args&&... args) {
@@ -48,7 +51,7 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = overlap_allowed();
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
@@ -135,12 +138,9 @@ int make_operand_map(CUtensorMap* map, const void* ptr, int inner, int outer, in
 // positions ascending within a sequence) over the keys and values of their sequences (kv
 // [n_kv][ldkv]: K of head g at column g * head_dim, V at v_off + g * head_dim). `tiles` (device
 // int4 [n_tiles]): first query row, query count (1..128), first key row, sequence length.
-// lists_from_device: the tiles and q_pos were written by a kernel earlier in the stream (read
-// after the grid dependency wait) rather than copied from the host.
 int attention_run(const void* q, int n_q, const void* kv, int n_kv, int ldkv, int v_off, void* o,
                   int ldo, const int4* tiles, int n_tiles, const int32_t* q_pos, int n_heads,
-                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum,
-                  bool lists_from_device = false);
+                  int n_kv_heads, int head_dim, int* status, cudaStream_t stream, double ctx_sum);
 constexpr int kAttnTileQ = 128;  // queries per attention tile
 // The same attention when every tile holds ONE query at its sequence's last position (a decode
 // step): tiles as above with query count 1; ctx_sum = the summed key counts.
@@ -163,9 +163,6 @@ int skip_scores_run(const float* logits, int V, int n_cand, const float* h, int 
                     float w1, float add_slc, float t_skip, int mode, float* s_skip, uint8_t* flag,
                     cudaStream_t stream, int32_t* admit = nullptr, uint8_t* target = nullptr,
                     int layer = 0, int tgt = 0);
-// An empty kernel launched without programmatic overlap: the kernels after it start only once all
-// earlier work in the stream has completed.
-int stream_barrier(cudaStream_t stream);
 // Layer l's row lists built on the device from admission layers (see plan_lists_kernel).
 constexpr int kPlanMaxSeqs = 1024;
 int plan_lists_run(int T, int B, const int32_t* cu, const int32_t* pos, const int32_t* admit,

@@ -29,12 +29,13 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 // out[orow(i)] = bf16(gain * h[irow(i)] / sqrt(mean(h^2) + eps)); out2[map2[irow]] gets the same
 // row when map2 is given and map2[irow] >= 0 (compact copy of the attention-active rows).
 __global__ void __launch_bounds__(kThreads)
-    rmsnorm_kernel(const float* __restrict__ h, int D, const uint16_t* __restrict__ gain, float eps,
-                   const int32_t* __restrict__ in_rows, __nv_bfloat16* __restrict__ out,
-                   const int32_t* __restrict__ map2, __nv_bfloat16* __restrict__ out2) {
+    rmsnorm_kernel(const float* h, int D, const uint16_t* __restrict__ gain, float eps,
+                   const int32_t* in_rows, __nv_bfloat16* __restrict__ out, const int32_t* map2,
+                   __nv_bfloat16* __restrict__ out2, unsigned long long* stamp) {
   __shared__ float red[kThreads / 32];
   pdl_launch_dependents();
   pdl_wait();
+  if (threadIdx.x == 0) stamp_start(stamp);
   const int i = blockIdx.x;
   const int r = in_rows ? in_rows[i] : i;
   if (r < 0) return;  // a padding entry of a device-built row list
@@ -64,9 +65,10 @@ __global__ void __launch_bounds__(kThreads)
     reinterpret_cast<uint2*>(out + size_t(i) * D)[c] = pk;
     if (r2 >= 0) reinterpret_cast<uint2*>(out2 + size_t(r2) * D)[c] = pk;
   }
+  if (threadIdx.x == 0) stamp_end(stamp);
 }
 
-__global__ void bf16_to_f32_kernel(const uint16_t* __restrict__ x, float* __restrict__ h, size_t n4) {
+__global__ void bf16_to_f32_kernel(const uint16_t* x, float* __restrict__ h, size_t n4) {
   pdl_launch_dependents();
   pdl_wait();
   for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < n4;
@@ -78,8 +80,8 @@ __global__ void bf16_to_f32_kernel(const uint16_t* __restrict__ x, float* __rest
   }
 }
 
-__global__ void scatter_rows_kernel(const uint16_t* __restrict__ src, int D,
-                                    const int32_t* __restrict__ rows, uint16_t* __restrict__ dst) {
+__global__ void scatter_rows_kernel(const uint16_t* src, int D, const int32_t* rows,
+                                    uint16_t* __restrict__ dst) {
   pdl_launch_dependents();
   pdl_wait();
   const int i = blockIdx.x;
@@ -90,9 +92,8 @@ __global__ void scatter_rows_kernel(const uint16_t* __restrict__ src, int D,
 
 // q_t of sequence b (ASL-Skip's text context, Sec. 4.2.1): the mean of h over the text tokens
 // text[ts[b] .. ts[b+1]), one thread per column, tokens in order (zero when there are none).
-__global__ void __launch_bounds__(kThreads) text_mean_kernel(const float* __restrict__ h, int D,
-                                                             const int32_t* __restrict__ ts,
-                                                             const int32_t* __restrict__ text,
+__global__ void __launch_bounds__(kThreads) text_mean_kernel(const float* h, int D, const int32_t* ts,
+                                                             const int32_t* text,
                                                              float* __restrict__ tmean) {
   pdl_launch_dependents();
   pdl_wait();
@@ -121,12 +122,10 @@ __device__ __forceinline__ float block_max(float v, float* red) {
 // row) / log V, F_itc = (cos(h_i, q_t) + 1) / 2 (0.5 without text), S_sa = ReLU(1 - E - F);
 // s_skip[i] += w1 S_sa + w2 SLC^Norm(l), flag[n] = s_skip[i] >= T_skip.
 __global__ void __launch_bounds__(kThreads)
-    skip_score_kernel(const float* __restrict__ logits, int V, const float* __restrict__ h, int D,
-                      const int32_t* __restrict__ cand, const int32_t* __restrict__ ts,
-                      const int32_t* __restrict__ seq_of, const float* __restrict__ tmean,
-                      float inv_log_v, float w1, float add_slc, float t_skip, int mode,
-                      float* __restrict__ s_skip, uint8_t* __restrict__ flag,
-                      int32_t* __restrict__ admit, uint8_t* __restrict__ target, int layer, int tgt) {
+    skip_score_kernel(const float* logits, int V, const float* h, int D, const int32_t* cand,
+                      const int32_t* ts, const int32_t* seq_of, const float* tmean, float inv_log_v,
+                      float w1, float add_slc, float t_skip, int mode, float* s_skip, uint8_t* flag,
+                      int32_t* admit, uint8_t* target, int layer, int tgt) {
   __shared__ float red[kThreads / 32];
   pdl_launch_dependents();
   pdl_wait();
@@ -221,11 +220,9 @@ __device__ int block_scan_excl(int v, int* tmp, int* total) {
 // sequence each; padded to max_tiles with copies of the last tile, whose recomputation writes the
 // same values, or a one-query tile when no token is a query). One CTA.
 __global__ void __launch_bounds__(1024)
-    plan_lists_kernel(int T, int B, const int32_t* __restrict__ cu, const int32_t* __restrict__ pos,
-                      const int32_t* __restrict__ admit, const uint8_t* __restrict__ target, int l,
-                      const int32_t* __restrict__ kv0, const int32_t* __restrict__ kvlen,
-                      int32_t* __restrict__ arows, int32_t* __restrict__ amap,
-                      int32_t* __restrict__ apos, int32_t* __restrict__ frows, int4* __restrict__ tiles,
+    plan_lists_kernel(int T, int B, const int32_t* cu, const int32_t* pos, const int32_t* admit,
+                      const uint8_t* target, int l, const int32_t* kv0, const int32_t* kvlen,
+                      int32_t* arows, int32_t* amap, int32_t* apos, int32_t* frows, int4* tiles,
                       int max_tiles) {
   __shared__ int tmp[32];
   __shared__ int seq_cnt[kPlanMaxSeqs];
@@ -301,26 +298,13 @@ int skip_scores_run(const float* logits, int V, int n_cand, const float* h, int 
   return SPD_OK;
 }
 
-namespace {
-__global__ void stream_barrier_kernel() {}
-}  // namespace
-
-int stream_barrier(cudaStream_t stream) {
-  stream_barrier_kernel<<<1, 32, 0, stream>>>();
-  SPD_CUDA_TRY(cudaGetLastError());
-  return SPD_OK;
-}
-
 int plan_lists_run(int T, int B, const int32_t* cu, const int32_t* pos, const int32_t* admit,
                    const uint8_t* target, int l, const int32_t* kv0, const int32_t* kvlen,
                    int32_t* arows, int32_t* amap, int32_t* apos, int32_t* frows, int4* tiles,
                    int max_tiles, cudaStream_t stream) {
   if (B > kPlanMaxSeqs) return fail(SPD_EUNSUPPORTED, "device plans support at most %d sequences", kPlanMaxSeqs);
-  // an ordinary launch (no programmatic overlap): it starts once all earlier work in the stream
-  // has completed, so every later kernel sees the decisions and the lists complete
-  plan_lists_kernel<<<1, 1024, 0, stream>>>(T, B, cu, pos, admit, target, l, kv0, kvlen, arows, amap,
-                                            apos, frows, tiles, max_tiles);
-  SPD_CUDA_TRY(cudaGetLastError());
+  SPD_CUDA_TRY(launch_pdl(plan_lists_kernel, dim3(1), dim3(1024), 0, stream, T, B, cu, pos, admit,
+                          target, l, kv0, kvlen, arows, amap, apos, frows, tiles, max_tiles));
   return SPD_OK;
 }
 
@@ -328,10 +312,11 @@ int rmsnorm_run(const float* h, int n_rows, int D, const uint16_t* gain, float e
                 const int32_t* in_rows, void* out, const int32_t* map2, void* out2,
                 cudaStream_t stream) {
   if (n_rows <= 0) return SPD_OK;
+  unsigned long long* stamp = stamp_slot(TR_ROWS, 4.0 * n_rows * D, double(n_rows) * D * (4.0 + 2.0));
   const int slot = trace_begin(stream);
   SPD_CUDA_TRY(launch_pdl(rmsnorm_kernel, dim3(n_rows), dim3(kThreads), 0, stream, h, D, gain, eps,
                           in_rows, static_cast<__nv_bfloat16*>(out), map2,
-                          static_cast<__nv_bfloat16*>(out2)));
+                          static_cast<__nv_bfloat16*>(out2), stamp));
   trace_end(slot, stream, TR_ROWS, 4.0 * n_rows * D, double(n_rows) * D * (4.0 + 2.0));
   return SPD_OK;
 }

@@ -156,7 +156,7 @@ __device__ __forceinline__ const float* feat_row(const PruneDims& p, int l, int 
 
 // ---- 1. a_v and inverse norms ---------------------------------------------------------------
 template <int SIM>
-__global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float* __restrict__ attn,
+__global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float* attn,
                                                        PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
@@ -904,7 +904,7 @@ __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
 // ---- received attention from full maps (Sec. 4.1.1 without [CLS]) ------------------------------
 // Column sums of attention maps: CTA (column block, map, row split) adds rows [q0, q1) of its 1024
 // columns (thread: four adjacent columns, float4 loads, eight rows in flight) in row order.
-__global__ void __launch_bounds__(256) received_colsum_kernel(const float* __restrict__ maps, int n_q,
+__global__ void __launch_bounds__(256) received_colsum_kernel(const float* maps, int n_q,
                                                               int n_k, int rows_per_split,
                                                               float* __restrict__ partial) {
   pdl_launch_dependents();
@@ -934,11 +934,11 @@ __global__ void __launch_bounds__(256) received_colsum_kernel(const float* __res
 
 // out[m][j] = sum over the members i of group j (ascending) of (sum over splits, in order, of the
 // partial column sums) / n_q; without groups j = i.
-__global__ void __launch_bounds__(256) received_finish_kernel(const float* __restrict__ partial,
+__global__ void __launch_bounds__(256) received_finish_kernel(const float* partial,
                                                               int n_maps, int n_k, int n_splits,
                                                               float inv_nq,
-                                                              const int32_t* __restrict__ gstart,
-                                                              const int32_t* __restrict__ gmem,
+                                                              const int32_t* gstart,
+                                                              const int32_t* gmem,
                                                               int n_out, float* __restrict__ out,
                                                               int* status) {
   pdl_launch_dependents();
@@ -1037,8 +1037,8 @@ __global__ void __launch_bounds__(1024) select_kernel(PruneDims p, PruneWs w, in
   }
 }
 
-__global__ void gather_bf16_kernel(const float* __restrict__ src, int n_tok, int d, int off,
-                                   const int32_t* __restrict__ idx, int keep,
+__global__ void gather_bf16_kernel(const float* src, int n_tok, int d, int off, const int32_t* idx,
+                                   int keep,
                                    __nv_bfloat16* __restrict__ dst, int* status) {
   pdl_launch_dependents();
   pdl_wait();
@@ -1143,7 +1143,7 @@ cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, size_t smem, cud
   cfg.stream = st;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = overlap_allowed();
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   attr[1].id = cudaLaunchAttributeClusterDimension;
   attr[1].val.clusterDim.x = KC;
   attr[1].val.clusterDim.y = 1;

@@ -301,6 +301,21 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 // when the kernel was launched without programmatic serialization.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// ---- launch stamps (measurement) ----------------------------------------------------------------
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Earliest start of a launch's work (call once per CTA after its grid dependency wait) and latest
+// end (once per CTA after its last store); s = [start, end] or null.
+__device__ __forceinline__ void stamp_start(unsigned long long* s) {
+  if (s) atomicMin(s, global_ns());
+}
+__device__ __forceinline__ void stamp_end(unsigned long long* s) {
+  if (s) atomicMax(s + 1, global_ns());
+}
+
 // Records the first device-side failure in a status word (0 = OK).
 __device__ __forceinline__ void set_status(int* status, int code) {
   if (status) atomicCAS(status, 0, code);

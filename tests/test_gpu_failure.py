@@ -26,8 +26,12 @@ def test_bounded_wait_times_out_and_context_survives():
 def test_host_side_rejections_touch_nothing():
     ws = torch.zeros(16, dtype=torch.uint8, device="cuda")
     X = torch.ones(4, 128, dtype=torch.bfloat16, device="cuda")
+    W = torch.ones(128, 128, dtype=torch.bfloat16, device="cuda")
     out = torch.zeros(4, 128, device="cuda")
     with pytest.raises(N.SpiderError) as e:
-        N.spd_linear(X, 4, 128, X, 128, N.EPI_F32, out, 128, ws)   # workspace too small
+        N.spd_linear(X, 4, 128, W, 128, N.EPI_F32, out, 128, ws)   # workspace too small
     assert e.value.code == N.SPD_ENOSPC
+    with pytest.raises(ValueError):                                 # weights too small (binding)
+        N.spd_linear(X, 4, 128, X, 128, N.EPI_F32, out, 128, ws)
+    torch.cuda.synchronize()
     assert not out.any()

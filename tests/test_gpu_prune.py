@@ -140,13 +140,19 @@ def test_received_attention_through_a_2x2_merger_feeds_prune():
     got = _gpu_received(maps, groups)
     ref = op.received_attention(maps.float().double().numpy(), groups)
     np.testing.assert_allclose(got, ref, rtol=1e-5, atol=1e-9)
-    a = torch.from_numpy(got.astype(np.float32))[None]  # [1 tile][H][320]
-    _, v, _ = conditioned_vision(20260701, 1, len(groups), 128, 2, H, 80, 1, has_cls=False,
-                                 attn_form=1)
-    v["attn"] = a.numpy()
-    res = op.prune(v["feats"], v["attn"], has_cls=False, attn_form=1, final_layer=1, keep=80)
-    if all(op.well_conditioned(r) for r in res):
-        assert_prune_parity(gpu_prune(v, 80, 1, has_cls=False, attn_form=1), res)
+    # the oracle prunes with its own received form, the GPU with the GPU's (equal within 1e-5):
+    # the first feature seed on which every decision of the oracle has a margin above 1e-3
+    a_ref = ref.astype(np.float32)[None]  # [1 tile][H][320]
+    for seed in range(20260701, 20260701 + 64):
+        v = synth.vision_tiles(seed, 1, len(groups), 128, 2, H, has_cls=False, attn_form=1)
+        v["attn"] = a_ref
+        res = op.prune(v["feats"], v["attn"], has_cls=False, attn_form=1, final_layer=1, keep=80)
+        if all(op.well_conditioned(r) for r in res):
+            break
+    else:
+        pytest.fail("no well-conditioned feature seed for the merged received form")
+    v["attn"] = got.astype(np.float32)[None]
+    assert_prune_parity(gpu_prune(v, 80, 1, has_cls=False, attn_form=1), res)
 
 
 def test_received_attention_repeat_runs_are_bitwise_identical():

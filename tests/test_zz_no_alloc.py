@@ -66,12 +66,18 @@ def test_noalloc_residual_add_into_rows():
         assert rowwise_rel(h.cpu().numpy(), ref.cpu().numpy()) < 1e-4
 
 
-def test_noalloc_rejects_outputs_beyond_its_scratch():
-    # 4097 output tiles of 128 weight rows x 256 tokens: refused on the host, nothing launched
-    M, K, N_ = 1, 64, 4097 * 128
+@pytest.mark.parametrize("M,N_", [
+    (1, 4097 * 128),  # 2 x 2049 counters for one token tile
+    (600, 1365 * 128),  # 2 x 683 x 3 = 4098 counters (CTA pairs count each half of a 256-row tile)
+])
+def test_noalloc_rejects_problems_beyond_its_scratch(M, N_):
+    # more tile counters than the static scratch holds: refused on the host, nothing enqueued
+    K = 64
     X = torch.zeros(M, K, dtype=torch.bfloat16, device="cuda")
-    W = torch.zeros(1, K, dtype=torch.bfloat16, device="cuda")  # never read
-    out = torch.zeros(1, dtype=torch.float32, device="cuda")     # never written
+    W = torch.zeros(N_, K, dtype=torch.bfloat16, device="cuda")  # never read
+    out = torch.zeros(M, N_, dtype=torch.float32, device="cuda")  # never written
     with pytest.raises(N.SpiderError) as e:
         N.spd_linear_noalloc(X, M, K, W, N_, N.EPI_F32, out, N_)
     assert e.value.code == N.SPD_ENOSPC
+    torch.cuda.synchronize()
+    assert not out.any()
