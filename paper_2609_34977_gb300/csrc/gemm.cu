@@ -96,6 +96,8 @@ struct KArgs {
   int* counters;
   int* status;
   long long budget;
+  int vec_red;  // residual epilogue: 16-byte reductions (n_out, ldo multiples of 4, out aligned)
+  int staged;  // rotary epilogues: the last whole segment of a CTA goes out through shared memory
   const float* norm_h;  // matrix-vector path: input RMSNorm (see GemmProblem)
   const uint16_t* norm_gain;
   const int32_t* norm_rows;
@@ -201,13 +203,12 @@ __device__ __forceinline__ void rope_cos_sin(int p, float2 f, float& c, float& s
 }
 
 // Rotary embedding of weight row nn (rows laid out in rotary pairs: lane l < 16 of a 32-row group
-// holds pair element j, lane l + 16 element j + head_dim / 2) for 8 tokens, stored as bf16 to row
-// row_of(t) (skipped when negative), column head * head_dim + rotated index. The angles are
-// computed in registers: a per-position table would cost an L2 round trip per 8 tokens.
-template <typename RowOf>
-__device__ __forceinline__ void rope_store8(const KArgs& a, __nv_bfloat16* o, int ldo, int nn,
-                                            int lane, int t0, const float (&v)[8], const int* tpos,
-                                            int tb, RowOf row_of) {
+// holds pair element j, lane l + 16 element j + head_dim / 2) for 8 tokens t0 + j, handed to
+// store(j, col, value) with col = head * head_dim + rotated index. The angles are computed in
+// registers: a per-position table would cost an L2 round trip per 8 tokens.
+template <typename Store>
+__device__ __forceinline__ void rope8(const KArgs& a, int nn, int lane, int t0, const float (&v)[8],
+                                      const int* tpos, int tb, Store store) {
   const int nt = a.n_tok;
   const int hd = a.head_dim, half = hd >> 1;
   const int head = nn / hd, g = (nn % hd) >> 5;
@@ -236,11 +237,63 @@ __device__ __forceinline__ void rope_store8(const KArgs& a, __nv_bfloat16* o, in
     y[i + 4] = fmaf(sgn * p_hi, s_hi, v[i + 4] * c_hi);
   }
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
+  for (int j = 0; j < 8; ++j) store(j, col, y[j]);
+}
+
+// rope8 stored as bf16 to row row_of(t) of o (skipped when negative or past the tokens).
+template <typename RowOf>
+__device__ __forceinline__ void rope_store8(const KArgs& a, __nv_bfloat16* o, int ldo, int nn,
+                                            int lane, int t0, const float (&v)[8], const int* tpos,
+                                            int tb, RowOf row_of) {
+  const int nt = a.n_tok;
+  rope8(a, nn, lane, t0, v, tpos, tb, [&](int j, int col, float y) {
     const int t = t0 + j;
     const int r = (t < nt) ? row_of(t) : -1;
-    if (r >= 0) o[size_t(r) * ldo + col] = __float2bfloat16_rn(y[j]);
+    if (r >= 0) o[size_t(r) * ldo + col] = __float2bfloat16_rn(y);
+  });
+}
+
+// Staged output of the rotary epilogues: the CTA's 128-column block of the output for 8 tokens,
+// written as bf16 into shared memory rows of kStgPitch bytes (token t0 + j - tb at row t0 + j -
+// tb, column col - c0) and copied out row by row afterwards (stage_copy_out).
+constexpr int kStgPitch = 256;
+template <int EPI>
+__device__ __forceinline__ void stage8(const KArgs& a, int n, int lane, int t0, const float (&v)[8],
+                                       const int* tpos, int tb, uint8_t* stg) {
+  const bool second = EPI == EPI_QKV_BF16 && n >= a.split;  // a K/V row of the fused QKV GEMM
+  const int nn = second ? n - a.split : n;                   // row within its output
+  const int c0 = nn & ~127;
+  uint8_t* base = stg + size_t(t0 - tb) * kStgPitch;
+  auto put = [&](int j, int col, float y) {
+    *reinterpret_cast<__nv_bfloat16*>(base + j * kStgPitch + 2 * (col - c0)) = __float2bfloat16_rn(y);
+  };
+  if ((EPI == EPI_QKV_BF16 && !second) || nn < a.rope_rows) {  // warp-uniform
+    rope8(a, nn, lane, t0, v, tpos, tb, put);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) put(j, nn, v[j]);
   }
+}
+
+// Copies the staged 128-column block of weight rows [n0, n0 + 128) out to global memory: one
+// 256-byte bulk copy per token row, issued by epilogue thread et for token tok0 + et (skipped past
+// the valid tokens and for negative rows). Every epilogue thread waits for its copies to complete.
+template <int EPI>
+__device__ __forceinline__ void stage_copy_out(const KArgs& a, int n0, int et, int tok0, int valid,
+                                               const int* trow, const uint8_t* stg) {
+  if (et < valid) {
+    const bool second = EPI == EPI_QKV_BF16 && n0 >= a.split;
+    const int nn0 = second ? n0 - a.split : n0;
+    const int t = tok0 + et;
+    const int r = second ? (a.rows2 ? a.rows2[t] : t) : trow[et];
+    if (r >= 0) {
+      __nv_bfloat16* o = static_cast<__nv_bfloat16*>(second ? a.out2 : a.out);
+      const int ldo = second ? a.ldo2 : a.ldo;
+      bulk_store(o + size_t(r) * ldo + nn0, stg + size_t(et) * kStgPitch, kStgPitch);
+    }
+  }
+  bulk_commit();
+  bulk_wait_all();
 }
 
 // Applies epilogue EPI to 8 consecutive tokens t0..t0+7 of weight row n (TMEM lane quarter q;
@@ -251,6 +304,42 @@ __device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane
                                           int t0, const float (&v)[8], const int* trow,
                                           const int* tpos, int tb) {
   const int nt = a.n_tok;
+  if constexpr (EPI == EPI_ADD_F32) {
+    if (a.vec_red) {
+      // 4 x 4 transposes inside each lane quad: lane k of a quad holds columns c0 .. c0 + 3 (c0 =
+      // n rounded down to 4) of tokens t0 + k and t0 + 4 + k afterwards, added with two 16-byte
+      // reductions instead of eight 4-byte ones (the residual update is bound by L2 atomics)
+      float w[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) w[j] = v[j];
+      const int k = lane & 3;
+#pragma unroll
+      for (int bit = 0; bit < 2; ++bit) {
+        const int m = 1 << bit;
+        const bool hi = (k >> bit) & 1;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (j & m) continue;
+          const float send = hi ? w[j] : w[j + m];
+          const float recv = __shfl_xor_sync(0xffffffffu, send, m);
+          if (hi) w[j] = recv;
+          else w[j + m] = recv;
+        }
+      }
+      const int c0 = n & ~3;
+      if (c0 < a.n_out) {  // n_out is a multiple of 4: a quad is in or out as a whole
+        float* o = static_cast<float*>(a.out);
+#pragma unroll
+        for (int blk = 0; blk < 2; ++blk) {
+          const int t = t0 + 4 * blk + k;
+          const int r = t < nt ? trow[t - tb] : -1;  // negative: a padding row of a device list
+          if (r >= 0) red_add_v4(o + size_t(r) * a.ldo + c0, w[4 * blk], w[4 * blk + 1],
+                                 w[4 * blk + 2], w[4 * blk + 3]);
+        }
+      }
+      return;
+    }
+  }
   if constexpr (EPI == EPI_F32 || EPI == EPI_ADD_F32) {
     if (n >= a.n_out) return;
     float* o = static_cast<float*>(a.out);
@@ -614,7 +703,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         tpos[et] = a.pos ? a.pos[tok0 + et] : 0;
       }
       epi_bar();
-      if ((kb_lo == 0 && seg_len == a.n_kb) || EPI == EPI_ADD_F32) {
+      constexpr bool kStaged = EPI == EPI_QKV_BF16 || EPI == EPI_ROPE_BF16;
+      if (kStaged && a.staged && j == plan.count - 1 && kb_lo == 0 && seg_len == a.n_kb) {
+        // the CTA's last segment, whole: every MMA has completed, so the stage ring is idle and
+        // holds the output block (bf16 rows of 256 bytes per 128 weight rows), which bulk copies
+        // move out row by row instead of 2-byte scattered stores
+        uint8_t* stg = smem;
+        for (int h = 0; h < a.nh; ++h) {
+          uint8_t* sh = stg + size_t(h) * a.tt * kStgPitch;
+#pragma unroll 1
+          for (int cc = half * 8; cc < valid; cc += 16) {
+            float v[8];
+            tmem_ld8(tq + h * a.hoff + cc, v);
+            stage8<EPI>(a, (blk0 + h) * kBM + row, lane, tok0 + cc, v, tpos, tok0, sh);
+          }
+        }
+        fence_proxy_async_smem();
+        epi_bar();
+        for (int h = 0; h < a.nh; ++h)
+          stage_copy_out<EPI>(a, (blk0 + h) * kBM, et, tok0, valid, trow,
+                              stg + size_t(h) * a.tt * kStgPitch);
+      } else if ((kb_lo == 0 && seg_len == a.n_kb) || EPI == EPI_ADD_F32) {
         for (int h = 0; h < a.nh; ++h) {
 #pragma unroll 1
           for (int cc = half * 8; cc < valid; cc += 16) {
@@ -1237,6 +1346,12 @@ unsigned long long* gemm_stamp(const GemmProblem& p) {
   return stamp_slot(TR_GEMM, fl, by);
 }
 
+// 16-byte residual reductions need 4-column groups that start 16-byte aligned in every row
+bool vec_red_ok(const GemmProblem& p) {
+  return p.epi == EPI_ADD_F32 && p.n_out % 4 == 0 && p.ldo % 4 == 0 &&
+         (reinterpret_cast<uintptr_t>(p.out) & 15) == 0;
+}
+
 bool gemv_eligible(const GemmProblem& p) {
   if (p.norm_h && ((reinterpret_cast<uintptr_t>(p.norm_h) | reinterpret_cast<uintptr_t>(p.norm_gain)) & 15))
     return false;
@@ -1269,6 +1384,7 @@ int gemv_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.norm_rows = p.norm_rows;
   a.norm_eps = p.norm_eps;
   a.stamp = gemm_stamp(p);
+  a.vec_red = vec_red_ok(p);
   const int groups = (p.n_out + 31) / 32, C = p.k / kGemvChunk;
   // residual epilogues split K until about two CTAs per SM stream (each at least one chunk column)
   int ksplit = 1;
@@ -1426,6 +1542,16 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.status = s.status;
   a.budget = kWaitBudget;
   a.stamp = gemm_stamp(p);
+  a.vec_red = vec_red_ok(p);
+  {
+    // staged rotary epilogues: whole 128-column output blocks of 16-byte aligned rows, the block
+    // of every token of the tile fitting in the idle stage ring
+    const bool rot = p.epi == EPI_QKV_BF16 || p.epi == EPI_ROPE_BF16;
+    const bool al = ((reinterpret_cast<uintptr_t>(p.out) | reinterpret_cast<uintptr_t>(p.out2)) & 15) == 0 &&
+                    p.ldo % 8 == 0 && (p.epi != EPI_QKV_BF16 || p.ldo2 % 8 == 0);
+    a.staged = rot && al && !a.cluster && p.n_out % kBM == 0 && (p.epi != EPI_QKV_BF16 || p.split % kBM == 0) &&
+               size_t(a.nh) * a.tt * kStgPitch <= size_t(a.stages) * stage_bytes;
+  }
 
   const size_t smem = size_t(a.stages) * stage_bytes + 1024 + 256 + 2048;
   const int slot = trace_begin(stream);

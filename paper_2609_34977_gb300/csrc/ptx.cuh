@@ -85,6 +85,20 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
       "l"(static_cast<uint64_t>(__cvta_generic_to_global(src))), "r"(bytes), "r"(smem_u32(bar))
       : "memory");
 }
+// 1D bulk copy of `bytes` (a multiple of 16; both addresses 16-byte aligned) from this CTA's shared
+// memory to global memory, in the issuing thread's current bulk group. Shared-memory data written
+// by generic stores needs fence_proxy_async_smem() (and a barrier) before the copy is issued.
+__device__ __forceinline__ void bulk_store(void* dst, const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(
+                   static_cast<uint64_t>(__cvta_generic_to_global(dst))),
+               "r"(smem_u32(src)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Waits until every bulk group the thread committed has completed (its global writes performed).
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
@@ -314,6 +328,12 @@ __device__ __forceinline__ void stamp_start(unsigned long long* s) {
 }
 __device__ __forceinline__ void stamp_end(unsigned long long* s) {
   if (s) atomicMax(s + 1, global_ns());
+}
+
+// Fire-and-forget 16-byte reduction p[0..3] += (a, b, c, d) at L2 (p 16-byte aligned).
+__device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c), "f"(d)
+               : "memory");
 }
 
 // Records the first device-side failure in a status word (0 = OK).
