@@ -55,6 +55,15 @@ int spd_workspace_status(void* ws, void* stream, int* status);
  * context stays usable. Asynchronous; read the result with spd_workspace_status. */
 int spd_selftest_bounded_wait(void* ws, long long budget_cycles, void* stream);
 
+/* Deterministic mode (library-wide; no counterpart in the paper). With on != 0, every GEMM sums
+ * each output element in a fixed order: K-split tiles store per-CTA fp32 partials that the tile's
+ * last CTA adds in CTA order, and residual updates of the fp32 stream are one read-modify-write per
+ * element. Repeated calls on the same inputs then give bit-identical results. With on = 0 (the
+ * default), split partial sums and residual updates are fire-and-forget fp32 reductions at L2,
+ * whose order varies, so the last bits (and, through bf16 roundings downstream, a bf16 unit) may
+ * differ between runs. Takes effect for launches enqueued after the call; returns SPD_OK. */
+int spd_set_deterministic(int on);
+
 /* Kernel-class tracing (no counterpart in the paper; measurement support). spd_trace_enable(n)
  * starts recording up to n launches: every launch of the library is bracketed by a CUDA event pair
  * on its stream and tagged with its class and algorithmic work; n <= 0 stops recording.

@@ -30,7 +30,7 @@ EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait"
            "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
            "spd_trace_read", "spd_prune_workspace", "spd_prefill_workspace", "spd_gather_bf16",
            "spd_last_error_detail", "spd_check", "spd_plan_from_layer_mask", "spd_prefill_admit",
-           "spd_stamp_enable", "spd_stamp_read", "spd_stamp_launch")
+           "spd_stamp_enable", "spd_stamp_read", "spd_stamp_launch", "spd_set_deterministic")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
 
 
@@ -132,6 +132,7 @@ def lib():
             "spd_linear": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, sz, vp]),
             "spd_linear_noalloc": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, vp]),
             "spd_trace_enable": (i, [i]),
+            "spd_set_deterministic": (i, [i]),
             "spd_stamp_enable": (i, [i]),
             "spd_stamp_launch": (i, [i, C.POINTER(i), C.POINTER(C.c_ulonglong), C.POINTER(C.c_ulonglong),
                                      C.POINTER(C.c_double), C.POINTER(C.c_double)]),
@@ -543,3 +544,8 @@ def spd_stamp_launches() -> list:
         out.append((cls.value, s0.value, s1.value, fl.value, by.value))
         k += 1
     return out
+
+
+def spd_set_deterministic(on: bool):
+    """Library-wide deterministic mode: GEMM sums in a fixed order (bit-identical repeated runs)."""
+    _check(lib().spd_set_deterministic(int(bool(on))))

@@ -111,6 +111,11 @@ struct spd_model {
 
 extern "C" const char* spd_last_error(void) { return g_err; }
 
+extern "C" int spd_set_deterministic(int on) {
+  set_deterministic(on);
+  return SPD_OK;
+}
+
 extern "C" int spd_workspace_status(void* ws, void* stream, int* status) {
   if (!ws || !status) return fail(SPD_EINVAL, "null workspace or status");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -307,8 +312,15 @@ static GemmScratch scratch_from(Carve& cv) {
   s.partial = cv.take<float>(s.partial_floats);
   s.n_counters = 1 << 16;
   s.counters = cv.take<int>(s.n_counters);
+  s.acc = nullptr;
+  s.acc_floats = 0;
   s.status = cv.status();
   return s;
+}
+// The accumulation buffers, carved last in a workspace (after the activation buffers).
+static void take_acc(Carve& cv, GemmScratch& s) {
+  s.acc_floats = kGemmAccFloats;
+  s.acc = cv.take<float>(s.acc_floats);
 }
 
 extern "C" int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, int N, int epilogue,
@@ -321,9 +333,10 @@ extern "C" int spd_linear(const uint16_t* X, int M, int K, const uint16_t* W, in
     return fail(SPD_EINVAL, "epilogue needs a bias");
   Carve cv(ws, ws_bytes);
   GemmScratch s = scratch_from(cv);
+  take_acc(cv, s);
   if (!cv.fits()) return fail(SPD_ENOSPC, "linear workspace too small");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  SPD_CUDA_TRY(cudaMemsetAsync(s.counters, 0, s.n_counters * sizeof(int), st));
+  if (int rc = gemm_scratch_clear(s, st)) return rc;
   GemmProblem p{};
   p.w = W;
   p.x = X;
@@ -388,10 +401,12 @@ extern "C" int spd_linear_noalloc(const uint16_t* X, int M, int K, const uint16_
   s.counters = cv.take<int>(s.n_counters);
   s.partial = cv.take<float>(0);
   s.partial_floats = (SPD_LINEAR_NOALLOC_SCRATCH_BYTES - cv.used) / sizeof(float);
+  s.acc = nullptr;  // no accumulation buffers: stream-K partial slots only
+  s.acc_floats = 0;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   // the status word and the counters start at zero (a failed earlier call may have left them set)
   SPD_CUDA_TRY(cudaMemsetAsync(base, 0, 256, st));
-  SPD_CUDA_TRY(cudaMemsetAsync(s.counters, 0, s.n_counters * sizeof(int), st));
+  if (int rc = gemm_scratch_clear(s, st)) return rc;
   GemmProblem p{};
   p.w = W;
   p.x = X;
@@ -413,8 +428,9 @@ extern "C" int spd_linear_noalloc(const uint16_t* X, int M, int K, const uint16_
 extern "C" size_t spd_project_workspace_size(const spd_model* m, int rows) {
   if (!m || rows < 0) return 0;
   Carve cv(nullptr, ~size_t(0));
-  scratch_from(cv);
+  GemmScratch s = scratch_from(cv);
   cv.take<uint16_t>(size_t(rows) * (m->cfg.d_proj > 0 ? m->cfg.d_proj : 1));
+  take_acc(cv, s);
   return cv.used;
 }
 
@@ -425,9 +441,10 @@ extern "C" int spd_project(const spd_model* m, const uint16_t* vis, int rows, co
   Carve cv(ws, ws_bytes);
   GemmScratch s = scratch_from(cv);
   uint16_t* hid = cv.take<uint16_t>(size_t(rows) * m->cfg.d_proj);
+  take_acc(cv, s);
   if (!cv.fits()) return fail(SPD_ENOSPC, "project workspace too small");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  SPD_CUDA_TRY(cudaMemsetAsync(s.counters, 0, s.n_counters * sizeof(int), st));
+  if (int rc = gemm_scratch_clear(s, st)) return rc;
   GemmProblem p{};
   p.map_w = &m->m_p1;
   p.w = m->pw1;
@@ -530,6 +547,7 @@ PrefillBufs carve_prefill(const spd_model_cfg& c, int T, int B, Carve& cv) {
   b.z = cv.take<uint16_t>(size_t(B) * D);
   b.list_ints = list_ints_for(c.n_layers, T, B);
   b.lists = cv.take<int32_t>(b.list_ints);
+  take_acc(cv, b.gs);
   return b;
 }
 
@@ -810,7 +828,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
   for (int l = 0; l < c.n_layers; ++l) plan_layer(P, l, mask ? mask + size_t(l) * T : nullptr, cu, B, T);
   int32_t* dl = bf.lists;
   SPD_CUDA_TRY(cudaMemcpyAsync(dl, P.hl.data(), P.end * sizeof(int32_t), cudaMemcpyHostToDevice, st));
-  SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
+  if (int rc = gemm_scratch_clear(bf.gs, st)) return rc;
   if (int rc = bf16_to_f32_run(x, h, size_t(T) * c.d_model, st)) return rc;
   for (int l = 0; l < c.n_layers; ++l)
     if (int rc = run_layer(m, l, P.ll[l], P, bf, dl, h, T, st)) return rc;
@@ -905,7 +923,7 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
     SPD_CUDA_TRY(cudaMemcpyAsync(ab.text, text.data(), text.size() * sizeof(int32_t),
                                  cudaMemcpyHostToDevice, st));
   SPD_CUDA_TRY(cudaMemsetAsync(ab.s_skip, 0, T * sizeof(float), st));
-  SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
+  if (int rc = gemm_scratch_clear(bf.gs, st)) return rc;
   if (int rc = bf16_to_f32_run(x, h, size_t(T) * D, st)) return rc;
 
   // logit lens of nc candidate tokens (device list): final RMSNorm, then the unembedding in fp32
@@ -1048,7 +1066,7 @@ extern "C" int spd_prefill_kv(const spd_model* m, const uint16_t* x, int T, cons
   for (int l = 0; l < c.n_layers; ++l) plan_layer(P, l, mask ? mask + size_t(l) * T : nullptr, cu, B, T);
   int32_t* dl = bf.lists;
   SPD_CUDA_TRY(cudaMemcpyAsync(dl, P.hl.data(), P.end * sizeof(int32_t), cudaMemcpyHostToDevice, st));
-  SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
+  if (int rc = gemm_scratch_clear(bf.gs, st)) return rc;
   if (int rc = bf16_to_f32_run(x, h, size_t(T) * c.d_model, st)) return rc;
   const size_t layer_rows = size_t(B) * max_len, row = 2 * size_t(c.n_kv_heads) * c.head_dim;
   for (int l = 0; l < c.n_layers; ++l) {
@@ -1096,7 +1114,7 @@ extern "C" int spd_decode(const spd_model* m, const uint16_t* x, int B, const in
   for (int l = 0; l < c.n_layers; ++l) plan_layer(P, l, nullptr, cu.data(), B, B);
   int32_t* dl = bf.lists;
   SPD_CUDA_TRY(cudaMemcpyAsync(dl, P.hl.data(), P.end * sizeof(int32_t), cudaMemcpyHostToDevice, st));
-  SPD_CUDA_TRY(cudaMemsetAsync(bf.gs.counters, 0, bf.gs.n_counters * sizeof(int), st));
+  if (int rc = gemm_scratch_clear(bf.gs, st)) return rc;
   if (int rc = bf16_to_f32_run(x, h, size_t(B) * c.d_model, st)) return rc;
   const size_t layer_rows = size_t(B) * max_len, row = 2 * size_t(c.n_kv_heads) * c.head_dim;
   for (int l = 0; l < c.n_layers; ++l) {

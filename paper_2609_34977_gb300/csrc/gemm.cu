@@ -54,6 +54,7 @@
 #include <cooperative_groups.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 
 #include "internal.h"
@@ -96,6 +97,9 @@ struct KArgs {
   int* counters;
   int* status;
   long long budget;
+  int determ;                 // deterministic mode: every output element summed in a fixed order
+  int dpr, rem_tiles, whole;  // data-parallel + remainder schedule (seg_plan_dpr)
+  float* acc;                 // dpr: fp32 accumulation buffers of the remainder tiles (zero at start)
   int vec_red;  // residual epilogue: 16-byte reductions (n_out, ldo multiples of 4, out aligned)
   int staged;  // rotary epilogues: the last whole segment of a CTA goes out through shared memory
   const float* norm_h;  // matrix-vector path: input RMSNorm (see GemmProblem)
@@ -109,6 +113,28 @@ __device__ __forceinline__ float warp_sum_f(float v) {
 #pragma unroll
   for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
   return v;
+}
+
+// 4 x 4 transposes inside each lane quad of a warp: lane k of a quad holds values v[j] of row n0 + k
+// (n0 = 4 (lane / 4)) for columns j = 0..7; afterwards w[4 b + c] = value of row n0 + c, column
+// 4 b + k (b = 0, 1), so that the lane owns four consecutive rows of two columns.
+__device__ __forceinline__ void quad_transpose8(const float (&v)[8], float (&w)[8], int lane) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) w[j] = v[j];
+  const int k = lane & 3;
+#pragma unroll
+  for (int bit = 0; bit < 2; ++bit) {
+    const int m = 1 << bit;
+    const bool hi = (k >> bit) & 1;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (j & m) continue;
+      const float send = hi ? w[j] : w[j + m];
+      const float recv = __shfl_xor_sync(0xffffffffu, send, m);
+      if (hi) w[j] = recv;
+      else w[j + m] = recv;
+    }
+  }
 }
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -129,9 +155,12 @@ __device__ __forceinline__ int cta_of_unit(int u, const KArgs& a) {
 struct SegPlan {
   int u0, u1, n_kb, first_b, last_b, count;
   bool natural, head, tail;
+  bool dpr;                     // data-parallel + remainder schedule (seg_plan_dpr)
+  int n_rsegs, whole0, n_whole;
 };
 __device__ __forceinline__ SegPlan seg_plan(int u0, int u1, int n_kb) {
-  SegPlan p;
+  SegPlan p{};
+  p.dpr = false;
   p.u0 = u0;
   p.u1 = u1;
   p.n_kb = n_kb;
@@ -150,7 +179,36 @@ __device__ __forceinline__ SegPlan seg_plan(int u0, int u1, int n_kb) {
   }
   return p;
 }
+// Data-parallel + remainder schedule: the first rem_tiles tiles are split in K over every work item,
+// item wc owning the remainder units [wc U_r / G, (wc + 1) U_r / G) (U_r = rem_tiles n_kb, G the
+// work items; the contributions of a remainder tile meet in an fp32 accumulation buffer at L2), then
+// the item runs the whole tiles rem_tiles + wc W .. + W - 1, which need no fixup. The remainder
+// comes first, so its fixups overlap the whole tiles' main loops.
+__device__ __forceinline__ SegPlan seg_plan_dpr(int wc, int grid, int rem_tiles, int whole, int n_kb) {
+  SegPlan p{};
+  p.dpr = true;
+  p.n_kb = n_kb;
+  const long long ur = (long long)rem_tiles * n_kb;
+  p.u0 = int(wc * ur / grid);
+  p.u1 = int((wc + 1) * ur / grid);
+  p.n_rsegs = p.u0 < p.u1 ? (p.u1 - 1) / n_kb - p.u0 / n_kb + 1 : 0;
+  p.whole0 = rem_tiles + wc * whole;
+  p.n_whole = whole;
+  p.count = p.n_rsegs + p.n_whole;
+  return p;
+}
 __device__ __forceinline__ void seg_get(const SegPlan& p, int j, int& s, int& e) {
+  if (p.dpr) {
+    if (j < p.n_rsegs) {
+      const int t = p.u0 / p.n_kb + j;
+      s = max(p.u0, t * p.n_kb);
+      e = min(p.u1, (t + 1) * p.n_kb);
+    } else {
+      s = (p.whole0 + j - p.n_rsegs) * p.n_kb;
+      e = s + p.n_kb;
+    }
+    return;
+  }
   if (p.natural) {
     const int te = (p.u0 / p.n_kb + 1) * p.n_kb;
     if (j == 0) {
@@ -305,27 +363,13 @@ __device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane
                                           const int* tpos, int tb) {
   const int nt = a.n_tok;
   if constexpr (EPI == EPI_ADD_F32) {
-    if (a.vec_red) {
+    if (a.vec_red && !a.determ) {
       // 4 x 4 transposes inside each lane quad: lane k of a quad holds columns c0 .. c0 + 3 (c0 =
       // n rounded down to 4) of tokens t0 + k and t0 + 4 + k afterwards, added with two 16-byte
       // reductions instead of eight 4-byte ones (the residual update is bound by L2 atomics)
       float w[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) w[j] = v[j];
+      quad_transpose8(v, w, lane);
       const int k = lane & 3;
-#pragma unroll
-      for (int bit = 0; bit < 2; ++bit) {
-        const int m = 1 << bit;
-        const bool hi = (k >> bit) & 1;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          if (j & m) continue;
-          const float send = hi ? w[j] : w[j + m];
-          const float recv = __shfl_xor_sync(0xffffffffu, send, m);
-          if (hi) w[j] = recv;
-          else w[j + m] = recv;
-        }
-      }
       const int c0 = n & ~3;
       if (c0 < a.n_out) {  // n_out is a multiple of 4: a quad is in or out as a whole
         float* o = static_cast<float*>(a.out);
@@ -349,7 +393,10 @@ __device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane
       const int r = t < nt ? trow[t - tb] : -1;  // negative: a padding row of a device-built list
       if (r >= 0) {
         float* p = o + size_t(r) * a.ldo + n;
-        if constexpr (EPI == EPI_ADD_F32) atomicAdd(p, v[j]);  // fire-and-forget red.add
+        if constexpr (EPI == EPI_ADD_F32) {
+          if (a.determ) *p += v[j];  // the tile's one finalizer: a plain read-modify-write
+          else atomicAdd(p, v[j]);   // fire-and-forget red.add
+        }
         else *p = v[j];
       }
     }
@@ -452,7 +499,11 @@ __device__ __forceinline__ void add4(float (&acc)[8], int o, const float4& x) {
 // even CTA issues the MMAs, each CTA's TMEM holds its 128 rows. Per weight byte that moves 5
 // bytes through shared memory instead of 6 (the token half is read by both tensor cores but
 // written once), the limit of the single-CTA main loop.
-template <int EPI, bool PAIR>
+// DET (residual epilogue only): deterministic mode, split tiles through the ordered partial slots
+// and plain read-modify-writes instead of red.add (a separate instance: the slot fixups would raise
+// the register count of the red.add instance, and with it the registers a co-resident kernel of the
+// programmatic launch chain can get).
+template <int EPI, bool PAIR, bool DET = false>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_sk_kernel(const __grid_constant__ CUtensorMap map_w,
                    const __grid_constant__ CUtensorMap map_x, const KArgs a) {
@@ -486,7 +537,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     u0 = unit_lo(wc, a);
     u1 = unit_lo(wc + 1, a);
   }
-  const SegPlan plan = seg_plan(u0, u1, a.n_kb);
+  const SegPlan plan = a.dpr ? seg_plan_dpr(wc, a.grid, a.rem_tiles, a.whole, a.n_kb)
+                             : seg_plan(u0, u1, a.n_kb);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < a.stages; ++s) {
@@ -723,7 +775,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int h = 0; h < a.nh; ++h)
           stage_copy_out<EPI>(a, (blk0 + h) * kBM, et, tok0, valid, trow,
                               stg + size_t(h) * a.tt * kStgPitch);
-      } else if ((kb_lo == 0 && seg_len == a.n_kb) || EPI == EPI_ADD_F32) {
+      } else if ((kb_lo == 0 && seg_len == a.n_kb) || (EPI == EPI_ADD_F32 && !DET)) {
         for (int h = 0; h < a.nh; ++h) {
 #pragma unroll 1
           for (int cc = half * 8; cc < valid; cc += 16) {
@@ -732,6 +784,50 @@ __global__ void __launch_bounds__(kThreads, 1)
             epilogue8<EPI>(a, (blk0 + h) * kBM + row, q, lane, blk0 + h, tok0 + cc, v, trow, tpos,
                            tok0);
           }
+        }
+      } else if (EPI != EPI_ADD_F32 && a.dpr) {
+        // a remainder tile (dpr schedule): every contributor adds its partial into the tile's fp32
+        // buffer at L2 ([tt tokens][CTA rows], token-major like the residual stream) with 16-byte
+        // reductions after quad transposes; the last to arrive reads the sum, runs the epilogue
+        // and leaves the buffer zero again. The order of the additions is not fixed (fp32 rounding
+        // may differ in the last bits between runs).
+        const int ctr = PAIR ? 2 * tile + prank : tile;
+        const int ar = a.nh * kBM;  // floats per token row of the buffer
+        float* acc = a.acc + size_t(ctr) * ar * a.tt;
+        for (int h = 0; h < a.nh; ++h) {
+#pragma unroll 1
+          for (int cc = half * 8; cc < valid; cc += 16) {
+            float v[8], w[8];
+            tmem_ld8(tq + h * a.hoff + cc, v);
+            quad_transpose8(v, w, lane);
+            const int k = lane & 3, c0 = h * kBM + (row & ~3);
+            red_add_v4(acc + size_t(cc + k) * ar + c0, w[0], w[1], w[2], w[3]);
+            red_add_v4(acc + size_t(cc + 4 + k) * ar + c0, w[4], w[5], w[6], w[7]);
+          }
+        }
+        __threadfence();  // the reductions are performed before the arrival below is seen
+        epi_bar();
+        if (threadIdx.x == 64) {
+          const int old = atomicAdd(&a.counters[ctr], seg_len);
+          flags[1] = (old + seg_len == a.n_kb);
+        }
+        epi_bar();
+        if (flags[1]) {
+          __threadfence();
+          for (int h = 0; h < a.nh; ++h) {
+#pragma unroll 1
+            for (int cc = half * 8; cc < valid; cc += 16) {
+              float* p = acc + size_t(cc) * ar + h * kBM + row;
+              float v[8];
+#pragma unroll
+              for (int jj = 0; jj < 8; ++jj) v[jj] = __ldcg(p + size_t(jj) * ar);
+#pragma unroll
+              for (int jj = 0; jj < 8; ++jj) __stcg(p + size_t(jj) * ar, 0.0f);
+              epilogue8<EPI>(a, (blk0 + h) * kBM + row, q, lane, blk0 + h, tok0 + cc, v, trow, tpos,
+                             tok0);
+            }
+          }
+          if (threadIdx.x == 64) a.counters[ctr] = 0;  // ready for the next launch
         }
       } else {
         // deterministic split tile: partial into this CTA's head (0) or tail (1) slot, laid out
@@ -1041,7 +1137,21 @@ int make_map(CUtensorMap* map, const void* ptr, int inner, int outer, int box_ou
 
 }  // namespace
 
-size_t gemm_scratch_bytes() { return kGemmSlotFloats * sizeof(float) + kCounters * sizeof(int) + 512; }
+int gemm_scratch_clear(const GemmScratch& s, cudaStream_t stream) {
+  SPD_CUDA_TRY(cudaMemsetAsync(s.counters, 0, s.n_counters * sizeof(int), stream));
+  if (s.acc_floats) SPD_CUDA_TRY(cudaMemsetAsync(s.acc, 0, s.acc_floats * sizeof(float), stream));
+  return SPD_OK;
+}
+
+namespace {
+std::atomic<int> g_deterministic{0};
+}
+int deterministic() { return g_deterministic.load(std::memory_order_relaxed); }
+void set_deterministic(int on) { g_deterministic.store(on ? 1 : 0, std::memory_order_relaxed); }
+
+size_t gemm_scratch_bytes() {
+  return (kGemmSlotFloats + kGemmAccFloats) * sizeof(float) + kCounters * sizeof(int) + 768;
+}
 
 int make_weight_map(CUtensorMap* map, const void* w, int n_out, int k) {
   return make_map(map, w, k, n_out, kBM);
@@ -1257,14 +1367,18 @@ KernelFn kernel_for(int epi) {
     case EPI_BF16: return gemm_sk_kernel<EPI_BF16, PAIR>;
     case EPI_BIAS_BF16: return gemm_sk_kernel<EPI_BIAS_BF16, PAIR>;
     case EPI_BIAS_GELU_BF16: return gemm_sk_kernel<EPI_BIAS_GELU_BF16, PAIR>;
-    case EPI_ADD_F32: return gemm_sk_kernel<EPI_ADD_F32, PAIR>;
+    case EPI_ADD_F32: return gemm_sk_kernel<EPI_ADD_F32, PAIR, false>;
     case EPI_ROPE_BF16: return gemm_sk_kernel<EPI_ROPE_BF16, PAIR>;
     case EPI_SWIGLU_BF16: return gemm_sk_kernel<EPI_SWIGLU_BF16, PAIR>;
     case EPI_QKV_BF16: return gemm_sk_kernel<EPI_QKV_BF16, PAIR>;
     default: return nullptr;
   }
 }
-KernelFn kernel_for(int epi, bool pair) { return pair ? kernel_for<true>(epi) : kernel_for<false>(epi); }
+KernelFn kernel_for(int epi, bool pair, bool det = false) {
+  if (det && epi == EPI_ADD_F32)
+    return pair ? gemm_sk_kernel<EPI_ADD_F32, true, true> : gemm_sk_kernel<EPI_ADD_F32, false, true>;
+  return pair ? kernel_for<true>(epi) : kernel_for<false>(epi);
+}
 
 // Sets the shared-memory limit of every instance once; returns the first error.
 cudaError_t set_kernel_attributes() {
@@ -1274,9 +1388,10 @@ cudaError_t set_kernel_attributes() {
     for (int e : {int(EPI_F32), int(EPI_BF16), int(EPI_BIAS_BF16), int(EPI_BIAS_GELU_BF16),
                   int(EPI_ADD_F32), int(EPI_ROPE_BF16), int(EPI_SWIGLU_BF16),
                   int(EPI_QKV_BF16)}) {
-      for (bool pair : {false, true}) {
+      for (int v = 0; v < 4; ++v) {
+        const bool pair = v & 1, det = v & 2;
         const cudaError_t r =
-            cudaFuncSetAttribute(reinterpret_cast<const void*>(kernel_for(e, pair)),
+            cudaFuncSetAttribute(reinterpret_cast<const void*>(kernel_for(e, pair, det)),
                                  cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kSmemPipe + 1024 + 256 + 16384);
         if (r != cudaSuccess && err == cudaSuccess) err = r;
@@ -1385,10 +1500,11 @@ int gemv_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.norm_eps = p.norm_eps;
   a.stamp = gemm_stamp(p);
   a.vec_red = vec_red_ok(p);
+  a.determ = deterministic();
   const int groups = (p.n_out + 31) / 32, C = p.k / kGemvChunk;
   // residual epilogues split K until about two CTAs per SM stream (each at least one chunk column)
   int ksplit = 1;
-  if (p.epi == EPI_ADD_F32)
+  if (p.epi == EPI_ADD_F32 && !a.determ)
     while (groups * ksplit < 2 * num_sms() && ksplit * 2 <= C && ksplit < 8) ksplit *= 2;
   const bool one = p.n_tok == 1;
   const int nt = one ? 1 : kGemvTok;
@@ -1489,7 +1605,8 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   // GPU at once.
   a.csplit = 1;
   a.cluster = 0;
-  if (tiles * 2 <= work_slots && p.epi == EPI_ADD_F32) {
+  a.determ = deterministic();
+  if (tiles * 2 <= work_slots && p.epi == EPI_ADD_F32 && !a.determ) {
     int C = 2;
     while (tiles * C * 2 <= work_slots && C * 4 <= a.n_kb) C *= 2;
     if (C * 2 <= a.n_kb) a.csplit = C;
@@ -1514,8 +1631,27 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   if (size_t(grid) * per_item > s.partial_floats) grid = s.partial_floats / per_item;
   if (grid < 1) grid = 1;
   if (units * (grid + 1) >= (1LL << 31)) return fail(SPD_EUNSUPPORTED, "GEMM too large");
+  // data-parallel + remainder (seg_plan_dpr) instead of stream-K for non-residual epilogues: W
+  // whole tiles per work item, the R leftover tiles split in K over all items, their partial sums
+  // accumulated at L2 (no fp32 partials stored per CTA and read back by one fixup CTA)
+  a.dpr = 0;
+  a.rem_tiles = 0;
+  a.whole = 0;
+  a.acc = s.acc;
+  if (a.csplit == 1 && p.epi != EPI_ADD_F32 && tiles > work_slots && !a.determ) {
+    const long long W = tiles / work_slots, R = tiles - W * work_slots;
+    const size_t acc_need = size_t(R) * tile_rows * a.tt;
+    if (R > 0 && R * a.n_kb >= 2 * work_slots && acc_need <= s.acc_floats) {
+      a.dpr = 1;
+      a.rem_tiles = int(R);
+      a.whole = int(W);
+      grid = work_slots;
+    }
+  }
   if (a.csplit > 1) {
     grid = tiles * a.csplit;
+  } else if (a.dpr) {
+    // grid set above
   } else if (tiles <= work_slots && tiles * 2 > work_slots && a.tt >= 128) {
     // between half and all of the work slots' worth of wide tiles: one whole tile per work item.
     // Stream-K's balance would split most tiles two or three ways, and the fixups of wide token
@@ -1523,7 +1659,7 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
     grid = tiles;
   }
   a.grid = int(grid);
-  const KernelFn kern = kernel_for(p.epi, pair);
+  const KernelFn kern = kernel_for(p.epi, pair, a.determ);
   a.out = p.out;
   a.ldo = p.ldo;
   a.out2 = p.out2;

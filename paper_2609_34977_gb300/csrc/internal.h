@@ -119,13 +119,26 @@ bool gemm_fuses_norm(const GemmProblem& p);
 // Scratch of stream-K partial slots (fp32, two per CTA) and per-tile arrival counters. The counters
 // must be zero before a GEMM runs; every GEMM leaves them zero again when it completes.
 constexpr size_t kGemmSlotFloats = size_t(10) << 20;
+// Accumulation buffers of the data-parallel + remainder schedule: zero when a GEMM starts, left
+// zero by every GEMM.
+constexpr size_t kGemmAccFloats = size_t(4) << 20;
 struct GemmScratch {
-  float* partial;
+  float* partial;     // stream-K partial slots
   size_t partial_floats;
+  float* acc;         // accumulation buffers (null: none)
+  size_t acc_floats;
   int* counters;
   int n_counters;
   int* status;
 };
+// Clears the tile counters and the accumulation buffers of a workspace scratch on `stream` (done
+// once per entry-point call, before its first GEMM).
+int gemm_scratch_clear(const GemmScratch& s, cudaStream_t stream);
+// Deterministic mode (process-wide): GEMMs sum every output element in a fixed order (split tiles
+// through per-CTA partial slots summed in CTA order, residual updates as one read-modify-write per
+// element) instead of fire-and-forget L2 reductions; repeated runs are then bit-identical.
+int deterministic();
+void set_deterministic(int on);
 
 size_t gemm_scratch_bytes();                           // fixed-capacity scratch for any problem
 int make_weight_map(CUtensorMap* map, const void* w, int n_out, int k);

@@ -84,24 +84,29 @@ def test_linear_split_tiles_are_deterministic():
     (200, 4096, 4096, N.EPI_ADD_F32),   # CTA pairs, split-K with red.add
     (160, 11008, 4096, N.EPI_ADD_F32),  # CTA pairs, split-K, long K
 ])
-def test_linear_cta_pairs(M, K, N_, epi):
+@pytest.mark.parametrize("determ", [0, 1])
+def test_linear_cta_pairs(M, K, N_, epi, determ):
     X, W = operands(M, K, N_, seed=M + K)
     ref = bf16_np(X) @ bf16_np(W).T
     ws = torch.zeros(N.spd_linear_workspace_size(M, N_), dtype=torch.uint8, device="cuda")
     h0 = torch.randn(M, N_, device="cuda") if epi == N.EPI_ADD_F32 else torch.zeros(M, N_, device="cuda")
     outs = []
-    for _ in range(2):
-        out = h0.clone() if epi == N.EPI_ADD_F32 else torch.full((M, N_), float("nan"), device="cuda")
-        N.spd_linear(X.cuda(), M, K, W.cuda(), N_, epi, out, N_, ws)
-        torch.cuda.synchronize()
-        assert N.spd_workspace_status(ws) == 0
-        outs.append(out)
+    N.spd_set_deterministic(determ)
+    try:
+        for _ in range(2):
+            out = h0.clone() if epi == N.EPI_ADD_F32 else torch.full((M, N_), float("nan"), device="cuda")
+            N.spd_linear(X.cuda(), M, K, W.cuda(), N_, epi, out, N_, ws)
+            torch.cuda.synchronize()
+            assert N.spd_workspace_status(ws) == 0
+            outs.append(out)
+    finally:
+        N.spd_set_deterministic(0)
     want = ref + (h0.cpu().double().numpy() if epi == N.EPI_ADD_F32 else 0.0)
     for out in outs:
         got = out.cpu().numpy()
         assert np.isfinite(got).all()
         assert rowwise_rel(got, want) < 1e-4
-    if epi == N.EPI_F32:  # split tiles are summed in CTA order: bit-identical runs
+    if determ:  # every element summed in a fixed order: bit-identical runs
         assert torch.equal(outs[0], outs[1])
 
 

@@ -114,3 +114,39 @@ def test_llava_width_spider_step_repeated_with_overlap():
             lgs.append(logits.cpu().numpy())
         assert N.spd_workspace_status(ws) == 0
         _check_repeats(hs, lgs, h_a, lg_a)
+
+
+def test_deterministic_mode_gives_bit_identical_prefills():
+    # spd_set_deterministic(1): every GEMM sums in a fixed order (partial slots in CTA order, one
+    # read-modify-write per residual element): repeated prefills agree bit for bit, and with the
+    # oracle as in the default mode. Two LLaVA-width layers with a skip plan on the visual tokens
+    # (fused QKV over 256 tokens, pair tiles split over K, the residual GEMMs' split tiles).
+    cfg = dict(n_layers=2, d_model=4096, n_heads=32, n_kv_heads=32, head_dim=128, d_ffn=11008,
+               vocab=1000, rope_theta=1e4, rms_eps=1e-5, d_vis=0, d_proj=0)
+    w = synth.decoder_weights(41, cfg, std=0.02, device="cuda")
+    model = N.SpdModel(cfg, w)
+    om = od.model_from_torch(w, cfg)
+    T = 256
+    x = torch.randn(T, 4096, generator=torch.Generator().manual_seed(42)).to(torch.bfloat16)
+    r = np.random.default_rng(43)
+    mask = np.zeros((2, T), np.uint8)
+    mask[:, :192] = r.integers(0, 4, size=(2, 192))
+    ws = torch.zeros(N.spd_prefill_workspace_size(model, T, 1), dtype=torch.uint8, device="cuda")
+    xd = x.cuda()
+    outs = []
+    N.spd_set_deterministic(1)
+    try:
+        for _ in range(5):
+            h = torch.full((T, 4096), float("nan"), device="cuda")
+            lg = torch.full((1, 1000), float("nan"), device="cuda")
+            N.spd_prefill(model, xd, T, [0, T], mask, h, lg, ws)
+            outs.append((h, lg))
+        torch.cuda.synchronize()
+        assert N.spd_workspace_status(ws) == 0
+    finally:
+        N.spd_set_deterministic(0)
+    for h, lg in outs[1:]:
+        assert torch.equal(h, outs[0][0]) and torch.equal(lg, outs[0][1])
+    h0, lg0 = od.prefill(om, bf16_np(x), [0, T], mask)
+    assert rowwise_rel(outs[0][0].cpu().numpy(), h0) < TOL
+    assert rowwise_rel(outs[0][1].cpu().numpy(), lg0) < TOL
