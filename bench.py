@@ -43,6 +43,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--keep", type=int, default=192)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true", help="skip the other workload shapes")
+    ap.add_argument("--sweep", action="store_true", help="the whole serving-sweep grid (batch up to 64)")
     ap.add_argument("--layers", type=int, default=32,
                     help="decoder layers (profiling captures only; the benchmark is 32)")
     return ap.parse_args()
@@ -310,6 +312,181 @@ def decode_steps(torch, N, spider, mask, dev, steps, warmup, hbm, max_len=512):
     return {"ms_per_token": ms, "tokens_per_s": 1000.0 / ms, "context": pos, "GB/s": gbs,
             "hbm_frac": gbs / hbm, "kernels": per,
             "what": "spd_decode, batch 1, after spd_prefill_kv of the SPIDER sequence (pruned, skip plan)"}
+
+
+def _time_calls(torch, fn, steps, warmup):
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(steps):
+        fn()
+    e.record()
+    torch.cuda.synchronize()
+    return s.elapsed_time(e) / steps
+
+
+def _pool_tiles(torch, synth, seed, n_pool, n_patch, d, n_layers, n_heads, has_cls=True, attn_form=0):
+    """A pool of seeded vision tiles on the device (requests draw their tiles from it)."""
+    v = synth.vision_tiles(seed, n_pool, n_patch, d, n_layers, n_heads, has_cls=has_cls, attn_form=attn_form)
+    return [torch.from_numpy(f).cuda() for f in v["feats"]], torch.from_numpy(v["attn"]).cuda()
+
+
+def tiled_workload(torch, N, synth, flops, model, name, tiles_per_req, text_lens, keep, skip_frac, targets,
+                   steps, warmup, seed, dense_ms=None, pool=None, n_patch=N_PATCH, d_vis=D_VIS, heads=H_VIS):
+    """SPIDER step (and, unless dense_ms is given, the dense step on the same kernels) of a batch of
+    requests with tiles_per_req[b] LLaVA tiles and text_lens[b] text tokens; tiles drawn from a pool
+    of 16 seeded tiles. Tokens counted: every original patch plus the text tokens."""
+    from paper_2609_34977_gb300.pipeline import SpiderPrefill
+    cfg = model.cfg
+    L = cfg["n_layers"]
+    n_tiles = int(sum(tiles_per_req))
+    if pool is None:
+        pool = _pool_tiles(torch, synth, seed, 16, n_patch, d_vis, 2, heads)
+    idx = torch.arange(n_tiles, device="cuda") % pool[1].shape[0]
+    feats = [f.index_select(0, idx).contiguous() for f in pool[0]]
+    attn = pool[1].index_select(0, idx).contiguous()
+    n_text = int(sum(text_lens))
+    text = torch.randn(n_text, cfg["d_model"], device="cuda").to(torch.bfloat16)
+    kw = dict(n_patch=n_patch, has_cls=True, d_vis=d_vis, n_feat_layers=2, final_layer=1, n_heads_vis=heads,
+              attn_form=0, tiles_per_req=tiles_per_req, text_lens=text_lens)
+    sp = SpiderPrefill(model, keep=keep, **kw)
+    admit, target = synth.adaptive_plan(seed, L, sp.token_is_visual, skip_frac, targets[:L], ADMIT_LO, L // 2)
+    mask = N.spd_plan_adaptive(L, admit, target)
+    ms = _time_calls(torch, lambda: sp.run(feats, attn, text, mask), steps, warmup)
+    assert sp.status() == 0, "device-side failure recorded"
+    seqs = [int(sp.cu[b + 1] - sp.cu[b]) for b in range(sp.B)]
+    w = flops.prefill_work(cfg, seqs, mask, n_proj_rows=n_tiles * keep)
+    del sp
+    if dense_ms is None:
+        dp = SpiderPrefill(model, keep=n_patch, dense=True, **kw)
+        dense_ms = _time_calls(torch, lambda: dp.run(feats, attn, text, None), max(2, steps // 2), 1)
+        del dp
+    torch.cuda.empty_cache()
+    tokens = n_tiles * n_patch + n_text
+    vanilla = sum(flops.paper_prefill_flops(tiles_per_req[b] * n_patch + text_lens[b], L, cfg["d_model"],
+                                            cfg["d_ffn"]) for b in range(len(text_lens)))
+    kept = sum(flops.paper_prefill_flops(tiles_per_req[b] * keep + text_lens[b], L, cfg["d_model"], cfg["d_ffn"])
+               for b in range(len(text_lens)))
+    return {"workload": name, "batch": len(text_lens), "tiles": n_tiles, "keep_per_tile": keep,
+            "text_tokens": n_text, "decoder_tokens": int(sum(seqs)), "visual_skip_fraction": skip_frac,
+            "ms_per_step": ms, "tokens_per_s": tokens / (ms / 1e3), "dense_ms_per_step": dense_ms,
+            "dense_tokens_per_s": tokens / (dense_ms / 1e3), "speedup_vs_dense": dense_ms / ms,
+            "decoder_flops_executed": w["gemm_flops"] + w["attn_flops"],
+            "paper_flops_vanilla": vanilla, "paper_flops_pruned_no_skip": kept}, dense_ms
+
+
+def varres_workload(torch, N, synth, flops, model, name, n_patches, text_lens, keep_ratio, skip_frac,
+                    targets, steps, warmup, seed, d_vis=1280, heads=16):
+    """Qwen2-style dynamic resolution: one image of n_patches[b] post-merger tokens per request
+    (no [CLS]: received-attention form), MSV-Prune to keep_ratio of them, projector d_vis -> D -> D,
+    the GQA decoder; and the dense step."""
+    from paper_2609_34977_gb300.pipeline import VarResSpiderPrefill
+    cfg = model.cfg
+    L = cfg["n_layers"]
+    feats, attn = [], []
+    for b, n in enumerate(n_patches):
+        f, a = _pool_tiles(torch, synth, seed + b, 1, n, d_vis, 2, heads, has_cls=False, attn_form=1)
+        feats.append(f)
+        attn.append(a)
+    n_text = int(sum(text_lens))
+    text = torch.randn(n_text, cfg["d_model"], device="cuda").to(torch.bfloat16)
+    kw = dict(n_patches=n_patches, d_vis=d_vis, n_feat_layers=2, final_layer=1, n_heads_vis=heads,
+              keep_ratio=keep_ratio, text_lens=text_lens)
+    sp = VarResSpiderPrefill(model, **kw)
+    admit, target = synth.adaptive_plan(seed, L, sp.token_is_visual, skip_frac, targets[:L], ADMIT_LO, L // 2)
+    mask = N.spd_plan_adaptive(L, admit, target)
+    ms = _time_calls(torch, lambda: sp.run(feats, attn, text, mask), steps, warmup)
+    assert sp.status() == 0, "device-side failure recorded"
+    seqs = [int(sp.cu[b + 1] - sp.cu[b]) for b in range(sp.B)]
+    w = flops.prefill_work(cfg, seqs, mask, n_proj_rows=int(sum(sp.keeps)))
+    del sp
+    dp = VarResSpiderPrefill(model, dense=True, **kw)
+    dense_ms = _time_calls(torch, lambda: dp.run(feats, attn, text, None), max(2, steps // 2), 1)
+    dense_T = dp.T
+    del dp
+    torch.cuda.empty_cache()
+    tokens = int(sum(n_patches)) + n_text
+    return {"workload": name, "batch": len(text_lens), "image_tokens": [int(n) for n in n_patches],
+            "keep_ratio": keep_ratio, "text_tokens": n_text, "decoder_tokens": int(sum(seqs)),
+            "dense_decoder_tokens": dense_T, "visual_skip_fraction": skip_frac,
+            "ms_per_step": ms, "tokens_per_s": tokens / (ms / 1e3), "dense_ms_per_step": dense_ms,
+            "dense_tokens_per_s": tokens / (dense_ms / 1e3), "speedup_vs_dense": dense_ms / ms,
+            "decoder_flops_executed": w["gemm_flops"] + w["attn_flops"]}
+
+
+def other_workloads(torch, N, synth, llava_model, dense_llava_ms, steps, warmup, full_sweep=False):
+    """The other workload shapes of the benchmark: LLaVA-1.5 keep 128 / 64, LLaVA-NeXT (5 crops,
+    keep 320 / 160 and the paper's N = 710 point, batch 1 and 8), the Qwen2-style GQA decoder (batch
+    4, dynamic resolution 1024-4096 tokens, keep 0.25) and a serving sweep over batch size, keep
+    ratio and skip fraction (a subset by default; --sweep runs the whole grid)."""
+    from paper_2609_34977_gb300 import flops
+    st, wu = max(3, steps // 4), 2
+    out = {}
+    m15 = synth.skip_targets("llava-1.5-7b")
+    mnx = synth.skip_targets("llava-next-7b")
+    pool = _pool_tiles(torch, synth, SEED + 11, 16, N_PATCH, D_VIS, 2, H_VIS)
+    res = []
+    for keep in (128, 64):
+        r, _ = tiled_workload(torch, N, synth, flops, llava_model, f"llava-1.5-7b keep {keep}", [1], [TEXT],
+                              keep, SKIP_FRAC, m15, st, wu, SEED + keep, dense_ms=dense_llava_ms, pool=pool)
+        res.append(r)
+    out["llava15_keep128_64"] = res
+    res = []
+    for B in (1, 8):
+        dense_ms = None
+        for keep, frac in ((64, SKIP_FRAC), (32, SKIP_FRAC), (142, 0.3)):
+            if B == 8 and keep != 64:
+                continue
+            r, dense_ms = tiled_workload(torch, N, synth, flops, llava_model,
+                                         f"llava-next-7b shape: {B} x 5 crops, keep {5 * keep}", [5] * B, [128] * B,
+                                         keep, frac, mnx, st, wu, SEED + 100 + keep, dense_ms=dense_ms, pool=pool)
+            res.append(r)
+    out["llava_next"] = res
+    # serving sweep: batch x keep per tile x skip fraction, tiles per request U{1..5}, text U[32, 512]
+    r = np.random.default_rng(SEED + 7)
+    Bs = (1, 2, 4, 8, 16, 32, 64) if full_sweep else (1, 8)
+    keeps = (64, 128, 192) if full_sweep else (64, 192)
+    fracs = (0.0, 0.25, 0.5) if full_sweep else (0.25,)
+    sweep = []
+    for B in Bs:
+        tiles = [int(x) for x in r.integers(1, 6, size=B)]
+        texts = [int(x) for x in r.integers(32, 513, size=B)]
+        dense_ms = None
+        for keep in keeps:
+            for frac in fracs:
+                rr, dense_ms = tiled_workload(torch, N, synth, flops, llava_model, "serving sweep, llava-1.5-7b",
+                                              tiles, texts, keep, frac, m15, st, wu, SEED + B, dense_ms=dense_ms,
+                                              pool=pool)
+                sweep.append({k: rr[k] for k in ("batch", "tiles", "keep_per_tile", "visual_skip_fraction",
+                                                  "decoder_tokens", "ms_per_step", "tokens_per_s",
+                                                  "dense_ms_per_step", "speedup_vs_dense")})
+    out["serving_sweep"] = {"points": sweep, "grid": "full" if full_sweep else "subset (--sweep for the full grid)",
+                            "keep_ratio_per_tile": {64: 0.11, 128: 0.22, 192: 0.33}}
+    del pool
+    torch.cuda.empty_cache()
+    return out
+
+
+def qwen_workload(torch, N, synth, steps, warmup):
+    """Qwen2-style GQA decoder (28 layers, 3584, 28 query / 4 KV heads, FFN 18944, vocab 152064,
+    projector 1280 -> 3584 -> 3584), batch 4 with seeded image sizes in [1024, 4096]."""
+    from paper_2609_34977_gb300 import flops
+    cfg = dict(synth.QWEN2_DECODER)
+    w = synth.decoder_weights(SEED + 3, cfg, device="cuda")
+    model = N.SpdModel(cfg, w)
+    del w
+    torch.cuda.empty_cache()
+    r = np.random.default_rng(SEED + 5)
+    n_patches = [int(x) for x in r.integers(1024, 4097, size=4)]
+    out = varres_workload(torch, N, synth, flops, model, "qwen2-gqa shape, batch 4", n_patches, [256] * 4, 0.25,
+                          SKIP_FRAC, synth.seeded_skip_targets(SEED, cfg["n_layers"]), max(3, steps // 4), 2,
+                          SEED + 9)
+    model.close()
+    torch.cuda.empty_cache()
+    return out
+
 
 
 def cpu_step_setup(keep, v, mask_fn):
@@ -581,6 +758,15 @@ def main():
     ra["peaks"] = ("hbm_frac: of the copy peak (MEASURED_PEAKS.json, read + write); frac_of_read_peak: "
                    "of a read-only stream measured in this run (torch sum over 2 GiB)")
     dec = decode_steps(torch, N, spider, mask, dev, a.steps, a.warmup, hbm)
+    # deterministic mode: the same step with every GEMM summed in a fixed order
+    N.spd_set_deterministic(1)
+    ms_det = timed(spider, mask, a.steps, a.warmup)
+    N.spd_set_deterministic(0)
+    determ = {"ms_per_step": ms_det, "cost_over_default": ms_det / ms,
+              "what": "spd_set_deterministic(1): ordered partial sums, read-modify-write residual updates"}
+    work = None
+    if not a.no_workloads and L == 32:
+        work = other_workloads(torch, N, synth, model, ms_dense, a.steps, a.warmup, a.sweep)
 
     # end to end through the public API: pinned host inputs -> device, step, logits -> host
     hf = [f.cpu().pin_memory() for f in feats]
@@ -604,6 +790,9 @@ def main():
     ms_e2e = s.elapsed_time(e) / a.steps
     h2d = sum(t.numel() * t.element_size() for t in hf + [ha, ht])
 
+    if work is not None:
+        work["qwen2_gqa"] = qwen_workload(torch, N, synth, a.steps, a.warmup)
+
     cpu = None
     if rank == 0 and not a.no_cpu_baseline:
         from oracle import decoder as od
@@ -626,6 +815,7 @@ def main():
                               "tokens_per_s": spider.T * world / (ms / 1000.0)},
                 "roofline": roof, "kernels": kernels, "dense_gemm": dense_gemm,
                 "prune_batch": pb, "received_attention": ra, "adaptive_plan": adaptive, "decode": dec,
+                "deterministic": determ, "workloads": work,
                 "cpu_baseline": cpu,
                 "e2e": {"value": tokens / (ms_e2e / 1000.0), "unit": "tokens/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": hl.numel() * 4,

@@ -132,3 +132,81 @@ class SpiderPrefill:
         codes = [N.spd_workspace_status(w) for w in (self.ws_prune, self.ws_proj, self.ws_prefill,
                                                      self.ws_adaptive) if w is not None]
         return next((c for c in codes if c), 0)
+
+
+class VarResSpiderPrefill:
+    """One image per request with its own token count (dynamic resolution, e.g. the Qwen2-VL
+    encoder after its 2 x 2 patch merger: no [CLS] token, so the received-attention form of
+    Sec. 4.1.1), pruned to round(keep_ratio * n_i) tokens each; then the projector, the sequence
+    assembly [visual; text] per request and the decoder prefill, as in SpiderPrefill.
+
+    n_patches[b] tokens in image b (its own spd_prune call); dense=True keeps every token."""
+
+    def __init__(self, model: N.SpdModel, *, n_patches, d_vis: int, n_feat_layers: int,
+                 final_layer: int, n_heads_vis: int, keep_ratio: float, text_lens,
+                 n_clusters: int = 4, kmeans_iters: int = 10, anchor_ratio: float = 0.7,
+                 dense: bool = False, device: str = "cuda"):
+        self.model = model
+        cfg = model.cfg
+        self.D = cfg["d_model"]
+        self.n_patches = [int(n) for n in n_patches]
+        self.text_lens = list(text_lens)
+        self.B = len(self.n_patches)
+        self.dense = dense
+        self.d_vis = d_vis
+        self.final_layer = final_layer
+        self.keeps = [n if dense else max(1, int(round(keep_ratio * n))) for n in self.n_patches]
+        self.cfgs = [N.prune_cfg(1, n, d_vis, n_feat_layers, final_layer, n_heads_vis, k, has_cls=False,
+                                 attn_form=1, n_clusters=n_clusters, kmeans_iters=kmeans_iters,
+                                 anchor_ratio=anchor_ratio)
+                     for n, k in zip(self.n_patches, self.keeps)]
+        dev = torch.device(device)
+        vis_rows, text_rows, cu = [], [], [0]
+        row = 0
+        for b in range(self.B):
+            vis_rows.extend(range(row, row + self.keeps[b]))
+            row += self.keeps[b]
+            text_rows.extend(range(row, row + self.text_lens[b]))
+            row += self.text_lens[b]
+            cu.append(row)
+        self.T = row
+        self.cu = np.array(cu, dtype=np.int32)
+        self.token_is_visual = np.zeros(self.T, dtype=bool)
+        self.token_is_visual[vis_rows] = True
+        self.vis_rows = torch.tensor(vis_rows, dtype=torch.int32, device=dev)
+        self.text_rows = torch.tensor(text_rows, dtype=torch.int32, device=dev)
+        self.keep_idx = [torch.arange(k, dtype=torch.int32, device=dev) if dense else
+                         torch.empty(k, dtype=torch.int32, device=dev) for k in self.keeps]
+        nv = sum(self.keeps)
+        self.vis = torch.empty(nv, d_vis, dtype=torch.bfloat16, device=dev)
+        self.x = torch.empty(self.T, self.D, dtype=torch.bfloat16, device=dev)
+        self.h = torch.empty(self.T, self.D, dtype=torch.float32, device=dev)
+        self.logits = torch.empty(self.B, cfg["vocab"], dtype=torch.float32, device=dev)
+        ws = max(N.spd_prune_workspace_size(c) for c in self.cfgs)
+        self.ws_prune = torch.zeros(ws, dtype=torch.uint8, device=dev)
+        self.ws_proj = torch.zeros(N.spd_project_workspace_size(model, nv), dtype=torch.uint8, device=dev)
+        self.ws_prefill = torch.zeros(N.spd_prefill_workspace_size(model, self.T, self.B), dtype=torch.uint8,
+                                      device=dev)
+
+    def run(self, feats, attn, text, skip_mask, stream=None):
+        """feats[b]: list of [1][n_b][d_vis] fp32 per tapped layer, attn[b]: [1][H][n_b] received
+        attention, text [sum(text_lens)][D] bf16. Returns the logits [B][vocab] (device)."""
+        off = 0
+        for b in range(self.B):
+            k = self.keeps[b]
+            if not self.dense:
+                N.spd_prune(self.cfgs[b], feats[b], attn[b], self.keep_idx[b], ws=self.ws_prune, stream=stream)
+            N.spd_gather_rows_bf16(feats[b][self.final_layer], 1, self.n_patches[b], self.d_vis, 0,
+                                   self.keep_idx[b], k, self.vis[off:off + k], ws=self.ws_prune,
+                                   stream=stream)
+            off += k
+        N.spd_project(self.model, self.vis, off, self.vis_rows, self.x, self.ws_proj, stream=stream)
+        if len(self.text_rows):
+            N.spd_scatter_rows(self.model, text, len(self.text_rows), self.text_rows, self.x, stream=stream)
+        N.spd_prefill(self.model, self.x, self.T, self.cu, skip_mask, self.h, self.logits, self.ws_prefill,
+                      stream=stream)
+        return self.logits
+
+    def status(self) -> int:
+        codes = [N.spd_workspace_status(w) for w in (self.ws_prune, self.ws_proj, self.ws_prefill)]
+        return next((c for c in codes if c), 0)

@@ -213,3 +213,39 @@ def test_gather_contract_form_equals_gather_rows():
     assert torch.equal(a, b)
     want = torch.from_numpy(v["feats"][1]).cuda()[torch.arange(3).repeat_interleave(64).cuda(), 1 + idx.flatten().long()]
     assert torch.equal(a, want.to(torch.bfloat16))
+
+
+def test_largest_accepted_tile_received_form_with_guard_bands():
+    # the top of the accepted range: n = 4096 post-merger tokens of width 1280 (the Qwen2-VL
+    # encoder after its patch merger, received-attention form), keep 0.25 n; its K-means runs the
+    # L2-streaming 8-CTA form. Seed 20260940: the first from 20260901 on whose tile every decision
+    # of the oracle has a margin above 1e-3 (few have, at 845 tokens a cluster). Every output sits
+    # between guard bands of canary values that must come back untouched.
+    seed, v, res = conditioned_vision(20260940, 1, 4096, 1280, 2, 16, 1024, 1, has_cls=False,
+                                      attn_form=1, tries=1)
+    feats = [torch.from_numpy(f).cuda() for f in v["feats"]]
+    attn = torch.from_numpy(v["attn"]).cuda()
+    cfg = N.prune_cfg(1, 4096, 1280, 2, 1, 16, 1024, has_cls=False, attn_form=1)
+    ws = torch.zeros(N.spd_prune_workspace_size(cfg), dtype=torch.uint8, device="cuda")
+    G = 256  # guard elements before and after every output
+    keep_b = torch.full((G + 1024 + G,), -7, dtype=torch.int32, device="cuda")
+    kind_b = torch.full((G + 4096 + G,), 9, dtype=torch.uint8, device="cuda")
+    clus_b = torch.full((G + 4096 + G,), 99, dtype=torch.int8, device="cuda")
+    score_b = torch.full((G + 4096 + G,), -1234.5, dtype=torch.float32, device="cuda")
+    N.spd_prune(cfg, feats, attn, keep_b[G:G + 1024], kind_b[G:G + 4096], clus_b[G:G + 4096],
+                score_b[G:G + 4096], ws=ws)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    for buf, n, canary in ((keep_b, 1024, -7), (kind_b, 4096, 9), (clus_b, 4096, 99), (score_b, 4096, -1234.5)):
+        assert torch.all(buf[:G] == canary) and torch.all(buf[G + n:] == canary)
+    g = dict(keep_idx=keep_b[G:G + 1024].cpu().numpy()[None], kind=kind_b[G:G + 4096].cpu().numpy()[None],
+             cluster=clus_b[G:G + 4096].cpu().numpy()[None], scores=score_b[G:G + 4096].cpu().numpy()[None])
+    assert_prune_parity(g, res)
+    # the gather of the kept rows (the projector's input) between guard rows
+    out_b = torch.full((1024 + 2, 1280), 3.0, dtype=torch.bfloat16, device="cuda")
+    N.spd_gather_rows_bf16(feats[1], 1, 4096, 1280, 0, keep_b[G:G + 1024], 1024, out_b[1:1025], ws=ws)
+    torch.cuda.synchronize()
+    assert N.spd_workspace_status(ws) == 0
+    assert torch.all(out_b[0] == 3.0) and torch.all(out_b[1025] == 3.0)
+    want = torch.from_numpy(v["feats"][1][0][res[0]["keep_idx"]]).to(torch.bfloat16)
+    assert torch.equal(out_b[1:1025].cpu(), want)
