@@ -1641,7 +1641,9 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   if (a.csplit == 1 && p.epi != EPI_ADD_F32 && tiles > work_slots && !a.determ) {
     const long long W = tiles / work_slots, R = tiles - W * work_slots;
     const size_t acc_need = size_t(R) * tile_rows * a.tt;
-    if (R > 0 && R * a.n_kb >= 2 * work_slots && acc_need <= s.acc_floats) {
+    // only a thin remainder (each item's share at most a quarter of a tile's k-blocks): with more,
+    // stream-K's ordered fixups beat the L2 reductions (measured on the dense LLaVA step)
+    if (R > 0 && R * 4 <= work_slots && R * a.n_kb >= 2 * work_slots && acc_need <= s.acc_floats) {
       a.dpr = 1;
       a.rem_tiles = int(R);
       a.whole = int(W);
