@@ -27,12 +27,36 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 }
 
 // out[orow(i)] = bf16(gain * h[irow(i)] / sqrt(mean(h^2) + eps)); out2[map2[irow]] gets the same
-// row when map2 is given and map2[irow] >= 0 (compact copy of the attention-active rows).
+// row when map2 is given and map2[irow] >= 0 (compact copy of the attention-active rows). Rows of
+// up to kRowVec * 4 * kThreads floats stay in registers between the sum of squares and the scaling
+// (one pass over the row); the gains (weights) are loaded before the grid dependency wait.
+constexpr int kRowVec = 4;
+__device__ __forceinline__ uint2 norm_pack(const float4& v, const ushort4& gg, float inv) {
+  const __nv_bfloat162 lo = __floats2bfloat162_rn(
+      v.x * inv * __bfloat162float(__ushort_as_bfloat16(gg.x)),
+      v.y * inv * __bfloat162float(__ushort_as_bfloat16(gg.y)));
+  const __nv_bfloat162 hi = __floats2bfloat162_rn(
+      v.z * inv * __bfloat162float(__ushort_as_bfloat16(gg.z)),
+      v.w * inv * __bfloat162float(__ushort_as_bfloat16(gg.w)));
+  return make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+}
+
 __global__ void __launch_bounds__(kThreads)
     rmsnorm_kernel(const float* h, int D, const uint16_t* __restrict__ gain, float eps,
                    const int32_t* in_rows, __nv_bfloat16* __restrict__ out, const int32_t* map2,
                    __nv_bfloat16* __restrict__ out2, unsigned long long* stamp) {
   __shared__ float red[kThreads / 32];
+  const int n4 = D / 4;
+  const bool in_regs = n4 <= kRowVec * kThreads;
+  const ushort4* g4 = reinterpret_cast<const ushort4*>(gain);
+  ushort4 gr[kRowVec];
+  if (in_regs) {
+#pragma unroll
+    for (int k = 0; k < kRowVec; ++k) {
+      const int c = threadIdx.x + k * kThreads;
+      if (c < n4) gr[k] = g4[c];
+    }
+  }
   pdl_launch_dependents();
   pdl_wait();
   if (threadIdx.x == 0) stamp_start(stamp);
@@ -40,30 +64,41 @@ __global__ void __launch_bounds__(kThreads)
   const int r = in_rows ? in_rows[i] : i;
   if (r < 0) return;  // a padding entry of a device-built row list
   const float4* src = reinterpret_cast<const float4*>(h + size_t(r) * D);
-  const int n4 = D / 4;
-  float ss = 0.0f;
-  for (int c = threadIdx.x; c < n4; c += kThreads) {
-    const float4 v = src[c];
-    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
-  }
-  const float tot = block_sum(ss, red);
-  const float inv = rsqrtf(tot / float(D) + eps);
   const int r2 = map2 ? map2[r] : -1;
-  const ushort4* g4 = reinterpret_cast<const ushort4*>(gain);
-  for (int c = threadIdx.x; c < n4; c += kThreads) {
-    const float4 v = src[c];
-    const ushort4 gg = g4[c];
-    __nv_bfloat162 lo = __floats2bfloat162_rn(
-        v.x * inv * __bfloat162float(__ushort_as_bfloat16(gg.x)),
-        v.y * inv * __bfloat162float(__ushort_as_bfloat16(gg.y)));
-    __nv_bfloat162 hi = __floats2bfloat162_rn(
-        v.z * inv * __bfloat162float(__ushort_as_bfloat16(gg.z)),
-        v.w * inv * __bfloat162float(__ushort_as_bfloat16(gg.w)));
-    uint2 pk;
-    pk.x = *reinterpret_cast<uint32_t*>(&lo);
-    pk.y = *reinterpret_cast<uint32_t*>(&hi);
-    reinterpret_cast<uint2*>(out + size_t(i) * D)[c] = pk;
-    if (r2 >= 0) reinterpret_cast<uint2*>(out2 + size_t(r2) * D)[c] = pk;
+  uint2* o = reinterpret_cast<uint2*>(out + size_t(i) * D);
+  uint2* o2 = r2 >= 0 ? reinterpret_cast<uint2*>(out2 + size_t(r2) * D) : nullptr;
+  float ss = 0.0f;
+  if (in_regs) {
+    float4 vr[kRowVec];
+#pragma unroll
+    for (int k = 0; k < kRowVec; ++k) {
+      const int c = threadIdx.x + k * kThreads;
+      vr[k] = c < n4 ? src[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < kRowVec; ++k)
+      ss += vr[k].x * vr[k].x + vr[k].y * vr[k].y + vr[k].z * vr[k].z + vr[k].w * vr[k].w;
+    const float inv = rsqrtf(block_sum(ss, red) / float(D) + eps);
+#pragma unroll
+    for (int k = 0; k < kRowVec; ++k) {
+      const int c = threadIdx.x + k * kThreads;
+      if (c < n4) {
+        const uint2 pk = norm_pack(vr[k], gr[k], inv);
+        o[c] = pk;
+        if (o2) o2[c] = pk;
+      }
+    }
+  } else {
+    for (int c = threadIdx.x; c < n4; c += kThreads) {
+      const float4 v = src[c];
+      ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+    }
+    const float inv = rsqrtf(block_sum(ss, red) / float(D) + eps);
+    for (int c = threadIdx.x; c < n4; c += kThreads) {
+      const uint2 pk = norm_pack(src[c], g4[c], inv);
+      o[c] = pk;
+      if (o2) o2[c] = pk;
+    }
   }
   if (threadIdx.x == 0) stamp_end(stamp);
 }
