@@ -156,9 +156,17 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
+LM_HEAD_SCALE = 12.0  # the LM head drawn with std 0.24 instead of 0.02 (see build_model)
+
+
 def build_model(torch, N, synth, device, layers=32):
+    """The LLaVA-1.5-7B-shaped decoder with random bf16 weights (std 0.02), except the LM head:
+    std 0.24, so that the logit lens of the online ASL-Skip plan sees peaked vocabulary
+    distributions (entropies that vary between tokens, as trained weights give) instead of nearly
+    uniform ones; no kernel's cost depends on the weights' values."""
     cfg = dict(synth.LLAVA_7B_DECODER, n_layers=layers)
     w = synth.decoder_weights(SEED, cfg, device=device)
+    w["lm_head"] = (w["lm_head"].float() * LM_HEAD_SCALE).to(torch.bfloat16)
     model = N.SpdModel(cfg, w)
     del w
     torch.cuda.empty_cache()

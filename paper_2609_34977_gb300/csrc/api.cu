@@ -838,7 +838,7 @@ extern "C" int spd_prefill(const spd_model* m, const uint16_t* x, int T, const i
 // ---- prefill with the online ASL-Skip plan (Alg. 1 stage 2) -----------------------------------
 namespace {
 struct AdaptiveBufs {
-  float* logits;  // [T][V] vocabulary logits of the candidates
+  float* logits;  // [T][lse_groups(V)] float4 logit-lens statistics of the candidates
   float* tmean;   // [B][D] mean text hidden state per sequence
   float* s_skip;  // [T] accumulated skippability
   uint8_t* flag;  // [T] admitted at this layer (per candidate)
@@ -855,7 +855,7 @@ struct AdaptiveBufs {
 };
 AdaptiveBufs carve_adaptive(const spd_model_cfg& c, int T, int B, Carve& cv) {
   AdaptiveBufs a;
-  a.logits = cv.take<float>(size_t(T) * c.vocab);
+  a.logits = cv.take<float>(size_t(T) * lse_groups(c.vocab) * 4);
   a.tmean = cv.take<float>(size_t(B) * c.d_model);
   a.s_skip = cv.take<float>(T);
   a.flag = cv.take<uint8_t>(T);
@@ -899,7 +899,7 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
   const bool no_slc = pol->ablate & SPD_SKIP_NO_SLC;
   const int mode = ((pol->w1 != 0.0f && !(pol->ablate & SPD_SKIP_NO_ENTROPY)) ? kSkipEntropy : 0) |
                    ((pol->w1 != 0.0f && !(pol->ablate & SPD_SKIP_NO_ITC)) ? kSkipItc : 0) |
-                   ((pol->ablate & SPD_SKIP_NO_ACCUM) ? 0 : kSkipAccumulate);
+                   ((pol->ablate & SPD_SKIP_NO_ACCUM) ? 0 : kSkipAccumulate) | kSkipLse;
   Carve cv(ws, ws_bytes);
   PrefillBufs bf = carve_prefill(c, T, B, cv);
   AdaptiveBufs ab = carve_adaptive(c, T, B, cv);
@@ -926,7 +926,9 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
   if (int rc = gemm_scratch_clear(bf.gs, st)) return rc;
   if (int rc = bf16_to_f32_run(x, h, size_t(T) * D, st)) return rc;
 
-  // logit lens of nc candidate tokens (device list): final RMSNorm, then the unembedding in fp32
+  // logit lens of nc candidate tokens (device list): final RMSNorm, then the unembedding with the
+  // entropy's statistics taken in the GEMM's epilogue (per 32 vocabulary words: max, sum of
+  // exponentials and their weighted sum; the fp32 logits never reach memory)
   auto lens = [&](const int32_t* cand_dev, int nc) -> int {
     if (int rc = rmsnorm_run(h, nc, D, m->final_norm, c.rms_eps, cand_dev, bf.xa, nullptr, nullptr, st))
       return rc;
@@ -937,9 +939,9 @@ extern "C" int spd_prefill_adaptive(const spd_model* m, const uint16_t* x, int T
     up.n_out = c.vocab;
     up.n_tok = nc;
     up.k = D;
-    up.epi = EPI_F32;
+    up.epi = EPI_LSE_F32;
     up.out = ab.logits;
-    up.ldo = c.vocab;
+    up.ldo = lse_groups(c.vocab);
     return gemm_run(up, bf.gs, st);
   };
 

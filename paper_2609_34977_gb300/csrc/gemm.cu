@@ -443,6 +443,35 @@ __device__ __forceinline__ void epilogue8(const KArgs& a, int n, int q, int lane
         }
       }
     }
+  } else if constexpr (EPI == EPI_LSE_F32) {
+    // the statistics of this warp's 32 weight rows (vocabulary words) for each of the 8 tokens:
+    // warp max, then the sums of e^(z - m) and e^(z - m) (z - m); lane j stores token t0 + j's
+    float m8[8], s8[8], u8[8];
+    const bool live = n < a.n_out;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      float m = live ? v[j] : -INFINITY;
+#pragma unroll
+      for (int off = 16; off; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+      const float d = live ? v[j] - m : 0.0f;
+      const float e = live ? __expf(d) : 0.0f;
+      float sj = e, uj = e * d;
+#pragma unroll
+      for (int off = 16; off; off >>= 1) {
+        sj += __shfl_xor_sync(0xffffffffu, sj, off);
+        uj += __shfl_xor_sync(0xffffffffu, uj, off);
+      }
+      m8[j] = m;
+      s8[j] = sj;
+      u8[j] = uj;
+    }
+    float4* o = static_cast<float4*>(a.out);
+    const int g = n >> 5;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int t = t0 + j;
+      if (lane == j && t < nt) o[size_t(t) * a.ldo + g] = make_float4(m8[j], s8[j], u8[j], 0.0f);
+    }
   } else if constexpr (EPI == EPI_SWIGLU_BF16) {
     // lanes l and l + 16 hold gate and up of the same FFN channel f: after one exchange lane l
     // finishes the even tokens of the group and lane l + 16 the odd ones
@@ -1371,6 +1400,7 @@ KernelFn kernel_for(int epi) {
     case EPI_ROPE_BF16: return gemm_sk_kernel<EPI_ROPE_BF16, PAIR>;
     case EPI_SWIGLU_BF16: return gemm_sk_kernel<EPI_SWIGLU_BF16, PAIR>;
     case EPI_QKV_BF16: return gemm_sk_kernel<EPI_QKV_BF16, PAIR>;
+    case EPI_LSE_F32: return gemm_sk_kernel<EPI_LSE_F32, PAIR>;
     default: return nullptr;
   }
 }
@@ -1387,7 +1417,7 @@ cudaError_t set_kernel_attributes() {
   std::call_once(once, [] {
     for (int e : {int(EPI_F32), int(EPI_BF16), int(EPI_BIAS_BF16), int(EPI_BIAS_GELU_BF16),
                   int(EPI_ADD_F32), int(EPI_ROPE_BF16), int(EPI_SWIGLU_BF16),
-                  int(EPI_QKV_BF16)}) {
+                  int(EPI_QKV_BF16), int(EPI_LSE_F32)}) {
       for (int v = 0; v < 4; ++v) {
         const bool pair = v & 1, det = v & 2;
         const cudaError_t r =
@@ -1440,7 +1470,7 @@ namespace {
 void gemm_work(const GemmProblem& p, double* flops, double* bytes) {
   const double cols = (p.epi == EPI_SWIGLU_BF16) ? 2.0 * p.out_cols : double(p.n_out);
   const double out_cols = (p.epi == EPI_SWIGLU_BF16) ? double(p.out_cols) : double(p.n_out);
-  const double ob = (p.epi == EPI_F32) ? 4.0 : (p.epi == EPI_ADD_F32) ? 8.0 : 2.0;
+  const double ob = (p.epi == EPI_F32) ? 4.0 : (p.epi == EPI_ADD_F32) ? 8.0 : (p.epi == EPI_LSE_F32) ? 0.5 : 2.0;
   double tok_cols = double(p.n_tok) * cols, tok_out = double(p.n_tok) * out_cols;
   if (p.epi == EPI_QKV_BF16) {
     tok_cols = double(p.n_tok_out) * p.split + double(p.n_tok) * (p.n_out - p.split);

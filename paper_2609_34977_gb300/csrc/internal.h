@@ -83,9 +83,14 @@ enum Epi : int {
   EPI_ADD_F32 = SPD_EPI_ADD_F32,
   EPI_ROPE_BF16 = 16,  // rotary embedding on weight rows [0, rope_rows) laid out in rotary pairs
   EPI_SWIGLU_BF16 = 17, // SiLU(gate) * up from weight rows interleaved in gate/up half-warps
-  EPI_QKV_BF16 = 18     // rows [0, split): rotary, to out at row rows[t] (skipped when < 0);
+  EPI_QKV_BF16 = 18,    // rows [0, split): rotary, to out at row rows[t] (skipped when < 0);
                         // rows [split, n_out): to out2 at row t, rotary on the first rope_rows
+  EPI_LSE_F32 = 19      // logit-lens statistics: for every group of 32 weight rows g and token t,
+                        // float4 (m, s, u, 0) at out[t * ldo + g] with m = max z, s = sum e^(z - m),
+                        // u = sum e^(z - m) (z - m) over the group's rows (rows past n_out left out)
 };
+// Number of 32-row groups of the logit-lens statistics of a V-word vocabulary.
+__host__ __device__ inline int lse_groups(int V) { return (V + 31) / 32; }
 
 struct GemmProblem {
   const CUtensorMap* map_w;  // weights [n_out][k] bf16, box 64 x 128 (optional)
@@ -164,13 +169,14 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream);
 
 // ---- ASL-Skip online scores (Sec. 4.2.1, Eq. 6) -------------------------------------------------
 // For candidate n (token cand[n], sequence seq_of[token]): E = entropy of softmax(logits[n]) / log V
-// (mode kSkipEntropy, else 0; logits unread), F = (cos of h[token] to the mean h of its sequence's
+// (mode kSkipEntropy, else 0; logits unread; with kSkipLse `logits` holds the float4 statistics of
+// EPI_LSE_F32 instead, [n_cand][lse_groups(V)], merged here), F = (cos of h[token] to the mean h of its sequence's
 // text tokens text[ts[b] .. ts[b+1]) (computed into tmean [B][D]) + 1) / 2 (mode kSkipItc, else 0),
 // S_sa = ReLU(1 - E - F); s_skip[token] = (kSkipAccumulate ? s_skip[token] : 0) + w1 S_sa + add_slc;
 // flag[n] = (s_skip[token] >= t_skip).
 // kSkipDevice: the decision stays on the device: candidates with admit >= 0 are left alone, and
 // one that reaches t_skip gets admit = layer, target = tgt (flag unused).
-constexpr int kSkipEntropy = 1, kSkipItc = 2, kSkipAccumulate = 4, kSkipDevice = 8;
+constexpr int kSkipEntropy = 1, kSkipItc = 2, kSkipAccumulate = 4, kSkipDevice = 8, kSkipLse = 16;
 int skip_scores_run(const float* logits, int V, int n_cand, const float* h, int D, const int32_t* cand,
                     const int32_t* ts, const int32_t* text, const int32_t* seq_of, int B, float* tmean,
                     float w1, float add_slc, float t_skip, int mode, float* s_skip, uint8_t* flag,

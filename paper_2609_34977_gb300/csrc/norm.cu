@@ -167,7 +167,29 @@ __global__ void __launch_bounds__(kThreads)
   const int n = blockIdx.x, i = cand[n], b = seq_of[i];
   if ((mode & kSkipDevice) && admit[i] >= 0) return;  // already in skip mode (block-uniform)
   float ent = 0.0f;
-  if (mode & kSkipEntropy) {
+  if ((mode & kSkipEntropy) && (mode & kSkipLse)) {
+    // merge of the per-32-word statistics (m_g, s_g, u_g): with m = max m_g,
+    // S = sum_g e^(m_g - m) s_g and U = sum_g e^(m_g - m) (u_g + (m_g - m) s_g), H = log S - U / S
+    const int G = lse_groups(V);
+    const float4* st = reinterpret_cast<const float4*>(logits) + size_t(n) * G;
+    float mx = -INFINITY;
+    for (int g = threadIdx.x; g < G; g += kThreads) mx = fmaxf(mx, st[g].x);
+    mx = block_max(mx, red);
+    float se = 0.0f, te = 0.0f;
+    for (int g = threadIdx.x; g < G; g += kThreads) {
+      const float4 q = st[g];
+      if (q.y > 0.0f) {
+        const float dm = q.x - mx, f = expf(dm);
+        se += f * q.y;
+        te += f * (q.z + dm * q.y);
+      }
+    }
+    __syncthreads();
+    se = block_sum(se, red);
+    __syncthreads();
+    te = block_sum(te, red);
+    ent = (logf(se) - te / se) * inv_log_v;
+  } else if (mode & kSkipEntropy) {
     const float* z = logits + size_t(n) * V;
     float mx = -INFINITY;
     for (int v = threadIdx.x; v < V; v += kThreads) mx = fmaxf(mx, z[v]);
