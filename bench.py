@@ -776,26 +776,20 @@ def main():
     if not a.no_workloads and L == 32:
         work = other_workloads(torch, N, synth, model, ms_dense, a.steps, a.warmup, a.sweep)
 
-    # end to end through the public API: pinned host inputs -> device, step, logits -> host
+    # end to end through the C ABI with host buffers: spd_step copies the pinned host inputs in,
+    # runs the whole step and copies the logits back to pinned host memory, every step
     hf = [f.cpu().pin_memory() for f in feats]
     ha, ht = attn.cpu().pin_memory(), text.cpu().pin_memory()
     hl = torch.empty_like(spider.logits, device="cpu").pin_memory()
-    for _ in range(a.warmup):
-        for d_, h_ in zip(feats + [attn, text], hf + [ha, ht]):
-            d_.copy_(h_, non_blocking=True)
-        spider.run(feats, attn, text, mask)
-        hl.copy_(spider.logits, non_blocking=True)
-    torch.cuda.synchronize()
-    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    s.record()
-    for _ in range(a.steps):
-        for d_, h_ in zip(feats + [attn, text], hf + [ha, ht]):
-            d_.copy_(h_, non_blocking=True)
-        spider.run(feats, attn, text, mask)
-        hl.copy_(spider.logits, non_blocking=True)
-    e.record()
-    torch.cuda.synchronize()
-    ms_e2e = s.elapsed_time(e) / a.steps
+    pc = spider.prune_cfg
+    ws_step = torch.zeros(N.spd_step_workspace_size(model, pc, [1], [TEXT]), dtype=torch.uint8, device=dev)
+
+    def e2e_step():
+        N.spd_step(model, pc, [1], [TEXT], hf, ha, ht, mask, hl, ws_step)
+
+    ms_e2e = _time_calls(torch, e2e_step, a.steps, a.warmup)
+    assert N.spd_step_status(ws_step, model, pc, [1], [TEXT]) == 0, "device-side failure recorded"
+    del ws_step
     h2d = sum(t.numel() * t.element_size() for t in hf + [ha, ht])
 
     if work is not None:
@@ -827,7 +821,8 @@ def main():
                 "cpu_baseline": cpu,
                 "e2e": {"value": tokens / (ms_e2e / 1000.0), "unit": "tokens/s",
                         "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": hl.numel() * 4,
-                        "ms_per_step": ms_e2e},
+                        "ms_per_step": ms_e2e,
+                        "call": "spd_step (C ABI): pinned host features, attention, text in; logits out"},
                 "gpu_launches": count_launches(spider, mask, False) * a.steps,
                 "clocks": clk,
                 "paper_context": "paper: LLaVA-1.5-7B prefill 67.4 ms (576 tokens) -> 48.2 ms (128), "

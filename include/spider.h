@@ -424,6 +424,37 @@ int spd_linear_noalloc(const uint16_t* X, int M, int K, const uint16_t* W, int N
                        void* stream);
 
 /* ------------------------------------------------------------------------------------------ */
+/* One whole step (Alg. 1: stage 1 then stage 2) in one call                                    */
+/* ------------------------------------------------------------------------------------------ */
+
+/* Workspace bytes of spd_step for this model, pruning configuration and batch layout (0 on
+ * invalid arguments). */
+size_t spd_step_workspace_size(const spd_model* m, const spd_prune_cfg* cfg, int n_seqs,
+                               const int32_t* tiles_per_seq, const int32_t* text_len);
+
+/* The whole SPIDER prefill of a batch (Alg. 1): MSV-Prune of every tile (spd_prune), the kept
+ * final-layer rows to bf16 (spd_gather_rows_bf16), the projector (spd_project; a row copy when the
+ * model has none), the text embeddings, and the decoder prefill with the skip mask (spd_prefill).
+ * Request b owns tiles_per_seq[b] consecutive tiles (host int32 [n_seqs], summing to cfg->n_tiles)
+ * and text_len[b] text tokens (host int32 [n_seqs]); its sequence is [cfg->keep kept tokens of each
+ * of its tiles, in tile order; its text tokens].
+ * feats[l], attn, text and logits may each be in host memory (pinned or pageable) or in device
+ * memory: host inputs are copied into the workspace on `stream` first and host logits are copied
+ * back at the end (the caller synchronises `stream` before reading them). Layouts: feats[l] fp32
+ * [n_tiles][n_tok][d_feat]; attn fp32 as in spd_prune; text bf16 [sum(text_len)][d_model], the
+ * requests' text rows in request order; skip_mask (host) uint8 [n_layers][T] over the packed
+ * tokens (NULL = no skipping); logits fp32 [n_seqs][vocab].
+ * Errors: SPD_EINVAL, SPD_ENOSPC, SPD_ECUDA; device-side failures through spd_step_status. */
+int spd_step(const spd_model* m, const spd_prune_cfg* cfg, int n_seqs, const int32_t* tiles_per_seq,
+             const int32_t* text_len, const float* const* feats, const float* attn, const uint16_t* text,
+             const uint8_t* skip_mask, float* logits, void* ws, size_t ws_bytes, void* stream);
+
+/* The first device-side failure recorded by the calls of a spd_step workspace (synchronises
+ * `stream`, clears the status words): SPD_OK or a negative spd_status. */
+int spd_step_status(void* ws, const spd_model* m, const spd_prune_cfg* cfg, int n_seqs,
+                    const int32_t* tiles_per_seq, const int32_t* text_len, void* stream);
+
+/* ------------------------------------------------------------------------------------------ */
 /* The hot path's contract names (thin forms of the calls above)                               */
 /* ------------------------------------------------------------------------------------------ */
 

@@ -30,7 +30,8 @@ EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait"
            "spd_linear_workspace_size", "spd_linear", "spd_linear_noalloc", "spd_trace_enable",
            "spd_trace_read", "spd_prune_workspace", "spd_prefill_workspace", "spd_gather_bf16",
            "spd_last_error_detail", "spd_check", "spd_plan_from_layer_mask", "spd_prefill_admit",
-           "spd_stamp_enable", "spd_stamp_read", "spd_stamp_launch", "spd_set_deterministic")
+           "spd_stamp_enable", "spd_stamp_read", "spd_stamp_launch", "spd_set_deterministic",
+           "spd_step_workspace_size", "spd_step", "spd_step_status")
 TRACE_GEMM, TRACE_ATTN, TRACE_ROWS, TRACE_PRUNE = 0, 1, 2, 3
 
 
@@ -133,6 +134,9 @@ def lib():
             "spd_linear_noalloc": (i, [vp, i, i, vp, i, i, vp, vp, vp, i, vp, vp]),
             "spd_trace_enable": (i, [i]),
             "spd_set_deterministic": (i, [i]),
+            "spd_step_workspace_size": (sz, [vp, C.POINTER(PruneCfg), i, vp, vp]),
+            "spd_step": (i, [vp, C.POINTER(PruneCfg), i, vp, vp, C.POINTER(vp), vp, vp, vp, vp, vp, sz, vp]),
+            "spd_step_status": (i, [vp, vp, C.POINTER(PruneCfg), i, vp, vp, vp]),
             "spd_stamp_enable": (i, [i]),
             "spd_stamp_launch": (i, [i, C.POINTER(i), C.POINTER(C.c_ulonglong), C.POINTER(C.c_ulonglong),
                                      C.POINTER(C.c_double), C.POINTER(C.c_double)]),
@@ -549,3 +553,63 @@ def spd_stamp_launches() -> list:
 def spd_set_deterministic(on: bool):
     """Library-wide deterministic mode: GEMM sums in a fixed order (bit-identical repeated runs)."""
     _check(lib().spd_set_deterministic(int(bool(on))))
+
+
+def _any(t, dt, n, name, optional=False):
+    """Pointer of an argument that may be in host or device memory (spd_step): a contiguous torch
+    tensor of element type dt with at least n elements, on the GPU or the CPU (pinned or not)."""
+    if t is None:
+        if optional:
+            return None
+        raise ValueError(f"{name}: a tensor is required")
+    if getattr(t, "is_cuda", False):
+        return _dev(t, dt, n, name)
+    if isinstance(t, np.ndarray) or not hasattr(t, "data_ptr"):
+        raise TypeError(f"{name}: a torch tensor is required")
+    if str(t.dtype) != "torch." + _DT[dt]:
+        raise ValueError(f"{name}: expected {_DT[dt]}, got {t.dtype}")
+    if t.numel() < n:
+        raise ValueError(f"{name}: {t.numel()} elements, the call touches {int(n)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: must be contiguous")
+    return t.data_ptr()
+
+
+def _step_layout(cfg, tiles_per_seq, text_len):
+    tps = np.ascontiguousarray(tiles_per_seq, dtype=np.int32)
+    tl = _host(text_len, np.int32, len(tps), "text_len")
+    return tps, tl
+
+
+def spd_step_workspace_size(model: SpdModel, cfg, tiles_per_seq, text_len) -> int:
+    tps, tl = _step_layout(cfg, tiles_per_seq, text_len)
+    return int(lib().spd_step_workspace_size(model.handle, C.byref(cfg), len(tps), tps.ctypes.data,
+                                             tl.ctypes.data))
+
+
+def spd_step(model: SpdModel, cfg, tiles_per_seq, text_len, feats, attn, text, skip_mask, logits, ws,
+             stream=None):
+    """The whole SPIDER step (prune, gather, projector, text rows, prefill) in one call; feats,
+    attn, text and logits may be host (CPU) or device tensors."""
+    tps, tl = _step_layout(cfg, tiles_per_seq, text_len)
+    B, D, L = len(tps), model.cfg["d_model"], model.cfg["n_layers"]
+    T = int(tps.sum()) * cfg.keep + int(tl.sum())
+    n = cfg.n_tok - (1 if cfg.has_cls else 0)
+    n_att = cfg.n_tok if cfg.attn_form == 0 else n
+    if len(feats) != cfg.n_layers:
+        raise ValueError(f"feats: {len(feats)} layers, cfg.n_layers = {cfg.n_layers}")
+    fa = (C.c_void_p * len(feats))(*[_any(f, "f32", cfg.n_tiles * cfg.n_tok * cfg.d_feat, f"feats[{i}]")
+                                      for i, f in enumerate(feats)])
+    mask = None if skip_mask is None else _host(skip_mask, np.uint8, L * T, "skip_mask")
+    wp, wb = _ws(ws)
+    _check(lib().spd_step(model.handle, C.byref(cfg), B, tps.ctypes.data, tl.ctypes.data, fa,
+                          _any(attn, "f32", cfg.n_tiles * cfg.n_heads * n_att, "attn"),
+                          _any(text, "bf16", int(tl.sum()) * D, "text", optional=int(tl.sum()) == 0),
+                          None if mask is None else mask.ctypes.data,
+                          _any(logits, "f32", B * model.cfg["vocab"], "logits"), wp, wb, _stream(stream)))
+
+
+def spd_step_status(ws, model: SpdModel, cfg, tiles_per_seq, text_len, stream=None) -> int:
+    tps, tl = _step_layout(cfg, tiles_per_seq, text_len)
+    return int(lib().spd_step_status(_p(ws), model.handle, C.byref(cfg), len(tps), tps.ctypes.data,
+                                     tl.ctypes.data, _stream(stream)))

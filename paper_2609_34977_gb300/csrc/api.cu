@@ -1171,3 +1171,169 @@ extern "C" int spd_prefill_admit(const spd_model* m, const uint16_t* x, int T, c
   if (int rc = spd_plan_adaptive(m->cfg.n_layers, T, admit_layer, target, mask.data())) return rc;
   return spd_prefill(m, x, T, cu, B, mask.data(), h, logits, ws, ws_bytes, stream);
 }
+
+// ---- one whole SPIDER step through the C ABI (host or device buffers) ------------------------------
+namespace {
+bool on_host(const void* p) {
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return true;  // unknown to CUDA: pageable host memory
+  }
+  return at.type == cudaMemoryTypeHost || at.type == cudaMemoryTypeUnregistered;
+}
+
+struct StepLayout {
+  int B = 0, T = 0, n_tiles = 0, n_vis = 0, n_text = 0, n_patch = 0;
+  std::vector<int32_t> cu, vis_rows, text_rows;
+};
+
+int step_layout(const spd_model* m, const spd_prune_cfg* pc, int B, const int32_t* tiles_per_seq,
+                const int32_t* text_len, StepLayout* L) {
+  if (!m || !pc || B < 1 || !tiles_per_seq || !text_len) return fail(SPD_EINVAL, "bad step arguments");
+  L->B = B;
+  L->n_patch = pc->n_tok - (pc->has_cls ? 1 : 0);
+  L->cu.assign(1, 0);
+  L->vis_rows.clear();
+  L->text_rows.clear();
+  int row = 0, tiles = 0;
+  for (int b = 0; b < B; ++b) {
+    if (tiles_per_seq[b] < 0 || text_len[b] < 0 || tiles_per_seq[b] + text_len[b] == 0)
+      return fail(SPD_EINVAL, "sequence %d: negative or empty", b);
+    const int nv = tiles_per_seq[b] * pc->keep;
+    for (int i = 0; i < nv; ++i) L->vis_rows.push_back(row++);
+    for (int i = 0; i < text_len[b]; ++i) L->text_rows.push_back(row++);
+    L->cu.push_back(row);
+    tiles += tiles_per_seq[b];
+  }
+  if (tiles != pc->n_tiles) return fail(SPD_EINVAL, "tiles_per_seq sums to %d, cfg.n_tiles is %d", tiles, pc->n_tiles);
+  L->T = row;
+  L->n_tiles = tiles;
+  L->n_vis = int(L->vis_rows.size());
+  L->n_text = int(L->text_rows.size());
+  if (!m->cfg.d_vis && pc->d_feat != m->cfg.d_model)
+    return fail(SPD_EINVAL, "without a projector the feature width must equal d_model");
+  if (m->cfg.d_vis && pc->d_feat != m->cfg.d_vis) return fail(SPD_EINVAL, "feature width != projector input");
+  return SPD_OK;
+}
+
+// Carves the step's buffers; sizes only when base is null.
+struct StepBufs {
+  const float* feats[SPD_MAX_FEAT_LAYERS];
+  float *feat_copy[SPD_MAX_FEAT_LAYERS], *attn_copy, *logits_dev;
+  uint16_t *text_copy, *vis, *x;
+  float* h;
+  int32_t *keep_idx, *rows;  // rows: vis_rows then text_rows
+  uint8_t *prune_ws, *proj_ws, *pre_ws;
+  size_t prune_bytes, proj_bytes, pre_bytes;
+};
+size_t step_carve(const spd_model* m, const spd_prune_cfg* pc, const StepLayout& L, void* base,
+                  StepBufs* s) {
+  Carve cv(base, ~size_t(0));
+  const size_t tile = size_t(pc->n_tok) * pc->d_feat;
+  for (int l = 0; l < pc->n_layers; ++l) s->feat_copy[l] = cv.take<float>(size_t(pc->n_tiles) * tile);
+  const int n_att = pc->attn_form == 0 ? pc->n_tok : L.n_patch;
+  s->attn_copy = cv.take<float>(size_t(pc->n_tiles) * pc->n_heads * n_att);
+  s->text_copy = cv.take<uint16_t>(size_t(L.n_text) * m->cfg.d_model);
+  s->logits_dev = cv.take<float>(size_t(L.B) * m->cfg.vocab);
+  s->keep_idx = cv.take<int32_t>(size_t(pc->n_tiles) * pc->keep);
+  s->rows = cv.take<int32_t>(size_t(L.n_vis + L.n_text));
+  s->vis = cv.take<uint16_t>(size_t(L.n_vis) * pc->d_feat);
+  s->x = cv.take<uint16_t>(size_t(L.T) * m->cfg.d_model);
+  s->h = cv.take<float>(size_t(L.T) * m->cfg.d_model);
+  s->prune_bytes = spd_prune_workspace_size(pc);
+  s->prune_ws = cv.take<uint8_t>(s->prune_bytes);
+  s->proj_bytes = m->cfg.d_vis ? spd_project_workspace_size(m, L.n_vis) : 0;
+  s->proj_ws = cv.take<uint8_t>(s->proj_bytes);
+  s->pre_bytes = spd_prefill_workspace_size(m, L.T, L.B);
+  s->pre_ws = cv.take<uint8_t>(s->pre_bytes);
+  return cv.used;
+}
+}  // namespace
+
+extern "C" size_t spd_step_workspace_size(const spd_model* m, const spd_prune_cfg* cfg, int n_seqs,
+                                          const int32_t* tiles_per_seq, const int32_t* text_len) {
+  StepLayout L;
+  if (step_layout(m, cfg, n_seqs, tiles_per_seq, text_len, &L)) return 0;
+  if (!spd_prune_workspace_size(cfg)) return 0;
+  StepBufs s;
+  return step_carve(m, cfg, L, nullptr, &s);
+}
+
+extern "C" int spd_step(const spd_model* m, const spd_prune_cfg* cfg, int n_seqs,
+                        const int32_t* tiles_per_seq, const int32_t* text_len,
+                        const float* const* feats, const float* attn, const uint16_t* text,
+                        const uint8_t* skip_mask, float* logits, void* ws, size_t ws_bytes, void* stream) {
+  StepLayout L;
+  if (int rc = step_layout(m, cfg, n_seqs, tiles_per_seq, text_len, &L)) return rc;
+  if (!feats || !attn || (L.n_text && !text) || !logits || !ws) return fail(SPD_EINVAL, "null step buffer");
+  if (cfg->n_layers < 1 || cfg->n_layers > SPD_MAX_FEAT_LAYERS) return fail(SPD_EINVAL, "bad feature layer count");
+  StepBufs s;
+  const size_t need = step_carve(m, cfg, L, ws, &s);
+  if (need > ws_bytes) return fail(SPD_ENOSPC, "step workspace too small (%zu < %zu)", ws_bytes, need);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t tile = size_t(cfg->n_tok) * cfg->d_feat;
+  // inputs in host memory are copied into the workspace first
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    if (!feats[l]) return fail(SPD_EINVAL, "null feature layer %d", l);
+    s.feats[l] = feats[l];
+    if (on_host(feats[l])) {
+      SPD_CUDA_TRY(cudaMemcpyAsync(s.feat_copy[l], feats[l], cfg->n_tiles * tile * sizeof(float),
+                                   cudaMemcpyHostToDevice, st));
+      s.feats[l] = s.feat_copy[l];
+    }
+  }
+  const int n_att = cfg->attn_form == 0 ? cfg->n_tok : L.n_patch;
+  const float* attn_d = attn;
+  if (on_host(attn)) {
+    SPD_CUDA_TRY(cudaMemcpyAsync(s.attn_copy, attn, size_t(cfg->n_tiles) * cfg->n_heads * n_att * sizeof(float),
+                                 cudaMemcpyHostToDevice, st));
+    attn_d = s.attn_copy;
+  }
+  const uint16_t* text_d = text;
+  const size_t D = m->cfg.d_model;
+  if (L.n_text && on_host(text)) {
+    SPD_CUDA_TRY(cudaMemcpyAsync(s.text_copy, text, L.n_text * D * sizeof(uint16_t), cudaMemcpyHostToDevice, st));
+    text_d = s.text_copy;
+  }
+  std::vector<int32_t> rows(L.vis_rows);
+  rows.insert(rows.end(), L.text_rows.begin(), L.text_rows.end());
+  if (!rows.empty())
+    SPD_CUDA_TRY(cudaMemcpyAsync(s.rows, rows.data(), rows.size() * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  // MSV-Prune, gather, projector (or row copy), text rows, prefill
+  if (int rc = spd_prune(cfg, s.feats, attn_d, s.keep_idx, nullptr, nullptr, nullptr, s.prune_ws, s.prune_bytes,
+                         stream))
+    return rc;
+  if (int rc = spd_gather_rows_bf16(s.feats[cfg->final_layer], cfg->n_tiles, cfg->n_tok, cfg->d_feat,
+                                    cfg->has_cls ? 1 : 0, s.keep_idx, cfg->keep, s.vis, s.prune_ws, stream))
+    return rc;
+  if (L.n_vis) {
+    const int rc = m->cfg.d_vis ? spd_project(m, s.vis, L.n_vis, s.rows, s.x, s.proj_ws, s.proj_bytes, stream)
+                                : spd_scatter_rows(m, s.vis, L.n_vis, s.rows, s.x, stream);
+    if (rc) return rc;
+  }
+  if (L.n_text)
+    if (int rc = spd_scatter_rows(m, text_d, L.n_text, s.rows + L.n_vis, s.x, stream)) return rc;
+  const bool host_logits = on_host(logits);
+  float* lg = host_logits ? s.logits_dev : logits;
+  if (int rc = spd_prefill(m, s.x, L.T, L.cu.data(), L.B, skip_mask, s.h, lg, s.pre_ws, s.pre_bytes, stream))
+    return rc;
+  if (host_logits)
+    SPD_CUDA_TRY(cudaMemcpyAsync(logits, lg, size_t(L.B) * m->cfg.vocab * sizeof(float), cudaMemcpyDeviceToHost, st));
+  return SPD_OK;
+}
+
+extern "C" int spd_step_status(void* ws, const spd_model* m, const spd_prune_cfg* cfg, int n_seqs,
+                               const int32_t* tiles_per_seq, const int32_t* text_len, void* stream) {
+  StepLayout L;
+  if (int rc = step_layout(m, cfg, n_seqs, tiles_per_seq, text_len, &L)) return rc;
+  StepBufs s;
+  step_carve(m, cfg, L, ws, &s);
+  for (void* w : {static_cast<void*>(s.prune_ws), static_cast<void*>(s.proj_ws), static_cast<void*>(s.pre_ws)}) {
+    if (w == s.proj_ws && !s.proj_bytes) continue;
+    int v = 0;
+    if (int rc = spd_workspace_status(w, stream, &v)) return rc;
+    if (v) return v;
+  }
+  return SPD_OK;
+}

@@ -54,3 +54,41 @@ def test_spider_step_at_the_llava15_shape():
     h_o, lg_o = od.prefill(om, x, pipe.cu, od.expand_adaptive_plan(admit, target, L))
     assert rowwise_rel(pipe.h.cpu().numpy(), h_o) < TOL
     assert rowwise_rel(logits.cpu().numpy(), lg_o) < TOL
+
+
+@pytest.mark.parametrize("host", [True, False])
+def test_whole_step_entry_with_host_or_device_buffers(host):
+    # spd_step (one C-ABI call: prune, gather, projector, text rows, prefill) with the inputs and
+    # the logits in pinned host memory (copied inside the call) or on the device, against the
+    # oracle's stages on the tiny decoder with a projector: 2 requests of 1 and 2 tiles
+    cfg = dict(synth.TINY_DECODER, d_vis=128, d_proj=192)
+    w = synth.decoder_weights(20260501, cfg, std=0.05)
+    model = N.SpdModel(cfg, {k: (v.cuda() if k != "layers" else [{kk: vv.cuda() for kk, vv in lw.items()}
+                                                                  for lw in v]) for k, v in w.items()})
+    keep, tiles, texts = 32, [1, 2], [16, 8]
+    seed, v, res = conditioned_vision(20260510, 3, 576, 128, 2, 8, keep, 1)
+    pc = N.prune_cfg(3, 577, 128, 2, 1, 8, keep)
+    text = synth.text_embeddings(seed, sum(texts), 256)
+    T = sum(t * keep for t in tiles) + sum(texts)
+    vis = np.concatenate([np.r_[np.ones(t * keep, bool), np.zeros(x, bool)] for t, x in zip(tiles, texts)])
+    mask = N.spd_plan_static(np.array([1, 2], np.uint8), vis.astype(np.uint8))
+    feats = [torch.from_numpy(f) for f in v["feats"]]
+    attn = torch.from_numpy(v["attn"])
+    tx = torch.from_numpy(text.view(np.int16)).view(torch.bfloat16)
+    if host:
+        feats, attn, tx = [f.pin_memory() for f in feats], attn.pin_memory(), tx.pin_memory()
+        logits = torch.full((2, 512), float("nan")).pin_memory()
+    else:
+        feats, attn, tx = [f.cuda() for f in feats], attn.cuda(), tx.cuda()
+        logits = torch.full((2, 512), float("nan"), device="cuda")
+    ws = torch.zeros(N.spd_step_workspace_size(model, pc, tiles, texts), dtype=torch.uint8, device="cuda")
+    N.spd_step(model, pc, tiles, texts, feats, attn, tx, mask, logits, ws)
+    torch.cuda.synchronize()
+    assert N.spd_step_status(ws, model, pc, tiles, texts) == 0
+    om = od.model_from_torch(w, cfg)
+    xv = od.project(om, np.concatenate([od.bf16_round(v["feats"][1][t, 1 + res[t]["keep_idx"]]) for t in range(3)]))
+    txt = synth.bf16_bits_to_f32(text).astype(np.float64)
+    x = np.concatenate([xv[:keep], txt[:16], xv[keep:], txt[16:]])
+    cu = [0, keep + 16, T]
+    _, lg_o = od.prefill(om, x, cu, mask)
+    assert rowwise_rel(logits.cpu().numpy(), lg_o) < TOL
