@@ -51,8 +51,9 @@ struct PruneDims {
 struct PruneWs {
   float* a_v;       // [T][n]
   float* inv;       // [L][T][n]
-  float* st1;       // [L][T][n] MSE: ||F_l,i||^2; KL: log-sum-exp of F_l,i
+  float* st1;       // [L][T][n] MSE: ||F_l,i||^2; KL: log-sum-exp of F_l,i (rounded to fp32)
   float* st2;       // [L][T][n] KL: sum_c P_c log P_c of P = softmax(F_l,i)
+  float* st3;       // [L][T][n] KL: log-sum-exp minus its fp32 rounding (st1 + st3 = the fp64 value)
   int8_t* role;     // [T][n] 1 anchor
   int32_t* alist;   // [T][n_anc]
   int32_t* ulist;   // [T][m]
@@ -62,7 +63,7 @@ struct PruneWs {
   int32_t* quotas;  // [T][16]
   float* asum;      // [T][16]
   float* csum;      // [T][L][K][d]
-  float* ssum;      // [T][L][16] MSE / KL: per-cluster sums of st1
+  double* ssum;     // [T][L][16] MSE / KL: per-cluster sums of st1 (+ st3), in fp64
   float* score;     // [T][m]
   int* status;
 };
@@ -77,6 +78,11 @@ __device__ __forceinline__ float ordered_val(uint32_t u) {
   return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
 }
 __device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+__device__ __forceinline__ double warp_sum_d(double v) {
 #pragma unroll
   for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
   return v;
@@ -174,7 +180,10 @@ __global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float*
     const size_t o = (size_t(l) * p.n_tiles + t) * p.n + i;
     if (lane == 0) w.inv[o] = 1.0f / sqrtf(ss);
     if (SIM == SPD_SIM_MSE && lane == 0) w.st1[o] = ss;
-    if (SIM == SPD_SIM_KL) {  // softmax over the row: max, then sum e^z and sum e^z z (z = x - max)
+    if (SIM == SPD_SIM_KL) {
+      // softmax over the row in fp64 (z = x - max exact, e^z, sums): the KL scores multiply the
+      // log-probabilities by log-ratios of tens, so an fp32 log-sum-exp (about 2e-6 off) would
+      // move them by about 1e-4
       float mx = -INFINITY;
       for (int c = lane; c < p.d / 4; c += 32) {
         const float4 v = r[c];
@@ -182,23 +191,25 @@ __global__ void __launch_bounds__(256) rowstats_kernel(PruneDims p, const float*
       }
 #pragma unroll
       for (int off = 16; off; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      float se = 0.0f, te = 0.0f;
+      double se = 0.0, te = 0.0;
       for (int c = lane; c < p.d / 4; c += 32) {
         const float4 v = r[c];
-        const float z[4] = {v.x - mx, v.y - mx, v.z - mx, v.w - mx};
+        const double z[4] = {double(v.x) - mx, double(v.y) - mx, double(v.z) - mx, double(v.w) - mx};
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          const float e = expf(z[u]);
+          const double e = exp(z[u]);
           se += e;
           te += e * z[u];
         }
       }
-      se = warp_sum(se);
-      te = warp_sum(te);
+      se = warp_sum_d(se);
+      te = warp_sum_d(te);
       if (lane == 0) {
-        const float lse = logf(se);
-        w.st1[o] = mx + lse;        // log sum_c e^x_c
-        w.st2[o] = te / se - lse;   // sum_c P_c log P_c
+        const double lse = double(mx) + log(se);  // log sum_c e^x_c
+        const float hi = float(lse);
+        w.st1[o] = hi;
+        w.st3[o] = float(lse - double(hi));
+        w.st2[o] = float(te / se - log(se));      // sum_c P_c log P_c
       }
     }
   }
@@ -286,13 +297,13 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
   constexpr bool kl = SIM == SPD_SIM_KL;
   const float* urow[8];
   const float* arow[8];
-  float ulse[8];  // KL: the non-anchor operand is softmax(F^L_i) = exp(F^L_i - lse_i)
+  double ulse[8];  // KL: the non-anchor operand is softmax(F^L_i) = exp(F^L_i - lse_i), in fp64
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const int r = r0 + 8 * i;
     urow[i] = (u0 + r < p.m) ? feat_row(p, p.fin, t, ul[u0 + r]) : nullptr;
     arow[i] = (p0 + r < p.n_anc) ? feat_row(p, p.fin, t, al[p0 + r]) : nullptr;
-    ulse[i] = (kl && urow[i]) ? w.st1[so + ul[u0 + r]] : 0.0f;
+    ulse[i] = (kl && urow[i]) ? double(w.st1[so + ul[u0 + r]]) + double(w.st3[so + ul[u0 + r]]) : 0.0;
   }
   const int nch = (p.d + 31) / 32, c0 = rank * nch / kAS, c1 = (rank + 1) * nch / kAS;
   float ru[8], ra[8];
@@ -301,7 +312,8 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const float x = (urow[i] && dcol < p.d) ? urow[i][dcol] : 0.0f;
-      ru[i] = (kl && urow[i] && dcol < p.d) ? expf(x - ulse[i]) : x;
+      if constexpr (kl) ru[i] = (urow[i] && dcol < p.d) ? float(exp(double(x) - ulse[i])) : 0.0f;
+      else ru[i] = x;
       ra[i] = (arow[i] && dcol < p.d) ? arow[i][dcol] : 0.0f;
     }
   };
@@ -366,7 +378,8 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
         const int ia = al[pa];
         const float v = SIM == SPD_SIM_COS ? sdot * iu * inv[ia]
                         : SIM == SPD_SIM_MSE ? 2.0f * sdot - w.st1[so + ia]
-                                             : sdot - w.st1[so + ia];
+                                             : float(double(sdot) - double(w.st1[so + ia]) -
+                                                     double(w.st3[so + ia]));
         best = fmaxf(best, v);
       }
     }
@@ -563,7 +576,7 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
   float* part = cent + size_t(K) * D;                         // [K][D] this CTA's column sums
   __shared__ int cnt[SPD_MAX_CLUSTERS];   // this CTA's cluster sizes
   __shared__ float asum_part[SPD_MAX_CLUSTERS];
-  __shared__ float ssum_part[SPD_MAX_CLUSTERS];  // MSE / KL: this CTA's sums of st1 per cluster
+  __shared__ double ssum_part[SPD_MAX_CLUSTERS];  // MSE / KL: this CTA's sums of st1 (+ st3) per cluster
   __shared__ int changed;      // this CTA's assignment changed in the current iteration
   __shared__ int any_changed;  // ... some CTA's of the cluster
   __shared__ int8_t asg[4096 / KC + 1];
@@ -776,9 +789,11 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
       }
     }
     __syncthreads();
-    if (!cos_sim && threadIdx.x == 0) {  // token order
-      for (int k = 0; k < K; ++k) ssum_part[k] = 0.0f;
-      for (int jj = 0; jj < nl; ++jj) ssum_part[asg[jj]] += rinv[jj];
+    if (!cos_sim && threadIdx.x == 0) {  // token order, fp64 (KL: the fp64 log-sum-exps)
+      const float* lo = p.sim == SPD_SIM_KL ? w.st3 + (size_t(l) * p.n_tiles + t) * p.n : nullptr;
+      for (int k = 0; k < K; ++k) ssum_part[k] = 0.0;
+      for (int jj = 0; jj < nl; ++jj)
+        ssum_part[asg[jj]] += double(rinv[jj]) + (lo ? double(lo[idx[jj]]) : 0.0);
     }
     column_sums<KN>(part, K, D, nl, asg,
                     RowAccess{RES ? rows : nullptr, fl, row0, idx, D, cos_sim ? rinv : static_cast<float*>(nullptr)});
@@ -788,8 +803,8 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
                               [&](int k, int c, float sum) { csum[k * D + c] = sum; });
     if (!cos_sim && rank == 0 && warp == 1) {  // CTA sums added in rank order
       for (int k = 0; k < K; ++k) {
-        const float sr = lane < KC ? cl.map_shared_rank(ssum_part, lane)[k] : 0.0f;
-        float a = 0.0f;
+        const double sr = lane < KC ? cl.map_shared_rank(ssum_part, lane)[k] : 0.0;
+        double a = 0.0;
         for (int rr = 0; rr < KC; ++rr) a += __shfl_sync(0xffffffffu, sr, rr);
         if (lane == 0) w.ssum[(size_t(t) * p.L + l) * 16 + k] = a;
       }
@@ -850,14 +865,15 @@ __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
       const float4* x4 = reinterpret_cast<const float4*>(feat_row(p, l, t, i));
       const size_t so = (size_t(l) * p.n_tiles + t) * p.n + i;
       const float iv = SIM == SPD_SIM_COS ? w.inv[so] : 1.0f;
-      const float lse = SIM == SPD_SIM_KL ? w.st1[so] : 0.0f;
-      const float inv_n = 1.0f / float(cnt);
-      const float sbar = SIM == SPD_SIM_KL ? w.ssum[(size_t(t) * p.L + l) * 16 + k] * inv_n : 0.0f;
+      // KL in fp64: log P_i,c = x_c - lse_i and the cluster mean of log P_j,c
+      const double lse = SIM == SPD_SIM_KL ? double(w.st1[so]) + double(w.st3[so]) : 0.0;
+      const double sbar = SIM == SPD_SIM_KL ? w.ssum[(size_t(t) * p.L + l) * 16 + k] / double(cnt) : 0.0;
       const float4* c4 =
           reinterpret_cast<const float4*>(w.csum + ((size_t(t) * p.L + l) * p.K + k) * p.d);
       // 16-byte loads, sixteen in flight per lane, two independent chains
       const int d4 = p.d / 4;
       float dot0 = 0.0f, dot1 = 0.0f;
+      double kdot = 0.0;  // KL
       for (int cb = lane; cb < d4; cb += 256) {
         float4 xv[8], cv[8];
 #pragma unroll
@@ -870,28 +886,30 @@ __global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
         for (int u = 0; u < 8; ++u) {
           // cos: f.(X - f) with f = x |x|^-1; MSE: x.(X - x); KL: P.(log P - mean_j log P_j)
           const float b0 = xv[u].x * iv, b1 = xv[u].y * iv, b2 = xv[u].z * iv, b3 = xv[u].w * iv;
-          float part;
-          if (SIM == SPD_SIM_KL) {
+          if constexpr (SIM == SPD_SIM_KL) {
             if (cb + 32 * u >= d4) continue;  // a zero-filled slot is no zero term here
-            const float l0 = b0 - lse, l1 = b1 - lse, l2 = b2 - lse, l3 = b3 - lse;
-            part = expf(l0) * (l0 - (cv[u].x * inv_n - sbar)) + expf(l1) * (l1 - (cv[u].y * inv_n - sbar)) +
-                   expf(l2) * (l2 - (cv[u].z * inv_n - sbar)) + expf(l3) * (l3 - (cv[u].w * inv_n - sbar));
+            const double dn = double(cnt);
+            const double l0 = double(b0) - lse, l1 = double(b1) - lse, l2 = double(b2) - lse,
+                         l3 = double(b3) - lse;
+            kdot += exp(l0) * (l0 - (double(cv[u].x) / dn - sbar)) +
+                    exp(l1) * (l1 - (double(cv[u].y) / dn - sbar)) +
+                    exp(l2) * (l2 - (double(cv[u].z) / dn - sbar)) +
+                    exp(l3) * (l3 - (double(cv[u].w) / dn - sbar));
           } else {
-            part = b0 * (cv[u].x - b0) + b1 * (cv[u].y - b1) + b2 * (cv[u].z - b2) + b3 * (cv[u].w - b3);
+            const float part =
+                b0 * (cv[u].x - b0) + b1 * (cv[u].y - b1) + b2 * (cv[u].z - b2) + b3 * (cv[u].w - b3);
+            if (u & 1) dot1 += part;
+            else dot0 += part;
           }
-          if (u & 1) dot1 += part;
-          else dot0 += part;
         }
       }
       const float dot = warp_sum(dot0 + dot1);
       float term = dot;
-      if (SIM != SPD_SIM_COS) {
-        if (SIM == SPD_SIM_MSE) {
-          const float sk = w.ssum[(size_t(t) * p.L + l) * 16 + k], st = w.st1[so];
-          term = -(float(cnt - 1) * st - 2.0f * dot + (sk - st)) / float(p.d);
-        } else {
-          term = -float(cnt) * dot;
-        }
+      if (SIM == SPD_SIM_MSE) {
+        const float sk = float(w.ssum[(size_t(t) * p.L + l) * 16 + k]), st = w.st1[so];
+        term = -(float(cnt - 1) * st - 2.0f * dot + (sk - st)) / float(p.d);
+      } else if (SIM == SPD_SIM_KL) {
+        term = float(-double(cnt) * warp_sum_d(kdot));
       }
       acc += wl * term;
     }
@@ -1116,6 +1134,7 @@ PruneWs carve(const PruneDims& p, Carve& cv) {
   const size_t nst = p.sim == SPD_SIM_COS ? 0 : T * p.n * p.L;
   w.st1 = cv.take<float>(nst);
   w.st2 = cv.take<float>(p.sim == SPD_SIM_KL ? nst : 0);
+  w.st3 = cv.take<float>(p.sim == SPD_SIM_KL ? nst : 0);
   w.role = cv.take<int8_t>(T * p.n);
   w.alist = cv.take<int32_t>(T * (p.n_anc + 1));
   w.ulist = cv.take<int32_t>(T * (p.m + 1));
@@ -1125,7 +1144,7 @@ PruneWs carve(const PruneDims& p, Carve& cv) {
   w.quotas = cv.take<int32_t>(T * 16);
   w.asum = cv.take<float>(T * 16);
   w.csum = cv.take<float>(T * p.L * p.K * p.d);
-  w.ssum = cv.take<float>(T * p.L * 16);
+  w.ssum = cv.take<double>(T * p.L * 16);
   w.score = cv.take<float>(T * (p.m + 1));
   return w;
 }

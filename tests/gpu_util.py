@@ -66,4 +66,6 @@ def assert_prune_parity(g, res, score_rtol=1e-5):
         assert np.isinf(s_g[anchors]).all()
         fin = ~anchors
         err = np.abs(s_g[fin] - s_o[fin]) / np.maximum(np.abs(s_o[fin]), 1e-2)
+        if err.size:
+            print(f"prune scores: max relative error {err.max():.3e} (tolerance {score_rtol:.0e})")
         assert err.max() <= score_rtol, err.max()

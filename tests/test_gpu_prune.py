@@ -162,11 +162,11 @@ def test_received_attention_repeat_runs_are_bitwise_identical():
 
 
 # ---- ablation variants of the MSV-Prune table ----
-# Scores of the KL kind within 5e-5 relative (floor 1e-2): the fp32 softmax exp(F - lse) of rows
-# whose entries reach |F| ~ 20 carries a relative error of about eps32 |F - lse| ~ 3e-6 in every
-# probability; times the log-ratios (~ 40) that KL sums, about 1e-4 absolute on scores of a few units.
+# Every kind's scores within 1e-5 relative (floor 1e-2). For KL the library takes the softmax and
+# its log-probabilities in fp64 (an fp32 exp(F - lse) of rows with |F| ~ 20 is about 3e-6 off in
+# every probability, which the log-ratios of tens that KL sums turn into about 1e-4 on the scores).
 def _score_rtol(kw):
-    return 5e-5 if kw.get("sim") == "kl" else 1e-5
+    return 1e-5
 
 
 @pytest.mark.parametrize("kw", [
