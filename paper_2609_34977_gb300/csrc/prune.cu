@@ -6,7 +6,7 @@
 //   anchors      top-N_anc of a_v by a bitonic sort of (a_v desc, index asc) keys (Eq. 1);
 //                stable lists of anchor and non-anchor tokens by block prefix sums
 //   anchor_sim   a_i = max_p cos(F^L_i, F^L_p) over anchors: 64 x 64 register-tiled fp32 products,
-//                the feature dimension split over a cluster of 4 CTAs whose partial tiles are summed
+//                the feature dimension split over a cluster of 4 (8 for few tiles) CTAs whose partial tiles are summed
 //                in rank order through distributed shared memory; max via atomicMax on
 //                order-preserving integer keys (exact, order independent)
 //   kmeans       one thread-block cluster of 16 CTAs per tile, each owning a contiguous slice of the
@@ -270,15 +270,13 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
 }
 
 // ---- 3. a_i = max over anchors of cos(F^L_i, F^L_p) -------------------------------------------
-// A cluster of kAS CTAs per 64 non-anchor tokens x 64 anchors tile, each CTA one slice of the
+// A cluster of AS CTAs per 64 non-anchor tokens x 64 anchors tile, each CTA one slice of the
 // feature dimension: 32-wide chunks through shared memory (stored transposed; the next chunk is
 // fetched into registers while the current one is multiplied), 4 x 4 dot products per thread.
 // The partial tiles are summed in rank order through distributed shared memory, each CTA
-// finishing 16 rows.
-constexpr int kAS = 4;
-
-template <int SIM>
-__global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
+// finishing 64 / AS rows. AS = 4 at serving batch; 8 for a few tiles (shorter chains per CTA).
+template <int SIM, int AS>
+__global__ void __cluster_dims__(AS, 1, 1) __launch_bounds__(256)
     anchor_sim_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
@@ -287,7 +285,7 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
   cg::cluster_group cl = cg::this_cluster();
   const int rank = int(cl.block_rank());
   const int t = blockIdx.z, tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  const int u0 = (blockIdx.x / kAS) * 64, p0 = blockIdx.y * 64;
+  const int u0 = (blockIdx.x / AS) * 64, p0 = blockIdx.y * 64;
   const int* ul = w.ulist + size_t(t) * p.m;
   const int* al = w.alist + size_t(t) * p.n_anc;
   // staging: thread loads column dd of rows r0 + 8 i (i < 8) of both operands
@@ -305,7 +303,7 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
     arow[i] = (p0 + r < p.n_anc) ? feat_row(p, p.fin, t, al[p0 + r]) : nullptr;
     ulse[i] = (kl && urow[i]) ? double(w.st1[so + ul[u0 + r]]) + double(w.st3[so + ul[u0 + r]]) : 0.0;
   }
-  const int nch = (p.d + 31) / 32, c0 = rank * nch / kAS, c1 = (rank + 1) * nch / kAS;
+  const int nch = (p.d + 31) / 32, c0 = rank * nch / AS, c1 = (rank + 1) * nch / AS;
   float ru[8], ra[8];
   auto fetch = [&](int ch) {
     const int dcol = ch * 32 + dd;
@@ -350,14 +348,16 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
 #pragma unroll
     for (int j = 0; j < 4; ++j) P[ty + 16 * i][tx + 16 * j] = acc[i][j];
   cl.sync();
-  // rows 16 rank .. 16 rank + 15 of the tile: all kAS partials loaded first, summed in rank order
-  const int lr = 16 * rank + ty;
-  float x[kAS][4];
+  // rows RPC rank .. RPC rank + RPC - 1 of the tile (TPR threads a row, CPT columns a thread): all
+  // AS partials loaded first, summed in rank order
+  constexpr int RPC = 64 / AS, TPR = 256 / RPC, CPT = 64 / TPR;
+  const int lr = RPC * rank + int(threadIdx.x) / TPR, cx = int(threadIdx.x) % TPR;
+  float x[AS][CPT];
 #pragma unroll
-  for (int src = 0; src < kAS; ++src) {
+  for (int src = 0; src < AS; ++src) {
     const float* pp = cl.map_shared_rank(&P[0][0], src) + lr * 65;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) x[src][j] = pp[tx + 16 * j];
+    for (int j = 0; j < CPT; ++j) x[src][j] = pp[cx + TPR * j];
   }
   const float* inv = w.inv + size_t(p.fin) * p.n_tiles * p.n + size_t(t) * p.n;
   const int ur = u0 + lr;
@@ -369,11 +369,11 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
   if (ur < p.m) {
     const float iu = inv[ul[ur]];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < CPT; ++j) {
       float sdot = 0.0f;
 #pragma unroll
-      for (int src = 0; src < kAS; ++src) sdot += x[src][j];
-      const int pa = p0 + tx + 16 * j;
+      for (int src = 0; src < AS; ++src) sdot += x[src][j];
+      const int pa = p0 + cx + TPR * j;
       if (pa < p.n_anc) {
         const int ia = al[pa];
         const float v = SIM == SPD_SIM_COS ? sdot * iu * inv[ia]
@@ -385,8 +385,8 @@ __global__ void __cluster_dims__(kAS, 1, 1) __launch_bounds__(256)
     }
   }
 #pragma unroll
-  for (int off = 8; off; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
-  if (tx == 0 && ur < p.m) {
+  for (int off = TPR / 2; off; off >>= 1) best = fmaxf(best, __shfl_xor_sync(0xffffffffu, best, off));
+  if (cx == 0 && ur < p.m) {
     const int iu = ul[ur];
     if (SIM == SPD_SIM_MSE) best = -(w.st1[so + iu] - best) / float(p.d);
     else if (SIM == SPD_SIM_KL) best = best - w.st2[so + iu];
@@ -1254,12 +1254,20 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
                           : p.sim == SPD_SIM_MSE ? rowstats_kernel<SPD_SIM_MSE> : rowstats_kernel<SPD_SIM_KL>,
                           dim3((p.n + 7) / 8, T), dim3(256), 0, st, p, attn, w));
   SPD_CUDA_TRY(launch_pdl(anchor_kernel, dim3(T), dim3(1024), 0, st, p, w));
-  if (p.n_anc > 0 && p.m > 0 && p.wa != 0.0f)
-    SPD_CUDA_TRY(launch_pdl(p.sim == SPD_SIM_COS ? anchor_sim_kernel<SPD_SIM_COS>
-                            : p.sim == SPD_SIM_MSE ? anchor_sim_kernel<SPD_SIM_MSE>
-                                                   : anchor_sim_kernel<SPD_SIM_KL>,
-                            dim3((p.m + 63) / 64 * kAS, (p.n_anc + 63) / 64, T), dim3(256), 0, st,
-                            p, w));
+  if (p.n_anc > 0 && p.m > 0 && p.wa != 0.0f) {
+    // the feature dimension over 8 CTAs while the tiles leave most SMs idle, else over 4
+    const dim3 g((p.m + 63) / 64, (p.n_anc + 63) / 64, T);
+    if (size_t(g.x) * g.y * T * 8 <= 2 * size_t(num_sms()))
+      SPD_CUDA_TRY(launch_pdl(p.sim == SPD_SIM_COS ? anchor_sim_kernel<SPD_SIM_COS, 8>
+                              : p.sim == SPD_SIM_MSE ? anchor_sim_kernel<SPD_SIM_MSE, 8>
+                                                     : anchor_sim_kernel<SPD_SIM_KL, 8>,
+                              dim3(g.x * 8, g.y, T), dim3(256), 0, st, p, w));
+    else
+      SPD_CUDA_TRY(launch_pdl(p.sim == SPD_SIM_COS ? anchor_sim_kernel<SPD_SIM_COS, 4>
+                              : p.sim == SPD_SIM_MSE ? anchor_sim_kernel<SPD_SIM_MSE, 4>
+                                                     : anchor_sim_kernel<SPD_SIM_KL, 4>,
+                              dim3(g.x * 4, g.y, T), dim3(256), 0, st, p, w));
+  }
   // K-means: the rows resident in shared memory over 16 CTAs per tile where they fit and all
   // tiles run in one wave of such clusters (latency); else re-read from L2 each pass by 8 CTAs per
   // tile, twice as many tiles at once (throughput)
