@@ -1586,7 +1586,11 @@ int gemm_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   // epilogues): there the single-CTA kernel runs.
   const int slots = sms / 2;  // pairs the GPU holds at once
   const long long pair_tiles = (long long)((p.n_out + 2 * kBM - 1) / (2 * kBM)) * a.n_ttiles;
-  const bool pair = a.tt >= 128 && !(p.epi != EPI_ADD_F32 && pair_tiles * 2 <= slots);
+  // Deterministic mode: residual GEMMs that few also take the single-CTA kernel, whose cluster
+  // reduction sums the split partials in rank order on every CTA of the cluster at once (the
+  // ordered stream-K fixup of the pair kernel leaves each tile's sum to one CTA).
+  const bool pair = a.tt >= 128 &&
+                    !((p.epi != EPI_ADD_F32 || deterministic()) && pair_tiles * 2 <= slots);
   // 256-row tiles in one CTA for token tiles of at most 64: their stages are mostly weights, and
   // two MMAs per token box double the weight bytes per stage (needs the row-major pointer)
   a.nh = (!pair && a.tt <= 64 && p.w) ? 2 : 1;

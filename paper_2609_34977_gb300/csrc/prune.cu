@@ -68,6 +68,14 @@ struct PruneWs {
   int* status;
 };
 
+// The outputs of a prune call (kind, cluster and scores optional).
+struct PruneOut {
+  int32_t* keep_idx;
+  uint8_t* kind;
+  int8_t* cluster;
+  float* scores;
+};
+
 namespace {
 
 __device__ __forceinline__ uint32_t ordered_key(float f) {
@@ -448,6 +456,104 @@ __device__ void compute_quotas(const int* sizes, int K, int n_cmp, int* quota) {
   }
 }
 
+// The fused tail of the K-means kernel: every CTA turns its tokens' accumulated terms into Eq. 3
+// scores (as score_kernel) and pushes their (cluster, score, index) keys into every CTA; each CTA
+// ranks its own tokens among all non-anchor keys and marks the selected ones in CTA 0, which
+// compacts the kept tokens in index order (as select_kernel). keys: 8 (m + 1) + n bytes of every
+// CTA's shared memory that nothing else reads any more (the resident rows); j0: this CTA's first
+// token of the tile's non-anchor list.
+template <int KC>
+__device__ void fused_select(const PruneDims& p, const PruneWs& w, const PruneOut& out,
+                             cg::cluster_group& cl, int rank, int t, int j0, int nl,
+                             const int8_t* asg, const int* idx, const float* av, float* sacc,
+                             const int* ncl, const float* ak, uint64_t* keys) {
+  const int m = p.m, K = p.K;
+  __shared__ int seg[SPD_MAX_CLUSTERS + 1];
+  __shared__ int quota[SPD_MAX_CLUSTERS];
+  __shared__ int tmp[32];
+  uint8_t* kept = reinterpret_cast<uint8_t*>(keys + m + 1);  // CTA 0: [n]
+  __syncthreads();  // every warp's terms of the last layer are in sacc
+  if (threadIdx.x == 0) {  // every CTA: segment offsets and the Eq. 2 quotas (same in all)
+    int sizes[SPD_MAX_CLUSTERS], q[SPD_MAX_CLUSTERS];
+    int acc = 0;
+    for (int k = 0; k < K; ++k) {
+      seg[k] = acc;
+      sizes[k] = ncl[k];
+      acc += ncl[k];
+    }
+    seg[K] = acc;
+    compute_quotas(sizes, K, p.n_cmp, q);
+    for (int k = 0; k < K; ++k) quota[k] = q[k];
+  }
+  uint64_t key[2];  // this thread's tokens jj = threadIdx.x + u blockDim.x (nl <= 2 blockDim.x)
+  for (int u = 0; u < 2; ++u) {
+    const int jj = threadIdx.x + u * blockDim.x;
+    key[u] = ~0ull;
+    if (jj < nl) {
+      const int k = asg[jj], cnt = ncl[k];
+      const float ai = av[jj];
+      float s;
+      if (cnt <= 1) {
+        s = p.wa * 2.0f * ai;
+      } else {
+        const float inv_c = 1.0f / float(cnt - 1);
+        s = sacc[jj] * inv_c + p.wa * (ai + (ak[k] - ai) * inv_c);
+      }
+      key[u] = (uint64_t(k) << 45) | (uint64_t(ordered_key(s)) << 13) | uint64_t(idx[jj]);
+    }
+  }
+  cl.sync();  // no CTA reads its resident rows any more
+  for (int u = 0; u < 2; ++u) {
+    const int jj = threadIdx.x + u * blockDim.x;
+    if (jj < nl)
+      for (int rr = 0; rr < KC; ++rr) cl.map_shared_rank(keys, rr)[j0 + jj] = key[u];
+  }
+  if (rank == 0)
+    for (int i = threadIdx.x; i < p.n; i += blockDim.x) kept[i] = uint8_t(w.role[size_t(t) * p.n + i]);
+  cl.sync();  // every CTA holds all m keys; CTA 0 the anchor flags
+  uint8_t* kept0 = cl.map_shared_rank(kept, 0);
+  for (int u = 0; u < 2; ++u) {
+    const int jj = threadIdx.x + u * blockDim.x;
+    if (jj >= nl) continue;
+    const uint64_t ki = key[u];
+    int r0 = 0, r1 = 0, r2 = 0, r3 = 0, j = 0;
+    for (; j + 4 <= m; j += 4) {
+      r0 += keys[j] < ki;
+      r1 += keys[j + 1] < ki;
+      r2 += keys[j + 2] < ki;
+      r3 += keys[j + 3] < ki;
+    }
+    for (; j < m; ++j) r0 += keys[j] < ki;
+    const int k = int(ki >> 45);
+    // the key at sorted position r of cluster k's segment is kept iff r - seg[k] < quota[k]
+    if (r0 + r1 + r2 + r3 - seg[k] < quota[k]) kept0[ki & 0x1fffu] = 2;
+    if (out.cluster) out.cluster[size_t(t) * p.n + (ki & 0x1fffu)] = int8_t(k);
+    if (out.scores) out.scores[size_t(t) * p.n + (ki & 0x1fffu)] = ordered_val(uint32_t(ki >> 13));
+  }
+  cl.sync();  // the selected flags are in CTA 0
+  if (rank != 0) return;
+  // compaction in index order: thread th owns tokens [th q, th q + q)
+  const int q = (p.n + blockDim.x - 1) / blockDim.x, base = threadIdx.x * q;
+  int nk = 0;
+  for (int u = 0; u < q; ++u)
+    if (base + u < p.n) nk += kept[base + u] != 0;
+  int pos = block_scan_excl(nk, tmp, nullptr);
+  for (int u = 0; u < q; ++u) {
+    const int i = base + u;
+    if (i >= p.n) break;
+    if (kept[i]) {
+      if (pos < p.keep) out.keep_idx[size_t(t) * p.keep + pos] = i;
+      else set_status(w.status, SPD_EINVAL);
+      ++pos;
+    }
+    if (out.kind) out.kind[size_t(t) * p.n + i] = kept[i];
+    if (kept[i] == 1) {
+      if (out.cluster) out.cluster[size_t(t) * p.n + i] = -1;
+      if (out.scores) out.scores[size_t(t) * p.n + i] = INFINITY;
+    }
+  }
+}
+
 // Row jj of this CTA's tokens: resident in shared memory (rows + jj D) or in global memory
 // (g + (row0 + idx[jj]) D), optionally scaled by scale[jj].
 struct RowAccess {
@@ -564,8 +670,14 @@ constexpr int kmeans_threads() { return KN == 4 ? 256 : 512; }
 
 // COS: the similarity kind is the cosine (the paper's); the MSE / KL ablations' extra sums are
 // compiled into the other instance only (the Lloyd loop is instruction-bound).
-template <int KC, bool RES, int KN, bool COS>
-__global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims p, PruneWs w) {
+// FUSED (RES and COS only): the kernel goes on to the Eq. 3 scores of its tokens, from the resident
+// rows of each layer and that layer's cluster sums pushed into every CTA, and the rank-0 CTA then
+// selects and compacts the kept tokens (the work of score_kernel and select_kernel, without their
+// launches and without reading the features again).
+template <int KC, bool RES, int KN, bool COS, bool FUSED = false>
+__global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims p, PruneWs w,
+                                                                       PruneOut out) {
+  static_assert(!FUSED || (RES && COS), "the fused tail reads resident rows of unit-norm scores");
   pdl_launch_dependents();
   pdl_wait();
   extern __shared__ __align__(16) float ksm[];
@@ -584,6 +696,8 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
   __shared__ float av[4096 / KC + 1];    // their a_j
   __shared__ float rinv[4096 / KC + 1];  // their 1 / ||F_l,j|| (cos) or st1 (MSE, KL) of the layer
   __shared__ int ncl[SPD_MAX_CLUSTERS];  // cluster sizes over the whole cluster of CTAs
+  __shared__ float ak[SPD_MAX_CLUSTERS];  // FUSED: the cluster's sums of a_j (rank order)
+  __shared__ float sacc[FUSED ? 4096 / KC + 1 : 1];  // FUSED: per token, sum_l w_l f_i.(S_l,k - f_i)
   __shared__ uint64_t rows_bar;
   cg::cluster_group cl = cg::this_cluster();
   const int rank = int(cl.block_rank());
@@ -593,6 +707,7 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
   const int* ul = w.ulist + size_t(t) * m;
   const size_t row0 = size_t(t) * p.n_tok + p.off;  // feature row of patch 0 of this tile
   const float* fin = p.feat[p.fin];
+  if (threadIdx.x < SPD_MAX_CLUSTERS) ncl[threadIdx.x] = 0;
   for (int jj = threadIdx.x; jj < nl; jj += blockDim.x) {
     idx[jj] = ul[j0 + jj];
     av[jj] = ordered_val(w.asim[size_t(t) * p.n + ul[j0 + jj]]);
@@ -799,14 +914,28 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
                     RowAccess{RES ? rows : nullptr, fl, row0, idx, D, cos_sim ? rinv : static_cast<float*>(nullptr)});
     cl.sync();
     float* csum = w.csum + (size_t(t) * p.L + l) * K * D;
-    cluster_column_reduce<KC>(cl, part, K, D, rank,
-                              [&](int k, int c, float sum) { csum[k * D + c] = sum; });
+    cluster_column_reduce<KC>(cl, part, K, D, rank, [&](int k, int c, float sum) {
+      csum[k * D + c] = sum;
+      if constexpr (FUSED)  // the layer's cluster sums into every CTA (the centroids are done)
+        for (int rr = 0; rr < KC; ++rr) cl.map_shared_rank(cent, rr)[k * D + c] = sum;
+    });
     if (!cos_sim && rank == 0 && warp == 1) {  // CTA sums added in rank order
       for (int k = 0; k < K; ++k) {
         const double sr = lane < KC ? cl.map_shared_rank(ssum_part, lane)[k] : 0.0;
         double a = 0.0;
         for (int rr = 0; rr < KC; ++rr) a += __shfl_sync(0xffffffffu, sr, rr);
         if (lane == 0) w.ssum[(size_t(t) * p.L + l) * 16 + k] = a;
+      }
+    }
+    if (FUSED && li == p.L - 1 && warp == 2) {
+      // every CTA: the cluster's sums of a_j over the CTAs, in rank order (lane r reads CTA r)
+      float ar[SPD_MAX_CLUSTERS];  // all of CTA lane's sums first (one remote round trip)
+      const float* peer = lane < KC ? cl.map_shared_rank(asum_part, lane) : nullptr;
+      for (int k = 0; k < K; ++k) ar[k] = peer ? peer[k] : 0.0f;
+      for (int k = 0; k < K; ++k) {
+        float a = 0.0f;
+        for (int rr = 0; rr < KC; ++rr) a += __shfl_sync(0xffffffffu, ar[k], rr);
+        if (lane == 0) ak[k] = a;
       }
     }
     if (li == p.L - 1 && rank == 0 && warp == 0) {
@@ -832,7 +961,29 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
       }
     }
     cl.sync();  // peers' shared memory is read above; keep it alive and unchanged until here
+    if constexpr (FUSED) {
+      // this CTA's tokens: f_i.(S_l,k - f_i) with f = F / |F| from the resident rows of layer l
+      const float wl = (l == p.fin) ? p.wf : p.w[l];
+      for (int jj = warp; jj < nl; jj += nw) {
+        if (li == 0 && lane == 0) sacc[jj] = 0.0f;
+        if (wl == 0.0f) continue;
+        const float* x = rows + size_t(jj) * D;
+        const float* sk = cent + size_t(asg[jj]) * D;
+        const float iv = rinv[jj];
+        float dot = 0.0f;
+        for (int c = 4 * lane; c < D; c += 128) {
+          const float4 xv = *reinterpret_cast<const float4*>(x + c);
+          const float4 sv = *reinterpret_cast<const float4*>(sk + c);
+          const float b0 = xv.x * iv, b1 = xv.y * iv, b2 = xv.z * iv, b3 = xv.w * iv;
+          dot += b0 * (sv.x - b0) + b1 * (sv.y - b1) + b2 * (sv.z - b2) + b3 * (sv.w - b3);
+        }
+        dot = warp_sum(dot);
+        if (lane == 0) sacc[jj] += wl * dot;
+      }
+    }
   }
+  if constexpr (FUSED) fused_select<KC>(p, w, out, cl, rank, t, j0, nl, asg, idx, av, sacc, ncl, ak,
+                                        reinterpret_cast<uint64_t*>(rows));
 }
 
 // ---- 6. per-token Eq. 3 scores ----------------------------------------------------------------
@@ -1152,9 +1303,11 @@ PruneWs carve(const PruneDims& p, Carve& cv) {
 constexpr size_t kResSmem = 200 * 1024;  // dynamic shared memory of the resident K-means
 int g_res_clusters = -1;                 // 16-CTA clusters of it the GPU holds at once
 
-template <int KC, bool RES, int KN>
-cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, size_t smem, cudaStream_t st) {
-  auto kern = p.sim == SPD_SIM_COS ? kmeans_kernel<KC, RES, KN, true> : kmeans_kernel<KC, RES, KN, false>;
+template <int KC, bool RES, int KN, bool FUSED = false>
+cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, const PruneOut& out, size_t smem,
+                          cudaStream_t st) {
+  auto kern = FUSED ? kmeans_kernel<KC, RES, KN, true, FUSED>
+              : p.sim == SPD_SIM_COS ? kmeans_kernel<KC, RES, KN, true> : kmeans_kernel<KC, RES, KN, false>;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(KC, p.n_tiles);
   cfg.blockDim = dim3(kmeans_threads<KN>());
@@ -1169,7 +1322,7 @@ cudaError_t launch_kmeans(const PruneDims& p, const PruneWs& w, size_t smem, cud
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, kern, p, w);
+  return cudaLaunchKernelEx(&cfg, kern, p, w, out);
 }
 
 // Kernel attributes (once per process) and whether 16-CTA clusters of the resident kernel fit.
@@ -1194,6 +1347,8 @@ int kmeans_setup() {
     if (err == cudaSuccess) err = streamed(kmeans_kernel<8, false, SPD_MAX_CLUSTERS, false>);
     if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, 4, false>);
     if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, SPD_MAX_CLUSTERS, false>);
+    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, 4, true, true>);
+    if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, SPD_MAX_CLUSTERS, true, true>);
     g_res_clusters = 0;
     if (err == cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
@@ -1275,21 +1430,33 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
   const size_t cent_bytes = size_t(2) * p.K * p.d * sizeof(float);
   const size_t res_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float) + cent_bytes;
   const bool res = p.m > 0 && res_bytes <= kResSmem && g_res_clusters > 0 && T <= g_res_clusters;
-  if (res && p.K == 4)
-    SPD_CUDA_TRY((launch_kmeans<16, true, 4>(p, w, res_bytes, st)));
+  // resident rows and the cosine kind: scores, selection and compaction in the same kernel (CTA 0's
+  // row buffer holds the m sort keys and the n kept flags by then)
+  const size_t row_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float);
+  const bool fused = res && p.sim == SPD_SIM_COS && (p.m + 15) / 16 <= 512 &&
+                     row_bytes >= size_t(8) * (p.m + 1) + p.n;
+  const PruneOut out{keep_idx, kind, cluster, scores};
+  if (fused && p.K == 4)
+    SPD_CUDA_TRY((launch_kmeans<16, true, 4, true>(p, w, out, res_bytes, st)));
+  else if (fused)
+    SPD_CUDA_TRY((launch_kmeans<16, true, SPD_MAX_CLUSTERS, true>(p, w, out, res_bytes, st)));
+  else if (res && p.K == 4)
+    SPD_CUDA_TRY((launch_kmeans<16, true, 4>(p, w, out, res_bytes, st)));
   else if (res)
-    SPD_CUDA_TRY((launch_kmeans<16, true, SPD_MAX_CLUSTERS>(p, w, res_bytes, st)));
+    SPD_CUDA_TRY((launch_kmeans<16, true, SPD_MAX_CLUSTERS>(p, w, out, res_bytes, st)));
   else if (p.K == 4)
-    SPD_CUDA_TRY((launch_kmeans<8, false, 4>(p, w, cent_bytes, st)));
+    SPD_CUDA_TRY((launch_kmeans<8, false, 4>(p, w, out, cent_bytes, st)));
   else
-    SPD_CUDA_TRY((launch_kmeans<8, false, SPD_MAX_CLUSTERS>(p, w, cent_bytes, st)));
-  if (p.m > 0) {
-    auto score = p.sim == SPD_SIM_COS ? score_kernel<SPD_SIM_COS>
-                 : p.sim == SPD_SIM_MSE ? score_kernel<SPD_SIM_MSE> : score_kernel<SPD_SIM_KL>;
-    SPD_CUDA_TRY(launch_pdl(score, dim3((p.m + 7) / 8, T), dim3(256), 0, st, p, w));
+    SPD_CUDA_TRY((launch_kmeans<8, false, SPD_MAX_CLUSTERS>(p, w, out, cent_bytes, st)));
+  if (!fused) {
+    if (p.m > 0) {
+      auto score = p.sim == SPD_SIM_COS ? score_kernel<SPD_SIM_COS>
+                   : p.sim == SPD_SIM_MSE ? score_kernel<SPD_SIM_MSE> : score_kernel<SPD_SIM_KL>;
+      SPD_CUDA_TRY(launch_pdl(score, dim3((p.m + 7) / 8, T), dim3(256), 0, st, p, w));
+    }
+    SPD_CUDA_TRY(launch_pdl(select_kernel, dim3(T), dim3(1024), 0, st, p, w, keep_idx, kind, cluster,
+                            scores));
   }
-  SPD_CUDA_TRY(launch_pdl(select_kernel, dim3(T), dim3(1024), 0, st, p, w, keep_idx, kind, cluster,
-                          scores));
   // algorithmic work per tile: every tapped layer's features and the attention read once, the
   // kept indices written; anchor similarities (n - N_anc) N_anc d multiply-adds
   trace_end(slot, st, TR_PRUNE, 2.0 * T * double(p.m) * p.n_anc * p.d,
