@@ -3,8 +3,8 @@
 //   rowstats     a_v = head-mean of the attention (Sec. 4.1.1); 1/||F_l,i|| for every tapped layer
 //                (and ||F_l,i||^2, or the log-sum-exp and negentropy of softmax(F_l,i), for the
 //                MSE and KL ablations of sim)
-//   anchors      top-N_anc of a_v by a bitonic sort of (a_v desc, index asc) keys (Eq. 1);
-//                stable lists of anchor and non-anchor tokens by block prefix sums
+//   anchors      top-N_anc of a_v by ranking (a_v desc, index asc) keys (Eq. 1); stable lists of
+//                anchor and non-anchor tokens by block prefix sums
 //   anchor_sim   a_i = max_p cos(F^L_i, F^L_p) over anchors: 64 x 64 register-tiled fp32 products,
 //                the feature dimension split over a cluster of 4 (8 for few tiles) CTAs whose partial tiles are summed
 //                in rank order through distributed shared memory; max via atomicMax on
@@ -22,6 +22,8 @@
 //                per-cluster sums of ||F_j||^2 or of the log-sum-exps)
 //   select       per cluster the N_k lowest (score, index) keys; kept = anchors + selected, compacted
 //                in ascending index order
+// Where the rows are resident and the similarity is the cosine, the K-means kernel goes on to the
+// scores and the selection itself (fused_select): four launches instead of six.
 // All reductions run in a fixed order, so repeated runs give identical bits.
 #include <cuda_bf16.h>
 #include <math.h>
