@@ -179,19 +179,24 @@ __device__ __forceinline__ SegPlan seg_plan(int u0, int u1, int n_kb) {
   }
   return p;
 }
-// Data-parallel + remainder schedule: the first rem_tiles tiles are split in K over every work item,
-// item wc owning the remainder units [wc U_r / G, (wc + 1) U_r / G) (U_r = rem_tiles n_kb, G the
-// work items; the contributions of a remainder tile meet in an fp32 accumulation buffer at L2), then
-// the item runs the whole tiles rem_tiles + wc W .. + W - 1, which need no fixup. The remainder
-// comes first, so its fixups overlap the whole tiles' main loops.
+// Data-parallel + remainder schedule: the first rem_tiles tiles are split in K over the work items,
+// each remainder tile over a contiguous group of G / rem_tiles items (G the work items) so that no
+// item holds parts of two remainder tiles (a second remainder segment would wait for the first
+// one's accumulator to drain); the contributions of a remainder tile meet in an fp32 accumulation
+// buffer at L2. Then the item runs the whole tiles rem_tiles + wc W .. + W - 1, which need no
+// fixup. The remainder comes first, so its fixups overlap the whole tiles' main loops.
 __device__ __forceinline__ SegPlan seg_plan_dpr(int wc, int grid, int rem_tiles, int whole, int n_kb) {
   SegPlan p{};
   p.dpr = true;
   p.n_kb = n_kb;
-  const long long ur = (long long)rem_tiles * n_kb;
-  p.u0 = int(wc * ur / grid);
-  p.u1 = int((wc + 1) * ur / grid);
-  p.n_rsegs = p.u0 < p.u1 ? (p.u1 - 1) / n_kb - p.u0 / n_kb + 1 : 0;
+  int rt = int((long long)wc * rem_tiles / grid);  // this item's remainder tile
+  while (rt + 1 < rem_tiles && (long long)(rt + 1) * grid / rem_tiles <= wc) ++rt;
+  while (rt > 0 && (long long)rt * grid / rem_tiles > wc) --rt;
+  const int g0 = int((long long)rt * grid / rem_tiles);
+  const int ng = int((long long)(rt + 1) * grid / rem_tiles) - g0, li = wc - g0;
+  p.u0 = rt * n_kb + li * n_kb / ng;
+  p.u1 = rt * n_kb + (li + 1) * n_kb / ng;
+  p.n_rsegs = p.u0 < p.u1 ? 1 : 0;
   p.whole0 = rem_tiles + wc * whole;
   p.n_whole = whole;
   p.count = p.n_rsegs + p.n_whole;
