@@ -174,12 +174,14 @@ def build_model(torch, N, synth, device, layers=32):
 
 
 def count_launches(pipe, mask, dense):
-    """Kernels of one step: MSV-Prune (6) and the gather, projector (2), text scatter, residual
-    initialisation, final norm and LM head (one matrix-vector launch with the norm fused for at most
-    four sequences); per layer RMSNorm and the QKV GEMM, attention and O when a token attends,
-    RMSNorm, gate/up and down when a token runs the FFN."""
+    """Kernels of one step: MSV-Prune (as many as the library reports for the configuration) and the
+    gather, projector (2), text scatter, residual initialisation, final norm and LM head (one
+    matrix-vector launch with the norm fused for at most four sequences); per layer RMSNorm and the
+    QKV GEMM, attention and O when a token attends, RMSNorm, gate/up and down when a token runs the
+    FFN."""
+    from paper_2609_34977_gb300 import _native as N
     L = mask.shape[0] if mask is not None else pipe.model.cfg["n_layers"]
-    n = (0 if dense else 7) + 2 + 1 + 1 + (1 if pipe.B <= 4 else 2)
+    n = (0 if dense else N.spd_prune_launches(pipe.prune_cfg) + 1) + 2 + 1 + 1 + (1 if pipe.B <= 4 else 2)
     for l in range(L):
         bits = mask[l] if mask is not None else np.zeros(pipe.T, np.uint8)
         n += 2 + (2 if ((bits & 1) == 0).any() else 0) + (3 if ((bits & 2) == 0).any() else 0)
@@ -710,7 +712,8 @@ def main():
     kernels = {k: {"launches_per_step": c["launches"] / a.steps, "ms_per_step": c["ms"] / a.steps,
                    "GB/s": c["bytes"] / max(c["ms"], 1e-9) / 1e6,
                    "TFLOP/s": c["flops"] / max(c["ms"], 1e-9) / 1e9} for k, c in cls.items()}
-    kernels["prune"]["timing"] = "one CUDA event pair around each spd_prune call (six kernels)"
+    kernels["prune"]["timing"] = (f"one CUDA event pair around each spd_prune call "
+                                  f"({N.spd_prune_launches(spider.prune_cfg)} kernels)")
 
     # the dense step's GEMMs (640 token rows, above the ridge) against the tensor roofline
     ms_dense_st = timed(dense, None, a.steps, 1, stamp=True)

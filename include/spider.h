@@ -138,6 +138,13 @@ typedef struct {
 /* Bytes of device workspace spd_prune needs for `cfg` (0 if cfg is invalid). */
 size_t spd_prune_workspace_size(const spd_prune_cfg* cfg);
 
+/* Number of kernels spd_prune enqueues for `cfg` on the current device (measurement support, no
+ * counterpart in the paper): 4 where the K-means kernel also scores, selects and compacts (rows
+ * resident in shared memory, cosine similarity), else 6; one less without the anchor maximum
+ * (no anchors, or the ablation without it), one less without non-anchor tokens. Negative
+ * spd_status on an invalid configuration. */
+int spd_prune_launches(const spd_prune_cfg* cfg);
+
 /* MSV-Prune of every tile (Sec. 4.1; Alg. 1 stage 1):
  *   a_v = head-mean of the attention (Sec. 4.1.1); anchors = the N_anc tokens of largest a_v
  *   (Eq. 1, ties to the lower index); K-means (Lloyd, squared Euclidean, seeds at the quantiles

@@ -20,7 +20,7 @@ EPI_F32, EPI_BF16, EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_ADD_F32 = 0, 1, 2, 3, 
 
 # every symbol include/spider.h declares
 EXPORTS = ("spd_last_error", "spd_workspace_status", "spd_selftest_bounded_wait",
-           "spd_prune_workspace_size", "spd_prune", "spd_received_attention_workspace_size",
+           "spd_prune_workspace_size", "spd_prune_launches", "spd_prune", "spd_received_attention_workspace_size",
            "spd_received_attention", "spd_gather_rows_bf16", "spd_model_create",
            "spd_model_destroy", "spd_plan_adaptive", "spd_plan_static", "spd_project_workspace_size",
            "spd_project", "spd_scatter_rows", "spd_attention_workspace_size", "spd_attention",
@@ -100,6 +100,7 @@ def lib():
             "spd_workspace_status": (i, [vp, vp, C.POINTER(i)]),
             "spd_selftest_bounded_wait": (i, [vp, ll, vp]),
             "spd_prune_workspace_size": (sz, [C.POINTER(PruneCfg)]),
+            "spd_prune_launches": (i, [C.POINTER(PruneCfg)]),
             "spd_prune": (i, [C.POINTER(PruneCfg), C.POINTER(vp), vp, vp, vp, vp, vp, vp, sz, vp]),
             "spd_received_attention_workspace_size": (sz, [i, i, i]),
             "spd_received_attention": (i, [vp, i, i, i, vp, vp, i, vp, vp, sz, vp]),
@@ -247,6 +248,13 @@ def prune_cfg(n_tiles, n_tok, d_feat, n_layers, final_layer, n_heads, keep, *, h
 
 def spd_prune_workspace_size(cfg: PruneCfg) -> int:
     return int(lib().spd_prune_workspace_size(C.byref(cfg)))
+
+
+def spd_prune_launches(cfg: PruneCfg) -> int:
+    """Kernels one spd_prune call with cfg enqueues on the current device."""
+    n = int(lib().spd_prune_launches(C.byref(cfg)))
+    _check(min(n, 0))
+    return n
 
 
 def spd_prune(cfg, feats, attn, keep_idx, kind=None, cluster=None, scores=None, ws=None, stream=None):

@@ -1377,10 +1377,40 @@ int kmeans_setup() {
   return SPD_OK;
 }
 
+// Which kernels spd_prune launches for p (after kmeans_setup).
+struct PrunePlan {
+  bool anchor_sim, res, fused;
+  int launches;
+};
+PrunePlan prune_plan(const PruneDims& p) {
+  PrunePlan q;
+  q.anchor_sim = p.n_anc > 0 && p.m > 0 && p.wa != 0.0f;
+  const size_t cent_bytes = size_t(2) * p.K * p.d * sizeof(float);
+  const size_t res_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float) + cent_bytes;
+  // K-means: the rows resident in shared memory over 16 CTAs per tile where they fit and all tiles
+  // run in one wave of such clusters (latency); else re-read from L2 each pass by 8 CTAs per tile,
+  // twice as many tiles at once (throughput)
+  q.res = p.m > 0 && res_bytes <= kResSmem && g_res_clusters > 0 && p.n_tiles <= g_res_clusters;
+  // resident rows and the cosine kind: scores, selection and compaction in the same kernel (CTA 0's
+  // row buffer holds the m sort keys and the n kept flags by then)
+  const size_t row_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float);
+  q.fused = q.res && p.sim == SPD_SIM_COS && (p.m + 15) / 16 <= 512 &&
+            row_bytes >= size_t(8) * (p.m + 1) + p.n;
+  q.launches = 2 + int(q.anchor_sim) + 1 + (q.fused ? 0 : int(p.m > 0) + 1);
+  return q;
+}
+
 }  // namespace
 }  // namespace spd
 
 using namespace spd;
+
+extern "C" int spd_prune_launches(const spd_prune_cfg* cfg) {
+  PruneDims p;
+  if (int rc = validate(cfg, &p)) return rc;
+  if (int rc = kmeans_setup()) return rc;
+  return prune_plan(p).launches;
+}
 
 extern "C" size_t spd_prune_workspace_size(const spd_prune_cfg* cfg) {
   PruneDims p;
@@ -1411,7 +1441,9 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
                           : p.sim == SPD_SIM_MSE ? rowstats_kernel<SPD_SIM_MSE> : rowstats_kernel<SPD_SIM_KL>,
                           dim3((p.n + 7) / 8, T), dim3(256), 0, st, p, attn, w));
   SPD_CUDA_TRY(launch_pdl(anchor_kernel, dim3(T), dim3(1024), 0, st, p, w));
-  if (p.n_anc > 0 && p.m > 0 && p.wa != 0.0f) {
+  if (int rc = kmeans_setup()) return rc;
+  const PrunePlan plan = prune_plan(p);
+  if (plan.anchor_sim) {
     // the feature dimension over 8 CTAs while the tiles leave most SMs idle, else over 4
     const dim3 g((p.m + 63) / 64, (p.n_anc + 63) / 64, T);
     if (size_t(g.x) * g.y * T * 8 <= 2 * size_t(num_sms()))
@@ -1425,32 +1457,22 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
                                                      : anchor_sim_kernel<SPD_SIM_KL, 4>,
                               dim3(g.x * 4, g.y, T), dim3(256), 0, st, p, w));
   }
-  // K-means: the rows resident in shared memory over 16 CTAs per tile where they fit and all
-  // tiles run in one wave of such clusters (latency); else re-read from L2 each pass by 8 CTAs per
-  // tile, twice as many tiles at once (throughput)
-  if (int rc = kmeans_setup()) return rc;
   const size_t cent_bytes = size_t(2) * p.K * p.d * sizeof(float);
   const size_t res_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float) + cent_bytes;
-  const bool res = p.m > 0 && res_bytes <= kResSmem && g_res_clusters > 0 && T <= g_res_clusters;
-  // resident rows and the cosine kind: scores, selection and compaction in the same kernel (CTA 0's
-  // row buffer holds the m sort keys and the n kept flags by then)
-  const size_t row_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float);
-  const bool fused = res && p.sim == SPD_SIM_COS && (p.m + 15) / 16 <= 512 &&
-                     row_bytes >= size_t(8) * (p.m + 1) + p.n;
   const PruneOut out{keep_idx, kind, cluster, scores};
-  if (fused && p.K == 4)
+  if (plan.fused && p.K == 4)
     SPD_CUDA_TRY((launch_kmeans<16, true, 4, true>(p, w, out, res_bytes, st)));
-  else if (fused)
+  else if (plan.fused)
     SPD_CUDA_TRY((launch_kmeans<16, true, SPD_MAX_CLUSTERS, true>(p, w, out, res_bytes, st)));
-  else if (res && p.K == 4)
+  else if (plan.res && p.K == 4)
     SPD_CUDA_TRY((launch_kmeans<16, true, 4>(p, w, out, res_bytes, st)));
-  else if (res)
+  else if (plan.res)
     SPD_CUDA_TRY((launch_kmeans<16, true, SPD_MAX_CLUSTERS>(p, w, out, res_bytes, st)));
   else if (p.K == 4)
     SPD_CUDA_TRY((launch_kmeans<8, false, 4>(p, w, out, cent_bytes, st)));
   else
     SPD_CUDA_TRY((launch_kmeans<8, false, SPD_MAX_CLUSTERS>(p, w, out, cent_bytes, st)));
-  if (!fused) {
+  if (!plan.fused) {
     if (p.m > 0) {
       auto score = p.sim == SPD_SIM_COS ? score_kernel<SPD_SIM_COS>
                    : p.sim == SPD_SIM_MSE ? score_kernel<SPD_SIM_MSE> : score_kernel<SPD_SIM_KL>;

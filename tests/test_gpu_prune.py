@@ -249,3 +249,14 @@ def test_largest_accepted_tile_received_form_with_guard_bands():
     assert torch.all(out_b[0] == 3.0) and torch.all(out_b[1025] == 3.0)
     want = torch.from_numpy(v["feats"][1][0][res[0]["keep_idx"]]).to(torch.bfloat16)
     assert torch.equal(out_b[1:1025].cpu(), want)
+
+
+def test_launch_count_query_follows_the_dispatch():
+    # spd_prune_launches: 4 kernels where K-means also scores, selects and compacts (one LLaVA tile,
+    # cosine), 6 for the ablation kinds and for more tiles than one wave of resident clusters, one
+    # less without anchors
+    one = N.prune_cfg(1, 577, 1024, 2, 1, 16, 192)
+    assert N.spd_prune_launches(one) == 4
+    assert N.spd_prune_launches(N.prune_cfg(1, 577, 1024, 2, 1, 16, 192, sim="mse")) == 6
+    assert N.spd_prune_launches(N.prune_cfg(64, 577, 1024, 2, 1, 16, 64)) == 6
+    assert N.spd_prune_launches(N.prune_cfg(1, 577, 1024, 2, 1, 16, 192, anchor_ratio=0.0)) == 3
