@@ -1537,10 +1537,11 @@ int gemv_run(const GemmProblem& p, const GemmScratch& s, cudaStream_t stream) {
   a.vec_red = vec_red_ok(p);
   a.determ = deterministic();
   const int groups = (p.n_out + 31) / 32, C = p.k / kGemvChunk;
-  // residual epilogues split K until about two CTAs per SM stream (each at least one chunk column)
+  // residual epilogues split K until about one CTA per SM streams (each at least one chunk column;
+  // two per SM measured slower at the decoder's O and down shapes: shorter rows per CTA)
   int ksplit = 1;
   if (p.epi == EPI_ADD_F32 && !a.determ)
-    while (groups * ksplit < 2 * num_sms() && ksplit * 2 <= C && ksplit < 8) ksplit *= 2;
+    while (groups * ksplit < num_sms() && ksplit * 2 <= C && ksplit < 8) ksplit *= 2;
   const bool one = p.n_tok == 1;
   const int nt = one ? 1 : kGemvTok;
   const size_t smem = size_t(nt) * ((C + ksplit - 1) / ksplit) * kGemvChunk * sizeof(uint16_t);
