@@ -3,7 +3,7 @@
 TEST INFRASTRUCTURE. Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg may import
 this module. It shares no code with the CUDA path.
 
-The paper does not describe the decoder beyond "Attention and FFN sub-layers". The architecture
+The paper does not describe the decoder beyond its attention and FFN sub-layers. The architecture
 is LLaMA-style, from the models it evaluates (LLaVA-1.5/NeXT on Vicuna-7B, Qwen2-style decoders):
 RMSNorm, rotary position embedding (rotate-half), causal multi-head or grouped-query attention,
 SwiGLU FFN, no biases. LLaVA's projector is Linear-GELU-Linear with biases.
@@ -90,7 +90,7 @@ def gelu(x):
 
 
 def project(model, vis, round_fn=bf16_round):
-    """LLaVA MLP projector (§2 "trainable connector"): Linear(d_vis->d_proj)+GELU, Linear(->D)."""
+    """LLaVA MLP projector (the connector of §2): Linear(d_vis->d_proj)+GELU, Linear(->D)."""
     p = model["proj"]
     hid = round_fn(gelu(np.asarray(vis, dtype=np.float64) @ p["w1"].T + p["b1"]))
     return round_fn(hid @ p["w2"].T + p["b2"])
