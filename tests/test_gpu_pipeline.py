@@ -92,3 +92,35 @@ def test_whole_step_entry_with_host_or_device_buffers(host):
     cu = [0, keep + 16, T]
     _, lg_o = od.prefill(om, x, cu, mask)
     assert rowwise_rel(logits.cpu().numpy(), lg_o) < TOL
+
+
+def test_whole_step_entry_equals_the_staged_calls_at_llava_width():
+    # spd_step with pinned host buffers at the LLaVA-1.5 shape (one tile, keep 192, projector
+    # 1024 -> 4096 -> 4096, 64 text tokens, 2 full-width decoder layers with a skip plan) against the
+    # same stages called one by one (SpiderPrefill): bit-identical logits in deterministic mode
+    L, keep, n_text = 2, 192, 64
+    cfg = dict(synth.LLAVA_7B_DECODER, n_layers=L, vocab=4096)
+    w = synth.decoder_weights(20261501, cfg, device="cuda")
+    model = N.SpdModel(cfg, w)
+    seed, v, res = conditioned_vision(20261510, 1, 576, 1024, 2, 16, keep, 1)
+    pipe = SpiderPrefill(model, n_patch=576, has_cls=True, d_vis=1024, n_feat_layers=2, final_layer=1,
+                         n_heads_vis=16, attn_form=0, keep=keep, tiles_per_req=[1], text_lens=[n_text])
+    admit, target = synth.adaptive_plan(seed, L, pipe.token_is_visual, 0.9,
+                                        synth.skip_targets("llava-1.5-7b")[:L], 0, L)
+    mask = N.spd_plan_adaptive(L, admit, target)
+    text = synth.text_embeddings(seed, n_text, 4096)
+    tx = torch.from_numpy(text.view(np.int16)).view(torch.bfloat16)
+    pc = N.prune_cfg(1, 577, 1024, 2, 1, 16, keep)
+    ws = torch.zeros(N.spd_step_workspace_size(model, pc, [1], [n_text]), dtype=torch.uint8, device="cuda")
+    feats_h = [torch.from_numpy(f).pin_memory() for f in v["feats"]]
+    attn_h = torch.from_numpy(v["attn"]).pin_memory()
+    logits_h = torch.full((1, 4096), float("nan")).pin_memory()
+    N.spd_set_deterministic(1)
+    try:
+        ref = pipe.run([f.cuda() for f in feats_h], attn_h.cuda(), tx.cuda(), mask).clone()
+        N.spd_step(model, pc, [1], [n_text], feats_h, attn_h, tx.pin_memory(), mask, logits_h, ws)
+        torch.cuda.synchronize()
+    finally:
+        N.spd_set_deterministic(0)
+    assert pipe.status() == 0 and N.spd_step_status(ws, model, pc, [1], [n_text]) == 0
+    assert torch.equal(logits_h, ref.cpu())
