@@ -10,8 +10,10 @@
 //   warps 0-3  softmax: thread r owns query row r (TMEM lane r); online softmax in fp32 with exp2;
 //              P rounded to bf16 into shared memory as a K-major swizzled operand; O rescaled in
 //              TMEM when a row's running maximum grows; at the end O / l goes to HBM in bf16
-// S of block j + 1 is computed while the softmax of block j runs. A query at position p sees keys
-// 0..p of its own sequence. Every wait is bounded (status SPD_ETIMEOUT, no hang).
+// S alternates between two TMEM buffers, so S of block j + 1 is computed while the softmax of
+// block j reads block j's (two passes: the maximum, then the exponentials, sum and P). A query at
+// position p sees keys 0..p of its own sequence. Every wait is bounded (status SPD_ETIMEOUT, no
+// hang).
 #include <cuda_bf16.h>
 #include <math.h>
 #include <stdint.h>
@@ -61,12 +63,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + L::bars);
   uint64_t* kv_full = q_full + 1;   // [2] K and V block landed
   uint64_t* kv_empty = q_full + 3;  // [2] its PV product has completed
-  uint64_t* s_full = q_full + 5;    // S of the current block is in TMEM
-  uint64_t* s_free = q_full + 6;    // the softmax warps have read S
-  uint64_t* p_full = q_full + 7;    // P written and O rescaled
-  uint64_t* o_done = q_full + 8;    // PV product of the current block completed
-  uint64_t* drain = q_full + 9;     // every MMA completed
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 10);
+  uint64_t* s_full = q_full + 5;    // [2] S of block j is in TMEM buffer j % 2
+  uint64_t* s_free = q_full + 7;    // [2] the softmax warps have read S buffer j % 2
+  uint64_t* p_full = q_full + 9;    // P written and O rescaled
+  uint64_t* o_done = q_full + 10;   // PV product of the current block completed
+  uint64_t* drain = q_full + 11;    // every MMA completed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 12);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -78,8 +80,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&kv_full[s], 1);
       mbar_init(&kv_empty[s], 1);
     }
-    mbar_init(s_full, 1);
-    mbar_init(s_free, 4);  // one arrival per softmax warp
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&s_free[b], 4);  // one arrival per softmax warp
+    }
     mbar_init(p_full, 4);
     mbar_init(o_done, 1);
     mbar_init(drain, 1);
@@ -89,14 +93,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&map_kv);
   }
   if (warp == 4) {
-    tmem_alloc(tmem_slot, 256);  // S: columns [0, 128); O: [128, 128 + HD)
+    tmem_alloc(tmem_slot, 512);  // S: two buffers, columns [0, 128) and [128, 256); O: [256, 256 + HD)
     tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t t_s = tmem, t_o = tmem + 128;
+  const uint32_t t_o = tmem + 256;  // S buffer b at tmem + 128 b
 
   // Nothing written by an earlier kernel of the stream is read before the grid dependency wait:
   // under programmatic overlap this kernel's prologue may run while several earlier kernels are
@@ -146,15 +150,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue_s = [&](int j) -> bool {
         const int s = j & 1;
         if (!mbar_wait(&kv_full[s], (j >> 1) & 1, abort_flag, budget)) return false;
-        if (j > 0 && !mbar_wait(s_free, (j - 1) & 1, abort_flag, budget)) return false;
+        // S buffer s was last read by the softmax of block j - 2
+        if (j > 1 && !mbar_wait(&s_free[s], ((j >> 1) - 1) & 1, abort_flag, budget)) return false;
         tc_fence_after();
         const uint32_t sk = smem_u32(smem + L::k + s * L::kChunks * kBox);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
-          mma_bf16(t_s, sdesc_k128(sq + off), sdesc_k128(sk + off), id_s, kk > 0 ? 1u : 0u);
+          mma_bf16(tmem + 128 * s, sdesc_k128(sq + off), sdesc_k128(sk + off), id_s, kk > 0 ? 1u : 0u);
         }
-        mma_commit(s_full);
+        mma_commit(&s_full[s]);
         return true;
       };
       if (ok) ok = issue_s(0);
@@ -188,43 +193,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     float m_run = -INFINITY, l_run = 0.0f;
     bool ok = true;
     for (int j = 0; j < nkb; ++j) {
-      if (!(ok = __all_sync(0xffffffffu, mbar_wait(s_full, j & 1, abort_flag, budget)))) break;
+      const int sb = j & 1;
+      if (!(ok = __all_sync(0xffffffffu, mbar_wait(&s_full[sb], (j >> 1) & 1, abort_flag, budget))))
+        break;
       tc_fence_after();
-      float s[kTK];
-#pragma unroll
+      const uint32_t t_s = tmem + 128 * sb + lanes;
+      const int kb = j * kTK;
+      // Two passes over the block's S row, 32 columns at a time in rolled loops (small code; the
+      // fully unrolled single pass held all 128 values in 254 registers and its first run cost
+      // 3 us against 1.4 for the second block): the row maximum, then 2^(s - m), the row sum and
+      // P. The next block's S goes to the other TMEM buffer meanwhile.
+      float mx = -INFINITY;
+#pragma unroll 1
       for (int c = 0; c < kTK / 32; ++c) {
         float v[32];
-        tmem_ld32(t_s + lanes + c * 32, v);
+        tmem_ld32(t_s + c * 32, v);
+        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-        for (int i = 0; i < 32; ++i) s[c * 32 + i] = v[i];
+        for (int i = 0; i < 32; ++i) {
+          const float x = (kb + c * 32 + i <= my_pos) ? v[i] * scale_log2 : -INFINITY;
+          m4[i & 3] = fmaxf(m4[i & 3], x);
+        }
+        mx = fmaxf(mx, fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])));
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(s_free);
-      const int kb = j * kTK;
-      // eight independent max / sum chains (one warp per sub-partition: latency, not throughput)
-      float mx8[8], rs8[8];
-#pragma unroll
-      for (int c = 0; c < 8; ++c) mx8[c] = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < kTK; ++i) {
-        s[i] = (kb + i <= my_pos) ? s[i] * scale_log2 : -INFINITY;
-        mx8[i & 7] = fmaxf(mx8[i & 7], s[i]);
-      }
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
       const float m_new = fmaxf(m_run, mx);  // finite: block 0 holds key 0 <= every position
       const float corr = exp2f(m_run - m_new);  // 0 on the first block
-#pragma unroll
-      for (int c = 0; c < 8; ++c) rs8[c] = 0.0f;
-#pragma unroll
-      for (int i = 0; i < kTK; ++i) {
-        s[i] = exp2f(s[i] - m_new);
-        rs8[i & 7] += s[i];
-      }
-      const float rs = ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
-      l_run = l_run * corr + rs;
-      m_run = m_new;
       if (j > 0) {
         // the previous PV product has completed: P's buffer is free and O can be rescaled
         if (!(ok = __all_sync(0xffffffffu, mbar_wait(o_done, (j - 1) & 1, abort_flag, budget))))
@@ -243,13 +236,33 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // P in bf16: row r of a K-major operand in the 128-byte swizzle layout (16-byte unit u of
       // the row at position u ^ (r % 8)), keys [0, 64) and [64, 128) in two boxes
+      float rs = 0.0f;
+#pragma unroll 1
+      for (int c = 0; c < kTK / 32; ++c) {
+        float v[32];
+        tmem_ld32(t_s + c * 32, v);
+        float r4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-      for (int u = 0; u < kTK / 8; ++u) {
-        const uint4 w = make_uint4(pack_bf16(s[8 * u], s[8 * u + 1]), pack_bf16(s[8 * u + 2], s[8 * u + 3]),
-                                   pack_bf16(s[8 * u + 4], s[8 * u + 5]),
-                                   pack_bf16(s[8 * u + 6], s[8 * u + 7]));
-        *reinterpret_cast<uint4*>(prow + (u >> 3) * kBox + (((u & 7) ^ (r & 7)) << 4)) = w;
+        for (int i = 0; i < 32; ++i) {
+          const float x = (kb + c * 32 + i <= my_pos) ? v[i] * scale_log2 : -INFINITY;
+          v[i] = exp2f(x - m_new);
+          r4[i & 3] += v[i];
+        }
+        rs += (r4[0] + r4[1]) + (r4[2] + r4[3]);
+#pragma unroll
+        for (int uu = 0; uu < 4; ++uu) {
+          const int u = 4 * c + uu;
+          const uint4 w = make_uint4(pack_bf16(v[8 * uu], v[8 * uu + 1]), pack_bf16(v[8 * uu + 2], v[8 * uu + 3]),
+                                     pack_bf16(v[8 * uu + 4], v[8 * uu + 5]),
+                                     pack_bf16(v[8 * uu + 6], v[8 * uu + 7]));
+          *reinterpret_cast<uint4*>(prow + (u >> 3) * kBox + (((u & 7) ^ (r & 7)) << 4)) = w;
+        }
       }
+      l_run = l_run * corr + rs;
+      m_run = m_new;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[sb]);  // S buffer sb read (both passes)
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
@@ -291,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncwarp();
   tc_fence_after();
-  if (warp == 4) tmem_dealloc(tmem, 256);
+  if (warp == 4) tmem_dealloc(tmem, 512);
   if (threadIdx.x == 0) stamp_end(stamp);
 }
 
