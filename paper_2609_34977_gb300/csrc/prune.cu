@@ -748,7 +748,10 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
     if (threadIdx.x == 0) changed = 0;
     __syncthreads();
     bool done_assign = false;
-    if constexpr (KN == 4) {
+    // K = 4 with the rows resident: the centroids in registers (242 registers a thread, one CTA an
+    // SM). The L2-streaming form takes the loop below instead: at 119 registers two of its CTAs
+    // share an SM, which hides more of the row loads' latency (64 tiles: 780 -> 606 us a call).
+    if constexpr (KN == 4 && RES) {
       if (D <= 1024) {
         done_assign = true;
         // lane's columns 4 lane + 128 j (j < 8) of the four centroids in registers
