@@ -11,7 +11,8 @@
 //                order-preserving integer keys (exact, order independent)
 //   kmeans       one thread-block cluster of 16 CTAs per tile, each owning a contiguous slice of the
 //                non-anchor tokens whose F^L rows it keeps in shared memory for every iteration (8
-//                CTAs re-reading them from L2 where they do not fit): Lloyd on raw F^L (assignment
+//                CTAs re-reading them from L2 where they do not fit, 4 beyond one wave of such
+//                clusters): Lloyd on raw F^L (assignment
 //                in each CTA, per-CTA sums in token order, cross-CTA sums in rank order through
 //                distributed shared memory), then the
 //                per-cluster, per-layer sums of unit feature rows, the sums of a_j, sizes and Eq. 2
@@ -282,7 +283,8 @@ __global__ void __launch_bounds__(1024) anchor_kernel(PruneDims p, PruneWs w) {
 // ---- 3. a_i = max over anchors of cos(F^L_i, F^L_p) -------------------------------------------
 // A cluster of AS CTAs per 64 non-anchor tokens x 64 anchors tile, each CTA one slice of the
 // feature dimension: 32-wide chunks through shared memory (stored transposed; the next chunk is
-// fetched into registers while the current one is multiplied), 4 x 4 dot products per thread.
+// fetched into registers while the current one is multiplied), 4 x 4 dot products per thread
+// (4 consecutive rows x 4 consecutive anchors: two 16-byte shared-memory loads per 16 FMAs).
 // The partial tiles are summed in rank order through distributed shared memory, each CTA
 // finishing 64 / AS rows. AS = 4 at serving batch; 8 for a few tiles (shorter chains per CTA).
 template <int SIM, int AS>
@@ -290,7 +292,7 @@ __global__ void __cluster_dims__(AS, 1, 1) __launch_bounds__(256)
     anchor_sim_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
-  __shared__ float Us[32][68], As[32][68];
+  __shared__ __align__(16) float Us[32][68], As[32][68];
   __shared__ float P[64][65];  // this CTA's partial dot products
   cg::cluster_group cl = cg::this_cluster();
   const int rank = int(cl.block_rank());
@@ -298,20 +300,23 @@ __global__ void __cluster_dims__(AS, 1, 1) __launch_bounds__(256)
   const int u0 = (blockIdx.x / AS) * 64, p0 = blockIdx.y * 64;
   const int* ul = w.ulist + size_t(t) * p.m;
   const int* al = w.alist + size_t(t) * p.n_anc;
-  // staging: thread loads column dd of rows r0 + 8 i (i < 8) of both operands
+  // staging: thread loads column dd of rows 8 r0 + i (i < 8) of both operands
   const int dd = threadIdx.x & 31, r0 = threadIdx.x >> 5;
   // per-row statistics of the final layer (MSE: squared norms; KL: log-sum-exps, negentropies)
   const size_t so = (size_t(p.fin) * p.n_tiles + t) * p.n;
   constexpr bool kl = SIM == SPD_SIM_KL;
-  const float* urow[8];
-  const float* arow[8];
+  // rows as 32-bit offsets into the tile's block of F^L (fewer registers than pointers; the block
+  // holds at most 4097 rows of at most 4096 floats); -1 for rows past the lists
+  const float* tile_f = feat_row(p, p.fin, t, -p.off);
+  int uo[8], ao[8];
   double ulse[8];  // KL: the non-anchor operand is softmax(F^L_i) = exp(F^L_i - lse_i), in fp64
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    const int r = r0 + 8 * i;
-    urow[i] = (u0 + r < p.m) ? feat_row(p, p.fin, t, ul[u0 + r]) : nullptr;
-    arow[i] = (p0 + r < p.n_anc) ? feat_row(p, p.fin, t, al[p0 + r]) : nullptr;
-    ulse[i] = (kl && urow[i]) ? double(w.st1[so + ul[u0 + r]]) + double(w.st3[so + ul[u0 + r]]) : 0.0;
+    const int r = 8 * r0 + i;
+    const bool uv = u0 + r < p.m;
+    uo[i] = uv ? (p.off + ul[u0 + r]) * p.d : -1;
+    ao[i] = (p0 + r < p.n_anc) ? (p.off + al[p0 + r]) * p.d : -1;
+    ulse[i] = (kl && uv) ? double(w.st1[so + ul[u0 + r]]) + double(w.st3[so + ul[u0 + r]]) : 0.0;
   }
   const int nch = (p.d + 31) / 32, c0 = rank * nch / AS, c1 = (rank + 1) * nch / AS;
   float ru[8], ra[8];
@@ -319,10 +324,10 @@ __global__ void __cluster_dims__(AS, 1, 1) __launch_bounds__(256)
     const int dcol = ch * 32 + dd;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const float x = (urow[i] && dcol < p.d) ? urow[i][dcol] : 0.0f;
-      if constexpr (kl) ru[i] = (urow[i] && dcol < p.d) ? float(exp(double(x) - ulse[i])) : 0.0f;
+      const float x = (uo[i] >= 0 && dcol < p.d) ? tile_f[uo[i] + dcol] : 0.0f;
+      if constexpr (kl) ru[i] = (uo[i] >= 0 && dcol < p.d) ? float(exp(double(x) - ulse[i])) : 0.0f;
       else ru[i] = x;
-      ra[i] = (arow[i] && dcol < p.d) ? arow[i][dcol] : 0.0f;
+      ra[i] = (ao[i] >= 0 && dcol < p.d) ? tile_f[ao[i] + dcol] : 0.0f;
     }
   };
   float acc[4][4];
@@ -332,20 +337,19 @@ __global__ void __cluster_dims__(AS, 1, 1) __launch_bounds__(256)
     for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
   if (c0 < c1) fetch(c0);
   for (int ch = c0; ch < c1; ++ch) {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      Us[dd][r0 + 8 * i] = ru[i];
-      As[dd][r0 + 8 * i] = ra[i];
-    }
+    // eight consecutive rows of column dd: two 16-byte stores per operand
+    *reinterpret_cast<float4*>(&Us[dd][8 * r0]) = make_float4(ru[0], ru[1], ru[2], ru[3]);
+    *reinterpret_cast<float4*>(&Us[dd][8 * r0 + 4]) = make_float4(ru[4], ru[5], ru[6], ru[7]);
+    *reinterpret_cast<float4*>(&As[dd][8 * r0]) = make_float4(ra[0], ra[1], ra[2], ra[3]);
+    *reinterpret_cast<float4*>(&As[dd][8 * r0 + 4]) = make_float4(ra[4], ra[5], ra[6], ra[7]);
     __syncthreads();
     if (ch + 1 < c1) fetch(ch + 1);  // in flight during the products below
 #pragma unroll 8
     for (int e = 0; e < 32; ++e) {
-      float a[4], b[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = Us[e][ty + 16 * i];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) b[j] = As[e][tx + 16 * j];
+      // rows 4 ty .. 4 ty + 3 and anchors 4 tx .. 4 tx + 3: one 16-byte load each
+      const float4 av = *reinterpret_cast<const float4*>(&Us[e][4 * ty]);
+      const float4 bv = *reinterpret_cast<const float4*>(&As[e][4 * tx]);
+      const float a[4] = {av.x, av.y, av.z, av.w}, b[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -356,7 +360,7 @@ __global__ void __cluster_dims__(AS, 1, 1) __launch_bounds__(256)
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) P[ty + 16 * i][tx + 16 * j] = acc[i][j];
+    for (int j = 0; j < 4; ++j) P[4 * ty + i][4 * tx + j] = acc[i][j];
   cl.sync();
   // rows RPC rank .. RPC rank + RPC - 1 of the tile (TPR threads a row, CPT columns a thread): all
   // AS partials loaded first, summed in rank order
@@ -999,8 +1003,10 @@ __global__ void __launch_bounds__(kmeans_threads<KN>()) kmeans_kernel(PruneDims 
 //        (the j = i term is 0; (X_k - S_k) / c is the cluster mean of log P_j, so every product
 //        is of a probability and an O(1) difference of logs, with no cancellation of large sums)
 // (Q_k, S_k: the cluster's sums of |F_j|^2 and of lse_j.)
+// One warp per token. The cosine instance is held to 80 registers so that three CTAs share an SM
+// (a few bytes of spills; 64 tiles about 10 us faster than at 97 registers and two CTAs).
 template <int SIM>
-__global__ void __launch_bounds__(256) score_kernel(PruneDims p, PruneWs w) {
+__global__ void __launch_bounds__(256, SIM == SPD_SIM_COS ? 3 : 1) score_kernel(PruneDims p, PruneWs w) {
   pdl_launch_dependents();
   pdl_wait();
   const int t = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1345,6 +1351,8 @@ int kmeans_setup() {
       return e;
     };
     err = streamed(kmeans_kernel<8, false, 4, true>);
+    if (err == cudaSuccess) err = streamed(kmeans_kernel<4, false, 4, true>);
+    if (err == cudaSuccess) err = streamed(kmeans_kernel<4, false, 4, false>);
     if (err == cudaSuccess) err = streamed(kmeans_kernel<8, false, SPD_MAX_CLUSTERS, true>);
     if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, 4, true>);
     if (err == cudaSuccess) err = resident(kmeans_kernel<16, true, SPD_MAX_CLUSTERS, true>);
@@ -1392,7 +1400,8 @@ PrunePlan prune_plan(const PruneDims& p) {
   const size_t res_bytes = size_t((p.m + 15) / 16) * p.d * sizeof(float) + cent_bytes;
   // K-means: the rows resident in shared memory over 16 CTAs per tile where they fit and all tiles
   // run in one wave of such clusters (latency); else re-read from L2 each pass by 8 CTAs per tile,
-  // twice as many tiles at once (throughput)
+  // twice as many tiles at once (throughput), or by 4 where 8-CTA clusters would take more than one
+  // wave at two CTAs an SM (the paper's K = 4)
   q.res = p.m > 0 && res_bytes <= kResSmem && g_res_clusters > 0 && p.n_tiles <= g_res_clusters;
   // resident rows and the cosine kind: scores, selection and compaction in the same kernel (CTA 0's
   // row buffer holds the m sort keys and the n kept flags by then)
@@ -1471,6 +1480,8 @@ extern "C" int spd_prune(const spd_prune_cfg* cfg, const float* const* feats, co
     SPD_CUDA_TRY((launch_kmeans<16, true, 4>(p, w, out, res_bytes, st)));
   else if (plan.res)
     SPD_CUDA_TRY((launch_kmeans<16, true, SPD_MAX_CLUSTERS>(p, w, out, res_bytes, st)));
+  else if (p.K == 4 && size_t(p.n_tiles) * 8 > 2 * size_t(num_sms()))
+    SPD_CUDA_TRY((launch_kmeans<4, false, 4>(p, w, out, cent_bytes, st)));
   else if (p.K == 4)
     SPD_CUDA_TRY((launch_kmeans<8, false, 4>(p, w, out, cent_bytes, st)));
   else

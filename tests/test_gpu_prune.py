@@ -37,12 +37,14 @@ def test_llava_next_anyres_tiles(keep):
     assert_prune_parity(gpu_prune(v, keep, 1), res)
 
 
-def test_many_tiles_streamed_kmeans():
+@pytest.mark.parametrize("n_tiles", [24, 40])
+def test_many_tiles_streamed_kmeans(n_tiles):
     # more tiles than one wave of resident 16-CTA K-means clusters: the form that re-reads the rows
-    # from L2 with 8 CTAs per tile runs (serving batches)
+    # from L2 runs (serving batches), with 8 CTAs per tile while those clusters fit in one wave at
+    # two CTAs an SM (24 tiles on 152 SMs), with 4 CTAs per tile beyond (40 tiles)
     # (tiles conditioned one by one: a seed whose 24 tiles all have margins above 1e-3 is rare)
     vs, res = [], []
-    for i in range(24):
+    for i in range(n_tiles):
         _, v1, r1 = conditioned_vision(20260601 + 97 * i, 1, 576, 1024, 2, 16, 64, 1)
         vs.append(v1)
         res += r1
