@@ -269,24 +269,33 @@ __device__ __forceinline__ void rope_cos_sin(int p, float2 f, float& c, float& s
 // holds pair element j, lane l + 16 element j + head_dim / 2) for 8 tokens t0 + j, handed to
 // store(j, col, value) with col = head * head_dim + rotated index. The angles are computed in
 // registers: a per-position table would cost an L2 round trip per 8 tokens.
-template <typename Store>
-__device__ __forceinline__ void rope8(const KArgs& a, int nn, int lane, int t0, const float (&v)[8],
-                                      const int* tpos, int tb, Store store) {
+// The angles of rope8: lanes l and l + 16 rotate by the same angles, so each evaluates those of four
+// of the 8 tokens t0 + j (lane l the first four, lane l + 16 the last four) and they trade them;
+// pos_of(t) is the rotary position of token t.
+template <typename PosOf>
+__device__ __forceinline__ void rope_angles4(const KArgs& a, int nn, int lane, int t0, PosOf pos_of,
+                                             float (&cm)[4], float (&sm)[4]) {
   const int nt = a.n_tok;
+  const int jf = 16 * ((nn % a.head_dim) >> 5) + (lane & 15);
+  const float2 fr = a.rope[jf];
+  const int hi = lane >> 4;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int t = min(t0 + 4 * hi + i, nt - 1);
+    rope_cos_sin(pos_of(t), fr, cm[i], sm[i]);
+  }
+}
+
+// rope8 with this lane's four angles given (cm, sm as computed by rope_angles4).
+template <typename Store>
+__device__ __forceinline__ void rope8_rot(const KArgs& a, int nn, int lane, const float (&v)[8],
+                                          const float (&cm)[4], const float (&sm)[4], Store store) {
   const int hd = a.head_dim, half = hd >> 1;
   const int head = nn / hd, g = (nn % hd) >> 5;
   const int jf = 16 * g + (lane & 15);
   const int col = head * hd + ((lane < 16) ? jf : half + jf);
-  const float2 fr = a.rope[jf];
   const float sgn = (lane < 16) ? -1.0f : 1.0f;
-  // lanes l and l + 16 rotate by the same angles: each evaluates four tokens' and they trade
   const int hi = lane >> 4;
-  float cm[4], sm[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int t = min(t0 + 4 * hi + i, nt - 1);
-    rope_cos_sin(tpos[t - tb], fr, cm[i], sm[i]);
-  }
   float y[8];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {  // branch-free math, then the stores
@@ -301,6 +310,14 @@ __device__ __forceinline__ void rope8(const KArgs& a, int nn, int lane, int t0, 
   }
 #pragma unroll
   for (int j = 0; j < 8; ++j) store(j, col, y[j]);
+}
+
+template <typename Store>
+__device__ __forceinline__ void rope8(const KArgs& a, int nn, int lane, int t0, const float (&v)[8],
+                                      const int* tpos, int tb, Store store) {
+  float cm[4], sm[4];
+  rope_angles4(a, nn, lane, t0, [&](int t) { return tpos[t - tb]; }, cm, sm);
+  rope8_rot(a, nn, lane, v, cm, sm, store);
 }
 
 // rope8 stored as bf16 to row row_of(t) of o (skipped when negative or past the tokens).
@@ -322,7 +339,8 @@ __device__ __forceinline__ void rope_store8(const KArgs& a, __nv_bfloat16* o, in
 constexpr int kStgPitch = 256;
 template <int EPI>
 __device__ __forceinline__ void stage8(const KArgs& a, int n, int lane, int t0, const float (&v)[8],
-                                       const int* tpos, int tb, uint8_t* stg) {
+                                       const int* tpos, int tb, uint8_t* stg,
+                                       const float* cs = nullptr) {
   const bool second = EPI == EPI_QKV_BF16 && n >= a.split;  // a K/V row of the fused QKV GEMM
   const int nn = second ? n - a.split : n;                   // row within its output
   const int c0 = nn & ~127;
@@ -331,7 +349,12 @@ __device__ __forceinline__ void stage8(const KArgs& a, int n, int lane, int t0, 
     *reinterpret_cast<__nv_bfloat16*>(base + j * kStgPitch + 2 * (col - c0)) = __float2bfloat16_rn(y);
   };
   if ((EPI == EPI_QKV_BF16 && !second) || nn < a.rope_rows) {  // warp-uniform
-    rope8(a, nn, lane, t0, v, tpos, tb, put);
+    if (cs) {  // the angles from the rotary table: (cos, sin) of the lane's four tokens
+      const float cm[4] = {cs[0], cs[2], cs[4], cs[6]}, sm[4] = {cs[1], cs[3], cs[5], cs[7]};
+      rope8_rot(a, nn, lane, v, cm, sm, put);
+    } else {
+      rope8(a, nn, lane, t0, v, tpos, tb, put);
+    }
   } else {
 #pragma unroll
     for (int j = 0; j < 8; ++j) put(j, nn, v[j]);
@@ -762,6 +785,39 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q = warp & 3;
     const int half = (warp - 2) >> 2;
     const int row = q * 32 + lane;
+    // Rotary table: where the CTA's only segment is a whole tile of a staged rotary epilogue, the
+    // second TMEM accumulator is unused, and the epilogue warps, idle during the main loop, fill it
+    // with the (cos, sin) of every 8-token group of their lanes (8 fp32 columns a group: the four
+    // tokens' angles the lane evaluates in rope8). The epilogue then loads them beside the
+    // accumulator instead of evaluating them after it is ready (the same function of the same
+    // inputs: identical values).
+    bool rtab = false;
+    const uint32_t ttab = tmem + a.accs + (static_cast<uint32_t>(q * 32) << 16);
+    if constexpr (EPI == EPI_QKV_BF16 || EPI == EPI_ROPE_BF16) {
+      if (a.staged && plan.count == 1 && a.nbuf == 2 && a.nh == 1) {
+        int u0s, u1s;
+        seg_get(plan, 0, u0s, u1s);
+        const int tile = u0s / a.n_kb;
+        if (u0s == tile * a.n_kb && u1s - u0s == a.n_kb) {
+          const int wt = tile / a.n_ttiles, tt_i = tile - wt * a.n_ttiles;
+          const int tok0 = tt_i * a.tt, valid = min(a.tt, a.n_tok - tok0);
+          const int n = (PAIR ? 2 * wt + prank : wt) * kBM + row;
+          const bool second = EPI == EPI_QKV_BF16 && n >= a.split;
+          const int nn = second ? n - a.split : n;
+          if ((EPI == EPI_QKV_BF16 && !second) || nn < a.rope_rows) {  // warp-uniform
+            rtab = true;
+#pragma unroll 1
+            for (int cc = half * 8; cc < valid; cc += 16) {
+              float cm[4], sm[4];
+              rope_angles4(a, nn, lane, tok0 + cc, [&](int t) { return a.pos ? a.pos[t] : 0; }, cm, sm);
+              const float w[8] = {cm[0], sm[0], cm[1], sm[1], cm[2], sm[2], cm[3], sm[3]};
+              tmem_st8(ttab + cc, w);
+            }
+            tmem_st_wait();
+          }
+        }
+      }
+    }
     for (int j = 0; j < plan.count; ++j) {
       int u, seg_end;
       seg_get(plan, j, u, seg_end);
@@ -800,8 +856,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
           for (int cc = half * 8; cc < valid; cc += 16) {
             float v[8];
-            tmem_ld8(tq + h * a.hoff + cc, v);
-            stage8<EPI>(a, (blk0 + h) * kBM + row, lane, tok0 + cc, v, tpos, tok0, sh);
+            if (rtab) {  // j == 0, h == 0: the table of this segment
+              float cs[8];
+              tmem_ld8x2(tq + cc, v, ttab + cc, cs);
+              stage8<EPI>(a, (blk0 + h) * kBM + row, lane, tok0 + cc, v, tpos, tok0, sh, cs);
+            } else {
+              tmem_ld8(tq + h * a.hoff + cc, v);
+              stage8<EPI>(a, (blk0 + h) * kBM + row, lane, tok0 + cc, v, tpos, tok0, sh);
+            }
           }
         }
         fence_proxy_async_smem();
