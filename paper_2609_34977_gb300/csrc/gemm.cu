@@ -911,12 +911,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (flags[1]) {
           __threadfence();
           for (int h = 0; h < a.nh; ++h) {
+            // the next group's sums are loaded before this group's epilogue (one L2 round trip
+            // per group instead of two dependent ones)
+            constexpr bool kPre = EPI == EPI_SWIGLU_BF16;  // the remainder schedule's GEMM
+            float nx[8];
+            if (kPre && half * 8 < valid) {
+              const float* p0 = acc + size_t(half * 8) * ar + h * kBM + row;
+#pragma unroll
+              for (int jj = 0; jj < 8; ++jj) nx[jj] = __ldcg(p0 + size_t(jj) * ar);
+            }
 #pragma unroll 1
             for (int cc = half * 8; cc < valid; cc += 16) {
               float* p = acc + size_t(cc) * ar + h * kBM + row;
               float v[8];
 #pragma unroll
-              for (int jj = 0; jj < 8; ++jj) v[jj] = __ldcg(p + size_t(jj) * ar);
+              for (int jj = 0; jj < 8; ++jj) v[jj] = kPre ? nx[jj] : __ldcg(p + size_t(jj) * ar);
+              if (kPre && cc + 16 < valid) {
+                const float* pn = p + size_t(16) * ar;
+#pragma unroll
+                for (int jj = 0; jj < 8; ++jj) nx[jj] = __ldcg(pn + size_t(jj) * ar);
+              }
 #pragma unroll
               for (int jj = 0; jj < 8; ++jj) __stcg(p + size_t(jj) * ar, 0.0f);
               epilogue8<EPI>(a, (blk0 + h) * kBM + row, q, lane, blk0 + h, tok0 + cc, v, trow, tpos,
